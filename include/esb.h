@@ -1,0 +1,245 @@
+/*
+ * esb.h -- C ABI of libesb.so: Elastic Significant Bit (ESB) quantization
+ * and ESB-coded contraction on one Blackwell-Ultra GPU (sm_103a).
+ *
+ * Method: Gong et al., "Elastic Significant Bit Quantization and
+ * Acceleration for Deep Neural Networks" (arXiv 2109.03513).
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ * - Pointers marked [device] are CUDA device pointers owned by the caller;
+ *   [host] pointers are ordinary host memory owned by the caller.  The
+ *   library never keeps a pointer after a call returns and allocates no
+ *   device memory; scratch memory is passed in by the caller (workspace).
+ * - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *   stream).  All device work is enqueued asynchronously on that stream;
+ *   nothing synchronises unless stated.
+ * - Arguments are validated on the host before any launch.  A non-zero
+ *   esb_status means nothing was enqueued.  ESB_ERR_CUDA means a launch
+ *   failed (cudaGetLastError is left set for the caller to inspect).
+ * - Kernels that wait on the tensor-core pipeline bound every wait; when a
+ *   wait gives up the kernel records ESB_ERR_TIMEOUT in a device status word
+ *   (read with esb_get_status) and returns without hanging.
+ *
+ * ESB format (Sec. III-B set, Sec. IV-A float format)
+ * ---------------------------------------------------
+ * fmt = {b, k, is_signed}, 2 <= b <= 8, 0 <= k <= b-1, N = 2^(b-k-1) - 1.
+ * A b-bit code is  sign (1 bit) | e (b-k-1 bits) | f (k bits), MSB..LSB.
+ * Its value in units of alpha is 0.f (= f * 2^-k) when e == N and
+ * 2^e * 1.f otherwise; its integer image is I = value * 2^k.  Zero is
+ * always encoded with sign 0 (e = N, f = 0), so the all-zero bit pattern
+ * is NOT zero.  Unsigned formats (is_signed = 0) use the non-negative half
+ * of the set with the same codes (sign bit always 0).
+ *
+ * Packed code matrices: floor(32/b) codes per little-endian 32-bit word,
+ * code j of a row in bits [b*(j % cpw), b*(j % cpw) + b) of word j / cpw;
+ * slots past the last column hold the zero code; unused high bits are 0.
+ * Each row starts at a word boundary; `ld*` arguments give the row stride
+ * in 32-bit words.
+ */
+#ifndef ESB_H_
+#define ESB_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum esb_status {
+    ESB_OK = 0,
+    ESB_ERR_INVALID_ARG = 1,  /* null pointer, negative size, bad enum, ld too small, alpha <= 0 ... */
+    ESB_ERR_UNSUPPORTED = 2,  /* (b,k) outside the range the entry point implements */
+    ESB_ERR_RANGE = 3,        /* an exactness bound (int32 / fp32 accumulation) would be exceeded */
+    ESB_ERR_ALIGN = 4,        /* a pointer or stride violates the stated alignment */
+    ESB_ERR_CUDA = 5,         /* a CUDA runtime call or launch failed */
+    ESB_ERR_TIMEOUT = 6       /* (device status only) a bounded pipeline wait gave up */
+} esb_status;
+
+typedef struct esb_format {
+    int32_t b;          /* total bits, 2..8 */
+    int32_t k;          /* fraction bits (k+1 significant bits), 0..b-1 */
+    int32_t is_signed;  /* 1: symmetric set; 0: non-negative half */
+} esb_format;
+
+/* Tie rule of the projection.  Sec. III-C gives half-open look-up
+ * intervals, so a value on a midpoint goes to the element of larger
+ * magnitude (ESB_ROUND_HALF_AWAY, the default).  ESB_ROUND_HALF_EVEN picks
+ * the neighbour whose multiple of the local spacing is even. */
+enum { ESB_ROUND_HALF_AWAY = 0, ESB_ROUND_HALF_EVEN = 1 };
+
+/* Activation of the fused epilogue (Sec. IV-B "MP&ReLU"; ReLU6 for
+ * MobileNetV2-shaped networks). */
+enum { ESB_ACT_NONE = 0, ESB_ACT_RELU = 1, ESB_ACT_RELU6 = 2 };
+
+/* Post-processing fused into the contraction (Sec. IV-C: "BN and DN"
+ * affine, activation, ESB quantization of the next layer's input).
+ * For accumulator acc[m][n] (exact int32) the epilogue computes, in fp32
+ * with this exact op order:
+ *   y = fmaf(scale[n], (float)acc, bias[n])
+ *   y = fmaf(res_scale, (float)I_res[m][n], y)         if residual != NULL
+ *   y = max(y, 0) (RELU) or min(max(y, 0), 6) (RELU6)
+ *   code = projection of y with alpha_out, fmt_out, rounding_out
+ *          (same as esb_project)
+ * The BN/DN fold of Sec. IV-C becomes scale[n]/bias[n] on the host. */
+typedef struct esb_epilogue {
+    const float* scale;        /* [device] N floats, or NULL -> scale0 for every n */
+    const float* bias;         /* [device] N floats, or NULL -> bias0 for every n */
+    float scale0;
+    float bias0;
+    int32_t act;               /* ESB_ACT_* */
+    const uint32_t* residual;  /* [device] packed codes, M rows of res_ld words, or NULL */
+    int64_t res_ld;            /* row stride of residual in words */
+    esb_format res_fmt;        /* format of the residual codes */
+    float res_scale;           /* multiplies the residual integer image */
+    float alpha_out;           /* requantisation scale (> 0), used if alpha_out_dev == NULL */
+    const float* alpha_out_dev;/* [device] 1 float, read by the kernel; overrides alpha_out */
+    esb_format fmt_out;        /* format of the output codes */
+    int32_t rounding_out;      /* ESB_ROUND_* */
+} esb_epilogue;
+
+/* Convolution geometry, NHWC activations, weights [cout][r][s][c]. */
+typedef struct esb_conv_desc {
+    int32_t n, h, w, c;        /* input batch, height, width, channels */
+    int32_t cout;              /* output channels (must equal c when groups == c) */
+    int32_t r, s;              /* filter height, width */
+    int32_t stride, pad;       /* same stride / zero padding in both dimensions */
+    int32_t groups;            /* 1 (dense) or c (depthwise) */
+} esb_conv_desc;
+
+/* ---------------------------------------------------------------- info */
+
+/* Library version: major*10000 + minor*100 + patch. */
+int32_t esb_version(void);
+
+/* Human-readable name of an esb_status value (static string). */
+const char* esb_status_string(int32_t status);
+
+/* ESB_OK if 2 <= b <= 8, 0 <= k <= b-1 and is_signed is 0 or 1. */
+esb_status esb_format_check(esb_format f);
+
+/* floor(32 / b) codes per 32-bit word; 0 for b outside 2..8. */
+int32_t esb_codes_per_word(int32_t b);
+
+/* Smallest row stride (words) for `cols` codes that keeps rows 16-byte
+ * aligned: ceil(cols / cpw) rounded up to a multiple of 4. */
+int64_t esb_row_words(int64_t cols, int32_t b);
+
+/* The code of zero (sign 0, e = N, f = 0); 0xFFFFFFFF for a bad format. */
+uint32_t esb_zero_code(esb_format f);
+
+/* alpha*(b,k) of Eq. optimal_alpha_seeking: the scale minimising the
+ * distribution difference D(alpha,b,k) of Eq. objective_function_expansion
+ * for N(0,1) data (Sec. III-D "Resolving extremum"; Table 1 prints it).
+ * Where D has several local minima (large N) the first one from small
+ * alpha is returned.  `dda` (nullable) receives the squared error over both
+ * halves, 2*D(alpha*), the quantity Table 1 prints as DDA.  Host only;
+ * cached per (b,k); thread-safe. */
+esb_status esb_alpha_star(int32_t b, int32_t k, double* alpha_star, double* dda);
+
+/* ----------------------------------------------------------- calibrate */
+
+/* Bytes of device workspace esb_calibrate_dda needs for n values. */
+size_t esb_calibrate_dda_workspace_bytes(int64_t n);
+
+/* DDA calibration of Sec. III-D ("Normalization" and "Resolving extremum"):
+ * statistics of x, then alpha = fl32(alpha*(b,k) * (spread + 1e-7)), where
+ * spread is the standard deviation sigma (signed formats: data normalised
+ * to zero mean and unit variance as in Sec. III-D) or the root mean square
+ * (unsigned formats: post-ReLU data, the scale of the underlying normal).
+ *   x          [device] n floats (16-byte aligned for the vector path; any
+ *              alignment accepted)
+ *   n          > 0
+ *   workspace  [device] >= esb_calibrate_dda_workspace_bytes(n) bytes,
+ *              8-byte aligned, contents ignored and overwritten
+ *   alpha_out  [device] 1 float written by the kernel (no host sync)
+ *   stats_out  [device] 3 doubles {mean, sigma or rms, n}, or NULL
+ * The reduction order is fixed, so results are bit-reproducible.
+ * Errors: INVALID_ARG, UNSUPPORTED (bad format), ALIGN (workspace), CUDA. */
+esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
+                             void* workspace, size_t workspace_bytes,
+                             float* alpha_out, double* stats_out, void* stream);
+
+/* ------------------------------------------------------------- project */
+
+/* Cheap projection operator of Eq. cheap_projection with the
+ * shift-and-round projection of Eq. fast_projection: for each element,
+ * v = x / alpha (IEEE fp32 division, round to nearest), clip to [-C, C]
+ * (C = largest set element), keep k+1 significant bits of |v| (the
+ * spacing of values below 1 is 2^-k), round by `rounding`, restore the
+ * sign, emit the b-bit code.  NaN -> zero code; +-Inf -> +-C; negative
+ * values -> zero code for unsigned formats.
+ *   x        [device] rows x cols floats, row stride ldx (>= cols) floats
+ *   alpha    > 0 and finite; used when alpha_dev == NULL
+ *   alpha_dev[device] 1 float (e.g. written by esb_calibrate_dda), or NULL
+ *   codes    [device] rows x ldc words, ldc >= ceil(cols / cpw); every word
+ *            of every row is written (slots past cols hold the zero code)
+ * Fast path when x, codes are 16-byte aligned and ldx, ldc are multiples
+ * of 4; otherwise a slower general path.  The two ranges must not overlap.
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx,
+                       float alpha, const float* alpha_dev, esb_format f, int32_t rounding,
+                       uint32_t* codes, int64_t ldc, void* stream);
+
+/* Dequantisation (test aid and fp32 export): y = fl32(alpha * q), q the
+ * value of each code in units of alpha (Sec. IV-A, Eq. q).
+ *   codes [device] rows x ldc words; y [device] rows x ldy floats. */
+esb_status esb_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_t ldc,
+                       float alpha, const float* alpha_dev, esb_format f,
+                       float* y, int64_t ldy, void* stream);
+
+/* ---------------------------------------------------------------- gemm */
+
+/* ESB-coded GEMM (Sec. III-B products of set elements; Sec. IV-B/IV-C
+ * computing logic): acc[m][n] = sum_k I(A[m][k]) * I(B[n][k]) exactly, then
+ * the fused epilogue (esb_epilogue) on each element.
+ *   A  [device] M rows of lda words (K codes each, K-major), 16-byte aligned rows
+ *   B  [device] N rows of ldb words (K codes each, K-major), 16-byte aligned rows
+ *   ep [host] epilogue parameters; may be NULL when codes_out == NULL and
+ *      y_out == NULL
+ *   acc_out   [device] M x N int32 (row stride N), or NULL
+ *   y_out     [device] M x N floats (row stride N), or NULL
+ *   codes_out [device] M rows of ldo words (N codes in fmt_out), or NULL
+ * The contraction runs on the tcgen05 tensor cores; it requires both
+ * formats to have k <= 3 and b-k-1 <= 4 (every config format qualifies),
+ * and K * max|I_A| * max|I_B| < 2^24 (else ESB_ERR_RANGE).
+ * Errors: INVALID_ARG, UNSUPPORTED, RANGE, ALIGN, CUDA. */
+esb_status esb_gemm(int64_t M, int64_t N, int64_t K,
+                    const uint32_t* A, int64_t lda, esb_format fa,
+                    const uint32_t* B, int64_t ldb, esb_format fb,
+                    const esb_epilogue* ep,
+                    int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
+                    void* stream);
+
+/* ---------------------------------------------------------------- conv */
+
+/* ESB-coded convolution, NHWC (Sec. IV-B: a K x K x c_in x c_out
+ * convolution over an h x w x c_in feature map), as an implicit GEMM with
+ * M = n*P*Q output pixels, N = cout, K = r*s*c, followed by the fused
+ * epilogue.  P = (h + 2 pad - r)/stride + 1, Q likewise.
+ *   X [device] n*h*w pixel rows of ldx words (c codes each), ldx % 4 == 0
+ *   W [device] cout*r*s rows of ldw words (c codes each); ldw == ldx
+ *   outputs as esb_gemm with M = n*P*Q rows (pixel-major NHWC).
+ * groups == c selects the depthwise path (one r x s filter per channel, W
+ * holds r*s rows of ldw words with c codes each, cout == c).
+ * Errors: INVALID_ARG, UNSUPPORTED, RANGE, ALIGN, CUDA. */
+esb_status esb_conv2d_nhwc(const esb_conv_desc* d,
+                           const uint32_t* X, int64_t ldx, esb_format fx,
+                           const uint32_t* W, int64_t ldw, esb_format fw,
+                           const esb_epilogue* ep,
+                           int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
+                           void* stream);
+
+/* ------------------------------------------------------------- status */
+
+/* Synchronises `stream`, then returns and clears the device status word
+ * (ESB_OK or ESB_ERR_TIMEOUT) in *device_status.  Returns ESB_ERR_CUDA if
+ * the synchronisation fails. */
+esb_status esb_get_status(void* stream, int32_t* device_status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ESB_H_ */

@@ -78,6 +78,7 @@ def _load():
         "oracle_unpack": (None, [p, i64, i64, i32, i64, p]),
         "oracle_D": (f64, [f64, i32, i32]),
         "oracle_alpha_star": (f64, [i32, i32, p]),
+        "oracle_dD": (f64, [f64, i32, i32]),
         "oracle_calibrate": (f32, [p, i64, i32, i32, i32, p]),
         "oracle_calibrate_with": (f32, [p, i64, f64, i32, p]),
         "oracle_gemm_i64": (None, [p, i64, i32, i32, p, i64, i32, i32, i64, i64, i64, p]),
@@ -221,6 +222,10 @@ def project_packed(x2d: np.ndarray, alpha: float, b: int, k: int, signed: bool =
 
 def D(alpha: float, b: int, k: int) -> float:
     return _load().oracle_D(alpha, b, k)
+
+
+def dD(alpha: float, b: int, k: int) -> float:
+    return _load().oracle_dD(alpha, b, k)
 
 
 def alpha_star(b: int, k: int) -> tuple[float, float]:

@@ -272,10 +272,36 @@ double oracle_D(double alpha, int b, int k)
     return D;
 }
 
+/* dD/dalpha.  Differentiating Eq. objective_function_expansion, the terms
+ * from the moving cell boundaries cancel (a boundary is the midpoint of its
+ * two elements, equally far from both), leaving
+ *   D'(alpha) = -2 sum_j q_j int_{cell j} (t - alpha q_j) phi(t) dt,
+ * with int t phi = phi(lo) - phi(hi) and int phi = Q(lo) - Q(hi). */
+double oracle_dD(double alpha, int b, int k)
+{
+    double s[ORACLE_MAX_SET];
+    int n = oracle_set_nonneg(b, k, s);
+    double g = 0.0;
+    for (int j = 0; j < n; j++) {
+        double lo = (j == 0) ? 0.0 : alpha * 0.5 * (s[j - 1] + s[j]);
+        double m1, m0;
+        if (j == n - 1) { m1 = std_phi(lo); m0 = std_Q(lo); }
+        else {
+            double hi = alpha * 0.5 * (s[j] + s[j + 1]);
+            m1 = std_phi(lo) - std_phi(hi);
+            m0 = std_Q(lo) - std_Q(hi);
+        }
+        g += -2.0 * s[j] * (m1 - alpha * s[j] * m0);
+    }
+    return g;
+}
+
 /* Eq. optimal_alpha_seeking: alpha* = argmin D.  D is not convex for large
  * N; the reading used here is "the first local minimum from small alpha"
- * on a 20000-point log grid over [1e-4, 4], refined by golden-section
- * search to 1e-12 relative.  Returns alpha*, and D(alpha*) via D_out. */
+ * (Sec. III-D resolves the extremum of the differentiable D; Fig. 7 plots
+ * D and its first and second derivatives).  The minimum is bracketed on a
+ * 20000-point log grid over [1e-4, 4], then located as the zero of D' by
+ * bisection to full fp64 precision.  Returns alpha*, and D(alpha*) via D_out. */
 double oracle_alpha_star(int b, int k, double *D_out)
 {
     const int G = 20000;
@@ -289,17 +315,16 @@ double oracle_alpha_star(int b, int k, double *D_out)
     int im = G - 1;
     for (int i = 1; i < G - 1; i++)
         if (d[i] <= d[i - 1] && d[i] < d[i + 1]) { im = i; break; }
-    double x0 = a[im > 0 ? im - 1 : 0], x3 = a[im < G - 1 ? im + 1 : G - 1];
+    double x0 = a[im > 0 ? im - 1 : 0], x1 = a[im < G - 1 ? im + 1 : G - 1];
     free(a);
     free(d);
-    const double gr = 0.5 * (sqrt(5.0) - 1.0);
-    double x1 = x3 - gr * (x3 - x0), x2 = x0 + gr * (x3 - x0);
-    double f1 = oracle_D(x1, b, k), f2 = oracle_D(x2, b, k);
-    while (x3 - x0 > 1e-12 * x3) {
-        if (f1 < f2) { x3 = x2; x2 = x1; f2 = f1; x1 = x3 - gr * (x3 - x0); f1 = oracle_D(x1, b, k); }
-        else         { x0 = x1; x1 = x2; f1 = f2; x2 = x0 + gr * (x3 - x0); f2 = oracle_D(x2, b, k); }
+    /* D' < 0 at x0 and > 0 at x1 around an interior minimum. */
+    for (int it = 0; it < 200; it++) {
+        double xm = 0.5 * (x0 + x1);
+        if (xm <= x0 || xm >= x1) break;
+        if (oracle_dD(xm, b, k) < 0.0) x0 = xm; else x1 = xm;
     }
-    double as = 0.5 * (x0 + x3);
+    double as = 0.5 * (x0 + x1);
     if (D_out) *D_out = oracle_D(as, b, k);
     return as;
 }
@@ -351,6 +376,12 @@ static int64_t image_of(uint32_t code, int b, int k)
     return (int64_t)ldexp(oracle_decode(code, b, k), k);
 }
 
+/* Table of image_of over all 2^b codes (built once per call). */
+static void image_table(int b, int k, int64_t *t)
+{
+    for (uint32_t c = 0; c < (1u << b); c++) t[c] = image_of(c, b, k);
+}
+
 /* C[m][n] = sum_k I(A[m][k]) * I(B[n][k]) in int64 (Sec. III-B: the product
  * of two set elements is the product of their fraction values and shifts;
  * Sec. IV-B: a convolution is a multiply-accumulate over c_in * K * K).
@@ -362,13 +393,16 @@ void oracle_gemm_i64(const uint32_t *A, int64_t lda, int ba, int ka,
 {
     int cpa = 32 / ba, cpb = 32 / bb;
     uint32_t ma = (1u << ba) - 1u, mb = (1u << bb) - 1u;
+    int64_t ta[256], tb[256];
+    image_table(ba, ka, ta);
+    image_table(bb, kb, tb);
     for (int64_t m = 0; m < M; m++)
         for (int64_t n = 0; n < N; n++) {
             int64_t acc = 0;
             for (int64_t kk = 0; kk < K; kk++) {
                 uint32_t ca = (A[m * lda + kk / cpa] >> (ba * (kk % cpa))) & ma;
                 uint32_t cb = (B[n * ldb + kk / cpb] >> (bb * (kk % cpb))) & mb;
-                acc += image_of(ca, ba, ka) * image_of(cb, bb, kb);
+                acc += ta[ca] * tb[cb];
             }
             C[m * N + n] = acc;
         }
@@ -381,11 +415,14 @@ int64_t oracle_gemm_entry(const uint32_t *A, int64_t lda, int ba, int ka,
 {
     int cpa = 32 / ba, cpb = 32 / bb;
     uint32_t ma = (1u << ba) - 1u, mb = (1u << bb) - 1u;
+    int64_t ta[256], tb[256];
+    image_table(ba, ka, ta);
+    image_table(bb, kb, tb);
     int64_t acc = 0;
     for (int64_t kk = 0; kk < K; kk++) {
         uint32_t ca = (A[m * lda + kk / cpa] >> (ba * (kk % cpa))) & ma;
         uint32_t cb = (B[n * ldb + kk / cpb] >> (bb * (kk % cpb))) & mb;
-        acc += image_of(ca, ba, ka) * image_of(cb, bb, kb);
+        acc += ta[ca] * tb[cb];
     }
     return acc;
 }
@@ -421,6 +458,9 @@ void oracle_conv2d_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
 {
     int cpx = 32 / bx, cpw_ = 32 / bw;
     uint32_t mx = (1u << bx) - 1u, mw = (1u << bw) - 1u;
+    int64_t tx[256], tw[256];
+    image_table(bx, kx, tx);
+    image_table(bw, kw, tw);
     for (int n = 0; n < Nb; n++)
         for (int p = 0; p < P; p++)
             for (int q = 0; q < Q; q++)
@@ -435,7 +475,7 @@ void oracle_conv2d_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
                             for (int c = 0; c < C; c++) {
                                 uint32_t cx = (xr[c / cpx] >> (bx * (c % cpx))) & mx;
                                 uint32_t cw = (wr[c / cpw_] >> (bw * (c % cpw_))) & mw;
-                                s += image_of(cx, bx, kx) * image_of(cw, bw, kw);
+                                s += tx[cx] * tw[cw];
                             }
                         }
                     acc[(((int64_t)n * P + p) * Q + q) * Cout + co] = s;
@@ -451,6 +491,9 @@ void oracle_dwconv_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
 {
     int cpx = 32 / bx, cpw_ = 32 / bw;
     uint32_t mx = (1u << bx) - 1u, mw = (1u << bw) - 1u;
+    int64_t tx[256], tw[256];
+    image_table(bx, kx, tx);
+    image_table(bw, kw, tw);
     for (int n = 0; n < Nb; n++)
         for (int p = 0; p < P; p++)
             for (int q = 0; q < Q; q++)
@@ -464,7 +507,7 @@ void oracle_dwconv_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
                             const uint32_t *wr = W + ((int64_t)r * S + t) * ldw;
                             uint32_t cx = (xr[c / cpx] >> (bx * (c % cpx))) & mx;
                             uint32_t cw = (wr[c / cpw_] >> (bw * (c % cpw_))) & mw;
-                            s += image_of(cx, bx, kx) * image_of(cw, bw, kw);
+                            s += tx[cx] * tw[cw];
                         }
                     acc[(((int64_t)n * P + p) * Q + q) * C + c] = s;
                 }

@@ -1,0 +1,260 @@
+// esb_api.cu -- the extern "C" entry points of libesb.so: host-side argument
+// validation, path selection and launches.  Declarations and contracts are
+// in include/esb.h.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include <cuda_runtime.h>
+
+#include "esb.h"
+#include "esb_common.cuh"
+#include "esb_internal.h"
+
+namespace esb {
+
+__device__ int g_esb_device_status = 0;
+
+int* device_status_ptr()
+{
+    static int* cache[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    if (!cache[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_esb_device_status) != cudaSuccess) return nullptr;
+        cache[dev] = static_cast<int*>(p);
+    }
+    return cache[dev];
+}
+
+int device_sm_count()
+{
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 132;
+    if (cache[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 132;
+        cache[dev] = n;
+    }
+    return cache[dev];
+}
+
+}  // namespace esb
+
+using namespace esb;
+
+namespace {
+
+bool fmt_ok(const esb_format& f)
+{
+    return f.b >= 2 && f.b <= 8 && f.k >= 0 && f.k <= f.b - 1 && (f.is_signed == 0 || f.is_signed == 1);
+}
+
+// The tensor-core operand route: the scaled-E4M3 image needs k <= 3 and an
+// exponent field of at most 4 bits, and must avoid the E4M3 NaN pattern
+// (exponent 15 with mantissa 111, i.e. b-k-1 = 4 and k = 3).
+bool fmt_tc_ok(const esb_format& f)
+{
+    const int ew = f.b - f.k - 1;
+    return f.k <= 3 && ew <= 4 && !(ew == 4 && f.k == 3);
+}
+
+int64_t words_for(int64_t cols, int b) { return (cols + (32 / b) - 1) / (32 / b); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+std::mutex g_astar_mu;
+double g_astar[9][9];
+double g_dda[9][9];
+bool g_astar_have[9][9];
+
+esb_status alpha_star_cached(int b, int k, double* a, double* d)
+{
+    std::lock_guard<std::mutex> lk(g_astar_mu);
+    if (!g_astar_have[b][k]) {
+        g_astar[b][k] = alpha_star_solve(b, k, &g_dda[b][k]);
+        g_astar_have[b][k] = true;
+    }
+    if (a) *a = g_astar[b][k];
+    if (d) *d = g_dda[b][k];
+    return ESB_OK;
+}
+
+esb_status check_epilogue(const esb_epilogue* ep, int64_t M, int64_t N, bool want_codes)
+{
+    if (!ep) return want_codes ? ESB_ERR_INVALID_ARG : ESB_OK;
+    if (ep->act < ESB_ACT_NONE || ep->act > ESB_ACT_RELU6) return ESB_ERR_INVALID_ARG;
+    if (ep->residual) {
+        if (!fmt_ok(ep->res_fmt)) return ESB_ERR_UNSUPPORTED;
+        if (ep->res_ld < words_for(N, ep->res_fmt.b)) return ESB_ERR_INVALID_ARG;
+        if (esb::fmt_max_image(ep->res_fmt.b, ep->res_fmt.k) >= 16777216.0) return ESB_ERR_RANGE;
+    }
+    if (want_codes) {
+        if (!fmt_ok(ep->fmt_out)) return ESB_ERR_UNSUPPORTED;
+        if (ep->rounding_out != ESB_ROUND_HALF_AWAY && ep->rounding_out != ESB_ROUND_HALF_EVEN) return ESB_ERR_INVALID_ARG;
+        if (!ep->alpha_out_dev && !(std::isfinite(ep->alpha_out) && ep->alpha_out > 0.0f)) return ESB_ERR_INVALID_ARG;
+    }
+    (void)M;
+    return ESB_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t esb_version(void) { return 100; }
+
+const char* esb_status_string(int32_t s)
+{
+    switch (s) {
+    case ESB_OK: return "ok";
+    case ESB_ERR_INVALID_ARG: return "invalid argument";
+    case ESB_ERR_UNSUPPORTED: return "unsupported format or configuration";
+    case ESB_ERR_RANGE: return "exactness bound exceeded";
+    case ESB_ERR_ALIGN: return "misaligned pointer or stride";
+    case ESB_ERR_CUDA: return "CUDA error";
+    case ESB_ERR_TIMEOUT: return "device pipeline wait timed out";
+    default: return "unknown status";
+    }
+}
+
+esb_status esb_format_check(esb_format f) { return fmt_ok(f) ? ESB_OK : ESB_ERR_UNSUPPORTED; }
+
+int32_t esb_codes_per_word(int32_t b) { return (b >= 2 && b <= 8) ? 32 / b : 0; }
+
+int64_t esb_row_words(int64_t cols, int32_t b)
+{
+    if (b < 2 || b > 8 || cols < 0) return 0;
+    return (words_for(cols, b) + 3) & ~int64_t(3);
+}
+
+uint32_t esb_zero_code(esb_format f) { return fmt_ok(f) ? fmt_zero_code(f.b, f.k) : 0xFFFFFFFFu; }
+
+esb_status esb_alpha_star(int32_t b, int32_t k, double* alpha_star, double* dda)
+{
+    if (b < 2 || b > 8 || k < 0 || k > b - 1) return ESB_ERR_UNSUPPORTED;
+    if (!alpha_star) return ESB_ERR_INVALID_ARG;
+    return alpha_star_cached(b, k, alpha_star, dda);
+}
+
+size_t esb_calibrate_dda_workspace_bytes(int64_t n) { return n > 0 ? calibrate_workspace_bytes(n) : 0; }
+
+esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f, void* workspace, size_t workspace_bytes,
+                             float* alpha_out, double* stats_out, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (!x || n <= 0 || !workspace || !alpha_out) return ESB_ERR_INVALID_ARG;
+    if (workspace_bytes < calibrate_workspace_bytes(n)) return ESB_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 7u) != 0) return ESB_ERR_ALIGN;
+    double as = 0.0;
+    alpha_star_cached(f.b, f.k, &as, nullptr);
+    cudaError_t e = launch_calibrate(x, n, f.is_signed, as, workspace, alpha_out, stats_out,
+                                     static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx, float alpha, const float* alpha_dev,
+                       esb_format f, int32_t rounding, uint32_t* codes, int64_t ldc, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (rows < 0 || cols < 0 || ldx < cols || ldc < words_for(cols, f.b)) return ESB_ERR_INVALID_ARG;
+    if (rounding != ESB_ROUND_HALF_AWAY && rounding != ESB_ROUND_HALF_EVEN) return ESB_ERR_INVALID_ARG;
+    if (!alpha_dev && !(std::isfinite(alpha) && alpha > 0.0f)) return ESB_ERR_INVALID_ARG;
+    if (rows == 0 || ldc == 0) return ESB_OK;
+    if (!codes || (cols > 0 && !x)) return ESB_ERR_INVALID_ARG;
+    cudaError_t e = launch_project(x, rows, cols, ldx, alpha, alpha_dev, f.b, f.k, f.is_signed, rounding, codes, ldc,
+                                   static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_t ldc, float alpha,
+                       const float* alpha_dev, esb_format f, float* y, int64_t ldy, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (rows < 0 || cols < 0 || ldc < words_for(cols, f.b) || ldy < cols) return ESB_ERR_INVALID_ARG;
+    if (!alpha_dev && !(std::isfinite(alpha) && alpha > 0.0f)) return ESB_ERR_INVALID_ARG;
+    if (rows == 0 || cols == 0) return ESB_OK;
+    if (!codes || !y) return ESB_ERR_INVALID_ARG;
+    cudaError_t e = launch_dequant(codes, rows, cols, ldc, alpha, alpha_dev, f.b, f.k, y, ldy,
+                                   static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, esb_format fa,
+                    const uint32_t* B, int64_t ldb, esb_format fb, const esb_epilogue* ep, int32_t* acc_out,
+                    float* y_out, uint32_t* codes_out, int64_t ldo, void* stream)
+{
+    if (!fmt_ok(fa) || !fmt_ok(fb)) return ESB_ERR_UNSUPPORTED;
+    if (M < 0 || N < 0 || K < 0) return ESB_ERR_INVALID_ARG;
+    if (lda < words_for(K, fa.b) || ldb < words_for(K, fb.b)) return ESB_ERR_INVALID_ARG;
+    if (!fmt_tc_ok(fa) || !fmt_tc_ok(fb)) return ESB_ERR_UNSUPPORTED;
+    const bool want_codes = codes_out != nullptr;
+    esb_status s = check_epilogue(ep, M, N, want_codes || y_out != nullptr);
+    if (s != ESB_OK) return s;
+    if (want_codes && ldo < words_for(N, ep->fmt_out.b)) return ESB_ERR_INVALID_ARG;
+    if ((double)K * fmt_max_image(fa.b, fa.k) * fmt_max_image(fb.b, fb.k) >= 16777216.0) return ESB_ERR_RANGE;
+    if (M > (int64_t)65535 * 128 * 256 || N > (int64_t)65535 * 16) return ESB_ERR_UNSUPPORTED;
+    if (M == 0 || N == 0) return ESB_OK;
+    if (!A || !B) return ESB_ERR_INVALID_ARG;
+    if (!acc_out && !y_out && !codes_out) return ESB_OK;
+    if (!aligned16(A) || !aligned16(B) || (lda & 3) || (ldb & 3)) return ESB_ERR_ALIGN;
+    if (!gemm_pick_ok(N, want_codes ? ep->fmt_out.b : 4)) return ESB_ERR_UNSUPPORTED;
+    GemmOutputs o{ep, acc_out, y_out, codes_out, ldo};
+    cudaError_t e = launch_gemm(M, N, K, A, lda, fa.b, fa.k, B, ldb, fb.b, fb.k, o, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_conv2d_nhwc(const esb_conv_desc* d, const uint32_t* X, int64_t ldx, esb_format fx, const uint32_t* W,
+                           int64_t ldw, esb_format fw, const esb_epilogue* ep, int32_t* acc_out, float* y_out,
+                           uint32_t* codes_out, int64_t ldo, void* stream)
+{
+    if (!d) return ESB_ERR_INVALID_ARG;
+    if (!fmt_ok(fx) || !fmt_ok(fw)) return ESB_ERR_UNSUPPORTED;
+    if (d->n < 0 || d->h <= 0 || d->w <= 0 || d->c <= 0 || d->cout <= 0 || d->r <= 0 || d->s <= 0 ||
+        d->stride <= 0 || d->pad < 0)
+        return ESB_ERR_INVALID_ARG;
+    if (d->h + 2 * d->pad < d->r || d->w + 2 * d->pad < d->s) return ESB_ERR_INVALID_ARG;
+    if (d->pad >= d->r || d->pad >= d->s) return ESB_ERR_INVALID_ARG;
+    if (ldx < words_for(d->c, fx.b) || ldw != ldx) return ESB_ERR_INVALID_ARG;
+    const int P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
+    const int Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
+    const int64_t M = (int64_t)d->n * P * Q;
+    const bool want_codes = codes_out != nullptr;
+    if (d->groups == d->c && d->c > 1) {
+        return ESB_ERR_UNSUPPORTED;  // depthwise path: not built yet
+    }
+    if (d->groups != 1) return ESB_ERR_UNSUPPORTED;
+    if (fx.b != fw.b) return ESB_ERR_UNSUPPORTED;
+    if (!fmt_tc_ok(fx) || !fmt_tc_ok(fw)) return ESB_ERR_UNSUPPORTED;
+    esb_status s = check_epilogue(ep, M, d->cout, want_codes || y_out != nullptr);
+    if (s != ESB_OK) return s;
+    if (want_codes && ldo < words_for(d->cout, ep->fmt_out.b)) return ESB_ERR_INVALID_ARG;
+    const int64_t K = (int64_t)d->r * d->s * ldx * (32 / fx.b);
+    if ((double)K * fmt_max_image(fx.b, fx.k) * fmt_max_image(fw.b, fw.k) >= 16777216.0) return ESB_ERR_RANGE;
+    if (M == 0) return ESB_OK;
+    if (!X || !W) return ESB_ERR_INVALID_ARG;
+    if (!acc_out && !y_out && !codes_out) return ESB_OK;
+    if (!aligned16(X) || !aligned16(W) || (ldx & 3)) return ESB_ERR_ALIGN;
+    if (M > (int64_t)65535 * 128 * 256) return ESB_ERR_UNSUPPORTED;
+    if (!gemm_pick_ok(d->cout, want_codes ? ep->fmt_out.b : 4)) return ESB_ERR_UNSUPPORTED;
+    GemmOutputs o{ep, acc_out, y_out, codes_out, ldo};
+    cudaError_t e = launch_conv_tc(*d, P, Q, X, ldx, fx.b, fx.k, W, ldw, fw.b, fw.k, o, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_get_status(void* stream, int32_t* device_status)
+{
+    if (!device_status) return ESB_ERR_INVALID_ARG;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return ESB_ERR_CUDA;
+    int v = 0;
+    if (cudaMemcpyFromSymbol(&v, esb::g_esb_device_status, sizeof(int)) != cudaSuccess) return ESB_ERR_CUDA;
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(esb::g_esb_device_status, &zero, sizeof(int)) != cudaSuccess) return ESB_ERR_CUDA;
+    *device_status = v;
+    return ESB_OK;
+}
+
+}  // extern "C"

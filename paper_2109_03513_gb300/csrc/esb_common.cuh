@@ -1,0 +1,287 @@
+// esb_common.cuh -- format arithmetic, the fp32-bit projection, and the
+// inline-PTX wrappers (mbarrier, tcgen05) shared by the kernels of libesb.
+//
+// ESB format: Sec. III-B (value set) and Sec. IV-A (float format) of
+// Gong et al., arXiv 2109.03513.  fmt = (b, k, signed), N = 2^(b-k-1) - 1,
+// code = sign | e (b-k-1 bits) | f (k bits); value = 0.f if e == N, else
+// 2^e * 1.f (units of alpha); integer image I = value * 2^k.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "esb.h"
+
+namespace esb {
+
+// ------------------------------------------------------------ format math
+
+__host__ __device__ inline int fmt_N(int b, int k) { return (1 << (b - k - 1)) - 1; }
+__host__ __device__ inline int fmt_ew(int b, int k) { return b - k - 1; }
+__host__ __device__ inline int fmt_cpw(int b) { return 32 / b; }
+__host__ __device__ inline uint32_t fmt_zero_code(int b, int k) { return (uint32_t)fmt_N(b, k) << k; }
+
+// Largest non-negative code: e = N-1, f = 2^k - 1 (or e = N = 0 when k = b-1).
+__host__ __device__ inline uint32_t fmt_max_code(int b, int k)
+{
+    int N = fmt_N(b, k);
+    uint32_t fmax = (1u << k) - 1u;
+    return N >= 1 ? (((uint32_t)(N - 1) << k) | fmax) : fmax;
+}
+
+// Largest integer image max|I| = (2^(k+1)-1) * 2^(N-1), or 2^k - 1 if N = 0.
+__host__ inline double fmt_max_image(int b, int k)
+{
+    int N = fmt_N(b, k);
+    if (N == 0) return (double)((1 << k) - 1);
+    double m = (double)((1 << (k + 1)) - 1);
+    for (int i = 0; i < N - 1; i++) m *= 2.0;
+    return m;
+}
+
+// C in units of alpha, the clip bound of Eq. cheap_projection.
+__host__ inline float fmt_C(int b, int k)
+{
+    double I = fmt_max_image(b, k);
+    double c = I;
+    for (int i = 0; i < k; i++) c *= 0.5;
+    return (float)c;   // exact: at most 8 significant bits
+}
+
+// ---------------------------------------------------- device status word
+
+// Kernels whose bounded waits give up record ESB_ERR_TIMEOUT in the
+// library's device status word (address passed as a kernel argument).
+__device__ __forceinline__ void record_status(int* status, int s)
+{
+    if (status) atomicCAS(status, 0, s);
+}
+
+// --------------------------------------------------------- projection
+
+struct ProjParams {
+    int b, k, is_signed, rounding;
+    int N;
+    uint32_t zero_code;
+    uint32_t max_code;   // non-negative code of C
+    uint32_t C_bits;     // fp32 bit pattern of C
+};
+
+__host__ inline ProjParams make_proj_params(int b, int k, int is_signed, int rounding)
+{
+    ProjParams p;
+    p.b = b; p.k = k; p.is_signed = is_signed; p.rounding = rounding;
+    p.N = fmt_N(b, k);
+    p.zero_code = fmt_zero_code(b, k);
+    p.max_code = fmt_max_code(b, k);
+    float C = fmt_C(b, k);
+    uint32_t cb;
+    __builtin_memcpy(&cb, &C, 4);
+    p.C_bits = cb;
+    return p;
+}
+
+// Code of v = x / alpha (already divided).  Eq. fast_projection on the
+// fp32 bits: the most significant 1 bit of |v| sets the binade n (values
+// below 1 use the spacing 2^-k of xi_0), the k+1 leading significant bits
+// are kept and the rest is rounded with one integer add and shift.  A
+// carry into the next binade is the next set element (f = 0, e + 1).
+__device__ __forceinline__ uint32_t project_scaled(float v, const ProjParams& p)
+{
+    const uint32_t u = __float_as_uint(v);
+    const uint32_t sign = u >> 31;
+    const uint32_t mag = u & 0x7fffffffu;
+    if (mag > 0x7f800000u) return p.zero_code;                 // NaN
+    if (sign && !p.is_signed) return p.zero_code;              // unsigned set: v < 0 -> 0
+    uint32_t code;
+    if (mag >= p.C_bits) {                                     // clip to C (incl. +-Inf)
+        code = p.max_code;
+    } else {
+        const int bexp = (int)(mag >> 23);
+        const uint32_t m24 = (mag & 0x7fffffu) | (bexp ? 0x800000u : 0u);
+        const int E = bexp ? bexp - 127 : -126;                // unbiased exponent
+        const int s = 23 - p.k - (E < 0 ? E : 0);              // bits to drop, >= 16
+        uint32_t r;
+        if (s > 24) {
+            r = 0u;                                            // below half a quantum
+        } else {
+            const uint32_t half = 1u << (s - 1);
+            const uint32_t add = p.rounding ? (half - 1u + ((m24 >> s) & 1u)) : half;
+            r = (m24 + add) >> s;
+        }
+        if (r == 0u) return p.zero_code;                       // zero carries sign 0
+        const uint32_t one = 1u << p.k;
+        uint32_t e, f;
+        if (E < 0) {                                           // r in [1, 2^k]
+            if (r < one) { e = (uint32_t)p.N; f = r; } else { e = 0u; f = 0u; }
+        } else {                                               // r in [2^k, 2^(k+1)]
+            if (r >= 2u * one) { e = (uint32_t)E + 1u; f = 0u; } else { e = (uint32_t)E; f = r - one; }
+        }
+        code = (e << p.k) | f;
+    }
+    return code | (sign << (p.b - 1));
+}
+
+__device__ __forceinline__ uint32_t project_code(float x, float alpha, const ProjParams& p)
+{
+    return project_scaled(__fdiv_rn(x, alpha), p);
+}
+
+// Value of a code in units of alpha (Sec. IV-A, Eq. q), exact in fp32 for b <= 8.
+__device__ __forceinline__ float code_value(uint32_t c, int b, int k)
+{
+    const int ew = b - k - 1;
+    const int N = (1 << ew) - 1;
+    const uint32_t s = (c >> (b - 1)) & 1u;
+    const uint32_t e = ew > 0 ? (c >> k) & ((1u << ew) - 1u) : 0u;
+    const uint32_t f = c & ((1u << k) - 1u);
+    const bool sub = (int)e == N;
+    const float m = (float)(sub ? f : ((1u << k) + f));
+    const float mag = ldexpf(m, (sub ? 0 : (int)e) - k);   // power-of-two scaling: exact
+    return s ? -mag : mag;
+}
+
+// Integer image of a code as float (exact; formats with max|I| < 2^24).
+__device__ __forceinline__ float code_image_f(uint32_t c, int b, int k)
+{
+    const int ew = b - k - 1;
+    const int N = (1 << ew) - 1;
+    const uint32_t s = (c >> (b - 1)) & 1u;
+    const uint32_t e = ew > 0 ? (c >> k) & ((1u << ew) - 1u) : 0u;
+    const uint32_t f = c & ((1u << k) - 1u);
+    const uint32_t mag = ((int)e == N) ? f : (((1u << k) + f) << e);
+    const float m = (float)mag;
+    return s ? -m : m;
+}
+
+// ------------------------------------------------------------- PTX helpers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init()
+{
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait: gives up after `limit_ns` of wall time (checked every 256
+// polls) and returns false; the caller records ESB_ERR_TIMEOUT.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, uint64_t limit_ns)
+{
+    const uint32_t a = smem_u32(bar);
+    if (mbar_try_wait(a, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try_wait(a, parity)) return true;
+        if ((it & 255u) == 0u && globaltimer_ns() - t0 > limit_ns) return false;
+    }
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// TMEM allocation (one full warp executes these).
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols)
+{
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                 ::"r"(smem_u32(slot)), "r"(ncols) : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
+{
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f8f6f4, issued by one thread.
+__device__ __forceinline__ void mma_f8f6f4(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                           uint32_t idesc, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive on an mbarrier once every previously issued tcgen05 op of this
+// thread has completed.
+__device__ __forceinline__ void mma_commit(uint64_t* bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+                 ::"r"(smem_u32(bar)) : "memory");
+}
+
+// 32 lanes x 16 columns of 32-bit TMEM words into 16 registers per thread.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor for a K-major operand in the 128-byte
+// swizzled layout: rows of 128 bytes, 8-row atoms of 1024 bytes (SBO).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);        // start address
+    d |= (uint64_t)1u << 16;                         // LBO (unused for swizzled K-major)
+    d |= (uint64_t)(1024u >> 4) << 32;               // SBO: 8 rows x 128 B
+    d |= (uint64_t)1u << 46;                         // descriptor version (sm_100 family)
+    d |= (uint64_t)2u << 61;                         // swizzle: 128 B
+    return d;
+}
+
+// Instruction descriptor: kind::f8f6f4, A = B = E4M3, D = F32, K-major
+// operands, M = 128, N = n.
+__host__ __device__ inline uint32_t idesc_e4m3_f32(int n)
+{
+    uint32_t d = 0;
+    d |= 1u << 4;                       // D format: F32
+    d |= 0u << 7;                       // A format: E4M3
+    d |= 0u << 10;                      // B format: E4M3
+    d |= (uint32_t)(n >> 3) << 17;      // N >> 3
+    d |= (uint32_t)(128 >> 4) << 24;    // M >> 4
+    return d;
+}
+
+}  // namespace esb

@@ -1,0 +1,48 @@
+// esb_internal.h -- launchers and host helpers shared by the libesb sources
+// (not part of the public C ABI).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "esb.h"
+
+namespace esb {
+
+int device_sm_count();
+
+// Device address of the library status word on the current device.
+int* device_status_ptr();
+
+cudaError_t launch_project(const float* x, int64_t rows, int64_t cols, int64_t ldx, float alpha,
+                           const float* alpha_dev, int b, int k, int is_signed, int rounding,
+                           uint32_t* codes, int64_t ldc, cudaStream_t st);
+
+cudaError_t launch_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_t ldc, float alpha,
+                           const float* alpha_dev, int b, int k, float* y, int64_t ldy, cudaStream_t st);
+
+size_t calibrate_workspace_bytes(int64_t n);
+cudaError_t launch_calibrate(const float* x, int64_t n, int is_signed, double alpha_star, void* workspace,
+                             float* alpha_out, double* stats_out, cudaStream_t st);
+
+struct GemmOutputs {
+    const esb_epilogue* ep;
+    int32_t* acc_out;
+    float* y_out;
+    uint32_t* codes_out;
+    int64_t ldo;
+};
+
+cudaError_t launch_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, int ba, int ka,
+                        const uint32_t* B, int64_t ldb, int bb, int kb, const GemmOutputs& o, cudaStream_t st);
+
+cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
+                           const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st);
+
+bool gemm_pick_ok(int64_t N, int out_b);
+
+// alpha*(b,k) and 2*D(alpha*) (Sec. III-D), solved on the host in fp64.
+double alpha_star_solve(int b, int k, double* dda);
+
+}  // namespace esb

@@ -1,0 +1,319 @@
+// esb_quant.cu -- HBM-bound element-wise kernels of libesb:
+//   * projection of fp32 tensors onto packed ESB codes (Eq. cheap_projection
+//     with the shift-and-round projection of Eq. fast_projection),
+//   * dequantisation (Sec. IV-A, Eq. q),
+//   * DDA calibration statistics and alpha (Sec. III-D).
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "esb_common.cuh"
+#include "esb_internal.h"
+
+namespace esb {
+
+// ----------------------------------------------------------- projection
+
+// Fast path: one thread turns 4*cpw consecutive floats of a row into 4
+// code words (one 16-byte store); cpw float4 loads in flight per thread,
+// streaming cache hints since every byte is touched once.
+template <int B>
+__global__ void __launch_bounds__(256)
+project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int64_t ldx,
+                   float alpha, const float* __restrict__ alpha_dev, ProjParams p,
+                   uint32_t* __restrict__ codes, int64_t ldc)
+{
+    constexpr int CPW = 32 / B;
+    const float a = alpha_dev ? __ldg(alpha_dev) : alpha;
+    const int64_t upr = ldc >> 2;                 // 4-word units per row
+    const int64_t total = rows * upr;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < total; u += stride) {
+        const int64_t r = (rows == 1) ? 0 : u / upr;
+        const int64_t w4 = u - r * upr;
+        const int64_t c0 = w4 * (4 * CPW);
+        const float* xr = x + r * ldx + c0;
+        uint32_t out[4];
+        if (c0 + 4 * CPW <= cols) {
+            float v[4 * CPW];
+#pragma unroll
+            for (int i = 0; i < CPW; i++) {
+                const float4 t = __ldcs(reinterpret_cast<const float4*>(xr) + i);
+                v[4 * i + 0] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
+            }
+#pragma unroll
+            for (int w = 0; w < 4; w++) {
+                uint32_t word = 0;
+#pragma unroll
+                for (int j = 0; j < CPW; j++) word |= project_code(v[w * CPW + j], a, p) << (B * j);
+                out[w] = word;
+            }
+        } else {
+#pragma unroll
+            for (int w = 0; w < 4; w++) {
+                uint32_t word = 0;
+#pragma unroll
+                for (int j = 0; j < CPW; j++) {
+                    const int64_t c = c0 + w * CPW + j;
+                    const uint32_t code = (c < cols) ? project_code(__ldcs(xr + w * CPW + j), a, p) : p.zero_code;
+                    word |= code << (B * j);
+                }
+                out[w] = word;
+            }
+        }
+        __stcs(reinterpret_cast<uint4*>(codes + r * ldc + (w4 << 2)), make_uint4(out[0], out[1], out[2], out[3]));
+    }
+}
+
+// General path: any alignment and strides; one thread per code word.
+template <int B>
+__global__ void __launch_bounds__(256)
+project_any_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int64_t ldx,
+                   float alpha, const float* __restrict__ alpha_dev, ProjParams p,
+                   uint32_t* __restrict__ codes, int64_t ldc)
+{
+    constexpr int CPW = 32 / B;
+    const float a = alpha_dev ? __ldg(alpha_dev) : alpha;
+    const int64_t total = rows * ldc;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < total; u += stride) {
+        const int64_t r = u / ldc;
+        const int64_t w = u - r * ldc;
+        uint32_t word = 0;
+#pragma unroll
+        for (int j = 0; j < CPW; j++) {
+            const int64_t c = w * CPW + j;
+            const uint32_t code = (c < cols) ? project_code(x[r * ldx + c], a, p) : p.zero_code;
+            word |= code << (B * j);
+        }
+        codes[u] = word;  // row-major: r * ldc + w == u
+    }
+}
+
+template <int B>
+static cudaError_t launch_project_b(const float* x, int64_t rows, int64_t cols, int64_t ldx, float alpha,
+                                    const float* alpha_dev, const ProjParams& p, uint32_t* codes,
+                                    int64_t ldc, bool vec, int sms, cudaStream_t st)
+{
+    const int threads = 256;
+    if (vec) {
+        const int64_t units = rows * (ldc >> 2);
+        int64_t blocks = (units + threads - 1) / threads;
+        const int64_t cap = (int64_t)sms * 8;
+        if (blocks > cap) blocks = cap;
+        if (blocks < 1) blocks = 1;
+        project_vec_kernel<B><<<(unsigned)blocks, threads, 0, st>>>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc);
+    } else {
+        const int64_t units = rows * ldc;
+        int64_t blocks = (units + threads - 1) / threads;
+        const int64_t cap = (int64_t)sms * 8;
+        if (blocks > cap) blocks = cap;
+        if (blocks < 1) blocks = 1;
+        project_any_kernel<B><<<(unsigned)blocks, threads, 0, st>>>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_project(const float* x, int64_t rows, int64_t cols, int64_t ldx, float alpha,
+                           const float* alpha_dev, int b, int k, int is_signed, int rounding,
+                           uint32_t* codes, int64_t ldc, cudaStream_t st)
+{
+    const ProjParams p = make_proj_params(b, k, is_signed, rounding);
+    const bool vec = ((reinterpret_cast<uintptr_t>(x) & 15u) == 0) && ((reinterpret_cast<uintptr_t>(codes) & 15u) == 0)
+                     && (ldx % 4 == 0) && (ldc % 4 == 0);
+    const int sms = device_sm_count();
+    switch (b) {
+    case 2: return launch_project_b<2>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc, vec, sms, st);
+    case 3: return launch_project_b<3>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc, vec, sms, st);
+    case 4: return launch_project_b<4>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc, vec, sms, st);
+    case 5: return launch_project_b<5>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc, vec, sms, st);
+    case 6: return launch_project_b<6>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc, vec, sms, st);
+    case 7: return launch_project_b<7>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc, vec, sms, st);
+    default: return launch_project_b<8>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc, vec, sms, st);
+    }
+}
+
+// ------------------------------------------------------------ dequant
+
+__global__ void __launch_bounds__(256)
+dequant_kernel(const uint32_t* __restrict__ codes, int64_t rows, int64_t cols, int64_t ldc, float alpha,
+               const float* __restrict__ alpha_dev, int b, int k, float* __restrict__ y, int64_t ldy)
+{
+    const float a = alpha_dev ? __ldg(alpha_dev) : alpha;
+    const int cpw = 32 / b;
+    const uint32_t mask = (1u << b) - 1u;
+    const int64_t total = rows * cols;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += stride) {
+        const int64_t r = i / cols;
+        const int64_t c = i - r * cols;
+        const uint32_t code = (codes[r * ldc + c / cpw] >> (b * (int)(c % cpw))) & mask;
+        y[r * ldy + c] = __fmul_rn(a, code_value(code, b, k));
+    }
+}
+
+cudaError_t launch_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_t ldc, float alpha,
+                           const float* alpha_dev, int b, int k, float* y, int64_t ldy, cudaStream_t st)
+{
+    const int threads = 256;
+    int64_t blocks = (rows * cols + threads - 1) / threads;
+    const int64_t cap = (int64_t)device_sm_count() * 8;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    dequant_kernel<<<(unsigned)blocks, threads, 0, st>>>(codes, rows, cols, ldc, alpha, alpha_dev, b, k, y, ldy);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------- DDA calibration
+
+// Pass 1.  The data is cut into chunks of 32 values.  Each thread keeps, in
+// fp64, the sums over its full chunks of a_c, a_c^2 and M2_c, where a_c is
+// the fp32 chunk mean and M2_c = sum (x - a_c)^2 in fp32 (both from the
+// chunk held in registers); partial chunks carry their count as a weight.
+// The law of total variance then gives mean and sigma from these sums with
+// no catastrophic cancellation inside a chunk.  Per-block partials go to
+// the workspace in a fixed layout; the finalize kernel adds them in a fixed
+// order, so the result does not depend on scheduling.
+constexpr int kCalThreads = 256;
+constexpr int kCalChunk = 32;
+constexpr int kCalMaxBlocks = 1024;
+
+struct CalPartial {
+    double n, s1, s2, s3;   // sum n_c, sum n_c a_c, sum n_c a_c^2, sum M2_c
+};
+
+__device__ __forceinline__ void cal_warp_sum(double& v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+}
+
+__global__ void __launch_bounds__(kCalThreads)
+calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalPartial* __restrict__ part)
+{
+    const int64_t nfull = n / kCalChunk;
+    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
+    double s1 = 0.0, s2 = 0.0, s3 = 0.0, cnt = 0.0;
+    for (int64_t c = tid; c < nfull; c += nthreads) {
+        float v[kCalChunk];
+        const float* xc = x + c * kCalChunk;
+        if (vec) {
+#pragma unroll
+            for (int i = 0; i < kCalChunk / 4; i++) {
+                const float4 t = __ldcs(reinterpret_cast<const float4*>(xc) + i);
+                v[4 * i] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < kCalChunk; i++) v[i] = __ldcs(xc + i);
+        }
+        float s = 0.0f;
+#pragma unroll
+        for (int i = 0; i < kCalChunk; i++) s += v[i];
+        const float a = s * (1.0f / kCalChunk);
+        float m2 = 0.0f;
+#pragma unroll
+        for (int i = 0; i < kCalChunk; i++) { const float d = v[i] - a; m2 = fmaf(d, d, m2); }
+        s1 += (double)a;
+        s2 = fma((double)a, (double)a, s2);
+        s3 += (double)m2;
+        cnt += 1.0;
+    }
+    double n_all = cnt * kCalChunk;
+    s1 *= kCalChunk;
+    s2 *= kCalChunk;
+    // The ragged tail (< 32 values) is one weighted chunk, owned by thread 0.
+    const int64_t tail0 = nfull * kCalChunk;
+    if (tid == 0 && tail0 < n) {
+        const int nt = (int)(n - tail0);
+        float s = 0.0f;
+        for (int i = 0; i < nt; i++) s += x[tail0 + i];
+        const float a = s / (float)nt;
+        float m2 = 0.0f;
+        for (int i = 0; i < nt; i++) { const float d = x[tail0 + i] - a; m2 = fmaf(d, d, m2); }
+        n_all += nt;
+        s1 += (double)nt * (double)a;
+        s2 += (double)nt * (double)a * (double)a;
+        s3 += (double)m2;
+    }
+    cal_warp_sum(n_all); cal_warp_sum(s1); cal_warp_sum(s2); cal_warp_sum(s3);
+    __shared__ CalPartial sh[kCalThreads / 32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) sh[warp] = CalPartial{n_all, s1, s2, s3};
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        CalPartial t{0.0, 0.0, 0.0, 0.0};
+        for (int w = 0; w < kCalThreads / 32; w++) {
+            t.n += sh[w].n; t.s1 += sh[w].s1; t.s2 += sh[w].s2; t.s3 += sh[w].s3;
+        }
+        part[blockIdx.x] = t;
+    }
+}
+
+// Pass 2 (one block): fixed-order sum of the block partials, then
+// mean = s1/n, M2 = s3 + (s2 - s1^2/n), sigma = sqrt(M2/n) (signed formats)
+// or rms = sqrt((s3 + s2)/n) (unsigned formats), alpha = fl32(alpha* (spread + 1e-7)).
+__global__ void __launch_bounds__(kCalThreads)
+calibrate_finalize_kernel(const CalPartial* __restrict__ part, int nblocks, double alpha_star, int is_signed,
+                          float* __restrict__ alpha_out, double* __restrict__ stats_out)
+{
+    __shared__ CalPartial sh[kCalThreads];
+    CalPartial t{0.0, 0.0, 0.0, 0.0};
+    for (int i = threadIdx.x; i < nblocks; i += kCalThreads) {
+        t.n += part[i].n; t.s1 += part[i].s1; t.s2 += part[i].s2; t.s3 += part[i].s3;
+    }
+    sh[threadIdx.x] = t;
+    __syncthreads();
+    for (int h = kCalThreads / 2; h > 0; h >>= 1) {
+        if (threadIdx.x < h) {
+            sh[threadIdx.x].n += sh[threadIdx.x + h].n;
+            sh[threadIdx.x].s1 += sh[threadIdx.x + h].s1;
+            sh[threadIdx.x].s2 += sh[threadIdx.x + h].s2;
+            sh[threadIdx.x].s3 += sh[threadIdx.x + h].s3;
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        const CalPartial r = sh[0];
+        const double mean = r.s1 / r.n;
+        double spread;
+        if (is_signed) {
+            double m2 = r.s3 + (r.s2 - r.s1 * mean);
+            if (m2 < 0.0) m2 = 0.0;
+            spread = sqrt(m2 / r.n);
+        } else {
+            spread = sqrt((r.s3 + r.s2) / r.n);
+        }
+        *alpha_out = (float)(alpha_star * (spread + 1e-7));
+        if (stats_out) { stats_out[0] = mean; stats_out[1] = spread; stats_out[2] = r.n; }
+    }
+}
+
+int calibrate_blocks(int64_t n)
+{
+    const int64_t per_block = (int64_t)kCalThreads * kCalChunk;
+    int64_t g = (n + per_block - 1) / per_block;
+    if (g > kCalMaxBlocks) g = kCalMaxBlocks;
+    if (g < 1) g = 1;
+    return (int)g;
+}
+
+size_t calibrate_workspace_bytes(int64_t n)
+{
+    return (size_t)calibrate_blocks(n) * sizeof(CalPartial);
+}
+
+cudaError_t launch_calibrate(const float* x, int64_t n, int is_signed, double alpha_star, void* workspace,
+                             float* alpha_out, double* stats_out, cudaStream_t st)
+{
+    const int g = calibrate_blocks(n);
+    const int vec = ((reinterpret_cast<uintptr_t>(x) & 15u) == 0) ? 1 : 0;
+    CalPartial* part = static_cast<CalPartial*>(workspace);
+    calibrate_pass1_kernel<<<g, kCalThreads, 0, st>>>(x, n, vec, part);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    calibrate_finalize_kernel<<<1, kCalThreads, 0, st>>>(part, g, alpha_star, is_signed, alpha_out, stats_out);
+    return cudaGetLastError();
+}
+
+}  // namespace esb

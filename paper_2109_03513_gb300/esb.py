@@ -1,0 +1,329 @@
+"""ctypes binding of libesb.so -- the C ABI declared in include/esb.h.
+
+Argument marshalling only: every step of the ESB path runs in the library's
+CUDA kernels.  PyTorch supplies device memory and streams.  Packed code
+tensors are torch.int32 tensors whose bits are the uint32 code words.
+If the library is missing this module raises; there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libesb.so")
+
+ESB_OK = 0
+ESB_ERR_INVALID_ARG = 1
+ESB_ERR_UNSUPPORTED = 2
+ESB_ERR_RANGE = 3
+ESB_ERR_ALIGN = 4
+ESB_ERR_CUDA = 5
+ESB_ERR_TIMEOUT = 6
+
+ESB_ROUND_HALF_AWAY = 0
+ESB_ROUND_HALF_EVEN = 1
+ESB_ACT_NONE = 0
+ESB_ACT_RELU = 1
+ESB_ACT_RELU6 = 2
+
+
+class EsbError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: esb_status {status}")
+
+
+class esb_format(ctypes.Structure):
+    _fields_ = [("b", ctypes.c_int32), ("k", ctypes.c_int32), ("is_signed", ctypes.c_int32)]
+
+
+class esb_epilogue(ctypes.Structure):
+    _fields_ = [
+        ("scale", ctypes.c_void_p), ("bias", ctypes.c_void_p),
+        ("scale0", ctypes.c_float), ("bias0", ctypes.c_float),
+        ("act", ctypes.c_int32),
+        ("residual", ctypes.c_void_p), ("res_ld", ctypes.c_int64), ("res_fmt", esb_format),
+        ("res_scale", ctypes.c_float),
+        ("alpha_out", ctypes.c_float), ("alpha_out_dev", ctypes.c_void_p),
+        ("fmt_out", esb_format), ("rounding_out", ctypes.c_int32),
+    ]
+
+
+class esb_conv_desc(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("n", "h", "w", "c", "cout", "r", "s", "stride", "pad", "groups")]
+
+
+@dataclass(frozen=True)
+class Fmt:
+    """ESB format: b total bits, k fraction bits (k+1 significant bits)."""
+    b: int
+    k: int
+    signed: bool = True
+
+    def c(self) -> esb_format:
+        return esb_format(self.b, self.k, 1 if self.signed else 0)
+
+
+_lib = None
+
+# (name, restype, argtypes) of every exported symbol of include/esb.h.
+_P, _I32, _I64, _F32, _SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+SIGNATURES = {
+    "esb_version": (_I32, []),
+    "esb_status_string": (ctypes.c_char_p, [_I32]),
+    "esb_format_check": (_I32, [esb_format]),
+    "esb_codes_per_word": (_I32, [_I32]),
+    "esb_row_words": (_I64, [_I64, _I32]),
+    "esb_zero_code": (ctypes.c_uint32, [esb_format]),
+    "esb_alpha_star": (_I32, [_I32, _I32, _P, _P]),
+    "esb_calibrate_dda_workspace_bytes": (_SZ, [_I64]),
+    "esb_calibrate_dda": (_I32, [_P, _I64, esb_format, _P, _SZ, _P, _P, _P]),
+    "esb_project": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _I32, _P, _I64, _P]),
+    "esb_dequant": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _P, _I64, _P]),
+    "esb_gemm": (_I32, [_I64, _I64, _I64, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
+    "esb_conv2d_nhwc": (_I32, [_P, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
+    "esb_get_status": (_I32, [_P, _P]),
+}
+
+
+def lib():
+    """Load libesb.so (built by __graft_entry__.build()).  Raises if absent."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libesb.so not built ({LIB_PATH}); run __graft_entry__.build()")
+        l = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(l, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = l
+    return _lib
+
+
+def _check(st: int, where: str):
+    if st != ESB_OK:
+        raise EsbError(st, where)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t: torch.Tensor, name: str):
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+# ------------------------------------------------------------------ info
+
+def esb_version() -> int:
+    return int(lib().esb_version())
+
+
+def esb_codes_per_word(b: int) -> int:
+    return int(lib().esb_codes_per_word(b))
+
+
+def esb_row_words(cols: int, b: int) -> int:
+    return int(lib().esb_row_words(cols, b))
+
+
+def esb_zero_code(f: Fmt) -> int:
+    return int(lib().esb_zero_code(f.c()))
+
+
+def esb_alpha_star(b: int, k: int) -> tuple[float, float]:
+    a = ctypes.c_double(0.0)
+    d = ctypes.c_double(0.0)
+    _check(lib().esb_alpha_star(b, k, ctypes.byref(a), ctypes.byref(d)), "esb_alpha_star")
+    return a.value, d.value
+
+
+# ------------------------------------------------------------- calibrate
+
+def esb_calibrate_dda(x: torch.Tensor, f: Fmt, alpha_out: Optional[torch.Tensor] = None,
+                      stats_out: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
+                      stream=None) -> tuple[torch.Tensor, Optional[torch.Tensor]]:
+    """Device alpha (1 float) and stats {mean, spread, n} of x (Sec. III-D)."""
+    _dev(x, "x")
+    assert x.dtype == torch.float32
+    n = x.numel()
+    if alpha_out is None:
+        alpha_out = torch.empty(1, dtype=torch.float32, device=x.device)
+    if workspace is None:
+        nb = int(lib().esb_calibrate_dda_workspace_bytes(n))
+        workspace = torch.empty(max(nb, 8), dtype=torch.uint8, device=x.device)
+    _check(lib().esb_calibrate_dda(_ptr(x), n, f.c(), _ptr(workspace), workspace.numel(), _ptr(alpha_out),
+                                   _ptr(stats_out), _stream(stream)), "esb_calibrate_dda")
+    return alpha_out, stats_out
+
+
+def esb_calibrate_dda_workspace_bytes(n: int) -> int:
+    return int(lib().esb_calibrate_dda_workspace_bytes(n))
+
+
+# --------------------------------------------------------------- project
+
+def esb_project(x: torch.Tensor, f: Fmt, alpha=None, rounding: int = ESB_ROUND_HALF_AWAY,
+                codes: Optional[torch.Tensor] = None, ldc: Optional[int] = None, stream=None) -> torch.Tensor:
+    """Project a (rows, cols) or 1-D fp32 tensor to packed codes (rows, ldc) int32.
+    alpha: python float or a 1-element CUDA float tensor (read on the device)."""
+    _dev(x, "x")
+    assert x.dtype == torch.float32
+    x2 = x.reshape(1, -1) if x.dim() == 1 else x.reshape(-1, x.shape[-1])
+    rows, cols = x2.shape
+    if ldc is None:
+        ldc = esb_row_words(cols, f.b)
+    if codes is None:
+        codes = torch.empty((rows, ldc), dtype=torch.int32, device=x.device)
+    a_host, a_dev = (float(alpha), None) if not isinstance(alpha, torch.Tensor) else (0.0, alpha)
+    _check(lib().esb_project(_ptr(x2), rows, cols, cols, a_host, _ptr(a_dev), f.c(), rounding, _ptr(codes), ldc,
+                             _stream(stream)), "esb_project")
+    return codes
+
+
+def esb_dequant(codes: torch.Tensor, cols: int, f: Fmt, alpha, stream=None) -> torch.Tensor:
+    _dev(codes, "codes")
+    c2 = codes.reshape(-1, codes.shape[-1])
+    rows, ldc = c2.shape
+    y = torch.empty((rows, cols), dtype=torch.float32, device=codes.device)
+    a_host, a_dev = (float(alpha), None) if not isinstance(alpha, torch.Tensor) else (0.0, alpha)
+    _check(lib().esb_dequant(_ptr(c2), rows, cols, ldc, a_host, _ptr(a_dev), f.c(), _ptr(y), cols, _stream(stream)),
+           "esb_dequant")
+    return y
+
+
+# ------------------------------------------------------------------ gemm
+
+@dataclass
+class Epilogue:
+    """Fused post-processing (include/esb.h, esb_epilogue)."""
+    scale: Optional[torch.Tensor] = None
+    bias: Optional[torch.Tensor] = None
+    scale0: float = 1.0
+    bias0: float = 0.0
+    act: int = ESB_ACT_NONE
+    residual: Optional[torch.Tensor] = None
+    res_fmt: Optional[Fmt] = None
+    res_scale: float = 0.0
+    alpha_out: float = 1.0
+    alpha_out_dev: Optional[torch.Tensor] = None
+    fmt_out: Fmt = Fmt(4, 2, True)
+    rounding_out: int = ESB_ROUND_HALF_AWAY
+
+    def c(self) -> esb_epilogue:
+        e = esb_epilogue()
+        e.scale = None if self.scale is None else self.scale.data_ptr()
+        e.bias = None if self.bias is None else self.bias.data_ptr()
+        e.scale0 = self.scale0
+        e.bias0 = self.bias0
+        e.act = self.act
+        if self.residual is not None:
+            e.residual = self.residual.data_ptr()
+            e.res_ld = self.residual.shape[-1]
+            e.res_fmt = self.res_fmt.c()
+        e.res_scale = self.res_scale
+        e.alpha_out = self.alpha_out
+        e.alpha_out_dev = None if self.alpha_out_dev is None else self.alpha_out_dev.data_ptr()
+        e.fmt_out = self.fmt_out.c()
+        e.rounding_out = self.rounding_out
+        return e
+
+
+def esb_gemm(A: torch.Tensor, fa: Fmt, B: torch.Tensor, fb: Fmt, K: int, ep: Optional[Epilogue] = None,
+             want_acc: bool = True, want_y: bool = False, want_codes: bool = False,
+             out_acc: Optional[torch.Tensor] = None, out_y: Optional[torch.Tensor] = None,
+             out_codes: Optional[torch.Tensor] = None, stream=None):
+    """(acc int32 (M,N) | None, y fp32 (M,N) | None, codes int32 (M, ldo) | None)."""
+    _dev(A, "A"); _dev(B, "B")
+    M, lda = A.shape
+    N, ldb = B.shape
+    dev = A.device
+    acc = out_acc if out_acc is not None else (torch.empty((M, N), dtype=torch.int32, device=dev) if want_acc else None)
+    y = out_y if out_y is not None else (torch.empty((M, N), dtype=torch.float32, device=dev) if want_y else None)
+    codes = out_codes
+    if codes is None and want_codes:
+        codes = torch.empty((M, esb_row_words(N, ep.fmt_out.b)), dtype=torch.int32, device=dev)
+    ldo = codes.shape[-1] if codes is not None else 0
+    epc = ep.c() if ep is not None else None
+    _check(lib().esb_gemm(M, N, K, _ptr(A), lda, fa.c(), _ptr(B), ldb, fb.c(),
+                          ctypes.byref(epc) if epc is not None else None,
+                          _ptr(acc), _ptr(y), _ptr(codes), ldo, _stream(stream)), "esb_gemm")
+    return acc, y, codes
+
+
+def conv_out_hw(h: int, w: int, r: int, s: int, stride: int, pad: int) -> tuple[int, int]:
+    return (h + 2 * pad - r) // stride + 1, (w + 2 * pad - s) // stride + 1
+
+
+def esb_conv2d_nhwc(X: torch.Tensor, fx: Fmt, W: torch.Tensor, fw: Fmt, n: int, h: int, w: int, c: int, cout: int,
+                    r: int, s: int, stride: int, pad: int, groups: int = 1, ep: Optional[Epilogue] = None,
+                    want_acc: bool = True, want_y: bool = False, want_codes: bool = False,
+                    out_acc: Optional[torch.Tensor] = None, out_y: Optional[torch.Tensor] = None,
+                    out_codes: Optional[torch.Tensor] = None, stream=None):
+    """NHWC conv on packed codes.  X: (n*h*w, ldx) int32; W: (cout*r*s, ldx) int32
+    (depthwise: (r*s, ldx)).  Outputs are (n*P*Q, cout)-shaped."""
+    _dev(X, "X"); _dev(W, "W")
+    ldx = X.shape[-1]
+    ldw = W.shape[-1]
+    P, Q = conv_out_hw(h, w, r, s, stride, pad)
+    M = n * P * Q
+    dev = X.device
+    acc = out_acc if out_acc is not None else (torch.empty((M, cout), dtype=torch.int32, device=dev) if want_acc else None)
+    y = out_y if out_y is not None else (torch.empty((M, cout), dtype=torch.float32, device=dev) if want_y else None)
+    codes = out_codes
+    if codes is None and want_codes:
+        codes = torch.empty((M, esb_row_words(cout, ep.fmt_out.b)), dtype=torch.int32, device=dev)
+    ldo = codes.shape[-1] if codes is not None else 0
+    d = esb_conv_desc(n, h, w, c, cout, r, s, stride, pad, groups)
+    epc = ep.c() if ep is not None else None
+    _check(lib().esb_conv2d_nhwc(ctypes.byref(d), _ptr(X), ldx, fx.c(), _ptr(W), ldw, fw.c(),
+                                 ctypes.byref(epc) if epc is not None else None,
+                                 _ptr(acc), _ptr(y), _ptr(codes), ldo, _stream(stream)), "esb_conv2d_nhwc")
+    return acc, y, codes
+
+
+def esb_get_status(stream=None) -> int:
+    v = ctypes.c_int32(0)
+    _check(lib().esb_get_status(_stream(stream), ctypes.byref(v)), "esb_get_status")
+    return int(v.value)
+
+
+# ------------------------------------------------------------ host helpers
+
+def default_scale(alpha_a: float, fa: Fmt, alpha_b: float, fb: Fmt) -> float:
+    """fp32 multiplier turning the integer accumulator into the real product:
+    alpha_a * 2^-ka * alpha_b * 2^-kb (one fp32 rounding of alpha_a * alpha_b)."""
+    import numpy as np
+    return float(np.float32(np.float32(alpha_a) * np.float32(alpha_b)) * np.float32(2.0 ** -(fa.k + fb.k)))
+
+
+def fold_bn_dn(alpha_w: float, kw: int, alpha_a: float, ka: int, bn_mean, bn_std, bn_gamma, bn_beta,
+               dn_mean: float, dn_std: float):
+    """Sec. IV-C "BN and DN" fold for this library's epilogue.  The paper folds
+    Scale, BN and DN (and the division by the next layer's alpha) into one
+    affine a*x + b of the accumulator x; here the division by alpha_out stays
+    in the requantisation, so scale[n] = alpha_out * a_n and bias[n] = alpha_out * b_n:
+      scale = alpha_w 2^-kw alpha_a 2^-ka gamma / (sigma_BN sigma_DN)
+      bias  = (sigma_BN beta - mu_BN gamma - sigma_BN mu_DN) / (sigma_DN sigma_BN)
+    Returns float64 numpy arrays (cast to fp32 by the caller)."""
+    import numpy as np
+    bn_mean, bn_std, bn_gamma, bn_beta = (np.asarray(v, dtype=np.float64) for v in (bn_mean, bn_std, bn_gamma, bn_beta))
+    s = (alpha_w * 2.0 ** -kw) * (alpha_a * 2.0 ** -ka)
+    scale = s * bn_gamma / (bn_std * dn_std)
+    bias = (bn_std * bn_beta - bn_mean * bn_gamma - bn_std * dn_mean) / (dn_std * bn_std)
+    return scale, bias

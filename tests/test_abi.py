@@ -1,0 +1,125 @@
+"""C-ABI library: loads, exports every declared symbol, host-only entry
+points and host-side validation (no device work; runs without a GPU)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle as o
+from conftest import ROOT, read_golden
+from paper_2109_03513_gb300 import esb
+
+HEADER = os.path.join(ROOT, "include", "esb.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import __graft_entry__
+    __graft_entry__.build()
+    return esb.lib()
+
+
+def declared_functions():
+    txt = open(HEADER).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"^\s*[A-Za-z_][A-Za-z0-9_ ]*?[\s\*]+(esb_[a-z0-9_]+)\s*\(", txt, flags=re.M)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert len(names) >= 14
+    for n in names:
+        assert hasattr(lib, n), n
+        assert n in esb.SIGNATURES, n
+    assert set(esb.SIGNATURES) == set(names)
+
+
+def test_info_functions(lib):
+    assert esb.esb_version() >= 100
+    for b in range(2, 9):
+        assert esb.esb_codes_per_word(b) == 32 // b
+        for k in range(0, b):
+            assert esb.esb_zero_code(esb.Fmt(b, k)) == o.zero_code(b, k)
+        for cols in (0, 1, 37, 64, 576):
+            rw = esb.esb_row_words(cols, b)
+            assert rw % 4 == 0 and rw * (32 // b) >= cols and (rw - 4) * (32 // b) < max(cols, 1)
+    assert esb.esb_codes_per_word(9) == 0
+    assert lib.esb_status_string(3) == b"exactness bound exceeded"
+
+
+@pytest.mark.parametrize("row", read_golden("table1_alpha_dda.txt"))
+def test_library_alpha_star_matches_table1(lib, row):
+    b, k, dda, astar = int(row[0]), int(row[1]), float(row[2]), float(row[3])
+    a, d = esb.esb_alpha_star(b, k)
+    assert abs(a - astar) <= 5e-5 + 1e-12
+    assert abs(d - dda) <= 5e-5 + 1e-12
+    ao, _ = o.alpha_star(b, k)
+    assert abs(a - ao) <= 1e-9 * ao
+
+
+def test_library_alpha_star_other_formats(lib):
+    for b in range(2, 8):
+        for k in range(0, b):
+            a, _ = esb.esb_alpha_star(b, k)
+            ao, _ = o.alpha_star(b, k)
+            assert abs(a - ao) <= 1e-9 * ao, (b, k, a, ao)
+
+
+def test_host_validation_without_device(lib):
+    f = esb.esb_format(4, 2, 1)
+    bad = esb.esb_format(9, 2, 1)
+    null = None
+    fake = ctypes.c_void_p(4096)
+    # unsupported / invalid formats and sizes are rejected before any launch
+    assert lib.esb_project(fake, 1, 8, 8, 1.0, null, bad, 0, fake, 4, null) == esb.ESB_ERR_UNSUPPORTED
+    assert lib.esb_project(fake, 1, 8, 8, 0.0, null, f, 0, fake, 4, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_project(fake, 1, 8, 8, float("nan"), null, f, 0, fake, 4, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_project(fake, 1, 8, 8, 1.0, null, f, 7, fake, 4, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_project(fake, 1, 64, 64, 1.0, null, f, 0, fake, 7, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_project(fake, 0, 8, 8, 1.0, null, f, 0, fake, 4, null) == esb.ESB_OK
+    assert lib.esb_calibrate_dda(fake, 0, f, fake, 64, fake, null, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_calibrate_dda(fake, 100, f, ctypes.c_void_p(4097), 1 << 20, fake, null, null) == esb.ESB_ERR_ALIGN
+    assert lib.esb_calibrate_dda(fake, 100, f, fake, 1, fake, null, null) == esb.ESB_ERR_INVALID_ARG
+    # contraction: exactness bound and unsupported formats
+    big = esb.esb_format(6, 3, 1)
+    ep = esb.Epilogue().c()
+    assert lib.esb_gemm(128, 64, 8192, fake, 2048, big, fake, 2048, big, ctypes.byref(ep), fake, null, null, 0,
+                        null) == esb.ESB_ERR_RANGE
+    f64 = esb.esb_format(6, 4, 1)     # 5 significant bits: not an E4M3 image
+    assert lib.esb_gemm(128, 64, 64, fake, 16, f64, fake, 16, f64, ctypes.byref(ep), fake, null, null, 0,
+                        null) == esb.ESB_ERR_UNSUPPORTED
+    assert lib.esb_gemm(128, 64, 64, fake, 4, f, fake, 8, f, ctypes.byref(ep), fake, null, null, 0,
+                        null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_gemm(128, 64, 64, ctypes.c_void_p(4100), 8, f, fake, 8, f, ctypes.byref(ep), fake, null, null, 0,
+                        null) == esb.ESB_ERR_ALIGN
+    assert lib.esb_gemm(0, 64, 64, fake, 8, f, fake, 8, f, ctypes.byref(ep), fake, null, null, 0,
+                        null) == esb.ESB_OK
+    d = esb.esb_conv_desc(1, 8, 8, 64, 64, 3, 3, 1, 1, 1)
+    assert lib.esb_conv2d_nhwc(ctypes.byref(d), fake, 8, f, fake, 12, f, ctypes.byref(ep), fake, null, null, 0,
+                               null) == esb.ESB_ERR_INVALID_ARG
+    d2 = esb.esb_conv_desc(1, 8, 8, 64, 64, 3, 3, 1, 3, 1)
+    assert lib.esb_conv2d_nhwc(ctypes.byref(d2), fake, 8, f, fake, 8, f, ctypes.byref(ep), fake, null, null, 0,
+                               null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_get_status(null, null) == esb.ESB_ERR_INVALID_ARG
+
+
+def test_bn_dn_fold_identity():
+    # Sec. IV-C: DN(BN(Scale(x))) / alpha_{l+1} = a x + b with the printed a, b.
+    rng = np.random.default_rng(4)
+    aw, ka, aa, kw = 0.37, 2, 1.3, 1
+    mu_bn, sd_bn, g, beta = rng.normal(size=5), rng.uniform(0.5, 2, 5), rng.normal(size=5), rng.normal(size=5)
+    mu_dn, sd_dn, a_next = 0.3, 1.7, 0.61
+    scale, bias = esb.fold_bn_dn(aw, kw, aa, ka, mu_bn, sd_bn, g, beta, mu_dn, sd_dn)
+    acc = rng.integers(-500, 500, size=5).astype(np.float64)
+    x = acc * (aw * 2.0 ** -kw) * (aa * 2.0 ** -ka)          # Scale: dequantised product
+    bn = g * (x - mu_bn) / sd_bn + beta                      # BN
+    dn = (bn - mu_dn) / sd_dn                                # DN
+    lhs = dn / a_next
+    # the paper's a and b (over the raw product x' = acc * alpha_W * alpha_A)
+    a_p = (aw * aa * g) / (a_next * sd_dn * sd_bn)
+    b_p = (sd_bn * beta - mu_bn * g - sd_bn * mu_dn) / (a_next * sd_dn * sd_bn)
+    xr = acc * 2.0 ** -(kw + ka)
+    assert np.allclose(lhs, a_p * xr + b_p, rtol=1e-12, atol=1e-12)
+    assert np.allclose(lhs, (scale * acc + bias) / a_next, rtol=1e-12, atol=1e-12)

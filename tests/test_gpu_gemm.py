@@ -1,0 +1,180 @@
+"""GPU parity of the ESB GEMM and implicit-GEMM convolution (tcgen05 path)
+against the CPU oracle: exact int32 accumulators, bit-exact fp32 epilogue
+outputs and requantised codes."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as o
+from paper_2109_03513_gb300 import esb, synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def u32(t):
+    return t.cpu().numpy().view(np.uint32)
+
+
+def dev_i32(a: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int32)).cuda()
+
+
+def random_packed(rows, cols, fmt, seed):
+    b, k = fmt[0], fmt[1]
+    codes = synth.uniform_ints((rows, cols), 0, 2 ** b, seed)
+    if len(fmt) > 2 and not fmt[2]:
+        codes &= np.uint32((1 << (b - 1)) - 1)        # unsigned: sign bit 0
+    return o.pack(codes, b, k, ld_words=esb.esb_row_words(cols, b))
+
+
+def projected_packed(x: np.ndarray, fmt, seed_alpha):
+    b, k, s = fmt
+    a, _ = o.calibrate(x, b, k, s)
+    return o.project_packed(x, a, b, k, s, ld_words=esb.esb_row_words(x.shape[1], b)), a
+
+
+GEMM_CASES = [
+    # (M, N, K, fa, fb)
+    (64, 64, 576, (4, 2, False), (4, 2, True)),     # a 3x3x64 conv tile
+    (128, 128, 128, (4, 2, True), (4, 2, True)),
+    (130, 70, 200, (4, 2, True), (4, 1, True)),     # ragged M, N, K
+    (257, 33, 1000, (3, 1, True), (6, 3, True)),
+    (300, 96, 515, (5, 2, True), (5, 2, True)),
+    (64, 48, 4096, (6, 3, True), (6, 3, True)),
+    (100, 200, 64, (4, 3, True), (5, 1, True)),
+    (1, 1, 1, (4, 2, True), (4, 2, True)),
+    (33, 17, 15, (2, 0, True), (3, 0, True)),
+    (256, 256, 1024, (4, 0, True), (4, 2, True)),
+]
+
+
+@pytest.mark.parametrize("M,N,K,fa,fb", GEMM_CASES)
+def test_gemm_acc_matches_oracle(M, N, K, fa, fb):
+    A = random_packed(M, K, fa, seed=M * 7 + K)
+    B = random_packed(N, K, fb, seed=N * 11 + K)
+    acc, _, _ = esb.esb_gemm(dev_i32(A), esb.Fmt(*fa[:2]), dev_i32(B), esb.Fmt(*fb[:2]), K)
+    exp = o.gemm_i64(A, fa[:2], B, fb[:2], M, N, K)
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), exp)
+
+
+def test_gemm_k_zero_and_empty():
+    A = np.zeros((5, 4), np.uint32)
+    B = np.zeros((3, 4), np.uint32)
+    acc, _, _ = esb.esb_gemm(dev_i32(A), esb.Fmt(4, 2), dev_i32(B), esb.Fmt(4, 2), 0)
+    assert np.array_equal(acc.cpu().numpy(), np.zeros((5, 3), np.int32))
+
+
+@pytest.mark.parametrize("fmt,K", [((4, 2), 16384), ((6, 3), 4600), ((5, 1), 450), ((3, 1), 262144)])
+def test_gemm_exact_near_the_accumulation_bound(fmt, K):
+    # Adversarial sums: A rows all at the largest image, B rows mixing the
+    # largest image with +-1 so partial sums grow towards 2^24 while small
+    # terms keep arriving; any loss of low bits in the fp32 TMEM
+    # accumulation shows up as an integer mismatch.
+    b, k = fmt
+    maxc = o.encode(o.C_of(b, k), b, k)
+    onep = o.encode(1.0 / 2 ** k, b, k)
+    onen = o.encode(-1.0 / 2 ** k, b, k)
+    M, N = 128, 64
+    ca = np.full((M, K), maxc, np.uint32)
+    rng = np.random.default_rng(K)
+    cb = np.where(rng.random((N, K)) < 0.7, maxc, np.where(rng.random((N, K)) < 0.5, onep, onen)).astype(np.uint32)
+    cb[0, :] = maxc
+    A = o.pack(ca, b, k, ld_words=esb.esb_row_words(K, b))
+    B = o.pack(cb, b, k, ld_words=esb.esb_row_words(K, b))
+    acc, _, _ = esb.esb_gemm(dev_i32(A), esb.Fmt(b, k), dev_i32(B), esb.Fmt(b, k), K)
+    exp = o.gemm_i64(A, fmt, B, fmt, M, N, K)
+    assert exp.max() < 2 ** 24
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), exp)
+
+
+def test_gemm_range_error():
+    A = np.zeros((128, 1024), np.uint32)
+    with pytest.raises(esb.EsbError) as e:
+        esb.esb_gemm(dev_i32(A), esb.Fmt(6, 3), dev_i32(A), esb.Fmt(6, 3), 8192)
+    assert e.value.status == esb.ESB_ERR_RANGE
+
+
+EPI_CASES = [
+    # (M, N, K, act, fmt_out, rounding, per_channel, residual)
+    (64, 64, 576, esb.ESB_ACT_RELU, (4, 2, False), 0, False, False),
+    (200, 128, 300, esb.ESB_ACT_NONE, (4, 2, True), 1, True, False),
+    (150, 80, 256, esb.ESB_ACT_RELU6, (6, 3, False), 0, True, True),     # 5 codes per word -> BN = 80
+    (129, 96, 640, esb.ESB_ACT_RELU, (5, 2, False), 0, False, True),     # 6 codes per word
+    (70, 60, 100, esb.ESB_ACT_NONE, (3, 1, True), 0, True, False),      # 10 codes per word
+]
+
+
+@pytest.mark.parametrize("M,N,K,act,fo,rnd,per_channel,residual", EPI_CASES)
+def test_gemm_fused_epilogue_matches_oracle(M, N, K, act, fo, rnd, per_channel, residual):
+    fa, fb = (4, 2, False), (4, 2, True)
+    xa = synth.half_normal((M, K), seed=M + 1).numpy()
+    xb = synth.he_normal((N, K), fan_in=K, seed=N + 2).numpy()
+    A, aa = projected_packed(xa, fa, 0)
+    B, ab = projected_packed(xb, fb, 0)
+    s0 = esb.default_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2))
+    if per_channel:
+        scale = (np.float32(s0) * synth.normal((N,), seed=3).numpy().__abs__() + np.float32(1e-3)).astype(np.float32)
+        bias = (0.1 * synth.normal((N,), seed=4).numpy()).astype(np.float32)
+    else:
+        scale = np.full(N, s0, np.float32)
+        bias = np.full(N, 0.05, np.float32)
+    res_fmt = (4, 2, True)
+    res_codes = random_packed(M, N, res_fmt, seed=77) if residual else None
+    ep = esb.Epilogue(scale=torch.from_numpy(scale).cuda() if per_channel else None,
+                      bias=torch.from_numpy(bias).cuda() if per_channel else None,
+                      scale0=float(s0), bias0=0.05, act=act,
+                      residual=dev_i32(res_codes) if residual else None, res_fmt=esb.Fmt(*res_fmt),
+                      res_scale=0.03125, alpha_out=0.173, fmt_out=esb.Fmt(*fo), rounding_out=rnd)
+    acc, y, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(4, 2, False), dev_i32(B), esb.Fmt(4, 2), K, ep=ep,
+                                 want_acc=True, want_y=True, want_codes=True)
+    acc_o = o.gemm_i64(A, fa[:2], B, fb[:2], M, N, K)
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), acc_o)
+    res_img = None
+    if residual:
+        rc = o.unpack(res_codes, N, 4)
+        res_img = np.vectorize(lambda c: o.image(int(c), 4, 2))(rc)
+    yo, co = o.epilogue(acc_o, scale, bias, act, 0.173, fo, rnd, res_images=res_img, res_scale=0.03125)
+    yg = y.cpu().numpy()
+    # pinned fp32 op order on both sides: identical bits (tolerance 1e-6 rel)
+    assert np.array_equal(yg, yo) or np.max(np.abs(yg - yo) / np.maximum(np.abs(yo), 1e-30)) <= 1e-6
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
+CONV_CASES = [
+    # n, h, w, c, cout, r, s, stride, pad, fx, fw
+    (2, 9, 7, 64, 64, 3, 3, 1, 1, (4, 2, False), (4, 2, True)),
+    (2, 56, 56, 64, 64, 3, 3, 1, 1, (4, 2, False), (4, 2, True)),     # ResNet18 3x3 layer shape, batch 2
+    (2, 14, 14, 128, 256, 3, 3, 2, 1, (4, 2, False), (4, 2, True)),
+    (3, 8, 8, 64, 128, 1, 1, 2, 0, (4, 2, False), (4, 2, True)),
+    (1, 23, 19, 3, 64, 7, 7, 2, 3, (4, 2, True), (4, 2, True)),       # first layer: c = 3
+    (2, 10, 10, 64, 64, 3, 3, 1, 1, (6, 3, False), (6, 3, True)),
+    (2, 10, 10, 40, 48, 3, 3, 1, 1, (5, 2, False), (5, 2, True)),
+    (2, 10, 10, 30, 32, 3, 3, 1, 1, (3, 1, False), (3, 1, True)),
+]
+
+
+@pytest.mark.parametrize("n,h,w,c,cout,r,s,stride,pad,fx,fw", CONV_CASES)
+def test_conv_matches_oracle(n, h, w, c, cout, r, s, stride, pad, fx, fw):
+    x = synth.half_normal((n * h * w, c), seed=h * 3 + c).numpy()
+    wt = synth.he_normal((cout * r * s, c), fan_in=r * s * c, seed=cout + r).numpy()
+    ldx = esb.esb_row_words(c, fx[0])
+    X, ax = projected_packed(x, fx, 0)
+    W, aw = projected_packed(wt, fw, 0)
+    assert X.shape[1] == ldx and W.shape[1] == ldx
+    fo = (fx[0], fx[1], False)
+    s0 = esb.default_scale(ax, esb.Fmt(*fx[:2]), aw, esb.Fmt(*fw[:2]))
+    ep = esb.Epilogue(scale0=s0, bias0=0.0, act=esb.ESB_ACT_RELU, alpha_out=0.7, fmt_out=esb.Fmt(*fo))
+    acc, y, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fx), dev_i32(W), esb.Fmt(*fw), n, h, w, c, cout, r, s,
+                                        stride, pad, ep=ep, want_acc=True, want_y=True, want_codes=True)
+    acc_o = o.conv2d_i64(X.reshape(n, h, w, ldx), fx[:2], W.reshape(cout, r, s, ldx), fw[:2],
+                         n, h, w, c, cout, r, s, stride, pad).reshape(-1, cout)
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), acc_o)
+    yo, co = o.epilogue(acc_o, np.full(cout, s0, np.float32), np.zeros(cout, np.float32), 1, 0.7, fo)
+    assert np.array_equal(y.cpu().numpy(), yo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))

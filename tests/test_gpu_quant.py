@@ -1,0 +1,153 @@
+"""GPU parity of projection, dequantisation and DDA calibration against the
+CPU oracle, through the C ABI (libesb.so)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as o
+from paper_2109_03513_gb300 import esb, synth
+
+pytestmark = pytest.mark.gpu
+
+FORMATS = [(b, k) for b in range(2, 9) for k in range(0, b)]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def u32(t: torch.Tensor) -> np.ndarray:
+    return t.cpu().numpy().view(np.uint32)
+
+
+def probe_values(b, k):
+    s = o.set_nonneg(b, k)
+    mids = 0.5 * (s[1:] + s[:-1])
+    pts = np.concatenate([s, mids, [o.C_of(b, k) * 1.5, 1e30, 1e-40, 3e-39]]).astype(np.float32)
+    out = [pts]
+    cur = pts
+    for _ in range(2):
+        out.append(np.nextafter(cur, np.float32(np.inf)))
+        out.append(np.nextafter(cur, np.float32(-np.inf)))
+        cur = out[-1]
+    v = np.concatenate(out)
+    return np.concatenate([v, -v, np.array([0.0, -0.0, np.inf, -np.inf, np.nan], np.float32)])
+
+
+@pytest.mark.parametrize("b,k", FORMATS)
+@pytest.mark.parametrize("signed", [True, False])
+@pytest.mark.parametrize("rounding", [0, 1])
+def test_project_matches_oracle(b, k, signed, rounding):
+    f = esb.Fmt(b, k, signed)
+    C = o.C_of(b, k)
+    x = np.concatenate([probe_values(b, k),
+                        synth.normal((6000,), seed=b * 100 + k).numpy() * np.float32(C),
+                        synth.laplace((2000,), seed=b * 100 + k + 1).numpy()]).astype(np.float32)
+    for alpha in (1.0, 0.7310585, 3.0):
+        # 1-D (vector path) and a ragged 2-D view (general path)
+        for shape in ((x.size,), (7, x.size // 7)):
+            xs = x[: int(np.prod(shape))].reshape(shape)
+            codes = esb.esb_project(torch.from_numpy(xs).cuda(), f, alpha=alpha, rounding=rounding)
+            exp = o.project_packed(xs.reshape(-1, shape[-1]), alpha, b, k, signed, rounding,
+                                   ld_words=codes.shape[-1])
+            assert np.array_equal(u32(codes), exp), (shape, alpha)
+
+
+def test_project_edge_shapes_and_device_alpha():
+    f = esb.Fmt(4, 2, True)
+    for rows, cols in [(1, 1), (1, 7), (3, 8), (5, 33), (2, 64), (130, 576)]:
+        x = synth.normal((rows, cols), seed=rows * 1000 + cols)
+        a = torch.tensor([0.41], dtype=torch.float32, device="cuda")
+        codes = esb.esb_project(x.cuda(), f, alpha=a)
+        exp = o.project_packed(x.numpy(), 0.41, 4, 2, True, 0, ld_words=codes.shape[-1])
+        assert np.array_equal(u32(codes), exp), (rows, cols)
+    # explicit wider row stride: padding words hold zero codes
+    x = synth.normal((4, 10), seed=3)
+    codes = esb.esb_project(x.cuda(), f, alpha=0.5, ldc=12)
+    assert np.array_equal(u32(codes), o.project_packed(x.numpy(), 0.5, 4, 2, ld_words=12))
+
+
+def test_project_full_size_sampled():
+    # 2^28 values, the size the projection sweep runs; check sampled words.
+    n = 1 << 28
+    f = esb.Fmt(4, 2, True)
+    x = torch.randn(n, generator=torch.Generator(device="cuda").manual_seed(5), device="cuda")
+    codes = esb.esb_project(x, f, alpha=0.37)
+    torch.cuda.synchronize()
+    cpw = 8
+    idx = np.unique(np.concatenate([np.arange(64), np.arange(codes.shape[1] - 64, codes.shape[1]),
+                                    np.random.default_rng(1).integers(0, codes.shape[1], 4000)]))
+    ti = torch.from_numpy(idx).cuda()
+    got = u32(codes[0, ti])
+    xs = x.view(-1, cpw)[ti].cpu().numpy()
+    exp = o.project_packed(xs, 0.37, 4, 2, True, 0, ld_words=1)[:, 0]
+    assert np.array_equal(got, exp)
+    del x, codes
+
+
+@pytest.mark.parametrize("b,k", [(2, 0), (3, 1), (4, 2), (5, 1), (6, 3), (8, 4), (8, 0)])
+def test_dequant_matches_oracle(b, k):
+    f = esb.Fmt(b, k, True)
+    rows, cols = 5, 77
+    codes = synth.uniform_ints((rows, cols), 0, 2 ** b, seed=b * 10 + k)
+    packed = o.pack(codes, b, k, ld_words=esb.esb_row_words(cols, b))
+    y = esb.esb_dequant(torch.from_numpy(packed.view(np.int32)).cuda(), cols, f, 0.8125)
+    vals = np.vectorize(lambda c: o.decode(int(c), b, k))(codes)
+    exp = (np.float32(0.8125) * vals.astype(np.float32)).astype(np.float32)
+    assert np.array_equal(y.cpu().numpy(), exp)
+
+
+CAL_CASES = [
+    ("normal", 1 << 20, True), ("half_normal", 1 << 20, False), ("laplace", 1 << 20, True),
+    ("normal", 1, True), ("normal", 31, True), ("normal", 33, True), ("normal", 1000003, True),
+    ("half_normal", 4097, False),
+]
+
+
+@pytest.mark.parametrize("dist,n,signed", CAL_CASES)
+@pytest.mark.parametrize("bk", [(4, 2), (6, 3)])
+def test_calibrate_matches_oracle(dist, n, signed, bk):
+    b, k = bk
+    x = synth.distribution(dist, (n,), seed=n % 1000 + b)
+    f = esb.Fmt(b, k, signed)
+    stats = torch.zeros(3, dtype=torch.float64, device="cuda")
+    a, _ = esb.esb_calibrate_dda(x.cuda(), f, stats_out=stats)
+    ao, so = o.calibrate(x.numpy(), b, k, signed)
+    ag = float(a.item())
+    st = stats.cpu().numpy()
+    assert abs(ag - ao) <= 1e-6 * ao, (ag, ao)
+    assert st[2] == n
+    assert abs(st[1] - so[1]) <= 1e-6 * max(so[1], 1e-30) + 1e-12
+    assert abs(st[0] - so[0]) <= 1e-6 * max(so[1], 1e-30) + 1e-12
+
+
+def test_calibrate_offset_constant_and_determinism():
+    f = esb.Fmt(4, 2, True)
+    x = synth.normal((1 << 18,), seed=9, mean=100.0)
+    a1, _ = esb.esb_calibrate_dda(x.cuda(), f)
+    a2, _ = esb.esb_calibrate_dda(x.cuda(), f)
+    ao, _ = o.calibrate(x.numpy(), 4, 2)
+    assert abs(a1.item() - ao) <= 1e-6 * ao
+    assert a1.item() == a2.item()
+    c = torch.full((1000,), 2.5, dtype=torch.float32)
+    ac, _ = esb.esb_calibrate_dda(c.cuda(), f)
+    assert ac.item() == np.float32(o.alpha_star(4, 2)[0] * 1e-7)
+    # unaligned base pointer takes the scalar path
+    xu = synth.normal((1 << 12) + 1, seed=4)
+    xd = xu.cuda()[1:]
+    au, _ = esb.esb_calibrate_dda(xd, f)
+    ao2, _ = o.calibrate(xu.numpy()[1:], 4, 2)
+    assert abs(au.item() - ao2) <= 1e-6 * ao2
+
+
+def test_calibrate_then_project_on_device():
+    # alpha stays on the device between the two calls (no host round trip)
+    f = esb.Fmt(5, 2, True)
+    x = synth.laplace((3, 1000), seed=12)
+    xd = x.cuda()
+    a, _ = esb.esb_calibrate_dda(xd, f)
+    codes = esb.esb_project(xd, f, alpha=a)
+    ah = float(a.item())
+    assert np.array_equal(u32(codes), o.project_packed(x.numpy(), ah, 5, 2, ld_words=codes.shape[-1]))

@@ -408,3 +408,15 @@ def test_epilogue_op_order():
             assert codes[m, n] == o.encode(o.project_value(float(t), 0.41, *fo), 4, 2, False)
     y6, _ = o.epilogue(acc * 100, scale, bias, 2, 0.41, fo)
     assert y6.max() <= 6.0 and y6.min() >= 0.0
+
+
+@pytest.mark.parametrize("b,k", [(4, 2), (5, 1), (6, 3), (3, 0), (2, 0)])
+def test_dD_is_the_derivative_of_D(b, k):
+    # D'(alpha) (used to locate alpha*) against central differences of D.
+    for a in (0.05, 0.3, 1.0, 1.7):
+        h = a * 1e-5
+        fd = (o.D(a + h, b, k) - o.D(a - h, b, k)) / (2 * h)
+        assert abs(fd - o.dD(a, b, k)) < 1e-6 * max(1.0, abs(fd)), (a, fd, o.dD(a, b, k))
+    a_star, _ = o.alpha_star(b, k)
+    assert abs(o.dD(a_star, b, k)) < 1e-12
+    assert o.dD(a_star * 0.99, b, k) < 0 < o.dD(a_star * 1.01, b, k)
