@@ -1,0 +1,451 @@
+#!/usr/bin/env python
+"""Benchmark of the ESB inference hot path on GB300 (one JSON line on stdout).
+
+Workload (default): a ResNet18-shaped 3x3 convolution layer, NHWC, batch 32,
+56x56, 64 -> 64 channels, stride 1, pad 1, weights and activations in
+ESB(4,2) (activations post-ReLU, unsigned).  Inputs are seeded synthetic
+tensors: X ~ |N(0,1)|, W ~ N(0, sqrt(2/576)) (He init).
+
+One step = one pass of the whole hot path over one batch, captured as a
+CUDA graph:
+  esb_calibrate_dda(X) -> esb_project(X)     (DDA alpha of the batch, codes)
+  esb_calibrate_dda(W) -> esb_project(W)
+  esb_conv2d_nhwc(Xc, Wc) with the fused epilogue (dequant scale from the two
+  device alphas, ReLU, ESB requantisation with the layer's calibrated
+  output alpha) -> next layer's packed codes.
+L2 is flushed (256 MiB write) before every timed step; each step is timed
+with CUDA events on the launching stream.  `value` is conv TOPS over the
+whole step (2 ops per MAC).  --impl reference times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ESB GEMM/conv int TOPS and esb_project GB/s, % of GB300 roofline (1 GPU)"
+UNIT = "TOPS"
+
+N_, H_, W_, C_, CO_, R_, S_ = 32, 56, 56, 64, 64, 3, 3
+STRIDE, PAD = 1, 1
+FB, FK = 4, 2
+P_ = (H_ + 2 * PAD - R_) // STRIDE + 1
+Q_ = (W_ + 2 * PAD - S_) // STRIDE + 1
+MACS = N_ * P_ * Q_ * CO_ * R_ * S_ * C_
+OPS = 2 * MACS
+WORKLOAD = {"workload": "resnet18_conv3x3_56x56_b32_esb42", "n": N_, "h": H_, "w": W_, "c": C_, "cout": CO_,
+            "r": R_, "s": S_, "stride": STRIDE, "pad": PAD, "b": FB, "k": FK, "ops_per_step": OPS,
+            "l2": "flushed (256 MiB write) before every timed step"}
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["hbm_gbs"], d["bf16_tflops"], "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+def _kernel_hash():
+    h = hashlib.sha256()
+    for f in ("esb_gemm.cu", "esb_common.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2109_03513_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def _traffic_from_profile(kernel_hash):
+    """DRAM bytes per launch of the conv kernel from the committed ncu summary,
+    if it was taken on the current kernel source; else None."""
+    p = os.path.join(ROOT, "profiles", "conv3x3_b32_ncu.txt")
+    if not os.path.exists(p):
+        return None
+    kv = {}
+    for line in open(p):
+        if ":" in line:
+            k, v = line.split(":", 1)
+            kv[k.strip()] = v.strip()
+    if kv.get("kernel_source_hash") != kernel_hash:
+        return None
+    try:
+        return float(kv["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    def __init__(self):
+        self.proc = None
+        self.path = os.path.join("/tmp", f"esb_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self, gpu_index=0):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9 and parts[0] == str(gpu_index):
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        mhz = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            for name, v in zip(names, r[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(mhz) if mhz else None, "sm_max_mhz": float(rows[0][2]),
+                "samples": len(rows), "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------------- GPU arm
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2109_03513_gb300 import esb, synth
+    import __graft_entry__
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0 or world == 1:
+        __graft_entry__.build()
+    if world > 1:
+        dist.barrier()
+    esb.lib()
+
+    fu, fs = esb.Fmt(FB, FK, False), esb.Fmt(FB, FK, True)
+    x_h = synth.half_normal((N_ * H_ * W_, C_), seed=1 + rank)
+    w_h = synth.he_normal((CO_ * R_ * S_, C_), fan_in=R_ * S_ * C_, seed=2)
+    X = x_h.to(dev)
+    Wt = w_h.to(dev)
+    ldx = esb.esb_row_words(C_, FB)
+    Xc = torch.empty((N_ * H_ * W_, ldx), dtype=torch.int32, device=dev)
+    Wc = torch.empty((CO_ * R_ * S_, ldx), dtype=torch.int32, device=dev)
+    M = N_ * P_ * Q_
+    Yc = torch.empty((M, esb.esb_row_words(CO_, FB)), dtype=torch.int32, device=dev)
+    ax = torch.empty(1, dtype=torch.float32, device=dev)
+    aw = torch.empty(1, dtype=torch.float32, device=dev)
+    wsx = torch.empty(esb.esb_calibrate_dda_workspace_bytes(X.numel()), dtype=torch.uint8, device=dev)
+    wsw = torch.empty(esb.esb_calibrate_dda_workspace_bytes(Wt.numel()), dtype=torch.uint8, device=dev)
+
+    # Calibration of the layer's output alpha (untimed, once): fp32 ReLU output -> DDA.
+    esb.esb_calibrate_dda(X, fu, alpha_out=ax, workspace=wsx)
+    esb.esb_project(X, fu, alpha=ax, codes=Xc)
+    esb.esb_calibrate_dda(Wt, fs, alpha_out=aw, workspace=wsw)
+    esb.esb_project(Wt, fs, alpha=aw, codes=Wc)
+    ep_cal = esb.Epilogue(scale0=1.0, alpha_a_dev=ax, alpha_b_dev=aw, act=esb.ESB_ACT_RELU, alpha_out=1.0,
+                          fmt_out=fu)
+    _, y32, _ = esb.esb_conv2d_nhwc(Xc, fu, Wc, fs, N_, H_, W_, C_, CO_, R_, S_, STRIDE, PAD, ep=ep_cal,
+                                    want_acc=False, want_y=True)
+    a_out, _ = esb.esb_calibrate_dda(y32, fu)
+    del y32
+    alpha_out = float(a_out.item())
+    ep = esb.Epilogue(scale0=1.0, alpha_a_dev=ax, alpha_b_dev=aw, act=esb.ESB_ACT_RELU, alpha_out=alpha_out,
+                      fmt_out=fu)
+
+    stream = torch.cuda.Stream(device=dev)
+    calls = [
+        ("calibrate_x", lambda: esb.esb_calibrate_dda(X, fu, alpha_out=ax, workspace=wsx, stream=stream), 2),
+        ("project_x", lambda: esb.esb_project(X, fu, alpha=ax, codes=Xc, stream=stream), 1),
+        ("calibrate_w", lambda: esb.esb_calibrate_dda(Wt, fs, alpha_out=aw, workspace=wsw, stream=stream), 2),
+        ("project_w", lambda: esb.esb_project(Wt, fs, alpha=aw, codes=Wc, stream=stream), 1),
+        ("conv", lambda: esb.esb_conv2d_nhwc(Xc, fu, Wc, fs, N_, H_, W_, C_, CO_, R_, S_, STRIDE, PAD, ep=ep,
+                                             want_acc=False, out_codes=Yc, stream=stream), 1),
+    ]
+    launches_per_step = sum(c[2] for c in calls)
+
+    def step():
+        for _, fn, _ in calls:
+            fn()
+
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            step()
+    torch.cuda.synchronize(dev)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        step()
+    torch.cuda.synchronize(dev)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            flush.fill_(1)
+            g.replay()
+    torch.cuda.synchronize(dev)
+
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    clocks = ClockSampler()
+    clocks.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    with torch.cuda.stream(stream):
+        for i in range(K):
+            flush.fill_(i & 255)
+            ev[i][0].record(stream)
+            g.replay()
+            ev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    ck = clocks.stop(local)
+    t_ms = sum(a.elapsed_time(b) for a, b in ev)
+    assert esb.esb_get_status(stream) == 0
+    t_max = t_ms
+    if world > 1:
+        tt = torch.tensor([t_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t_max = float(tt.item())
+    value = world * K * OPS / (t_max * 1e-3) / 1e12
+
+    # Per-kernel durations (same launches, un-graphed, cold L2) for the roofline.
+    reps = max(20, min(200, K // 10))
+    per = {name: 0.0 for name, _, _ in calls}
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            flush.fill_(3)
+            evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(calls) + 1)]
+            evs[0].record(stream)
+            for j, (_, fn, _) in enumerate(calls):
+                fn()
+                evs[j + 1].record(stream)
+            torch.cuda.synchronize(dev)
+            for j, (name, _, _) in enumerate(calls):
+                per[name] += evs[j].elapsed_time(evs[j + 1]) / reps
+
+    # End to end through the public API with host buffers: H2D of X, the step,
+    # D2H of the output codes, all inside the timed region.
+    x_pin = x_h.pin_memory()
+    y_pin = torch.empty(Yc.shape, dtype=torch.int32).pin_memory()
+    ke = max(10, min(200, K // 10))
+    e2e_ms = 0.0
+    with torch.cuda.stream(stream):
+        for _ in range(ke):
+            flush.fill_(5)
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            X.copy_(x_pin, non_blocking=True)
+            g.replay()
+            y_pin.copy_(Yc, non_blocking=True)
+            a1.record(stream)
+            torch.cuda.synchronize(dev)
+            e2e_ms += a0.elapsed_time(a1)
+    e2e_ms /= ke
+    e2e_value = world * OPS / (e2e_ms * 1e-3) / 1e12
+    if world > 1:
+        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_value = world * OPS / (float(tt.item()) * 1e-3) / 1e12
+
+    hbm, bf16, src = _peaks()
+    n_x, n_w = X.numel(), Wt.numel()
+    algo = {  # algorithmic bytes / ops per launch
+        "calibrate_x": ("hbm", 4.0 * n_x), "project_x": ("hbm", 4.0 * n_x + 4.0 * Xc.numel()),
+        "calibrate_w": ("hbm", 4.0 * n_w), "project_w": ("hbm", 4.0 * n_w + 4.0 * Wc.numel()),
+        "conv": ("tensor", float(OPS)),
+    }
+    dominant = max(per, key=per.get)
+    bound, amount = algo[dominant]
+    t_k = per[dominant] * 1e-3
+    khash = _kernel_hash()
+    if bound == "tensor":
+        achieved = amount / t_k / 1e12
+        peak = 2.0 * bf16
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "kernel": dominant,
+                "peak_note": f"fp8 dense = {src} bf16 burst {bf16} x nominal fp8:bf16 ratio 2",
+                "traffic": _traffic_from_profile(khash) if dominant == "conv" else None}
+    else:
+        achieved = amount / t_k / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                "kernel": dominant, "peak_note": f"{src} HBM copy", "traffic": None}
+    kernels = {}
+    for name, (b, amt) in algo.items():
+        t = per[name] * 1e-3
+        if b == "tensor":
+            kernels[name] = {"us": per[name] * 1e3, "TFLOP/s": amt / t / 1e12, "frac": amt / t / 1e12 / (2.0 * bf16)}
+        else:
+            kernels[name] = {"us": per[name] * 1e3, "GB/s": amt / t / 1e9, "frac": amt / t / 1e9 / hbm}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
+        "ms_per_step": t_max / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "e4m3", "data": "synthetic (seeded |N(0,1)| activations, He-init N(0,sqrt(2/576)) weights)",
+        "config": dict(WORKLOAD, parallelism="replicas" if world > 1 else "single"),
+        "roofline": roof, "kernels": kernels,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(x_pin.numel() * 4),
+                "d2h_bytes_per_step": int(y_pin.numel() * 4), "ms_per_step": e2e_ms},
+        "gpu_launches": launches_per_step * K,
+        "clocks": ck, "kernel_source_hash": khash,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+# ----------------------------------------------------------- CPU oracle arm
+
+class OracleSample:
+    """The hot path by the CPU oracle on a bounded sample of the workload:
+    DDA calibration of all of X and W, projection of W and of the input
+    images the sample touches, then conv + epilogue of `rows` output rows
+    (image-major).  run() returns the conv ops it performed."""
+
+    def __init__(self, pool):
+        import numpy as np
+
+        import oracle as o
+        from paper_2109_03513_gb300 import synth
+
+        o.build()
+        self.np, self.o, self.pool = np, o, pool
+        self.x = synth.half_normal((N_ * H_ * W_, C_), seed=1).numpy()
+        self.w = synth.he_normal((CO_ * R_ * S_, C_), fan_in=R_ * S_ * C_, seed=2).numpy()
+        self.ldx = (-(-C_ // (32 // FB)) + 3) // 4 * 4
+
+    def run(self, rows):
+        np, o = self.np, self.o
+        ax, _ = o.calibrate(self.x, FB, FK, signed=False)
+        aw, _ = o.calibrate(self.w, FB, FK, signed=True)
+        Wc = o.project_packed(self.w, aw, FB, FK, True, ld_words=self.ldx).reshape(CO_, R_, S_, self.ldx)
+        units = [(i // P_, i % P_) for i in range(rows)]
+        imgs = sorted({n for n, _ in units})
+        pix = H_ * W_
+        Xi = {}
+
+        def proj(n):
+            Xi[n] = o.project_packed(self.x[n * pix:(n + 1) * pix], ax, FB, FK, False,
+                                     ld_words=self.ldx).reshape(1, H_, W_, self.ldx)
+
+        list(self.pool.map(proj, imgs))
+        scale = np.float32(np.float32(ax) * np.float32(aw)) * np.float32(2.0 ** -(2 * FK))
+
+        def one(u):
+            n, p = u
+            acc = o.conv2d_rows_i64(Xi[n], (FB, FK), Wc, (FB, FK), 1, H_, W_, C_, CO_, R_, S_, STRIDE, PAD, p, p + 1)
+            o.epilogue(acc.reshape(-1, CO_), np.full(CO_, scale, np.float32), np.zeros(CO_, np.float32), 1,
+                       0.25, (FB, FK, False))
+            return 1
+
+        done = sum(self.pool.map(one, units))
+        return 2 * done * Q_ * CO_ * R_ * S_ * C_
+
+    def rows_for_budget(self, seconds):
+        import time as _t
+        t0 = _t.perf_counter()
+        self.run(1)
+        t1 = _t.perf_counter() - t0
+        cores = self.pool._max_workers
+        return max(1, min(N_ * P_, int(seconds / max(t1, 1e-3) * cores * 0.8)))
+
+
+def _cores():
+    return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+
+
+def cpu_baseline(budget_s=12.0):
+    from concurrent.futures import ThreadPoolExecutor
+
+    cores = _cores()
+    with ThreadPoolExecutor(max_workers=cores) as pool:
+        smp = OracleSample(pool)
+        rows = smp.rows_for_budget(budget_s)
+        t0 = time.perf_counter()
+        ops = smp.run(rows)
+        dt = time.perf_counter() - t0
+    return {"value": ops / dt / 1e12, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"DDA calibration of all of X ({N_}x{H_}x{W_}x{C_}) and W, projection of W and of the "
+                      f"touched images, conv + epilogue of {rows} of the {N_ * P_} output rows "
+                      f"({ops / 1e9:.3f} GOP); {dt:.2f} s wall",
+            "seconds": dt}
+
+
+def run_reference(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from concurrent.futures import ThreadPoolExecutor
+
+    cores = _cores()
+    times = []
+    ops = 0
+    with ThreadPoolExecutor(max_workers=cores) as pool:
+        smp = OracleSample(pool)
+        budget = 150.0 / (args.steps + args.warmup)           # whole run within a few minutes
+        rows = smp.rows_for_budget(budget)
+        for i in range(args.warmup + args.steps):
+            t0 = time.perf_counter()
+            ops = smp.run(rows)
+            dt = time.perf_counter() - t0
+            if i >= args.warmup:
+                times.append(dt)
+    total = sum(times)
+    value = len(times) * ops / total / 1e12
+    sample = (f"per step: DDA calibration of all of X and W, projection of W and of the touched images, "
+              f"conv + epilogue of {rows} of the {N_ * P_} output rows ({ops / 1e9:.3f} GOP)")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+            "data": "synthetic", "config": dict(WORKLOAD, parallelism="cpu oracle"),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

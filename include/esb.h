@@ -77,7 +77,9 @@ enum { ESB_ACT_NONE = 0, ESB_ACT_RELU = 1, ESB_ACT_RELU6 = 2 };
  * affine, activation, ESB quantization of the next layer's input).
  * For accumulator acc[m][n] (exact int32) the epilogue computes, in fp32
  * with this exact op order:
- *   y = fmaf(scale[n], (float)acc, bias[n])
+ *   s = scale[n] (or scale0)
+ *   s = s * (fl32(alpha_a * alpha_b) * 2^-(kA+kB))     if alpha_a_dev and alpha_b_dev
+ *   y = fmaf(s, (float)acc, bias[n])
  *   y = fmaf(res_scale, (float)I_res[m][n], y)         if residual != NULL
  *   y = max(y, 0) (RELU) or min(max(y, 0), 6) (RELU6)
  *   code = projection of y with alpha_out, fmt_out, rounding_out
@@ -85,6 +87,8 @@ enum { ESB_ACT_NONE = 0, ESB_ACT_RELU = 1, ESB_ACT_RELU6 = 2 };
  * The BN/DN fold of Sec. IV-C becomes scale[n]/bias[n] on the host. */
 typedef struct esb_epilogue {
     const float* scale;        /* [device] N floats, or NULL -> scale0 for every n */
+    const float* alpha_a_dev;  /* [device] 1 float (scale of A / X), or NULL; with alpha_b_dev */
+    const float* alpha_b_dev;  /* [device] 1 float (scale of B / W), or NULL: the "Scale" stage */
     const float* bias;         /* [device] N floats, or NULL -> bias0 for every n */
     float scale0;
     float bias0;

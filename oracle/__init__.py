@@ -84,7 +84,9 @@ def _load():
         "oracle_gemm_i64": (None, [p, i64, i32, i32, p, i64, i32, i32, i64, i64, i64, p]),
         "oracle_gemm_entry": (i64, [p, i64, i32, i32, p, i64, i32, i32, i64, i64, i64]),
         "oracle_epilogue_one": (f32, [i64, f32, f32, i32, i64, f32, i32, f32, i32, i32, i32, i32, p]),
+        "oracle_epilogue_array": (None, [p, i64, i64, p, p, p, f32, i32, f32, i32, i32, i32, i32, p, p]),
         "oracle_conv2d_i64": (None, [p, i64, i32, i32, p, i64, i32, i32] + [i32] * 11 + [p]),
+        "oracle_conv2d_rows_i64": (None, [p, i64, i32, i32, p, i64, i32, i32] + [i32] * 13 + [p]),
         "oracle_dwconv_i64": (None, [p, i64, i32, i32, p, i64, i32, i32] + [i32] * 10 + [p]),
         "oracle_maxpool_codes": (None, [p, i64, i32, i32] + [i32] * 9 + [i64, p]),
         "oracle_avgpool_sum_i64": (None, [p, i64, i32, i32, i32, i32, i32, p]),
@@ -275,20 +277,16 @@ def epilogue(acc: np.ndarray, scale: np.ndarray, bias: np.ndarray, act: int, alp
              res_scale: float = 0.0) -> tuple[np.ndarray, np.ndarray]:
     """Per-element post-processing of an (M, N) accumulator; scale/bias are
     per column n.  Returns (y fp32 (M,N), unpacked output codes (M,N))."""
-    lib = _load()
+    acc = np.ascontiguousarray(acc, dtype=np.int64)
     M, N = acc.shape
+    scale = np.ascontiguousarray(scale, dtype=np.float32)
+    bias = np.ascontiguousarray(bias, dtype=np.float32)
     y = np.zeros((M, N), dtype=np.float32)
     codes = np.zeros((M, N), dtype=np.uint32)
-    cbuf = ctypes.c_uint32(0)
-    has_res = res_images is not None
-    for m in range(M):
-        for n in range(N):
-            r = int(res_images[m, n]) if has_res else 0
-            y[m, n] = lib.oracle_epilogue_one(int(acc[m, n]), float(scale[n]), float(bias[n]),
-                                              int(has_res), r, float(res_scale), act,
-                                              float(alpha_out), fo[0], fo[1], int(fo[2]), rounding,
-                                              ctypes.byref(cbuf))
-            codes[m, n] = cbuf.value
+    res = None if res_images is None else np.ascontiguousarray(res_images, dtype=np.int64)
+    _load().oracle_epilogue_array(_ptr(acc), M, N, _ptr(scale), _ptr(bias),
+                                  None if res is None else _ptr(res), float(res_scale), act, float(alpha_out),
+                                  fo[0], fo[1], int(fo[2]), rounding, _ptr(y), _ptr(codes))
     return y, codes
 
 
@@ -300,6 +298,18 @@ def conv2d_i64(X, fx, W, fw, Nb, H, Wd, C, Cout, R, S, stride, pad):
     acc = np.zeros((Nb, P, Q, Cout), dtype=np.int64)
     _load().oracle_conv2d_i64(_ptr(X), X.shape[-1], fx[0], fx[1], _ptr(W), W.shape[-1], fw[0], fw[1],
                               Nb, H, Wd, C, Cout, R, S, stride, pad, P, Q, _ptr(acc))
+    return acc
+
+
+def conv2d_rows_i64(X, fx, W, fw, Nb, H, Wd, C, Cout, R, S, stride, pad, p0, p1):
+    """conv2d_i64 restricted to output rows [p0, p1)."""
+    P = (H + 2 * pad - R) // stride + 1
+    Q = (Wd + 2 * pad - S) // stride + 1
+    X = np.ascontiguousarray(X, dtype=np.uint32)
+    W = np.ascontiguousarray(W, dtype=np.uint32)
+    acc = np.zeros((Nb, p1 - p0, Q, Cout), dtype=np.int64)
+    _load().oracle_conv2d_rows_i64(_ptr(X), X.shape[-1], fx[0], fx[1], _ptr(W), W.shape[-1], fw[0], fw[1],
+                                   Nb, H, Wd, C, Cout, R, S, stride, pad, P, Q, p0, p1, _ptr(acc))
     return acc
 
 

@@ -447,6 +447,24 @@ float oracle_epilogue_one(int64_t acc, float scale, float bias, int has_res, int
     return y;
 }
 
+/* oracle_epilogue_one over an M x N accumulator; scale/bias per column n;
+ * res_images (nullable) is M x N; y (nullable) M x N; codes M x N unpacked. */
+void oracle_epilogue_array(const int64_t *acc, int64_t M, int64_t N, const float *scale, const float *bias,
+                           const int64_t *res_images, float res_scale, int act, float alpha_out,
+                           int bo, int ko, int so, int rounding, float *y, uint32_t *codes)
+{
+    for (int64_t m = 0; m < M; m++)
+        for (int64_t n = 0; n < N; n++) {
+            int64_t i = m * N + n;
+            uint32_t c = 0;
+            float v = oracle_epilogue_one(acc[i], scale[n], bias[n], res_images != 0,
+                                          res_images ? res_images[i] : 0, res_scale, act, alpha_out,
+                                          bo, ko, so, rounding, &c);
+            if (y) y[i] = v;
+            if (codes) codes[i] = c;
+        }
+}
+
 /* Sec. IV-B computing logic of a convolution layer, NHWC: X codes are rows
  * of C codes per pixel (ldx words), W codes are rows of C codes per
  * (cout, r, s) (ldw words).  acc[n][p][q][co] = sum_{r,s,c} I(X)*I(W) with
@@ -479,6 +497,41 @@ void oracle_conv2d_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
                             }
                         }
                     acc[(((int64_t)n * P + p) * Q + q) * Cout + co] = s;
+                }
+}
+
+/* oracle_conv2d_i64 restricted to output rows p in [p0, p1) (acc holds
+ * (p1 - p0) rows per image); used to time bounded samples. */
+void oracle_conv2d_rows_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
+                            const uint32_t *W, int64_t ldw, int bw, int kw,
+                            int Nb, int H, int Wd, int C, int Cout, int R, int S,
+                            int stride, int pad, int P, int Q, int p0, int p1, int64_t *acc)
+{
+    int cpx = 32 / bx, cpw_ = 32 / bw;
+    uint32_t mx = (1u << bx) - 1u, mw = (1u << bw) - 1u;
+    int64_t tx[256], tw[256];
+    image_table(bx, kx, tx);
+    image_table(bw, kw, tw);
+    int rows = p1 - p0;
+    (void)P;
+    for (int n = 0; n < Nb; n++)
+        for (int p = p0; p < p1; p++)
+            for (int q = 0; q < Q; q++)
+                for (int co = 0; co < Cout; co++) {
+                    int64_t s = 0;
+                    for (int r = 0; r < R; r++)
+                        for (int t = 0; t < S; t++) {
+                            int h = p * stride - pad + r, w = q * stride - pad + t;
+                            if (h < 0 || h >= H || w < 0 || w >= Wd) continue;
+                            const uint32_t *xr = X + (((int64_t)n * H + h) * Wd + w) * ldx;
+                            const uint32_t *wr = W + (((int64_t)co * R + r) * S + t) * ldw;
+                            for (int c = 0; c < C; c++) {
+                                uint32_t cx = (xr[c / cpx] >> (bx * (c % cpx))) & mx;
+                                uint32_t cw = (wr[c / cpw_] >> (bw * (c % cpw_))) & mw;
+                                s += tx[cx] * tw[cw];
+                            }
+                        }
+                    acc[(((int64_t)n * rows + (p - p0)) * Q + q) * Cout + co] = s;
                 }
 }
 

@@ -161,6 +161,9 @@ __device__ __forceinline__ uint4 decode_unit(const Src& src, const typename Src:
 
 struct EpiParams {
     const float* scale;
+    const float* alpha_a_dev;
+    const float* alpha_b_dev;
+    float dq_pow2;            // 2^-(kA+kB)
     const float* bias;
     float scale0, bias0;
     int act;
@@ -290,6 +293,8 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
         const int64_t m = m0 + row;
         const bool mrow = m < M;
         float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
+        const bool dq = ep.alpha_a_dev && ep.alpha_b_dev;
+        const float dqs = dq ? __fmul_rn(__ldg(ep.alpha_a_dev), __ldg(ep.alpha_b_dev)) * ep.dq_pow2 : 1.0f;
         uint8_t* stage_codes = smem;               // 128 x BN bytes, stages are free now
         const int rcpw = ep.residual ? 32 / ep.res_b : 1;
         const uint32_t rmask = ep.residual ? (1u << ep.res_b) - 1u : 0u;
@@ -309,7 +314,8 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
                 if (mrow && n < N) {
                     const float af = __uint_as_float(r[j]) * acc_scale;   // exact integer
                     if (ep.acc_out) ep.acc_out[m * N + n] = __float2int_rn(af);
-                    const float sc = ep.scale ? __ldg(ep.scale + n) : ep.scale0;
+                    float sc = ep.scale ? __ldg(ep.scale + n) : ep.scale0;
+                    if (dq) sc = __fmul_rn(sc, dqs);
                     const float bi = ep.bias ? __ldg(ep.bias + n) : ep.bias0;
                     float y = __fmaf_rn(sc, af, bi);
                     if (ep.residual) {
@@ -395,6 +401,9 @@ static EpiParams make_epi(const GemmOutputs& o)
     EpiParams ep;
     const esb_epilogue* e = o.ep;
     ep.scale = e ? e->scale : nullptr;
+    ep.alpha_a_dev = e ? e->alpha_a_dev : nullptr;
+    ep.alpha_b_dev = e ? e->alpha_b_dev : nullptr;
+    ep.dq_pow2 = 1.0f;
     ep.bias = e ? e->bias : nullptr;
     ep.scale0 = e ? e->scale0 : 1.0f;
     ep.bias0 = e ? e->bias0 : 0.0f;
@@ -422,7 +431,8 @@ static EpiParams make_epi(const GemmOutputs& o)
 cudaError_t launch_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, int ba, int ka,
                         const uint32_t* B, int64_t ldb, int bb, int kb, const GemmOutputs& o, cudaStream_t st)
 {
-    const EpiParams ep = make_epi(o);
+    EpiParams ep = make_epi(o);
+    ep.dq_pow2 = ldexpf(1.0f, -(ka + kb));
     const int BN = pick_bn(N, ep.out_cpw);
     RowsSrc a{A, lda, M};
     RowsSrc b{B, ldb, N};
@@ -432,7 +442,8 @@ cudaError_t launch_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int6
 cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
                            const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st)
 {
-    const EpiParams ep = make_epi(o);
+    EpiParams ep = make_epi(o);
+    ep.dq_pow2 = ldexpf(1.0f, -(kx + kw));
     const int64_t M = (int64_t)d.n * P * Q;
     const int64_t N = d.cout;
     const int64_t K = (int64_t)d.r * d.s * ldx * (32 / bx);

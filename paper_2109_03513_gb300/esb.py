@@ -44,7 +44,8 @@ class esb_format(ctypes.Structure):
 
 class esb_epilogue(ctypes.Structure):
     _fields_ = [
-        ("scale", ctypes.c_void_p), ("bias", ctypes.c_void_p),
+        ("scale", ctypes.c_void_p), ("alpha_a_dev", ctypes.c_void_p), ("alpha_b_dev", ctypes.c_void_p),
+        ("bias", ctypes.c_void_p),
         ("scale0", ctypes.c_float), ("bias0", ctypes.c_float),
         ("act", ctypes.c_int32),
         ("residual", ctypes.c_void_p), ("res_ld", ctypes.c_int64), ("res_fmt", esb_format),
@@ -214,6 +215,8 @@ class Epilogue:
     """Fused post-processing (include/esb.h, esb_epilogue)."""
     scale: Optional[torch.Tensor] = None
     bias: Optional[torch.Tensor] = None
+    alpha_a_dev: Optional[torch.Tensor] = None
+    alpha_b_dev: Optional[torch.Tensor] = None
     scale0: float = 1.0
     bias0: float = 0.0
     act: int = ESB_ACT_NONE
@@ -229,6 +232,8 @@ class Epilogue:
         e = esb_epilogue()
         e.scale = None if self.scale is None else self.scale.data_ptr()
         e.bias = None if self.bias is None else self.bias.data_ptr()
+        e.alpha_a_dev = None if self.alpha_a_dev is None else self.alpha_a_dev.data_ptr()
+        e.alpha_b_dev = None if self.alpha_b_dev is None else self.alpha_b_dev.data_ptr()
         e.scale0 = self.scale0
         e.bias0 = self.bias0
         e.act = self.act

@@ -94,7 +94,7 @@ def test_gemm_exact_near_the_accumulation_bound(fmt, K):
 
 
 def test_gemm_range_error():
-    A = np.zeros((128, 1024), np.uint32)
+    A = np.zeros((128, esb.esb_row_words(8192, 6)), np.uint32)
     with pytest.raises(esb.EsbError) as e:
         esb.esb_gemm(dev_i32(A), esb.Fmt(6, 3), dev_i32(A), esb.Fmt(6, 3), 8192)
     assert e.value.status == esb.ESB_ERR_RANGE
@@ -178,3 +178,32 @@ def test_conv_matches_oracle(n, h, w, c, cout, r, s, stride, pad, fx, fw):
     yo, co = o.epilogue(acc_o, np.full(cout, s0, np.float32), np.zeros(cout, np.float32), 1, 0.7, fo)
     assert np.array_equal(y.cpu().numpy(), yo)
     assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
+def test_conv_dequant_scale_from_device_alphas():
+    # calibrate -> project -> conv with the "Scale" stage taken from the two
+    # device alphas (no host round trip), as bench.py runs it.
+    n, h, w, c, cout = 2, 12, 12, 64, 64
+    fu, fs = esb.Fmt(4, 2, False), esb.Fmt(4, 2, True)
+    x = synth.half_normal((n * h * w, c), seed=21)
+    wt = synth.he_normal((cout * 9, c), fan_in=576, seed=22)
+    xd, wd = x.cuda(), wt.cuda()
+    ax, _ = esb.esb_calibrate_dda(xd, fu)
+    aw, _ = esb.esb_calibrate_dda(wd, fs)
+    Xc = esb.esb_project(xd, fu, alpha=ax)
+    Wc = esb.esb_project(wd, fs, alpha=aw)
+    ep = esb.Epilogue(scale0=1.0, alpha_a_dev=ax, alpha_b_dev=aw, bias0=-0.01, act=esb.ESB_ACT_RELU,
+                      alpha_out=0.3, fmt_out=fu)
+    acc, y, codes = esb.esb_conv2d_nhwc(Xc, fu, Wc, fs, n, h, w, c, cout, 3, 3, 1, 1, ep=ep, want_acc=True,
+                                        want_y=True, want_codes=True)
+    axh, awh = np.float32(ax.item()), np.float32(aw.item())
+    dq = np.float32(np.float32(axh * awh) * np.float32(2.0 ** -4))
+    sc = np.float32(np.float32(1.0) * dq)
+    Xo = o.project_packed(x.numpy(), float(axh), 4, 2, False, ld_words=Xc.shape[1])
+    Wo = o.project_packed(wt.numpy(), float(awh), 4, 2, True, ld_words=Wc.shape[1])
+    acc_o = o.conv2d_i64(Xo.reshape(n, h, w, -1), (4, 2), Wo.reshape(cout, 3, 3, -1), (4, 2),
+                         n, h, w, c, cout, 3, 3, 1, 1).reshape(-1, cout)
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), acc_o)
+    yo, co = o.epilogue(acc_o, np.full(cout, sc, np.float32), np.full(cout, -0.01, np.float32), 1, 0.3, (4, 2, False))
+    assert np.array_equal(y.cpu().numpy(), yo)
+    assert np.array_equal(u32(codes), o.pack(co, 4, 2, ld_words=codes.shape[1]))

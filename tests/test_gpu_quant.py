@@ -135,7 +135,7 @@ def test_calibrate_offset_constant_and_determinism():
     ac, _ = esb.esb_calibrate_dda(c.cuda(), f)
     assert ac.item() == np.float32(o.alpha_star(4, 2)[0] * 1e-7)
     # unaligned base pointer takes the scalar path
-    xu = synth.normal((1 << 12) + 1, seed=4)
+    xu = synth.normal(((1 << 12) + 1,), seed=4)
     xd = xu.cuda()[1:]
     au, _ = esb.esb_calibrate_dda(xd, f)
     ao2, _ = o.calibrate(xu.numpy()[1:], 4, 2)
