@@ -165,6 +165,34 @@ esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
                              void* workspace, size_t workspace_bytes,
                              float* alpha_out, double* stats_out, void* stream);
 
+/* Size of the fixed scratch array behind esb_calibrate_dda_noalloc. */
+#define ESB_CALIBRATE_NOALLOC_SCRATCH_BYTES 32768
+
+/* esb_calibrate_dda without a workspace argument (the paper has no
+ * counterpart; this is a deployment convenience).  Some callers cannot
+ * allocate device memory: a plug-in that only receives input and output
+ * pointers from its host application and has no allocator to call, a
+ * framework whose caching allocator already holds the device's memory (a
+ * direct cudaMalloc can then fail, or fragment memory it manages), or a
+ * serving loop that must not allocate after start-up.  This entry point
+ * computes the same alpha and statistics as esb_calibrate_dda but keeps its
+ * scratch (one 32-byte record per reduction block, at most
+ * ESB_CALIBRATE_NOALLOC_SCRATCH_BYTES) in a fixed array inside the library;
+ * every GPU that loads the library holds that array until the process
+ * exits.  It calls no cudaMalloc, cudaFree or other allocating routine.
+ *   x          [device] n floats; n > 0
+ *   alpha_out  [device] 1 float; stats_out [device] 3 doubles or NULL
+ * The first call on a device looks up the array's device address (with
+ * that device current) and caches it; make that first call before any
+ * stream capture.  All calls share the one array and it keeps the last
+ * call's contents (each call overwrites every record it later reads, so
+ * nothing has to be cleared): calls whose kernels overlap on the GPU (on
+ * different streams without ordering) race on it and must be serialised.
+ * Errors: INVALID_ARG, UNSUPPORTED, RANGE (scratch need above the array's
+ * size; the reduction uses at most 1024 blocks, so no n exceeds it), CUDA. */
+esb_status esb_calibrate_dda_noalloc(const float* x, int64_t n, esb_format f,
+                                     float* alpha_out, double* stats_out, void* stream);
+
 /* ------------------------------------------------------------- project */
 
 /* Cheap projection operator of Eq. cheap_projection with the

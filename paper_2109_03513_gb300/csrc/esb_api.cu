@@ -156,6 +156,19 @@ esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f, void* work
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 
+esb_status esb_calibrate_dda_noalloc(const float* x, int64_t n, esb_format f, float* alpha_out, double* stats_out,
+                                     void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (!x || n <= 0 || !alpha_out) return ESB_ERR_INVALID_ARG;
+    if (calibrate_workspace_bytes(n) > calibrate_noalloc_capacity()) return ESB_ERR_RANGE;
+    double as = 0.0;
+    alpha_star_cached(f.b, f.k, &as, nullptr);
+    cudaError_t e = launch_calibrate_noalloc(x, n, f.is_signed, as, alpha_out, stats_out,
+                                             static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
 esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx, float alpha, const float* alpha_dev,
                        esb_format f, int32_t rounding, uint32_t* codes, int64_t ldc, void* stream)
 {

@@ -4,6 +4,7 @@
 //   * dequantisation (Sec. IV-A, Eq. q),
 //   * DDA calibration statistics and alpha (Sec. III-D).
 #include <cstdint>
+#include <mutex>
 #include <cuda_runtime.h>
 
 #include "esb_common.cuh"
@@ -314,6 +315,54 @@ cudaError_t launch_calibrate(const float* x, int64_t n, int is_signed, double al
     if (e != cudaSuccess) return e;
     calibrate_finalize_kernel<<<1, kCalThreads, 0, st>>>(part, g, alpha_star, is_signed, alpha_out, stats_out);
     return cudaGetLastError();
+}
+
+// ------------------------------------------- calibration without workspace
+
+// Scratch of esb_calibrate_dda_noalloc: room for the partial record of every
+// block the reduction can launch (kCalMaxBlocks x 32 bytes = 32 KiB).  It is
+// a file-scope device array, so it exists on every GPU that loads the
+// library until the process exits, and every call of the variant shares it.
+static_assert(sizeof(CalPartial) == 32, "partial record layout");
+static __device__ __align__(256) unsigned char g_cal_noalloc_scratch[kCalMaxBlocks * 32];
+
+namespace {
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[64] = {nullptr};
+}  // namespace
+
+size_t calibrate_noalloc_capacity() { return sizeof(g_cal_noalloc_scratch); }
+
+// The host-side name of the array is only a stand-in, never a device
+// address: the address is looked up once per device (with that device
+// current) and cached.
+static cudaError_t noalloc_scratch_address(void** out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_cal_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return cudaSuccess;
+}
+
+cudaError_t launch_calibrate_noalloc(const float* x, int64_t n, int is_signed, double alpha_star, float* alpha_out,
+                                     double* stats_out, cudaStream_t st)
+{
+    if (calibrate_workspace_bytes(n) > sizeof(g_cal_noalloc_scratch)) return cudaErrorInvalidValue;
+    void* ws = nullptr;
+    cudaError_t e = noalloc_scratch_address(&ws);
+    if (e != cudaSuccess) return e;
+    // Pass 1 writes every partial record that pass 2 reads, so nothing in the
+    // shared scratch has to be cleared between calls.
+    return launch_calibrate(x, n, is_signed, alpha_star, ws, alpha_out, stats_out, st);
 }
 
 }  // namespace esb

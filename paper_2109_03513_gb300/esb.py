@@ -84,6 +84,7 @@ SIGNATURES = {
     "esb_alpha_star": (_I32, [_I32, _I32, _P, _P]),
     "esb_calibrate_dda_workspace_bytes": (_SZ, [_I64]),
     "esb_calibrate_dda": (_I32, [_P, _I64, esb_format, _P, _SZ, _P, _P, _P]),
+    "esb_calibrate_dda_noalloc": (_I32, [_P, _I64, esb_format, _P, _P, _P]),
     "esb_project": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _I32, _P, _I64, _P]),
     "esb_dequant": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _P, _I64, _P]),
     "esb_gemm": (_I32, [_I64, _I64, _I64, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
@@ -170,6 +171,22 @@ def esb_calibrate_dda(x: torch.Tensor, f: Fmt, alpha_out: Optional[torch.Tensor]
         workspace = torch.empty(max(nb, 8), dtype=torch.uint8, device=x.device)
     _check(lib().esb_calibrate_dda(_ptr(x), n, f.c(), _ptr(workspace), workspace.numel(), _ptr(alpha_out),
                                    _ptr(stats_out), _stream(stream)), "esb_calibrate_dda")
+    return alpha_out, stats_out
+
+
+def esb_calibrate_dda_noalloc(x: torch.Tensor, f: Fmt, alpha_out: Optional[torch.Tensor] = None,
+                              stats_out: Optional[torch.Tensor] = None,
+                              stream=None) -> tuple[torch.Tensor, Optional[torch.Tensor]]:
+    """esb_calibrate_dda for callers that cannot allocate device memory: the
+    scratch is a fixed array inside libesb.so, so no workspace is passed (the
+    caller still supplies x, alpha_out and stats_out).  Calls that overlap on
+    the GPU share that array and must be serialised."""
+    _dev(x, "x")
+    assert x.dtype == torch.float32
+    if alpha_out is None:
+        alpha_out = torch.empty(1, dtype=torch.float32, device=x.device)
+    _check(lib().esb_calibrate_dda_noalloc(_ptr(x), x.numel(), f.c(), _ptr(alpha_out), _ptr(stats_out),
+                                           _stream(stream)), "esb_calibrate_dda_noalloc")
     return alpha_out, stats_out
 
 
