@@ -254,7 +254,10 @@ esb_status esb_gemm(int64_t M, int64_t N, int64_t K,
  *   W [device] cout*r*s rows of ldw words (c codes each); ldw == ldx
  *   outputs as esb_gemm with M = n*P*Q rows (pixel-major NHWC).
  * groups == c selects the depthwise path (one r x s filter per channel, W
- * holds r*s rows of ldw words with c codes each, cout == c).
+ * holds r*s rows of ldw words with c codes each, cout == c), which runs on
+ * CUDA cores (no dense contraction): exact int32 sums of r*s products, the
+ * same epilogue; there fmt_out.b must equal fx.b and
+ * r*s*max|I_X|*max|I_W| < 2^31.
  * Errors: INVALID_ARG, UNSUPPORTED, RANGE, ALIGN, CUDA. */
 esb_status esb_conv2d_nhwc(const esb_conv_desc* d,
                            const uint32_t* X, int64_t ldx, esb_format fx,
@@ -262,6 +265,35 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d,
                            const esb_epilogue* ep,
                            int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
                            void* stream);
+
+/* -------------------------------------------------------------- pooling */
+
+/* Max pooling of ESB codes, NHWC (Sec. IV-B "MP" stage with the
+ * intersection window: a window that runs past the border is cut to the
+ * part inside the image).  The projection is monotone, so the maximum of
+ * the codes' values is the value of the projected maximum; each output
+ * slot holds the input code of largest value (the zero code for zero).
+ *   X [device] n*h*w pixel rows of ldx words (c codes each, format f)
+ *   Y [device] n*P*Q rows of ldy words, P = (h + 2 pad - win)/stride + 1
+ *     (for 3x3/2 pad 1 this is ceil(h/2), the paper's output size)
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+esb_status esb_maxpool_nhwc(const uint32_t* X, int64_t ldx, esb_format f,
+                            int32_t n, int32_t h, int32_t w, int32_t c,
+                            int32_t win, int32_t stride, int32_t pad,
+                            uint32_t* Y, int64_t ldy, void* stream);
+
+/* Global average pooling of ESB codes (the pooling before ResNet18's and
+ * MobileNetV2's classifier): s[i][ch] = sum over the hw pixels of the
+ * integer images (exact int32), y = fl32(scale * (float)s) (scale carries
+ * alpha * 2^-k / hw), then y is projected with alpha_out / fmt_out as in
+ * esb_project.  fmt_out.b must equal f.b.
+ *   X [device] n*hw pixel rows of ldx words; y_out [device] n x c floats
+ *   or NULL; codes_out [device] n rows of ldo words or NULL.
+ * Errors: INVALID_ARG, UNSUPPORTED, RANGE, CUDA. */
+esb_status esb_avgpool_nhwc(const uint32_t* X, int64_t ldx, esb_format f,
+                            int32_t n, int32_t hw, int32_t c, float scale,
+                            float alpha_out, esb_format fmt_out, int32_t rounding,
+                            float* y_out, uint32_t* codes_out, int64_t ldo, void* stream);
 
 /* ------------------------------------------------------------- status */
 

@@ -231,15 +231,28 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d, const uint32_t* X, int64_t ld
         return ESB_ERR_INVALID_ARG;
     if (d->h + 2 * d->pad < d->r || d->w + 2 * d->pad < d->s) return ESB_ERR_INVALID_ARG;
     if (d->pad >= d->r || d->pad >= d->s) return ESB_ERR_INVALID_ARG;
-    if (ldx < words_for(d->c, fx.b) || ldw != ldx) return ESB_ERR_INVALID_ARG;
+    if (ldx < words_for(d->c, fx.b)) return ESB_ERR_INVALID_ARG;
     const int P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
     const int Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
     const int64_t M = (int64_t)d->n * P * Q;
     const bool want_codes = codes_out != nullptr;
     if (d->groups == d->c && d->c > 1) {
-        return ESB_ERR_UNSUPPORTED;  // depthwise path: not built yet
+        if (d->cout != d->c) return ESB_ERR_INVALID_ARG;
+        if (ldw < words_for(d->c, fw.b)) return ESB_ERR_INVALID_ARG;
+        esb_status s = check_epilogue(ep, M, d->c, want_codes || y_out != nullptr);
+        if (s != ESB_OK) return s;
+        if (want_codes && (ep->fmt_out.b != fx.b || ldo < words_for(d->c, fx.b))) return ESB_ERR_INVALID_ARG;
+        if ((double)d->r * d->s * fmt_max_image(fx.b, fx.k) * fmt_max_image(fw.b, fw.k) >= 2147483648.0)
+            return ESB_ERR_RANGE;
+        if (M == 0 || (!acc_out && !y_out && !codes_out)) return ESB_OK;
+        if (!X || !W) return ESB_ERR_INVALID_ARG;
+        GemmOutputs o{ep, acc_out, y_out, codes_out, ldo};
+        cudaError_t e = launch_dwconv(*d, P, Q, X, ldx, fx.b, fx.k, W, ldw, fw.b, fw.k, o,
+                                      static_cast<cudaStream_t>(stream));
+        return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
     }
     if (d->groups != 1) return ESB_ERR_UNSUPPORTED;
+    if (ldw != ldx) return ESB_ERR_INVALID_ARG;
     if (fx.b != fw.b) return ESB_ERR_UNSUPPORTED;
     if (!fmt_tc_ok(fx) || !fmt_tc_ok(fw)) return ESB_ERR_UNSUPPORTED;
     esb_status s = check_epilogue(ep, M, d->cout, want_codes || y_out != nullptr);
@@ -255,6 +268,40 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d, const uint32_t* X, int64_t ld
     if (!gemm_pick_ok(d->cout, want_codes ? ep->fmt_out.b : 4)) return ESB_ERR_UNSUPPORTED;
     GemmOutputs o{ep, acc_out, y_out, codes_out, ldo};
     cudaError_t e = launch_conv_tc(*d, P, Q, X, ldx, fx.b, fx.k, W, ldw, fw.b, fw.k, o, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_maxpool_nhwc(const uint32_t* X, int64_t ldx, esb_format f, int32_t n, int32_t h, int32_t w, int32_t c,
+                            int32_t win, int32_t stride, int32_t pad, uint32_t* Y, int64_t ldy, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (n < 0 || h <= 0 || w <= 0 || c <= 0 || win <= 0 || stride <= 0 || pad < 0 || pad >= win) return ESB_ERR_INVALID_ARG;
+    if (h + 2 * pad < win || w + 2 * pad < win) return ESB_ERR_INVALID_ARG;
+    if (ldx < words_for(c, f.b) || ldy < words_for(c, f.b)) return ESB_ERR_INVALID_ARG;
+    const int P = (h + 2 * pad - win) / stride + 1, Q = (w + 2 * pad - win) / stride + 1;
+    if (n == 0) return ESB_OK;
+    if (!X || !Y) return ESB_ERR_INVALID_ARG;
+    cudaError_t e = launch_maxpool(X, ldx, f.b, f.k, n, h, w, c, win, stride, pad, P, Q, Y, ldy,
+                                   static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_avgpool_nhwc(const uint32_t* X, int64_t ldx, esb_format f, int32_t n, int32_t hw, int32_t c, float scale,
+                            float alpha_out, esb_format fmt_out, int32_t rounding, float* y_out, uint32_t* codes_out,
+                            int64_t ldo, void* stream)
+{
+    if (!fmt_ok(f) || !fmt_ok(fmt_out)) return ESB_ERR_UNSUPPORTED;
+    if (n < 0 || hw <= 0 || c <= 0 || ldx < words_for(c, f.b)) return ESB_ERR_INVALID_ARG;
+    if (fmt_out.b != f.b) return ESB_ERR_INVALID_ARG;
+    if (codes_out && ldo < words_for(c, f.b)) return ESB_ERR_INVALID_ARG;
+    if (rounding != ESB_ROUND_HALF_AWAY && rounding != ESB_ROUND_HALF_EVEN) return ESB_ERR_INVALID_ARG;
+    if (!std::isfinite(scale) || !(std::isfinite(alpha_out) && alpha_out > 0.0f)) return ESB_ERR_INVALID_ARG;
+    if ((double)hw * fmt_max_image(f.b, f.k) >= 2147483648.0) return ESB_ERR_RANGE;
+    if (n == 0 || (!y_out && !codes_out)) return ESB_OK;
+    if (!X) return ESB_ERR_INVALID_ARG;
+    if ((int64_t)n > 65535) return ESB_ERR_UNSUPPORTED;
+    cudaError_t e = launch_avgpool(X, ldx, f.b, f.k, n, hw, c, scale, alpha_out, fmt_out.b, fmt_out.k, fmt_out.is_signed,
+                                   rounding, y_out, codes_out, ldo, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 

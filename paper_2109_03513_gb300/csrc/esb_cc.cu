@@ -275,6 +275,14 @@ esb_avgpool_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int k, in
     const uint32_t mask = (1u << b) - 1u;
     const int64_t nn = blockIdx.y;
     const int w = blockIdx.x;                           // code word of the channel group
+    if (w * cpw >= C) {                                 // padding word of the output row
+        if (threadIdx.x == 0 && codes_out && w < ldo) {
+            uint32_t word = 0;
+            for (int j = 0; j < 32 / out.b; j++) word |= out.zero_code << (out.b * j);
+            codes_out[nn * ldo + w] = word;
+        }
+        return;
+    }
     __shared__ int32_t red[256][16];
     int32_t acc[16];
 #pragma unroll
@@ -316,7 +324,8 @@ cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
                            int64_t ldo, cudaStream_t st)
 {
     ProjParams out = make_proj_params(bo, ko, so, rounding);
-    const int words = (C + (32 / b) - 1) / (32 / b);
+    int64_t words = (C + (32 / b) - 1) / (32 / b);
+    if (codes_out && ldo > words) words = ldo;          // also write the row's padding words
     dim3 grid((unsigned)words, (unsigned)n);
     esb_avgpool_kernel<<<grid, 256, 0, st>>>(X, ldx, b, k, HW, C, scale, alpha_out, out, y_out, codes_out, ldo);
     return cudaGetLastError();

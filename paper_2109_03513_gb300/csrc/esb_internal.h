@@ -46,6 +46,14 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
 
 bool gemm_pick_ok(int64_t N, int out_b);
 
+cudaError_t launch_dwconv(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
+                          const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st);
+cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int H, int Wd, int C, int win,
+                           int stride, int pad, int P, int Q, uint32_t* Y, int64_t ldy, cudaStream_t st);
+cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int HW, int C, float scale,
+                           float alpha_out, int bo, int ko, int so, int rounding, float* y_out, uint32_t* codes_out,
+                           int64_t ldo, cudaStream_t st);
+
 // alpha*(b,k) and 2*D(alpha*) (Sec. III-D), solved on the host in fp64.
 double alpha_star_solve(int b, int k, double* dda);
 

@@ -89,6 +89,9 @@ SIGNATURES = {
     "esb_dequant": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _P, _I64, _P]),
     "esb_gemm": (_I32, [_I64, _I64, _I64, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
     "esb_conv2d_nhwc": (_I32, [_P, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
+    "esb_maxpool_nhwc": (_I32, [_P, _I64, esb_format] + [_I32] * 7 + [_P, _I64, _P]),
+    "esb_avgpool_nhwc": (_I32, [_P, _I64, esb_format, _I32, _I32, _I32, _F32, _F32, esb_format, _I32, _P, _P, _I64,
+                                _P]),
     "esb_get_status": (_I32, [_P, _P]),
 }
 
@@ -317,6 +320,31 @@ def esb_conv2d_nhwc(X: torch.Tensor, fx: Fmt, W: torch.Tensor, fw: Fmt, n: int, 
                                  ctypes.byref(epc) if epc is not None else None,
                                  _ptr(acc), _ptr(y), _ptr(codes), ldo, _stream(stream)), "esb_conv2d_nhwc")
     return acc, y, codes
+
+
+def esb_maxpool_nhwc(X: torch.Tensor, f: Fmt, n: int, h: int, w: int, c: int, win: int = 3, stride: int = 2,
+                     pad: int = 1, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Max pooling of NHWC codes; returns (n*P*Q, ldx) int32 codes."""
+    _dev(X, "X")
+    ldx = X.shape[-1]
+    P, Q = conv_out_hw(h, w, win, win, stride, pad)
+    Y = out if out is not None else torch.empty((n * P * Q, ldx), dtype=torch.int32, device=X.device)
+    _check(lib().esb_maxpool_nhwc(_ptr(X), ldx, f.c(), n, h, w, c, win, stride, pad, _ptr(Y), Y.shape[-1],
+                                  _stream(stream)), "esb_maxpool_nhwc")
+    return Y
+
+
+def esb_avgpool_nhwc(X: torch.Tensor, f: Fmt, n: int, hw: int, c: int, scale: float, alpha_out: float, fmt_out: Fmt,
+                     rounding: int = ESB_ROUND_HALF_AWAY, want_y: bool = False, stream=None):
+    """Global average pooling of NHWC codes -> (y (n, c) fp32 | None, codes (n, ldo) int32)."""
+    _dev(X, "X")
+    ldx = X.shape[-1]
+    y = torch.empty((n, c), dtype=torch.float32, device=X.device) if want_y else None
+    ldo = esb_row_words(c, fmt_out.b)
+    codes = torch.empty((n, ldo), dtype=torch.int32, device=X.device)
+    _check(lib().esb_avgpool_nhwc(_ptr(X), ldx, f.c(), n, hw, c, scale, alpha_out, fmt_out.c(), rounding, _ptr(y),
+                                  _ptr(codes), ldo, _stream(stream)), "esb_avgpool_nhwc")
+    return y, codes
 
 
 def esb_get_status(stream=None) -> int:
