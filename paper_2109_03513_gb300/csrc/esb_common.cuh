@@ -127,6 +127,125 @@ __device__ __forceinline__ uint32_t project_code(float x, float alpha, const Pro
     return project_scaled(__fdiv_rn(x, alpha), p);
 }
 
+// ------------------------------------------- projection by thresholds
+
+// For a fixed alpha the code of x depends only on which midpoints t_j
+// (between consecutive non-negative set elements q_j < q_(j+1)) the value
+// v = fl(|x| / alpha) reaches.  IEEE division is monotone in |x|, so
+// "v >= t_j" is exactly "|x| >= T_j" for the smallest float T_j with that
+// property ("v > t_j" when the tie at t_j goes down under half-to-even).
+// The T_j are found once per kernel with the same division, after which a
+// projection needs no division at all -- a different evaluation order of
+// Eq. cheap_projection with identical results.
+constexpr int kMaxThresholds = 127;    // 2^(b-1) - 1 for b = 8
+
+// Element j (0-based, ascending) of the non-negative set, in units of alpha.
+__device__ __forceinline__ float set_element(int j, int k)
+{
+    const int one = 1 << k;
+    if (j < one) return ldexpf((float)j, -k);
+    return ldexpf((float)(one + (j & (one - 1))), (j >> k) - 1 - k);
+}
+
+// T_j computed by one full warp.  Start from x0 = fl(t * alpha), which is
+// within a few ulps of T_j; 32 consecutive candidates around it are tested
+// at once.  If they do not bracket T_j (over/underflow ranges), fall back to
+// a bisection over all non-negative fp32 bit patterns.
+__device__ inline float warp_threshold(float alpha, float t, bool strict, int lane)
+{
+    const uint32_t b0 = __float_as_uint(__fmul_rn(t, alpha));
+    if (b0 >= 16u && b0 < 0x7f800000u - 16u) {
+        const uint32_t cand = b0 - 16u + (uint32_t)lane;
+        const float v = __fdiv_rn(__uint_as_float(cand), alpha);
+        const bool ok = strict ? (v > t) : (v >= t);
+        const unsigned m = __ballot_sync(0xffffffffu, ok);
+        if ((m & 1u) == 0u && (m >> 31) != 0u) return __uint_as_float(b0 - 16u + (uint32_t)(__ffs(m) - 1));
+    }
+    uint32_t lo = 0u, hi = 0x7f800000u;        // fl(0/alpha) < t (t > 0); fl(inf/alpha) >= t
+    while (hi - lo > 1u) {
+        const uint32_t mid = lo + ((hi - lo) >> 1);
+        const float v = __fdiv_rn(__uint_as_float(mid), alpha);
+        if (strict ? (v > t) : (v >= t)) hi = mid; else lo = mid;
+    }
+    return __uint_as_float(hi);
+}
+
+// Fill T[0 .. L-2] (L = 2^(b-1)) using the warps [warp0, warp0 + nwarps).
+// The caller synchronises before reading T.
+__device__ inline void build_thresholds(float* T, const ProjParams& p, float alpha, int warp, int lane, int warp0,
+                                        int nwarps)
+{
+    const int L = 1 << (p.b - 1);
+    for (int j = warp - warp0; j < L - 1; j += nwarps) {
+        const float q0 = set_element(j, p.k), q1 = set_element(j + 1, p.k);
+        const float t = 0.5f * (q0 + q1);                 // exact
+        bool strict = false;
+        if (p.rounding) {                                 // half-even: tie goes to the even multiple
+            const int r = (int)(q1 / (q1 - q0));          // spacing is a power of two: exact
+            strict = (r & 1) != 0;
+        }
+        const float Tj = warp_threshold(alpha, t, strict, lane);
+        if (lane == 0) T[j] = Tj;
+    }
+}
+
+// Code of x by the thresholds (bucket = number of T_j <= |x|).
+__device__ __forceinline__ uint32_t project_by_table(float x, const float* T, const ProjParams& p)
+{
+    const uint32_t u = __float_as_uint(x);
+    const uint32_t sign = u >> 31;
+    const float a = __uint_as_float(u & 0x7fffffffu);
+    const int L = 1 << (p.b - 1);
+    int j = 0;
+#pragma unroll 1
+    for (int step = L >> 1; step > 0; step >>= 1)
+        if (a >= T[j + step - 1]) j += step;
+    if (j == 0 || (sign && !p.is_signed)) return p.zero_code;    // zero (and NaN) carry sign 0
+    const int one = 1 << p.k;
+    const uint32_t mag = (j >= one) ? (uint32_t)(j - one) : (((uint32_t)p.N << p.k) | (uint32_t)j);
+    return mag | (sign << (p.b - 1));
+}
+
+// The same with the table in registers for b = 4 (7 thresholds).
+struct Thr7 { float t[7]; };
+
+__device__ __forceinline__ uint32_t project_by_thr7(float x, const Thr7& T, const ProjParams& p)
+{
+    const uint32_t u = __float_as_uint(x);
+    const uint32_t sign = u >> 31;
+    const float a = __uint_as_float(u & 0x7fffffffu);
+    int j = (a >= T.t[3]) ? 4 : 0;
+    j += (a >= (j ? T.t[5] : T.t[1])) ? 2 : 0;
+    const float t3 = (j & 4) ? ((j & 2) ? T.t[6] : T.t[4]) : ((j & 2) ? T.t[2] : T.t[0]);
+    j += (a >= t3) ? 1 : 0;
+    if (j == 0 || (sign && !p.is_signed)) return p.zero_code;
+    const int one = 1 << p.k;
+    const uint32_t mag = (j >= one) ? (uint32_t)(j - one) : (((uint32_t)p.N << p.k) | (uint32_t)j);
+    return mag | (sign << 3);
+}
+
+// Bucket (0..7) of a against 7 ascending thresholds: the number of T_j <= a.
+__device__ __forceinline__ uint32_t bucket7(float a, const Thr7& T)
+{
+    uint32_t j = (a >= T.t[3]) ? 4u : 0u;
+    j |= (a >= (j ? T.t[5] : T.t[1])) ? 2u : 0u;
+    const float t3 = (j & 4u) ? ((j & 2u) ? T.t[6] : T.t[4]) : ((j & 2u) ? T.t[2] : T.t[0]);
+    j |= (a >= t3) ? 1u : 0u;
+    return j;
+}
+
+// Eight 4-bit codes at once from their buckets J (one per nibble, 0..7) and
+// sign bits S (bit 3 of each nibble).  Element j of the non-negative set has
+// the code (j - 2^k) mod 2^(b-1) -- the exponent field rotated by one, as in
+// the decode -- so the whole word is one add and a mask; zero (j = 0) keeps
+// sign 0.
+__device__ __forceinline__ uint32_t codes8_b4(uint32_t J, uint32_t S, int k)
+{
+    const uint32_t C1 = 0x88888888u - (0x11111111u << k);   // 8 - 2^k per nibble: no borrow across nibbles
+    const uint32_t nz = (J + 0x77777777u) & 0x88888888u;      // bit 3 set where j >= 1
+    return ((J + C1) & 0x77777777u) | (S & nz);
+}
+
 // Value of a code in units of alpha (Sec. IV-A, Eq. q), exact in fp32 for b <= 8.
 __device__ __forceinline__ float code_value(uint32_t c, int b, int k)
 {

@@ -16,15 +16,21 @@
 // K * max|I_A| * max|I_B| < 2^24 (checked on the host), and the epilogue
 // scales it back to the exact int32 sum.
 //
-// Pipeline (per CTA, one 128 x BN output tile): all warps load packed code
-// words and decode them into a kStages-deep ring of shared-memory stages in
-// the 128-byte-swizzled K-major layout; one thread issues
-// tcgen05.mma.kind::f8f6f4 (M = 128, N = BN, K = 32) into a TMEM
-// accumulator and commits each stage to an mbarrier, which gates the reuse
-// of that stage.  The MMAs of one stage run while the next stages are being
-// decoded (the paper's ping-pong buffers, Sec. IV-C/IV-D).  The epilogue
-// reads TMEM with tcgen05.ld and runs the fused affine / residual /
-// activation / requantisation.
+// Two kernels share the decode and the epilogue:
+//  * esb_gemm_ws_kernel (B resident): persistent, warp-specialised.  The
+//    CTA decodes its N-tile of B once into shared memory; 8 producer warps
+//    decode A tiles into an 8-deep ring of shared-memory stages; one MMA
+//    warp issues tcgen05.mma (M = 128, N = BN, K = 32) into one of two TMEM
+//    accumulators and commits each stage to the mbarrier that frees it;
+//    4 epilogue warps drain the other accumulator with tcgen05.ld, so the
+//    post-processing of tile i overlaps the MMAs of tile i+1 and the decode
+//    of later tiles (the paper's ping-pong buffers and overlapped timing
+//    graph, Sec. IV-C/IV-D).
+//  * esb_gemm_tc_kernel (B streamed): one 128 x BN tile per CTA; all warps
+//    decode A and B K-blocks into a ring of stages, one thread issues the
+//    MMAs.  Used when B does not fit in shared memory.
+// Every mbarrier wait is bounded (kWaitLimitNs); on expiry the kernel records
+// ESB_ERR_TIMEOUT, stops issuing work, frees TMEM and returns.
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -35,8 +41,8 @@ namespace esb {
 
 constexpr int kBM = 128;           // rows per tile (TMEM lanes)
 constexpr int kBK = 128;           // codes (= E4M3 bytes) per K-block: one 128-byte swizzle row
-constexpr int kStages = 4;
-constexpr int kGemmThreads = 256;
+constexpr int kStages = 4;         // streamed kernel
+constexpr int kGemmThreads = 256;  // streamed kernel
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
 
 struct OpFmt {
@@ -90,72 +96,123 @@ struct RowsSrc {
     int64_t ld;
     int64_t rows;
     struct Row { const uint32_t* p; };
+    struct Cursor { int64_t w; };
     __device__ __forceinline__ Row row(int64_t r) const { Row x; x.p = (r < rows) ? base + r * ld : nullptr; return x; }
     __device__ __forceinline__ const uint32_t* words(const Row& x, int64_t w) const { return x.p ? x.p + w : nullptr; }
+    __device__ __forceinline__ Cursor cursor(int64_t w) const { Cursor c; c.w = w; return c; }
+    __device__ __forceinline__ void advance(Cursor& c, int dw) const { c.w += dw; }
+    __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const { return x.p ? x.p + c.w : nullptr; }
 };
 
 // Implicit im2col of NHWC codes: row m = (n, p, q) output pixel; logical
 // word w = tap * ldx + word, tap = (r, s); out-of-image taps read as zero.
+// All index arithmetic is 32-bit except the final pixel offset.
 struct ConvSrc {
     const uint32_t* X;
-    int64_t ldx;
-    int64_t rows;                 // n * P * Q
+    int ldx;
+    int rows;                     // n * P * Q
     int H, W, P, Q, S, stride, pad;
-    struct Row { int64_t pix0; int h0, w0; bool valid; };
-    __device__ __forceinline__ Row row(int64_t m) const
+    struct Row { int pix0; int h0, w0; bool valid; };
+    struct Cursor { int r, s, word; };
+    __device__ __forceinline__ Row row(int64_t m64) const
     {
         Row x;
-        x.valid = m < rows;
-        const int64_t pq = (int64_t)P * Q;
-        const int64_t n = x.valid ? m / pq : 0;
-        const int64_t rem = x.valid ? m - n * pq : 0;
-        const int p = (int)(rem / Q), q = (int)(rem - (int64_t)(rem / Q) * Q);
+        const int m = (int)m64;
+        x.valid = m64 < rows;
+        const int pq = P * Q;
+        const int n = x.valid ? m / pq : 0;
+        const int rem = x.valid ? m - n * pq : 0;
+        const int p = rem / Q, q = rem - (rem / Q) * Q;
         x.h0 = p * stride - pad;
         x.w0 = q * stride - pad;
         x.pix0 = n * H;
         return x;
     }
+    __device__ __forceinline__ const uint32_t* tap_ptr(const Row& x, int r, int s, int word) const
+    {
+        const int h = x.h0 + r, ww = x.w0 + s;
+        if (!x.valid || h < 0 || h >= H || ww < 0 || ww >= W) return nullptr;
+        return X + ((int64_t)(x.pix0 + h) * W + ww) * ldx + word;
+    }
     __device__ __forceinline__ const uint32_t* words(const Row& x, int64_t w) const
     {
-        if (!x.valid) return nullptr;
-        const int64_t tap = w / ldx;
-        const int64_t word = w - tap * ldx;
-        const int r = (int)(tap / S), s = (int)(tap - (int64_t)(tap / S) * S);
-        const int h = x.h0 + r, ww = x.w0 + s;
-        if (h < 0 || h >= H || ww < 0 || ww >= W) return nullptr;
-        return X + ((x.pix0 + h) * W + ww) * ldx + word;
+        const int tap = (int)(w / ldx);
+        const int word = (int)(w - (int64_t)tap * ldx);
+        return tap_ptr(x, tap / S, tap - (tap / S) * S, word);
     }
+    __device__ __forceinline__ Cursor cursor(int64_t w) const
+    {
+        Cursor c;
+        const int tap = (int)(w / ldx);
+        c.word = (int)(w - (int64_t)tap * ldx);
+        c.r = tap / S;
+        c.s = tap - c.r * S;
+        return c;
+    }
+    __device__ __forceinline__ void advance(Cursor& c, int dw) const
+    {
+        c.word += dw;
+        while (c.word >= ldx) {
+            c.word -= ldx;
+            if (++c.s == S) { c.s = 0; ++c.r; }
+        }
+    }
+    __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const { return tap_ptr(x, c.r, c.s, c.word); }
 };
+
+// General decode of the 16-code unit [k0, k0 + 16) of one row (any b, K tail).
+template <class Src>
+__device__ __noinline__ uint4 decode_unit_any(const Src& src, const typename Src::Row& row, int64_t k0, int64_t K,
+                                              const OpFmt f)
+{
+    uint32_t o0 = 0u, o1 = 0u, o2 = 0u, o3 = 0u;
+#pragma unroll 1
+    for (int j = 0; j < 16; j++) {
+        const int64_t kk = k0 + j;
+        if (kk >= K) break;
+        const int64_t wi = kk / f.cpw;
+        const int slot = (int)(kk - wi * f.cpw);
+        const uint32_t* p = src.words(row, wi);
+        if (!p) continue;
+        const uint32_t c = (__ldg(p) >> (f.b * slot)) & f.mask;
+        const uint32_t byte = code_to_e4m3(c, f);
+        const int pos = unit_pos(j);
+        const uint32_t v = byte << (8 * (pos & 3));
+        switch (pos >> 2) {
+        case 0: o0 |= v; break;
+        case 1: o1 |= v; break;
+        case 2: o2 |= v; break;
+        default: o3 |= v; break;
+        }
+    }
+    return make_uint4(o0, o1, o2, o3);
+}
+
+// Fast decode of a full b = 4 unit (two words) at a cursor.
+template <class Src>
+__device__ __forceinline__ uint4 decode_unit_b4(const Src& src, const typename Src::Row& row,
+                                                const typename Src::Cursor& c, const OpFmt& f)
+{
+    uint32_t o[4] = {0u, 0u, 0u, 0u};
+    const uint32_t* p = src.at(row, c);
+    if (p) {
+        const uint2 w = __ldg(reinterpret_cast<const uint2*>(p));
+        decode_word_b4(w.x, f.k, f.ew, o[0], o[1]);
+        decode_word_b4(w.y, f.k, f.ew, o[2], o[3]);
+    }
+    return make_uint4(o[0], o[1], o[2], o[3]);
+}
 
 // Decode the 16-code unit [k0, k0 + 16) of one row into 16 bytes.
 template <class Src>
 __device__ __forceinline__ uint4 decode_unit(const Src& src, const typename Src::Row& row, int64_t k0, int64_t K,
                                              const OpFmt& f)
 {
-    uint32_t o[4] = {0u, 0u, 0u, 0u};
-    if (f.b == 4 && k0 + 16 <= K) {
-        const uint32_t* p = src.words(row, k0 >> 3);
-        if (p) {
-            const uint2 w = __ldg(reinterpret_cast<const uint2*>(p));
-            decode_word_b4(w.x, f.k, f.ew, o[0], o[1]);
-            decode_word_b4(w.y, f.k, f.ew, o[2], o[3]);
-        }
-    } else {
-        uint8_t* ob = reinterpret_cast<uint8_t*>(o);
-#pragma unroll 1
-        for (int j = 0; j < 16; j++) {
-            const int64_t kk = k0 + j;
-            if (kk >= K) break;
-            const int64_t wi = kk / f.cpw;
-            const int slot = (int)(kk - wi * f.cpw);
-            const uint32_t* p = src.words(row, wi);
-            if (!p) continue;
-            const uint32_t c = (__ldg(p) >> (f.b * slot)) & f.mask;
-            ob[unit_pos(j)] = (uint8_t)code_to_e4m3(c, f);
-        }
-    }
-    return make_uint4(o[0], o[1], o[2], o[3]);
+    if (f.b == 4 && k0 + 16 <= K) return decode_unit_b4(src, row, src.cursor(k0 >> 3), f);
+    return decode_unit_any(src, row, k0, K, f);
 }
+
+__device__ __forceinline__ uint32_t swz(int r, int g) { return (uint32_t)(r * 128 + ((g ^ (r & 7)) << 4)); }
 
 // ------------------------------------------------------------ epilogue
 
@@ -193,7 +250,70 @@ __device__ __forceinline__ float apply_act(float y, int act)
     return y;
 }
 
-// ------------------------------------------------------------ the kernel
+// Per-kernel constants of the epilogue.
+struct EpiCtx {
+    bool dq;
+    float dqs;
+    const float* T;     // requantisation thresholds (shared memory)
+    Thr7 t7;
+    bool b4;
+};
+
+__device__ __forceinline__ EpiCtx make_epi_ctx(const EpiParams& ep, const float* T)
+{
+    EpiCtx c;
+    c.dq = ep.alpha_a_dev && ep.alpha_b_dev;
+    c.dqs = c.dq ? __fmul_rn(__ldg(ep.alpha_a_dev), __ldg(ep.alpha_b_dev)) * ep.dq_pow2 : 1.0f;
+    c.T = T;
+    c.b4 = ep.out.b == 4;
+#pragma unroll
+    for (int i = 0; i < 7; i++) c.t7.t[i] = (ep.codes_out && c.b4) ? T[i] : 0.0f;
+    return c;
+}
+
+// One output element: affine, residual, activation, optional stores, code.
+__device__ __forceinline__ uint32_t epi_element(const EpiParams& ep, const EpiCtx& cx, float af, int64_t m, int64_t n,
+                                                int64_t N)
+{
+    if (ep.acc_out) ep.acc_out[m * N + n] = __float2int_rn(af);
+    float sc = ep.scale ? __ldg(ep.scale + n) : ep.scale0;
+    if (cx.dq) sc = __fmul_rn(sc, cx.dqs);
+    const float bi = ep.bias ? __ldg(ep.bias + n) : ep.bias0;
+    float y = __fmaf_rn(sc, af, bi);
+    if (ep.residual) {
+        const int rcpw = 32 / ep.res_b;
+        const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >> (ep.res_b * (int)(n % rcpw))) &
+                            ((1u << ep.res_b) - 1u);
+        y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+    }
+    y = apply_act(y, ep.act);
+    if (ep.y_out) ep.y_out[m * N + n] = y;
+    if (!ep.codes_out) return 0u;
+    return cx.b4 ? project_by_thr7(y, cx.t7, ep.out) : project_by_table(y, cx.T, ep.out);
+}
+
+// Wait on an mbarrier phase with a wall-clock bound and an abort flag
+// raised by another role of the CTA.
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* err)
+{
+    const uint32_t a = smem_u32(bar);
+    if (mbar_try_wait(a, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try_wait(a, parity)) return true;
+        if ((it & 255u) == 0u) {
+            if (*err) return false;
+            if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// ------------------------------------------------- streamed-B kernel
 
 template <class SrcA, class SrcB>
 __global__ void __launch_bounds__(kGemmThreads, 1)
@@ -201,7 +321,6 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
                    float acc_scale, EpiParams ep)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    // 1024-byte aligned base for the swizzled stages.
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int a_bytes = kBM * kBK;
     const int b_bytes = BN * kBK;
@@ -209,6 +328,7 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
     uint64_t* mma_bar = reinterpret_cast<uint64_t*>(smem + kStages * stage_bytes);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_bar + kStages);
     volatile int* err_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    float* thr = reinterpret_cast<float*>(tmem_slot + 4);
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
@@ -226,6 +346,10 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
         tmem_alloc(tmem_slot, tmem_cols);
         tc_fence_before();
     }
+    if (ep.codes_out) {
+        const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
+        build_thresholds(thr, ep.out, alpha_out, warp, lane, 0, kGemmThreads / 32);
+    }
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_d = *tmem_slot;
@@ -233,7 +357,6 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
     const int64_t nkb = (K + kBK - 1) / kBK;
     const uint32_t idesc = idesc_e4m3_f32(BN);
 
-    // Each thread owns fixed rows of the A and B tiles across all K-blocks.
     constexpr int kAUnits = kBM * (kBK / 16) / kGemmThreads;   // 4
     typename SrcA::Row arow[kAUnits];
 #pragma unroll
@@ -253,14 +376,11 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
         for (int i = 0; i < kAUnits; i++) {
             const int u = tid + i * kGemmThreads;
             const int r = u >> 3, g = u & 7;
-            const uint4 v = decode_unit(srcA, arow[i], kbase + g * 16, K, fa);
-            *reinterpret_cast<uint4*>(sa + r * 128 + ((g ^ (r & 7)) << 4)) = v;
+            *reinterpret_cast<uint4*>(sa + swz(r, g)) = decode_unit(srcA, arow[i], kbase + g * 16, K, fa);
         }
         for (int u = tid; u < BN * 8; u += kGemmThreads) {
             const int r = u >> 3, g = u & 7;
-            const typename SrcB::Row brow = srcB.row(n0 + r);
-            const uint4 v = decode_unit(srcB, brow, kbase + g * 16, K, fb);
-            *reinterpret_cast<uint4*>(sb + r * 128 + ((g ^ (r & 7)) << 4)) = v;
+            *reinterpret_cast<uint4*>(sb + swz(r, g)) = decode_unit(srcB, srcB.row(n0 + r), kbase + g * 16, K, fb);
         }
         fence_proxy_async_smem();
         __syncthreads();
@@ -286,18 +406,13 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
     if (failed && tid == 0) record_status(ep.status, ESB_ERR_TIMEOUT);
 
     if (!failed) {
-        // ---------------------------------------------------- epilogue
         const int quarter = warp & 3;              // TMEM lanes 32*quarter .. +31
         const int half = warp >> 2;                // column chunks of this warp
         const int row = quarter * 32 + lane;
         const int64_t m = m0 + row;
         const bool mrow = m < M;
-        float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
-        const bool dq = ep.alpha_a_dev && ep.alpha_b_dev;
-        const float dqs = dq ? __fmul_rn(__ldg(ep.alpha_a_dev), __ldg(ep.alpha_b_dev)) * ep.dq_pow2 : 1.0f;
+        const EpiCtx cx = make_epi_ctx(ep, thr);
         uint8_t* stage_codes = smem;               // 128 x BN bytes, stages are free now
-        const int rcpw = ep.residual ? 32 / ep.res_b : 1;
-        const uint32_t rmask = ep.residual ? (1u << ep.res_b) - 1u : 0u;
         for (int c16 = half; c16 < BN / 16; c16 += 2) {
             uint32_t r[16];
             if (nkb > 0) {
@@ -311,21 +426,7 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
                 const int col = c16 * 16 + j;
                 const int64_t n = n0 + col;
                 uint32_t code = ep.out.zero_code;
-                if (mrow && n < N) {
-                    const float af = __uint_as_float(r[j]) * acc_scale;   // exact integer
-                    if (ep.acc_out) ep.acc_out[m * N + n] = __float2int_rn(af);
-                    float sc = ep.scale ? __ldg(ep.scale + n) : ep.scale0;
-                    if (dq) sc = __fmul_rn(sc, dqs);
-                    const float bi = ep.bias ? __ldg(ep.bias + n) : ep.bias0;
-                    float y = __fmaf_rn(sc, af, bi);
-                    if (ep.residual) {
-                        const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >> (ep.res_b * (int)(n % rcpw))) & rmask;
-                        y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
-                    }
-                    y = apply_act(y, ep.act);
-                    if (ep.y_out) ep.y_out[m * N + n] = y;
-                    if (ep.codes_out) code = project_code(y, alpha_out, ep.out);
-                }
+                if (mrow && n < N) code = epi_element(ep, cx, __uint_as_float(r[j]) * acc_scale, m, n, N);
                 if (ep.codes_out) stage_codes[row * BN + col] = (uint8_t)code;
             }
         }
@@ -354,6 +455,407 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
     }
 }
 
+// ----------------------------------------- resident-B persistent kernel
+
+constexpr int kWsEpiWarps = 8;                 // warps 0-7: epilogue (lanes 32*(w&3).., column half w>>2)
+constexpr int kWsMmaWarp = 8;                  // warp 8: TMEM allocation and MMA issue
+constexpr int kWsProdWarp0 = 9;                // warps 9-15: A producers, one stage at a time each
+constexpr int kWsProdWarps = 7;
+constexpr int kWsThreads = (kWsProdWarp0 + kWsProdWarps) * 32;   // 512: 4 warps per SM sub-partition
+constexpr int kWsMaxStages = 8;
+
+struct WsLayout {
+    int nkb;          // K-blocks
+    int BN;
+    int stages;
+    int b_bytes;      // resident B: nkb * BN * 128
+    int smem_bytes;   // total dynamic shared memory incl. alignment slack
+};
+
+__host__ inline WsLayout ws_layout(int64_t K, int BN, int max_smem)
+{
+    WsLayout L;
+    L.nkb = (int)((K + kBK - 1) / kBK);
+    L.BN = BN;
+    L.b_bytes = L.nkb * BN * kBK;
+    const int fixed = 1024 + L.b_bytes + 4 * 128 + 512;      // slack, B, thresholds, barriers
+    int st = (max_smem - fixed) / (kBM * kBK);
+    if (st > kWsMaxStages) st = kWsMaxStages;
+    L.stages = st;
+    L.smem_bytes = fixed + st * kBM * kBK;
+    return L;
+}
+
+// Byte masks of the decoded lo/hi words of one b = 4 word when only its
+// first v codes (0..8) are inside K.
+__device__ __forceinline__ void tail_masks(int v, uint32_t& mlo, uint32_t& mhi)
+{
+    const int nlo = (v + 1) >> 1, nhi = v >> 1;       // lo holds codes 0,2,4,6; hi 1,3,5,7
+    mlo = nlo >= 4 ? 0xffffffffu : ((1u << (8 * nlo)) - 1u);
+    mhi = nhi >= 4 ? 0xffffffffu : ((1u << (8 * nhi)) - 1u);
+}
+
+// Decode one 128-code K-block slice (16 words, four 16-byte pieces) of a
+// b = 4 row and store its 8 units to a swizzled stage row.  The loads of
+// all four pieces are issued before any decode.
+// Pieces outside the operand (rows past M or N, out-of-image taps, words
+// past K) are filled with the zero code -- the all-zero bit pattern is not
+// zero in this format (it is the value 1).
+template <class Src>
+__device__ __forceinline__ void load_row_b4(const Src& src, const typename Src::Row& row,
+                                            const typename Src::Cursor (&cur)[4], int64_t kw0, int64_t K,
+                                            uint32_t zero_word, uint4 (&v)[4])
+{
+#pragma unroll
+    for (int pc = 0; pc < 4; pc++) {
+        const int64_t kk0 = (kw0 + 4 * pc) * 8;       // first code of the piece
+        const uint32_t* p = (kk0 < K) ? src.at(row, cur[pc]) : nullptr;
+        v[pc] = p ? __ldg(reinterpret_cast<const uint4*>(p)) : make_uint4(zero_word, zero_word, zero_word, zero_word);
+    }
+}
+
+__device__ __forceinline__ void store_row_b4(uint8_t* stage, int r, const uint4 (&v)[4], int64_t kw0, int64_t K,
+                                             const OpFmt& f)
+{
+    const bool tail = (kw0 + 16) * 8 > K;             // only the last K-block can reach past K
+#pragma unroll
+    for (int pc = 0; pc < 4; pc++) {
+        const uint32_t w[4] = {v[pc].x, v[pc].y, v[pc].z, v[pc].w};
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+            uint32_t o0, o1, o2, o3;
+            decode_word_b4(w[2 * h], f.k, f.ew, o0, o1);
+            decode_word_b4(w[2 * h + 1], f.k, f.ew, o2, o3);
+            const int64_t wi = kw0 + 4 * pc + 2 * h;  // word index of w[2h]
+            if (tail && (wi + 2) * 8 > K) {           // K tail: zero the codes past K
+                uint32_t ml, mh;
+                int va = (int)(K - wi * 8);
+                va = va < 0 ? 0 : (va > 8 ? 8 : va);
+                tail_masks(va, ml, mh);
+                o0 &= ml; o1 &= mh;
+                int vb = (int)(K - (wi + 1) * 8);
+                vb = vb < 0 ? 0 : (vb > 8 ? 8 : vb);
+                tail_masks(vb, ml, mh);
+                o2 &= ml; o3 &= mh;
+            }
+            *reinterpret_cast<uint4*>(stage + swz(r, 2 * pc + h)) = make_uint4(o0, o1, o2, o3);
+        }
+    }
+}
+
+// Stage fill for formats other than b = 4 (general decode, out of line to
+// keep the hot b = 4 loop small).
+template <class Src>
+__device__ __noinline__ void fill_stage_any(const Src& src, const typename Src::Row (&rows)[4], uint8_t* st, int lane,
+                                            int64_t k0, int64_t K, const OpFmt f)
+{
+#pragma unroll 1
+    for (int q = 0; q < 4; q++)
+#pragma unroll 1
+        for (int g = 0; g < 8; g++)
+            *reinterpret_cast<uint4*>(st + swz(lane + 32 * q, g)) = decode_unit_any(src, rows[q], k0 + g * 16, K, f);
+}
+
+// Epilogue of one 16-column chunk for outputs other than b = 4 codes
+// (general packing), out of line.
+__device__ __noinline__ void epi_chunk_any(const EpiParams& ep, const EpiCtx& cx, const uint32_t (&r)[16], float acc_scale,
+                                           int64_t m, bool mrow, int64_t n_first, int64_t N, uint32_t& word, int& slot,
+                                           int64_t& wcol)
+{
+    const int cpw = ep.out_cpw;
+#pragma unroll 1
+    for (int j = 0; j < 16; j++) {
+        const int64_t n = n_first + j;
+        uint32_t code = ep.out.zero_code;
+        if (mrow && n < N) code = epi_element(ep, cx, __uint_as_float(r[j]) * acc_scale, m, n, N);
+        word |= code << (ep.out.b * slot);
+        if (++slot == cpw) {
+            if (ep.codes_out && mrow && wcol < ep.ldo) ep.codes_out[m * ep.ldo + wcol] = word;
+            word = 0;
+            slot = 0;
+            wcol++;
+        }
+    }
+}
+
+template <class SrcA>
+__global__ void __launch_bounds__(kWsThreads, 1)
+esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpFmt fa, OpFmt fb, int BN, int nkb,
+                   int stages, int n_tiles, int64_t m_tiles, float acc_scale, EpiParams ep)
+{
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sB = smem;                                        // nkb blocks of BN x 128 bytes
+    uint8_t* sA = sB + nkb * BN * kBK;                         // stages x 16 KiB
+    float* thr = reinterpret_cast<float*>(sA + stages * kBM * kBK);
+    uint64_t* full = reinterpret_cast<uint64_t*>(thr + 128);
+    uint64_t* empty = full + kWsMaxStages;
+    uint64_t* tfull = empty + kWsMaxStages;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* err = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int n_tile = (int)(blockIdx.x % n_tiles);
+    const int64_t cta_in_n = blockIdx.x / n_tiles;
+    const int64_t ctas_per_n = gridDim.x / n_tiles;
+    const int64_t n0 = (int64_t)n_tile * BN;
+    const int64_t my_tiles = (m_tiles > cta_in_n) ? (m_tiles - cta_in_n + ctas_per_n - 1) / ctas_per_n : 0;
+    uint32_t tmem_cols = 32;
+    while ((int)tmem_cols < 2 * BN) tmem_cols <<= 1;
+    // Epilogue column split: both halves of BN must be whole 16-column chunks
+    // and whole output words; otherwise warps 0-3 take every column.
+    const int half_cols = BN / 2;
+    const bool split = (half_cols % 16 == 0) && (half_cols % ep.out_cpw == 0);
+    const int epi_warps = split ? 8 : 4;
+
+    if (tid == 0) {
+        for (int s = 0; s < stages; s++) {
+            mbar_init(&full[s], 1);                   // the producer warp that filled the stage
+            mbar_init(&empty[s], 1);                  // the MMA commit that drained it
+        }
+        for (int a = 0; a < 2; a++) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], epi_warps);
+        }
+        mbar_init(drain, 1);
+        *err = 0;
+        fence_mbar_init();
+    }
+    if (warp == kWsMmaWarp) {
+        tmem_alloc(tmem_slot, tmem_cols);
+        tc_fence_before();
+    }
+    // Resident B: this CTA's N-tile, every K-block, decoded once.
+    if (fb.b == 4) {
+        const RowsSrc::Row dummy{nullptr};
+        (void)dummy;
+        for (int pr = tid; pr < nkb * BN; pr += kWsThreads) {
+            const int kb = pr / BN, r = pr - kb * BN;
+            const RowsSrc::Row row = srcB.row(n0 + r);
+            const int64_t kw0 = (int64_t)kb * 16;
+            RowsSrc::Cursor cur[4];
+#pragma unroll
+            for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
+            uint4 v[4];
+            load_row_b4(srcB, row, cur, kw0, K, fmt_zero_code(4, fb.k) * 0x11111111u, v);
+            store_row_b4(sB + kb * BN * kBK, r, v, kw0, K, fb);
+        }
+    } else {
+        for (int u = tid; u < nkb * BN * 8; u += kWsThreads) {
+            const int kb = u / (BN * 8);
+            const int rem = u - kb * BN * 8;
+            const int r = rem >> 3, g = rem & 7;
+            *reinterpret_cast<uint4*>(sB + kb * BN * kBK + swz(r, g)) =
+                decode_unit_any(srcB, srcB.row(n0 + r), (int64_t)kb * kBK + g * 16, K, fb);
+        }
+    }
+    fence_proxy_async_smem();
+    if (ep.codes_out) {
+        const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
+        build_thresholds(thr, ep.out, alpha_out, warp, lane, 0, kWsThreads / 32);
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp >= kWsProdWarp0) {
+        // ---------------------------------------------- A producers
+        // Warp p fills the stages of iterations p, p + 7, ... of this CTA's
+        // (tile, K-block) sequence, so up to 7 K-blocks are loading at once.
+        // Lane l owns rows l, l + 32, l + 64, l + 96 of the tile.
+        // At most `stages` producers are active: a producer then never waits
+        // on a stage more than one phase ahead of the MMA's progress, which
+        // is all the parity of an mbarrier can tell apart.
+        const int p = warp - kWsProdWarp0;
+        const int nprod = stages < kWsProdWarps ? stages : kWsProdWarps;
+        const int64_t total_it = (p < nprod) ? my_tiles * nkb : 0;
+        const uint32_t zwa = fmt_zero_code(4, fa.k) * 0x11111111u;
+        int64_t cur_tile = -1;
+        typename SrcA::Row rows[4];
+        for (int64_t it = p; it < total_it && !*err; it += nprod) {
+            const int64_t ti = it / nkb;
+            const int kb = (int)(it - ti * nkb);
+            if (ti != cur_tile) {
+                cur_tile = ti;
+                const int64_t m0 = (cta_in_n + ti * ctas_per_n) * kBM;
+#pragma unroll
+                for (int q = 0; q < 4; q++) rows[q] = srcA.row(m0 + lane + 32 * q);
+            }
+            const int s = (int)(it % stages);
+            const uint32_t ph = (uint32_t)((it / stages) & 1);
+            if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
+            uint8_t* st = sA + s * kBM * kBK;
+            if (fa.b == 4) {
+                const int64_t kw0 = (int64_t)kb * 16;
+                typename SrcA::Cursor cur[4];
+#pragma unroll
+                for (int pc = 0; pc < 4; pc++) cur[pc] = srcA.cursor(kw0 + 4 * pc);
+                uint4 v[4][4];
+#pragma unroll
+                for (int q = 0; q < 4; q++) load_row_b4(srcA, rows[q], cur, kw0, K, zwa, v[q]);
+#pragma unroll
+                for (int q = 0; q < 4; q++) store_row_b4(st, lane + 32 * q, v[q], kw0, K, fa);
+            } else {
+                fill_stage_any(srcA, rows, st, lane, (int64_t)kb * kBK, K, fa);
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&full[s]);
+        }
+    } else if (warp == kWsMmaWarp) {
+        // ---------------------------------------------- MMA issue
+        if (lane == 0) {
+            const uint32_t idesc = idesc_e4m3_f32(BN);
+            const uint32_t b_base = smem_u32(sB), a_base = smem_u32(sA);
+            int64_t it = 0;
+            for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
+                const int a = (int)(ti & 1);
+                if (!wait_or_abort(&tempty[a], (uint32_t)((ti >> 1) & 1) ^ 1u, err)) { *err = 1; break; }
+                tc_fence_after();
+                const uint32_t d = tmem_base + (uint32_t)(a * BN);
+                for (int kb = 0; kb < nkb; kb++, it++) {
+                    const int s = (int)(it % stages);
+                    if (!wait_or_abort(&full[s], (uint32_t)((it / stages) & 1), err)) { *err = 1; break; }
+                    tc_fence_after();
+                    const uint32_t a0 = a_base + (uint32_t)(s * kBM * kBK);
+                    const uint32_t b0 = b_base + (uint32_t)(kb * BN * kBK);
+#pragma unroll
+                    for (int j = 0; j < kBK / 32; j++)
+                        mma_f8f6f4(d, smem_desc_sw128(a0 + j * 32), smem_desc_sw128(b0 + j * 32), idesc,
+                                   (kb > 0 || j > 0) ? 1u : 0u);
+                    mma_commit(&empty[s]);
+                }
+                if (*err) break;
+                mma_commit(&tfull[a]);
+            }
+            // Every MMA this thread issued has completed before TMEM is freed
+            // (also on the abort path).
+            mma_commit(drain);
+            volatile int no_abort = 0;
+            if (!wait_or_abort(drain, 0u, &no_abort)) *err = 1;
+        }
+    } else if (warp < epi_warps) {
+        // ---------------------------------------------- epilogue
+        const int quarter = warp & 3;
+        const int row = quarter * 32 + lane;          // TMEM lane = tile row
+        const int c_lo = split ? (warp >> 2) * half_cols : 0;
+        const int c_hi = split ? c_lo + half_cols : BN;
+        const EpiCtx cx = make_epi_ctx(ep, thr);
+        const int cpw = ep.out_cpw;
+        const bool swar = ep.codes_out && ep.out.b == 4;
+        const float sc_fixed = ep.scale ? 0.0f : (cx.dq ? __fmul_rn(ep.scale0, cx.dqs) : ep.scale0);
+        const float sc_lean = sc_fixed * acc_scale;
+        const bool out_signed = ep.out.is_signed != 0;
+        // the lean path needs every column of the chunk inside N and a finite folded scale
+        const bool lean_ok = swar && !ep.scale && !ep.bias && !ep.residual && !ep.acc_out && !ep.y_out &&
+                             isfinite(sc_lean) && (sc_lean != 0.0f || sc_fixed == 0.0f);
+        for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
+            const int a = (int)(ti & 1);
+            if (!wait_or_abort(&tfull[a], (uint32_t)((ti >> 1) & 1), err)) { *err = 1; break; }
+            tc_fence_after();
+            const int64_t m = (cta_in_n + ti * ctas_per_n) * kBM + row;
+            const bool mrow = m < M;
+            const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(a * BN);
+            uint32_t word = 0;
+            int slot = 0;
+            int64_t wcol = (n0 + c_lo) / cpw;
+            for (int c = c_lo; c < c_hi; c += 16) {
+                uint32_t r[16];
+                tmem_ld16(taddr + (uint32_t)c, r);
+                const bool lean = lean_ok && (n0 + c + 16 <= N);
+                if (c + 16 >= c_hi) {                 // every column of this warp is in registers
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&tempty[a]);
+                }
+                if (lean) {
+                    // 4-bit output codes only, scalar scale/bias, no residual:
+                    // y = fma(scale * 2^(kA+kB+12), raw, bias) equals
+                    // fma(scale, acc, bias) exactly (power-of-two scaling),
+                    // then the bucket of y among the 7 thresholds, eight codes
+                    // per word at once.
+                    uint32_t wds[2];
+#pragma unroll
+                    for (int h = 0; h < 2; h++) {
+                        uint32_t J = 0u, S = 0u;
+#pragma unroll
+                        for (int j = 0; j < 8; j++) {
+                            float y = __fmaf_rn(sc_lean, __uint_as_float(r[8 * h + j]), ep.bias0);
+                            y = apply_act(y, ep.act);
+                            const float a = out_signed ? fabsf(y) : y;
+                            const bool b2 = a >= cx.t7.t[3];
+                            const bool b1 = a >= (b2 ? cx.t7.t[5] : cx.t7.t[1]);
+                            const bool b0 = a >= (b2 ? (b1 ? cx.t7.t[6] : cx.t7.t[4]) : (b1 ? cx.t7.t[2] : cx.t7.t[0]));
+                            J |= ((b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u)) << (4 * j);
+                            if (out_signed) S |= (__float_as_uint(y) >> 31) << (4 * j + 3);
+                        }
+                        wds[h] = codes8_b4(J, S, ep.out.k);
+                    }
+                    const int64_t w0 = (n0 + c) >> 3;
+                    if (mrow) {
+                        if (w0 + 1 < ep.ldo) {
+                            *reinterpret_cast<uint2*>(ep.codes_out + m * ep.ldo + w0) = make_uint2(wds[0], wds[1]);
+                        } else if (w0 < ep.ldo) {
+                            ep.codes_out[m * ep.ldo + w0] = wds[0];
+                        }
+                    }
+                } else if (swar) {
+                    // 4-bit output codes with per-channel parameters, residual or extra outputs
+                    uint32_t wds[2];
+#pragma unroll
+                    for (int h = 0; h < 2; h++) {
+                        uint32_t J = 0u, S = 0u;
+#pragma unroll 1
+                        for (int j = 0; j < 8; j++) {
+                            const int64_t n = n0 + c + 8 * h + j;
+                            const float af = __uint_as_float(r[8 * h + j]) * acc_scale;
+                            if (mrow && n < N) {
+                                if (ep.acc_out) ep.acc_out[m * N + n] = __float2int_rn(af);
+                                float sc = sc_fixed;
+                                if (ep.scale) { sc = __ldg(ep.scale + n); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
+                                const float bi = ep.bias ? __ldg(ep.bias + n) : ep.bias0;
+                                float y = __fmaf_rn(sc, af, bi);
+                                if (ep.residual) {
+                                    const int rcpw = 32 / ep.res_b;
+                                    const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >>
+                                                         (ep.res_b * (int)(n % rcpw))) & ((1u << ep.res_b) - 1u);
+                                    y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+                                }
+                                y = apply_act(y, ep.act);
+                                if (ep.y_out) ep.y_out[m * N + n] = y;
+                                const uint32_t u = __float_as_uint(y);
+                                J |= bucket7(ep.out.is_signed ? fabsf(y) : y, cx.t7) << (4 * j);
+                                S |= ((u >> 31) & (uint32_t)ep.out.is_signed) << (4 * j + 3);
+                            }
+                        }
+                        wds[h] = codes8_b4(J, S, ep.out.k);
+                    }
+                    const int64_t w0 = (n0 + c) >> 3;
+                    if (mrow) {
+                        if (w0 + 1 < ep.ldo) {
+                            *reinterpret_cast<uint2*>(ep.codes_out + m * ep.ldo + w0) = make_uint2(wds[0], wds[1]);
+                        } else if (w0 < ep.ldo) {
+                            ep.codes_out[m * ep.ldo + w0] = wds[0];
+                        }
+                    }
+                } else {
+                    epi_chunk_any(ep, cx, r, acc_scale, m, mrow, n0 + c, N, word, slot, wcol);
+                }
+            }
+        }
+    }
+
+    __syncthreads();
+    if (*err && tid == 0) record_status(ep.status, ESB_ERR_TIMEOUT);
+    if (warp == kWsMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, tmem_cols);
+    }
+}
+
 // ------------------------------------------------------------ host side
 
 static int pick_bn(int64_t N, int out_cpw)
@@ -375,7 +877,21 @@ static int pick_bn(int64_t N, int out_cpw)
 
 static size_t gemm_smem_bytes(int BN)
 {
-    return 1024 + (size_t)kStages * (kBM * kBK + (size_t)BN * kBK) + kStages * 8 + 16;
+    return 1024 + (size_t)kStages * (kBM * kBK + (size_t)BN * kBK) + kStages * 8 + 16 + 512;
+}
+
+static int max_dyn_smem()
+{
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 227 * 1024;
+    if (!cache[dev]) {
+        int v = 0;
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess || v <= 0)
+            v = 227 * 1024;
+        cache[dev] = v;
+    }
+    return cache[dev];
 }
 
 template <class SrcA, class SrcB>
@@ -394,6 +910,35 @@ static cudaError_t launch_tc(const SrcA& a, const SrcB& b, int64_t M, int64_t N,
     dim3 grid((unsigned)((M + kBM - 1) / kBM), (unsigned)((N + BN - 1) / BN));
     esb_gemm_tc_kernel<SrcA, SrcB><<<grid, kGemmThreads, smem, st>>>(a, b, M, N, K, fa, fb, BN, acc_scale, ep);
     return cudaGetLastError();
+}
+
+// Resident-B launch when B's N-tile fits in shared memory with at least
+// three A stages; returns false (nothing launched) otherwise.
+template <class SrcA>
+static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int64_t K, const OpFmt& fa,
+                      const OpFmt& fb, int BN, const EpiParams& ep, cudaStream_t st, cudaError_t* err)
+{
+    const int maxs = max_dyn_smem();
+    const WsLayout L = ws_layout(K, BN, maxs);
+    if (L.stages < 3) return false;
+    static bool configured = false;
+    if (!configured) {
+        *err = cudaFuncSetAttribute(esb_gemm_ws_kernel<SrcA>, cudaFuncAttributeMaxDynamicSharedMemorySize, maxs);
+        if (*err != cudaSuccess) return true;
+        configured = true;
+    }
+    const int n_tiles = (int)((N + BN - 1) / BN);
+    const int64_t m_tiles = (M + kBM - 1) / kBM;
+    int64_t per_n = device_sm_count() / n_tiles;
+    if (per_n < 1) per_n = 1;
+    if (per_n > m_tiles) per_n = m_tiles;
+    const int64_t grid = per_n * n_tiles;
+    const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
+    esb_gemm_ws_kernel<SrcA><<<(unsigned)grid, kWsThreads, L.smem_bytes, st>>>(a, b, M, N, K, fa, fb, BN, L.nkb,
+                                                                               L.stages, n_tiles, m_tiles, acc_scale,
+                                                                               ep);
+    *err = cudaGetLastError();
+    return true;
 }
 
 static EpiParams make_epi(const GemmOutputs& o)
@@ -436,7 +981,12 @@ cudaError_t launch_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int6
     const int BN = pick_bn(N, ep.out_cpw);
     RowsSrc a{A, lda, M};
     RowsSrc b{B, ldb, N};
-    return launch_tc(a, b, M, N, K, make_opfmt(ba, ka), make_opfmt(bb, kb), BN, ep, st);
+    const OpFmt fa = make_opfmt(ba, ka), fb = make_opfmt(bb, kb);
+    if (K > 0) {
+        cudaError_t e = cudaSuccess;
+        if (launch_ws(a, b, M, N, K, fa, fb, BN, ep, st, &e)) return e;
+    }
+    return launch_tc(a, b, M, N, K, fa, fb, BN, ep, st);
 }
 
 cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
@@ -449,10 +999,13 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
     const int64_t K = (int64_t)d.r * d.s * ldx * (32 / bx);
     const int BN = pick_bn(N, ep.out_cpw);
     ConvSrc a;
-    a.X = X; a.ldx = ldx; a.rows = M; a.H = d.h; a.W = d.w; a.P = P; a.Q = Q; a.S = d.s;
+    a.X = X; a.ldx = (int)ldx; a.rows = (int)M; a.H = d.h; a.W = d.w; a.P = P; a.Q = Q; a.S = d.s;
     a.stride = d.stride; a.pad = d.pad;
     RowsSrc b{W, (int64_t)d.r * d.s * ldw, N};
-    return launch_tc(a, b, M, N, K, make_opfmt(bx, kx), make_opfmt(bw, kw), BN, ep, st);
+    const OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
+    cudaError_t e = cudaSuccess;
+    if (K > 0 && launch_ws(a, b, M, N, K, fa, fb, BN, ep, st, &e)) return e;
+    return launch_tc(a, b, M, N, K, fa, fb, BN, ep, st);
 }
 
 bool gemm_pick_ok(int64_t N, int out_b) { return pick_bn(N, 32 / out_b) != 0; }

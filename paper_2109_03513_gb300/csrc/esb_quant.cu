@@ -14,6 +14,10 @@ namespace esb {
 
 // ----------------------------------------------------------- projection
 
+// Both projection kernels first build the threshold table of the current
+// alpha (all warps, see build_thresholds), then project every element with
+// it: no division per element.
+
 // Fast path: one thread turns 4*cpw consecutive floats of a row into 4
 // code words (one 16-byte store); cpw float4 loads in flight per thread,
 // streaming cache hints since every byte is touched once.
@@ -24,7 +28,17 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
                    uint32_t* __restrict__ codes, int64_t ldc)
 {
     constexpr int CPW = 32 / B;
+    constexpr int L = 1 << (B - 1);
+    __shared__ float T[L];
     const float a = alpha_dev ? __ldg(alpha_dev) : alpha;
+    build_thresholds(T, p, a, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
+    __syncthreads();
+    Thr7 t7;
+    if (B == 4) {
+#pragma unroll
+        for (int i = 0; i < 7; i++) t7.t[i] = T[i];
+    }
+    auto proj = [&](float v) -> uint32_t { return B == 4 ? project_by_thr7(v, t7, p) : project_by_table(v, T, p); };
     const int64_t upr = ldc >> 2;                 // 4-word units per row
     const int64_t total = rows * upr;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -41,12 +55,28 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
                 const float4 t = __ldcs(reinterpret_cast<const float4*>(xr) + i);
                 v[4 * i + 0] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
             }
+            if (B == 4) {
+                // buckets of |x| (x for the unsigned set: negatives land in bucket 0)
 #pragma unroll
-            for (int w = 0; w < 4; w++) {
-                uint32_t word = 0;
+                for (int w = 0; w < 4; w++) {
+                    uint32_t J = 0u, S = 0u;
 #pragma unroll
-                for (int j = 0; j < CPW; j++) word |= project_code(v[w * CPW + j], a, p) << (B * j);
-                out[w] = word;
+                    for (int j = 0; j < 8; j++) {
+                        const float xv = v[w * 8 + j];
+                        const uint32_t u = __float_as_uint(xv);
+                        J |= bucket7(p.is_signed ? fabsf(xv) : xv, t7) << (4 * j);
+                        S |= ((u >> 31) & (uint32_t)p.is_signed) << (4 * j + 3);
+                    }
+                    out[w] = codes8_b4(J, S, p.k);
+                }
+            } else {
+#pragma unroll
+                for (int w = 0; w < 4; w++) {
+                    uint32_t word = 0;
+#pragma unroll
+                    for (int j = 0; j < CPW; j++) word |= proj(v[w * CPW + j]) << (B * j);
+                    out[w] = word;
+                }
             }
         } else {
 #pragma unroll
@@ -55,7 +85,7 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
 #pragma unroll
                 for (int j = 0; j < CPW; j++) {
                     const int64_t c = c0 + w * CPW + j;
-                    const uint32_t code = (c < cols) ? project_code(__ldcs(xr + w * CPW + j), a, p) : p.zero_code;
+                    const uint32_t code = (c < cols) ? proj(__ldcs(xr + w * CPW + j)) : p.zero_code;
                     word |= code << (B * j);
                 }
                 out[w] = word;
@@ -73,7 +103,11 @@ project_any_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
                    uint32_t* __restrict__ codes, int64_t ldc)
 {
     constexpr int CPW = 32 / B;
+    constexpr int L = 1 << (B - 1);
+    __shared__ float T[L];
     const float a = alpha_dev ? __ldg(alpha_dev) : alpha;
+    build_thresholds(T, p, a, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
+    __syncthreads();
     const int64_t total = rows * ldc;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < total; u += stride) {
@@ -83,7 +117,7 @@ project_any_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
 #pragma unroll
         for (int j = 0; j < CPW; j++) {
             const int64_t c = w * CPW + j;
-            const uint32_t code = (c < cols) ? project_code(x[r * ldx + c], a, p) : p.zero_code;
+            const uint32_t code = (c < cols) ? project_by_table(x[r * ldx + c], T, p) : p.zero_code;
             word |= code << (B * j);
         }
         codes[u] = word;  // row-major: r * ldc + w == u
@@ -166,26 +200,67 @@ cudaError_t launch_dequant(const uint32_t* codes, int64_t rows, int64_t cols, in
 
 // ------------------------------------------------------- DDA calibration
 
-// Pass 1.  The data is cut into chunks of 32 values.  Each thread keeps, in
-// fp64, the sums over its full chunks of a_c, a_c^2 and M2_c, where a_c is
-// the fp32 chunk mean and M2_c = sum (x - a_c)^2 in fp32 (both from the
-// chunk held in registers); partial chunks carry their count as a weight.
-// The law of total variance then gives mean and sigma from these sums with
-// no catastrophic cancellation inside a chunk.  Per-block partials go to
-// the workspace in a fixed layout; the finalize kernel adds them in a fixed
-// order, so the result does not depend on scheduling.
+// Pass 1.  The data is cut into chunks of 32 values.  For each chunk the
+// thread computes, from registers, the fp32 chunk mean a_c and
+// M2_c = sum (x - a_c)^2; the law of total variance then gives the
+// statistics from the sums of a_c, a_c^2 and M2_c with no cancellation
+// inside a chunk.  Those sums are carried as unevaluated pairs of fp32
+// numbers (hi + lo, error-free transformations: ~48 significant bits), so
+// the reduction runs on the fp32 pipes -- GB300 has very little fp64
+// throughput -- and fp64 is used only for the final few operations.
+// Per-block partials go to the workspace in a fixed layout; the finalize
+// kernel adds them in a fixed order, so results do not depend on
+// scheduling.
 constexpr int kCalThreads = 256;
 constexpr int kCalChunk = 32;
 constexpr int kCalMaxBlocks = 1024;
+constexpr int kCalChunksPerThread = 1;
 
 struct CalPartial {
     double n, s1, s2, s3;   // sum n_c, sum n_c a_c, sum n_c a_c^2, sum M2_c
 };
 
-__device__ __forceinline__ void cal_warp_sum(double& v)
+// (hi, lo) += x, Knuth's TwoSum with the rounding error kept in lo.
+__device__ __forceinline__ void df_add(float& hi, float& lo, float x)
 {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const float s = hi + x;
+    const float bp = s - hi;
+    const float e = (hi - (s - bp)) + (x - bp);
+    hi = s;
+    lo += e;
+}
+
+// (hi, lo) += (h2, l2)
+__device__ __forceinline__ void df_add2(float& hi, float& lo, float h2, float l2)
+{
+    df_add(hi, lo, h2);
+    lo += l2;
+}
+
+// (hi, lo) += a * a, exactly split by an fma.
+__device__ __forceinline__ void df_add_sq(float& hi, float& lo, float a)
+{
+    const float p = a * a;
+    const float pe = fmaf(a, a, -p);
+    df_add(hi, lo, p);
+    lo += pe;
+}
+
+struct CalAcc {
+    unsigned long long n;
+    float s1h, s1l, s2h, s2l, s3h, s3l;
+};
+
+__device__ __forceinline__ void cal_shfl(CalAcc& A, int o)
+{
+    const unsigned long long n = __shfl_xor_sync(0xffffffffu, A.n, o);
+    const float a1 = __shfl_xor_sync(0xffffffffu, A.s1h, o), b1 = __shfl_xor_sync(0xffffffffu, A.s1l, o);
+    const float a2 = __shfl_xor_sync(0xffffffffu, A.s2h, o), b2 = __shfl_xor_sync(0xffffffffu, A.s2l, o);
+    const float a3 = __shfl_xor_sync(0xffffffffu, A.s3h, o), b3 = __shfl_xor_sync(0xffffffffu, A.s3l, o);
+    A.n += n;
+    df_add2(A.s1h, A.s1l, a1, b1);
+    df_add2(A.s2h, A.s2l, a2, b2);
+    df_add2(A.s3h, A.s3l, a3, b3);
 }
 
 __global__ void __launch_bounds__(kCalThreads)
@@ -194,7 +269,11 @@ calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalParti
     const int64_t nfull = n / kCalChunk;
     const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
-    double s1 = 0.0, s2 = 0.0, s3 = 0.0, cnt = 0.0;
+    CalAcc A{0ull, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+    float sa_h = 0.0f, sa_l = 0.0f;   // sum of a over full chunks (weight 32 applied at the end)
+    float sq_h = 0.0f, sq_l = 0.0f;   // sum of a^2 over full chunks
+    unsigned long long cnt = 0ull;
+#pragma unroll 2
     for (int64_t c = tid; c < nfull; c += nthreads) {
         float v[kCalChunk];
         const float* xc = x + c * kCalChunk;
@@ -215,14 +294,15 @@ calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalParti
         float m2 = 0.0f;
 #pragma unroll
         for (int i = 0; i < kCalChunk; i++) { const float d = v[i] - a; m2 = fmaf(d, d, m2); }
-        s1 += (double)a;
-        s2 = fma((double)a, (double)a, s2);
-        s3 += (double)m2;
-        cnt += 1.0;
+        df_add(sa_h, sa_l, a);
+        df_add_sq(sq_h, sq_l, a);
+        df_add(A.s3h, A.s3l, m2);
+        cnt += 1ull;
     }
-    double n_all = cnt * kCalChunk;
-    s1 *= kCalChunk;
-    s2 *= kCalChunk;
+    // full chunks carry weight 32: scaling a pair by a power of two is exact
+    A.n = cnt * (unsigned long long)kCalChunk;
+    A.s1h = sa_h * kCalChunk; A.s1l = sa_l * kCalChunk;
+    A.s2h = sq_h * kCalChunk; A.s2l = sq_l * kCalChunk;
     // The ragged tail (< 32 values) is one weighted chunk, owned by thread 0.
     const int64_t tail0 = nfull * kCalChunk;
     if (tid == 0 && tail0 < n) {
@@ -232,22 +312,32 @@ calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalParti
         const float a = s / (float)nt;
         float m2 = 0.0f;
         for (int i = 0; i < nt; i++) { const float d = x[tail0 + i] - a; m2 = fmaf(d, d, m2); }
-        n_all += nt;
-        s1 += (double)nt * (double)a;
-        s2 += (double)nt * (double)a * (double)a;
-        s3 += (double)m2;
+        // n_t * a and n_t * a^2 as exact pairs: split the products with fmas
+        const float w = (float)nt;
+        const float p1 = w * a, e1 = fmaf(w, a, -p1);
+        df_add(A.s1h, A.s1l, p1); A.s1l += e1;
+        const float q = a * a, qe = fmaf(a, a, -q);          // a^2 = q + qe exactly
+        const float p2 = w * q, e2 = fmaf(w, q, -p2);         // w q = p2 + e2 exactly
+        df_add(A.s2h, A.s2l, p2); A.s2l += e2 + w * qe;
+        df_add(A.s3h, A.s3l, m2);
+        A.n += (unsigned long long)nt;
     }
-    cal_warp_sum(n_all); cal_warp_sum(s1); cal_warp_sum(s2); cal_warp_sum(s3);
-    __shared__ CalPartial sh[kCalThreads / 32];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cal_shfl(A, o);
+    __shared__ CalAcc sh[kCalThreads / 32];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) sh[warp] = CalPartial{n_all, s1, s2, s3};
+    if (lane == 0) sh[warp] = A;
     __syncthreads();
     if (threadIdx.x == 0) {
-        CalPartial t{0.0, 0.0, 0.0, 0.0};
-        for (int w = 0; w < kCalThreads / 32; w++) {
-            t.n += sh[w].n; t.s1 += sh[w].s1; t.s2 += sh[w].s2; t.s3 += sh[w].s3;
+        CalAcc t = sh[0];
+        for (int w = 1; w < kCalThreads / 32; w++) {
+            t.n += sh[w].n;
+            df_add2(t.s1h, t.s1l, sh[w].s1h, sh[w].s1l);
+            df_add2(t.s2h, t.s2l, sh[w].s2h, sh[w].s2l);
+            df_add2(t.s3h, t.s3l, sh[w].s3h, sh[w].s3l);
         }
-        part[blockIdx.x] = t;
+        part[blockIdx.x] = CalPartial{(double)t.n, (double)t.s1h + (double)t.s1l, (double)t.s2h + (double)t.s2l,
+                                      (double)t.s3h + (double)t.s3l};
     }
 }
 
@@ -292,7 +382,7 @@ calibrate_finalize_kernel(const CalPartial* __restrict__ part, int nblocks, doub
 
 int calibrate_blocks(int64_t n)
 {
-    const int64_t per_block = (int64_t)kCalThreads * kCalChunk;
+    const int64_t per_block = (int64_t)kCalThreads * kCalChunk * kCalChunksPerThread;
     int64_t g = (n + per_block - 1) / per_block;
     if (g > kCalMaxBlocks) g = kCalMaxBlocks;
     if (g < 1) g = 1;
