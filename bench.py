@@ -8,7 +8,8 @@ tensors: X ~ |N(0,1)|, W ~ N(0, sqrt(2/576)) (He init).
 
 One step = one pass of the hot path over one batch, captured as a CUDA
 graph:
-  esb_calibrate_dda(X) -> esb_project(X)     (DDA alpha of the batch, codes)
+  esb_project_dda(X)   (DDA statistics and alpha of the batch, then its
+                        projection to packed codes, in one launch)
   esb_conv2d_nhwc(Xc, Wc) with the fused epilogue (dequant scale from the two
   device alphas, ReLU, ESB requantisation with the layer's calibrated
   output alpha) -> next layer's packed codes.
@@ -190,8 +191,8 @@ def run_gpu(args):
     def calls_for(i):
         Xi, Xci = Xs[i], Xcs[i]
         return [
-            ("calibrate_x", lambda: esb.esb_calibrate_dda(Xi, fu, alpha_out=ax, workspace=wsx, stream=stream), 2),
-            ("project_x", lambda: esb.esb_project(Xi, fu, alpha=ax, codes=Xci, stream=stream), 1),
+            ("project_dda_x", lambda: esb.esb_project_dda(Xi, fu, alpha_out=ax, workspace=wsx, codes=Xci,
+                                                          stream=stream), 1),
             ("conv", lambda: esb.esb_conv2d_nhwc(Xci, fu, Wc, fs, N_, H_, W_, C_, CO_, R_, S_, STRIDE, PAD, ep=ep,
                                                  want_acc=False, out_codes=Yc, stream=stream), 1),
         ]
@@ -291,7 +292,8 @@ def run_gpu(args):
     hbm, bf16, src = _peaks()
     n_x, n_w = X.numel(), Wt.numel()
     algo = {  # algorithmic bytes / ops per launch
-        "calibrate_x": ("hbm", 4.0 * n_x), "project_x": ("hbm", 4.0 * n_x + 4.0 * Xc.numel()),
+        # one HBM read of x (the second pass reads it from L2) + the code words written
+        "project_dda_x": ("hbm", 4.0 * n_x + 4.0 * Xc.numel()),
         "conv": ("tensor", float(OPS)),
     }
     dominant = max(per, key=per.get)

@@ -144,7 +144,8 @@ esb_status esb_alpha_star(int32_t b, int32_t k, double* alpha_star, double* dda)
 
 /* ----------------------------------------------------------- calibrate */
 
-/* Bytes of device workspace esb_calibrate_dda needs for n values. */
+/* Bytes of device workspace esb_calibrate_dda needs for n values on the
+ * current device (the reduction grid follows its SM count). */
 size_t esb_calibrate_dda_workspace_bytes(int64_t n);
 
 /* DDA calibration of Sec. III-D ("Normalization" and "Resolving extremum"):
@@ -159,7 +160,8 @@ size_t esb_calibrate_dda_workspace_bytes(int64_t n);
  *              8-byte aligned, contents ignored and overwritten
  *   alpha_out  [device] 1 float written by the kernel (no host sync)
  *   stats_out  [device] 3 doubles {mean, sigma or rms, n}, or NULL
- * The reduction order is fixed, so results are bit-reproducible.
+ * One memset of the workspace's ticket word and one kernel launch; the
+ * reduction order is fixed, so results are bit-reproducible on a device.
  * Errors: INVALID_ARG, UNSUPPORTED (bad format), ALIGN (workspace), CUDA. */
 esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
                              void* workspace, size_t workspace_bytes,
@@ -189,7 +191,8 @@ esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
  * nothing has to be cleared): calls whose kernels overlap on the GPU (on
  * different streams without ordering) race on it and must be serialised.
  * Errors: INVALID_ARG, UNSUPPORTED, RANGE (scratch need above the array's
- * size; the reduction uses at most 1024 blocks, so no n exceeds it), CUDA. */
+ * size; the reduction uses at most 1023 blocks plus one ticket record, so
+ * no n exceeds it), CUDA. */
 esb_status esb_calibrate_dda_noalloc(const float* x, int64_t n, esb_format f,
                                      float* alpha_out, double* stats_out, void* stream);
 
@@ -213,6 +216,23 @@ esb_status esb_calibrate_dda_noalloc(const float* x, int64_t n, esb_format f,
 esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx,
                        float alpha, const float* alpha_dev, esb_format f, int32_t rounding,
                        uint32_t* codes, int64_t ldc, void* stream);
+
+/* DDA-calibrated projection of one tensor: the statistics and alpha of
+ * esb_calibrate_dda (Sec. III-D), then esb_project of the same tensor with
+ * that alpha (Eq. cheap_projection), in one cooperative launch that keeps
+ * the tensor in L2 between the two passes.
+ *   x          [device] rows x cols floats, contiguous (row stride cols)
+ *   workspace  [device] >= esb_calibrate_dda_workspace_bytes(rows * cols),
+ *              8-byte aligned, contents ignored
+ *   alpha_out  [device] 1 float written with the alpha used
+ *   stats_out  [device] 3 doubles {mean, sigma or rms, n}, or NULL
+ *   codes      [device] rows x ldc words, as esb_project
+ * 16-byte-aligned x and codes with cols and ldc multiples of 4 take the
+ * fused path; other layouts run the two steps as separate launches.
+ * Errors: INVALID_ARG, UNSUPPORTED, ALIGN (workspace), CUDA. */
+esb_status esb_project_dda(const float* x, int64_t rows, int64_t cols, esb_format f, int32_t rounding,
+                           void* workspace, size_t workspace_bytes, float* alpha_out, double* stats_out,
+                           uint32_t* codes, int64_t ldc, void* stream);
 
 /* Dequantisation (test aid and fp32 export): y = fl32(alpha * q), q the
  * value of each code in units of alpha (Sec. IV-A, Eq. q).

@@ -183,6 +183,23 @@ esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx, 
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 
+esb_status esb_project_dda(const float* x, int64_t rows, int64_t cols, esb_format f, int32_t rounding,
+                           void* workspace, size_t workspace_bytes, float* alpha_out, double* stats_out,
+                           uint32_t* codes, int64_t ldc, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (rows <= 0 || cols <= 0 || ldc < words_for(cols, f.b)) return ESB_ERR_INVALID_ARG;
+    if (rounding != ESB_ROUND_HALF_AWAY && rounding != ESB_ROUND_HALF_EVEN) return ESB_ERR_INVALID_ARG;
+    if (!x || !workspace || !alpha_out || !codes) return ESB_ERR_INVALID_ARG;
+    if (workspace_bytes < calibrate_workspace_bytes(rows * cols)) return ESB_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 7u) != 0) return ESB_ERR_ALIGN;
+    double as = 0.0;
+    alpha_star_cached(f.b, f.k, &as, nullptr);
+    cudaError_t e = launch_calibrate_project(x, rows, cols, f.b, f.k, f.is_signed, rounding, as, workspace, alpha_out,
+                                             stats_out, codes, ldc, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
 esb_status esb_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_t ldc, float alpha,
                        const float* alpha_dev, esb_format f, float* y, int64_t ldy, void* stream)
 {

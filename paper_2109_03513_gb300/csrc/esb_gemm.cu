@@ -544,26 +544,36 @@ __device__ __forceinline__ void store_row_b4(uint8_t* stage, int r, const uint4 
 }
 
 // Stage fill for formats other than b = 4 (general decode, out of line to
-// keep the hot b = 4 loop small).
+// keep the hot b = 4 loop small; takes scalars only, so no register array of
+// the caller has to live in memory).
 template <class Src>
-__device__ __noinline__ void fill_stage_any(const Src& src, const typename Src::Row (&rows)[4], uint8_t* st, int lane,
-                                            int64_t k0, int64_t K, const OpFmt f)
+__device__ __noinline__ void fill_stage_any(const Src src, int64_t m0, uint8_t* st, int lane, int64_t k0, int64_t K,
+                                            const OpFmt f)
 {
 #pragma unroll 1
-    for (int q = 0; q < 4; q++)
+    for (int q = 0; q < 4; q++) {
+        const typename Src::Row row = src.row(m0 + lane + 32 * q);
 #pragma unroll 1
         for (int g = 0; g < 8; g++)
-            *reinterpret_cast<uint4*>(st + swz(lane + 32 * q, g)) = decode_unit_any(src, rows[q], k0 + g * 16, K, f);
+            *reinterpret_cast<uint4*>(st + swz(lane + 32 * q, g)) = decode_unit_any(src, row, k0 + g * 16, K, f);
+    }
 }
 
-// Epilogue of one 16-column chunk for outputs other than b = 4 codes
-// (general packing), out of line.
-__device__ __noinline__ void epi_chunk_any(const EpiParams& ep, const EpiCtx& cx, const uint32_t (&r)[16], float acc_scale,
-                                           int64_t m, bool mrow, int64_t n_first, int64_t N, uint32_t& word, int& slot,
-                                           int64_t& wcol)
+// Epilogue of one 16-column chunk for outputs other than the lean 4-bit
+// path (general packing), out of line; reads its own TMEM chunk.
+__device__ __noinline__ void epi_chunk_any(const EpiParams* __restrict__ sep, const EpiCtx* __restrict__ scx,
+                                           uint32_t taddr, float acc_scale, int64_t m, bool mrow, int64_t n_first,
+                                           int64_t N, uint32_t* word_slot_w)
 {
+    const EpiParams& ep = *sep;
+    const EpiCtx cx = *scx;
+    uint32_t r[16];
+    tmem_ld16(taddr, r);
     const int cpw = ep.out_cpw;
-#pragma unroll 1
+    uint32_t word = word_slot_w[0];
+    int slot = (int)word_slot_w[1];
+    int64_t wcol = (int64_t)word_slot_w[2] | ((int64_t)word_slot_w[3] << 32);
+#pragma unroll
     for (int j = 0; j < 16; j++) {
         const int64_t n = n_first + j;
         uint32_t code = ep.out.zero_code;
@@ -576,6 +586,10 @@ __device__ __noinline__ void epi_chunk_any(const EpiParams& ep, const EpiCtx& cx
             wcol++;
         }
     }
+    word_slot_w[0] = word;
+    word_slot_w[1] = (uint32_t)slot;
+    word_slot_w[2] = (uint32_t)(wcol & 0xffffffff);
+    word_slot_w[3] = (uint32_t)(wcol >> 32);
 }
 
 template <class SrcA>
@@ -624,42 +638,49 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
         *err = 0;
         fence_mbar_init();
     }
-    if (warp == kWsMmaWarp) {
-        tmem_alloc(tmem_slot, tmem_cols);
-        tc_fence_before();
-    }
-    // Resident B: this CTA's N-tile, every K-block, decoded once.
-    if (fb.b == 4) {
-        const RowsSrc::Row dummy{nullptr};
-        (void)dummy;
-        for (int pr = tid; pr < nkb * BN; pr += kWsThreads) {
-            const int kb = pr / BN, r = pr - kb * BN;
-            const RowsSrc::Row row = srcB.row(n0 + r);
-            const int64_t kw0 = (int64_t)kb * 16;
-            RowsSrc::Cursor cur[4];
+    __syncthreads();                                  // barriers initialised
+
+    // Producers start loading A at once; meanwhile the MMA and epilogue
+    // warps decode the resident B, allocate TMEM and build the
+    // requantisation thresholds, then meet on named barrier 1.
+    constexpr int kSetupThreads = kWsProdWarp0 * 32;  // warps 0..8
+    uint32_t tmem_base = 0;
+    if (warp < kWsProdWarp0) {
+        if (warp == kWsMmaWarp) {
+            tmem_alloc(tmem_slot, tmem_cols);
+            tc_fence_before();
+        }
+        // Resident B: this CTA's N-tile, every K-block, decoded once.
+        if (fb.b == 4) {
+            for (int pr = tid; pr < nkb * BN; pr += kSetupThreads) {
+                const int kb = pr / BN, r = pr - kb * BN;
+                const RowsSrc::Row row = srcB.row(n0 + r);
+                const int64_t kw0 = (int64_t)kb * 16;
+                RowsSrc::Cursor cur[4];
 #pragma unroll
-            for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
-            uint4 v[4];
-            load_row_b4(srcB, row, cur, kw0, K, fmt_zero_code(4, fb.k) * 0x11111111u, v);
-            store_row_b4(sB + kb * BN * kBK, r, v, kw0, K, fb);
+                for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
+                uint4 v[4];
+                load_row_b4(srcB, row, cur, kw0, K, fmt_zero_code(4, fb.k) * 0x11111111u, v);
+                store_row_b4(sB + kb * BN * kBK, r, v, kw0, K, fb);
+            }
+        } else {
+            for (int u = tid; u < nkb * BN * 8; u += kSetupThreads) {
+                const int kb = u / (BN * 8);
+                const int rem = u - kb * BN * 8;
+                const int r = rem >> 3, g = rem & 7;
+                *reinterpret_cast<uint4*>(sB + kb * BN * kBK + swz(r, g)) =
+                    decode_unit_any(srcB, srcB.row(n0 + r), (int64_t)kb * kBK + g * 16, K, fb);
+            }
         }
-    } else {
-        for (int u = tid; u < nkb * BN * 8; u += kWsThreads) {
-            const int kb = u / (BN * 8);
-            const int rem = u - kb * BN * 8;
-            const int r = rem >> 3, g = rem & 7;
-            *reinterpret_cast<uint4*>(sB + kb * BN * kBK + swz(r, g)) =
-                decode_unit_any(srcB, srcB.row(n0 + r), (int64_t)kb * kBK + g * 16, K, fb);
+        fence_proxy_async_smem();
+        if (ep.codes_out) {
+            const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
+            build_thresholds(thr, ep.out, alpha_out, warp, lane, 0, kWsProdWarp0);
         }
+        asm volatile("bar.sync 1, %0;" ::"n"(kSetupThreads) : "memory");
+        tc_fence_after();
+        tmem_base = *tmem_slot;
     }
-    fence_proxy_async_smem();
-    if (ep.codes_out) {
-        const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
-        build_thresholds(thr, ep.out, alpha_out, warp, lane, 0, kWsThreads / 32);
-    }
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem_base = *tmem_slot;
 
     if (warp >= kWsProdWarp0) {
         // ---------------------------------------------- A producers
@@ -699,7 +720,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
 #pragma unroll
                 for (int q = 0; q < 4; q++) store_row_b4(st, lane + 32 * q, v[q], kw0, K, fa);
             } else {
-                fill_stage_any(srcA, rows, st, lane, (int64_t)kb * kBK, K, fa);
+                fill_stage_any(srcA, (cta_in_n + ti * ctas_per_n) * kBM, st, lane, (int64_t)kb * kBK, K, fa);
             }
             fence_proxy_async_smem();
             __syncwarp();
@@ -741,11 +762,17 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
         // ---------------------------------------------- epilogue
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;          // TMEM lane = tile row
+        __shared__ EpiParams sh_ep;                   // copies for the out-of-line general path
+        __shared__ EpiCtx sh_cx;
         const int c_lo = split ? (warp >> 2) * half_cols : 0;
         const int c_hi = split ? c_lo + half_cols : BN;
         const EpiCtx cx = make_epi_ctx(ep, thr);
+        if (warp == 0 && lane == 0) { sh_ep = ep; sh_cx = cx; }
+        asm volatile("bar.sync 2, %0;" ::"r"(epi_warps * 32) : "memory");   // exactly the epilogue warps in use
         const int cpw = ep.out_cpw;
         const bool swar = ep.codes_out && ep.out.b == 4;
+        const float T0 = cx.t7.t[0], T1 = cx.t7.t[1], T2 = cx.t7.t[2], T3 = cx.t7.t[3], T4 = cx.t7.t[4],
+                    T5 = cx.t7.t[5], T6 = cx.t7.t[6];
         const float sc_fixed = ep.scale ? 0.0f : (cx.dq ? __fmul_rn(ep.scale0, cx.dqs) : ep.scale0);
         const float sc_lean = sc_fixed * acc_scale;
         const bool out_signed = ep.out.is_signed != 0;
@@ -759,10 +786,18 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
             const int64_t m = (cta_in_n + ti * ctas_per_n) * kBM + row;
             const bool mrow = m < M;
             const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(a * BN);
-            uint32_t word = 0;
-            int slot = 0;
-            int64_t wcol = (n0 + c_lo) / cpw;
+            uint32_t wsw[4] = {0u, 0u, (uint32_t)(((n0 + c_lo) / cpw) & 0xffffffff),
+                               (uint32_t)(((n0 + c_lo) / cpw) >> 32)};   // general path: word, slot, column
             for (int c = c_lo; c < c_hi; c += 16) {
+                if (!swar) {
+                    epi_chunk_any(&sh_ep, &sh_cx, taddr + (uint32_t)c, acc_scale, m, mrow, n0 + c, N, wsw);
+                    if (c + 16 >= c_hi) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&tempty[a]);
+                    }
+                    continue;
+                }
                 uint32_t r[16];
                 tmem_ld16(taddr + (uint32_t)c, r);
                 const bool lean = lean_ok && (n0 + c + 16 <= N);
@@ -786,9 +821,9 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
                             float y = __fmaf_rn(sc_lean, __uint_as_float(r[8 * h + j]), ep.bias0);
                             y = apply_act(y, ep.act);
                             const float a = out_signed ? fabsf(y) : y;
-                            const bool b2 = a >= cx.t7.t[3];
-                            const bool b1 = a >= (b2 ? cx.t7.t[5] : cx.t7.t[1]);
-                            const bool b0 = a >= (b2 ? (b1 ? cx.t7.t[6] : cx.t7.t[4]) : (b1 ? cx.t7.t[2] : cx.t7.t[0]));
+                            const bool b2 = a >= T3;
+                            const bool b1 = a >= (b2 ? T5 : T1);
+                            const bool b0 = a >= (b2 ? (b1 ? T6 : T4) : (b1 ? T2 : T0));
                             J |= ((b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u)) << (4 * j);
                             if (out_signed) S |= (__float_as_uint(y) >> 31) << (4 * j + 3);
                         }
@@ -841,8 +876,6 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
                             ep.codes_out[m * ep.ldo + w0] = wds[0];
                         }
                     }
-                } else {
-                    epi_chunk_any(ep, cx, r, acc_scale, m, mrow, n0 + c, N, word, slot, wcol);
                 }
             }
         }
@@ -918,7 +951,15 @@ template <class SrcA>
 static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int64_t K, const OpFmt& fa,
                       const OpFmt& fb, int BN, const EpiParams& ep, cudaStream_t st, cudaError_t* err)
 {
-    const int maxs = max_dyn_smem();
+    // dynamic shared memory = the opt-in maximum minus the kernel's static shared memory
+    static int static_smem = -1;
+    if (static_smem < 0) {
+        cudaFuncAttributes fa_attr;
+        *err = cudaFuncGetAttributes(&fa_attr, esb_gemm_ws_kernel<SrcA>);
+        if (*err != cudaSuccess) return true;
+        static_smem = (int)fa_attr.sharedSizeBytes;
+    }
+    const int maxs = max_dyn_smem() - static_smem;
     const WsLayout L = ws_layout(K, BN, maxs);
     if (L.stages < 3) return false;
     static bool configured = false;

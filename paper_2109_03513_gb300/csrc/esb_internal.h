@@ -26,6 +26,10 @@ size_t calibrate_workspace_bytes(int64_t n);
 cudaError_t launch_calibrate(const float* x, int64_t n, int is_signed, double alpha_star, void* workspace,
                              float* alpha_out, double* stats_out, cudaStream_t st);
 
+cudaError_t launch_calibrate_project(const float* x, int64_t rows, int64_t cols, int b, int k, int is_signed,
+                                     int rounding, double alpha_star, void* workspace, float* alpha_out,
+                                     double* stats_out, uint32_t* codes, int64_t ldc, cudaStream_t st);
+
 size_t calibrate_noalloc_capacity();
 cudaError_t launch_calibrate_noalloc(const float* x, int64_t n, int is_signed, double alpha_star, float* alpha_out,
                                      double* stats_out, cudaStream_t st);

@@ -14,6 +14,49 @@ namespace esb {
 
 // ----------------------------------------------------------- projection
 
+// Projection of a flat (row stride = cols, code rows without padding)
+// tensor to 4-bit codes in warp tiles of 1024 values: coalesced 16-byte
+// loads, lane l projects values 4(32j + l) .. +3 to 16 bits of codes, and
+// lane pairs (l, l + 1) join their halves into one word with a shuffle.
+template <bool SIGNED, bool STREAM>
+__device__ __forceinline__ void project_flat_b4(const float* __restrict__ x, int64_t n, const Thr7& t7, int k,
+                                                uint32_t* __restrict__ codes)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t tiles = (n + 1023) / 1024;
+#pragma unroll 1
+    for (int64_t t = gwarp; t < tiles; t += nwarps) {
+        const int64_t e0 = t * 1024;
+        const bool whole = e0 + 1024 <= n;
+        const float4* xt = reinterpret_cast<const float4*>(x + e0) + lane;
+        float4 q[8];
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            const int64_t e = e0 + 4 * (32 * j + lane);
+            if (whole || e < n) q[j] = STREAM ? __ldcs(xt + 32 * j) : __ldg(xt + 32 * j);
+            else q[j] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            const float xv[4] = {q[j].x, q[j].y, q[j].z, q[j].w};
+            uint32_t J = 0u, S = 0u;
+#pragma unroll
+            for (int i = 0; i < 4; i++) {
+                J |= bucket7(SIGNED ? fabsf(xv[i]) : xv[i], t7) << (4 * i);
+                if (SIGNED) S |= (__float_as_uint(xv[i]) >> 31) << (4 * i + 3);
+            }
+            const uint32_t h = codes8_b4(J, S, k) & 0xffffu;          // four codes: low 16 bits
+            const uint32_t other = __shfl_down_sync(0xffffffffu, h, 1);
+            if ((lane & 1) == 0) {
+                const int64_t wi = (e0 >> 3) + 16 * j + (lane >> 1);
+                if (whole || wi < (n >> 3)) codes[wi] = h | (other << 16);
+            }
+        }
+    }
+}
+
 // Both projection kernels first build the threshold table of the current
 // alpha (all warps, see build_thresholds), then project every element with
 // it: no division per element.
@@ -30,6 +73,35 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
     constexpr int CPW = 32 / B;
     constexpr int L = 1 << (B - 1);
     __shared__ float T[L];
+    const int64_t upr = ldc >> 2;                 // 4-word units per row
+    const int64_t total = rows * upr;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+
+    // The first unit's loads are issued before the threshold table is built,
+    // and every later unit's loads before the previous unit's store, so the
+    // table set-up and the stores overlap memory latency.
+    float v[4 * CPW];
+    int64_t r = 0, w4 = 0, c0 = 0;
+    bool full = false;
+    auto fetch = [&](int64_t uu) {
+        if (uu >= total) return;
+        r = (rows == 1) ? 0 : uu / upr;
+        w4 = uu - r * upr;
+        c0 = w4 * (4 * CPW);
+        full = c0 + 4 * CPW <= cols;
+        if (full) {
+            const float4* xr = reinterpret_cast<const float4*>(x + r * ldx + c0);
+#pragma unroll
+            for (int i = 0; i < CPW; i++) {
+                const float4 t = __ldcs(xr + i);
+                v[4 * i + 0] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
+            }
+        }
+    };
+    int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const bool flat = (ldx == cols) && (cols % 8 == 0) && (ldc * 8 == cols);
+    if (!(B == 4 && flat)) fetch(u);
+
     const float a = alpha_dev ? __ldg(alpha_dev) : alpha;
     build_thresholds(T, p, a, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
     __syncthreads();
@@ -38,23 +110,18 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
 #pragma unroll
         for (int i = 0; i < 7; i++) t7.t[i] = T[i];
     }
-    auto proj = [&](float v) -> uint32_t { return B == 4 ? project_by_thr7(v, t7, p) : project_by_table(v, T, p); };
-    const int64_t upr = ldc >> 2;                 // 4-word units per row
-    const int64_t total = rows * upr;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < total; u += stride) {
-        const int64_t r = (rows == 1) ? 0 : u / upr;
-        const int64_t w4 = u - r * upr;
-        const int64_t c0 = w4 * (4 * CPW);
-        const float* xr = x + r * ldx + c0;
+    auto proj = [&](float xv) -> uint32_t { return B == 4 ? project_by_thr7(xv, t7, p) : project_by_table(xv, T, p); };
+
+    if (B == 4 && flat) {                                 // flat codes: coalesced warp tiles
+        if (p.is_signed) project_flat_b4<true, true>(x, rows * cols, t7, p.k, codes);
+        else project_flat_b4<false, true>(x, rows * cols, t7, p.k, codes);
+        return;
+    }
+
+    for (; u < total; u += stride) {
         uint32_t out[4];
-        if (c0 + 4 * CPW <= cols) {
-            float v[4 * CPW];
-#pragma unroll
-            for (int i = 0; i < CPW; i++) {
-                const float4 t = __ldcs(reinterpret_cast<const float4*>(xr) + i);
-                v[4 * i + 0] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
-            }
+        const int64_t rr = r, ww4 = w4, cc0 = c0;
+        if (full) {
             if (B == 4) {
                 // buckets of |x| (x for the unsigned set: negatives land in bucket 0)
 #pragma unroll
@@ -63,9 +130,9 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
 #pragma unroll
                     for (int j = 0; j < 8; j++) {
                         const float xv = v[w * 8 + j];
-                        const uint32_t u = __float_as_uint(xv);
+                        const uint32_t uxv = __float_as_uint(xv);
                         J |= bucket7(p.is_signed ? fabsf(xv) : xv, t7) << (4 * j);
-                        S |= ((u >> 31) & (uint32_t)p.is_signed) << (4 * j + 3);
+                        S |= ((uxv >> 31) & (uint32_t)p.is_signed) << (4 * j + 3);
                     }
                     out[w] = codes8_b4(J, S, p.k);
                 }
@@ -79,19 +146,21 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
                 }
             }
         } else {
+            const float* xr = x + rr * ldx + cc0;
 #pragma unroll
             for (int w = 0; w < 4; w++) {
                 uint32_t word = 0;
 #pragma unroll
                 for (int j = 0; j < CPW; j++) {
-                    const int64_t c = c0 + w * CPW + j;
+                    const int64_t c = cc0 + w * CPW + j;
                     const uint32_t code = (c < cols) ? proj(__ldcs(xr + w * CPW + j)) : p.zero_code;
                     word |= code << (B * j);
                 }
                 out[w] = word;
             }
         }
-        __stcs(reinterpret_cast<uint4*>(codes + r * ldc + (w4 << 2)), make_uint4(out[0], out[1], out[2], out[3]));
+        fetch(u + stride);
+        __stcs(reinterpret_cast<uint4*>(codes + rr * ldc + (ww4 << 2)), make_uint4(out[0], out[1], out[2], out[3]));
     }
 }
 
@@ -213,7 +282,7 @@ cudaError_t launch_dequant(const uint32_t* codes, int64_t rows, int64_t cols, in
 // scheduling.
 constexpr int kCalThreads = 256;
 constexpr int kCalChunk = 32;
-constexpr int kCalMaxBlocks = 1024;
+constexpr int kCalMaxBlocks = 1023;   // + one 32-byte ticket record = 32 KiB of workspace
 constexpr int kCalChunksPerThread = 1;
 
 struct CalPartial {
@@ -263,109 +332,30 @@ __device__ __forceinline__ void cal_shfl(CalAcc& A, int o)
     df_add2(A.s3h, A.s3l, a3, b3);
 }
 
-__global__ void __launch_bounds__(kCalThreads)
-calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalPartial* __restrict__ part)
+// Sum of the block partials in a fixed order and the final statistics,
+// run by the last block of the pass (see calibrate_pass1_kernel).
+__device__ void calibrate_finalize_block(const CalPartial* part, int nblocks, double alpha_star, int is_signed,
+                                         float* alpha_out, double* stats_out)
 {
-    const int64_t nfull = n / kCalChunk;
-    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
-    CalAcc A{0ull, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
-    float sa_h = 0.0f, sa_l = 0.0f;   // sum of a over full chunks (weight 32 applied at the end)
-    float sq_h = 0.0f, sq_l = 0.0f;   // sum of a^2 over full chunks
-    unsigned long long cnt = 0ull;
-#pragma unroll 2
-    for (int64_t c = tid; c < nfull; c += nthreads) {
-        float v[kCalChunk];
-        const float* xc = x + c * kCalChunk;
-        if (vec) {
-#pragma unroll
-            for (int i = 0; i < kCalChunk / 4; i++) {
-                const float4 t = __ldcs(reinterpret_cast<const float4*>(xc) + i);
-                v[4 * i] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
-            }
-        } else {
-#pragma unroll
-            for (int i = 0; i < kCalChunk; i++) v[i] = __ldcs(xc + i);
-        }
-        float s = 0.0f;
-#pragma unroll
-        for (int i = 0; i < kCalChunk; i++) s += v[i];
-        const float a = s * (1.0f / kCalChunk);
-        float m2 = 0.0f;
-#pragma unroll
-        for (int i = 0; i < kCalChunk; i++) { const float d = v[i] - a; m2 = fmaf(d, d, m2); }
-        df_add(sa_h, sa_l, a);
-        df_add_sq(sq_h, sq_l, a);
-        df_add(A.s3h, A.s3l, m2);
-        cnt += 1ull;
-    }
-    // full chunks carry weight 32: scaling a pair by a power of two is exact
-    A.n = cnt * (unsigned long long)kCalChunk;
-    A.s1h = sa_h * kCalChunk; A.s1l = sa_l * kCalChunk;
-    A.s2h = sq_h * kCalChunk; A.s2l = sq_l * kCalChunk;
-    // The ragged tail (< 32 values) is one weighted chunk, owned by thread 0.
-    const int64_t tail0 = nfull * kCalChunk;
-    if (tid == 0 && tail0 < n) {
-        const int nt = (int)(n - tail0);
-        float s = 0.0f;
-        for (int i = 0; i < nt; i++) s += x[tail0 + i];
-        const float a = s / (float)nt;
-        float m2 = 0.0f;
-        for (int i = 0; i < nt; i++) { const float d = x[tail0 + i] - a; m2 = fmaf(d, d, m2); }
-        // n_t * a and n_t * a^2 as exact pairs: split the products with fmas
-        const float w = (float)nt;
-        const float p1 = w * a, e1 = fmaf(w, a, -p1);
-        df_add(A.s1h, A.s1l, p1); A.s1l += e1;
-        const float q = a * a, qe = fmaf(a, a, -q);          // a^2 = q + qe exactly
-        const float p2 = w * q, e2 = fmaf(w, q, -p2);         // w q = p2 + e2 exactly
-        df_add(A.s2h, A.s2l, p2); A.s2l += e2 + w * qe;
-        df_add(A.s3h, A.s3l, m2);
-        A.n += (unsigned long long)nt;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) cal_shfl(A, o);
-    __shared__ CalAcc sh[kCalThreads / 32];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) sh[warp] = A;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        CalAcc t = sh[0];
-        for (int w = 1; w < kCalThreads / 32; w++) {
-            t.n += sh[w].n;
-            df_add2(t.s1h, t.s1l, sh[w].s1h, sh[w].s1l);
-            df_add2(t.s2h, t.s2l, sh[w].s2h, sh[w].s2l);
-            df_add2(t.s3h, t.s3l, sh[w].s3h, sh[w].s3l);
-        }
-        part[blockIdx.x] = CalPartial{(double)t.n, (double)t.s1h + (double)t.s1l, (double)t.s2h + (double)t.s2l,
-                                      (double)t.s3h + (double)t.s3l};
-    }
-}
-
-// Pass 2 (one block): fixed-order sum of the block partials, then
-// mean = s1/n, M2 = s3 + (s2 - s1^2/n), sigma = sqrt(M2/n) (signed formats)
-// or rms = sqrt((s3 + s2)/n) (unsigned formats), alpha = fl32(alpha* (spread + 1e-7)).
-__global__ void __launch_bounds__(kCalThreads)
-calibrate_finalize_kernel(const CalPartial* __restrict__ part, int nblocks, double alpha_star, int is_signed,
-                          float* __restrict__ alpha_out, double* __restrict__ stats_out)
-{
-    __shared__ CalPartial sh[kCalThreads];
+    __shared__ CalPartial red[kCalThreads];
     CalPartial t{0.0, 0.0, 0.0, 0.0};
     for (int i = threadIdx.x; i < nblocks; i += kCalThreads) {
-        t.n += part[i].n; t.s1 += part[i].s1; t.s2 += part[i].s2; t.s3 += part[i].s3;
+        const double* q = reinterpret_cast<const double*>(part + i);   // written by other blocks: read from L2
+        t.n += __ldcg(q); t.s1 += __ldcg(q + 1); t.s2 += __ldcg(q + 2); t.s3 += __ldcg(q + 3);
     }
-    sh[threadIdx.x] = t;
+    red[threadIdx.x] = t;
     __syncthreads();
     for (int h = kCalThreads / 2; h > 0; h >>= 1) {
-        if (threadIdx.x < h) {
-            sh[threadIdx.x].n += sh[threadIdx.x + h].n;
-            sh[threadIdx.x].s1 += sh[threadIdx.x + h].s1;
-            sh[threadIdx.x].s2 += sh[threadIdx.x + h].s2;
-            sh[threadIdx.x].s3 += sh[threadIdx.x + h].s3;
+        if ((int)threadIdx.x < h) {
+            red[threadIdx.x].n += red[threadIdx.x + h].n;
+            red[threadIdx.x].s1 += red[threadIdx.x + h].s1;
+            red[threadIdx.x].s2 += red[threadIdx.x + h].s2;
+            red[threadIdx.x].s3 += red[threadIdx.x + h].s3;
         }
         __syncthreads();
     }
     if (threadIdx.x == 0) {
-        const CalPartial r = sh[0];
+        const CalPartial r = red[0];
         const double mean = r.s1 / r.n;
         double spread;
         if (is_signed) {
@@ -380,18 +370,268 @@ calibrate_finalize_kernel(const CalPartial* __restrict__ part, int nblocks, doub
     }
 }
 
+// One launch: every block writes its partial record; the block that takes
+// the last ticket (the ticket word is zeroed by a memset before the launch)
+// adds all records in index order and finalises alpha.
+// Adds one group of `cnt` values (cnt = 32: weight folded in at the end; any
+// other count: weighted exactly) to the accumulators.
+__device__ __forceinline__ void cal_group(const float* v, int cnt, float& sa_h, float& sa_l, float& sq_h, float& sq_l,
+                                          CalAcc& A, unsigned long long& full_groups)
+{
+    float s = 0.0f;
+    for (int i = 0; i < cnt; i++) s += v[i];
+    const float a = (cnt == kCalChunk) ? s * (1.0f / kCalChunk) : s / (float)cnt;
+    float m2 = 0.0f;
+    for (int i = 0; i < cnt; i++) { const float d = v[i] - a; m2 = fmaf(d, d, m2); }
+    if (cnt == kCalChunk) {
+        df_add(sa_h, sa_l, a);
+        df_add_sq(sq_h, sq_l, a);
+        full_groups += 1ull;
+    } else {
+        // n_c * a and n_c * a^2 as exact pairs: split the products with fmas
+        const float w = (float)cnt;
+        const float p1 = w * a, e1 = fmaf(w, a, -p1);
+        df_add(A.s1h, A.s1l, p1); A.s1l += e1;
+        const float q = a * a, qe = fmaf(a, a, -q);          // a^2 = q + qe exactly
+        const float p2 = w * q, e2 = fmaf(w, q, -p2);         // w q = p2 + e2 exactly
+        df_add(A.s2h, A.s2l, p2); A.s2l += e2 + w * qe;
+        A.n += (unsigned long long)cnt;
+    }
+    df_add(A.s3h, A.s3l, m2);
+}
+
+// Statistics of this block's share of x, reduced over the block; thread 0
+// returns the block's partial record.  The data is read in warp tiles of
+// 1024 values with coalesced 16-byte loads (lane l takes values
+// 4(32j + l) .. +3, j = 0..7, as its group of 32 -- any partition into groups
+// serves the law of total variance).  Values past the last full tile are
+// taken by warp 0 of block 0 in contiguous groups of at most 32.
+// `stream_loads` selects evict-first loads (data read once) or default loads
+// (data kept in L2 for a second pass).
+__device__ __forceinline__ CalPartial cal_block_partial(const float* __restrict__ x, int64_t n, int vec,
+                                                        bool stream_loads)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t tiles = vec ? n / 1024 : 0;
+    CalAcc A{0ull, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+    float sa_h = 0.0f, sa_l = 0.0f;   // sum of a over full groups (weight 32 applied at the end)
+    float sq_h = 0.0f, sq_l = 0.0f;   // sum of a^2 over full groups
+    unsigned long long full_groups = 0ull;
+#pragma unroll 1
+    for (int64_t t = gwarp; t < tiles; t += nwarps) {
+        const float4* xt = reinterpret_cast<const float4*>(x + t * 1024) + lane;
+        float v[kCalChunk];
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            const float4 q = stream_loads ? __ldcs(xt + 32 * j) : __ldg(xt + 32 * j);
+            v[4 * j] = q.x; v[4 * j + 1] = q.y; v[4 * j + 2] = q.z; v[4 * j + 3] = q.w;
+        }
+        cal_group(v, kCalChunk, sa_h, sa_l, sq_h, sq_l, A, full_groups);
+    }
+    const int64_t rem0 = tiles * 1024;
+    if (blockIdx.x == 0 && threadIdx.x < 32 && rem0 < n) {
+        // up to 32 contiguous groups of 32 per lane pass
+        for (int64_t g0 = rem0 + 32 * (int64_t)lane; g0 < n; g0 += 32 * 32) {
+            const int cnt = (int)((n - g0) < 32 ? (n - g0) : 32);
+            float v[kCalChunk];
+            for (int i = 0; i < cnt; i++) v[i] = x[g0 + i];
+            cal_group(v, cnt, sa_h, sa_l, sq_h, sq_l, A, full_groups);
+        }
+    }
+    // full groups carry weight 32: scaling a pair by a power of two is exact
+    A.n += full_groups * (unsigned long long)kCalChunk;
+    df_add2(A.s1h, A.s1l, sa_h * kCalChunk, sa_l * kCalChunk);
+    df_add2(A.s2h, A.s2l, sq_h * kCalChunk, sq_l * kCalChunk);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cal_shfl(A, o);
+    __shared__ CalAcc sh[kCalThreads / 32];
+    const int warp = threadIdx.x >> 5;
+    if (lane == 0) sh[warp] = A;
+    __syncthreads();
+    CalPartial out{0.0, 0.0, 0.0, 0.0};
+    if (threadIdx.x == 0) {
+        CalAcc t = sh[0];
+        for (int w = 1; w < kCalThreads / 32; w++) {
+            t.n += sh[w].n;
+            df_add2(t.s1h, t.s1l, sh[w].s1h, sh[w].s1l);
+            df_add2(t.s2h, t.s2l, sh[w].s2h, sh[w].s2l);
+            df_add2(t.s3h, t.s3l, sh[w].s3h, sh[w].s3l);
+        }
+        out = CalPartial{(double)t.n, (double)t.s1h + (double)t.s1l, (double)t.s2h + (double)t.s2l,
+                         (double)t.s3h + (double)t.s3l};
+    }
+    return out;
+}
+
+// Workspace head record: the ticket counter, the release flag of the fused
+// kernel's grid barrier, and the alpha it publishes.
+struct CalSync {
+    unsigned int ticket;
+    unsigned int flag;
+    float alpha;
+    unsigned int pad[5];
+};
+static_assert(sizeof(CalSync) == sizeof(CalPartial), "head record is one partial record wide");
+
+// One launch: every block writes its partial record; the block that takes
+// the last ticket (the ticket word is zeroed by a memset before the launch)
+// adds all records in index order and finalises alpha.
+__global__ void __launch_bounds__(kCalThreads)
+calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalPartial* __restrict__ part,
+                       CalSync* __restrict__ sync, double alpha_star, int is_signed,
+                       float* __restrict__ alpha_out, double* __restrict__ stats_out)
+{
+    const CalPartial mine = cal_block_partial(x, n, vec, true);
+    __shared__ bool is_last;
+    if (threadIdx.x == 0) {
+        part[blockIdx.x] = mine;
+        __threadfence();
+        is_last = atomicAdd(&sync->ticket, 1u) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (is_last) {
+        __threadfence();
+        calibrate_finalize_block(part, gridDim.x, alpha_star, is_signed, alpha_out, stats_out);
+    }
+}
+
+// ------------------------------------- DDA-calibrated projection, fused
+
+// Calibration and projection of the same tensor in one cooperative launch
+// (all blocks co-resident).  Phase 1 reduces the statistics with loads that
+// leave x in L2; the last block to arrive finalises alpha, publishes it and
+// raises the release flag, which every other block waits for (bounded).
+// Phase 2 projects x, now read from L2, with that alpha.
+template <int B>
+__global__ void __launch_bounds__(kCalThreads)
+calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, CalPartial* __restrict__ part,
+                         CalSync* __restrict__ sync, double alpha_star, ProjParams p, float* __restrict__ alpha_out,
+                         double* __restrict__ stats_out, uint32_t* __restrict__ codes, int64_t ldc,
+                         int* __restrict__ status)
+{
+    constexpr int CPW = 32 / B;
+    constexpr int L = 1 << (B - 1);
+    const int64_t n = rows * cols;
+    const CalPartial mine = cal_block_partial(x, n, 1, false);
+    __shared__ bool is_last;
+    __shared__ int timed_out;
+    __shared__ float T[L];
+    if (threadIdx.x == 0) {
+        part[blockIdx.x] = mine;
+        __threadfence();
+        is_last = atomicAdd(&sync->ticket, 1u) == gridDim.x - 1;
+        timed_out = 0;
+    }
+    __syncthreads();
+    if (is_last) {
+        __threadfence();
+        calibrate_finalize_block(part, gridDim.x, alpha_star, p.is_signed, &sync->alpha, stats_out);
+        if (threadIdx.x == 0) {
+            *alpha_out = sync->alpha;
+            __threadfence();
+            atomicExch(&sync->flag, 1u);
+        }
+    } else if (threadIdx.x == 0) {
+        const volatile unsigned int* f = &sync->flag;
+        const uint64_t t0 = globaltimer_ns();
+        uint32_t it = 0;
+        while (*f == 0u) {
+            if ((++it & 255u) == 0u && globaltimer_ns() - t0 > 2000000000ull) { timed_out = 1; break; }
+            __nanosleep(64);
+        }
+        __threadfence();
+    }
+    __syncthreads();
+    if (timed_out) {
+        if (threadIdx.x == 0) record_status(status, ESB_ERR_TIMEOUT);
+        return;
+    }
+    const float a = __ldcg(&sync->alpha);
+    build_thresholds(T, p, a, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
+    __syncthreads();
+    Thr7 t7;
+    if (B == 4) {
+#pragma unroll
+        for (int i = 0; i < 7; i++) t7.t[i] = T[i];
+        if (cols % 8 == 0 && ldc * 8 == cols) {         // flat codes: coalesced warp tiles
+            if (p.is_signed) project_flat_b4<true, true>(x, n, t7, p.k, codes);
+            else project_flat_b4<false, true>(x, n, t7, p.k, codes);
+            return;
+        }
+    }
+    const int64_t upr = ldc >> 2;
+    const int64_t total = rows * upr;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < total; u += stride) {
+        const int64_t r = (rows == 1) ? 0 : u / upr;
+        const int64_t w4 = u - r * upr;
+        const int64_t c0 = w4 * (4 * CPW);
+        const float* xr = x + r * cols + c0;
+        uint32_t out[4];
+        if (c0 + 4 * CPW <= cols) {
+            float v[4 * CPW];
+#pragma unroll
+            for (int i = 0; i < CPW; i++) {
+                const float4 t = __ldcs(reinterpret_cast<const float4*>(xr) + i);
+                v[4 * i + 0] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
+            }
+            if (B == 4) {
+#pragma unroll
+                for (int w = 0; w < 4; w++) {
+                    uint32_t J = 0u, S = 0u;
+#pragma unroll
+                    for (int j = 0; j < 8; j++) {
+                        const float xv = v[w * 8 + j];
+                        J |= bucket7(p.is_signed ? fabsf(xv) : xv, t7) << (4 * j);
+                        S |= ((__float_as_uint(xv) >> 31) & (uint32_t)p.is_signed) << (4 * j + 3);
+                    }
+                    out[w] = codes8_b4(J, S, p.k);
+                }
+            } else {
+#pragma unroll
+                for (int w = 0; w < 4; w++) {
+                    uint32_t word = 0;
+#pragma unroll
+                    for (int j = 0; j < CPW; j++) word |= project_by_table(v[w * CPW + j], T, p) << (B * j);
+                    out[w] = word;
+                }
+            }
+        } else {
+#pragma unroll
+            for (int w = 0; w < 4; w++) {
+                uint32_t word = 0;
+#pragma unroll
+                for (int j = 0; j < CPW; j++) {
+                    const int64_t c = c0 + w * CPW + j;
+                    const uint32_t code = (c < cols) ? project_by_table(__ldcs(xr + w * CPW + j), T, p) : p.zero_code;
+                    word |= code << (B * j);
+                }
+                out[w] = word;
+            }
+        }
+        __stcs(reinterpret_cast<uint4*>(codes + r * ldc + (w4 << 2)), make_uint4(out[0], out[1], out[2], out[3]));
+    }
+}
+
+// Grid: one chunk per thread up to one resident wave (4 blocks of 256
+// threads per SM at this kernel's register use), at most kCalMaxBlocks.
 int calibrate_blocks(int64_t n)
 {
     const int64_t per_block = (int64_t)kCalThreads * kCalChunk * kCalChunksPerThread;
     int64_t g = (n + per_block - 1) / per_block;
+    const int64_t wave = (int64_t)device_sm_count() * 4;
+    if (g > wave) g = wave;
     if (g > kCalMaxBlocks) g = kCalMaxBlocks;
     if (g < 1) g = 1;
     return (int)g;
 }
 
+// Workspace: [ticket record (32 B)][one CalPartial per block].
 size_t calibrate_workspace_bytes(int64_t n)
 {
-    return (size_t)calibrate_blocks(n) * sizeof(CalPartial);
+    return sizeof(CalPartial) + (size_t)calibrate_blocks(n) * sizeof(CalPartial);
 }
 
 cudaError_t launch_calibrate(const float* x, int64_t n, int is_signed, double alpha_star, void* workspace,
@@ -399,22 +639,77 @@ cudaError_t launch_calibrate(const float* x, int64_t n, int is_signed, double al
 {
     const int g = calibrate_blocks(n);
     const int vec = ((reinterpret_cast<uintptr_t>(x) & 15u) == 0) ? 1 : 0;
-    CalPartial* part = static_cast<CalPartial*>(workspace);
-    calibrate_pass1_kernel<<<g, kCalThreads, 0, st>>>(x, n, vec, part);
-    cudaError_t e = cudaGetLastError();
+    CalSync* sync = static_cast<CalSync*>(workspace);
+    CalPartial* part = static_cast<CalPartial*>(workspace) + 1;
+    cudaError_t e = cudaMemsetAsync(sync, 0, 2 * sizeof(unsigned int), st);
     if (e != cudaSuccess) return e;
-    calibrate_finalize_kernel<<<1, kCalThreads, 0, st>>>(part, g, alpha_star, is_signed, alpha_out, stats_out);
+    calibrate_pass1_kernel<<<g, kCalThreads, 0, st>>>(x, n, vec, part, sync, alpha_star, is_signed, alpha_out,
+                                                        stats_out);
     return cudaGetLastError();
+}
+
+template <int B>
+static cudaError_t launch_calibrate_project_b(const float* x, int64_t rows, int64_t cols, const ProjParams& p,
+                                              double alpha_star, void* workspace, float* alpha_out, double* stats_out,
+                                              uint32_t* codes, int64_t ldc, cudaStream_t st, bool* launched)
+{
+    *launched = false;
+    int per_sm = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, calibrate_project_kernel<B>, kCalThreads, 0);
+    if (e != cudaSuccess) return e;
+    int64_t g = calibrate_blocks(rows * cols);
+    const int64_t co_resident = (int64_t)per_sm * device_sm_count();
+    if (co_resident < 1) return cudaSuccess;
+    if (g > co_resident) g = co_resident;
+    CalSync* sync = static_cast<CalSync*>(workspace);
+    CalPartial* part = static_cast<CalPartial*>(workspace) + 1;
+    e = cudaMemsetAsync(sync, 0, 2 * sizeof(unsigned int), st);
+    if (e != cudaSuccess) return e;
+    int* status = device_status_ptr();
+    void* args[] = {(void*)&x, (void*)&rows, (void*)&cols, (void*)&part, (void*)&sync, (void*)&alpha_star,
+                    (void*)&p, (void*)&alpha_out, (void*)&stats_out, (void*)&codes, (void*)&ldc, (void*)&status};
+    e = cudaLaunchCooperativeKernel((const void*)calibrate_project_kernel<B>, dim3((unsigned)g), dim3(kCalThreads),
+                                    args, 0, st);
+    *launched = true;
+    return e;
+}
+
+cudaError_t launch_calibrate_project(const float* x, int64_t rows, int64_t cols, int b, int k, int is_signed,
+                                     int rounding, double alpha_star, void* workspace, float* alpha_out,
+                                     double* stats_out, uint32_t* codes, int64_t ldc, cudaStream_t st)
+{
+    const bool vec = ((reinterpret_cast<uintptr_t>(x) & 15u) == 0) && ((reinterpret_cast<uintptr_t>(codes) & 15u) == 0)
+                     && (cols % 4 == 0) && (ldc % 4 == 0);
+    bool launched = false;
+    cudaError_t e = cudaSuccess;
+    if (vec) {
+        const ProjParams p = make_proj_params(b, k, is_signed, rounding);
+        switch (b) {
+        case 2: e = launch_calibrate_project_b<2>(x, rows, cols, p, alpha_star, workspace, alpha_out, stats_out, codes, ldc, st, &launched); break;
+        case 3: e = launch_calibrate_project_b<3>(x, rows, cols, p, alpha_star, workspace, alpha_out, stats_out, codes, ldc, st, &launched); break;
+        case 4: e = launch_calibrate_project_b<4>(x, rows, cols, p, alpha_star, workspace, alpha_out, stats_out, codes, ldc, st, &launched); break;
+        case 5: e = launch_calibrate_project_b<5>(x, rows, cols, p, alpha_star, workspace, alpha_out, stats_out, codes, ldc, st, &launched); break;
+        case 6: e = launch_calibrate_project_b<6>(x, rows, cols, p, alpha_star, workspace, alpha_out, stats_out, codes, ldc, st, &launched); break;
+        case 7: e = launch_calibrate_project_b<7>(x, rows, cols, p, alpha_star, workspace, alpha_out, stats_out, codes, ldc, st, &launched); break;
+        default: e = launch_calibrate_project_b<8>(x, rows, cols, p, alpha_star, workspace, alpha_out, stats_out, codes, ldc, st, &launched); break;
+        }
+        if (e != cudaSuccess || launched) return e;
+    }
+    // General layouts: the two-launch form.
+    e = launch_calibrate(x, rows * cols, is_signed, alpha_star, workspace, alpha_out, stats_out, st);
+    if (e != cudaSuccess) return e;
+    return launch_project(x, rows, cols, cols, 0.0f, alpha_out, b, k, is_signed, rounding, codes, ldc, st);
 }
 
 // ------------------------------------------- calibration without workspace
 
-// Scratch of esb_calibrate_dda_noalloc: room for the partial record of every
-// block the reduction can launch (kCalMaxBlocks x 32 bytes = 32 KiB).  It is
+// Scratch of esb_calibrate_dda_noalloc: room for the ticket record and the
+// partial record of every block the reduction can launch
+// ((kCalMaxBlocks + 1) x 32 bytes = 32 KiB).  It is
 // a file-scope device array, so it exists on every GPU that loads the
 // library until the process exits, and every call of the variant shares it.
 static_assert(sizeof(CalPartial) == 32, "partial record layout");
-static __device__ __align__(256) unsigned char g_cal_noalloc_scratch[kCalMaxBlocks * 32];
+static __device__ __align__(256) unsigned char g_cal_noalloc_scratch[(kCalMaxBlocks + 1) * 32];
 
 namespace {
 std::mutex g_noalloc_mu;
@@ -450,8 +745,9 @@ cudaError_t launch_calibrate_noalloc(const float* x, int64_t n, int is_signed, d
     void* ws = nullptr;
     cudaError_t e = noalloc_scratch_address(&ws);
     if (e != cudaSuccess) return e;
-    // Pass 1 writes every partial record that pass 2 reads, so nothing in the
-    // shared scratch has to be cleared between calls.
+    // The ticket and flag words are zeroed by a memset node of the launch;
+    // every partial record is written before it is read, so nothing else has
+    // to be cleared.
     return launch_calibrate(x, n, is_signed, alpha_star, ws, alpha_out, stats_out, st);
 }
 

@@ -86,6 +86,7 @@ SIGNATURES = {
     "esb_calibrate_dda": (_I32, [_P, _I64, esb_format, _P, _SZ, _P, _P, _P]),
     "esb_calibrate_dda_noalloc": (_I32, [_P, _I64, esb_format, _P, _P, _P]),
     "esb_project": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _I32, _P, _I64, _P]),
+    "esb_project_dda": (_I32, [_P, _I64, _I64, esb_format, _I32, _P, _SZ, _P, _P, _P, _I64, _P]),
     "esb_dequant": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _P, _I64, _P]),
     "esb_gemm": (_I32, [_I64, _I64, _I64, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
     "esb_conv2d_nhwc": (_I32, [_P, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
@@ -215,6 +216,30 @@ def esb_project(x: torch.Tensor, f: Fmt, alpha=None, rounding: int = ESB_ROUND_H
     _check(lib().esb_project(_ptr(x2), rows, cols, cols, a_host, _ptr(a_dev), f.c(), rounding, _ptr(codes), ldc,
                              _stream(stream)), "esb_project")
     return codes
+
+
+def esb_project_dda(x: torch.Tensor, f: Fmt, rounding: int = ESB_ROUND_HALF_AWAY,
+                    alpha_out: Optional[torch.Tensor] = None, stats_out: Optional[torch.Tensor] = None,
+                    workspace: Optional[torch.Tensor] = None, codes: Optional[torch.Tensor] = None,
+                    ldc: Optional[int] = None, stream=None) -> tuple[torch.Tensor, torch.Tensor]:
+    """DDA calibration and projection of x in one launch -> (codes (rows, ldc) int32, alpha (1,) float)."""
+    _dev(x, "x")
+    assert x.dtype == torch.float32
+    x2 = x.reshape(1, -1) if x.dim() == 1 else x.reshape(-1, x.shape[-1])
+    rows, cols = x2.shape
+    if ldc is None:
+        ldc = esb_row_words(cols, f.b)
+    if codes is None:
+        codes = torch.empty((rows, ldc), dtype=torch.int32, device=x.device)
+    if alpha_out is None:
+        alpha_out = torch.empty(1, dtype=torch.float32, device=x.device)
+    if workspace is None:
+        nb = int(lib().esb_calibrate_dda_workspace_bytes(rows * cols))
+        workspace = torch.empty(max(nb, 8), dtype=torch.uint8, device=x.device)
+    _check(lib().esb_project_dda(_ptr(x2), rows, cols, f.c(), rounding, _ptr(workspace), workspace.numel(),
+                                 _ptr(alpha_out), _ptr(stats_out), _ptr(codes), ldc, _stream(stream)),
+           "esb_project_dda")
+    return codes, alpha_out
 
 
 def esb_dequant(codes: torch.Tensor, cols: int, f: Fmt, alpha, stream=None) -> torch.Tensor:

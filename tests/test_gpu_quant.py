@@ -151,3 +151,38 @@ def test_calibrate_then_project_on_device():
     codes = esb.esb_project(xd, f, alpha=a)
     ah = float(a.item())
     assert np.array_equal(u32(codes), o.project_packed(x.numpy(), ah, 5, 2, ld_words=codes.shape[-1]))
+
+
+PD_CASES = [
+    ("half_normal", (200704, 64), (4, 2, False)),      # the bench layer's activations (6.4 M values)
+    ("normal", (1000, 96), (4, 2, True)),
+    ("laplace", (333, 40), (6, 3, True)),
+    ("normal", (7, 37), (5, 2, True)),                  # ragged: cols % 4 != 0 takes the two-launch form
+    ("half_normal", (1, 8), (3, 1, False)),
+    ("normal", (4096, 128), (4, 1, True)),
+]
+
+
+@pytest.mark.parametrize("dist,shape,fmt", PD_CASES)
+@pytest.mark.parametrize("rounding", [0, 1])
+def test_project_dda_matches_oracle(dist, shape, fmt, rounding):
+    b, k, signed = fmt
+    f = esb.Fmt(b, k, signed)
+    x = synth.distribution(dist, shape, seed=shape[0] + b)
+    stats = torch.zeros(3, dtype=torch.float64, device="cuda")
+    codes, a = esb.esb_project_dda(x.cuda(), f, rounding=rounding, stats_out=stats)
+    ag = float(a.item())
+    ao, so = o.calibrate(x.numpy(), b, k, signed)
+    assert abs(ag - ao) <= 1e-6 * ao, (ag, ao)
+    st = stats.cpu().numpy()
+    assert st[2] == x.numel() and abs(st[1] - so[1]) <= 1e-6 * so[1]
+    if x.numel() > 100000:   # full-size case: sampled rows
+        idx = np.unique(np.concatenate([np.arange(16), np.arange(shape[0] - 16, shape[0]),
+                                        np.random.default_rng(3).integers(0, shape[0], 2000)]))
+        got = u32(codes)[idx]
+        exp = o.project_packed(x.numpy()[idx], ag, b, k, signed, rounding, ld_words=codes.shape[1])
+    else:
+        got = u32(codes)
+        exp = o.project_packed(x.numpy(), ag, b, k, signed, rounding, ld_words=codes.shape[1])
+    assert np.array_equal(got, exp)
+    assert esb.esb_get_status() == 0
