@@ -286,6 +286,27 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d,
                            int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
                            void* stream);
 
+/* Kernels behind esb_conv2d_nhwc. */
+enum {
+    ESB_CONV_KERNEL_HALO = 1,      /* stride 1, 4-bit X: input rows decoded once,
+                                      each filter tap a shifted view (tcgen05) */
+    ESB_CONV_KERNEL_IM2COL = 2,    /* implicit im2col, filters resident in shared memory */
+    ESB_CONV_KERNEL_STREAMED = 3,  /* implicit im2col, filters streamed per K-block */
+    ESB_CONV_KERNEL_DEPTHWISE = 4  /* groups == c, CUDA cores */
+};
+
+/* Which of the kernels above esb_conv2d_nhwc launches for geometry d, X
+ * row stride ldx and formats fx, fw, when its packed output codes have
+ * out_b bits (0: no code output).  The choice depends only on these and on
+ * the device's shared memory (queried on the current device); results are
+ * identical whichever kernel runs.  Setting ESB_CONV_IM2COL=1 in the
+ * environment before the first call disables the halo kernel.
+ *   kernel [host] receives one ESB_CONV_KERNEL_* value
+ * Errors: INVALID_ARG (bad geometry, or the call would be rejected),
+ * CUDA (no device). */
+esb_status esb_conv2d_kernel(const esb_conv_desc* d, int64_t ldx, esb_format fx, esb_format fw, int32_t out_b,
+                             int32_t* kernel);
+
 /* -------------------------------------------------------------- pooling */
 
 /* Max pooling of ESB codes, NHWC (Sec. IV-B "MP" stage with the

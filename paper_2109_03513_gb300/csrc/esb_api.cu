@@ -288,6 +288,30 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d, const uint32_t* X, int64_t ld
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 
+esb_status esb_conv2d_kernel(const esb_conv_desc* d, int64_t ldx, esb_format fx, esb_format fw, int32_t out_b,
+                             int32_t* kernel)
+{
+    if (!d || !kernel) return ESB_ERR_INVALID_ARG;
+    if (!fmt_ok(fx) || !fmt_ok(fw)) return ESB_ERR_INVALID_ARG;
+    if (d->n < 0 || d->h <= 0 || d->w <= 0 || d->c <= 0 || d->cout <= 0 || d->r <= 0 || d->s <= 0 ||
+        d->stride <= 0 || d->pad < 0 || d->pad >= d->r || d->pad >= d->s)
+        return ESB_ERR_INVALID_ARG;
+    if (d->h + 2 * d->pad < d->r || d->w + 2 * d->pad < d->s) return ESB_ERR_INVALID_ARG;
+    if (ldx < words_for(d->c, fx.b)) return ESB_ERR_INVALID_ARG;
+    if (out_b != 0 && (out_b < 2 || out_b > 8)) return ESB_ERR_INVALID_ARG;
+    if (d->groups == d->c && d->c > 1) {
+        *kernel = ESB_CONV_KERNEL_DEPTHWISE;
+        return ESB_OK;
+    }
+    if (d->groups != 1 || fx.b != fw.b || !fmt_tc_ok(fx) || !fmt_tc_ok(fw) || (ldx & 3)) return ESB_ERR_INVALID_ARG;
+    const int P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
+    const int Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
+    const int k = conv_kernel_choice(*d, P, Q, ldx, fx.b, fx.k, out_b ? out_b : 4);
+    if (k < 0) return ESB_ERR_CUDA;
+    *kernel = k;
+    return ESB_OK;
+}
+
 esb_status esb_maxpool_nhwc(const uint32_t* X, int64_t ldx, esb_format f, int32_t n, int32_t h, int32_t w, int32_t c,
                             int32_t win, int32_t stride, int32_t pad, uint32_t* Y, int64_t ldy, void* stream)
 {

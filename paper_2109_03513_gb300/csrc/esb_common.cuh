@@ -390,6 +390,20 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
     return d;
 }
 
+// Shared-memory matrix descriptor, K-major without swizzle: core matrices
+// of 8 rows x 16 bytes (rows 16 bytes apart); sbo = byte stride between
+// 8-row groups along M/N, lbo = byte stride between 16-byte column chunks
+// along K.  Any 16-byte aligned start address.
+__device__ __forceinline__ uint64_t smem_desc_noswz(uint32_t saddr, uint32_t lbo, uint32_t sbo)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);        // start address
+    d |= (uint64_t)((lbo & 0x3FFFFu) >> 4) << 16;    // leading (K) byte offset
+    d |= (uint64_t)((sbo & 0x3FFFFu) >> 4) << 32;    // stride (M/N) byte offset
+    d |= (uint64_t)1u << 46;                         // descriptor version (sm_100 family)
+    return d;                                        // swizzle field 0: none
+}
+
 // Instruction descriptor: kind::f8f6f4, A = B = E4M3, D = F32, K-major
 // operands, M = 128, N = n.
 __host__ __device__ inline uint32_t idesc_e4m3_f32(int n)

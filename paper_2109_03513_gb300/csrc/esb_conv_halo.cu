@@ -1,0 +1,351 @@
+// esb_conv_halo.cu -- stride-1 ESB convolution from a decoded input halo
+// (Sec. IV-B: the r x s x c_in x c_out convolution of the computing logic).
+//
+// The im2col kernel (esb_gemm.cu) decodes every input code once per filter
+// tap.  Here a 128-row output tile is rows_out = 128 / Ws whole output rows
+// of one image, each padded to a pitch of Ws pixel slots (Ws = the power of
+// two >= w + pad).  The producers decode the rows_out + r - 1 input rows
+// that tile needs ONCE into shared memory, pixel-linear: slot
+// (i * Ws + j + pad) holds input pixel (row p0 - pad + i, column j), and the
+// slots of columns w .. Ws - 1, of the left padding and of rows outside the
+// image hold E4M3 zero bytes (the decoded zero code).  Each 16-code channel
+// chunk is its own plane of slots x 16 bytes.
+//
+// Output pixel (p0 + pl, q) is tile row pl * Ws + q, and its tap (r, s)
+// reads slot (pl * Ws + q) + r * Ws + s.  So tap (r, s) of the whole tile is
+// the same buffer seen from a start address shifted by (r * Ws + s) * 16
+// bytes: with A in the K-major no-swizzle layout (rows 16 bytes apart in
+// 8-row core matrices, SBO = 128 bytes between them, LBO = one plane between
+// 16-code chunks), every tap is one descriptor, and the MMA warp issues
+// r * s * (chunks / 2) tcgen05.mma (K = 32) per tile from a single decode.
+// B (the filters, K = (tap, channel)) is resident as in the GEMM kernel, and
+// the epilogue is the shared one; rows with q >= Q or past the image's last
+// output row are computed from zero slots and not stored.
+//
+// Channel blocks of 128 codes are separate stages, so a tile's halo never
+// needs more than 8 planes of shared memory at once.
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "esb_tc.cuh"
+
+namespace esb {
+
+struct HaloGeom {
+    const uint32_t* X;   // n*h*w pixels of ldx words
+    int ldx;             // words per pixel (multiple of 4)
+    int H, W, P, Q, R, S, pad;
+    int lws;             // log2(Ws)
+    int rows_out;        // output rows per tile (128 / Ws)
+    int tpi;             // tiles per image
+    int hr;              // halo rows (rows_out + R - 1)
+    int ns;              // slots per plane (128 + (R-1) * Ws + S - 1)
+    int pb;              // bytes per plane (ns * 16)
+    int cblocks;         // channel blocks of 16 words
+    int stage_bytes;     // planes of one channel block (<= 8 planes)
+};
+
+// Producer: decode one channel block of one tile's halo into stage st.
+// Lane l owns slots l, l + 32, ...; each slot takes NPC 16-byte pieces
+// (4 words = two 16-code chunks each) of its pixel.  The pieces of up to
+// 16 / NPC slot groups are loaded before any decode, so a fill makes at
+// most a few round trips to memory.
+template <int NPC>
+__device__ __forceinline__ void halo_fill_t(const HaloGeom& g, int p0, const uint32_t* xi, uint8_t* st, int lane,
+                                            int k, int ew)
+{
+    constexpr int GB = 16 / NPC;                                   // slot groups per batch
+    const int groups = (g.ns + 31) >> 5;
+    const int nb = (groups + GB - 1) / GB;
+    const int per = (groups + nb - 1) / nb;                        // balanced batches
+    const int wsm = (1 << g.lws) - 1;
+#pragma unroll 1
+    for (int g0 = 0; g0 < groups; g0 += per) {
+        uint4 v[GB][NPC];
+        uint32_t okm = 0u;
+#pragma unroll
+        for (int u = 0; u < GB; u++) {
+            const int slot = (g0 + u) * 32 + lane;
+            const int rel = slot - g.pad;
+            const int hi = rel >> g.lws;                           // halo row (-1: left guard)
+            const int j = rel & wsm;
+            const int h = p0 - g.pad + hi;
+            const bool ok = u < per && slot < g.ns && rel >= 0 && hi < g.hr && j < g.W && (unsigned)h < (unsigned)g.H;
+            const uint4* px = reinterpret_cast<const uint4*>(xi + ((int64_t)h * g.W + j) * g.ldx);
+#pragma unroll
+            for (int pc = 0; pc < NPC; pc++) v[u][pc] = ok ? __ldg(px + pc) : make_uint4(0u, 0u, 0u, 0u);
+            okm |= (ok ? 1u : 0u) << u;
+        }
+#pragma unroll
+        for (int u = 0; u < GB; u++) {
+            const int slot = (g0 + u) * 32 + lane;
+            if (u >= per || slot >= g.ns) break;
+            const bool ok = (okm >> u) & 1u;
+#pragma unroll
+            for (int pc = 0; pc < NPC; pc++) {
+                uint4 c0 = make_uint4(0u, 0u, 0u, 0u), c1 = c0;
+                if (ok) {
+                    decode_word_b4(v[u][pc].x, k, ew, c0.x, c0.y);
+                    decode_word_b4(v[u][pc].y, k, ew, c0.z, c0.w);
+                    decode_word_b4(v[u][pc].z, k, ew, c1.x, c1.y);
+                    decode_word_b4(v[u][pc].w, k, ew, c1.z, c1.w);
+                }
+                uint8_t* dst = st + (2 * pc) * g.pb + slot * 16;
+                *reinterpret_cast<uint4*>(dst) = c0;
+                *reinterpret_cast<uint4*>(dst + g.pb) = c1;
+            }
+        }
+    }
+}
+
+// Channel block cb (words 16 cb .. of each pixel) of tile T's halo.
+__device__ __noinline__ void halo_fill(const HaloGeom g, int64_t T, int cb, uint8_t* st, int lane, int k, int ew)
+{
+    const int nimg = (int)(T / g.tpi);
+    const int p0 = (int)(T - (int64_t)nimg * g.tpi) * g.rows_out;
+    const int w0 = cb * 16;
+    const int npc = min(16, g.ldx - w0) >> 2;                      // pieces per slot (1..4)
+    const uint32_t* xi = g.X + (int64_t)nimg * g.H * g.W * g.ldx + w0;
+    switch (npc) {
+    case 1: halo_fill_t<1>(g, p0, xi, st, lane, k, ew); break;
+    case 2: halo_fill_t<2>(g, p0, xi, st, lane, k, ew); break;
+    case 3: halo_fill_t<3>(g, p0, xi, st, lane, k, ew); break;
+    default: halo_fill_t<4>(g, p0, xi, st, lane, k, ew); break;
+    }
+}
+
+__global__ void __launch_bounds__(kWsThreads, 1)
+esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, OpFmt fb, int BN, int nkb,
+                     int stages, int n_tiles, int64_t m_tiles, float acc_scale, EpiParams ep)
+{
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sB = smem;                                        // nkb blocks of BN x 128 bytes (SW128)
+    uint8_t* sA = sB + nkb * BN * kBK;                         // stages x stage_bytes (halo planes)
+    float* thr = reinterpret_cast<float*>(sA + stages * g.stage_bytes);
+    uint64_t* full = reinterpret_cast<uint64_t*>(thr + 128);
+    uint64_t* empty = full + kWsMaxStages;
+    uint64_t* tfull = empty + kWsMaxStages;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* err = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int n_tile = (int)(blockIdx.x % n_tiles);
+    const int64_t cta_in_n = blockIdx.x / n_tiles;
+    const int64_t ctas_per_n = gridDim.x / n_tiles;
+    const int64_t n0 = (int64_t)n_tile * BN;
+    const int64_t my_tiles = (m_tiles > cta_in_n) ? (m_tiles - cta_in_n + ctas_per_n - 1) / ctas_per_n : 0;
+    uint32_t tmem_cols = 32;
+    while ((int)tmem_cols < 2 * BN) tmem_cols <<= 1;
+    const int half_cols = BN / 2;
+    const bool split = (half_cols % 16 == 0) && (half_cols % ep.out_cpw == 0);
+    const int epi_warps = split ? 8 : 4;
+    const int cbs = g.cblocks;
+
+    if (tid == 0) {
+        for (int s = 0; s < stages; s++) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; a++) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], epi_warps);
+        }
+        mbar_init(drain, 1);
+        *err = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+
+    uint32_t tmem_base = 0;
+    if (warp < kWsProdWarp0)
+        tmem_base = ws_setup(srcB, n0, K, fb, BN, nkb, sB, thr, ep, tmem_slot, tmem_cols, tid);
+
+    if (warp >= kWsProdWarp0) {
+        // ---------------------------------------------- halo producers
+        // Warp p fills iterations p, p + nprod, ... of this CTA's (tile,
+        // channel block) sequence; at most `stages` producers are active
+        // (an mbarrier's parity tells apart only adjacent phases).
+        const int p = warp - kWsProdWarp0;
+        const int nprod = stages < kWsProdWarps ? stages : kWsProdWarps;
+        const int64_t total_it = (p < nprod) ? my_tiles * cbs : 0;
+        for (int64_t it = p; it < total_it && !*err; it += nprod) {
+            const int64_t ti = it / cbs;
+            const int cb = (int)(it - ti * cbs);
+            const int s = (int)(it % stages);
+            const uint32_t ph = (uint32_t)((it / stages) & 1);
+            if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
+            halo_fill(g, cta_in_n + ti * ctas_per_n, cb, sA + s * g.stage_bytes, lane, fa.k, fa.ew);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&full[s]);
+        }
+    } else if (warp == kWsMmaWarp) {
+        // ---------------------------------------------- MMA issue
+        if (lane == 0) {
+            const uint32_t idesc = idesc_e4m3_f32(BN);
+            const uint32_t b_base = smem_u32(sB), a_base = smem_u32(sA);
+            const int ctap = g.ldx * 8;                        // codes per tap
+            const int ws = 1 << g.lws;
+            int64_t it = 0;
+            for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
+                const int a = (int)(ti & 1);
+                if (!wait_or_abort(&tempty[a], (uint32_t)((ti >> 1) & 1) ^ 1u, err)) { *err = 1; break; }
+                tc_fence_after();
+                const uint32_t d = tmem_base + (uint32_t)(a * BN);
+                for (int cb = 0; cb < cbs; cb++, it++) {
+                    const int s = (int)(it % stages);
+                    if (!wait_or_abort(&full[s], (uint32_t)((it / stages) & 1), err)) { *err = 1; break; }
+                    tc_fence_after();
+                    const uint32_t a0 = a_base + (uint32_t)(s * g.stage_bytes);
+                    const int pairs = min(16, g.ldx - cb * 16) >> 2;   // K = 32 steps in this block
+                    for (int t = 0; t < g.R * g.S; t++) {
+                        const int r = t / g.S, sx = t - r * g.S;
+                        const uint32_t at = a0 + (uint32_t)((r * ws + sx) * 16);
+                        for (int j = 0; j < pairs; j++) {
+                            const int k0 = t * ctap + cb * 128 + 32 * j;
+                            const uint32_t bb = b_base + (uint32_t)((k0 >> 7) * BN * kBK + ((k0 & 127) >> 5) * 32);
+                            mma_f8f6f4(d, smem_desc_noswz(at + (uint32_t)(2 * j * g.pb), (uint32_t)g.pb, 128u),
+                                       smem_desc_sw128(bb), idesc, (cb > 0 || t > 0 || j > 0) ? 1u : 0u);
+                        }
+                    }
+                    mma_commit(&empty[s]);
+                }
+                if (*err) break;
+                mma_commit(&tfull[a]);
+            }
+            ws_drain(drain, err);
+        }
+    } else if (warp < epi_warps) {
+        // ---------------------------------------------- epilogue
+        const int64_t ctas = ctas_per_n, first = cta_in_n;
+        const HaloGeom gg = g;
+        auto rows = [=](int64_t ti, int row, int64_t& m) -> bool {
+            const int64_t T = first + ti * ctas;
+            const int64_t nimg = T / gg.tpi;
+            const int p = (int)(T - nimg * gg.tpi) * gg.rows_out + (row >> gg.lws);
+            const int q = row & ((1 << gg.lws) - 1);
+            m = (nimg * gg.P + p) * gg.Q + q;
+            return q < gg.Q && p < gg.P;
+        };
+        ws_epilogue(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
+                    warp, lane);
+    }
+
+    __syncthreads();
+    if (*err && tid == 0) record_status(ep.status, ESB_ERR_TIMEOUT);
+    if (warp == kWsMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, tmem_cols);
+    }
+}
+
+// Minimum share of the computed tile rows that are real output pixels for
+// the halo path to be taken (56 x 56: 87.5 %; 7 x 7: 38 %, im2col instead).
+constexpr double kHaloMinUse = 0.7;
+
+struct HaloPlan {
+    HaloGeom g;
+    int BN, nkb, stages;
+    int64_t K, smem;
+};
+
+static int halo_static_smem(cudaError_t* err)
+{
+    static int v = -1;
+    if (v < 0) {
+        cudaFuncAttributes a;
+        *err = cudaFuncGetAttributes(&a, esb_conv_halo_kernel);
+        if (*err != cudaSuccess) return -1;
+        v = (int)a.sharedSizeBytes;
+    }
+    return v;
+}
+
+// Geometry, N-tile width and shared-memory budget of the halo path, or
+// false when the shape does not suit it.  BN starts at bn0 and shrinks
+// (keeping whole output words) until the resident B and two halo stages fit.
+static bool halo_plan(const esb_conv_desc& d, int P, int Q, int64_t ldx, const OpFmt& fa, int bn0, int out_cpw,
+                      HaloPlan* hp, cudaError_t* err)
+{
+    *err = cudaSuccess;
+    if (d.stride != 1 || fa.b != 4 || ldx % 4 != 0 || ldx > (1 << 20) || d.pad > d.r - 1 || d.pad > d.s - 1)
+        return false;
+    int lws = 0;
+    while ((1 << lws) < d.w + d.pad) lws++;
+    const int ws = 1 << lws;
+    if (ws > kBM || Q > ws) return false;
+    HaloGeom& g = hp->g;
+    g.X = nullptr; g.ldx = (int)ldx; g.H = d.h; g.W = d.w; g.P = P; g.Q = Q; g.R = d.r; g.S = d.s; g.pad = d.pad;
+    g.lws = lws;
+    g.rows_out = kBM / ws;
+    g.tpi = (P + g.rows_out - 1) / g.rows_out;
+    if ((double)P * Q / ((double)g.tpi * kBM) < kHaloMinUse) return false;
+    g.hr = g.rows_out + d.r - 1;
+    g.ns = kBM + (d.r - 1) * ws + d.s - 1;
+    g.pb = g.ns * 16;
+    g.cblocks = (int)((ldx + 15) / 16);
+    const int planes = (int)(ldx >= 16 ? 8 : ldx / 2);
+    g.stage_bytes = ((planes * g.pb + 127) / 128) * 128;
+    const int st_smem = halo_static_smem(err);
+    if (st_smem < 0) return false;
+    const int maxs = max_dyn_smem() - st_smem;
+    hp->K = (int64_t)d.r * d.s * ldx * 8;
+    hp->nkb = (int)((hp->K + kBK - 1) / kBK);
+    static const int cands[] = {256, 240, 224, 208, 192, 176, 160, 144, 128, 112, 96, 80, 64, 48, 32, 16};
+    for (int i = -1; i < (int)(sizeof(cands) / sizeof(cands[0])); i++) {
+        const int bn = i < 0 ? bn0 : cands[i];
+        if (bn <= 0 || (i >= 0 && bn >= bn0) || bn % out_cpw != 0) continue;
+        const int64_t fixed = 1024 + (int64_t)hp->nkb * bn * kBK + 4 * 128 + 512;
+        int64_t stg = (maxs - fixed) / g.stage_bytes;
+        if (stg > kWsMaxStages) stg = kWsMaxStages;
+        if (stg < 2) continue;
+        hp->BN = bn;
+        hp->stages = (int)stg;
+        hp->smem = fixed + stg * (int64_t)g.stage_bytes;
+        return true;
+    }
+    return false;
+}
+
+bool conv_halo_ok(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int kx, int out_cpw)
+{
+    HaloPlan hp;
+    cudaError_t e;
+    return halo_plan(d, P, Q, ldx, make_opfmt(bx, kx), pick_bn(d.cout, out_cpw), out_cpw, &hp, &e);
+}
+
+bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, const OpFmt& fa,
+                      const uint32_t* W, int64_t ldw, const OpFmt& fb, int BN, const EpiParams& ep, cudaStream_t st,
+                      cudaError_t* err)
+{
+    HaloPlan hp;
+    if (!halo_plan(d, P, Q, ldx, fa, BN, ep.out_cpw, &hp, err)) return *err != cudaSuccess;
+    hp.g.X = X;
+    static bool configured = false;
+    if (!configured) {
+        *err = cudaFuncSetAttribute(esb_conv_halo_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    max_dyn_smem() - halo_static_smem(err));
+        if (*err != cudaSuccess) return true;
+        configured = true;
+    }
+    const int64_t N = d.cout;
+    const int n_tiles = (int)((N + hp.BN - 1) / hp.BN);
+    const int64_t m_tiles = (int64_t)d.n * hp.g.tpi;
+    int64_t per_n = device_sm_count() / n_tiles;
+    if (per_n < 1) per_n = 1;
+    if (per_n > m_tiles) per_n = m_tiles;
+    const int64_t grid = per_n * n_tiles;
+    RowsSrc b{W, (int64_t)d.r * d.s * ldw, N};
+    const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
+    esb_conv_halo_kernel<<<(unsigned)grid, kWsThreads, (size_t)hp.smem, st>>>(hp.g, b, N, hp.K, fa, fb, hp.BN, hp.nkb,
+                                                                             hp.stages, n_tiles, m_tiles, acc_scale,
+                                                                             ep);
+    *err = cudaGetLastError();
+    return true;
+}
+
+}  // namespace esb

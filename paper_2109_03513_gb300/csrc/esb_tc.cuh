@@ -1,0 +1,507 @@
+// esb_tc.cuh -- device code shared by the tcgen05 contraction kernels
+// (esb_gemm.cu: GEMM and im2col convolution; esb_conv_halo.cu: stride-1
+// convolution from a decoded input halo): operand decode of ESB codes to
+// scaled E4M3 bytes, the fused post-processing epilogue (Sec. IV-C), the
+// bounded mbarrier waits, and the setup and epilogue roles of the
+// persistent warp-specialised kernels.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "esb_common.cuh"
+#include "esb_internal.h"
+
+namespace esb {
+
+constexpr int kBM = 128;           // rows per tile (TMEM lanes)
+constexpr int kBK = 128;           // codes (= E4M3 bytes) per K-block: one 128-byte swizzle row
+constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
+
+struct OpFmt {
+    int b, k, ew, cpw;
+    uint32_t mask;
+};
+
+__host__ inline OpFmt make_opfmt(int b, int k)
+{
+    OpFmt o;
+    o.b = b; o.k = k; o.ew = b - k - 1; o.cpw = 32 / b; o.mask = (1u << b) - 1u;
+    return o;
+}
+
+// Byte position of code j (0..15) of a 16-code unit.  The fast b = 4
+// decode emits codes 0,2,4,6 | 1,3,5,7 of each word; every path uses the
+// same order, so A and B agree on the K permutation (a contraction is
+// invariant under a common permutation of K).
+__device__ __forceinline__ int unit_pos(int j) { return ((j >> 3) << 3) | ((j & 1) << 2) | ((j & 7) >> 1); }
+
+// One code -> scaled E4M3 byte.
+__device__ __forceinline__ uint32_t code_to_e4m3(uint32_t c, const OpFmt& f)
+{
+    const uint32_t s = (c >> (f.b - 1)) & 1u;
+    const uint32_t fr = c & ((1u << f.k) - 1u);
+    uint32_t E = 0u;
+    if (f.ew > 0) {
+        const uint32_t em = (1u << f.ew) - 1u;
+        E = (((c >> f.k) & em) + 1u) & em;
+    }
+    return (s << 7) | (E << 3) | (fr << (3 - f.k));
+}
+
+// 8 four-bit codes (one word) -> 8 scaled E4M3 bytes (lo: codes 0,2,4,6; hi: 1,3,5,7).
+__device__ __forceinline__ void decode_word_b4(uint32_t w, int k, int ew, uint32_t& lo, uint32_t& hi)
+{
+    uint32_t u = w;
+    if (ew > 0) u = (((w & 0x77777777u) + (0x11111111u << k)) & 0x77777777u) | (w & 0x88888888u);
+    const uint32_t a = u & 0x0F0F0F0Fu;
+    const uint32_t b = (u >> 4) & 0x0F0F0F0Fu;
+    const int sh = 3 - k;
+    lo = ((a & 0x07070707u) << sh) | ((a & 0x08080808u) << 4);
+    hi = ((b & 0x07070707u) << sh) | ((b & 0x08080808u) << 4);
+}
+
+// ------------------------------------------------------------ row sources
+
+// Plain K-major rows: logical word w of row r is base[r * ld + w].
+struct RowsSrc {
+    const uint32_t* base;
+    int64_t ld;
+    int64_t rows;
+    struct Row { const uint32_t* p; };
+    struct Cursor { int64_t w; };
+    __device__ __forceinline__ Row row(int64_t r) const { Row x; x.p = (r < rows) ? base + r * ld : nullptr; return x; }
+    __device__ __forceinline__ const uint32_t* words(const Row& x, int64_t w) const { return x.p ? x.p + w : nullptr; }
+    __device__ __forceinline__ Cursor cursor(int64_t w) const { Cursor c; c.w = w; return c; }
+    __device__ __forceinline__ void advance(Cursor& c, int dw) const { c.w += dw; }
+    __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const { return x.p ? x.p + c.w : nullptr; }
+};
+
+// General decode of the 16-code unit [k0, k0 + 16) of one row (any b, K tail).
+template <class Src>
+__device__ __noinline__ uint4 decode_unit_any(const Src& src, const typename Src::Row& row, int64_t k0, int64_t K,
+                                              const OpFmt f)
+{
+    uint32_t o0 = 0u, o1 = 0u, o2 = 0u, o3 = 0u;
+#pragma unroll 1
+    for (int j = 0; j < 16; j++) {
+        const int64_t kk = k0 + j;
+        if (kk >= K) break;
+        const int64_t wi = kk / f.cpw;
+        const int slot = (int)(kk - wi * f.cpw);
+        const uint32_t* p = src.words(row, wi);
+        if (!p) continue;
+        const uint32_t c = (__ldg(p) >> (f.b * slot)) & f.mask;
+        const uint32_t byte = code_to_e4m3(c, f);
+        const int pos = unit_pos(j);
+        const uint32_t v = byte << (8 * (pos & 3));
+        switch (pos >> 2) {
+        case 0: o0 |= v; break;
+        case 1: o1 |= v; break;
+        case 2: o2 |= v; break;
+        default: o3 |= v; break;
+        }
+    }
+    return make_uint4(o0, o1, o2, o3);
+}
+
+__device__ __forceinline__ uint32_t swz(int r, int g) { return (uint32_t)(r * 128 + ((g ^ (r & 7)) << 4)); }
+
+// ------------------------------------------------------------ epilogue
+
+struct EpiParams {
+    const float* scale;
+    const float* alpha_a_dev;
+    const float* alpha_b_dev;
+    float dq_pow2;            // 2^-(kA+kB)
+    const float* bias;
+    float scale0, bias0;
+    int act;
+    const uint32_t* residual;
+    int64_t res_ld;
+    int res_b, res_k;
+    float res_scale;
+    float alpha_out;
+    const float* alpha_out_dev;
+    ProjParams out;
+    int out_cpw;
+    int32_t* acc_out;
+    float* y_out;
+    uint32_t* codes_out;
+    int64_t ldo;
+    int* status;
+};
+
+__device__ __forceinline__ float apply_act(float y, int act)
+{
+    if (act == ESB_ACT_RELU) {
+        y = (y > 0.0f) ? y : 0.0f;
+    } else if (act == ESB_ACT_RELU6) {
+        y = (y > 0.0f) ? y : 0.0f;
+        y = (y < 6.0f) ? y : 6.0f;
+    }
+    return y;
+}
+
+// Per-kernel constants of the epilogue.
+struct EpiCtx {
+    bool dq;
+    float dqs;
+    const float* T;     // requantisation thresholds (shared memory)
+    Thr7 t7;
+    bool b4;
+};
+
+__device__ __forceinline__ EpiCtx make_epi_ctx(const EpiParams& ep, const float* T)
+{
+    EpiCtx c;
+    c.dq = ep.alpha_a_dev && ep.alpha_b_dev;
+    c.dqs = c.dq ? __fmul_rn(__ldg(ep.alpha_a_dev), __ldg(ep.alpha_b_dev)) * ep.dq_pow2 : 1.0f;
+    c.T = T;
+    c.b4 = ep.out.b == 4;
+#pragma unroll
+    for (int i = 0; i < 7; i++) c.t7.t[i] = (ep.codes_out && c.b4) ? T[i] : 0.0f;
+    return c;
+}
+
+// One output element: affine, residual, activation, optional stores, code.
+__device__ __forceinline__ uint32_t epi_element(const EpiParams& ep, const EpiCtx& cx, float af, int64_t m, int64_t n,
+                                                int64_t N)
+{
+    if (ep.acc_out) ep.acc_out[m * N + n] = __float2int_rn(af);
+    float sc = ep.scale ? __ldg(ep.scale + n) : ep.scale0;
+    if (cx.dq) sc = __fmul_rn(sc, cx.dqs);
+    const float bi = ep.bias ? __ldg(ep.bias + n) : ep.bias0;
+    float y = __fmaf_rn(sc, af, bi);
+    if (ep.residual) {
+        const int rcpw = 32 / ep.res_b;
+        const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >> (ep.res_b * (int)(n % rcpw))) &
+                            ((1u << ep.res_b) - 1u);
+        y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+    }
+    y = apply_act(y, ep.act);
+    if (ep.y_out) ep.y_out[m * N + n] = y;
+    if (!ep.codes_out) return 0u;
+    return cx.b4 ? project_by_thr7(y, cx.t7, ep.out) : project_by_table(y, cx.T, ep.out);
+}
+
+// Wait on an mbarrier phase with a wall-clock bound and an abort flag
+// raised by another role of the CTA.
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* err)
+{
+    const uint32_t a = smem_u32(bar);
+    if (mbar_try_wait(a, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try_wait(a, parity)) return true;
+        if ((it & 255u) == 0u) {
+            if (*err) return false;
+            if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// ----------------------------------------- resident-B persistent kernel
+
+constexpr int kWsEpiWarps = 8;                 // warps 0-7: epilogue (lanes 32*(w&3).., column half w>>2)
+constexpr int kWsMmaWarp = 8;                  // warp 8: TMEM allocation and MMA issue
+constexpr int kWsProdWarp0 = 9;                // warps 9-15: A producers, one stage at a time each
+constexpr int kWsProdWarps = 7;
+constexpr int kWsThreads = (kWsProdWarp0 + kWsProdWarps) * 32;   // 512: 4 warps per SM sub-partition
+constexpr int kWsMaxStages = 8;
+
+// Byte masks of the decoded lo/hi words of one b = 4 word when only its
+// first v codes (0..8) are inside K.
+__device__ __forceinline__ void tail_masks(int v, uint32_t& mlo, uint32_t& mhi)
+{
+    const int nlo = (v + 1) >> 1, nhi = v >> 1;       // lo holds codes 0,2,4,6; hi 1,3,5,7
+    mlo = nlo >= 4 ? 0xffffffffu : ((1u << (8 * nlo)) - 1u);
+    mhi = nhi >= 4 ? 0xffffffffu : ((1u << (8 * nhi)) - 1u);
+}
+
+// Decode one 128-code K-block slice (16 words, four 16-byte pieces) of a
+// b = 4 row and store its 8 units to a swizzled stage row.  The loads of
+// all four pieces are issued before any decode.
+// Pieces outside the operand (rows past M or N, out-of-image taps, words
+// past K) are filled with the zero code -- the all-zero bit pattern is not
+// zero in this format (it is the value 1).
+template <class Src>
+__device__ __forceinline__ void load_row_b4(const Src& src, const typename Src::Row& row,
+                                            const typename Src::Cursor (&cur)[4], int64_t kw0, int64_t K,
+                                            uint32_t zero_word, uint4 (&v)[4])
+{
+#pragma unroll
+    for (int pc = 0; pc < 4; pc++) {
+        const int64_t kk0 = (kw0 + 4 * pc) * 8;       // first code of the piece
+        const uint32_t* p = (kk0 < K) ? src.at(row, cur[pc]) : nullptr;
+        v[pc] = p ? __ldg(reinterpret_cast<const uint4*>(p)) : make_uint4(zero_word, zero_word, zero_word, zero_word);
+    }
+}
+
+__device__ __forceinline__ void store_row_b4(uint8_t* stage, int r, const uint4 (&v)[4], int64_t kw0, int64_t K,
+                                             const OpFmt& f)
+{
+    const bool tail = (kw0 + 16) * 8 > K;             // only the last K-block can reach past K
+#pragma unroll
+    for (int pc = 0; pc < 4; pc++) {
+        const uint32_t w[4] = {v[pc].x, v[pc].y, v[pc].z, v[pc].w};
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+            uint32_t o0, o1, o2, o3;
+            decode_word_b4(w[2 * h], f.k, f.ew, o0, o1);
+            decode_word_b4(w[2 * h + 1], f.k, f.ew, o2, o3);
+            const int64_t wi = kw0 + 4 * pc + 2 * h;  // word index of w[2h]
+            if (tail && (wi + 2) * 8 > K) {           // K tail: zero the codes past K
+                uint32_t ml, mh;
+                int va = (int)(K - wi * 8);
+                va = va < 0 ? 0 : (va > 8 ? 8 : va);
+                tail_masks(va, ml, mh);
+                o0 &= ml; o1 &= mh;
+                int vb = (int)(K - (wi + 1) * 8);
+                vb = vb < 0 ? 0 : (vb > 8 ? 8 : vb);
+                tail_masks(vb, ml, mh);
+                o2 &= ml; o3 &= mh;
+            }
+            *reinterpret_cast<uint4*>(stage + swz(r, 2 * pc + h)) = make_uint4(o0, o1, o2, o3);
+        }
+    }
+}
+
+// Epilogue of one 16-column chunk for outputs other than the lean 4-bit
+// path (general packing), out of line; reads its own TMEM chunk.
+static __device__ __noinline__ void epi_chunk_any(const EpiParams* __restrict__ sep, const EpiCtx* __restrict__ scx,
+                                           uint32_t taddr, float acc_scale, int64_t m, bool mrow, int64_t n_first,
+                                           int64_t N, uint32_t* word_slot_w)
+{
+    const EpiParams& ep = *sep;
+    const EpiCtx cx = *scx;
+    uint32_t r[16];
+    tmem_ld16(taddr, r);
+    const int cpw = ep.out_cpw;
+    uint32_t word = word_slot_w[0];
+    int slot = (int)word_slot_w[1];
+    int64_t wcol = (int64_t)word_slot_w[2] | ((int64_t)word_slot_w[3] << 32);
+#pragma unroll
+    for (int j = 0; j < 16; j++) {
+        const int64_t n = n_first + j;
+        uint32_t code = ep.out.zero_code;
+        if (mrow && n < N) code = epi_element(ep, cx, __uint_as_float(r[j]) * acc_scale, m, n, N);
+        word |= code << (ep.out.b * slot);
+        if (++slot == cpw) {
+            if (ep.codes_out && mrow && wcol < ep.ldo) ep.codes_out[m * ep.ldo + wcol] = word;
+            word = 0;
+            slot = 0;
+            wcol++;
+        }
+    }
+    word_slot_w[0] = word;
+    word_slot_w[1] = (uint32_t)slot;
+    word_slot_w[2] = (uint32_t)(wcol & 0xffffffff);
+    word_slot_w[3] = (uint32_t)(wcol >> 32);
+}
+
+
+// ------------------------------------ roles of the warp-specialised kernels
+
+// Setup role (warps 0 .. kWsProdWarp0 - 1, while the producers already load
+// A): the MMA warp allocates tmem_cols TMEM columns; all setup warps decode
+// the CTA's N-tile of B (rows n0 .. n0 + BN, every K-block) once into sB in
+// the SW128 K-major layout, and build the requantisation thresholds; then
+// they meet on named barrier 1.  Returns the TMEM base address.
+__device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, int64_t K, const OpFmt& fb, int BN,
+                                             int nkb, uint8_t* sB, float* thr, const EpiParams& ep,
+                                             uint32_t* tmem_slot, uint32_t tmem_cols, int tid)
+{
+    constexpr int kSetupThreads = kWsProdWarp0 * 32;
+    const int warp = tid >> 5, lane = tid & 31;
+    if (warp == kWsMmaWarp) {
+        tmem_alloc(tmem_slot, tmem_cols);
+        tc_fence_before();
+    }
+    if (fb.b == 4) {
+        for (int pr = tid; pr < nkb * BN; pr += kSetupThreads) {
+            const int kb = pr / BN, r = pr - kb * BN;
+            const RowsSrc::Row row = srcB.row(n0 + r);
+            const int64_t kw0 = (int64_t)kb * 16;
+            RowsSrc::Cursor cur[4];
+#pragma unroll
+            for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
+            uint4 v[4];
+            load_row_b4(srcB, row, cur, kw0, K, fmt_zero_code(4, fb.k) * 0x11111111u, v);
+            store_row_b4(sB + kb * BN * kBK, r, v, kw0, K, fb);
+        }
+    } else {
+        for (int u = tid; u < nkb * BN * 8; u += kSetupThreads) {
+            const int kb = u / (BN * 8);
+            const int rem = u - kb * BN * 8;
+            const int r = rem >> 3, g = rem & 7;
+            *reinterpret_cast<uint4*>(sB + kb * BN * kBK + swz(r, g)) =
+                decode_unit_any(srcB, srcB.row(n0 + r), (int64_t)kb * kBK + g * 16, K, fb);
+        }
+    }
+    fence_proxy_async_smem();
+    if (ep.codes_out) {
+        const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
+        build_thresholds(thr, ep.out, alpha_out, warp, lane, 0, kWsProdWarp0);
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(kSetupThreads) : "memory");
+    tc_fence_after();
+    return *tmem_slot;
+}
+
+// Epilogue role (warps 0 .. epi_warps - 1): drains the accumulator tiles of
+// this CTA in order, tile ti from TMEM buffer ti & 1 (columns (ti & 1) * BN
+// ..), and frees the buffer on tempty once its columns are in registers.
+// Warp w reads TMEM lanes 32 (w & 3) .. +31 (= tile rows); with split, warps
+// 0-3 take the columns [0, BN/2) and warps 4-7 [BN/2, BN).  rows(ti, row, m)
+// gives the output row m of a tile row and whether it exists.
+template <class RowMap>
+__device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* thr, const RowMap& rows,
+                                            int64_t my_tiles, int64_t n0, int64_t N, int BN, bool split,
+                                            int epi_warps, uint32_t tmem_base, float acc_scale, uint64_t* tfull,
+                                            uint64_t* tempty, volatile int* err, int warp, int lane)
+{
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;              // TMEM lane = tile row
+    __shared__ EpiParams sh_ep;                       // copies for the out-of-line general path
+    __shared__ EpiCtx sh_cx;
+    const int half_cols = BN / 2;
+    const int c_lo = split ? (warp >> 2) * half_cols : 0;
+    const int c_hi = split ? c_lo + half_cols : BN;
+    const EpiCtx cx = make_epi_ctx(ep, thr);
+    if (warp == 0 && lane == 0) { sh_ep = ep; sh_cx = cx; }
+    asm volatile("bar.sync 2, %0;" ::"r"(epi_warps * 32) : "memory");   // exactly the epilogue warps in use
+    const int cpw = ep.out_cpw;
+    const bool swar = ep.codes_out && ep.out.b == 4;
+    const float T0 = cx.t7.t[0], T1 = cx.t7.t[1], T2 = cx.t7.t[2], T3 = cx.t7.t[3], T4 = cx.t7.t[4],
+                T5 = cx.t7.t[5], T6 = cx.t7.t[6];
+    const float sc_fixed = ep.scale ? 0.0f : (cx.dq ? __fmul_rn(ep.scale0, cx.dqs) : ep.scale0);
+    const float sc_lean = sc_fixed * acc_scale;
+    const bool out_signed = ep.out.is_signed != 0;
+    // the lean path needs every column of the chunk inside N and a finite folded scale
+    const bool lean_ok = swar && !ep.scale && !ep.bias && !ep.residual && !ep.acc_out && !ep.y_out &&
+                         isfinite(sc_lean) && (sc_lean != 0.0f || sc_fixed == 0.0f);
+    for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
+        const int a = (int)(ti & 1);
+        if (!wait_or_abort(&tfull[a], (uint32_t)((ti >> 1) & 1), err)) { *err = 1; break; }
+        tc_fence_after();
+        int64_t m = 0;
+        const bool mrow = rows(ti, row, m);
+        const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(a * BN);
+        uint32_t wsw[4] = {0u, 0u, (uint32_t)(((n0 + c_lo) / cpw) & 0xffffffff),
+                           (uint32_t)(((n0 + c_lo) / cpw) >> 32)};   // general path: word, slot, column
+        for (int c = c_lo; c < c_hi; c += 16) {
+            if (!swar) {
+                epi_chunk_any(&sh_ep, &sh_cx, taddr + (uint32_t)c, acc_scale, m, mrow, n0 + c, N, wsw);
+                if (c + 16 >= c_hi) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&tempty[a]);
+                }
+                continue;
+            }
+            uint32_t r[16];
+            tmem_ld16(taddr + (uint32_t)c, r);
+            const bool lean = lean_ok && (n0 + c + 16 <= N);
+            if (c + 16 >= c_hi) {                     // every column of this warp is in registers
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[a]);
+            }
+            uint32_t wds[2];
+            if (lean) {
+                // 4-bit output codes only, scalar scale/bias, no residual:
+                // y = fma(scale * 2^(kA+kB+12), raw, bias) equals
+                // fma(scale, acc, bias) exactly (power-of-two scaling),
+                // then the bucket of y among the 7 thresholds, eight codes
+                // per word at once.
+#pragma unroll
+                for (int h = 0; h < 2; h++) {
+                    uint32_t J = 0u, S = 0u;
+#pragma unroll
+                    for (int j = 0; j < 8; j++) {
+                        float y = __fmaf_rn(sc_lean, __uint_as_float(r[8 * h + j]), ep.bias0);
+                        y = apply_act(y, ep.act);
+                        const float av = out_signed ? fabsf(y) : y;
+                        const bool b2 = av >= T3;
+                        const bool b1 = av >= (b2 ? T5 : T1);
+                        const bool b0 = av >= (b2 ? (b1 ? T6 : T4) : (b1 ? T2 : T0));
+                        J |= ((b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u)) << (4 * j);
+                        if (out_signed) S |= (__float_as_uint(y) >> 31) << (4 * j + 3);
+                    }
+                    wds[h] = codes8_b4(J, S, ep.out.k);
+                }
+            } else {
+                // 4-bit output codes with per-channel parameters, residual or extra outputs
+#pragma unroll
+                for (int h = 0; h < 2; h++) {
+                    uint32_t J = 0u, S = 0u;
+#pragma unroll 1
+                    for (int j = 0; j < 8; j++) {
+                        const int64_t n = n0 + c + 8 * h + j;
+                        const float af = __uint_as_float(r[8 * h + j]) * acc_scale;
+                        if (mrow && n < N) {
+                            if (ep.acc_out) ep.acc_out[m * N + n] = __float2int_rn(af);
+                            float sc = sc_fixed;
+                            if (ep.scale) { sc = __ldg(ep.scale + n); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
+                            const float bi = ep.bias ? __ldg(ep.bias + n) : ep.bias0;
+                            float y = __fmaf_rn(sc, af, bi);
+                            if (ep.residual) {
+                                const int rcpw = 32 / ep.res_b;
+                                const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >>
+                                                     (ep.res_b * (int)(n % rcpw))) & ((1u << ep.res_b) - 1u);
+                                y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+                            }
+                            y = apply_act(y, ep.act);
+                            if (ep.y_out) ep.y_out[m * N + n] = y;
+                            const uint32_t u = __float_as_uint(y);
+                            J |= bucket7(ep.out.is_signed ? fabsf(y) : y, cx.t7) << (4 * j);
+                            S |= ((u >> 31) & (uint32_t)ep.out.is_signed) << (4 * j + 3);
+                        }
+                    }
+                    wds[h] = codes8_b4(J, S, ep.out.k);
+                }
+            }
+            const int64_t w0 = (n0 + c) >> 3;
+            if (mrow) {
+                if (w0 + 1 < ep.ldo) {
+                    *reinterpret_cast<uint2*>(ep.codes_out + m * ep.ldo + w0) = make_uint2(wds[0], wds[1]);
+                } else if (w0 < ep.ldo) {
+                    ep.codes_out[m * ep.ldo + w0] = wds[0];
+                }
+            }
+        }
+    }
+}
+
+// Bounded wait of the MMA thread for its own last commit before TMEM is
+// freed (also on the abort path).
+__device__ __forceinline__ void ws_drain(uint64_t* drain, volatile int* err)
+{
+    mma_commit(drain);
+    volatile int no_abort = 0;
+    if (!wait_or_abort(drain, 0u, &no_abort)) *err = 1;
+}
+
+// ------------------------------------------------------------- host side
+
+int pick_bn(int64_t N, int out_cpw);          // N-tile width (esb_gemm.cu)
+int max_dyn_smem();                           // opt-in shared memory per block
+EpiParams make_epi(const GemmOutputs& o);     // epilogue parameters of a call
+
+// Stride-1 convolution from a decoded input halo (esb_conv_halo.cu).  Returns
+// false, launching nothing, when the shape does not suit it (stride != 1,
+// A not 4-bit, rows wider than 128 - pad, too little of the tile used, or
+// too little shared memory); otherwise launches and stores the launch
+// status in *err.  BN is the preferred N-tile width; a smaller one is used
+// when the resident filters would not fit.
+bool conv_halo_ok(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int kx, int out_cpw);
+bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, const OpFmt& fa,
+                      const uint32_t* W, int64_t ldw, const OpFmt& fb, int BN, const EpiParams& ep, cudaStream_t st,
+                      cudaError_t* err);
+
+}  // namespace esb

@@ -90,6 +90,7 @@ SIGNATURES = {
     "esb_dequant": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _P, _I64, _P]),
     "esb_gemm": (_I32, [_I64, _I64, _I64, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
     "esb_conv2d_nhwc": (_I32, [_P, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
+    "esb_conv2d_kernel": (_I32, [_P, _I64, esb_format, esb_format, _I32, _P]),
     "esb_maxpool_nhwc": (_I32, [_P, _I64, esb_format] + [_I32] * 7 + [_P, _I64, _P]),
     "esb_avgpool_nhwc": (_I32, [_P, _I64, esb_format, _I32, _I32, _I32, _F32, _F32, esb_format, _I32, _P, _P, _I64,
                                 _P]),
@@ -345,6 +346,19 @@ def esb_conv2d_nhwc(X: torch.Tensor, fx: Fmt, W: torch.Tensor, fw: Fmt, n: int, 
                                  ctypes.byref(epc) if epc is not None else None,
                                  _ptr(acc), _ptr(y), _ptr(codes), ldo, _stream(stream)), "esb_conv2d_nhwc")
     return acc, y, codes
+
+
+ESB_CONV_KERNEL_HALO, ESB_CONV_KERNEL_IM2COL, ESB_CONV_KERNEL_STREAMED, ESB_CONV_KERNEL_DEPTHWISE = 1, 2, 3, 4
+
+
+def esb_conv2d_kernel(n: int, h: int, w: int, c: int, cout: int, r: int, s: int, stride: int, pad: int,
+                      fx: Fmt, fw: Fmt, out_b: int = 4, groups: int = 1, ldx: Optional[int] = None) -> int:
+    """Which kernel esb_conv2d_nhwc runs for this convolution (ESB_CONV_KERNEL_*)."""
+    d = esb_conv_desc(n, h, w, c, cout, r, s, stride, pad, groups)
+    out = ctypes.c_int32(0)
+    _check(lib().esb_conv2d_kernel(ctypes.byref(d), esb_row_words(c, fx.b) if ldx is None else ldx, fx.c(), fw.c(),
+                                   out_b, ctypes.byref(out)), "esb_conv2d_kernel")
+    return int(out.value)
 
 
 def esb_maxpool_nhwc(X: torch.Tensor, f: Fmt, n: int, h: int, w: int, c: int, win: int = 3, stride: int = 2,

@@ -159,9 +159,9 @@ CONV_CASES = [
 ]
 
 
-@pytest.mark.parametrize("n,h,w,c,cout,r,s,stride,pad,fx,fw", CONV_CASES)
-def test_conv_matches_oracle(n, h, w, c, cout, r, s, stride, pad, fx, fw):
-    x = synth.half_normal((n * h * w, c), seed=h * 3 + c).numpy()
+def check_conv(n, h, w, c, cout, r, s, stride, pad, fx, fw):
+    x = synth.half_normal((n * h * w, c), seed=h * 3 + c).numpy() if not fx[2] else \
+        synth.normal((n * h * w, c), seed=h * 3 + c).numpy()
     wt = synth.he_normal((cout * r * s, c), fan_in=r * s * c, seed=cout + r).numpy()
     ldx = esb.esb_row_words(c, fx[0])
     X, ax = projected_packed(x, fx, 0)
@@ -178,6 +178,71 @@ def test_conv_matches_oracle(n, h, w, c, cout, r, s, stride, pad, fx, fw):
     yo, co = o.epilogue(acc_o, np.full(cout, s0, np.float32), np.zeros(cout, np.float32), 1, 0.7, fo)
     assert np.array_equal(y.cpu().numpy(), yo)
     assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
+@pytest.mark.parametrize("n,h,w,c,cout,r,s,stride,pad,fx,fw", CONV_CASES)
+def test_conv_matches_oracle(n, h, w, c, cout, r, s, stride, pad, fx, fw):
+    check_conv(n, h, w, c, cout, r, s, stride, pad, fx, fw)
+
+
+HALO_CASES = [
+    # n, h, w, c, cout, r, s, pad, fx, fw  (stride 1, 4-bit activations)
+    (2, 56, 56, 64, 64, 3, 3, 1, (4, 2, False), (4, 2, True)),        # ResNet18 layer-1 3x3 shape
+    (2, 28, 28, 128, 128, 3, 3, 1, (4, 2, False), (4, 2, True)),      # layer-2 shape: 4 pieces per pixel
+    (2, 14, 14, 256, 256, 3, 3, 1, (4, 2, False), (4, 2, True)),      # layer-3 shape: 2 channel blocks, 2 N-tiles
+    (3, 15, 30, 40, 48, 3, 3, 1, (4, 2, False), (4, 2, True)),        # channel padding codes, last tile ragged
+    (2, 12, 28, 64, 32, 5, 5, 2, (4, 1, False), (4, 1, True)),        # 5x5, pad 2
+    (2, 16, 31, 96, 80, 1, 1, 0, (4, 2, False), (4, 2, True)),        # 1x1: 3 pieces per pixel, N tail
+    (2, 18, 60, 64, 64, 3, 3, 0, (4, 2, False), (4, 2, True)),        # no padding: Q = w - 2
+    (2, 20, 24, 64, 64, 3, 3, 1, (4, 2, True), (4, 1, True)),         # signed activations
+    (1, 14, 14, 320, 64, 3, 3, 1, (4, 2, False), (4, 2, True)),       # partial last channel block
+    (1, 6, 63, 64, 64, 3, 3, 1, (4, 3, False), (4, 3, True)),         # w + pad = slot pitch
+    (1, 5, 100, 32, 64, 3, 3, 1, (4, 0, False), (4, 0, True)),        # pitch 128: one output row per tile
+]
+
+
+@pytest.mark.parametrize("n,h,w,c,cout,r,s,pad,fx,fw", HALO_CASES)
+def test_conv_halo_matches_oracle(n, h, w, c, cout, r, s, pad, fx, fw):
+    assert esb.esb_conv2d_kernel(n, h, w, c, cout, r, s, 1, pad, esb.Fmt(*fx), esb.Fmt(*fw),
+                                 out_b=fx[0]) == esb.ESB_CONV_KERNEL_HALO
+    check_conv(n, h, w, c, cout, r, s, 1, pad, fx, fw)
+
+
+def test_conv_kernel_choice():
+    f4, f6 = esb.Fmt(4, 2), esb.Fmt(6, 3)
+    k = esb.esb_conv2d_kernel
+    assert k(32, 56, 56, 64, 64, 3, 3, 1, 1, f4, f4) == esb.ESB_CONV_KERNEL_HALO
+    assert k(2, 7, 7, 512, 512, 3, 3, 1, 1, f4, f4) != esb.ESB_CONV_KERNEL_HALO      # 38 % of a tile used
+    assert k(2, 56, 56, 64, 128, 3, 3, 2, 1, f4, f4) != esb.ESB_CONV_KERNEL_HALO     # stride 2
+    assert k(2, 10, 10, 64, 64, 3, 3, 1, 1, f6, f6) != esb.ESB_CONV_KERNEL_HALO      # 6-bit activations
+    assert k(2, 10, 10, 64, 64, 3, 3, 1, 1, f4, f4, groups=64) == esb.ESB_CONV_KERNEL_DEPTHWISE
+
+
+def test_conv_full_size_sampled_rows():
+    # The timed workload at full size (batch 32, 56x56x64 -> 64, 3x3), in
+    # the launch configuration the benchmark times; output rows of a few
+    # images checked against the oracle.
+    n, h, w, c, cout = 32, 56, 56, 64, 64
+    fu, fs = (4, 2, False), (4, 2, True)
+    x = synth.half_normal((n * h * w, c), seed=7).numpy()
+    wt = synth.he_normal((cout * 9, c), fan_in=576, seed=8).numpy()
+    X, ax = projected_packed(x, fu, 0)
+    W, aw = projected_packed(wt, fs, 0)
+    s0 = esb.default_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2))
+    ep = esb.Epilogue(scale0=s0, act=esb.ESB_ACT_RELU, alpha_out=0.7, fmt_out=esb.Fmt(4, 2, False))
+    acc, _, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fu), dev_i32(W), esb.Fmt(*fs), n, h, w, c, cout, 3, 3,
+                                        1, 1, ep=ep, want_acc=True, want_codes=True)
+    acc = acc.cpu().numpy().astype(np.int64).reshape(n, h, w, cout)
+    codes = u32(codes).reshape(n, h, w, -1)
+    for img in (0, 13, 31):
+        for (p0, p1) in ((0, 3), (27, 29), (53, 56)):
+            ao = o.conv2d_rows_i64(X.reshape(n, h, w, -1)[img:img + 1], fu[:2], W.reshape(cout, 3, 3, -1), fs[:2],
+                                   1, h, w, c, cout, 3, 3, 1, 1, p0, p1)[0]
+            assert np.array_equal(acc[img, p0:p1], ao)
+            _, co = o.epilogue(ao.reshape(-1, cout), np.full(cout, s0, np.float32), np.zeros(cout, np.float32), 1,
+                               0.7, (4, 2, False))
+            assert np.array_equal(codes[img, p0:p1].reshape(-1, codes.shape[-1]),
+                                  o.pack(co, 4, 2, ld_words=codes.shape[-1]))
 
 
 def test_conv_dequant_scale_from_device_alphas():
