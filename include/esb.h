@@ -54,7 +54,9 @@ typedef enum esb_status {
     ESB_ERR_RANGE = 3,        /* an exactness bound (int32 / fp32 accumulation) would be exceeded */
     ESB_ERR_ALIGN = 4,        /* a pointer or stride violates the stated alignment */
     ESB_ERR_CUDA = 5,         /* a CUDA runtime call or launch failed */
-    ESB_ERR_TIMEOUT = 6       /* (device status only) a bounded pipeline wait gave up */
+    ESB_ERR_TIMEOUT = 6,      /* (device status only) a bounded pipeline wait gave up */
+    ESB_ERR_INTERNAL = 7      /* (device status only) a kernel found its shared-memory
+                                 allocation smaller than its layout and did no work */
 } esb_status;
 
 typedef struct esb_format {

@@ -117,6 +117,7 @@ const char* esb_status_string(int32_t s)
     case ESB_ERR_ALIGN: return "misaligned pointer or stride";
     case ESB_ERR_CUDA: return "CUDA error";
     case ESB_ERR_TIMEOUT: return "device pipeline wait timed out";
+    case ESB_ERR_INTERNAL: return "kernel launch configuration inconsistent (no work done)";
     default: return "unknown status";
     }
 }

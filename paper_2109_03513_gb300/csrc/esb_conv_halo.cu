@@ -45,6 +45,31 @@ struct HaloGeom {
     int stage_bytes;     // planes of one channel block (<= 8 planes)
 };
 
+// The MMAs of one stage (channel block) with every offset a compile-time
+// constant: slot pitch WS, an R x S filter, UT K steps of 32 codes per tap
+// of which this block holds PAIRS, N-tile BN.  Straight-line issue, nothing
+// but the tcgen05.mma between two MMAs.
+template <int WS, int R, int S, int UT, int PAIRS, int BN>
+__device__ __forceinline__ void halo_mma_fixed(uint32_t d, uint32_t a_st, uint32_t b_blk, uint32_t idesc,
+                                               uint32_t& acc)
+{
+    constexpr int NS = 128 + (R - 1) * WS + S - 1;
+    constexpr uint32_t PB = NS * 16;
+    const uint64_t a_desc = smem_desc_noswz(a_st, PB, 128u);
+    const uint64_t b_desc = smem_desc_sw128(b_blk);
+#pragma unroll
+    for (int t = 0; t < R * S; t++) {
+#pragma unroll
+        for (int j = 0; j < PAIRS; j++) {
+            const uint32_t ao = (uint32_t)((((t / S) * WS + (t % S)) * 16 + 2 * j * (int)PB) >> 4);
+            const int kq = t * UT + j;
+            const uint32_t bo = (uint32_t)(((kq >> 2) * BN * 128 + (kq & 3) * 32) >> 4);
+            mma_f8f6f4(d, a_desc + ao, b_desc + bo, idesc, acc);
+            acc = 1u;
+        }
+    }
+}
+
 // Producer: decode one channel block of one tile's halo into stage st.
 // Lane l owns slots l, l + 32, ...; each slot takes NPC 16-byte pieces
 // (4 words = two 16-code chunks each) of its pixel.  The pieces of up to
@@ -144,6 +169,11 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
     const bool split = (half_cols % 16 == 0) && (half_cols % ep.out_cpw == 0);
     const int epi_warps = split ? 8 : 4;
     const int cbs = g.cblocks;
+    // the layout above must fit the dynamic allocation (uniform for the CTA)
+    if ((uintptr_t)(reinterpret_cast<const volatile uint8_t*>(err) + 4 - smem_raw) > dynamic_smem_bytes()) {
+        if (tid == 0) record_status(ep.status, ESB_ERR_INTERNAL);
+        return;
+    }
 
     if (tid == 0) {
         for (int s = 0; s < stages; s++) {
@@ -185,31 +215,49 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
         }
     } else if (warp == kWsMmaWarp) {
         // ---------------------------------------------- MMA issue
+        // Common geometries issue straight-line MMAs with constant offsets
+        // (halo_mma_fixed); others compute the offsets in the loop.
+        // Descriptors never come from shared memory: the tensor core's own
+        // operand reads keep it close to saturated.
         if (lane == 0) {
             const uint32_t idesc = idesc_e4m3_f32(BN);
             const uint32_t b_base = smem_u32(sB), a_base = smem_u32(sA);
-            const int ctap = g.ldx * 8;                        // codes per tap
             const int ws = 1 << g.lws;
+            const int units_tap = g.ldx >> 2;                  // 32-code K steps per tap
+            const bool r3 = g.R == 3 && g.S == 3;
             int64_t it = 0;
             for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
                 const int a = (int)(ti & 1);
                 if (!wait_or_abort(&tempty[a], (uint32_t)((ti >> 1) & 1) ^ 1u, err)) { *err = 1; break; }
                 tc_fence_after();
                 const uint32_t d = tmem_base + (uint32_t)(a * BN);
+                uint32_t acc = 0u;
                 for (int cb = 0; cb < cbs; cb++, it++) {
                     const int s = (int)(it % stages);
                     if (!wait_or_abort(&full[s], (uint32_t)((it / stages) & 1), err)) { *err = 1; break; }
                     tc_fence_after();
-                    const uint32_t a0 = a_base + (uint32_t)(s * g.stage_bytes);
-                    const int pairs = min(16, g.ldx - cb * 16) >> 2;   // K = 32 steps in this block
-                    for (int t = 0; t < g.R * g.S; t++) {
-                        const int r = t / g.S, sx = t - r * g.S;
-                        const uint32_t at = a0 + (uint32_t)((r * ws + sx) * 16);
-                        for (int j = 0; j < pairs; j++) {
-                            const int k0 = t * ctap + cb * 128 + 32 * j;
-                            const uint32_t bb = b_base + (uint32_t)((k0 >> 7) * BN * kBK + ((k0 & 127) >> 5) * 32);
-                            mma_f8f6f4(d, smem_desc_noswz(at + (uint32_t)(2 * j * g.pb), (uint32_t)g.pb, 128u),
-                                       smem_desc_sw128(bb), idesc, (cb > 0 || t > 0 || j > 0) ? 1u : 0u);
+                    const uint32_t a_st = a_base + (uint32_t)(s * g.stage_bytes);
+                    const uint32_t b_blk = b_base + (uint32_t)(cb * BN * kBK);   // block cb: 4 K steps on
+                    const int pairs = min(16, g.ldx - cb * 16) >> 2;
+                    if (r3 && ws == 64 && units_tap == 2 && BN == 64) {           // 56 x 56 x 64
+                        halo_mma_fixed<64, 3, 3, 2, 2, 64>(d, a_st, b_blk, idesc, acc);
+                    } else if (r3 && ws == 32 && units_tap == 4 && BN == 128) {   // 28 x 28 x 128
+                        halo_mma_fixed<32, 3, 3, 4, 4, 128>(d, a_st, b_blk, idesc, acc);
+                    } else if (r3 && ws == 16 && units_tap == 8 && pairs == 4 && BN == 64) {   // 14 x 14 x 256
+                        halo_mma_fixed<16, 3, 3, 8, 4, 64>(d, a_st, b_blk, idesc, acc);
+                    } else {
+                        for (int r = 0; r < g.R; r++) {
+                            for (int sx = 0; sx < g.S; sx++) {
+                                const uint32_t at = a_st + (uint32_t)((r * ws + sx) * 16);
+                                const int kq0 = (r * g.S + sx) * units_tap + cb * 4;
+                                for (int j = 0; j < pairs; j++) {
+                                    const int kq = kq0 + j;
+                                    const uint32_t bb = b_base + (uint32_t)((kq >> 2) * BN * kBK + (kq & 3) * 32);
+                                    mma_f8f6f4(d, smem_desc_noswz(at + (uint32_t)(2 * j * g.pb), (uint32_t)g.pb, 128u),
+                                               smem_desc_sw128(bb), idesc, acc);
+                                    acc = 1u;
+                                }
+                            }
                         }
                     }
                     mma_commit(&empty[s]);
@@ -221,15 +269,15 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
         }
     } else if (warp < epi_warps) {
         // ---------------------------------------------- epilogue
-        const int64_t ctas = ctas_per_n, first = cta_in_n;
-        const HaloGeom gg = g;
+        const int ctas = (int)ctas_per_n, first = (int)cta_in_n;   // tile counts fit in 32 bits (host check)
+        const int tpi = g.tpi, rows_out = g.rows_out, lws = g.lws, P = g.P, Q = g.Q;
         auto rows = [=](int64_t ti, int row, int64_t& m) -> bool {
-            const int64_t T = first + ti * ctas;
-            const int64_t nimg = T / gg.tpi;
-            const int p = (int)(T - nimg * gg.tpi) * gg.rows_out + (row >> gg.lws);
-            const int q = row & ((1 << gg.lws) - 1);
-            m = (nimg * gg.P + p) * gg.Q + q;
-            return q < gg.Q && p < gg.P;
+            const int T = first + (int)ti * ctas;
+            const int nimg = T / tpi;
+            const int p = (T - nimg * tpi) * rows_out + (row >> lws);
+            const int q = row & ((1 << lws) - 1);
+            m = ((int64_t)nimg * P + p) * Q + q;
+            return q < Q && p < P;
         };
         ws_epilogue(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
                     warp, lane);
@@ -290,6 +338,7 @@ static bool halo_plan(const esb_conv_desc& d, int P, int Q, int64_t ldx, const O
     g.cblocks = (int)((ldx + 15) / 16);
     const int planes = (int)(ldx >= 16 ? 8 : ldx / 2);
     g.stage_bytes = ((planes * g.pb + 127) / 128) * 128;
+    if ((int64_t)d.n * g.tpi >= (1ll << 30)) return false;
     const int st_smem = halo_static_smem(err);
     if (st_smem < 0) return false;
     const int maxs = max_dyn_smem() - st_smem;
@@ -324,6 +373,10 @@ bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, i
 {
     HaloPlan hp;
     if (!halo_plan(d, P, Q, ldx, fa, BN, ep.out_cpw, &hp, err)) return *err != cudaSuccess;
+    if (hp.smem <= 0 || hp.smem > max_dyn_smem() - halo_static_smem(err)) {
+        *err = cudaErrorInvalidConfiguration;
+        return true;
+    }
     hp.g.X = X;
     static bool configured = false;
     if (!configured) {

@@ -337,6 +337,11 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
     const int half_cols = BN / 2;
     const bool split = (half_cols % 16 == 0) && (half_cols % ep.out_cpw == 0);
     const int epi_warps = split ? 8 : 4;
+    // the layout above must fit the dynamic allocation (uniform for the CTA)
+    if ((uintptr_t)(reinterpret_cast<const volatile uint8_t*>(err) + 4 - smem_raw) > dynamic_smem_bytes()) {
+        if (tid == 0) record_status(ep.status, ESB_ERR_INTERNAL);
+        return;
+    }
 
     if (tid == 0) {
         for (int s = 0; s < stages; s++) {
@@ -552,6 +557,14 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
     return true;
 }
 
+// Bound + 2 on |acc| for the epilogue's FMA-pipe requantisation, or 0 when
+// K max|I_A| max|I_B| reaches 2^20.
+static float acc_fma_limit(int64_t K, int ba, int ka, int bb, int kb)
+{
+    const double bound = (double)K * fmt_max_image(ba, ka) * fmt_max_image(bb, kb);
+    return bound < 1048576.0 ? (float)(bound + 2.0) : 0.0f;
+}
+
 EpiParams make_epi(const GemmOutputs& o)
 {
     EpiParams ep;
@@ -580,6 +593,11 @@ EpiParams make_epi(const GemmOutputs& o)
     ep.y_out = o.y_out;
     ep.codes_out = o.codes_out;
     ep.ldo = o.ldo;
+    {
+        const uintptr_t pa = reinterpret_cast<uintptr_t>(o.codes_out);
+        ep.codes_vec = ((pa & 15u) == 0 && (o.ldo & 3) == 0) ? 4 : ((pa & 7u) == 0 && (o.ldo & 1) == 0) ? 2 : 1;
+    }
+    ep.acc_lim = 0.0f;
     ep.status = device_status_ptr();
     return ep;
 }
@@ -589,6 +607,7 @@ cudaError_t launch_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int6
 {
     EpiParams ep = make_epi(o);
     ep.dq_pow2 = ldexpf(1.0f, -(ka + kb));
+    ep.acc_lim = acc_fma_limit(K, ba, ka, bb, kb);
     const int BN = pick_bn(N, ep.out_cpw);
     RowsSrc a{A, lda, M};
     RowsSrc b{B, ldb, N};
@@ -617,6 +636,7 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
 {
     EpiParams ep = make_epi(o);
     ep.dq_pow2 = ldexpf(1.0f, -(kx + kw));
+    ep.acc_lim = acc_fma_limit((int64_t)d.r * d.s * ldx * (32 / bx), bx, kx, bw, kw);
     const int64_t M = (int64_t)d.n * P * Q;
     const int64_t N = d.cout;
     const int64_t K = (int64_t)d.r * d.s * ldx * (32 / bx);

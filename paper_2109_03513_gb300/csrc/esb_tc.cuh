@@ -128,6 +128,8 @@ struct EpiParams {
     float* y_out;
     uint32_t* codes_out;
     int64_t ldo;
+    int codes_vec;            // widest safe store of code words: 1, 2 or 4 (pointer and ldo alignment)
+    float acc_lim;            // K max|I_A| max|I_B| + 2 when that bound is below 2^20, else 0
     int* status;
 };
 
@@ -185,18 +187,19 @@ __device__ __forceinline__ uint32_t epi_element(const EpiParams& ep, const EpiCt
 }
 
 // Wait on an mbarrier phase with a wall-clock bound and an abort flag
-// raised by another role of the CTA.
+// raised by another role of the CTA.  The waiting thread is parked by the
+// hardware between tries (suspend hint), so a waiting warp takes no issue
+// slots from the working warps of its sub-partition.
+constexpr uint32_t kSuspendHintNs = 20000;
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* err)
 {
     const uint32_t a = smem_u32(bar);
     if (mbar_try_wait(a, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
-    for (uint32_t it = 1;; ++it) {
-        if (mbar_try_wait(a, parity)) return true;
-        if ((it & 255u) == 0u) {
-            if (*err) return false;
-            if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
-        }
+    for (;;) {
+        if (mbar_try_wait_hint(a, parity, kSuspendHintNs)) return true;
+        if (*err) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
     }
 }
 
@@ -305,6 +308,66 @@ static __device__ __noinline__ void epi_chunk_any(const EpiParams* __restrict__ 
 }
 
 
+// Lean-path threshold on the raw accumulator.  For a scale sc > 0,
+// y(a) = fma(sc, a, b) is non-decreasing in the integer accumulator a
+// (|a| < 2^24, checked on the host), and so is the activation of y; an
+// output code's bucket counts the thresholds T_j (all > 0) at or below
+// act(y).  For ReLU and no activation, act(y) >= T  <=>  y >= T (T > 0);
+// ReLU6 never reaches a T above 6.  Returns A * rs for the smallest
+// integer A with y(A) >= T (raw = a * rs exactly), +inf if none, -inf if
+// every accumulator qualifies.  26 bounded bisection steps on integers.
+__device__ __forceinline__ float acc_raw_threshold(float sc, float b, float T, int act, float rs)
+{
+    if (act == ESB_ACT_RELU6 && T > 6.0f) return __int_as_float(0x7f800000);
+    const int lim = 1 << 24;
+    if (!(__fmaf_rn(sc, (float)lim, b) >= T)) return __int_as_float(0x7f800000);
+    if (__fmaf_rn(sc, (float)-lim, b) >= T) return __int_as_float(0xff800000);
+    int lo = -lim, hi = lim;                           // y(lo) < T <= y(hi)
+    for (int it = 0; it < 32 && hi - lo > 1; it++) {
+        const int mid = lo + ((hi - lo) >> 1);
+        if (__fmaf_rn(sc, (float)mid, b) >= T) hi = mid; else lo = mid;
+    }
+    return (float)hi * rs;
+}
+
+struct Raw8 { uint32_t r[8]; };
+
+// One packed word of 4-bit output codes (8 columns from n_first) with
+// per-channel scale/bias, residual or extra outputs; out of line so the
+// caller's accumulator registers stay in registers.
+static __device__ __noinline__ uint32_t epi_word_b4(const EpiParams* __restrict__ sep, const EpiCtx* __restrict__ scx,
+                                                    Raw8 v, float acc_scale, float sc_fixed, int64_t m, bool mrow,
+                                                    int64_t n_first, int64_t N)
+{
+    const EpiParams& ep = *sep;
+    const EpiCtx& cx = *scx;
+    uint32_t J = 0u, S = 0u;
+#pragma unroll 1
+    for (int j = 0; j < 8; j++) {
+        const int64_t n = n_first + j;
+        const float af = __uint_as_float(v.r[j]) * acc_scale;
+        if (mrow && n < N) {
+            if (ep.acc_out) ep.acc_out[m * N + n] = __float2int_rn(af);
+            float sc = sc_fixed;
+            if (ep.scale) { sc = __ldg(ep.scale + n); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
+            const float bi = ep.bias ? __ldg(ep.bias + n) : ep.bias0;
+            float y = __fmaf_rn(sc, af, bi);
+            if (ep.residual) {
+                const int rcpw = 32 / ep.res_b;
+                const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >> (ep.res_b * (int)(n % rcpw))) &
+                                    ((1u << ep.res_b) - 1u);
+                y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+            }
+            y = apply_act(y, ep.act);
+            if (ep.y_out) ep.y_out[m * N + n] = y;
+            const uint32_t u = __float_as_uint(y);
+            J |= bucket7(ep.out.is_signed ? fabsf(y) : y, cx.t7) << (4 * j);
+            S |= ((u >> 31) & (uint32_t)ep.out.is_signed) << (4 * j + 3);
+        }
+    }
+    return codes8_b4(J, S, ep.out.k);
+}
+
 // ------------------------------------ roles of the warp-specialised kernels
 
 // Setup role (warps 0 .. kWsProdWarp0 - 1, while the producers already load
@@ -373,18 +436,48 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
     const int c_lo = split ? (warp >> 2) * half_cols : 0;
     const int c_hi = split ? c_lo + half_cols : BN;
     const EpiCtx cx = make_epi_ctx(ep, thr);
-    if (warp == 0 && lane == 0) { sh_ep = ep; sh_cx = cx; }
-    asm volatile("bar.sync 2, %0;" ::"r"(epi_warps * 32) : "memory");   // exactly the epilogue warps in use
-    const int cpw = ep.out_cpw;
     const bool swar = ep.codes_out && ep.out.b == 4;
-    const float T0 = cx.t7.t[0], T1 = cx.t7.t[1], T2 = cx.t7.t[2], T3 = cx.t7.t[3], T4 = cx.t7.t[4],
-                T5 = cx.t7.t[5], T6 = cx.t7.t[6];
     const float sc_fixed = ep.scale ? 0.0f : (cx.dq ? __fmul_rn(ep.scale0, cx.dqs) : ep.scale0);
     const float sc_lean = sc_fixed * acc_scale;
     const bool out_signed = ep.out.is_signed != 0;
     // the lean path needs every column of the chunk inside N and a finite folded scale
     const bool lean_ok = swar && !ep.scale && !ep.bias && !ep.residual && !ep.acc_out && !ep.y_out &&
                          isfinite(sc_lean) && (sc_lean != 0.0f || sc_fixed == 0.0f);
+    // With a positive scalar scale the requantised bucket is a monotone step
+    // function of the exact integer accumulator, so the 7 thresholds on y
+    // become 7 thresholds on the raw TMEM value (acc_raw_threshold, one lane
+    // each); a signed output without activation keeps the general lean path.
+    const bool raw_ok = lean_ok && sc_fixed > 0.0f && (!out_signed || ep.act != ESB_ACT_NONE);
+    __shared__ float sh_raw[8];
+    if (warp == 0) {
+        if (lane == 0) { sh_ep = ep; sh_cx = cx; }
+        if (raw_ok && lane < 7) sh_raw[lane] = acc_raw_threshold(sc_fixed, ep.bias0, thr[lane], ep.act, 1.0f / acc_scale);
+    }
+    asm volatile("bar.sync 2, %0;" ::"r"(epi_warps * 32) : "memory");   // exactly the epilogue warps in use
+    const int cpw = ep.out_cpw;
+    const float T0 = cx.t7.t[0], T1 = cx.t7.t[1], T2 = cx.t7.t[2], T3 = cx.t7.t[3], T4 = cx.t7.t[4],
+                T5 = cx.t7.t[5], T6 = cx.t7.t[6];
+    float R0 = 0.0f, R1 = 0.0f, R2 = 0.0f, R3 = 0.0f, R4 = 0.0f, R5 = 0.0f, R6 = 0.0f;
+    if (raw_ok) {
+        R0 = sh_raw[0]; R1 = sh_raw[1]; R2 = sh_raw[2]; R3 = sh_raw[3]; R4 = sh_raw[4]; R5 = sh_raw[5]; R6 = sh_raw[6];
+    }
+    // The same search on the FMA pipe when |acc| <= L - 2 < 2^20 (the ALU
+    // pipe is the epilogue's bottleneck): with A_j = R_j / rs clamped to
+    // [-L, L] and k_j = 1 - 2 A_j, sat(fma(raw, 2/rs, k_j)) = sat(2 acc -
+    // 2 A_j + 1) is exactly [acc >= A_j] (an odd integer below 2^24 before
+    // the clamp to [0, 1]); the next threshold is chosen by fmas with those
+    // 0/1 factors, and the bucket bits are packed by fmas with powers of 16
+    // (every intermediate an integer below 2^24: exact).
+    const bool fma_ok = raw_ok && ep.acc_lim > 0.0f;
+    float cK = 0.0f, K0 = 0.0f, K1 = 0.0f, K3 = 0.0f, D51 = 0.0f, D20 = 0.0f, D40 = 0.0f, E3 = 0.0f;
+    if (fma_ok) {
+        const float L = ep.acc_lim;
+        auto kf = [&](float R) { return 1.0f - 2.0f * fminf(fmaxf(R * acc_scale, -L), L); };
+        const float k0 = kf(R0), k1 = kf(R1), k2 = kf(R2), k3 = kf(R3), k4 = kf(R4), k5 = kf(R5), k6 = kf(R6);
+        cK = 2.0f * acc_scale;
+        K0 = k0; K1 = k1; K3 = k3;
+        D51 = k5 - k1; D20 = k2 - k0; D40 = k4 - k0; E3 = (k6 - k4) - (k2 - k0);
+    }
     for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
         const int a = (int)(ti & 1);
         if (!wait_or_abort(&tfull[a], (uint32_t)((ti >> 1) & 1), err)) { *err = 1; break; }
@@ -404,24 +497,61 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 }
                 continue;
             }
-            uint32_t r[16];
-            tmem_ld16(taddr + (uint32_t)c, r);
-            const bool lean = lean_ok && (n0 + c + 16 <= N);
-            if (c + 16 >= c_hi) {                     // every column of this warp is in registers
+            // 4-bit output codes: 32 (or 16) columns per TMEM load
+            const int nc = (c + 32 <= c_hi) ? 32 : 16;
+            uint32_t r[32];
+            if (nc == 32) {
+                tmem_ld32(taddr + (uint32_t)c, r);
+            } else {
+                tmem_ld16(taddr + (uint32_t)c, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+            }
+            if (c + nc >= c_hi) {                     // every column of this warp is in registers
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&tempty[a]);
             }
-            uint32_t wds[2];
-            if (lean) {
-                // 4-bit output codes only, scalar scale/bias, no residual:
-                // y = fma(scale * 2^(kA+kB+12), raw, bias) equals
-                // fma(scale, acc, bias) exactly (power-of-two scaling),
-                // then the bucket of y among the 7 thresholds, eight codes
-                // per word at once.
+            const bool lean = lean_ok && (n0 + c + nc <= N);
+            uint32_t wds[4];
 #pragma unroll
-                for (int h = 0; h < 2; h++) {
-                    uint32_t J = 0u, S = 0u;
+            for (int h = 0; h < 4; h++) {
+                if (h * 8 >= nc) break;
+                uint32_t J = 0u, S = 0u;
+                if (lean && fma_ok) {
+                    float jh[2];
+#pragma unroll
+                    for (int q = 0; q < 2; q++) {
+                        float jf = 0.0f;
+#pragma unroll
+                        for (int j = 3; j >= 0; j--) {
+                            const float v = __uint_as_float(r[8 * h + 4 * q + j]);
+                            const float b2 = __saturatef(__fmaf_rn(v, cK, K3));
+                            const float b1 = __saturatef(__fmaf_rn(v, cK, __fmaf_rn(b2, D51, K1)));
+                            const float t0 = __fmaf_rn(b1, __fmaf_rn(b2, E3, D20), __fmaf_rn(b2, D40, K0));
+                            const float b0 = __saturatef(__fmaf_rn(v, cK, t0));
+                            const float nb = __fmaf_rn(b2, 4.0f, __fmaf_rn(b1, 2.0f, b0));
+                            jf = __fmaf_rn(jf, 16.0f, nb);       // nibbles of elements 3..0, element 0 lowest
+                        }
+                        jh[q] = jf + 8388608.0f;                   // integer jf < 2^16 in the low mantissa bits
+                    }
+                    J = (__float_as_uint(jh[0]) & 0xffffu) | (__float_as_uint(jh[1]) << 16);
+                    wds[h] = codes8_b4(J, 0u, ep.out.k);
+                } else if (lean && raw_ok) {
+                    // bucket = number of raw thresholds <= raw accumulator
+#pragma unroll
+                    for (int j = 0; j < 8; j++) {
+                        const float v = __uint_as_float(r[8 * h + j]);
+                        const bool b2 = v >= R3;
+                        const bool b1 = v >= (b2 ? R5 : R1);
+                        const bool b0 = v >= (b2 ? (b1 ? R6 : R4) : (b1 ? R2 : R0));
+                        J |= ((b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u)) << (4 * j);
+                    }
+                    wds[h] = codes8_b4(J, 0u, ep.out.k);
+                } else if (lean) {
+                    // 4-bit output codes only, scalar scale/bias, no residual:
+                    // y = fma(scale * 2^(kA+kB+12), raw, bias) equals
+                    // fma(scale, acc, bias) exactly (power-of-two scaling),
+                    // then the bucket of y among the 7 thresholds, eight
+                    // codes per word at once.
 #pragma unroll
                     for (int j = 0; j < 8; j++) {
                         float y = __fmaf_rn(sc_lean, __uint_as_float(r[8 * h + j]), ep.bias0);
@@ -434,46 +564,29 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                         if (out_signed) S |= (__float_as_uint(y) >> 31) << (4 * j + 3);
                     }
                     wds[h] = codes8_b4(J, S, ep.out.k);
-                }
-            } else {
-                // 4-bit output codes with per-channel parameters, residual or extra outputs
+                } else {
+                    Raw8 v;
 #pragma unroll
-                for (int h = 0; h < 2; h++) {
-                    uint32_t J = 0u, S = 0u;
-#pragma unroll 1
-                    for (int j = 0; j < 8; j++) {
-                        const int64_t n = n0 + c + 8 * h + j;
-                        const float af = __uint_as_float(r[8 * h + j]) * acc_scale;
-                        if (mrow && n < N) {
-                            if (ep.acc_out) ep.acc_out[m * N + n] = __float2int_rn(af);
-                            float sc = sc_fixed;
-                            if (ep.scale) { sc = __ldg(ep.scale + n); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
-                            const float bi = ep.bias ? __ldg(ep.bias + n) : ep.bias0;
-                            float y = __fmaf_rn(sc, af, bi);
-                            if (ep.residual) {
-                                const int rcpw = 32 / ep.res_b;
-                                const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >>
-                                                     (ep.res_b * (int)(n % rcpw))) & ((1u << ep.res_b) - 1u);
-                                y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
-                            }
-                            y = apply_act(y, ep.act);
-                            if (ep.y_out) ep.y_out[m * N + n] = y;
-                            const uint32_t u = __float_as_uint(y);
-                            J |= bucket7(ep.out.is_signed ? fabsf(y) : y, cx.t7) << (4 * j);
-                            S |= ((u >> 31) & (uint32_t)ep.out.is_signed) << (4 * j + 3);
-                        }
-                    }
-                    wds[h] = codes8_b4(J, S, ep.out.k);
+                    for (int j = 0; j < 8; j++) v.r[j] = r[8 * h + j];
+                    wds[h] = epi_word_b4(&sh_ep, &sh_cx, v, acc_scale, sc_fixed, m, mrow, n0 + c + 8 * h, N);
                 }
             }
-            const int64_t w0 = (n0 + c) >> 3;
             if (mrow) {
-                if (w0 + 1 < ep.ldo) {
-                    *reinterpret_cast<uint2*>(ep.codes_out + m * ep.ldo + w0) = make_uint2(wds[0], wds[1]);
-                } else if (w0 < ep.ldo) {
-                    ep.codes_out[m * ep.ldo + w0] = wds[0];
+                // words w0 .. w0 + nc/8 - 1 of row m; vector stores only where
+                // the address is aligned and every word is inside the row
+                const int64_t w0 = (n0 + c) >> 3;
+                uint32_t* dst = ep.codes_out + m * ep.ldo + w0;
+                const int nw = nc >> 3;
+                if (nw == 4 && ep.codes_vec >= 4 && (w0 & 3) == 0 && w0 + 4 <= ep.ldo) {
+                    *reinterpret_cast<uint4*>(dst) = make_uint4(wds[0], wds[1], wds[2], wds[3]);
+                } else if (ep.codes_vec >= 2 && (w0 & 1) == 0 && w0 + nw <= ep.ldo) {
+                    for (int q = 0; q < nw; q += 2) *reinterpret_cast<uint2*>(dst + q) = make_uint2(wds[q], wds[q + 1]);
+                } else {
+                    for (int q = 0; q < nw; q++)
+                        if (w0 + q < ep.ldo) dst[q] = wds[q];
                 }
             }
+            c += nc - 16;                             // the loop adds the other 16
         }
     }
 }

@@ -24,6 +24,7 @@ ESB_ERR_RANGE = 3
 ESB_ERR_ALIGN = 4
 ESB_ERR_CUDA = 5
 ESB_ERR_TIMEOUT = 6
+ESB_ERR_INTERNAL = 7
 
 ESB_ROUND_HALF_AWAY = 0
 ESB_ROUND_HALF_EVEN = 1

@@ -146,6 +146,97 @@ def test_gemm_fused_epilogue_matches_oracle(M, N, K, act, fo, rnd, per_channel, 
     assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
 
 
+LEAN_CASES = [
+    # (act, fmt_out, bias0, scale factor): codes-only outputs with a scalar
+    # scale and bias -- the epilogue's requantisation-only path
+    (esb.ESB_ACT_RELU, (4, 2, False), 0.05, 1.0),
+    (esb.ESB_ACT_RELU, (4, 2, False), -0.3, 3.7),
+    (esb.ESB_ACT_NONE, (4, 2, False), 0.2, 1.0),
+    (esb.ESB_ACT_NONE, (4, 2, True), -0.1, 2.0),       # signed, no activation: sign per element
+    (esb.ESB_ACT_RELU6, (4, 0, False), 0.0, 40.0),      # thresholds above 6 are never reached
+    (esb.ESB_ACT_RELU6, (4, 1, True), 0.5, 9.0),
+    (esb.ESB_ACT_RELU, (4, 3, True), 0.0, 0.01),
+    (esb.ESB_ACT_RELU, (4, 2, False), 0.1, -1.0),      # negative scale
+    (esb.ESB_ACT_NONE, (4, 2, True), 0.0, 0.0),        # zero scale: every output is the bias
+]
+
+
+def lean_epilogue(fo, act, bias0, s):
+    return esb.Epilogue(scale0=float(s), bias0=bias0, act=act, alpha_out=0.173, fmt_out=esb.Fmt(*fo))
+
+
+@pytest.mark.parametrize("act,fo,bias0,sf", LEAN_CASES)
+def test_gemm_codes_only_epilogue(act, fo, bias0, sf):
+    M, N, K = 300, 64, 576
+    fa, fb = (4, 2, False), (4, 2, True)
+    A, aa = projected_packed(synth.half_normal((M, K), seed=M + 5).numpy(), fa, 0)
+    B, ab = projected_packed(synth.he_normal((N, K), fan_in=K, seed=N + 6).numpy(), fb, 0)
+    s = np.float32(esb.default_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2)) * sf)
+    _, _, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(*fa), dev_i32(B), esb.Fmt(*fb), K, ep=lean_epilogue(fo, act, bias0, s),
+                               want_acc=False, want_y=False, want_codes=True)
+    acc_o = o.gemm_i64(A, fa[:2], B, fb[:2], M, N, K)
+    _, co = o.epilogue(acc_o, np.full(N, s, np.float32), np.full(N, bias0, np.float32), act, 0.173, fo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
+@pytest.mark.parametrize("M,N,K,fab", [(200, 64, 4096, (6, 3)), (130, 96, 2000, (5, 2))])
+@pytest.mark.parametrize("act", [esb.ESB_ACT_RELU, esb.ESB_ACT_NONE])
+def test_gemm_codes_only_epilogue_large_accumulators(M, N, K, fab, act):
+    # K max|I_A| max|I_B| above 2^20: the requantisation compares raw
+    # accumulators on the ALU pipe instead of the FMA-pipe form
+    fa, fb = (fab[0], fab[1], False), (fab[0], fab[1], True)
+    A, aa = projected_packed(synth.half_normal((M, K), seed=K + 1).numpy(), fa, 0)
+    B, ab = projected_packed(synth.he_normal((N, K), fan_in=K, seed=K + 2).numpy(), fb, 0)
+    s = np.float32(esb.default_scale(aa, esb.Fmt(*fab), ab, esb.Fmt(*fab)))
+    fo = (4, 2, False)
+    _, _, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(*fa), dev_i32(B), esb.Fmt(*fb), K,
+                               ep=lean_epilogue(fo, act, -0.02, s), want_acc=False, want_codes=True)
+    acc_o = o.gemm_i64(A, fa[:2], B, fb[:2], M, N, K)
+    _, co = o.epilogue(acc_o, np.full(N, s, np.float32), np.full(N, -0.02, np.float32), act, 0.173, fo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
+@pytest.mark.parametrize("shape", [(2, 56, 56, 64, 64, 1), (2, 9, 7, 64, 64, 1), (2, 14, 14, 128, 256, 2)])
+@pytest.mark.parametrize("act,fo,bias0,sf", LEAN_CASES[:6])
+def test_conv_codes_only_epilogue(shape, act, fo, bias0, sf):
+    n, h, w, c, cout, stride = shape
+    fx, fw = (4, 2, False), (4, 2, True)
+    X, ax = projected_packed(synth.half_normal((n * h * w, c), seed=h + c).numpy(), fx, 0)
+    W, aw = projected_packed(synth.he_normal((cout * 9, c), fan_in=9 * c, seed=cout).numpy(), fw, 0)
+    s = np.float32(esb.default_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2)) * sf)
+    _, _, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fx), dev_i32(W), esb.Fmt(*fw), n, h, w, c, cout, 3, 3,
+                                      stride, 1, ep=lean_epilogue(fo, act, bias0, s), want_acc=False,
+                                      want_codes=True)
+    ldx = X.shape[1]
+    acc_o = o.conv2d_i64(X.reshape(n, h, w, ldx), fx[:2], W.reshape(cout, 3, 3, ldx), fw[:2], n, h, w, c, cout, 3, 3,
+                         stride, 1).reshape(-1, cout)
+    _, co = o.epilogue(acc_o, np.full(cout, s, np.float32), np.full(cout, bias0, np.float32), act, 0.173, fo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
+@pytest.mark.parametrize("ldo_extra,offset_words", [(1, 0), (2, 1), (3, 2), (0, 1)])
+def test_codes_store_alignment(ldo_extra, offset_words):
+    # output rows at any word stride and start (no 8/16-byte alignment)
+    n, h, w, c, cout = 2, 20, 24, 64, 64
+    fx, fw = (4, 2, False), (4, 2, True)
+    X, ax = projected_packed(synth.half_normal((n * h * w, c), seed=31).numpy(), fx, 0)
+    W, aw = projected_packed(synth.he_normal((cout * 9, c), fan_in=576, seed=32).numpy(), fw, 0)
+    s = np.float32(esb.default_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2)))
+    ldo = esb.esb_row_words(cout, 4) + ldo_extra
+    M = n * h * w
+    buf = torch.full((M * ldo + offset_words + 8,), -1, dtype=torch.int32, device="cuda")
+    out = buf[offset_words:offset_words + M * ldo].view(M, ldo)
+    esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fx), dev_i32(W), esb.Fmt(*fw), n, h, w, c, cout, 3, 3, 1, 1,
+                        ep=lean_epilogue((4, 2, False), esb.ESB_ACT_RELU, 0.0, s), want_acc=False, out_codes=out)
+    acc_o = o.conv2d_i64(X.reshape(n, h, w, -1), fx[:2], W.reshape(cout, 3, 3, -1), fw[:2], n, h, w, c, cout, 3, 3,
+                         1, 1).reshape(-1, cout)
+    _, co = o.epilogue(acc_o, np.full(cout, s, np.float32), np.zeros(cout, np.float32), 1, 0.173, (4, 2, False))
+    got = u32(out)
+    assert np.array_equal(got[:, :8], o.pack(co, 4, 2, ld_words=8))
+    b = u32(buf)
+    assert (b[:offset_words] == 0xFFFFFFFF).all() and (b[offset_words + M * ldo:] == 0xFFFFFFFF).all()
+
+
 CONV_CASES = [
     # n, h, w, c, cout, r, s, stride, pad, fx, fw
     (2, 9, 7, 64, 64, 3, 3, 1, 1, (4, 2, False), (4, 2, True)),
