@@ -159,10 +159,10 @@ size_t esb_calibrate_dda_workspace_bytes(int64_t n);
  *              alignment accepted)
  *   n          > 0
  *   workspace  [device] >= esb_calibrate_dda_workspace_bytes(n) bytes,
- *              8-byte aligned, contents ignored and overwritten
+ *              16-byte aligned, contents ignored and overwritten
  *   alpha_out  [device] 1 float written by the kernel (no host sync)
  *   stats_out  [device] 3 doubles {mean, sigma or rms, n}, or NULL
- * One memset of the workspace's ticket word and one kernel launch; the
+ * One memset of the workspace's ticket words and one kernel launch; the
  * reduction order is fixed, so results are bit-reproducible on a device.
  * Errors: INVALID_ARG, UNSUPPORTED (bad format), ALIGN (workspace), CUDA. */
 esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
@@ -225,7 +225,7 @@ esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx,
  * the tensor in L2 between the two passes.
  *   x          [device] rows x cols floats, contiguous (row stride cols)
  *   workspace  [device] >= esb_calibrate_dda_workspace_bytes(rows * cols),
- *              8-byte aligned, contents ignored
+ *              16-byte aligned, contents ignored
  *   alpha_out  [device] 1 float written with the alpha used
  *   stats_out  [device] 3 doubles {mean, sigma or rms, n}, or NULL
  *   codes      [device] rows x ldc words, as esb_project

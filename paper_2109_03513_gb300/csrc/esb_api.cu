@@ -149,7 +149,7 @@ esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f, void* work
     if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
     if (!x || n <= 0 || !workspace || !alpha_out) return ESB_ERR_INVALID_ARG;
     if (workspace_bytes < calibrate_workspace_bytes(n)) return ESB_ERR_INVALID_ARG;
-    if ((reinterpret_cast<uintptr_t>(workspace) & 7u) != 0) return ESB_ERR_ALIGN;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 15u) != 0) return ESB_ERR_ALIGN;
     double as = 0.0;
     alpha_star_cached(f.b, f.k, &as, nullptr);
     cudaError_t e = launch_calibrate(x, n, f.is_signed, as, workspace, alpha_out, stats_out,
@@ -193,7 +193,7 @@ esb_status esb_project_dda(const float* x, int64_t rows, int64_t cols, esb_forma
     if (rounding != ESB_ROUND_HALF_AWAY && rounding != ESB_ROUND_HALF_EVEN) return ESB_ERR_INVALID_ARG;
     if (!x || !workspace || !alpha_out || !codes) return ESB_ERR_INVALID_ARG;
     if (workspace_bytes < calibrate_workspace_bytes(rows * cols)) return ESB_ERR_INVALID_ARG;
-    if ((reinterpret_cast<uintptr_t>(workspace) & 7u) != 0) return ESB_ERR_ALIGN;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 15u) != 0) return ESB_ERR_ALIGN;
     double as = 0.0;
     alpha_star_cached(f.b, f.k, &as, nullptr);
     cudaError_t e = launch_calibrate_project(x, rows, cols, f.b, f.k, f.is_signed, rounding, as, workspace, alpha_out,

@@ -202,16 +202,20 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
         const int p = warp - kWsProdWarp0;
         const int nprod = stages < kWsProdWarps ? stages : kWsProdWarps;
         const int64_t total_it = (p < nprod) ? my_tiles * cbs : 0;
+        // stage s and its phase ph follow it incrementally (no division in
+        // the loop): it advances by nprod <= stages, so s wraps at most once
+        int s = p;
+        uint32_t ph = 0u;
         for (int64_t it = p; it < total_it && !*err; it += nprod) {
-            const int64_t ti = it / cbs;
+            const int64_t ti = (cbs == 1) ? it : it / cbs;
             const int cb = (int)(it - ti * cbs);
-            const int s = (int)(it % stages);
-            const uint32_t ph = (uint32_t)((it / stages) & 1);
             if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
             halo_fill(g, cta_in_n + ti * ctas_per_n, cb, sA + s * g.stage_bytes, lane, fa.k, fa.ew);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&full[s]);
+            s += nprod;
+            if (s >= stages) { s -= stages; ph ^= 1u; }
         }
     } else if (warp == kWsMmaWarp) {
         // ---------------------------------------------- MMA issue
@@ -225,16 +229,16 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
             const int ws = 1 << g.lws;
             const int units_tap = g.ldx >> 2;                  // 32-code K steps per tap
             const bool r3 = g.R == 3 && g.S == 3;
-            int64_t it = 0;
+            int s = 0;                                         // stage and phase of the next K-block
+            uint32_t ph = 0u;
             for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
                 const int a = (int)(ti & 1);
                 if (!wait_or_abort(&tempty[a], (uint32_t)((ti >> 1) & 1) ^ 1u, err)) { *err = 1; break; }
                 tc_fence_after();
                 const uint32_t d = tmem_base + (uint32_t)(a * BN);
                 uint32_t acc = 0u;
-                for (int cb = 0; cb < cbs; cb++, it++) {
-                    const int s = (int)(it % stages);
-                    if (!wait_or_abort(&full[s], (uint32_t)((it / stages) & 1), err)) { *err = 1; break; }
+                for (int cb = 0; cb < cbs; cb++) {
+                    if (!wait_or_abort(&full[s], ph, err)) { *err = 1; break; }
                     tc_fence_after();
                     const uint32_t a_st = a_base + (uint32_t)(s * g.stage_bytes);
                     const uint32_t b_blk = b_base + (uint32_t)(cb * BN * kBK);   // block cb: 4 K steps on
@@ -261,6 +265,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
                         }
                     }
                     mma_commit(&empty[s]);
+                    if (++s == stages) { s = 0; ph ^= 1u; }
                 }
                 if (*err) break;
                 mma_commit(&tfull[a]);

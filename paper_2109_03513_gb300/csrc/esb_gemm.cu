@@ -379,6 +379,10 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
         const uint32_t zwa = fmt_zero_code(4, fa.k) * 0x11111111u;
         int64_t cur_tile = -1;
         typename SrcA::Row rows[4];
+        // stage s and its phase ph follow it incrementally (no division in
+        // the loop): it advances by nprod <= stages, so s wraps at most once
+        int s = p;
+        uint32_t ph = 0u;
         for (int64_t it = p; it < total_it && !*err; it += nprod) {
             const int64_t ti = it / nkb;
             const int kb = (int)(it - ti * nkb);
@@ -388,8 +392,6 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
 #pragma unroll
                 for (int q = 0; q < 4; q++) rows[q] = srcA.row(m0 + lane + 32 * q);
             }
-            const int s = (int)(it % stages);
-            const uint32_t ph = (uint32_t)((it / stages) & 1);
             if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
             uint8_t* st = sA + s * kBM * kBK;
             if (fa.b == 4) {
@@ -408,21 +410,23 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&full[s]);
+            s += nprod;
+            if (s >= stages) { s -= stages; ph ^= 1u; }
         }
     } else if (warp == kWsMmaWarp) {
         // ---------------------------------------------- MMA issue
         if (lane == 0) {
             const uint32_t idesc = idesc_e4m3_f32(BN);
             const uint32_t b_base = smem_u32(sB), a_base = smem_u32(sA);
-            int64_t it = 0;
+            int s = 0;                                         // stage and phase of the next K-block
+            uint32_t ph = 0u;
             for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
                 const int a = (int)(ti & 1);
                 if (!wait_or_abort(&tempty[a], (uint32_t)((ti >> 1) & 1) ^ 1u, err)) { *err = 1; break; }
                 tc_fence_after();
                 const uint32_t d = tmem_base + (uint32_t)(a * BN);
-                for (int kb = 0; kb < nkb; kb++, it++) {
-                    const int s = (int)(it % stages);
-                    if (!wait_or_abort(&full[s], (uint32_t)((it / stages) & 1), err)) { *err = 1; break; }
+                for (int kb = 0; kb < nkb; kb++) {
+                    if (!wait_or_abort(&full[s], ph, err)) { *err = 1; break; }
                     tc_fence_after();
                     const uint32_t a0 = a_base + (uint32_t)(s * kBM * kBK);
                     const uint32_t b0 = b_base + (uint32_t)(kb * BN * kBK);
@@ -431,6 +435,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
                         mma_f8f6f4(d, smem_desc_sw128(a0 + j * 32), smem_desc_sw128(b0 + j * 32), idesc,
                                    (kb > 0 || j > 0) ? 1u : 0u);
                     mma_commit(&empty[s]);
+                    if (++s == stages) { s = 0; ph ^= 1u; }
                 }
                 if (*err) break;
                 mma_commit(&tfull[a]);

@@ -14,46 +14,82 @@ namespace esb {
 
 // ----------------------------------------------------------- projection
 
-// Projection of a flat (row stride = cols, code rows without padding)
-// tensor to 4-bit codes in warp tiles of 1024 values: coalesced 16-byte
-// loads, lane l projects values 4(32j + l) .. +3 to 16 bits of codes, and
-// lane pairs (l, l + 1) join their halves into one word with a shuffle.
-template <bool SIGNED, bool STREAM>
-__device__ __forceinline__ void project_flat_b4(const float* __restrict__ x, int64_t n, const Thr7& t7, int k,
-                                                uint32_t* __restrict__ codes)
+// Granules of 128 values (lane l holds values 4l .. 4l + 3): the warps of
+// the grid take equal contiguous runs of them, in the same order in every
+// pass over x, so a warp's share differs by at most one granule from any
+// other's.
+__device__ __forceinline__ void warp_granules(int64_t gran, int64_t& g_lo, int64_t& g_hi)
 {
-    const int lane = threadIdx.x & 31;
     const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    const int64_t tiles = (n + 1023) / 1024;
+    g_lo = gran * gwarp / nwarps;
+    g_hi = gran * (gwarp + 1) / nwarps;
+}
+
+// Codes of one granule (warp-collective): lane l turns its values 4l .. 4l
+// + 3 into 16 bits of codes, lane pairs (l, l + 1) join their halves into
+// code word 16 g + l / 2 with a shuffle.
+template <bool SIGNED>
+__device__ __forceinline__ void project_granule_b4(const float4 q, int64_t g, int64_t nw, const Thr7& t7, int k,
+                                                   uint32_t* __restrict__ codes)
+{
+    const int lane = threadIdx.x & 31;
+    const float xv4[4] = {q.x, q.y, q.z, q.w};
+    uint32_t J = 0u, S = 0u;
+#pragma unroll
+    for (int i = 0; i < 4; i++) {
+        J |= bucket7(SIGNED ? fabsf(xv4[i]) : xv4[i], t7) << (4 * i);
+        if (SIGNED) S |= (__float_as_uint(xv4[i]) >> 31) << (4 * i + 3);
+    }
+    const uint32_t h = codes8_b4(J, S, k) & 0xffffu;          // four codes: low 16 bits
+    const uint32_t other = __shfl_down_sync(0xffffffffu, h, 1);
+    const int64_t wi = g * 16 + (lane >> 1);
+    if ((lane & 1) == 0 && wi < nw) codes[wi] = h | (other << 16);
+}
+
+// Projection of a flat (row stride = cols, code rows without padding)
+// tensor of n values (n % 8 == 0) to 4-bit codes.  The full granules are
+// split among the warps exactly as in the statistics pass (warp_granules);
+// each warp reads its first `stash_g` granules from its shared-memory stash
+// (written by that pass) and the rest in batches of 8 coalesced 16-byte
+// loads per lane; the last warp also takes the partial granule at the end.
+template <bool SIGNED, bool STREAM>
+__device__ __forceinline__ void project_flat_b4(const float* __restrict__ x, int64_t n, const Thr7& t7, int k,
+                                                uint32_t* __restrict__ codes, const float4* stash = nullptr,
+                                                int stash_g = 0)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t gran = n / 128;
+    int64_t g_lo, g_hi;
+    warp_granules(gran, g_lo, g_hi);
+    const float4* xv = reinterpret_cast<const float4*>(x) + lane;
+    const int64_t nw = n >> 3;                        // code words
+    int64_t g0 = g_lo;
+    if (stash) {
+        const int64_t g_st = g_lo + stash_g < g_hi ? g_lo + stash_g : g_hi;
+#pragma unroll 4
+        for (; g0 < g_st; g0++) project_granule_b4<SIGNED>(stash[(g0 - g_lo) * 32 + lane], g0, nw, t7, k, codes);
+    }
 #pragma unroll 1
-    for (int64_t t = gwarp; t < tiles; t += nwarps) {
-        const int64_t e0 = t * 1024;
-        const bool whole = e0 + 1024 <= n;
-        const float4* xt = reinterpret_cast<const float4*>(x + e0) + lane;
+    for (; g0 < g_hi; g0 += 8) {
         float4 q[8];
 #pragma unroll
-        for (int j = 0; j < 8; j++) {
-            const int64_t e = e0 + 4 * (32 * j + lane);
-            if (whole || e < n) q[j] = STREAM ? __ldcs(xt + 32 * j) : __ldg(xt + 32 * j);
-            else q[j] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        for (int u = 0; u < 8; u++) {
+            q[u] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (g0 + u < g_hi) q[u] = STREAM ? __ldcs(xv + (g0 + u) * 32) : __ldg(xv + (g0 + u) * 32);
         }
 #pragma unroll
-        for (int j = 0; j < 8; j++) {
-            const float xv[4] = {q[j].x, q[j].y, q[j].z, q[j].w};
-            uint32_t J = 0u, S = 0u;
-#pragma unroll
-            for (int i = 0; i < 4; i++) {
-                J |= bucket7(SIGNED ? fabsf(xv[i]) : xv[i], t7) << (4 * i);
-                if (SIGNED) S |= (__float_as_uint(xv[i]) >> 31) << (4 * i + 3);
-            }
-            const uint32_t h = codes8_b4(J, S, k) & 0xffffu;          // four codes: low 16 bits
-            const uint32_t other = __shfl_down_sync(0xffffffffu, h, 1);
-            if ((lane & 1) == 0) {
-                const int64_t wi = (e0 >> 3) + 16 * j + (lane >> 1);
-                if (whole || wi < (n >> 3)) codes[wi] = h | (other << 16);
-            }
+        for (int u = 0; u < 8; u++) {
+            if (g0 + u >= g_hi) break;                // warp-uniform
+            project_granule_b4<SIGNED>(q[u], g0 + u, nw, t7, k, codes);
         }
+    }
+    const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    if (gwarp == nwarps - 1 && gran * 128 < n) {      // partial last granule
+        const int64_t e = gran * 128 + 4 * lane;
+        const float4 q = e < n ? __ldg(xv + gran * 32) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        project_granule_b4<SIGNED>(q, gran, nw, t7, k, codes);
     }
 }
 
@@ -202,7 +238,12 @@ static cudaError_t launch_project_b(const float* x, int64_t rows, int64_t cols, 
     if (vec) {
         const int64_t units = rows * (ldc >> 2);
         int64_t blocks = (units + threads - 1) / threads;
-        const int64_t cap = (int64_t)sms * 8;
+        // one resident wave: every warp's share is then loaded at once
+        static int per_sm = 0;
+        if (!per_sm && (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, project_vec_kernel<B>, threads, 0) !=
+                            cudaSuccess || per_sm < 1))
+            per_sm = 2;
+        const int64_t cap = (int64_t)sms * per_sm;
         if (blocks > cap) blocks = cap;
         if (blocks < 1) blocks = 1;
         project_vec_kernel<B><<<(unsigned)blocks, threads, 0, st>>>(x, rows, cols, ldx, alpha, alpha_dev, p, codes, ldc);
@@ -284,10 +325,7 @@ constexpr int kCalThreads = 256;
 constexpr int kCalChunk = 32;
 constexpr int kCalMaxBlocks = 1023;   // + one 32-byte ticket record = 32 KiB of workspace
 constexpr int kCalChunksPerThread = 1;
-
-struct CalPartial {
-    double n, s1, s2, s3;   // sum n_c, sum n_c a_c, sum n_c a_c^2, sum M2_c
-};
+constexpr int kCalStashMax = 13;      // granules per warp kept in shared memory (4 x 8 x 13 x 512 B = 208 KiB per SM)
 
 // (hi, lo) += x, Knuth's TwoSum with the rounding error kept in lo.
 __device__ __forceinline__ void df_add(float& hi, float& lo, float x)
@@ -315,170 +353,245 @@ __device__ __forceinline__ void df_add_sq(float& hi, float& lo, float a)
     lo += pe;
 }
 
-struct CalAcc {
+// Statistics of a set of values split into groups c of n_c values with
+// mean a_c and within-group sum of squared deviations M2_c (law of total
+// variance): n = sum n_c, s1 = sum n_c a_c, s2 = sum n_c a_c^2,
+// s3 = sum M2_c, each sum an fp32 (hi, lo) pair.  One record per block in
+// the workspace (32 bytes).
+struct __align__(16) CalAcc {
     unsigned long long n;
     float s1h, s1l, s2h, s2l, s3h, s3l;
 };
+typedef CalAcc CalPartial;
+
+__device__ __forceinline__ void cal_add(CalAcc& A, const CalAcc& B)
+{
+    A.n += B.n;
+    df_add2(A.s1h, A.s1l, B.s1h, B.s1l);
+    df_add2(A.s2h, A.s2l, B.s2h, B.s2l);
+    df_add2(A.s3h, A.s3l, B.s3h, B.s3l);
+}
 
 __device__ __forceinline__ void cal_shfl(CalAcc& A, int o)
 {
-    const unsigned long long n = __shfl_xor_sync(0xffffffffu, A.n, o);
-    const float a1 = __shfl_xor_sync(0xffffffffu, A.s1h, o), b1 = __shfl_xor_sync(0xffffffffu, A.s1l, o);
-    const float a2 = __shfl_xor_sync(0xffffffffu, A.s2h, o), b2 = __shfl_xor_sync(0xffffffffu, A.s2l, o);
-    const float a3 = __shfl_xor_sync(0xffffffffu, A.s3h, o), b3 = __shfl_xor_sync(0xffffffffu, A.s3l, o);
-    A.n += n;
-    df_add2(A.s1h, A.s1l, a1, b1);
-    df_add2(A.s2h, A.s2l, a2, b2);
-    df_add2(A.s3h, A.s3l, a3, b3);
+    CalAcc B;
+    B.n = __shfl_xor_sync(0xffffffffu, A.n, o);
+    B.s1h = __shfl_xor_sync(0xffffffffu, A.s1h, o); B.s1l = __shfl_xor_sync(0xffffffffu, A.s1l, o);
+    B.s2h = __shfl_xor_sync(0xffffffffu, A.s2h, o); B.s2l = __shfl_xor_sync(0xffffffffu, A.s2l, o);
+    B.s3h = __shfl_xor_sync(0xffffffffu, A.s3h, o); B.s3l = __shfl_xor_sync(0xffffffffu, A.s3l, o);
+    cal_add(A, B);
 }
 
-// Sum of the block partials in a fixed order and the final statistics,
-// run by the last block of the pass (see calibrate_pass1_kernel).
+// Sum over the block's threads (every thread passes its share; thread 0
+// gets the total).
+__device__ __forceinline__ CalAcc cal_block_reduce(CalAcc A)
+{
+    __shared__ CalAcc sh[kCalThreads / 32];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cal_shfl(A, o);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) sh[warp] = A;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 1; w < kCalThreads / 32; w++) cal_add(A, sh[w]);
+    }
+    return A;
+}
+
+// Sum of the nblocks block records in index order (fp32 pair arithmetic
+// across the block: this part runs double precision at a small fraction of
+// the fp32 rate); thread 0 gets the total.  Every block that calls it on
+// the same records gets the same bits.
+__device__ __forceinline__ CalAcc cal_reduce_records(const CalPartial* part, int nblocks)
+{
+    CalAcc t{0ull, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+    // nblocks <= kCalMaxBlocks < 4 * kCalThreads: at most 4 records a thread,
+    // all loaded (two 16-byte loads each, from L2: other blocks wrote them)
+    // before any is added
+    static_assert(kCalMaxBlocks <= 4 * kCalThreads, "records per thread");
+    uint4 w[4][2];
+#pragma unroll
+    for (int u = 0; u < 4; u++) {
+        const int i = threadIdx.x + u * kCalThreads;
+        const uint4* q = reinterpret_cast<const uint4*>(part + (i < nblocks ? i : 0));
+        w[u][0] = __ldcg(q);
+        w[u][1] = __ldcg(q + 1);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; u++) {
+        if (threadIdx.x + u * kCalThreads < nblocks) {
+            CalAcc r;
+            r.n = (unsigned long long)w[u][0].x | ((unsigned long long)w[u][0].y << 32);
+            r.s1h = __uint_as_float(w[u][0].z); r.s1l = __uint_as_float(w[u][0].w);
+            r.s2h = __uint_as_float(w[u][1].x); r.s2l = __uint_as_float(w[u][1].y);
+            r.s3h = __uint_as_float(w[u][1].z); r.s3l = __uint_as_float(w[u][1].w);
+            cal_add(t, r);
+        }
+    }
+    return cal_block_reduce(t);
+}
+
+// alpha = fl32(alpha* (spread + 1e-7)) from the totals (Sec. III-D); the
+// spread is the standard deviation for the symmetric set and the RMS for
+// the non-negative one.  fp32 pair arithmetic only (double precision runs
+// at a small fraction of the fp32 rate on this part): the mean is kept as a
+// pair, so s2 - s1 * mean loses nothing to the rounding of the mean even
+// when |mean| >> spread; the final quotient and square root are single
+// fp32 operations (relative error ~1e-7).  stats (may be null) gets
+// {mean, spread, n}.
+__device__ __forceinline__ float cal_alpha(const CalAcc& t, double alpha_star, int is_signed, double* stats)
+{
+    const float nh = (float)t.n;                                   // n as a pair (exact below 2^48)
+    const float nl = (float)(t.n - (unsigned long long)nh);
+    float vh, vl;                                                  // the centred (or raw) second moment sum
+    // mean = s1 / n to pair precision: quotient, then the remainder's
+    // quotient (products with one rounded reciprocal: ~1 ulp)
+    const float rn = 1.0f / nh;
+    const float mh = t.s1h * rn;
+    const float ml = (fmaf(-mh, nh, t.s1h) - mh * nl + t.s1l) * rn;
+    if (is_signed) {
+        // s1 * mean as a pair (fma gives the product's rounding error exactly)
+        const float ph = t.s1h * mh;
+        const float pl = fmaf(t.s1h, mh, -ph) + t.s1h * ml + t.s1l * mh;
+        // m2 = s3 + (s2 - s1 * mean)
+        float dh = t.s2h, dl = t.s2l;
+        df_add2(dh, dl, -ph, -pl);
+        vh = t.s3h; vl = t.s3l;
+        df_add2(vh, vl, dh, dl);
+    } else {
+        vh = t.s3h; vl = t.s3l;
+        df_add2(vh, vl, t.s2h, t.s2l);
+    }
+    float v = vh + vl;
+    if (!(v > 0.0f)) v = 0.0f;
+    const float spread = sqrtf(v * rn);
+    if (stats) { stats[0] = (double)mh + (double)ml; stats[1] = (double)spread; stats[2] = (double)t.n; }
+    return (float)alpha_star * (spread + 1e-7f);
+}
+
+// The last block of a pass: totals and alpha.
 __device__ void calibrate_finalize_block(const CalPartial* part, int nblocks, double alpha_star, int is_signed,
                                          float* alpha_out, double* stats_out)
 {
-    __shared__ CalPartial red[kCalThreads];
-    CalPartial t{0.0, 0.0, 0.0, 0.0};
-    for (int i = threadIdx.x; i < nblocks; i += kCalThreads) {
-        const double* q = reinterpret_cast<const double*>(part + i);   // written by other blocks: read from L2
-        t.n += __ldcg(q); t.s1 += __ldcg(q + 1); t.s2 += __ldcg(q + 2); t.s3 += __ldcg(q + 3);
-    }
-    red[threadIdx.x] = t;
-    __syncthreads();
-    for (int h = kCalThreads / 2; h > 0; h >>= 1) {
-        if ((int)threadIdx.x < h) {
-            red[threadIdx.x].n += red[threadIdx.x + h].n;
-            red[threadIdx.x].s1 += red[threadIdx.x + h].s1;
-            red[threadIdx.x].s2 += red[threadIdx.x + h].s2;
-            red[threadIdx.x].s3 += red[threadIdx.x + h].s3;
-        }
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) {
-        const CalPartial r = red[0];
-        const double mean = r.s1 / r.n;
-        double spread;
-        if (is_signed) {
-            double m2 = r.s3 + (r.s2 - r.s1 * mean);
-            if (m2 < 0.0) m2 = 0.0;
-            spread = sqrt(m2 / r.n);
-        } else {
-            spread = sqrt((r.s3 + r.s2) / r.n);
-        }
-        *alpha_out = (float)(alpha_star * (spread + 1e-7));
-        if (stats_out) { stats_out[0] = mean; stats_out[1] = spread; stats_out[2] = r.n; }
-    }
+    const CalAcc t = cal_reduce_records(part, nblocks);
+    if (threadIdx.x == 0) *alpha_out = cal_alpha(t, alpha_star, is_signed, stats_out);
 }
 
-// One launch: every block writes its partial record; the block that takes
-// the last ticket (the ticket word is zeroed by a memset before the launch)
-// adds all records in index order and finalises alpha.
-// Adds one group of `cnt` values (cnt = 32: weight folded in at the end; any
-// other count: weighted exactly) to the accumulators.
-__device__ __forceinline__ void cal_group(const float* v, int cnt, float& sa_h, float& sa_l, float& sq_h, float& sq_l,
+// Adds one group of CNT values to the accumulators: CNT = 32 keeps its mean
+// in the (sa, sq) sums whose weight 32 is applied once at the end; any
+// other count is weighted exactly here.
+template <int CNT>
+__device__ __forceinline__ void cal_group(const float (&v)[CNT], float& sa_h, float& sa_l, float& sq_h, float& sq_l,
                                           CalAcc& A, unsigned long long& full_groups)
 {
     float s = 0.0f;
-    for (int i = 0; i < cnt; i++) s += v[i];
-    const float a = (cnt == kCalChunk) ? s * (1.0f / kCalChunk) : s / (float)cnt;
+#pragma unroll
+    for (int i = 0; i < CNT; i++) s += v[i];
+    const float a = s * (1.0f / CNT);                 // CNT is a power of two: exact scaling of the sum
     float m2 = 0.0f;
-    for (int i = 0; i < cnt; i++) { const float d = v[i] - a; m2 = fmaf(d, d, m2); }
-    if (cnt == kCalChunk) {
+#pragma unroll
+    for (int i = 0; i < CNT; i++) { const float d = v[i] - a; m2 = fmaf(d, d, m2); }
+    if (CNT == kCalChunk) {
         df_add(sa_h, sa_l, a);
         df_add_sq(sq_h, sq_l, a);
         full_groups += 1ull;
     } else {
         // n_c * a and n_c * a^2 as exact pairs: split the products with fmas
-        const float w = (float)cnt;
+        const float w = (float)CNT;
         const float p1 = w * a, e1 = fmaf(w, a, -p1);
         df_add(A.s1h, A.s1l, p1); A.s1l += e1;
         const float q = a * a, qe = fmaf(a, a, -q);          // a^2 = q + qe exactly
         const float p2 = w * q, e2 = fmaf(w, q, -p2);         // w q = p2 + e2 exactly
         df_add(A.s2h, A.s2l, p2); A.s2l += e2 + w * qe;
-        A.n += (unsigned long long)cnt;
+        A.n += (unsigned long long)CNT;
     }
     df_add(A.s3h, A.s3l, m2);
 }
 
+// One value as its own group (n_c = 1, M2_c = 0).
+__device__ __forceinline__ void cal_single(float a, CalAcc& A)
+{
+    df_add(A.s1h, A.s1l, a);
+    df_add_sq(A.s2h, A.s2l, a);
+    A.n += 1ull;
+}
+
 // Statistics of this block's share of x, reduced over the block; thread 0
-// returns the block's partial record.  The data is read in warp tiles of
-// 1024 values with coalesced 16-byte loads (lane l takes values
-// 4(32j + l) .. +3, j = 0..7, as its group of 32 -- any partition into groups
-// serves the law of total variance).  Values past the last full tile are
-// taken by warp 0 of block 0 in contiguous groups of at most 32.
+// returns the block's record.  With a stash (this warp's region of shared
+// memory) the warp also keeps its first stash_g granules there.  Each warp reads its granules in batches of
+// 8 (eight coalesced 16-byte loads per lane in flight); a lane's 32 values
+// of a full batch form one group, a shorter batch gives groups of 4 (any
+// partition into groups serves the law of total variance).  The n % 128
+// values past the last granule (all of x when it is not 16-byte aligned)
+// are taken by warp 0 of block 0 one by one.
 // `stream_loads` selects evict-first loads (data read once) or default loads
-// (data kept in L2 for a second pass).
-__device__ __forceinline__ CalPartial cal_block_partial(const float* __restrict__ x, int64_t n, int vec,
-                                                        bool stream_loads)
+// (data kept in the caches for a second pass).
+__device__ __forceinline__ CalAcc cal_block_partial(const float* __restrict__ x, int64_t n, int vec, bool stream_loads,
+                                                    float4* stash = nullptr, int stash_g = 0)
 {
     const int lane = threadIdx.x & 31;
-    const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    const int64_t tiles = vec ? n / 1024 : 0;
+    const int64_t gran = vec ? n / 128 : 0;
+    int64_t g_lo, g_hi;
+    warp_granules(gran, g_lo, g_hi);
     CalAcc A{0ull, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
     float sa_h = 0.0f, sa_l = 0.0f;   // sum of a over full groups (weight 32 applied at the end)
     float sq_h = 0.0f, sq_l = 0.0f;   // sum of a^2 over full groups
     unsigned long long full_groups = 0ull;
+    const float4* xv = reinterpret_cast<const float4*>(x) + lane;
 #pragma unroll 1
-    for (int64_t t = gwarp; t < tiles; t += nwarps) {
-        const float4* xt = reinterpret_cast<const float4*>(x + t * 1024) + lane;
-        float v[kCalChunk];
+    for (int64_t g0 = g_lo; g0 < g_hi; g0 += 8) {
+        const int cnt = (int)((g_hi - g0) < 8 ? (g_hi - g0) : 8);
+        float4 q[8];
 #pragma unroll
-        for (int j = 0; j < 8; j++) {
-            const float4 q = stream_loads ? __ldcs(xt + 32 * j) : __ldg(xt + 32 * j);
-            v[4 * j] = q.x; v[4 * j + 1] = q.y; v[4 * j + 2] = q.z; v[4 * j + 3] = q.w;
+        for (int u = 0; u < 8; u++) {
+            q[u] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (u < cnt) q[u] = stream_loads ? __ldcs(xv + (g0 + u) * 32) : __ldg(xv + (g0 + u) * 32);
         }
-        cal_group(v, kCalChunk, sa_h, sa_l, sq_h, sq_l, A, full_groups);
-    }
-    const int64_t rem0 = tiles * 1024;
-    if (blockIdx.x == 0 && threadIdx.x < 32 && rem0 < n) {
-        // up to 32 contiguous groups of 32 per lane pass
-        for (int64_t g0 = rem0 + 32 * (int64_t)lane; g0 < n; g0 += 32 * 32) {
-            const int cnt = (int)((n - g0) < 32 ? (n - g0) : 32);
+        if (stash) {                                  // keep the warp's first stash_g granules on chip
+#pragma unroll
+            for (int u = 0; u < 8; u++)
+                if (u < cnt && g0 + u - g_lo < stash_g) stash[(g0 + u - g_lo) * 32 + lane] = q[u];
+        }
+        if (cnt == 8) {
             float v[kCalChunk];
-            for (int i = 0; i < cnt; i++) v[i] = x[g0 + i];
-            cal_group(v, cnt, sa_h, sa_l, sq_h, sq_l, A, full_groups);
+#pragma unroll
+            for (int u = 0; u < 8; u++) { v[4 * u] = q[u].x; v[4 * u + 1] = q[u].y; v[4 * u + 2] = q[u].z; v[4 * u + 3] = q[u].w; }
+            cal_group<kCalChunk>(v, sa_h, sa_l, sq_h, sq_l, A, full_groups);
+        } else {
+#pragma unroll
+            for (int u = 0; u < 8; u++) {
+                if (u < cnt) {
+                    const float v[4] = {q[u].x, q[u].y, q[u].z, q[u].w};
+                    cal_group<4>(v, sa_h, sa_l, sq_h, sq_l, A, full_groups);
+                }
+            }
         }
+    }
+    const int64_t rem0 = gran * 128;
+    if (blockIdx.x == 0 && threadIdx.x < 32) {
+        for (int64_t i = rem0 + lane; i < n; i += 32) cal_single(x[i], A);
     }
     // full groups carry weight 32: scaling a pair by a power of two is exact
     A.n += full_groups * (unsigned long long)kCalChunk;
     df_add2(A.s1h, A.s1l, sa_h * kCalChunk, sa_l * kCalChunk);
     df_add2(A.s2h, A.s2l, sq_h * kCalChunk, sq_l * kCalChunk);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) cal_shfl(A, o);
-    __shared__ CalAcc sh[kCalThreads / 32];
-    const int warp = threadIdx.x >> 5;
-    if (lane == 0) sh[warp] = A;
-    __syncthreads();
-    CalPartial out{0.0, 0.0, 0.0, 0.0};
-    if (threadIdx.x == 0) {
-        CalAcc t = sh[0];
-        for (int w = 1; w < kCalThreads / 32; w++) {
-            t.n += sh[w].n;
-            df_add2(t.s1h, t.s1l, sh[w].s1h, sh[w].s1l);
-            df_add2(t.s2h, t.s2l, sh[w].s2h, sh[w].s2l);
-            df_add2(t.s3h, t.s3l, sh[w].s3h, sh[w].s3l);
-        }
-        out = CalPartial{(double)t.n, (double)t.s1h + (double)t.s1l, (double)t.s2h + (double)t.s2l,
-                         (double)t.s3h + (double)t.s3l};
-    }
-    return out;
+    return cal_block_reduce(A);
 }
 
 // Workspace head record: the ticket counter, the release flag of the fused
 // kernel's grid barrier, and the alpha it publishes.
 struct CalSync {
     unsigned int ticket;
-    unsigned int flag;
-    float alpha;
-    unsigned int pad[5];
+    unsigned int pad0;
+    unsigned long long release;   // fused kernel: (1 << 32) | bits(alpha) once alpha is known
+    unsigned int pad[4];
 };
 static_assert(sizeof(CalSync) == sizeof(CalPartial), "head record is one partial record wide");
 
 // One launch: every block writes its partial record; the block that takes
 // the last ticket (the ticket word is zeroed by a memset before the launch)
 // adds all records in index order and finalises alpha.
-__global__ void __launch_bounds__(kCalThreads)
+__global__ void __launch_bounds__(kCalThreads, 4)
 calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalPartial* __restrict__ part,
                        CalSync* __restrict__ sync, double alpha_star, int is_signed,
                        float* __restrict__ alpha_out, double* __restrict__ stats_out)
@@ -505,19 +618,28 @@ calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalParti
 // raises the release flag, which every other block waits for (bounded).
 // Phase 2 projects x, now read from L2, with that alpha.
 template <int B>
-__global__ void __launch_bounds__(kCalThreads)
+__global__ void __launch_bounds__(kCalThreads, 4)
 calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, CalPartial* __restrict__ part,
                          CalSync* __restrict__ sync, double alpha_star, ProjParams p, float* __restrict__ alpha_out,
                          double* __restrict__ stats_out, uint32_t* __restrict__ codes, int64_t ldc,
-                         int* __restrict__ status)
+                         int* __restrict__ status, int stash_g)
 {
+    // stash: stash_g granules (512 bytes each) per warp of dynamic shared memory
+    extern __shared__ float4 stash_all[];
+    float4* stash = stash_g > 0 ? stash_all + (size_t)(threadIdx.x >> 5) * stash_g * 32 : nullptr;
     constexpr int CPW = 32 / B;
     constexpr int L = 1 << (B - 1);
     const int64_t n = rows * cols;
-    const CalPartial mine = cal_block_partial(x, n, 1, false);
-    __shared__ bool is_last;
+    const bool flat = B == 4 && cols % 8 == 0 && ldc * 8 == cols;
+    const CalPartial mine = cal_block_partial(x, n, 1, false, flat ? stash : nullptr, stash_g);
     __shared__ int timed_out;
+    __shared__ float s_alpha;
     __shared__ float T[L];
+    // Grid barrier: every block publishes its record; the block that takes
+    // the last ticket sums the records and publishes alpha in the release
+    // word (one 64-bit store: flag and value together), which the others
+    // wait for (bounded).
+    __shared__ bool is_last;
     if (threadIdx.x == 0) {
         part[blockIdx.x] = mine;
         __threadfence();
@@ -527,37 +649,44 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
     __syncthreads();
     if (is_last) {
         __threadfence();
-        calibrate_finalize_block(part, gridDim.x, alpha_star, p.is_signed, &sync->alpha, stats_out);
+        const CalAcc tot = cal_reduce_records(part, gridDim.x);
         if (threadIdx.x == 0) {
-            *alpha_out = sync->alpha;
-            __threadfence();
-            atomicExch(&sync->flag, 1u);
+            double st[3];
+            const float al = cal_alpha(tot, alpha_star, p.is_signed, stats_out ? st : nullptr);
+            // alpha travels in the release word itself: nothing else has to
+            // be visible to the other blocks first
+            atomicExch(&sync->release, (1ull << 32) | (unsigned long long)__float_as_uint(al));
+            s_alpha = al;
+            *alpha_out = al;
+            if (stats_out) { stats_out[0] = st[0]; stats_out[1] = st[1]; stats_out[2] = st[2]; }
         }
     } else if (threadIdx.x == 0) {
-        const volatile unsigned int* f = &sync->flag;
+        const volatile unsigned long long* rel = &sync->release;
         const uint64_t t0 = globaltimer_ns();
         uint32_t it = 0;
-        while (*f == 0u) {
-            if ((++it & 255u) == 0u && globaltimer_ns() - t0 > 2000000000ull) { timed_out = 1; break; }
-            __nanosleep(64);
+        unsigned long long w = *rel;
+        while ((w >> 32) == 0ull) {
+            if ((++it & 63u) == 0u && globaltimer_ns() - t0 > 2000000000ull) { timed_out = 1; break; }
+            __nanosleep(32);
+            w = *rel;
         }
-        __threadfence();
+        s_alpha = __uint_as_float((unsigned int)(w & 0xffffffffull));
     }
     __syncthreads();
     if (timed_out) {
         if (threadIdx.x == 0) record_status(status, ESB_ERR_TIMEOUT);
         return;
     }
-    const float a = __ldcg(&sync->alpha);
+    const float a = s_alpha;
     build_thresholds(T, p, a, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
     __syncthreads();
     Thr7 t7;
     if (B == 4) {
 #pragma unroll
         for (int i = 0; i < 7; i++) t7.t[i] = T[i];
-        if (cols % 8 == 0 && ldc * 8 == cols) {         // flat codes: coalesced warp tiles
-            if (p.is_signed) project_flat_b4<true, true>(x, n, t7, p.k, codes);
-            else project_flat_b4<false, true>(x, n, t7, p.k, codes);
+        if (flat) {                                     // flat codes: the statistics pass's granules
+            if (p.is_signed) project_flat_b4<true, true>(x, n, t7, p.k, codes, stash, stash_g);
+            else project_flat_b4<false, true>(x, n, t7, p.k, codes, stash, stash_g);
             return;
         }
     }
@@ -615,6 +744,14 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
     }
 }
 
+// These kernels use almost no shared memory: ask for the largest L1 (the
+// fused kernel's second pass re-reads x, which then stays on chip).
+template <class F>
+static void prefer_l1(F* kernel)
+{
+    (void)cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 0);
+}
+
 // Grid: one chunk per thread up to one resident wave (4 blocks of 256
 // threads per SM at this kernel's register use), at most kCalMaxBlocks.
 int calibrate_blocks(int64_t n)
@@ -641,8 +778,10 @@ cudaError_t launch_calibrate(const float* x, int64_t n, int is_signed, double al
     const int vec = ((reinterpret_cast<uintptr_t>(x) & 15u) == 0) ? 1 : 0;
     CalSync* sync = static_cast<CalSync*>(workspace);
     CalPartial* part = static_cast<CalPartial*>(workspace) + 1;
-    cudaError_t e = cudaMemsetAsync(sync, 0, 2 * sizeof(unsigned int), st);
+    cudaError_t e = cudaMemsetAsync(sync, 0, 16, st);
     if (e != cudaSuccess) return e;
+    static bool l1_set = false;
+    if (!l1_set) { prefer_l1(calibrate_pass1_kernel); l1_set = true; }
     calibrate_pass1_kernel<<<g, kCalThreads, 0, st>>>(x, n, vec, part, sync, alpha_star, is_signed, alpha_out,
                                                         stats_out);
     return cudaGetLastError();
@@ -654,22 +793,44 @@ static cudaError_t launch_calibrate_project_b(const float* x, int64_t rows, int6
                                               uint32_t* codes, int64_t ldc, cudaStream_t st, bool* launched)
 {
     *launched = false;
+    const int64_t n = rows * cols;
+    const int sms = device_sm_count();
+    int64_t g = calibrate_blocks(n);                  // up to 4 blocks per SM
+    // Stash (flat 4-bit codes): every warp keeps its granules in shared
+    // memory between the two passes, up to kCalStashMax granules (4 blocks
+    // of 8 warps x kCalStashMax x 512 bytes fit one SM); any rest is re-read.
+    const bool flat = B == 4 && cols % 8 == 0 && ldc * 8 == cols;
+    int stash_g = 0;
+    if (flat) {
+        const int64_t nwarps = g * (kCalThreads / 32);
+        const int64_t gs = (n / 128 + nwarps - 1) / nwarps;
+        stash_g = (int)(gs < kCalStashMax ? gs : kCalStashMax);
+    }
+    const size_t smem = (size_t)stash_g * 512 * (kCalThreads / 32);
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e0 = cudaFuncSetAttribute(calibrate_project_kernel<B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              kCalStashMax * 512 * (kCalThreads / 32));
+        if (e0 != cudaSuccess) return e0;
+        (void)cudaFuncSetAttribute(calibrate_project_kernel<B>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+        configured = true;
+    }
     int per_sm = 0;
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, calibrate_project_kernel<B>, kCalThreads, 0);
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, calibrate_project_kernel<B>, kCalThreads, smem);
     if (e != cudaSuccess) return e;
-    int64_t g = calibrate_blocks(rows * cols);
-    const int64_t co_resident = (int64_t)per_sm * device_sm_count();
+    const int64_t co_resident = (int64_t)per_sm * sms;
     if (co_resident < 1) return cudaSuccess;
-    if (g > co_resident) g = co_resident;
+    if (g > co_resident) g = co_resident;             // a partial stash still works: the rest is re-read
     CalSync* sync = static_cast<CalSync*>(workspace);
     CalPartial* part = static_cast<CalPartial*>(workspace) + 1;
-    e = cudaMemsetAsync(sync, 0, 2 * sizeof(unsigned int), st);
+    e = cudaMemsetAsync(sync, 0, 16, st);
     if (e != cudaSuccess) return e;
     int* status = device_status_ptr();
     void* args[] = {(void*)&x, (void*)&rows, (void*)&cols, (void*)&part, (void*)&sync, (void*)&alpha_star,
-                    (void*)&p, (void*)&alpha_out, (void*)&stats_out, (void*)&codes, (void*)&ldc, (void*)&status};
+                    (void*)&p, (void*)&alpha_out, (void*)&stats_out, (void*)&codes, (void*)&ldc, (void*)&status,
+                    (void*)&stash_g};
     e = cudaLaunchCooperativeKernel((const void*)calibrate_project_kernel<B>, dim3((unsigned)g), dim3(kCalThreads),
-                                    args, 0, st);
+                                    args, smem, st);
     *launched = true;
     return e;
 }
@@ -745,7 +906,7 @@ cudaError_t launch_calibrate_noalloc(const float* x, int64_t n, int is_signed, d
     void* ws = nullptr;
     cudaError_t e = noalloc_scratch_address(&ws);
     if (e != cudaSuccess) return e;
-    // The ticket and flag words are zeroed by a memset node of the launch;
+    // The ticket and release words are zeroed by a memset node of the launch;
     // every partial record is written before it is read, so nothing else has
     // to be cleared.
     return launch_calibrate(x, n, is_signed, alpha_star, ws, alpha_out, stats_out, st);
