@@ -159,11 +159,15 @@ size_t esb_calibrate_dda_workspace_bytes(int64_t n);
  *              alignment accepted)
  *   n          > 0
  *   workspace  [device] >= esb_calibrate_dda_workspace_bytes(n) bytes,
- *              16-byte aligned, contents ignored and overwritten
+ *              16-byte aligned, zero-filled before its first use (e.g.
+ *              cudaMemset once); every call that completes leaves its first
+ *              32 bytes zero again (the block records after them are
+ *              scratch), so it needs no clearing between calls.  After a
+ *              device status of ESB_ERR_TIMEOUT zero it again.
  *   alpha_out  [device] 1 float written by the kernel (no host sync)
  *   stats_out  [device] 3 doubles {mean, sigma or rms, n}, or NULL
- * One memset of the workspace's ticket words and one kernel launch; the
- * reduction order is fixed, so results are bit-reproducible on a device.
+ * One kernel launch; the reduction order is fixed, so results are
+ * bit-reproducible on a device.
  * Errors: INVALID_ARG, UNSUPPORTED (bad format), ALIGN (workspace), CUDA. */
 esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
                              void* workspace, size_t workspace_bytes,
@@ -188,9 +192,9 @@ esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
  *   alpha_out  [device] 1 float; stats_out [device] 3 doubles or NULL
  * The first call on a device looks up the array's device address (with
  * that device current) and caches it; make that first call before any
- * stream capture.  All calls share the one array and it keeps the last
- * call's contents (each call overwrites every record it later reads, so
- * nothing has to be cleared): calls whose kernels overlap on the GPU (on
+ * stream capture.  All calls share the one array (zero-filled when the
+ * library loads; each call leaves its head record zero and overwrites every
+ * block record it later reads): calls whose kernels overlap on the GPU (on
  * different streams without ordering) race on it and must be serialised.
  * Errors: INVALID_ARG, UNSUPPORTED, RANGE (scratch need above the array's
  * size; the reduction uses at most 1023 blocks plus one ticket record, so
@@ -221,11 +225,14 @@ esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx,
 
 /* DDA-calibrated projection of one tensor: the statistics and alpha of
  * esb_calibrate_dda (Sec. III-D), then esb_project of the same tensor with
- * that alpha (Eq. cheap_projection), in one cooperative launch that keeps
- * the tensor in L2 between the two passes.
+ * that alpha (Eq. cheap_projection), in one cooperative launch: each
+ * warp keeps its share of the tensor on chip (shared memory) between the
+ * two passes, so x is read from memory once.
  *   x          [device] rows x cols floats, contiguous (row stride cols)
  *   workspace  [device] >= esb_calibrate_dda_workspace_bytes(rows * cols),
- *              16-byte aligned, contents ignored
+ *              16-byte aligned, zero-filled before its first use, as for
+ *              esb_calibrate_dda (the two may share one workspace when
+ *              their calls are ordered)
  *   alpha_out  [device] 1 float written with the alpha used
  *   stats_out  [device] 3 doubles {mean, sigma or rms, n}, or NULL
  *   codes      [device] rows x ldc words, as esb_project

@@ -280,6 +280,15 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p)
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// Programmatic dependent launch.  griddep_wait: block until the grids this
+// one depends on have completed and their memory is visible (returns at
+// once when the launch has no programmatic dependency); every read of data
+// an earlier launch may have written, and every write an earlier launch may
+// still read, comes after it.  griddep_launch_dependents: this CTA no longer
+// holds back the launch of a dependent grid.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // Bytes of dynamic shared memory this launch was given.
 __device__ __forceinline__ uint32_t dynamic_smem_bytes()
 {

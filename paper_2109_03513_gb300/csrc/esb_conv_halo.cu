@@ -202,6 +202,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
         const int p = warp - kWsProdWarp0;
         const int nprod = stages < kWsProdWarps ? stages : kWsProdWarps;
         const int64_t total_it = (p < nprod) ? my_tiles * cbs : 0;
+        griddep_wait();                               // X may come from the previous launch
         // stage s and its phase ph follow it incrementally (no division in
         // the loop): it advances by nprod <= stages, so s wraps at most once
         int s = p;
@@ -399,10 +400,8 @@ bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, i
     const int64_t grid = per_n * n_tiles;
     RowsSrc b{W, (int64_t)d.r * d.s * ldw, N};
     const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
-    esb_conv_halo_kernel<<<(unsigned)grid, kWsThreads, (size_t)hp.smem, st>>>(hp.g, b, N, hp.K, fa, fb, hp.BN, hp.nkb,
-                                                                             hp.stages, n_tiles, m_tiles, acc_scale,
-                                                                             ep);
-    *err = cudaGetLastError();
+    *err = launch_pdl(esb_conv_halo_kernel, dim3((unsigned)grid), dim3(kWsThreads), (size_t)hp.smem, st, hp.g, b, N,
+                      hp.K, fa, fb, hp.BN, hp.nkb, hp.stages, n_tiles, m_tiles, acc_scale, ep);
     return true;
 }
 

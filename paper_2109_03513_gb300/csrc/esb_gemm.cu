@@ -376,6 +376,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
         const int p = warp - kWsProdWarp0;
         const int nprod = stages < kWsProdWarps ? stages : kWsProdWarps;
         const int64_t total_it = (p < nprod) ? my_tiles * nkb : 0;
+        griddep_wait();                               // A may come from the previous launch
         const uint32_t zwa = fmt_zero_code(4, fa.k) * 0x11111111u;
         int64_t cur_tile = -1;
         typename SrcA::Row rows[4];
@@ -555,10 +556,8 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
     if (per_n > m_tiles) per_n = m_tiles;
     const int64_t grid = per_n * n_tiles;
     const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
-    esb_gemm_ws_kernel<SrcA><<<(unsigned)grid, kWsThreads, L.smem_bytes, st>>>(a, b, M, N, K, fa, fb, BN, L.nkb,
-                                                                               L.stages, n_tiles, m_tiles, acc_scale,
-                                                                               ep);
-    *err = cudaGetLastError();
+    *err = launch_pdl(esb_gemm_ws_kernel<SrcA>, dim3((unsigned)grid), dim3(kWsThreads), (size_t)L.smem_bytes, st, a, b,
+                      M, N, K, fa, fb, BN, L.nkb, L.stages, n_tiles, m_tiles, acc_scale, ep);
     return true;
 }
 

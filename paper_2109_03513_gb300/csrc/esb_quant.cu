@@ -580,9 +580,11 @@ __device__ __forceinline__ CalAcc cal_block_partial(const float* __restrict__ x,
 
 // Workspace head record: the ticket counter, the release flag of the fused
 // kernel's grid barrier, and the alpha it publishes.
+// All three words are zero when a launch starts and zero again when it
+// ends: the last block to leave resets them (no memset between calls).
 struct CalSync {
-    unsigned int ticket;
-    unsigned int pad0;
+    unsigned int ticket;          // blocks that have published their record
+    unsigned int depart;          // fused kernel: blocks past the release
     unsigned long long release;   // fused kernel: (1 << 32) | bits(alpha) once alpha is known
     unsigned int pad[4];
 };
@@ -607,6 +609,7 @@ calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalParti
     if (is_last) {
         __threadfence();
         calibrate_finalize_block(part, gridDim.x, alpha_star, is_signed, alpha_out, stats_out);
+        if (threadIdx.x == 0) sync->ticket = 0u;      // every block has counted itself: ready for the next call
     }
 }
 
@@ -672,12 +675,23 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
         }
         s_alpha = __uint_as_float((unsigned int)(w & 0xffffffffull));
     }
+    if (threadIdx.x == 0 && !timed_out) {
+        // leave the barrier; the last block out returns the words to zero
+        if (atomicAdd(&sync->depart, 1u) == gridDim.x - 1) {
+            sync->ticket = 0u;
+            sync->release = 0ull;
+            sync->depart = 0u;
+        }
+    }
     __syncthreads();
     if (timed_out) {
         if (threadIdx.x == 0) record_status(status, ESB_ERR_TIMEOUT);
         return;
     }
     const float a = s_alpha;
+    // every block is resident (cooperative launch) and past the barrier: a
+    // dependent grid may take the SMs as these blocks finish
+    griddep_launch_dependents();
     build_thresholds(T, p, a, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
     __syncthreads();
     Thr7 t7;
@@ -778,8 +792,6 @@ cudaError_t launch_calibrate(const float* x, int64_t n, int is_signed, double al
     const int vec = ((reinterpret_cast<uintptr_t>(x) & 15u) == 0) ? 1 : 0;
     CalSync* sync = static_cast<CalSync*>(workspace);
     CalPartial* part = static_cast<CalPartial*>(workspace) + 1;
-    cudaError_t e = cudaMemsetAsync(sync, 0, 16, st);
-    if (e != cudaSuccess) return e;
     static bool l1_set = false;
     if (!l1_set) { prefer_l1(calibrate_pass1_kernel); l1_set = true; }
     calibrate_pass1_kernel<<<g, kCalThreads, 0, st>>>(x, n, vec, part, sync, alpha_star, is_signed, alpha_out,
@@ -823,8 +835,6 @@ static cudaError_t launch_calibrate_project_b(const float* x, int64_t rows, int6
     if (g > co_resident) g = co_resident;             // a partial stash still works: the rest is re-read
     CalSync* sync = static_cast<CalSync*>(workspace);
     CalPartial* part = static_cast<CalPartial*>(workspace) + 1;
-    e = cudaMemsetAsync(sync, 0, 16, st);
-    if (e != cudaSuccess) return e;
     int* status = device_status_ptr();
     void* args[] = {(void*)&x, (void*)&rows, (void*)&cols, (void*)&part, (void*)&sync, (void*)&alpha_star,
                     (void*)&p, (void*)&alpha_out, (void*)&stats_out, (void*)&codes, (void*)&ldc, (void*)&status,
@@ -906,9 +916,8 @@ cudaError_t launch_calibrate_noalloc(const float* x, int64_t n, int is_signed, d
     void* ws = nullptr;
     cudaError_t e = noalloc_scratch_address(&ws);
     if (e != cudaSuccess) return e;
-    // The ticket and release words are zeroed by a memset node of the launch;
-    // every partial record is written before it is read, so nothing else has
-    // to be cleared.
+    // The array starts zero-filled and every call leaves its head record
+    // zero again; every partial record is written before it is read.
     return launch_calibrate(x, n, is_signed, alpha_star, ws, alpha_out, stats_out, st);
 }
 

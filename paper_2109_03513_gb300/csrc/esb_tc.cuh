@@ -371,7 +371,9 @@ static __device__ __noinline__ uint32_t epi_word_b4(const EpiParams* __restrict_
 // ------------------------------------ roles of the warp-specialised kernels
 
 // Setup role (warps 0 .. kWsProdWarp0 - 1, while the producers already load
-// A): the MMA warp allocates tmem_cols TMEM columns; all setup warps decode
+// A): the MMA warp allocates tmem_cols TMEM columns (before the
+// programmatic-launch wait: it touches no data of earlier launches); all
+// setup warps decode
 // the CTA's N-tile of B (rows n0 .. n0 + BN, every K-block) once into sB in
 // the SW128 K-major layout, and build the requantisation thresholds; then
 // they meet on named barrier 1.  Returns the TMEM base address.
@@ -385,6 +387,7 @@ __device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, in
         tmem_alloc(tmem_slot, tmem_cols);
         tc_fence_before();
     }
+    griddep_wait();                                   // B and the alphas may come from the previous launch
     if (fb.b == 4) {
         for (int pr = tid; pr < nkb * BN; pr += kSetupThreads) {
             const int kb = pr / BN, r = pr - kb * BN;
@@ -601,6 +604,25 @@ __device__ __forceinline__ void ws_drain(uint64_t* drain, volatile int* err)
 }
 
 // ------------------------------------------------------------- host side
+
+// Launch with programmatic stream serialisation: the grid may start while
+// the previous kernel of the stream finishes; the kernel's griddep_wait
+// orders its dependent reads and writes after it.
+template <class... KArgs, class... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
 
 int pick_bn(int64_t N, int out_cpw);          // N-tile width (esb_gemm.cu)
 int max_dyn_smem();                           // opt-in shared memory per block

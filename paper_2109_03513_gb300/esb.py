@@ -174,7 +174,7 @@ def esb_calibrate_dda(x: torch.Tensor, f: Fmt, alpha_out: Optional[torch.Tensor]
         alpha_out = torch.empty(1, dtype=torch.float32, device=x.device)
     if workspace is None:
         nb = int(lib().esb_calibrate_dda_workspace_bytes(n))
-        workspace = torch.empty(max(nb, 8), dtype=torch.uint8, device=x.device)
+        workspace = torch.zeros(max(nb, 16), dtype=torch.uint8, device=x.device)
     _check(lib().esb_calibrate_dda(_ptr(x), n, f.c(), _ptr(workspace), workspace.numel(), _ptr(alpha_out),
                                    _ptr(stats_out), _stream(stream)), "esb_calibrate_dda")
     return alpha_out, stats_out
@@ -237,7 +237,7 @@ def esb_project_dda(x: torch.Tensor, f: Fmt, rounding: int = ESB_ROUND_HALF_AWAY
         alpha_out = torch.empty(1, dtype=torch.float32, device=x.device)
     if workspace is None:
         nb = int(lib().esb_calibrate_dda_workspace_bytes(rows * cols))
-        workspace = torch.empty(max(nb, 8), dtype=torch.uint8, device=x.device)
+        workspace = torch.zeros(max(nb, 16), dtype=torch.uint8, device=x.device)
     _check(lib().esb_project_dda(_ptr(x2), rows, cols, f.c(), rounding, _ptr(workspace), workspace.numel(),
                                  _ptr(alpha_out), _ptr(stats_out), _ptr(codes), ldc, _stream(stream)),
            "esb_project_dda")

@@ -186,3 +186,27 @@ def test_project_dda_matches_oracle(dist, shape, fmt, rounding):
         exp = o.project_packed(x.numpy(), ag, b, k, signed, rounding, ld_words=codes.shape[1])
     assert np.array_equal(got, exp)
     assert esb.esb_get_status() == 0
+
+
+def test_workspace_left_zero_and_reusable():
+    # the calibration workspace is zero-filled once; every call leaves its
+    # 32-byte head record zero again, so one workspace serves any sequence
+    # of calibrations and fused projections
+    f = esb.Fmt(4, 2, False)
+    xa = synth.half_normal((3000, 64), seed=41).cuda()
+    xb = synth.half_normal((777, 64), seed=42).cuda()
+    nb = max(esb.esb_calibrate_dda_workspace_bytes(xa.numel()), esb.esb_calibrate_dda_workspace_bytes(xb.numel()))
+    ws = torch.zeros(nb, dtype=torch.uint8, device="cuda")
+    alphas = []
+    for x, fused in [(xa, True), (xb, False), (xa, False), (xb, True), (xa, True)]:
+        if fused:
+            _, a = esb.esb_project_dda(x, f, workspace=ws)
+        else:
+            a, _ = esb.esb_calibrate_dda(x, f, workspace=ws)
+        assert esb.esb_get_status() == 0
+        assert int(ws[:32].cpu().sum()) == 0
+        alphas.append(float(a.item()))
+    fresh_a = float(esb.esb_calibrate_dda(xa, f)[0].item())
+    fresh_b = float(esb.esb_calibrate_dda(xb, f)[0].item())
+    for a, ref in zip(alphas, [fresh_a, fresh_b, fresh_a, fresh_b, fresh_a]):
+        assert abs(a - ref) <= 1e-6 * ref
