@@ -31,6 +31,8 @@
 
 namespace esb {
 
+constexpr int kHaloDecoders = kWsProdWarps - 1;   // bulk path: warps decoding each tile together
+
 struct HaloGeom {
     const uint32_t* X;   // n*h*w pixels of ldx words
     int ldx;             // words per pixel (multiple of 4)
@@ -42,7 +44,9 @@ struct HaloGeom {
     int ns;              // slots per plane (128 + (R-1) * Ws + S - 1)
     int pb;              // bytes per plane (ns * 16)
     int cblocks;         // channel blocks of 16 words
-    int stage_bytes;     // planes of one channel block (<= 8 planes)
+    int stage_bytes;     // planes of one channel block (<= 8 planes), then raw rows
+    int planes_bytes;    // the planes part of a stage
+    int raw_bytes;       // raw code rows of a tile (one channel block only), or 0: register path
 };
 
 // The MMAs of one stage (channel block) with every offset a compile-time
@@ -123,6 +127,75 @@ __device__ __forceinline__ void halo_fill_t(const HaloGeom& g, int p0, const uin
     }
 }
 
+// Bulk-copy fills (one channel block, ldx <= 16 words).  The copy issuer
+// (one thread) copies the input rows of tile T that lie inside the image,
+// whole (w pixels of ldx words, contiguous in NHWC), into the stage's raw
+// area with one cp.async.bulk each, completing on mbarrier `raw_bar`.
+__device__ __forceinline__ void halo_issue_rows(const HaloGeom& g, int64_t T, uint8_t* st, uint64_t* raw_bar)
+{
+    const int nimg = (int)(T / g.tpi);
+    const int p0 = (int)(T - (int64_t)nimg * g.tpi) * g.rows_out;
+    uint8_t* raw = st + g.planes_bytes;
+    const int row_words = g.W * g.ldx;
+    int valid = 0;
+    for (int i = 0; i < g.hr; i++) {
+        const int h = p0 - g.pad + i;
+        valid += (h >= 0 && h < g.H) ? 1 : 0;
+    }
+    mbar_arrive_expect_tx(raw_bar, (uint32_t)(valid * row_words * 4));
+    for (int i = 0; i < g.hr; i++) {
+        const int h = p0 - g.pad + i;
+        if (h >= 0 && h < g.H)
+            bulk_copy_g2s(raw + (size_t)i * row_words * 4, g.X + ((int64_t)nimg * g.H + h) * row_words,
+                          (uint32_t)(row_words * 4), raw_bar);
+    }
+}
+
+// The decoders' share of one bulk-filled tile: slots first, first + stride,
+// ... (zeros for padding slots and rows outside the image).
+template <int NPC>
+__device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint8_t* st, int first, int stride, int k,
+                                              int ew)
+{
+    const int nimg = (int)(T / g.tpi);
+    const int p0 = (int)(T - (int64_t)nimg * g.tpi) * g.rows_out;
+    const uint8_t* raw = st + g.planes_bytes;
+    const int wsm = (1 << g.lws) - 1;
+#pragma unroll 2
+    for (int slot = first; slot < g.ns; slot += stride) {
+        const int rel = slot - g.pad;
+        const int hi = rel >> g.lws;
+        const int j = rel & wsm;
+        const int h = p0 - g.pad + hi;
+        const bool ok = rel >= 0 && hi < g.hr && j < g.W && (unsigned)h < (unsigned)g.H;
+        const uint4* src = reinterpret_cast<const uint4*>(raw + ((size_t)hi * g.W + j) * g.ldx * 4);
+#pragma unroll
+        for (int pc = 0; pc < NPC; pc++) {
+            uint4 c0 = make_uint4(0u, 0u, 0u, 0u), c1 = c0;
+            if (ok) {
+                const uint4 v = src[pc];
+                decode_word_b4(v.x, k, ew, c0.x, c0.y);
+                decode_word_b4(v.y, k, ew, c0.z, c0.w);
+                decode_word_b4(v.z, k, ew, c1.x, c1.y);
+                decode_word_b4(v.w, k, ew, c1.z, c1.w);
+            }
+            uint8_t* dst = st + (2 * pc) * g.pb + slot * 16;
+            *reinterpret_cast<uint4*>(dst) = c0;
+            *reinterpret_cast<uint4*>(dst + g.pb) = c1;
+        }
+    }
+}
+
+__device__ __noinline__ void halo_decode(const HaloGeom g, int64_t T, uint8_t* st, int first, int stride, int k, int ew)
+{
+    switch (g.ldx >> 2) {
+    case 1: halo_decode_t<1>(g, T, st, first, stride, k, ew); break;
+    case 2: halo_decode_t<2>(g, T, st, first, stride, k, ew); break;
+    case 3: halo_decode_t<3>(g, T, st, first, stride, k, ew); break;
+    default: halo_decode_t<4>(g, T, st, first, stride, k, ew); break;
+    }
+}
+
 // Channel block cb (words 16 cb .. of each pixel) of tile T's halo.
 __device__ __noinline__ void halo_fill(const HaloGeom g, int64_t T, int cb, uint8_t* st, int lane, int k, int ew)
 {
@@ -153,7 +226,8 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
     uint64_t* tfull = empty + kWsMaxStages;
     uint64_t* tempty = tfull + 2;
     uint64_t* drain = tempty + 2;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* rawb = drain + 1;                                // kWsMaxStages: bulk-copy fills
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rawb + kWsMaxStages);
     volatile int* err = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int tid = threadIdx.x;
@@ -177,8 +251,10 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
 
     if (tid == 0) {
         for (int s = 0; s < stages; s++) {
-            mbar_init(&full[s], 1);
+            // bulk path: the kKHaloDecoders decoder warps fill a stage together
+            mbar_init(&full[s], g.raw_bytes > 0 ? kHaloDecoders : 1);
             mbar_init(&empty[s], 1);
+            mbar_init(&rawb[s], 1);                   // the issuer's arrive.expect_tx, then the copies' bytes
         }
         for (int a = 0; a < 2; a++) {
             mbar_init(&tfull[a], 1);
@@ -196,13 +272,42 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
 
     if (warp >= kWsProdWarp0) {
         // ---------------------------------------------- halo producers
-        // Warp p fills iterations p, p + nprod, ... of this CTA's (tile,
-        // channel block) sequence; at most `stages` producers are active
-        // (an mbarrier's parity tells apart only adjacent phases).
         const int p = warp - kWsProdWarp0;
+        griddep_wait();                               // X may come from the previous launch
+        if (g.raw_bytes > 0) {
+            // Bulk path, tiles in order: producer warp 0 issues the row copies
+            // of every tile as soon as its stage is free (up to `stages` tiles
+            // ahead); the other kHaloDecoders warps decode each tile together,
+            // so the first tile is ready after one copy and a short decode.
+            int s = 0;
+            uint32_t ph = 0u;
+            if (p == 0) {
+                if (lane == 0) {
+                    for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
+                        if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
+                        halo_issue_rows(g, cta_in_n + ti * ctas_per_n, sA + s * g.stage_bytes, &rawb[s]);
+                        if (++s == stages) { s = 0; ph ^= 1u; }
+                    }
+                }
+            } else {
+                const int d = p - 1;                  // decoder index 0 .. kHaloDecoders - 1
+                for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
+                    if (!wait_or_abort(&rawb[s], ph, err)) { *err = 1; break; }
+                    halo_decode(g, cta_in_n + ti * ctas_per_n, sA + s * g.stage_bytes, d * 32 + lane,
+                                kHaloDecoders * 32, fa.k, fa.ew);
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&full[s]);
+                    if (++s == stages) { s = 0; ph ^= 1u; }
+                }
+            }
+        } else {
+        // Register path (several channel blocks): warp p fills iterations p,
+        // p + nprod, ... of this CTA's (tile, channel block) sequence; at most
+        // `stages` producers are active (an mbarrier's parity tells apart
+        // only adjacent phases).
         const int nprod = stages < kWsProdWarps ? stages : kWsProdWarps;
         const int64_t total_it = (p < nprod) ? my_tiles * cbs : 0;
-        griddep_wait();                               // X may come from the previous launch
         // stage s and its phase ph follow it incrementally (no division in
         // the loop): it advances by nprod <= stages, so s wraps at most once
         int s = p;
@@ -217,6 +322,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
             if (lane == 0) mbar_arrive(&full[s]);
             s += nprod;
             if (s >= stages) { s -= stages; ph ^= 1u; }
+        }
         }
     } else if (warp == kWsMmaWarp) {
         // ---------------------------------------------- MMA issue
@@ -343,7 +449,10 @@ static bool halo_plan(const esb_conv_desc& d, int P, int Q, int64_t ldx, const O
     g.pb = g.ns * 16;
     g.cblocks = (int)((ldx + 15) / 16);
     const int planes = (int)(ldx >= 16 ? 8 : ldx / 2);
-    g.stage_bytes = ((planes * g.pb + 127) / 128) * 128;
+    g.planes_bytes = ((planes * g.pb + 127) / 128) * 128;
+    // one channel block: the fill bulk-copies whole input rows to a raw area of the stage
+    g.raw_bytes = (g.cblocks == 1) ? ((g.hr * d.w * (int)ldx * 4 + 127) / 128) * 128 : 0;
+    g.stage_bytes = g.planes_bytes + g.raw_bytes;
     if ((int64_t)d.n * g.tpi >= (1ll << 30)) return false;
     const int st_smem = halo_static_smem(err);
     if (st_smem < 0) return false;

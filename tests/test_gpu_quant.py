@@ -210,3 +210,23 @@ def test_workspace_left_zero_and_reusable():
     fresh_b = float(esb.esb_calibrate_dda(xb, f)[0].item())
     for a, ref in zip(alphas, [fresh_a, fresh_b, fresh_a, fresh_b, fresh_a]):
         assert abs(a - ref) <= 1e-6 * ref
+
+
+def test_sharded_calibration_from_device_statistics():
+    # per-shard statistics from the device (esb_calibrate_dda stats_out),
+    # combined on the host (shard.combine_dda_stats), against the oracle on
+    # the whole tensor
+    from paper_2109_03513_gb300 import shard
+    for signed, x in [(True, synth.normal((200003,), seed=21, mean=2.0)), (False, synth.half_normal((131072,), seed=22))]:
+        f = esb.Fmt(4, 2, signed)
+        cuts = [0, 50000, 50001, x.numel()]
+        stats = []
+        for i in range(3):
+            st = torch.zeros(3, dtype=torch.float64, device="cuda")
+            esb.esb_calibrate_dda(x[cuts[i]:cuts[i + 1]].contiguous().cuda(), f, stats_out=st)
+            stats.append(st.cpu().numpy())
+        n, mean, spread = shard.combine_dda_stats(stats, signed)
+        a = shard.dda_alpha(esb.esb_alpha_star(4, 2)[0], spread)
+        a_ref, st_ref = o.calibrate(x.numpy(), 4, 2, signed)
+        assert n == x.numel()
+        assert abs(a - a_ref) <= 1e-6 * a_ref
