@@ -206,6 +206,26 @@ __device__ __forceinline__ uint32_t project_by_table(float x, const float* T, co
     return mag | (sign << (p.b - 1));
 }
 
+// The same for a compile-time width B: the b - 1 levels of the search are
+// unrolled (the 2^(B-1) - 1 <= 127 thresholds are in shared memory; for
+// B <= 6 they sit in distinct banks, so lanes never conflict).
+template <int B>
+__device__ __forceinline__ uint32_t project_by_table_t(float x, const float* T, const ProjParams& p)
+{
+    constexpr int L = 1 << (B - 1);
+    const uint32_t u = __float_as_uint(x);
+    const uint32_t sign = u >> 31;
+    const float a = __uint_as_float(u & 0x7fffffffu);
+    int j = 0;
+#pragma unroll
+    for (int step = L >> 1; step > 0; step >>= 1)
+        j += (a >= T[j + step - 1]) ? step : 0;
+    const int one = 1 << p.k;
+    const uint32_t mag = (j >= one) ? (uint32_t)(j - one) : (((uint32_t)p.N << p.k) | (uint32_t)j);
+    const bool zero = j == 0 || (sign && !p.is_signed);        // zero (and NaN) carry sign 0
+    return zero ? p.zero_code : (mag | (sign << (B - 1)));
+}
+
 // The same with the table in registers for b = 4 (7 thresholds).
 struct Thr7 { float t[7]; };
 

@@ -146,7 +146,7 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
 #pragma unroll
         for (int i = 0; i < 7; i++) t7.t[i] = T[i];
     }
-    auto proj = [&](float xv) -> uint32_t { return B == 4 ? project_by_thr7(xv, t7, p) : project_by_table(xv, T, p); };
+    auto proj = [&](float xv) -> uint32_t { return B == 4 ? project_by_thr7(xv, t7, p) : project_by_table_t<B>(xv, T, p); };
 
     if (B == 4 && flat) {                                 // flat codes: coalesced warp tiles
         if (p.is_signed) project_flat_b4<true, true>(x, rows * cols, t7, p.k, codes);
@@ -222,7 +222,7 @@ project_any_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
 #pragma unroll
         for (int j = 0; j < CPW; j++) {
             const int64_t c = w * CPW + j;
-            const uint32_t code = (c < cols) ? project_by_table(x[r * ldx + c], T, p) : p.zero_code;
+            const uint32_t code = (c < cols) ? project_by_table_t<B>(x[r * ldx + c], T, p) : p.zero_code;
             word |= code << (B * j);
         }
         codes[u] = word;  // row-major: r * ldc + w == u
@@ -737,7 +737,7 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
                 for (int w = 0; w < 4; w++) {
                     uint32_t word = 0;
 #pragma unroll
-                    for (int j = 0; j < CPW; j++) word |= project_by_table(v[w * CPW + j], T, p) << (B * j);
+                    for (int j = 0; j < CPW; j++) word |= project_by_table_t<B>(v[w * CPW + j], T, p) << (B * j);
                     out[w] = word;
                 }
             }
@@ -748,7 +748,7 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
 #pragma unroll
                 for (int j = 0; j < CPW; j++) {
                     const int64_t c = c0 + w * CPW + j;
-                    const uint32_t code = (c < cols) ? project_by_table(__ldcs(xr + w * CPW + j), T, p) : p.zero_code;
+                    const uint32_t code = (c < cols) ? project_by_table_t<B>(__ldcs(xr + w * CPW + j), T, p) : p.zero_code;
                     word |= code << (B * j);
                 }
                 out[w] = word;
