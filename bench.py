@@ -18,8 +18,10 @@ entry points (esb_calibrate_dda, esb_project), as a deployed layer stores
 W already in ESB codes.
 Consecutive steps take their input from a rotation of NBATCH seeded
 batches whose fp32 activations together exceed the 129 MB L2 (no step
-finds its input in L2); the K timed steps are bracketed by CUDA events on
-the launching stream.  `value` is conv TOPS over the whole step (2 ops per
+finds its input in L2).  One CUDA graph holds NBATCH consecutive steps (so
+kernel boundaries inside it keep their programmatic launch edges); the K
+timed steps are K // NBATCH replays of it plus a graph of the remaining
+steps, bracketed by CUDA events on the launching stream.  `value` is conv TOPS over the whole step (2 ops per
 MAC).  --impl reference times the CPU oracle instead.
 """
 from __future__ import annotations
@@ -215,18 +217,25 @@ def run_gpu(args):
             for _, fn, _ in calls_for(i):
                 fn()
     torch.cuda.synchronize(dev)
-    graphs = []
-    for i in range(NBATCH):
+    def capture(steps):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            for _, fn, _ in calls_for(i):
-                fn()
-        graphs.append(g)
+            for i in range(steps):
+                for _, fn, _ in calls_for(i):
+                    fn()
+        return g
+
+    # graph_all: NBATCH consecutive steps (batches 0 .. NBATCH-1); graph_one:
+    # the step of batch 0 (end-to-end timing); graph_rem: the first
+    # K % NBATCH steps, so that exactly K steps are timed
+    graph_all = capture(NBATCH)
+    graph_one = capture(1)
+    graph_rem = capture(args.steps % NBATCH) if args.steps % NBATCH else None
     torch.cuda.synchronize(dev)
 
     with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            graphs[i % NBATCH].replay()
+        for i in range((args.warmup + NBATCH - 1) // NBATCH):
+            graph_all.replay()
     torch.cuda.synchronize(dev)
 
     K = args.steps
@@ -239,8 +248,10 @@ def run_gpu(args):
     torch.cuda.synchronize(dev)
     with torch.cuda.stream(stream):
         t0e.record(stream)
-        for i in range(K):
-            graphs[i % NBATCH].replay()
+        for i in range(K // NBATCH):
+            graph_all.replay()
+        if graph_rem is not None:
+            graph_rem.replay()
         t1e.record(stream)
     torch.cuda.synchronize(dev)
     if world > 1:
@@ -281,14 +292,14 @@ def run_gpu(args):
     with torch.cuda.stream(stream):
         for i in range(3):
             X.copy_(x_pin, non_blocking=True)
-            graphs[0].replay()
+            graph_one.replay()
             y_pin.copy_(Yc, non_blocking=True)
         torch.cuda.synchronize(dev)
         a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a0.record(stream)
         for _ in range(ke):
             X.copy_(x_pin, non_blocking=True)
-            graphs[0].replay()
+            graph_one.replay()
             y_pin.copy_(Yc, non_blocking=True)
         a1.record(stream)
         torch.cuda.synchronize(dev)

@@ -212,6 +212,7 @@ __device__ __noinline__ void halo_fill(const HaloGeom g, int64_t T, int cb, uint
     }
 }
 
+template <bool FAST>
 __global__ void __launch_bounds__(kWsThreads, 1)
 esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, OpFmt fb, int BN, int nkb,
                      int stages, int n_tiles, int64_t m_tiles, float acc_scale, EpiParams ep)
@@ -264,17 +265,34 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
         *err = 0;
         fence_mbar_init();
     }
-    __syncthreads();
+    ws_alloc(warp, tmem_slot, tmem_cols);
+    __syncthreads();                                  // barriers initialised, TMEM allocated
+    griddep_wait();                                   // X, B and the alphas may come from the previous launch
+    griddep_launch_dependents();                      // every CTA is resident: the next grid may queue behind it
 
-    uint32_t tmem_base = 0;
-    if (warp < kWsProdWarp0)
-        tmem_base = ws_setup(srcB, n0, K, fb, BN, nkb, sB, thr, ep, tmem_slot, tmem_cols, tid);
+    // Setup.  B is decoded by the MMA warp and the producer warps (all but
+    // the bulk issuer, which starts the first tiles' copies at once); the
+    // MMA warp waits for it on named barrier 1.  The epilogue warps build
+    // the requantisation thresholds meanwhile (named barrier 3), so neither
+    // chain waits for the other.
+    const bool bulk = FAST || g.raw_bytes > 0;
+    const int nbdec = bulk ? 7 * 32 : 8 * 32;
+    if (warp < kWsEpiWarps) {
+        ws_thresholds(thr, ep, warp, lane);
+    } else if (!(bulk && warp == kWsProdWarp0)) {
+        const int t = (bulk && warp > kWsProdWarp0) ? tid - (kWsProdWarp0 + 1) * 32 + 32 : tid - kWsMmaWarp * 32;
+        ws_decode_b<FAST>(srcB, n0, K, fb, BN, nkb, sB, t, nbdec);
+        fence_proxy_async_smem();
+        if (warp == kWsMmaWarp) asm volatile("bar.sync 1, %0;" ::"r"(nbdec) : "memory");
+        else asm volatile("bar.arrive 1, %0;" ::"r"(nbdec) : "memory");
+    }
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
 
     if (warp >= kWsProdWarp0) {
         // ---------------------------------------------- halo producers
         const int p = warp - kWsProdWarp0;
-        griddep_wait();                               // X may come from the previous launch
-        if (g.raw_bytes > 0) {
+        if (bulk) {
             // Bulk path, tiles in order: producer warp 0 issues the row copies
             // of every tile as soon as its stage is free (up to `stages` tiles
             // ahead); the other kHaloDecoders warps decode each tile together,
@@ -391,7 +409,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
             m = ((int64_t)nimg * P + p) * Q + q;
             return q < Q && p < P;
         };
-        ws_epilogue(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
+        ws_epilogue<FAST>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
                     warp, lane);
     }
 
@@ -413,14 +431,17 @@ struct HaloPlan {
     int64_t K, smem;
 };
 
+// Static shared memory of the kernel (the larger of its two instances).
 static int halo_static_smem(cudaError_t* err)
 {
     static int v = -1;
     if (v < 0) {
-        cudaFuncAttributes a;
-        *err = cudaFuncGetAttributes(&a, esb_conv_halo_kernel);
+        cudaFuncAttributes a0, a1;
+        *err = cudaFuncGetAttributes(&a0, esb_conv_halo_kernel<false>);
         if (*err != cudaSuccess) return -1;
-        v = (int)a.sharedSizeBytes;
+        *err = cudaFuncGetAttributes(&a1, esb_conv_halo_kernel<true>);
+        if (*err != cudaSuccess) return -1;
+        v = (int)(a0.sharedSizeBytes > a1.sharedSizeBytes ? a0.sharedSizeBytes : a1.sharedSizeBytes);
     }
     return v;
 }
@@ -495,7 +516,10 @@ bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, i
     hp.g.X = X;
     static bool configured = false;
     if (!configured) {
-        *err = cudaFuncSetAttribute(esb_conv_halo_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        *err = cudaFuncSetAttribute(esb_conv_halo_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    max_dyn_smem() - halo_static_smem(err));
+        if (*err != cudaSuccess) return true;
+        *err = cudaFuncSetAttribute(esb_conv_halo_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     max_dyn_smem() - halo_static_smem(err));
         if (*err != cudaSuccess) return true;
         configured = true;
@@ -509,7 +533,13 @@ bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, i
     const int64_t grid = per_n * n_tiles;
     RowsSrc b{W, (int64_t)d.r * d.s * ldw, N};
     const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
-    *err = launch_pdl(esb_conv_halo_kernel, dim3((unsigned)grid), dim3(kWsThreads), (size_t)hp.smem, st, hp.g, b, N,
+    // The specialised instance: 4-bit B, bulk-copied input rows and 4-bit
+    // codes as the only output, with a scalar scale and bias, in whole N-tiles
+    // and with a monotone requantisation (unsigned codes or an activation).
+    const bool fast = fb.b == 4 && hp.g.raw_bytes > 0 && ep.codes_out && ep.out.b == 4 && !ep.scale && !ep.bias &&
+                      !ep.residual && !ep.acc_out && !ep.y_out && ep.acc_lim > 0.0f && N % hp.BN == 0 &&
+                      (!ep.out.is_signed || ep.act != ESB_ACT_NONE);
+    *err = launch_pdl(fast ? esb_conv_halo_kernel<true> : esb_conv_halo_kernel<false>, dim3((unsigned)grid), dim3(kWsThreads), (size_t)hp.smem, st, hp.g, b, N,
                       hp.K, fa, fb, hp.BN, hp.nkb, hp.stages, n_tiles, m_tiles, acc_scale, ep);
     return true;
 }

@@ -356,14 +356,15 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
         *err = 0;
         fence_mbar_init();
     }
-    __syncthreads();                                  // barriers initialised
+    ws_alloc(warp, tmem_slot, tmem_cols);
+    __syncthreads();                                  // barriers initialised, TMEM allocated
 
     // Producers start loading A at once; meanwhile the MMA and epilogue
-    // warps decode the resident B, allocate TMEM and build the
-    // requantisation thresholds (ws_setup).
+    // warps decode the resident B and build the requantisation thresholds
+    // (ws_setup).
     uint32_t tmem_base = 0;
     if (warp < kWsProdWarp0)
-        tmem_base = ws_setup(srcB, n0, K, fb, BN, nkb, sB, thr, ep, tmem_slot, tmem_cols, tid);
+        tmem_base = ws_setup<false>(srcB, n0, K, fb, BN, nkb, sB, thr, ep, tmem_slot, tid);
 
     if (warp >= kWsProdWarp0) {
         // ---------------------------------------------- A producers
@@ -450,7 +451,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
             m = (first + ti * ctas) * kBM + row;
             return m < M;
         };
-        ws_epilogue(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
+        ws_epilogue<false>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
                     warp, lane);
     }
 

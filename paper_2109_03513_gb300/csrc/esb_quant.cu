@@ -4,6 +4,7 @@
 //   * dequantisation (Sec. IV-A, Eq. q),
 //   * DDA calibration statistics and alpha (Sec. III-D).
 #include <cstdint>
+#include <cstdlib>
 #include <mutex>
 #include <cuda_runtime.h>
 
@@ -392,8 +393,20 @@ __device__ __forceinline__ CalAcc cal_block_reduce(CalAcc A)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) sh[warp] = A;
     __syncthreads();
-    if (threadIdx.x == 0) {
-        for (int w = 1; w < kCalThreads / 32; w++) cal_add(A, sh[w]);
+    if (warp == 0) {
+        // the warp totals, added pairwise by lanes 0-7 (index order fixed)
+        constexpr int kW = kCalThreads / 32;
+        static_assert((kW & (kW - 1)) == 0 && kW <= 32, "warp count");
+        A = sh[lane < kW ? lane : 0];
+#pragma unroll
+        for (int o = 1; o < kW; o <<= 1) {
+            CalAcc B;
+            B.n = __shfl_down_sync(0xffffffffu, A.n, o);
+            B.s1h = __shfl_down_sync(0xffffffffu, A.s1h, o); B.s1l = __shfl_down_sync(0xffffffffu, A.s1l, o);
+            B.s2h = __shfl_down_sync(0xffffffffu, A.s2h, o); B.s2l = __shfl_down_sync(0xffffffffu, A.s2l, o);
+            B.s3h = __shfl_down_sync(0xffffffffu, A.s3h, o); B.s3l = __shfl_down_sync(0xffffffffu, A.s3l, o);
+            cal_add(A, B);
+        }
     }
     return A;
 }
@@ -590,6 +603,18 @@ struct CalSync {
 };
 static_assert(sizeof(CalSync) == sizeof(CalPartial), "head record is one partial record wide");
 
+// Leaving the fused kernel's grid barrier, at the end of the block's work
+// (every block read the release word long before): the last block out
+// returns the sync words to zero.
+__device__ __forceinline__ void cal_depart(CalSync* sync)
+{
+    if (threadIdx.x == 0 && atomicAdd(&sync->depart, 1u) == gridDim.x - 1) {
+        sync->ticket = 0u;
+        sync->release = 0ull;
+        sync->depart = 0u;
+    }
+}
+
 // One launch: every block writes its partial record; the block that takes
 // the last ticket (the ticket word is zeroed by a memset before the launch)
 // adds all records in index order and finalises alpha.
@@ -615,8 +640,8 @@ calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalParti
 
 // ------------------------------------- DDA-calibrated projection, fused
 
-// Calibration and projection of the same tensor in one cooperative launch
-// (all blocks co-resident).  Phase 1 reduces the statistics with loads that
+// Calibration and projection of the same tensor in one launch of one
+// resident wave (all blocks co-resident).  Phase 1 reduces the statistics with loads that
 // leave x in L2; the last block to arrive finalises alpha, publishes it and
 // raises the release flag, which every other block waits for (bounded).
 // Phase 2 projects x, now read from L2, with that alpha.
@@ -630,6 +655,7 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
     // stash: stash_g granules (512 bytes each) per warp of dynamic shared memory
     extern __shared__ float4 stash_all[];
     float4* stash = stash_g > 0 ? stash_all + (size_t)(threadIdx.x >> 5) * stash_g * 32 : nullptr;
+    griddep_wait();                                   // x and the workspace may be in use by the previous launch
     constexpr int CPW = 32 / B;
     constexpr int L = 1 << (B - 1);
     const int64_t n = rows * cols;
@@ -675,21 +701,13 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
         }
         s_alpha = __uint_as_float((unsigned int)(w & 0xffffffffull));
     }
-    if (threadIdx.x == 0 && !timed_out) {
-        // leave the barrier; the last block out returns the words to zero
-        if (atomicAdd(&sync->depart, 1u) == gridDim.x - 1) {
-            sync->ticket = 0u;
-            sync->release = 0ull;
-            sync->depart = 0u;
-        }
-    }
     __syncthreads();
     if (timed_out) {
         if (threadIdx.x == 0) record_status(status, ESB_ERR_TIMEOUT);
         return;
     }
     const float a = s_alpha;
-    // every block is resident (cooperative launch) and past the barrier: a
+    // every block is resident and past the barrier: a
     // dependent grid may take the SMs as these blocks finish
     griddep_launch_dependents();
     build_thresholds(T, p, a, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
@@ -701,6 +719,7 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
         if (flat) {                                     // flat codes: the statistics pass's granules
             if (p.is_signed) project_flat_b4<true, true>(x, n, t7, p.k, codes, stash, stash_g);
             else project_flat_b4<false, true>(x, n, t7, p.k, codes, stash, stash_g);
+            cal_depart(sync);
             return;
         }
     }
@@ -756,6 +775,7 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
         }
         __stcs(reinterpret_cast<uint4*>(codes + r * ldc + (w4 << 2)), make_uint4(out[0], out[1], out[2], out[3]));
     }
+    cal_depart(sync);
 }
 
 // These kernels use almost no shared memory: ask for the largest L1 (the
@@ -839,8 +859,34 @@ static cudaError_t launch_calibrate_project_b(const float* x, int64_t rows, int6
     void* args[] = {(void*)&x, (void*)&rows, (void*)&cols, (void*)&part, (void*)&sync, (void*)&alpha_star,
                     (void*)&p, (void*)&alpha_out, (void*)&stats_out, (void*)&codes, (void*)&ldc, (void*)&status,
                     (void*)&stash_g};
-    e = cudaLaunchCooperativeKernel((const void*)calibrate_project_kernel<B>, dim3((unsigned)g), dim3(kCalThreads),
-                                    args, smem, st);
+    // The grid is one resident wave (sized by the occupancy query above), so
+    // every block becomes resident once the previous kernel of the stream
+    // has left the SMs; the grid barrier's wait is bounded and reports
+    // ESB_ERR_TIMEOUT should another tenant's work keep SMs occupied.  The
+    // launch is programmatic (it may overlap the previous kernel's end; the
+    // kernel's griddep_wait orders its reads and writes after it) rather
+    // than cooperative: a cooperative launch waits for the whole device to
+    // drain first.  ESB_FUSED_COOPERATIVE=1 selects the cooperative launch.
+    static const int coop = [] {
+        const char* v = getenv("ESB_FUSED_COOPERATIVE");
+        return (v && v[0] == '1') ? 1 : 0;
+    }();
+    if (coop) {
+        e = cudaLaunchCooperativeKernel((const void*)calibrate_project_kernel<B>, dim3((unsigned)g), dim3(kCalThreads),
+                                        args, smem, st);
+    } else {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)g);
+        cfg.blockDim = dim3(kCalThreads);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = st;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelExC(&cfg, (const void*)calibrate_project_kernel<B>, args);
+    }
     *launched = true;
     return e;
 }

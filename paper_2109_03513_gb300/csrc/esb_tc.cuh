@@ -370,38 +370,53 @@ static __device__ __noinline__ uint32_t epi_word_b4(const EpiParams* __restrict_
 
 // ------------------------------------ roles of the warp-specialised kernels
 
-// Setup role (warps 0 .. kWsProdWarp0 - 1, while the producers already load
-// A): the MMA warp allocates tmem_cols TMEM columns (before the
-// programmatic-launch wait: it touches no data of earlier launches); all
-// setup warps decode
-// the CTA's N-tile of B (rows n0 .. n0 + BN, every K-block) once into sB in
-// the SW128 K-major layout, and build the requantisation thresholds; then
-// they meet on named barrier 1.  Returns the TMEM base address.
-__device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, int64_t K, const OpFmt& fb, int BN,
-                                             int nkb, uint8_t* sB, float* thr, const EpiParams& ep,
-                                             uint32_t* tmem_slot, uint32_t tmem_cols, int tid)
+// TMEM for the two accumulator buffers, allocated by the MMA warp before the
+// CTA's first barrier (the caller then runs __syncthreads, and ws_setup reads
+// the base address after it).
+__device__ __forceinline__ void ws_alloc(int warp, uint32_t* tmem_slot, uint32_t tmem_cols)
 {
-    constexpr int kSetupThreads = kWsProdWarp0 * 32;
-    const int warp = tid >> 5, lane = tid & 31;
     if (warp == kWsMmaWarp) {
         tmem_alloc(tmem_slot, tmem_cols);
         tc_fence_before();
     }
-    griddep_wait();                                   // B and the alphas may come from the previous launch
-    if (fb.b == 4) {
-        for (int pr = tid; pr < nkb * BN; pr += kSetupThreads) {
-            const int kb = pr / BN, r = pr - kb * BN;
-            const RowsSrc::Row row = srcB.row(n0 + r);
-            const int64_t kw0 = (int64_t)kb * 16;
-            RowsSrc::Cursor cur[4];
+}
+
+// Decode of the CTA's N-tile of B (rows n0 .. n0 + BN, every K-block) once
+// into sB in the SW128 K-major layout, by threads t = 0 .. nthreads - 1 of
+// the calling warps.  B4: B is known to be 4-bit.  The caller fences
+// (fence_proxy_async_smem) and synchronises before the MMA reads sB.
+template <bool B4>
+__device__ __forceinline__ void ws_decode_b(const RowsSrc& srcB, int64_t n0, int64_t K, const OpFmt& fb, int BN,
+                                            int nkb, uint8_t* sB, int t, int nthreads)
+{
+    if (B4 || fb.b == 4) {
+        // two rows per thread and pass, both loaded before either is stored
+        const uint32_t zw = fmt_zero_code(4, fb.k) * 0x11111111u;
+        const int rows_total = nkb * BN;
+        for (int pr0 = t; pr0 < rows_total; pr0 += 2 * nthreads) {
+            uint4 v[2][4];
+            int kbs[2], rs[2];
 #pragma unroll
-            for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
-            uint4 v[4];
-            load_row_b4(srcB, row, cur, kw0, K, fmt_zero_code(4, fb.k) * 0x11111111u, v);
-            store_row_b4(sB + kb * BN * kBK, r, v, kw0, K, fb);
+            for (int u = 0; u < 2; u++) {
+                const int pr = pr0 + u * nthreads;
+                kbs[u] = pr / BN;
+                rs[u] = pr - kbs[u] * BN;
+                if (pr < rows_total) {
+                    const RowsSrc::Row row = srcB.row(n0 + rs[u]);
+                    const int64_t kw0 = (int64_t)kbs[u] * 16;
+                    RowsSrc::Cursor cur[4];
+#pragma unroll
+                    for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
+                    load_row_b4(srcB, row, cur, kw0, K, zw, v[u]);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 2; u++)
+                if (pr0 + u * nthreads < rows_total)
+                    store_row_b4(sB + kbs[u] * BN * kBK, rs[u], v[u], (int64_t)kbs[u] * 16, K, fb);
         }
     } else {
-        for (int u = tid; u < nkb * BN * 8; u += kSetupThreads) {
+        for (int u = t; u < nkb * BN * 8; u += nthreads) {
             const int kb = u / (BN * 8);
             const int rem = u - kb * BN * 8;
             const int r = rem >> 3, g = rem & 7;
@@ -409,12 +424,41 @@ __device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, in
                 decode_unit_any(srcB, srcB.row(n0 + r), (int64_t)kb * kBK + g * 16, K, fb);
         }
     }
-    fence_proxy_async_smem();
+}
+
+// Requantisation thresholds of the output format, built by warps 0-7 (the
+// epilogue warps), which then meet on named barrier 3.
+__device__ __forceinline__ void ws_thresholds(float* thr, const EpiParams& ep, int warp, int lane)
+{
     if (ep.codes_out) {
         const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
-        build_thresholds(thr, ep.out, alpha_out, warp, lane, 0, kWsProdWarp0);
+        build_thresholds(thr, ep.out, alpha_out, warp, lane, 0, kWsEpiWarps);
     }
-    asm volatile("bar.sync 1, %0;" ::"n"(kSetupThreads) : "memory");
+    asm volatile("bar.sync 3, %0;" ::"n"(kWsEpiWarps * 32) : "memory");
+}
+
+// Setup role (warps 0 .. kWsProdWarp0 - 1, while the producers already load
+// A): all setup warps decode B (ws_decode_b); the MMA warp waits for that on
+// named barrier 1 and leaves, while warps 0-7 build the thresholds
+// (ws_thresholds: the MMA does not wait for them).  B4: B is known to be
+// 4-bit.  Returns the TMEM base address (allocated by ws_alloc before the
+// CTA barrier).
+template <bool B4>
+__device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, int64_t K, const OpFmt& fb, int BN,
+                                             int nkb, uint8_t* sB, float* thr, const EpiParams& ep,
+                                             uint32_t* tmem_slot, int tid)
+{
+    constexpr int kSetupThreads = kWsProdWarp0 * 32;
+    const int warp = tid >> 5, lane = tid & 31;
+    griddep_wait();                                   // B and the alphas may come from the previous launch
+    ws_decode_b<B4>(srcB, n0, K, fb, BN, nkb, sB, tid, kSetupThreads);
+    fence_proxy_async_smem();
+    if (warp == kWsMmaWarp) {
+        asm volatile("bar.sync 1, %0;" ::"n"(kSetupThreads) : "memory");
+    } else {
+        asm volatile("bar.arrive 1, %0;" ::"n"(kSetupThreads) : "memory");
+        ws_thresholds(thr, ep, warp, lane);
+    }
     tc_fence_after();
     return *tmem_slot;
 }
@@ -424,8 +468,12 @@ __device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, in
 // ..), and frees the buffer on tempty once its columns are in registers.
 // Warp w reads TMEM lanes 32 (w & 3) .. +31 (= tile rows); with split, warps
 // 0-3 take the columns [0, BN/2) and warps 4-7 [BN/2, BN).  rows(ti, row, m)
-// gives the output row m of a tile row and whether it exists.
-template <class RowMap>
+// gives the output row m of a tile row and whether it exists.  LEAN4: the
+// host has established 4-bit codes as the only output with a scalar scale
+// and bias (every column chunk inside N); the instance then holds just the
+// FMA-pipe requantisation and, for device values that rule it out, the
+// out-of-line per-word path.
+template <bool LEAN4, class RowMap>
 __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* thr, const RowMap& rows,
                                             int64_t my_tiles, int64_t n0, int64_t N, int BN, bool split,
                                             int epi_warps, uint32_t tmem_base, float acc_scale, uint64_t* tfull,
@@ -491,7 +539,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
         uint32_t wsw[4] = {0u, 0u, (uint32_t)(((n0 + c_lo) / cpw) & 0xffffffff),
                            (uint32_t)(((n0 + c_lo) / cpw) >> 32)};   // general path: word, slot, column
         for (int c = c_lo; c < c_hi; c += 16) {
-            if (!swar) {
+            if (!LEAN4 && !swar) {
                 epi_chunk_any(&sh_ep, &sh_cx, taddr + (uint32_t)c, acc_scale, m, mrow, n0 + c, N, wsw);
                 if (c + 16 >= c_hi) {
                     tc_fence_before();
@@ -538,7 +586,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                     }
                     J = (__float_as_uint(jh[0]) & 0xffffu) | (__float_as_uint(jh[1]) << 16);
                     wds[h] = codes8_b4(J, 0u, ep.out.k);
-                } else if (lean && raw_ok) {
+                } else if (!LEAN4 && lean && raw_ok) {
                     // bucket = number of raw thresholds <= raw accumulator
 #pragma unroll
                     for (int j = 0; j < 8; j++) {
@@ -549,7 +597,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                         J |= ((b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u)) << (4 * j);
                     }
                     wds[h] = codes8_b4(J, 0u, ep.out.k);
-                } else if (lean) {
+                } else if (!LEAN4 && lean) {
                     // 4-bit output codes only, scalar scale/bias, no residual:
                     // y = fma(scale * 2^(kA+kB+12), raw, bias) equals
                     // fma(scale, acc, bias) exactly (power-of-two scaling),

@@ -363,3 +363,35 @@ def test_conv_dequant_scale_from_device_alphas():
     yo, co = o.epilogue(acc_o, np.full(cout, sc, np.float32), np.full(cout, -0.01, np.float32), 1, 0.3, (4, 2, False))
     assert np.array_equal(y.cpu().numpy(), yo)
     assert np.array_equal(u32(codes), o.pack(co, 4, 2, ld_words=codes.shape[1]))
+
+
+@pytest.mark.parametrize("alpha_scale", [1.0, 0.0])
+def test_conv_codes_only_from_device_alphas(alpha_scale):
+    # The timed layer's call (codes only, scale from the two device alphas)
+    # through the specialised halo instance; with a zero activation alpha the
+    # folded scale is 0 and the kernel takes its per-word path (every output
+    # is act(bias) requantised).
+    n, h, w, c, cout = 2, 28, 28, 64, 64
+    fu, fs = esb.Fmt(4, 2, False), esb.Fmt(4, 2, True)
+    assert esb.esb_conv2d_kernel(n, h, w, c, cout, 3, 3, 1, 1, fu, fs, out_b=4) == esb.ESB_CONV_KERNEL_HALO
+    x = synth.half_normal((n * h * w, c), seed=31)
+    wt = synth.he_normal((cout * 9, c), fan_in=576, seed=32)
+    xd, wd = x.cuda(), wt.cuda()
+    ax, _ = esb.esb_calibrate_dda(xd, fu)
+    aw, _ = esb.esb_calibrate_dda(wd, fs)
+    Xc = esb.esb_project(xd, fu, alpha=ax)
+    Wc = esb.esb_project(wd, fs, alpha=aw)
+    axe = ax * alpha_scale
+    ep = esb.Epilogue(scale0=1.0, alpha_a_dev=axe, alpha_b_dev=aw, bias0=0.02, act=esb.ESB_ACT_RELU,
+                      alpha_out=0.3, fmt_out=fu)
+    _, _, codes = esb.esb_conv2d_nhwc(Xc, fu, Wc, fs, n, h, w, c, cout, 3, 3, 1, 1, ep=ep, want_acc=False,
+                                      want_codes=True)
+    axh, awh = np.float32(ax.item()), np.float32(aw.item())
+    dq = np.float32(np.float32(np.float32(axh * np.float32(alpha_scale)) * awh) * np.float32(2.0 ** -4))
+    sc = np.float32(np.float32(1.0) * dq)
+    Xo = o.project_packed(x.numpy(), float(axh), 4, 2, False, ld_words=Xc.shape[1])
+    Wo = o.project_packed(wt.numpy(), float(awh), 4, 2, True, ld_words=Wc.shape[1])
+    acc_o = o.conv2d_i64(Xo.reshape(n, h, w, -1), (4, 2), Wo.reshape(cout, 3, 3, -1), (4, 2),
+                         n, h, w, c, cout, 3, 3, 1, 1).reshape(-1, cout)
+    _, co = o.epilogue(acc_o, np.full(cout, sc, np.float32), np.full(cout, 0.02, np.float32), 1, 0.3, (4, 2, False))
+    assert np.array_equal(u32(codes), o.pack(co, 4, 2, ld_words=codes.shape[1]))
