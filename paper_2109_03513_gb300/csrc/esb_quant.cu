@@ -591,6 +591,82 @@ __device__ __forceinline__ CalAcc cal_block_partial(const float* __restrict__ x,
     return cal_block_reduce(A);
 }
 
+// The statistics pass of the fused kernel on a flat tensor: each warp's
+// first min(granules, stash_g) granules -- a contiguous byte range, laid out
+// in the stash exactly as in memory -- arrive by one bulk copy per warp
+// (every byte in flight at once, no registers held), the rest by loads as
+// in cal_block_partial; the statistics of the stashed granules are then
+// read from shared memory.  A copy that does not complete within the wait
+// limit sets *copy_timeout (after a second bounded wait for the copy).
+__device__ __forceinline__ CalAcc cal_block_partial_bulk(const float* __restrict__ x, int64_t n, float4* stash,
+                                                         int stash_g, int* copy_timeout)
+{
+    __shared__ uint64_t wbar[kCalThreads / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t gran = n / 128;
+    int64_t g_lo, g_hi;
+    warp_granules(gran, g_lo, g_hi);
+    const int ns = (int)((g_hi - g_lo) < stash_g ? (g_hi - g_lo) : stash_g);
+    if (lane == 0 && ns > 0) {
+        mbar_init(&wbar[warp], 1);
+        fence_mbar_init();
+        mbar_arrive_expect_tx(&wbar[warp], (uint32_t)ns * 512u);
+        bulk_copy_g2s(stash, x + g_lo * 128, (uint32_t)ns * 512u, &wbar[warp]);
+    }
+    __syncwarp();
+    CalAcc A{0ull, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f, 0.0f};
+    float sa_h = 0.0f, sa_l = 0.0f, sq_h = 0.0f, sq_l = 0.0f;
+    unsigned long long full_groups = 0ull;
+    auto batch = [&](const float4 (&q)[8], int cnt) {
+        if (cnt == 8) {
+            float v[kCalChunk];
+#pragma unroll
+            for (int u = 0; u < 8; u++) { v[4 * u] = q[u].x; v[4 * u + 1] = q[u].y; v[4 * u + 2] = q[u].z; v[4 * u + 3] = q[u].w; }
+            cal_group<kCalChunk>(v, sa_h, sa_l, sq_h, sq_l, A, full_groups);
+        } else {
+#pragma unroll
+            for (int u = 0; u < 8; u++) {
+                if (u < cnt) {
+                    const float v[4] = {q[u].x, q[u].y, q[u].z, q[u].w};
+                    cal_group<4>(v, sa_h, sa_l, sq_h, sq_l, A, full_groups);
+                }
+            }
+        }
+    };
+    // granules past the stash: loads, while the copy is in flight
+    const float4* xv = reinterpret_cast<const float4*>(x) + lane;
+#pragma unroll 1
+    for (int64_t g0 = g_lo + ns; g0 < g_hi; g0 += 8) {
+        const int cnt = (int)((g_hi - g0) < 8 ? (g_hi - g0) : 8);
+        float4 q[8];
+#pragma unroll
+        for (int u = 0; u < 8; u++) q[u] = (u < cnt) ? __ldcs(xv + (g0 + u) * 32) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        batch(q, cnt);
+    }
+    if (ns > 0) {
+        if (!mbar_wait_bounded(&wbar[warp], 0u, 2000000000ull)) {
+            if (lane == 0) *copy_timeout = 1;
+            (void)mbar_wait_bounded(&wbar[warp], 0u, 1000000000ull);
+        }
+#pragma unroll 1
+        for (int g0 = 0; g0 < ns; g0 += 8) {
+            const int cnt = (ns - g0) < 8 ? (ns - g0) : 8;
+            float4 q[8];
+#pragma unroll
+            for (int u = 0; u < 8; u++) q[u] = (u < cnt) ? stash[(g0 + u) * 32 + lane] : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            batch(q, cnt);
+        }
+    }
+    const int64_t rem0 = gran * 128;
+    if (blockIdx.x == 0 && threadIdx.x < 32) {
+        for (int64_t i = rem0 + lane; i < n; i += 32) cal_single(x[i], A);
+    }
+    A.n += full_groups * (unsigned long long)kCalChunk;
+    df_add2(A.s1h, A.s1l, sa_h * kCalChunk, sa_l * kCalChunk);
+    df_add2(A.s2h, A.s2l, sq_h * kCalChunk, sq_l * kCalChunk);
+    return cal_block_reduce(A);
+}
+
 // Workspace head record: the ticket counter, the release flag of the fused
 // kernel's grid barrier, and the alpha it publishes.
 // All three words are zero when a launch starts and zero again when it
@@ -660,10 +736,13 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
     constexpr int L = 1 << (B - 1);
     const int64_t n = rows * cols;
     const bool flat = B == 4 && cols % 8 == 0 && ldc * 8 == cols;
-    const CalPartial mine = cal_block_partial(x, n, 1, false, flat ? stash : nullptr, stash_g);
-    __shared__ int timed_out;
+    __shared__ int copy_timeout, timed_out;
     __shared__ float s_alpha;
     __shared__ float T[L];
+    if (threadIdx.x == 0) { copy_timeout = 0; timed_out = 0; }
+    __syncthreads();
+    const CalPartial mine = (flat && stash) ? cal_block_partial_bulk(x, n, stash, stash_g, &copy_timeout)
+                                            : cal_block_partial(x, n, 1, false, nullptr, 0);
     // Grid barrier: every block publishes its record; the block that takes
     // the last ticket sums the records and publishes alpha in the release
     // word (one 64-bit store: flag and value together), which the others
@@ -673,7 +752,6 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
         part[blockIdx.x] = mine;
         __threadfence();
         is_last = atomicAdd(&sync->ticket, 1u) == gridDim.x - 1;
-        timed_out = 0;
     }
     __syncthreads();
     if (is_last) {
@@ -702,8 +780,9 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
         s_alpha = __uint_as_float((unsigned int)(w & 0xffffffffull));
     }
     __syncthreads();
-    if (timed_out) {
+    if (timed_out || copy_timeout) {
         if (threadIdx.x == 0) record_status(status, ESB_ERR_TIMEOUT);
+        if (!timed_out) cal_depart(sync);
         return;
     }
     const float a = s_alpha;
