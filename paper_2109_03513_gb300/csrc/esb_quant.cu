@@ -48,6 +48,20 @@ __device__ __forceinline__ void project_granule_b4(const float4 q, int64_t g, in
     if ((lane & 1) == 0 && wi < nw) codes[wi] = h | (other << 16);
 }
 
+// One code word (8 values, 2 x float4) of a flat tensor.
+template <bool SIGNED>
+__device__ __forceinline__ uint32_t word_b4(const float4 qa, const float4 qb, const Thr7& t7, int k)
+{
+    const float v[8] = {qa.x, qa.y, qa.z, qa.w, qb.x, qb.y, qb.z, qb.w};
+    uint32_t J = 0u, S = 0u;
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+        J |= bucket7(SIGNED ? fabsf(v[j]) : v[j], t7) << (4 * j);
+        if (SIGNED) S |= (__float_as_uint(v[j]) >> 31) << (4 * j + 3);
+    }
+    return codes8_b4(J, S, k);
+}
+
 // Projection of a flat (row stride = cols, code rows without padding)
 // tensor of n values (n % 8 == 0) to 4-bit codes.  The full granules are
 // split among the warps exactly as in the statistics pass (warp_granules);
@@ -67,9 +81,18 @@ __device__ __forceinline__ void project_flat_b4(const float* __restrict__ x, int
     const int64_t nw = n >> 3;                        // code words
     int64_t g0 = g_lo;
     if (stash) {
-        const int64_t g_st = g_lo + stash_g < g_hi ? g_lo + stash_g : g_hi;
-#pragma unroll 4
-        for (; g0 < g_st; g0++) project_granule_b4<SIGNED>(stash[(g0 - g_lo) * 32 + lane], g0, nw, t7, k, codes);
+        // stashed granules in pairs: lane l makes word l & 15 of granule
+        // l >> 4 of the pair from two float4 (no shuffle, one store)
+        const int ns = (int)(g_hi - g_lo < stash_g ? g_hi - g_lo : stash_g);
+        const int half = lane >> 4, wl = lane & 15;
+        int i = 0;
+#pragma unroll 2
+        for (; i + 2 <= ns; i += 2) {
+            const float4* sp = stash + (i + half) * 32 + 2 * wl;
+            codes[(g_lo + i + half) * 16 + wl] = word_b4<SIGNED>(sp[0], sp[1], t7, k);
+        }
+        for (g0 = g_lo + i; g0 < g_lo + ns; g0++)
+            project_granule_b4<SIGNED>(stash[(g0 - g_lo) * 32 + lane], g0, nw, t7, k, codes);
     }
 #pragma unroll 1
     for (; g0 < g_hi; g0 += 8) {

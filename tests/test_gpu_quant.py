@@ -55,6 +55,26 @@ def test_project_matches_oracle(b, k, signed, rounding):
             assert np.array_equal(u32(codes), exp), (shape, alpha)
 
 
+@pytest.mark.parametrize("k", [0, 1, 2, 3])
+@pytest.mark.parametrize("signed", [True, False])
+def test_project_b4_flat_probes(k, signed):
+    # 4-bit codes of flat tensors take the FMA-pipe bucket search; probes on
+    # and next to every threshold, binade edges, subnormals, infinities and
+    # NaN, for alphas whose thresholds span many binades, and alphas so small
+    # or large that the kernel keeps the compare-based search
+    f = esb.Fmt(4, k, signed)
+    C = o.C_of(4, k)
+    base = np.concatenate([probe_values(4, k), synth.normal((4000,), seed=40 + k).numpy() * np.float32(C)])
+    for alpha in (1.0, 0.7310585, 3.0, 2.0 ** -20, 1e-35, 1e35, 6.0e-8):
+        pts = np.concatenate([base * np.float32(alpha), base]).astype(np.float32)
+        pts = pts[: pts.size // 64 * 64]
+        for shape in ((1, pts.size), (pts.size // 64, 64)):
+            xs = pts.reshape(shape)
+            codes = esb.esb_project(torch.from_numpy(xs).cuda(), f, alpha=alpha)
+            exp = o.project_packed(xs, alpha, 4, k, signed, 0, ld_words=codes.shape[-1])
+            assert np.array_equal(u32(codes), exp), (shape, alpha)
+
+
 def test_project_edge_shapes_and_device_alpha():
     f = esb.Fmt(4, 2, True)
     for rows, cols in [(1, 1), (1, 7), (3, 8), (5, 33), (2, 64), (130, 576)]:
