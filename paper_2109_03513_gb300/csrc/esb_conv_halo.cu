@@ -270,22 +270,22 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
     griddep_wait();                                   // X, B and the alphas may come from the previous launch
     griddep_launch_dependents();                      // every CTA is resident: the next grid may queue behind it
 
-    // Setup.  B is decoded by the MMA warp and the producer warps (all but
-    // the bulk issuer, which starts the first tiles' copies at once); the
-    // MMA warp waits for it on named barrier 1.  The epilogue warps build
-    // the requantisation thresholds meanwhile (named barrier 3), so neither
-    // chain waits for the other.
+    // Setup.  Every warp but the bulk issuer (which starts the first tiles'
+    // row copies at once) decodes its share of B, one row chunk per thread
+    // where it can, so that B is ready after about one load round trip; the
+    // MMA warp waits for all of it on named barrier 1, the others only
+    // arrive.  The epilogue warps then build the requantisation thresholds
+    // (named barrier 3) while the first tile is filled and multiplied.
     const bool bulk = FAST || g.raw_bytes > 0;
-    const int nbdec = bulk ? 7 * 32 : 8 * 32;
-    if (warp < kWsEpiWarps) {
-        ws_thresholds(thr, ep, warp, lane);
-    } else if (!(bulk && warp == kWsProdWarp0)) {
-        const int t = (bulk && warp > kWsProdWarp0) ? tid - (kWsProdWarp0 + 1) * 32 + 32 : tid - kWsMmaWarp * 32;
+    if (!(bulk && warp == kWsProdWarp0)) {
+        const int nbdec = bulk ? kWsThreads - 32 : kWsThreads;
+        const int t = (bulk && warp > kWsProdWarp0) ? tid - 32 : tid;
         ws_decode_b<FAST>(srcB, n0, K, fb, BN, nkb, sB, t, nbdec);
         fence_proxy_async_smem();
         if (warp == kWsMmaWarp) asm volatile("bar.sync 1, %0;" ::"r"(nbdec) : "memory");
         else asm volatile("bar.arrive 1, %0;" ::"r"(nbdec) : "memory");
     }
+    if (warp < kWsEpiWarps) ws_thresholds(thr, ep, warp, lane);
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
