@@ -161,7 +161,7 @@ __device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint
     const int p0 = (int)(T - (int64_t)nimg * g.tpi) * g.rows_out;
     const uint8_t* raw = st + g.planes_bytes;
     const int wsm = (1 << g.lws) - 1;
-#pragma unroll 2
+#pragma unroll 1                                      // compact: it shares the SM's instruction cache
     for (int slot = first; slot < g.ns; slot += stride) {
         const int rel = slot - g.pad;
         const int hi = rel >> g.lws;
@@ -536,9 +536,11 @@ bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, i
     // The specialised instance: 4-bit B, bulk-copied input rows and 4-bit
     // codes as the only output, with a scalar scale and bias, in whole N-tiles
     // and with a monotone requantisation (unsigned codes or an activation).
+    const int half = hp.BN / 2;
+    const bool split = (half % 16 == 0) && (half % ep.out_cpw == 0);
     const bool fast = fb.b == 4 && hp.g.raw_bytes > 0 && ep.codes_out && ep.out.b == 4 && !ep.scale && !ep.bias &&
                       !ep.residual && !ep.acc_out && !ep.y_out && ep.acc_lim > 0.0f && N % hp.BN == 0 &&
-                      (!ep.out.is_signed || ep.act != ESB_ACT_NONE);
+                      (!ep.out.is_signed || ep.act != ESB_ACT_NONE) && (split ? half : hp.BN) % 32 == 0;
     *err = launch_pdl(fast ? esb_conv_halo_kernel<true> : esb_conv_halo_kernel<false>, dim3((unsigned)grid), dim3(kWsThreads), (size_t)hp.smem, st, hp.g, b, N,
                       hp.K, fa, fb, hp.BN, hp.nkb, hp.stages, n_tiles, m_tiles, acc_scale, ep);
     return true;

@@ -470,7 +470,8 @@ __device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, in
 // 0-3 take the columns [0, BN/2) and warps 4-7 [BN/2, BN).  rows(ti, row, m)
 // gives the output row m of a tile row and whether it exists.  LEAN4: the
 // host has established 4-bit codes as the only output with a scalar scale
-// and bias (every column chunk inside N); the instance then holds just the
+// and bias (every column chunk inside N, each warp's columns a multiple of
+// 32); the instance then holds just the
 // FMA-pipe requantisation and, for device values that rule it out, the
 // out-of-line per-word path.
 template <bool LEAN4, class RowMap>
@@ -549,7 +550,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 continue;
             }
             // 4-bit output codes: 32 (or 16) columns per TMEM load
-            const int nc = (c + 32 <= c_hi) ? 32 : 16;
+            const int nc = (LEAN4 || c + 32 <= c_hi) ? 32 : 16;   // LEAN4: whole 32-column chunks
             uint32_t r[32];
             if (nc == 32) {
                 tmem_ld32(taddr + (uint32_t)c, r);
