@@ -702,6 +702,20 @@ struct CalSync {
 };
 static_assert(sizeof(CalSync) == sizeof(CalPartial), "head record is one partial record wide");
 
+// Publishes the block's record and takes a ticket (thread 0); true for the
+// last block.  The ticket's read-modify-write has release and acquire
+// semantics at GPU scope: it releases this block's record, and the last
+// block's thread 0 acquires every earlier record through it; that block's
+// other threads are ordered after it by the CTA barrier that follows, and
+// read the records from L2 (cal_reduce_records).
+__device__ __forceinline__ bool cal_arrive(CalPartial* part, const CalAcc& mine, CalSync* sync)
+{
+    part[blockIdx.x] = mine;
+    unsigned int old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(&sync->ticket) : "memory");
+    return old == gridDim.x - 1;
+}
+
 // Leaving the fused kernel's grid barrier, at the end of the block's work
 // (every block read the release word long before): the last block out
 // returns the sync words to zero.
@@ -724,14 +738,9 @@ calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalParti
 {
     const CalPartial mine = cal_block_partial(x, n, vec, true);
     __shared__ bool is_last;
-    if (threadIdx.x == 0) {
-        part[blockIdx.x] = mine;
-        __threadfence();
-        is_last = atomicAdd(&sync->ticket, 1u) == gridDim.x - 1;
-    }
+    if (threadIdx.x == 0) is_last = cal_arrive(part, mine, sync);
     __syncthreads();
     if (is_last) {
-        __threadfence();
         calibrate_finalize_block(part, gridDim.x, alpha_star, is_signed, alpha_out, stats_out);
         if (threadIdx.x == 0) sync->ticket = 0u;      // every block has counted itself: ready for the next call
     }
@@ -771,14 +780,9 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
     // word (one 64-bit store: flag and value together), which the others
     // wait for (bounded).
     __shared__ bool is_last;
-    if (threadIdx.x == 0) {
-        part[blockIdx.x] = mine;
-        __threadfence();
-        is_last = atomicAdd(&sync->ticket, 1u) == gridDim.x - 1;
-    }
+    if (threadIdx.x == 0) is_last = cal_arrive(part, mine, sync);
     __syncthreads();
     if (is_last) {
-        __threadfence();
         const CalAcc tot = cal_reduce_records(part, gridDim.x);
         if (threadIdx.x == 0) {
             double st[3];
