@@ -321,6 +321,11 @@ __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32
 // an earlier launch may have written, and every write an earlier launch may
 // still read, comes after it.  griddep_launch_dependents: this CTA no longer
 // holds back the launch of a dependent grid.
+// L2 prefetch of the line holding p.  It returns nothing to the SM, so it
+// may be issued before griddep_wait: the loads after the wait still read
+// whatever the previous grid leaves in L2, the point of coherence.
+__device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
+
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 

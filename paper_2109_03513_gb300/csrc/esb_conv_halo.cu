@@ -250,6 +250,14 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
         return;
     }
 
+    {
+        // the CTA's rows of B into L2 while the previous grid may still be
+        // finishing (weights are often no longer in L2 by the next call)
+        const int64_t rows_b = (srcB.rows - n0) < (int64_t)BN ? (srcB.rows - n0) : (int64_t)BN;
+        const char* b0 = reinterpret_cast<const char*>(srcB.base + n0 * srcB.ld);
+        const int64_t bytes = rows_b > 0 ? rows_b * srcB.ld * 4 : 0;
+        for (int64_t off = (int64_t)tid * 128; off < bytes; off += (int64_t)kWsThreads * 128) prefetch_l2(b0 + off);
+    }
     if (tid == 0) {
         for (int s = 0; s < stages; s++) {
             // bulk path: the kKHaloDecoders decoder warps fill a stage together
