@@ -390,30 +390,21 @@ __device__ __forceinline__ void ws_decode_b(const RowsSrc& srcB, int64_t n0, int
                                             int nkb, uint8_t* sB, int t, int nthreads)
 {
     if (B4 || fb.b == 4) {
-        // two rows per thread and pass, both loaded before either is stored
+        // one row chunk per thread and pass (compact: this code runs cold,
+        // once per CTA, on the path to the first MMA)
         const uint32_t zw = fmt_zero_code(4, fb.k) * 0x11111111u;
         const int rows_total = nkb * BN;
-        for (int pr0 = t; pr0 < rows_total; pr0 += 2 * nthreads) {
-            uint4 v[2][4];
-            int kbs[2], rs[2];
+#pragma unroll 1
+        for (int pr = t; pr < rows_total; pr += nthreads) {
+            const int kb = pr / BN, r = pr - kb * BN;
+            const RowsSrc::Row row = srcB.row(n0 + r);
+            const int64_t kw0 = (int64_t)kb * 16;
+            RowsSrc::Cursor cur[4];
 #pragma unroll
-            for (int u = 0; u < 2; u++) {
-                const int pr = pr0 + u * nthreads;
-                kbs[u] = pr / BN;
-                rs[u] = pr - kbs[u] * BN;
-                if (pr < rows_total) {
-                    const RowsSrc::Row row = srcB.row(n0 + rs[u]);
-                    const int64_t kw0 = (int64_t)kbs[u] * 16;
-                    RowsSrc::Cursor cur[4];
-#pragma unroll
-                    for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
-                    load_row_b4(srcB, row, cur, kw0, K, zw, v[u]);
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < 2; u++)
-                if (pr0 + u * nthreads < rows_total)
-                    store_row_b4(sB + kbs[u] * BN * kBK, rs[u], v[u], (int64_t)kbs[u] * 16, K, fb);
+            for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
+            uint4 v[4];
+            load_row_b4(srcB, row, cur, kw0, K, zw, v);
+            store_row_b4(sB + kb * BN * kBK, r, v, kw0, K, fb);
         }
     } else {
         for (int u = t; u < nkb * BN * 8; u += nthreads) {
