@@ -541,7 +541,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 continue;
             }
             // 4-bit output codes: 32 (or 16) columns per TMEM load
-            const int nc = (LEAN4 || c + 32 <= c_hi) ? 32 : 16;   // LEAN4: whole 32-column chunks
+            const int nc = LEAN4 ? 16 : ((c + 32 <= c_hi) ? 32 : 16);   // LEAN4: 16 columns a load (compact code)
             uint32_t r[32];
             if (nc == 32) {
                 tmem_ld32(taddr + (uint32_t)c, r);
