@@ -225,9 +225,14 @@ esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx,
 
 /* DDA-calibrated projection of one tensor: the statistics and alpha of
  * esb_calibrate_dda (Sec. III-D), then esb_project of the same tensor with
- * that alpha (Eq. cheap_projection), in one cooperative launch: each
- * warp keeps its share of the tensor on chip (shared memory) between the
- * two passes, so x is read from memory once.
+ * that alpha (Eq. cheap_projection), in one launch of one resident wave
+ * with a grid barrier between the passes: each warp keeps its share of the
+ * tensor on chip (shared memory) between them, so x is read from memory
+ * once.  The barrier needs every block resident; its wait is bounded, and
+ * should another tenant's work keep SMs occupied for seconds the call
+ * reports ESB_ERR_TIMEOUT through esb_get_status.  (ESB_FUSED_COOPERATIVE=1
+ * in the environment selects a cooperative launch, which waits for the
+ * whole device instead.)
  *   x          [device] rows x cols floats, contiguous (row stride cols)
  *   workspace  [device] >= esb_calibrate_dda_workspace_bytes(rows * cols),
  *              16-byte aligned, zero-filled before its first use, as for
