@@ -278,6 +278,28 @@ esb_status esb_gemm(int64_t M, int64_t N, int64_t K,
                     int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
                     void* stream);
 
+/* The same contraction and epilogue as esb_gemm for large operands, with
+ * caller-provided scratch: each operand is first decoded once into a tiled
+ * image of E4M3 bytes in the workspace (tiles of 128 rows of A or 256 rows
+ * of B by 128 codes, each one contiguous block in the MMA operand layout),
+ * then a persistent tcgen05 kernel streams whole tiles into shared memory
+ * by bulk copies.  Arguments, outputs, the exactness bound and the errors
+ * are those of esb_gemm, plus
+ *   workspace  [device] >= esb_gemm_tiled_workspace_bytes(M, N, K) bytes,
+ *              16-byte aligned, contents undefined before and after (the
+ *              call overwrites it)
+ * Shapes the tiled kernel does not take (N < 256, or 256 not a multiple of
+ * the output's codes per word) run esb_gemm's kernels; the workspace is
+ * then unused.  Errors: as esb_gemm, and ALIGN (workspace) or INVALID_ARG
+ * (workspace too small). */
+size_t esb_gemm_tiled_workspace_bytes(int64_t M, int64_t N, int64_t K);
+esb_status esb_gemm_tiled(int64_t M, int64_t N, int64_t K,
+                          const uint32_t* A, int64_t lda, esb_format fa,
+                          const uint32_t* B, int64_t ldb, esb_format fb,
+                          const esb_epilogue* ep,
+                          int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
+                          void* workspace, size_t workspace_bytes, void* stream);
+
 /* ---------------------------------------------------------------- conv */
 
 /* ESB-coded convolution, NHWC (Sec. IV-B: a K x K x c_in x c_out

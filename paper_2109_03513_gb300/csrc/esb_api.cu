@@ -214,10 +214,13 @@ esb_status esb_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 
-esb_status esb_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, esb_format fa,
-                    const uint32_t* B, int64_t ldb, esb_format fb, const esb_epilogue* ep, int32_t* acc_out,
-                    float* y_out, uint32_t* codes_out, int64_t ldo, void* stream)
+// Validation shared by esb_gemm and esb_gemm_tiled: ESB_OK with *run set
+// when there is work to launch.
+static esb_status gemm_check(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, esb_format fa,
+                             const uint32_t* B, int64_t ldb, esb_format fb, const esb_epilogue* ep,
+                             int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo, bool* run)
 {
+    *run = false;
     if (!fmt_ok(fa) || !fmt_ok(fb)) return ESB_ERR_UNSUPPORTED;
     if (M < 0 || N < 0 || K < 0) return ESB_ERR_INVALID_ARG;
     if (lda < words_for(K, fa.b) || ldb < words_for(K, fb.b)) return ESB_ERR_INVALID_ARG;
@@ -233,8 +236,45 @@ esb_status esb_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t 
     if (!acc_out && !y_out && !codes_out) return ESB_OK;
     if (!aligned16(A) || !aligned16(B) || (lda & 3) || (ldb & 3)) return ESB_ERR_ALIGN;
     if (!gemm_pick_ok(N, want_codes ? ep->fmt_out.b : 4)) return ESB_ERR_UNSUPPORTED;
+    *run = true;
+    return ESB_OK;
+}
+
+esb_status esb_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, esb_format fa,
+                    const uint32_t* B, int64_t ldb, esb_format fb, const esb_epilogue* ep, int32_t* acc_out,
+                    float* y_out, uint32_t* codes_out, int64_t ldo, void* stream)
+{
+    bool run = false;
+    const esb_status s = gemm_check(M, N, K, A, lda, fa, B, ldb, fb, ep, acc_out, y_out, codes_out, ldo, &run);
+    if (s != ESB_OK || !run) return s;
     GemmOutputs o{ep, acc_out, y_out, codes_out, ldo};
     cudaError_t e = launch_gemm(M, N, K, A, lda, fa.b, fa.k, B, ldb, fb.b, fb.k, o, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+size_t esb_gemm_tiled_workspace_bytes(int64_t M, int64_t N, int64_t K)
+{
+    return (M > 0 && N > 0 && K > 0) ? gemm_tiled_workspace_bytes(M, N, K) : 0;
+}
+
+esb_status esb_gemm_tiled(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, esb_format fa,
+                          const uint32_t* B, int64_t ldb, esb_format fb, const esb_epilogue* ep, int32_t* acc_out,
+                          float* y_out, uint32_t* codes_out, int64_t ldo, void* workspace, size_t workspace_bytes,
+                          void* stream)
+{
+    bool run = false;
+    const esb_status s = gemm_check(M, N, K, A, lda, fa, B, ldb, fb, ep, acc_out, y_out, codes_out, ldo, &run);
+    if (s != ESB_OK || !run) return s;
+    GemmOutputs o{ep, acc_out, y_out, codes_out, ldo};
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int out_cpw = codes_out ? 32 / ep->fmt_out.b : 8;
+    if (!gemm_tiled_ok(M, N, K, out_cpw)) {
+        const cudaError_t e = launch_gemm(M, N, K, A, lda, fa.b, fa.k, B, ldb, fb.b, fb.k, o, st);
+        return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+    }
+    if (!workspace || workspace_bytes < gemm_tiled_workspace_bytes(M, N, K)) return ESB_ERR_INVALID_ARG;
+    if (!aligned16(workspace)) return ESB_ERR_ALIGN;
+    const cudaError_t e = launch_gemm_tiled(M, N, K, A, lda, fa.b, fa.k, B, ldb, fb.b, fb.k, o, workspace, st);
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 

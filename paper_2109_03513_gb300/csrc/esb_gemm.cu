@@ -564,7 +564,7 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
 
 // Bound + 2 on |acc| for the epilogue's FMA-pipe requantisation, or 0 when
 // K max|I_A| max|I_B| reaches 2^20.
-static float acc_fma_limit(int64_t K, int ba, int ka, int bb, int kb)
+float acc_fma_limit(int64_t K, int ba, int ka, int bb, int kb)
 {
     const double bound = (double)K * fmt_max_image(ba, ka) * fmt_max_image(bb, kb);
     return bound < 1048576.0 ? (float)(bound + 2.0) : 0.0f;

@@ -1,0 +1,299 @@
+// ESB GEMM for large operands (Sec. III-B products, Sec. IV-B/IV-C
+// computing logic): C[m, n] = sum_k I(A[m, k]) I(B[n, k]) with the fused
+// epilogue, for shapes whose B does not stay resident in shared memory.
+//
+// Two steps on the caller's stream:
+//  1. esb_tile_kernel decodes each operand once into a tiled image of E4M3
+//     bytes in the caller's workspace: tile (rb, kb) holds rows
+//     rb*TH .. rb*TH + TH - 1 and codes 128 kb .. 128 kb + 127 as TH x 128
+//     bytes in the SW128 K-major layout of an MMA operand (row r, 16-byte
+//     chunk g at r*128 + ((g ^ (r & 7)) * 16)); tiles follow in (rb, kb)
+//     order, so every tile is one contiguous block.  Rows past the operand
+//     and codes past K are E4M3 zeros.  HBM-bound: code bytes in, one byte
+//     per code out.
+//  2. esb_gemm_tiled_kernel, persistent and warp-specialised: one producer
+//     thread bulk-copies whole tiles (A: 128 rows, 16 KiB; B: 256 rows,
+//     32 KiB) into a ring of shared-memory stages (cp.async.bulk completing
+//     on mbarriers), the MMA thread issues four 128 x 256 x 32 tcgen05.mma
+//     per K-block into one of two 256-column TMEM accumulators, and eight
+//     epilogue warps drain them through the epilogue of the other tcgen05
+//     kernels (ws_epilogue).  Each CTA keeps one 256-column N-tile and walks
+//     the M-tiles.
+// The contraction is exact under the same bound as esb_gemm (fp32 TMEM
+// accumulation of integer-valued products, K max|I_A| max|I_B| < 2^24).
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "esb_tc.cuh"
+#include "esb_internal.h"
+
+namespace esb {
+
+namespace {
+
+constexpr int kTiledBN = 256;                  // N-tile width (rows of a B tile)
+constexpr int kTiledThreads = 320;             // warps 0-7 epilogue, 8 MMA, 9 producer
+constexpr int kTiledProdWarp = 9;
+constexpr int kTileA = kBM * kBK;              // 16 KiB
+constexpr int kTileB = kTiledBN * kBK;         // 32 KiB
+
+}  // namespace
+
+// One 16-byte chunk (16 codes) per thread and pass: u enumerates (tile,
+// row, physical chunk), so consecutive threads write consecutive bytes.
+__global__ void __launch_bounds__(256) esb_tile_kernel(RowsSrc src, int64_t K, OpFmt f, int TH, int nkb,
+                                                       int64_t rblocks, uint8_t* __restrict__ out)
+{
+    const int64_t total = rblocks * nkb * (int64_t)TH * 8;
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < total; u += (int64_t)gridDim.x * blockDim.x) {
+        const int gp = (int)(u & 7);                         // physical chunk in the 128-byte row
+        const int64_t rt = u >> 3;
+        const int r = (int)(rt % TH);
+        const int64_t t = rt / TH;                           // tile index rb * nkb + kb
+        const int64_t rb = t / nkb;
+        const int kb = (int)(t - rb * nkb);
+        const int g = gp ^ (r & 7);                          // logical chunk: codes 16 g .. 16 g + 15
+        const int64_t row = rb * TH + r;
+        const int64_t k0 = (int64_t)kb * kBK + g * 16;
+        uint4 o = make_uint4(0u, 0u, 0u, 0u);
+        if (row < src.rows && k0 < K) {
+            const RowsSrc::Row rw = src.row(row);
+            if (f.b == 4) {
+                // two words (16 codes) at word k0 / 8 (even: 8-byte aligned);
+                // rows are padded to whole 16-byte groups, so both exist
+                const uint2 w = __ldg(reinterpret_cast<const uint2*>(src.words(rw, k0 >> 3)));
+                uint32_t o0, o1, o2, o3;
+                decode_word_b4(w.x, f.k, f.ew, o0, o1);
+                decode_word_b4(w.y, f.k, f.ew, o2, o3);
+                if (k0 + 16 > K) {                           // K tail: zero the codes past K
+                    uint32_t ml, mh;
+                    int va = (int)(K - k0);
+                    va = va < 0 ? 0 : (va > 8 ? 8 : va);
+                    tail_masks(va, ml, mh);
+                    o0 &= ml; o1 &= mh;
+                    int vb = (int)(K - k0 - 8);
+                    vb = vb < 0 ? 0 : (vb > 8 ? 8 : vb);
+                    tail_masks(vb, ml, mh);
+                    o2 &= ml; o3 &= mh;
+                }
+                o = make_uint4(o0, o1, o2, o3);
+            } else {
+                o = decode_unit_any(src, rw, k0, K, f);
+            }
+        }
+        reinterpret_cast<uint4*>(out + t * (int64_t)TH * kBK + (int64_t)r * kBK)[gp] = o;
+    }
+}
+
+template <bool LEAN4>
+__global__ void __launch_bounds__(kTiledThreads, 1)
+esb_gemm_tiled_kernel(const uint8_t* __restrict__ At, const uint8_t* __restrict__ Bt, int64_t M, int64_t N, int nkb,
+                      int stages, int n_tiles, int64_t m_tiles, float acc_scale, EpiParams ep)
+{
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    constexpr int BN = kTiledBN;
+    constexpr int kStage = kTileA + kTileB;                      // A tile then B tile (both 1024-aligned)
+    float* thr = reinterpret_cast<float*>(smem + stages * kStage);
+    uint64_t* full = reinterpret_cast<uint64_t*>(thr + 128);
+    uint64_t* empty = full + kWsMaxStages;
+    uint64_t* tfull = empty + kWsMaxStages;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* err = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int n_tile = (int)(blockIdx.x % n_tiles);
+    const int64_t cta_in_n = blockIdx.x / n_tiles;
+    const int64_t ctas_per_n = gridDim.x / n_tiles;
+    const int64_t n0 = (int64_t)n_tile * BN;
+    const int64_t my_tiles = (m_tiles > cta_in_n) ? (m_tiles - cta_in_n + ctas_per_n - 1) / ctas_per_n : 0;
+    constexpr uint32_t tmem_cols = 2 * BN;
+    const int half_cols = BN / 2;
+    const bool split = (half_cols % 16 == 0) && (half_cols % ep.out_cpw == 0);
+    const int epi_warps = split ? 8 : 4;
+    // the layout above must fit the dynamic allocation (uniform for the CTA)
+    if ((uintptr_t)(reinterpret_cast<const volatile uint8_t*>(err) + 4 - smem_raw) > dynamic_smem_bytes()) {
+        if (tid == 0) record_status(ep.status, ESB_ERR_INTERNAL);
+        return;
+    }
+    if (tid == 0) {
+        for (int s = 0; s < stages; s++) {
+            mbar_init(&full[s], 1);                      // the producer's arrive.expect_tx, then the copies' bytes
+            mbar_init(&empty[s], 1);                     // the MMA commit that drained it
+        }
+        for (int a = 0; a < 2; a++) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], epi_warps);
+        }
+        mbar_init(drain, 1);
+        *err = 0;
+        fence_mbar_init();
+    }
+    ws_alloc(warp, tmem_slot, tmem_cols);
+    __syncthreads();                                     // barriers initialised, TMEM allocated
+    griddep_wait();                                      // the tiled operands come from the tile kernels
+    if (warp < kWsEpiWarps) ws_thresholds(thr, ep, warp, lane);
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == kTiledProdWarp) {
+        // ---------------------------------------------- producer
+        if (lane == 0) {
+            int s = 0;
+            uint32_t ph = 0u;
+            const uint8_t* bt = Bt + (int64_t)n_tile * nkb * kTileB;
+            for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
+                const uint8_t* at = At + (cta_in_n + ti * ctas_per_n) * nkb * (int64_t)kTileA;
+                for (int kb = 0; kb < nkb; kb++) {
+                    if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
+                    uint8_t* st = smem + s * kStage;
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)kStage);
+                    bulk_copy_g2s(st, at + (int64_t)kb * kTileA, (uint32_t)kTileA, &full[s]);
+                    bulk_copy_g2s(st + kTileA, bt + (int64_t)kb * kTileB, (uint32_t)kTileB, &full[s]);
+                    if (++s == stages) { s = 0; ph ^= 1u; }
+                }
+            }
+        }
+    } else if (warp == kWsMmaWarp) {
+        // ---------------------------------------------- MMA issue
+        if (lane == 0) {
+            const uint32_t idesc = idesc_e4m3_f32(BN);
+            const uint32_t base = smem_u32(smem);
+            int s = 0;
+            uint32_t ph = 0u;
+            for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
+                const int a = (int)(ti & 1);
+                if (!wait_or_abort(&tempty[a], (uint32_t)((ti >> 1) & 1) ^ 1u, err)) { *err = 1; break; }
+                tc_fence_after();
+                const uint32_t d = tmem_base + (uint32_t)(a * BN);
+                uint32_t acc = 0u;
+                for (int kb = 0; kb < nkb; kb++) {
+                    if (!wait_or_abort(&full[s], ph, err)) { *err = 1; break; }
+                    tc_fence_after();
+                    const uint32_t st = base + (uint32_t)(s * kStage);
+                    const uint64_t ad = smem_desc_sw128(st), bd = smem_desc_sw128(st + kTileA);
+                    // four K steps of 32 codes: 32 bytes along the swizzled row
+                    mma_f8f6f4(d, ad, bd, idesc, acc);
+                    mma_f8f6f4(d, ad + 2, bd + 2, idesc, 1u);
+                    mma_f8f6f4(d, ad + 4, bd + 4, idesc, 1u);
+                    mma_f8f6f4(d, ad + 6, bd + 6, idesc, 1u);
+                    acc = 1u;
+                    mma_commit(&empty[s]);
+                    if (++s == stages) { s = 0; ph ^= 1u; }
+                }
+                if (*err) break;
+                mma_commit(&tfull[a]);
+            }
+            ws_drain(drain, err);
+        }
+    } else if (warp < epi_warps) {
+        // ---------------------------------------------- epilogue
+        const int64_t first = cta_in_n, ctas = ctas_per_n;
+        auto rows = [=](int64_t ti, int row, int64_t& m) -> bool {
+            m = (first + ti * ctas) * kBM + row;
+            return m < M;
+        };
+        ws_epilogue<LEAN4>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty,
+                           err, warp, lane);
+    }
+
+    __syncthreads();
+    if (*err && tid == 0) record_status(ep.status, ESB_ERR_TIMEOUT);
+    if (warp == kWsMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, tmem_cols);
+    }
+}
+
+// ------------------------------------------------------------- host side
+
+static int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+size_t gemm_tiled_workspace_bytes(int64_t M, int64_t N, int64_t K)
+{
+    const int64_t nkb = cdiv(K, kBK);
+    return (size_t)(cdiv(M, kBM) * nkb * kTileA + cdiv(N, kTiledBN) * nkb * kTileB);
+}
+
+bool gemm_tiled_ok(int64_t M, int64_t N, int64_t K, int out_cpw)
+{
+    return M > 0 && N >= kTiledBN && K > 0 && kTiledBN % out_cpw == 0;
+}
+
+static int tiled_static_smem(cudaError_t* err)
+{
+    static int v = -1;
+    if (v < 0) {
+        cudaFuncAttributes a0, a1;
+        *err = cudaFuncGetAttributes(&a0, esb_gemm_tiled_kernel<false>);
+        if (*err != cudaSuccess) return -1;
+        *err = cudaFuncGetAttributes(&a1, esb_gemm_tiled_kernel<true>);
+        if (*err != cudaSuccess) return -1;
+        v = (int)(a0.sharedSizeBytes > a1.sharedSizeBytes ? a0.sharedSizeBytes : a1.sharedSizeBytes);
+    }
+    return v;
+}
+
+static cudaError_t launch_tile(const RowsSrc& src, int64_t K, const OpFmt& f, int TH, int nkb, int64_t rblocks,
+                               uint8_t* out, cudaStream_t st)
+{
+    const int64_t total = rblocks * nkb * (int64_t)TH * 8;
+    int64_t grid = cdiv(total, 256);
+    const int64_t cap = (int64_t)device_sm_count() * 8;
+    if (grid > cap) grid = cap;
+    esb_tile_kernel<<<(unsigned)grid, 256, 0, st>>>(src, K, f, TH, nkb, rblocks, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_tiled(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, int ba, int ka,
+                              const uint32_t* B, int64_t ldb, int bb, int kb, const GemmOutputs& o, void* workspace,
+                              cudaStream_t st)
+{
+    EpiParams ep = make_epi(o);
+    ep.dq_pow2 = ldexpf(1.0f, -(ka + kb));
+    ep.acc_lim = acc_fma_limit(K, ba, ka, bb, kb);
+    const OpFmt fa = make_opfmt(ba, ka), fb = make_opfmt(bb, kb);
+    const int nkb = (int)cdiv(K, kBK);
+    const int64_t m_tiles = cdiv(M, kBM), n_tiles = cdiv(N, kTiledBN);
+    uint8_t* At = static_cast<uint8_t*>(workspace);
+    uint8_t* Bt = At + m_tiles * nkb * (int64_t)kTileA;
+    cudaError_t e = launch_tile(RowsSrc{A, lda, M}, K, fa, kBM, nkb, m_tiles, At, st);
+    if (e != cudaSuccess) return e;
+    e = launch_tile(RowsSrc{B, ldb, N}, K, fb, kTiledBN, nkb, n_tiles, Bt, st);
+    if (e != cudaSuccess) return e;
+
+    const int st_smem = tiled_static_smem(&e);
+    if (st_smem < 0) return e;
+    const int maxs = max_dyn_smem() - st_smem;
+    const int64_t fixed = 1024 + 4 * 128 + 512;
+    int stages = (int)((maxs - fixed) / (kTileA + kTileB));
+    if (stages > kWsMaxStages) stages = kWsMaxStages;
+    if (stages < 2) return cudaErrorInvalidConfiguration;
+    const size_t smem = (size_t)(fixed + (int64_t)stages * (kTileA + kTileB));
+    static bool configured = false;
+    if (!configured) {
+        e = cudaFuncSetAttribute(esb_gemm_tiled_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, maxs);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(esb_gemm_tiled_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, maxs);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    int64_t per_n = device_sm_count() / n_tiles;
+    if (per_n < 1) per_n = 1;
+    if (per_n > m_tiles) per_n = m_tiles;
+    const int64_t grid = per_n * n_tiles;
+    const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
+    // the specialised epilogue: 4-bit codes as the only output with a scalar
+    // scale and bias, whole N-tiles, a monotone requantisation
+    const bool fast = ep.codes_out && ep.out.b == 4 && !ep.scale && !ep.bias && !ep.residual && !ep.acc_out &&
+                      !ep.y_out && ep.acc_lim > 0.0f && N % kTiledBN == 0 &&
+                      (!ep.out.is_signed || ep.act != ESB_ACT_NONE);
+    return launch_pdl(fast ? esb_gemm_tiled_kernel<true> : esb_gemm_tiled_kernel<false>, dim3((unsigned)grid),
+                      dim3(kTiledThreads), smem, st, (const uint8_t*)At, (const uint8_t*)Bt, M, N, nkb, stages,
+                      (int)n_tiles, m_tiles, acc_scale, ep);
+}
+
+}  // namespace esb

@@ -49,6 +49,15 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
                            const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st);
 
 bool gemm_pick_ok(int64_t N, int out_b);
+
+// Large GEMMs (esb_gemm_tiled.cu): both operands decoded once into tiled
+// E4M3 images in the caller's workspace, then a persistent tcgen05 kernel
+// over whole-tile bulk copies.
+size_t gemm_tiled_workspace_bytes(int64_t M, int64_t N, int64_t K);
+bool gemm_tiled_ok(int64_t M, int64_t N, int64_t K, int out_cpw);
+cudaError_t launch_gemm_tiled(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, int ba, int ka,
+                              const uint32_t* B, int64_t ldb, int bb, int kb, const GemmOutputs& o, void* workspace,
+                              cudaStream_t st);
 // Kernel esb_conv2d_nhwc launches for a dense convolution (an
 // esb_conv_kernel value), or -1 when the device cannot be queried.
 int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int kx, int out_b);

@@ -667,6 +667,7 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 int pick_bn(int64_t N, int out_cpw);          // N-tile width (esb_gemm.cu)
 int max_dyn_smem();                           // opt-in shared memory per block
 EpiParams make_epi(const GemmOutputs& o);     // epilogue parameters of a call
+float acc_fma_limit(int64_t K, int ba, int ka, int bb, int kb);   // FMA-pipe requantisation bound (esb_gemm.cu)
 
 // Stride-1 convolution from a decoded input halo (esb_conv_halo.cu).  Returns
 // false, launching nothing, when the shape does not suit it (stride != 1,

@@ -90,6 +90,9 @@ SIGNATURES = {
     "esb_project_dda": (_I32, [_P, _I64, _I64, esb_format, _I32, _P, _SZ, _P, _P, _P, _I64, _P]),
     "esb_dequant": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _P, _I64, _P]),
     "esb_gemm": (_I32, [_I64, _I64, _I64, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
+    "esb_gemm_tiled_workspace_bytes": (_SZ, [_I64, _I64, _I64]),
+    "esb_gemm_tiled": (_I32, [_I64, _I64, _I64, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64,
+                              _P, _SZ, _P]),
     "esb_conv2d_nhwc": (_I32, [_P, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
     "esb_conv2d_kernel": (_I32, [_P, _I64, esb_format, esb_format, _I32, _P]),
     "esb_maxpool_nhwc": (_I32, [_P, _I64, esb_format] + [_I32] * 7 + [_P, _I64, _P]),
@@ -296,11 +299,17 @@ class Epilogue:
         return e
 
 
+def esb_gemm_tiled_workspace_bytes(M: int, N: int, K: int) -> int:
+    return int(lib().esb_gemm_tiled_workspace_bytes(M, N, K))
+
+
 def esb_gemm(A: torch.Tensor, fa: Fmt, B: torch.Tensor, fb: Fmt, K: int, ep: Optional[Epilogue] = None,
              want_acc: bool = True, want_y: bool = False, want_codes: bool = False,
              out_acc: Optional[torch.Tensor] = None, out_y: Optional[torch.Tensor] = None,
-             out_codes: Optional[torch.Tensor] = None, stream=None):
-    """(acc int32 (M,N) | None, y fp32 (M,N) | None, codes int32 (M, ldo) | None)."""
+             out_codes: Optional[torch.Tensor] = None, stream=None, workspace: Optional[torch.Tensor] = None):
+    """(acc int32 (M,N) | None, y fp32 (M,N) | None, codes int32 (M, ldo) | None).
+    With a workspace (a CUDA uint8 tensor of at least
+    esb_gemm_tiled_workspace_bytes(M, N, K) bytes) the call is esb_gemm_tiled."""
     _dev(A, "A"); _dev(B, "B")
     M, lda = A.shape
     N, ldb = B.shape
@@ -312,6 +321,13 @@ def esb_gemm(A: torch.Tensor, fa: Fmt, B: torch.Tensor, fb: Fmt, K: int, ep: Opt
         codes = torch.empty((M, esb_row_words(N, ep.fmt_out.b)), dtype=torch.int32, device=dev)
     ldo = codes.shape[-1] if codes is not None else 0
     epc = ep.c() if ep is not None else None
+    if workspace is not None:
+        _dev(workspace, "workspace")
+        _check(lib().esb_gemm_tiled(M, N, K, _ptr(A), lda, fa.c(), _ptr(B), ldb, fb.c(),
+                                    ctypes.byref(epc) if epc is not None else None,
+                                    _ptr(acc), _ptr(y), _ptr(codes), ldo, _ptr(workspace),
+                                    workspace.numel() * workspace.element_size(), _stream(stream)), "esb_gemm_tiled")
+        return acc, y, codes
     _check(lib().esb_gemm(M, N, K, _ptr(A), lda, fa.c(), _ptr(B), ldb, fb.c(),
                           ctypes.byref(epc) if epc is not None else None,
                           _ptr(acc), _ptr(y), _ptr(codes), ldo, _stream(stream)), "esb_gemm")

@@ -395,3 +395,76 @@ def test_conv_codes_only_from_device_alphas(alpha_scale):
                          n, h, w, c, cout, 3, 3, 1, 1).reshape(-1, cout)
     _, co = o.epilogue(acc_o, np.full(cout, sc, np.float32), np.full(cout, 0.02, np.float32), 1, 0.3, (4, 2, False))
     assert np.array_equal(u32(codes), o.pack(co, 4, 2, ld_words=codes.shape[1]))
+
+
+TILED_CASES = [
+    # (M, N, K, fa, fb): the tiled large-operand path (esb_gemm_tiled)
+    (300, 512, 1000, (4, 2, False), (4, 2, True)),    # ragged M and K tail, two N-tiles
+    (257, 300, 515, (4, 1, True), (4, 2, True)),      # ragged N (last N-tile partly past N)
+    (130, 256, 2000, (6, 3, True), (6, 3, True)),     # 6-bit codes: the general tile decode
+    (520, 768, 128, (3, 1, True), (3, 1, True)),      # one K-block
+    (128, 1024, 4608, (4, 2, False), (4, 2, True)),   # deep K, four N-tiles
+]
+
+
+def tiled_ws(M, N, K):
+    nb = esb.esb_gemm_tiled_workspace_bytes(M, N, K)
+    # garbage in the workspace: the tile pass overwrites every byte it uses
+    return torch.full((max(nb, 16),), 0xA5, dtype=torch.uint8, device="cuda")
+
+
+@pytest.mark.parametrize("M,N,K,fa,fb", TILED_CASES)
+def test_gemm_tiled_matches_oracle(M, N, K, fa, fb):
+    A = random_packed(M, K, fa, seed=M * 5 + K)
+    B = random_packed(N, K, fb, seed=N * 3 + K)
+    fo = (4, 2, False)
+    s0 = np.float32(3e-4)
+    ep = esb.Epilogue(scale0=float(s0), bias0=0.01, act=esb.ESB_ACT_RELU, alpha_out=0.41, fmt_out=esb.Fmt(*fo))
+    acc, y, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(*fa[:2]), dev_i32(B), esb.Fmt(*fb[:2]), K, ep=ep,
+                                 want_acc=True, want_y=True, want_codes=True, workspace=tiled_ws(M, N, K))
+    exp = o.gemm_i64(A, fa[:2], B, fb[:2], M, N, K)
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), exp)
+    yo, co = o.epilogue(exp, np.full(N, s0, np.float32), np.full(N, 0.01, np.float32), 1, 0.41, fo)
+    assert np.array_equal(y.cpu().numpy(), yo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+    assert esb.esb_get_status() == 0
+
+
+@pytest.mark.parametrize("act,fo,bias0,sf", LEAN_CASES[:6])
+def test_gemm_tiled_codes_only(act, fo, bias0, sf):
+    # codes as the only output in whole N-tiles: the specialised epilogue
+    M, N, K = 300, 512, 576
+    fa, fb = (4, 2, False), (4, 2, True)
+    A, aa = projected_packed(synth.half_normal((M, K), seed=M + 9).numpy(), fa, 0)
+    B, ab = projected_packed(synth.he_normal((N, K), fan_in=K, seed=N + 8).numpy(), fb, 0)
+    s = np.float32(esb.default_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2)) * sf)
+    _, _, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(*fa), dev_i32(B), esb.Fmt(*fb), K,
+                               ep=lean_epilogue(fo, act, bias0, s), want_acc=False, want_codes=True,
+                               workspace=tiled_ws(M, N, K))
+    acc_o = o.gemm_i64(A, fa[:2], B, fb[:2], M, N, K)
+    _, co = o.epilogue(acc_o, np.full(N, s, np.float32), np.full(N, bias0, np.float32), act, 0.173, fo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
+def test_gemm_tiled_small_n_falls_back():
+    # N < 256: esb_gemm_tiled runs esb_gemm's kernels and leaves the workspace alone
+    M, N, K = 200, 96, 300
+    A = random_packed(M, K, (4, 2, True), seed=1)
+    B = random_packed(N, K, (4, 2, True), seed=2)
+    ws = torch.zeros(16, dtype=torch.uint8, device="cuda")
+    acc, _, _ = esb.esb_gemm(dev_i32(A), esb.Fmt(4, 2), dev_i32(B), esb.Fmt(4, 2), K, workspace=ws)
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), o.gemm_i64(A, (4, 2), B, (4, 2), M, N, K))
+    assert int(ws.sum()) == 0
+
+
+def test_gemm_tiled_full_size_sampled_rows():
+    # the square 4096^3 sweep size in (4,2): int32 accumulators of sampled
+    # rows against the oracle
+    n = 4096
+    A = random_packed(n, n, (4, 2, False), seed=41)
+    B = random_packed(n, n, (4, 2, True), seed=42)
+    acc, _, _ = esb.esb_gemm(dev_i32(A), esb.Fmt(4, 2), dev_i32(B), esb.Fmt(4, 2), n, workspace=tiled_ws(n, n, n))
+    rows = np.array([0, 1, 127, 128, 2047, 4094, 4095] + list(np.random.default_rng(5).integers(0, n, 9)))
+    exp = o.gemm_i64(A[rows], (4, 2), B, (4, 2), len(rows), n, n)
+    assert np.array_equal(acc.cpu().numpy()[rows].astype(np.int64), exp)
+    assert esb.esb_get_status() == 0
