@@ -283,14 +283,20 @@ esb_status esb_gemm(int64_t M, int64_t N, int64_t K,
  * image of E4M3 bytes in the workspace (tiles of 128 rows of A or 256 rows
  * of B by 128 codes, each one contiguous block in the MMA operand layout),
  * then a persistent tcgen05 kernel streams whole tiles into shared memory
- * by bulk copies.  Arguments, outputs, the exactness bound and the errors
- * are those of esb_gemm, plus
+ * by bulk copies.  Arguments, outputs and errors are those of esb_gemm; the
+ * exactness bound is wider: with K max|I_A| max|I_B| >= 2^24 the kernel
+ * splits K into up to four chunks that each stay below 2^24 (each chunk
+ * exact in fp32) and adds them as integers (the int32 accumulator, and
+ * float(acc) rounded to nearest for the epilogue), so the call takes
+ * K max|I_A| max|I_B| < 2^31 when the chunks fit (four) and the output
+ * codes hold a divisor of 16 per word; RANGE otherwise.  Plus
  *   workspace  [device] >= esb_gemm_tiled_workspace_bytes(M, N, K) bytes,
  *              16-byte aligned, contents undefined before and after (the
  *              call overwrites it)
- * Shapes the tiled kernel does not take (N < 256, or 256 not a multiple of
- * the output's codes per word) run esb_gemm's kernels; the workspace is
- * then unused.  Errors: as esb_gemm, and ALIGN (workspace) or INVALID_ARG
+ * Shapes the tiled kernel does not take (N < 256, 256 not a multiple of the
+ * output's codes per word, or fewer than 2^32 multiply-adds, where the
+ * other kernels finish first) run esb_gemm's kernels; the workspace is then
+ * unused.  Errors: as esb_gemm, and ALIGN (workspace) or INVALID_ARG
  * (workspace too small). */
 size_t esb_gemm_tiled_workspace_bytes(int64_t M, int64_t N, int64_t K);
 esb_status esb_gemm_tiled(int64_t M, int64_t N, int64_t K,

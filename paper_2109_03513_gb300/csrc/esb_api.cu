@@ -215,10 +215,13 @@ esb_status esb_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_
 }
 
 // Validation shared by esb_gemm and esb_gemm_tiled: ESB_OK with *run set
-// when there is work to launch.
+// when there is work to launch.  acc_bound: the exactness bound on
+// K max|I_A| max|I_B| of the path (2^24 for one fp32 accumulation, 2^31
+// for the chunked one of the tiled path, which checks the rest itself).
 static esb_status gemm_check(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, esb_format fa,
                              const uint32_t* B, int64_t ldb, esb_format fb, const esb_epilogue* ep,
-                             int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo, bool* run)
+                             int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo, bool* run,
+                             double acc_bound = 16777216.0)
 {
     *run = false;
     if (!fmt_ok(fa) || !fmt_ok(fb)) return ESB_ERR_UNSUPPORTED;
@@ -229,7 +232,7 @@ static esb_status gemm_check(int64_t M, int64_t N, int64_t K, const uint32_t* A,
     esb_status s = check_epilogue(ep, M, N, want_codes || y_out != nullptr);
     if (s != ESB_OK) return s;
     if (want_codes && ldo < words_for(N, ep->fmt_out.b)) return ESB_ERR_INVALID_ARG;
-    if ((double)K * fmt_max_image(fa.b, fa.k) * fmt_max_image(fb.b, fb.k) >= 16777216.0) return ESB_ERR_RANGE;
+    if ((double)K * fmt_max_image(fa.b, fa.k) * fmt_max_image(fb.b, fb.k) >= acc_bound) return ESB_ERR_RANGE;
     if (M > (int64_t)65535 * 128 * 256 || N > (int64_t)65535 * 16) return ESB_ERR_UNSUPPORTED;
     if (M == 0 || N == 0) return ESB_OK;
     if (!A || !B) return ESB_ERR_INVALID_ARG;
@@ -263,12 +266,15 @@ esb_status esb_gemm_tiled(int64_t M, int64_t N, int64_t K, const uint32_t* A, in
                           void* stream)
 {
     bool run = false;
-    const esb_status s = gemm_check(M, N, K, A, lda, fa, B, ldb, fb, ep, acc_out, y_out, codes_out, ldo, &run);
+    const esb_status s =
+        gemm_check(M, N, K, A, lda, fa, B, ldb, fb, ep, acc_out, y_out, codes_out, ldo, &run, 2147483648.0);
     if (s != ESB_OK || !run) return s;
     GemmOutputs o{ep, acc_out, y_out, codes_out, ldo};
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
     const int out_cpw = codes_out ? 32 / ep->fmt_out.b : 8;
-    if (!gemm_tiled_ok(M, N, K, out_cpw)) {
+    if (!gemm_tiled_ok(M, N, K, fa.b, fa.k, fb.b, fb.k, out_cpw)) {
+        // esb_gemm's kernels: one fp32 accumulation
+        if ((double)K * fmt_max_image(fa.b, fa.k) * fmt_max_image(fb.b, fb.k) >= 16777216.0) return ESB_ERR_RANGE;
         const cudaError_t e = launch_gemm(M, N, K, A, lda, fa.b, fa.k, B, ldb, fb.b, fb.k, o, st);
         return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
     }

@@ -54,7 +54,7 @@ bool gemm_pick_ok(int64_t N, int out_b);
 // E4M3 images in the caller's workspace, then a persistent tcgen05 kernel
 // over whole-tile bulk copies.
 size_t gemm_tiled_workspace_bytes(int64_t M, int64_t N, int64_t K);
-bool gemm_tiled_ok(int64_t M, int64_t N, int64_t K, int out_cpw);
+bool gemm_tiled_ok(int64_t M, int64_t N, int64_t K, int ba, int ka, int bb, int kb, int out_cpw);
 cudaError_t launch_gemm_tiled(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, int ba, int ka,
                               const uint32_t* B, int64_t ldb, int bb, int kb, const GemmOutputs& o, void* workspace,
                               cudaStream_t st);

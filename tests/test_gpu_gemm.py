@@ -407,6 +407,12 @@ TILED_CASES = [
 ]
 
 
+@pytest.fixture
+def tiled_always(monkeypatch):
+    # every shape the tiled kernel takes goes to it (not only the large ones)
+    monkeypatch.setenv("ESB_GEMM_TILED_MIN_MACS", "0")
+
+
 def tiled_ws(M, N, K):
     nb = esb.esb_gemm_tiled_workspace_bytes(M, N, K)
     # garbage in the workspace: the tile pass overwrites every byte it uses
@@ -414,7 +420,7 @@ def tiled_ws(M, N, K):
 
 
 @pytest.mark.parametrize("M,N,K,fa,fb", TILED_CASES)
-def test_gemm_tiled_matches_oracle(M, N, K, fa, fb):
+def test_gemm_tiled_matches_oracle(M, N, K, fa, fb, tiled_always):
     A = random_packed(M, K, fa, seed=M * 5 + K)
     B = random_packed(N, K, fb, seed=N * 3 + K)
     fo = (4, 2, False)
@@ -431,7 +437,7 @@ def test_gemm_tiled_matches_oracle(M, N, K, fa, fb):
 
 
 @pytest.mark.parametrize("act,fo,bias0,sf", LEAN_CASES[:6])
-def test_gemm_tiled_codes_only(act, fo, bias0, sf):
+def test_gemm_tiled_codes_only(act, fo, bias0, sf, tiled_always):
     # codes as the only output in whole N-tiles: the specialised epilogue
     M, N, K = 300, 512, 576
     fa, fb = (4, 2, False), (4, 2, True)
@@ -446,7 +452,7 @@ def test_gemm_tiled_codes_only(act, fo, bias0, sf):
     assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
 
 
-def test_gemm_tiled_small_n_falls_back():
+def test_gemm_tiled_small_n_falls_back(tiled_always):
     # N < 256: esb_gemm_tiled runs esb_gemm's kernels and leaves the workspace alone
     M, N, K = 200, 96, 300
     A = random_packed(M, K, (4, 2, True), seed=1)
@@ -467,4 +473,38 @@ def test_gemm_tiled_full_size_sampled_rows():
     rows = np.array([0, 1, 127, 128, 2047, 4094, 4095] + list(np.random.default_rng(5).integers(0, n, 9)))
     exp = o.gemm_i64(A[rows], (4, 2), B, (4, 2), len(rows), n, n)
     assert np.array_equal(acc.cpu().numpy()[rows].astype(np.int64), exp)
+    assert esb.esb_get_status() == 0
+
+
+@pytest.mark.parametrize("M,N,K", [(200, 256, 6000), (130, 300, 16384)])
+def test_gemm_tiled_chunked_k(M, N, K, tiled_always):
+    # K max|I_A| max|I_B| past 2^24 with 6-bit codes: the K chunks of the
+    # tiled kernel (two, then four with 128-column N-tiles), added as exact
+    # integers; y and codes from float(acc) rounded to nearest
+    f = (6, 3, True)
+    # random codes, except that a band of rows of A and of B holds the code
+    # of the largest image (positive in A, both signs in B): their sums reach
+    # K max|I|^2 > 2^24, the others stay small
+    cmax = max(range(2 ** 6), key=lambda c: o.image(c, 6, 3))
+    cneg = min(range(2 ** 6), key=lambda c: o.image(c, 6, 3))
+    ca = synth.uniform_ints((M, K), 0, 2 ** 6, K + 1)
+    cb = synth.uniform_ints((N, K), 0, 2 ** 6, K + 2)
+    ca[:20] = cmax
+    cb[:10] = cmax
+    cb[10:20] = cneg
+    A = o.pack(ca, 6, 3, ld_words=esb.esb_row_words(K, 6))
+    B = o.pack(cb, 6, 3, ld_words=esb.esb_row_words(K, 6))
+    s0 = np.float32(2e-6)
+    fo = (4, 2, True)
+    ep = esb.Epilogue(scale0=float(s0), bias0=-0.03, act=esb.ESB_ACT_NONE, alpha_out=0.2, fmt_out=esb.Fmt(*fo))
+    with pytest.raises(RuntimeError):           # one fp32 accumulation cannot hold it
+        esb.esb_gemm(dev_i32(A), esb.Fmt(6, 3), dev_i32(B), esb.Fmt(6, 3), K)
+    acc, y, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(6, 3), dev_i32(B), esb.Fmt(6, 3), K, ep=ep, want_acc=True,
+                                 want_y=True, want_codes=True, workspace=tiled_ws(M, N, K))
+    exp = o.gemm_i64(A, (6, 3), B, (6, 3), M, N, K)
+    assert np.abs(exp).max() >= 2 ** 24            # the case needs the chunks
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), exp)
+    yo, co = o.epilogue(exp, np.full(N, s0, np.float32), np.full(N, -0.03, np.float32), 0, 0.2, fo)
+    assert np.array_equal(y.cpu().numpy(), yo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
     assert esb.esb_get_status() == 0
