@@ -469,6 +469,80 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_sweep(args):
+    """The sweeps of the large-operand workloads, one JSON line: esb_gemm_tiled
+    on square M=N=K in {1024, 4096, 8192, 16384} at ESB (4,2) and (6,3)
+    (unsigned A, signed B, codes out), and esb_project on 2^28 fp32 values
+    N(0,1) for every b in 3..6, k in 1..b-1.  Each point: CUDA events over
+    repeated calls after 3 warm-ups (operands larger than L2 from 4096 up;
+    the projection reads 1 GiB per call)."""
+    import torch
+
+    from paper_2109_03513_gb300 import esb, synth
+    import __graft_entry__
+
+    __graft_entry__.build()
+    dev = torch.device("cuda")
+    hbm, bf16, _ = _peaks()
+    fp8 = 2.0 * bf16
+    st, en = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timeit(f, reps):
+        for _ in range(3):
+            f()
+        torch.cuda.synchronize()
+        st.record()
+        for _ in range(reps):
+            f()
+        en.record()
+        torch.cuda.synchronize()
+        return st.elapsed_time(en) / reps * 1e3
+
+    out = []
+    g = torch.Generator().manual_seed(0)
+    for b, k in [(4, 2), (6, 3)]:
+        fu, fs = esb.Fmt(b, k, False), esb.Fmt(b, k, True)
+        for n in [1024, 4096, 8192, 16384]:
+            ld = esb.esb_row_words(n, b)
+            # uniformly drawn codes (sign bit cleared for the unsigned A)
+            ca = torch.randint(0, 2 ** b, (n, n), generator=g, dtype=torch.int64)
+            cb = torch.randint(0, 2 ** b, (n, n), generator=g, dtype=torch.int64)
+            ca &= (1 << (b - 1)) - 1
+            cpw = 32 // b
+
+            def pack(c):
+                c = torch.nn.functional.pad(c, (0, ld * cpw - n)).reshape(n, ld, cpw)
+                sh = torch.arange(cpw, dtype=torch.int64) * b
+                return ((c << sh).sum(-1) & 0xffffffff).to(torch.int64).to(torch.int32)
+
+            A, B = pack(ca).to(dev), pack(cb).to(dev)
+            del ca, cb
+            ep = esb.Epilogue(scale0=1e-4, act=esb.ESB_ACT_RELU, alpha_out=0.3, fmt_out=esb.Fmt(4, 2, False))
+            oc = torch.empty((n, esb.esb_row_words(n, 4)), dtype=torch.int32, device=dev)
+            ws = torch.empty(esb.esb_gemm_tiled_workspace_bytes(n, n, n), dtype=torch.uint8, device=dev)
+            f = lambda: esb.esb_gemm(A, fu, B, fs, n, ep=ep, want_acc=False, want_codes=True, out_codes=oc,
+                                     workspace=ws)
+            reps = max(3, min(200, int(1e11 / (2.0 * n ** 3))))
+            us = timeit(f, reps)
+            tf = 2.0 * n ** 3 / us / 1e6
+            out.append({"gemm": [n, n, n], "fmt": [b, k], "us": round(us, 2), "TFLOP/s": round(tf, 1),
+                        "frac_fp8": round(tf / fp8, 3), "status": esb.esb_get_status()})
+            del A, B, oc, ws
+            torch.cuda.empty_cache()
+    x = synth.normal((1 << 28,), seed=0).to(dev)
+    for b in range(3, 7):
+        for k in range(1, b):
+            f = esb.Fmt(b, k, True)
+            codes = torch.empty((1, esb.esb_row_words(1 << 28, b)), dtype=torch.int32, device=dev)
+            us = timeit(lambda: esb.esb_project(x, f, alpha=0.7, codes=codes), 20)
+            byt = (1 << 28) * (4 + 4 / (32 // b))
+            out.append({"project": 1 << 28, "fmt": [b, k], "us": round(us, 1), "GB/s": round(byt / us / 1e3, 1),
+                        "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
+    print(json.dumps({"workload": "sweeps (esb_gemm_tiled M=N=K, esb_project 2^28)", "peaks": {
+        "hbm_gbs": hbm, "fp8_tflops": fp8, "note": "measured HBM copy; fp8 = 2 x measured bf16 burst"},
+        "results": out}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -476,10 +550,13 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweeps", action="store_true", help="the large-operand sweeps instead of the step")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.sweeps:
+        run_sweep(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)
