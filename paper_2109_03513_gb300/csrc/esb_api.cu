@@ -322,7 +322,9 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d, const uint32_t* X, int64_t ld
     esb_status s = check_epilogue(ep, M, d->cout, want_codes || y_out != nullptr);
     if (s != ESB_OK) return s;
     if (want_codes && ldo < words_for(d->cout, ep->fmt_out.b)) return ESB_ERR_INVALID_ARG;
-    const int64_t K = (int64_t)d->r * d->s * ldx * (32 / fx.b);
+    // the exactness bound counts the r*s*c real terms: padding slots hold the
+    // zero code, whose image is 0
+    const int64_t K = (int64_t)d->r * d->s * d->c;
     if ((double)K * fmt_max_image(fx.b, fx.k) * fmt_max_image(fw.b, fw.k) >= 16777216.0) return ESB_ERR_RANGE;
     if (M == 0) return ESB_OK;
     if (!X || !W) return ESB_ERR_INVALID_ARG;

@@ -641,7 +641,7 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
 {
     EpiParams ep = make_epi(o);
     ep.dq_pow2 = ldexpf(1.0f, -(kx + kw));
-    ep.acc_lim = acc_fma_limit((int64_t)d.r * d.s * ldx * (32 / bx), bx, kx, bw, kw);
+    ep.acc_lim = acc_fma_limit((int64_t)d.r * d.s * d.c, bx, kx, bw, kw);   // padding slots add exact zeros
     const int64_t M = (int64_t)d.n * P * Q;
     const int64_t N = d.cout;
     const int64_t K = (int64_t)d.r * d.s * ldx * (32 / bx);
