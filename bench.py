@@ -473,7 +473,8 @@ def run_sweep(args):
     """The sweeps of the large-operand workloads, one JSON line: esb_gemm_tiled
     on square M=N=K in {1024, 4096, 8192, 16384} at ESB (4,2) and (6,3)
     (unsigned A, signed B, codes out), and esb_project on 2^28 fp32 values
-    N(0,1) for every b in 3..6, k in 1..b-1.  Each point: CUDA events over
+    N(0,1) for every b in 3..6, k in 1..b-1 (`--sweeps gemm` / `--sweeps
+    project` run one half).  Each point: CUDA events over
     repeated calls after 3 warm-ups (operands larger than L2 from 4096 up;
     the projection reads 1 GiB per call)."""
     import torch
@@ -500,7 +501,7 @@ def run_sweep(args):
 
     out = []
     g = torch.Generator().manual_seed(0)
-    for b, k in [(4, 2), (6, 3)]:
+    for b, k in ([(4, 2), (6, 3)] if args.sweeps in ("all", "gemm") else []):
         fu, fs = esb.Fmt(b, k, False), esb.Fmt(b, k, True)
         for n in [1024, 4096, 8192, 16384]:
             ld = esb.esb_row_words(n, b)
@@ -530,7 +531,7 @@ def run_sweep(args):
             del A, B, oc, ws
             torch.cuda.empty_cache()
     x = synth.normal((1 << 28,), seed=0).to(dev)
-    for b in range(3, 7):
+    for b in (range(3, 7) if args.sweeps in ("all", "project") else []):
         for k in range(1, b):
             f = esb.Fmt(b, k, True)
             codes = torch.empty((1, esb.esb_row_words(1 << 28, b)), dtype=torch.int32, device=dev)
@@ -550,7 +551,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--sweeps", action="store_true", help="the large-operand sweeps instead of the step")
+    ap.add_argument("--sweeps", nargs="?", const="all", choices=["all", "gemm", "project"],
+                    help="the large-operand sweeps instead of the step (all, or only the GEMM or projection half)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -226,6 +226,84 @@ __device__ __forceinline__ uint32_t project_by_table_t(float x, const float* T, 
     return zero ? p.zero_code : (mag | (sign << (B - 1)));
 }
 
+// ------------------------------------------------ projection by cells
+//
+// For b = 3 and b >= 5 the bisection above costs b - 1 dependent
+// shared-memory loads per value.  Instead the non-negative fp32 bit patterns are cut into cells
+// of 2^(21-k) patterns (k + 2 leading fraction bits per binade).  Within a
+// binade e of v = |x| / alpha the set's spacing is 2^(e-k) (also below 1),
+// so consecutive thresholds lie at least alpha * 2^(e-k) >= two cells apart
+// for every normal alpha: a cell holds at most one T_j, which the table
+// build checks (and the caller keeps the bisection when it does not hold:
+// subnormal thresholds, thresholds that overflow, tables over capacity).
+// Entry c: the first threshold above the cell's start s_c, and the codes
+// below and at/above it -- the code of x is then one load and one compare.
+__host__ __device__ constexpr int cell_shift(int k) { return 21 - k; }
+
+// Code of bucket j (0 .. L-1) of the non-negative set with the sign bit set
+// where a sign is allowed (signed set, j != 0); the projection ANDs it with
+// the value's sign.
+__device__ __forceinline__ uint32_t bucket_code(int j, const ProjParams& p)
+{
+    if (j == 0) return p.zero_code;
+    const int one = 1 << p.k;
+    const uint32_t mag = (j >= one) ? (uint32_t)(j - one) : (((uint32_t)p.N << p.k) | (uint32_t)j);
+    return mag | (p.is_signed ? (1u << (p.b - 1)) : 0u);
+}
+
+// Build the cell table of the thresholds T (all threads of the block; T is
+// complete and visible).  Returns, identically in every thread, whether the
+// table is usable; then h0 is the first cell's index and hmax the last
+// entry.  The last cell lies above T_(L-2): every number there (and +Inf,
+// and every value clamped to it) takes the top code, NaN the zero code.
+template <int B, int CAP>
+__device__ inline bool build_cells(uint2* cells, int& h0, int& hmax, const float* T, const ProjParams& p)
+{
+    constexpr int L = 1 << (B - 1);
+    const int sh = cell_shift(p.k);
+    const uint32_t tl = __float_as_uint(T[L - 2]);
+    h0 = (int)(__float_as_uint(T[0]) >> sh) - 1;
+    if (h0 < 0) h0 = 0;
+    const int H = (int)(tl >> sh) + 2 - h0;
+    hmax = H - 1;
+    if (tl >= 0x7f800000u || H > CAP) return false;             // uniform across the block
+    bool bad = false;
+    for (int c = threadIdx.x; c < H; c += blockDim.x) {
+        const float s = __uint_as_float((uint32_t)(h0 + c) << sh);
+        int g = 0;                                              // #{T_j <= s_c}
+#pragma unroll
+        for (int step = L >> 1; step > 0; step >>= 1)
+            g += (s >= T[g + step - 1]) ? step : 0;
+        float thr;
+        uint32_t lo, hi;
+        if (c == H - 1) {
+            thr = 0.0f; lo = p.zero_code; hi = bucket_code(L - 1, p);
+        } else if (g == L - 1) {
+            thr = __uint_as_float(0x7f800000u); lo = hi = bucket_code(L - 1, p);
+        } else {
+            if (g + 1 <= L - 2 && T[g + 1] < __uint_as_float((uint32_t)(h0 + c + 1) << sh)) bad = true;
+            thr = T[g]; lo = bucket_code(g, p); hi = bucket_code(g + 1, p);
+        }
+        cells[c] = make_uint2(__float_as_uint(thr), lo | (hi << 16));
+    }
+    return !__syncthreads_or(bad);
+}
+
+// Code of x by the cell table.  amask clears the sign for a signed set; for
+// the unsigned set the raw pattern is used, so negative values (negative as
+// int32) clamp to cell 0, below T_0: the zero code.
+template <int B>
+__device__ __forceinline__ uint32_t project_by_cells(float x, const uint2* cells, int h0, int hmax, int sh,
+                                                     uint32_t amask)
+{
+    const uint32_t u = __float_as_uint(x);
+    const uint32_t ab = u & amask;
+    const int h = min(max(((int)ab >> sh) - h0, 0), hmax);
+    const uint2 e = cells[h];
+    const uint32_t c = (__uint_as_float(ab) >= __uint_as_float(e.x)) ? (e.y >> 16) : e.y;
+    return c & ((u >> (32 - B)) | ((1u << (B - 1)) - 1u));
+}
+
 // The same with the table in registers for b = 4 (7 thresholds).
 struct Thr7 { float t[7]; };
 

@@ -132,7 +132,13 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
 {
     constexpr int CPW = 32 / B;
     constexpr int L = 1 << (B - 1);
+    // b = 3 and b >= 5: one 8-byte cell entry per value instead of b - 1
+    // threshold loads (b = 4 keeps its register bucket search, which is faster
+    // there)
+    constexpr bool CELLS = B == 3 || B >= 5;
+    constexpr int CAP = B <= 6 ? 1024 : 2048;
     __shared__ float T[L];
+    __shared__ uint2 cells[CELLS ? CAP : 1];
     const int64_t upr = ldc >> 2;                 // 4-word units per row
     const int64_t total = rows * upr;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -170,7 +176,10 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
 #pragma unroll
         for (int i = 0; i < 7; i++) t7.t[i] = T[i];
     }
-    auto proj = [&](float xv) -> uint32_t { return B == 4 ? project_by_thr7(xv, t7, p) : project_by_table_t<B>(xv, T, p); };
+    int h0 = 0, hmax = 0;
+    const bool by_cells = CELLS && build_cells<B, CAP>(cells, h0, hmax, T, p);
+    const int sh = cell_shift(p.k);
+    const uint32_t amask = p.is_signed ? 0x7fffffffu : 0xffffffffu;
 
     if (B == 4 && flat) {                                 // flat codes: coalesced warp tiles
         if (p.is_signed) project_flat_b4<true, true>(x, rows * cols, t7, p.k, codes);
@@ -178,50 +187,59 @@ project_vec_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, int6
         return;
     }
 
-    for (; u < total; u += stride) {
-        uint32_t out[4];
-        const int64_t rr = r, ww4 = w4, cc0 = c0;
-        if (full) {
-            if (B == 4) {
-                // buckets of |x| (x for the unsigned set: negatives land in bucket 0)
+    // the loop once per per-value projection (the choice is block-uniform)
+    auto run = [&](auto proj) {
+        for (; u < total; u += stride) {
+            uint32_t out[4];
+            const int64_t rr = r, ww4 = w4, cc0 = c0;
+            if (full) {
+                if (B == 4) {
+                    // buckets of |x| (x for the unsigned set: negatives land in bucket 0)
 #pragma unroll
-                for (int w = 0; w < 4; w++) {
-                    uint32_t J = 0u, S = 0u;
+                    for (int w = 0; w < 4; w++) {
+                        uint32_t J = 0u, S = 0u;
 #pragma unroll
-                    for (int j = 0; j < 8; j++) {
-                        const float xv = v[w * 8 + j];
-                        const uint32_t uxv = __float_as_uint(xv);
-                        J |= bucket7(p.is_signed ? fabsf(xv) : xv, t7) << (4 * j);
-                        S |= ((uxv >> 31) & (uint32_t)p.is_signed) << (4 * j + 3);
+                        for (int j = 0; j < 8; j++) {
+                            const float xv = v[w * 8 + j];
+                            const uint32_t uxv = __float_as_uint(xv);
+                            J |= bucket7(p.is_signed ? fabsf(xv) : xv, t7) << (4 * j);
+                            S |= ((uxv >> 31) & (uint32_t)p.is_signed) << (4 * j + 3);
+                        }
+                        out[w] = codes8_b4(J, S, p.k);
                     }
-                    out[w] = codes8_b4(J, S, p.k);
+                } else {
+#pragma unroll
+                    for (int w = 0; w < 4; w++) {
+                        uint32_t word = 0;
+#pragma unroll
+                        for (int j = 0; j < CPW; j++) word |= proj(v[w * CPW + j]) << (B * j);
+                        out[w] = word;
+                    }
                 }
             } else {
+                const float* xr = x + rr * ldx + cc0;
 #pragma unroll
                 for (int w = 0; w < 4; w++) {
                     uint32_t word = 0;
 #pragma unroll
-                    for (int j = 0; j < CPW; j++) word |= proj(v[w * CPW + j]) << (B * j);
+                    for (int j = 0; j < CPW; j++) {
+                        const int64_t c = cc0 + w * CPW + j;
+                        const uint32_t code = (c < cols) ? proj(__ldcs(xr + w * CPW + j)) : p.zero_code;
+                        word |= code << (B * j);
+                    }
                     out[w] = word;
                 }
             }
-        } else {
-            const float* xr = x + rr * ldx + cc0;
-#pragma unroll
-            for (int w = 0; w < 4; w++) {
-                uint32_t word = 0;
-#pragma unroll
-                for (int j = 0; j < CPW; j++) {
-                    const int64_t c = cc0 + w * CPW + j;
-                    const uint32_t code = (c < cols) ? proj(__ldcs(xr + w * CPW + j)) : p.zero_code;
-                    word |= code << (B * j);
-                }
-                out[w] = word;
-            }
+            fetch(u + stride);
+            __stcs(reinterpret_cast<uint4*>(codes + rr * ldc + (ww4 << 2)), make_uint4(out[0], out[1], out[2], out[3]));
         }
-        fetch(u + stride);
-        __stcs(reinterpret_cast<uint4*>(codes + rr * ldc + (ww4 << 2)), make_uint4(out[0], out[1], out[2], out[3]));
-    }
+    };
+    if (by_cells)
+        run([&](float xv) -> uint32_t { return project_by_cells<B>(xv, cells, h0, hmax, sh, amask); });
+    else
+        run([&](float xv) -> uint32_t {
+            return B == 4 ? project_by_thr7(xv, t7, p) : project_by_table_t<B>(xv, T, p);
+        });
 }
 
 // General path: any alignment and strides; one thread per code word.

@@ -58,7 +58,7 @@ def test_project_matches_oracle(b, k, signed, rounding):
 @pytest.mark.parametrize("k", [0, 1, 2, 3])
 @pytest.mark.parametrize("signed", [True, False])
 def test_project_b4_flat_probes(k, signed):
-    # 4-bit codes of flat tensors take the FMA-pipe bucket search; probes on
+    # 4-bit codes of flat tensors take the warp-tile path; probes on
     # and next to every threshold, binade edges, subnormals, infinities and
     # NaN, for alphas whose thresholds span many binades, and alphas so small
     # or large that the kernel keeps the compare-based search
@@ -73,6 +73,31 @@ def test_project_b4_flat_probes(k, signed):
             codes = esb.esb_project(torch.from_numpy(xs).cuda(), f, alpha=alpha)
             exp = o.project_packed(xs, alpha, 4, k, signed, 0, ld_words=codes.shape[-1])
             assert np.array_equal(u32(codes), exp), (shape, alpha)
+
+
+CELL_FORMATS = ([(3, k) for k in range(3)] + [(5, k) for k in range(5)] + [(6, k) for k in range(6)]
+                + [(7, 0), (7, 3), (7, 5), (7, 6), (8, 0), (8, 4), (8, 6), (8, 7)])
+
+
+@pytest.mark.parametrize("b,k", CELL_FORMATS)
+@pytest.mark.parametrize("signed", [True, False])
+def test_project_cell_table_probes(b, k, signed):
+    # b = 3 and b >= 5 project through the per-block cell table (at most one
+    # threshold per cell of 2^(21-k) fp32 patterns); probes on and next to
+    # every threshold, for alphas that keep the table, and for alphas whose
+    # thresholds overflow or run subnormal (or whose table is over capacity,
+    # (8, 7)), where the block keeps the bisection; both tie rules
+    f = esb.Fmt(b, k, signed)
+    C = o.C_of(b, k)
+    base = np.concatenate([probe_values(b, k), synth.normal((3000,), seed=50 + 8 * b + k).numpy() * np.float32(C)])
+    for alpha in (1.0, 0.7310585, 3.0, 2.0 ** -20, 1e-35, 1e35, 6.0e-8):
+        pts = np.concatenate([base * np.float32(alpha), base]).astype(np.float32)
+        for rounding in (0, 1):
+            for shape in ((1, pts.size), (pts.size // 96, 96)):
+                xs = np.ascontiguousarray(pts[: int(np.prod(shape))].reshape(shape))
+                codes = esb.esb_project(torch.from_numpy(xs).cuda(), f, alpha=alpha, rounding=rounding)
+                exp = o.project_packed(xs, alpha, b, k, signed, rounding, ld_words=codes.shape[-1])
+                assert np.array_equal(u32(codes), exp), (shape, alpha, rounding)
 
 
 def test_project_edge_shapes_and_device_alpha():
