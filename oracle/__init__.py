@@ -12,9 +12,11 @@ Parity status of each function (what pins it, see ``tests/test_oracle_pins.py``)
   set of Fig. 10, linear/PoT/ternary special cases of Sec. III-B, the
   multiplication identity Eq. esb_multiplication over all code pairs).
 * projection -- pinned (worked example of Sec. III-C, equality of the two
-  formulations Eq. thresholing_func / Eq. fast_projection on every fp32 of
-  small formats' ranges, idempotence, symmetry, monotonicity, brute-force
-  nearest search with numpy).
+  formulations Eq. thresholing_func / Eq. fast_projection on a strided sweep
+  of the fp32 patterns of small formats' ranges plus every midpoint and its
+  neighbours, idempotence, symmetry, monotonicity, brute-force nearest
+  search with numpy, and the step-function form the GPU's projection of all
+  2^32 patterns is compared with).
 * alpha*, D -- pinned (all 18 alpha* and DDA values of Table 1; the 3-level
   Lloyd-Max quantizer of N(0,1); the scale identity alpha*(b,b-1) = 2 alpha*(b,b-2)).
 * calibration -- pinned (closed-form moments of constructed inputs).

@@ -5,6 +5,7 @@ import pytest
 import torch
 
 import oracle as o
+from conftest import oracle_step_function, step_function_codes
 from paper_2109_03513_gb300 import esb, synth
 
 pytestmark = pytest.mark.gpu
@@ -98,6 +99,35 @@ def test_project_cell_table_probes(b, k, signed):
                 codes = esb.esb_project(torch.from_numpy(xs).cuda(), f, alpha=alpha, rounding=rounding)
                 exp = o.project_packed(xs, alpha, b, k, signed, rounding, ld_words=codes.shape[-1])
                 assert np.array_equal(u32(codes), exp), (shape, alpha, rounding)
+
+
+EVERY_FP32_CASES = [(2, 0, True, 0, 1.0), (3, 1, True, 0, 3.0), (4, 2, True, 0, 0.7310585), (4, 2, False, 1, 1.0),
+                    (5, 2, False, 0, 0.7310585), (6, 3, True, 1, 0.7310585), (8, 4, True, 0, 0.37), (8, 7, True, 0, 1.0)]
+
+
+@pytest.mark.parametrize("b,k,signed,rounding,alpha", EVERY_FP32_CASES)
+def test_project_every_fp32_pattern(b, k, signed, rounding, alpha):
+    # All 2^32 fp32 bit patterns, projected as flat tensors of 2^26 values
+    # (b = 4: the warp-tile path; b = 3, 5, 6, 8: the cell table; (8, 7) and
+    # (2, 0): the bisection), against the oracle's step function (breakpoints
+    # and bucket codes computed by the oracle alone, see conftest)
+    step = oracle_step_function(alpha, b, k, signed, rounding)
+    f = esb.Fmt(b, k, signed)
+    cpw = 32 // b
+    n = 1 << 26
+    shifts = torch.arange(cpw, device="cuda", dtype=torch.int64) * b
+    codes = torch.empty((1, esb.esb_row_words(n, b)), dtype=torch.int32, device="cuda")
+    for c in range((1 << 32) // n):
+        bits = torch.arange(c * n, (c + 1) * n, dtype=torch.int64, device="cuda")
+        x = torch.where(bits >= (1 << 31), bits - (1 << 32), bits).to(torch.int32).view(torch.float32)
+        esb.esb_project(x, f, alpha=alpha, rounding=rounding, codes=codes)
+        w = codes[0].to(torch.int64) & 0xFFFFFFFF
+        got = ((w[:, None] >> shifts[None, :]) & ((1 << b) - 1)).reshape(-1)[:n]
+        exp = step_function_codes(bits, step)
+        if not torch.equal(got, exp):
+            i = int(torch.nonzero(got != exp)[0, 0])
+            raise AssertionError((hex(c * n + i), int(exp[i]), int(got[i])))
+    assert esb.esb_get_status() == 0
 
 
 def test_project_edge_shapes_and_device_alpha():

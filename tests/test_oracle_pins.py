@@ -12,7 +12,7 @@ import numpy as np
 import pytest
 
 import oracle as o
-from conftest import read_golden
+from conftest import oracle_step_function, read_golden, step_function_codes
 
 ALL_FORMATS = [(b, k) for b in range(2, 9) for k in range(0, b)]
 SMALL_FORMATS = [(b, k) for b in range(2, 7) for k in range(0, b)]
@@ -420,3 +420,29 @@ def test_dD_is_the_derivative_of_D(b, k):
     a_star, _ = o.alpha_star(b, k)
     assert abs(o.dD(a_star, b, k)) < 1e-12
     assert o.dD(a_star * 0.99, b, k) < 0 < o.dD(a_star * 1.01, b, k)
+
+
+STEP_CASES = [(2, 0, True, 0, 1.0), (3, 1, True, 0, 3.0), (4, 2, True, 0, 0.7310585), (4, 2, False, 1, 1.0),
+              (5, 2, False, 0, 0.7310585), (6, 3, True, 1, 0.7310585), (8, 4, True, 0, 0.37), (8, 7, True, 0, 1.0)]
+
+
+@pytest.mark.parametrize("b,k,signed,rounding,alpha", STEP_CASES)
+def test_projection_is_the_step_function_of_its_breakpoints(b, k, signed, rounding, alpha):
+    # The oracle's projection of any fp32 is fixed by the L-1 breakpoints
+    # found from it by bisection (monotone in |x|, symmetric or clamped for
+    # x < 0, NaN alone): checked on random bit patterns, every breakpoint and
+    # its neighbours, and the special values.  The GPU test that projects
+    # every one of the 2^32 patterns compares against this step function.
+    import torch
+    step = oracle_step_function(alpha, b, k, signed, rounding)
+    T = step[0]
+    rng = np.random.default_rng(b * 100 + k)
+    bits = np.concatenate([rng.integers(0, 1 << 32, 1 << 17, dtype=np.int64),
+                           T, T - 1, T + 1, T | (1 << 31), (T - 1) | (1 << 31),
+                           [0, 1 << 31, 0x7F800000, 0xFF800000, 0x7F800001, 0x7FC00000, 0xFFC00000, 1, 0x80000001,
+                            0x7F7FFFFF, 0xFF7FFFFF]]).astype(np.int64)
+    x = bits.astype(np.uint32).view(np.float32)
+    exp = o.project_codes(x, alpha, b, k, signed, rounding).astype(np.int64)
+    got = step_function_codes(torch.from_numpy(bits), step).numpy()
+    bad = np.nonzero(got != exp)[0]
+    assert bad.size == 0, [(hex(int(bits[i])), int(exp[i]), int(got[i])) for i in bad[:5]]
