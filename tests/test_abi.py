@@ -105,6 +105,70 @@ def test_host_validation_without_device(lib):
     assert lib.esb_get_status(null, null) == esb.ESB_ERR_INVALID_ARG
 
 
+def test_host_validation_other_entry_points(lib):
+    # every check below returns before any launch or device query
+    f = esb.esb_format(4, 2, 1)
+    f63 = esb.esb_format(6, 3, 1)
+    null = None
+    fake = ctypes.c_void_p(4096)
+    ep = ctypes.byref(esb.Epilogue().c())
+    R = esb.ESB_ERR_RANGE
+    # tiled GEMM: K max|I_A| max|I_B| < 2^31 for the chunked path ((6,3): 60 x 60)
+    K = 600000                         # 600000 * 3600 >= 2^31
+    ld = esb.esb_row_words(K, 6)
+    assert lib.esb_gemm_tiled(256, 256, K, fake, ld, f63, fake, ld, f63, ep, fake, null, null, 0, fake, 1 << 40,
+                              null) == R
+    # below it the chunked path runs (K past 2^24 / 3600): it needs a workspace
+    K = 8192
+    ld = esb.esb_row_words(K, 6)
+    ws = lib.esb_gemm_tiled_workspace_bytes(256, 256, K)
+    assert ws > 0
+    assert lib.esb_gemm_tiled(256, 256, K, fake, ld, f63, fake, ld, f63, ep, fake, null, null, 0, null, 0,
+                              null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_gemm_tiled(256, 256, K, fake, ld, f63, fake, ld, f63, ep, fake, null, null, 0, fake, ws - 1,
+                              null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_gemm_tiled(256, 256, K, fake, ld, f63, fake, ld, f63, ep, fake, null, null, 0,
+                              ctypes.c_void_p(4104), ws, null) == esb.ESB_ERR_ALIGN
+    # ... which esb_gemm (one fp32 accumulation, bound 2^24) refuses
+    assert lib.esb_gemm(256, 256, K, fake, ld, f63, fake, ld, f63, ep, fake, null, null, 0, null) == R
+    assert lib.esb_gemm_tiled_workspace_bytes(0, 256, K) == 0
+    # fused calibration + projection
+    wsb = lib.esb_calibrate_dda_workspace_bytes(64)
+    assert lib.esb_project_dda(fake, 1, 64, f, 2, fake, wsb, fake, null, fake, 8, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_project_dda(fake, 1, 64, f, 0, fake, wsb - 1, fake, null, fake, 8, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_project_dda(fake, 1, 64, f, 0, ctypes.c_void_p(4100), wsb, fake, null, fake, 8,
+                               null) == esb.ESB_ERR_ALIGN
+    assert lib.esb_project_dda(fake, 1, 64, f, 0, fake, wsb, fake, null, fake, 7, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_project_dda(fake, 0, 64, f, 0, fake, wsb, fake, null, fake, 8, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_project_dda(fake, 1, 64, esb.esb_format(4, 4, 1), 0, fake, wsb, fake, null, fake, 8,
+                               null) == esb.ESB_ERR_UNSUPPORTED
+    # dequantisation
+    assert lib.esb_dequant(fake, 2, 64, 8, 1.0, null, f, fake, 63, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_dequant(fake, 2, 64, 7, 1.0, null, f, fake, 64, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_dequant(fake, 2, 64, 8, -1.0, null, f, fake, 64, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_dequant(fake, 0, 64, 8, 1.0, null, f, fake, 64, null) == esb.ESB_OK
+    # depthwise convolution (groups = C): Cout = C, output width = input width, bound 2^31
+    dw = esb.esb_conv_desc(1, 8, 8, 64, 32, 3, 3, 1, 1, 64)
+    assert lib.esb_conv2d_nhwc(ctypes.byref(dw), fake, 8, f, fake, 8, f, ep, fake, null, null, 0,
+                               null) == esb.ESB_ERR_INVALID_ARG
+    f81 = esb.esb_format(8, 1, 1)      # max|I| = 3 * 2^62: any window exceeds 2^31
+    dw = esb.esb_conv_desc(1, 8, 8, 64, 64, 3, 3, 1, 1, 64)
+    assert lib.esb_conv2d_nhwc(ctypes.byref(dw), fake, 16, f81, fake, 16, f81, ep, fake, null, null, 0, null) == R
+    # grouped convolution other than depthwise
+    g2 = esb.esb_conv_desc(1, 8, 8, 64, 64, 3, 3, 1, 1, 2)
+    assert lib.esb_conv2d_nhwc(ctypes.byref(g2), fake, 8, f, fake, 8, f, ep, fake, null, null, 0,
+                               null) == esb.ESB_ERR_UNSUPPORTED
+    # pooling
+    assert lib.esb_maxpool_nhwc(fake, 8, f, 1, 8, 8, 64, 3, 2, 3, fake, 8, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_maxpool_nhwc(fake, 8, f, 1, 8, 8, 64, 3, 2, 1, fake, 7, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_maxpool_nhwc(fake, 8, f, 0, 8, 8, 64, 3, 2, 1, fake, 8, null) == esb.ESB_OK
+    f52 = esb.esb_format(5, 2, 0)
+    assert lib.esb_avgpool_nhwc(fake, 8, f, 1, 49, 64, 1.0, 0.5, f52, 0, null, fake, 8,
+                                null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_avgpool_nhwc(fake, 8, f, 1, 49, 64, 1.0, 0.0, f, 0, null, fake, 8, null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_avgpool_nhwc(fake, 16, f81, 1, 49, 64, 1.0, 0.5, f81, 0, null, fake, 16, null) == R
+
+
 def test_bn_dn_fold_identity():
     # Sec. IV-C: DN(BN(Scale(x))) / alpha_{l+1} = a x + b with the printed a, b.
     rng = np.random.default_rng(4)
