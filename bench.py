@@ -121,23 +121,33 @@ class ClockSampler:
             self.proc.wait(timeout=5)
         except Exception:
             self.proc.kill()
-        rows = []
-        for line in open(self.path):
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) >= 9 and parts[0] == str(gpu_index):
-                rows.append(parts)
+        with open(self.path) as fh:
+            lines = fh.readlines()
         os.unlink(self.path)
-        if not rows:
-            return None
-        mhz = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
-        reasons = set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for r in rows:
-            for name, v in zip(names, r[5:9]):
-                if v.lower().startswith("active"):
-                    reasons.add(name)
-        return {"sm_mhz": statistics.median(mhz) if mhz else None, "sm_max_mhz": float(rows[0][2]),
-                "samples": len(rows), "reasons": sorted(reasons)}
+        return summarise_clocks(lines, gpu_index)
+
+
+def summarise_clocks(lines, gpu_index=0):
+    """The clocks object of the JSON line from nvidia-smi CSV samples (index,
+    clocks.sm, clocks.max.sm, power.draw, reasons.active, hw_slowdown,
+    hw_thermal_slowdown, sw_thermal_slowdown, sw_power_cap): median SM clock,
+    the maximum, and every throttle reason seen active in any sample."""
+    rows = []
+    for line in lines:
+        parts = [x.strip() for x in line.split(",")]
+        if len(parts) >= 9 and parts[0] == str(gpu_index):
+            rows.append(parts)
+    if not rows:
+        return None
+    mhz = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+    reasons = set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for r in rows:
+        for name, v in zip(names, r[5:9]):
+            if v.lower().startswith("active"):
+                reasons.add(name)
+    return {"sm_mhz": statistics.median(mhz) if mhz else None, "sm_max_mhz": float(rows[0][2]),
+            "samples": len(rows), "reasons": sorted(reasons)}
 
 
 # --------------------------------------------------------------------- GPU arm
