@@ -540,7 +540,7 @@ def run_sweep(args):
                         "frac_fp8": round(tf / fp8, 3), "status": esb.esb_get_status()})
             del A, B, oc, ws
             torch.cuda.empty_cache()
-    x = synth.normal((1 << 28,), seed=0).to(dev)
+    x = synth.normal((1 << 28,), seed=0).to(dev) if args.sweeps in ("all", "project") else None
     for b in (range(3, 7) if args.sweeps in ("all", "project") else []):
         for k in range(1, b):
             f = esb.Fmt(b, k, True)
@@ -549,9 +549,91 @@ def run_sweep(args):
             byt = (1 << 28) * (4 + 4 / (32 // b))
             out.append({"project": 1 << 28, "fmt": [b, k], "us": round(us, 1), "GB/s": round(byt / us / 1e3, 1),
                         "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
-    print(json.dumps({"workload": "sweeps (esb_gemm_tiled M=N=K, esb_project 2^28)", "peaks": {
+    del x
+    if args.sweeps in ("all", "cc"):
+        out += _cc_sweep(esb, torch, timeit, hbm)
+    print(json.dumps({"workload": "sweeps (esb_gemm_tiled M=N=K, esb_project 2^28, depthwise conv and pooling)",
+                      "peaks": {
         "hbm_gbs": hbm, "fp8_tflops": fp8, "note": "measured HBM copy; fp8 = 2 x measured bf16 burst"},
         "results": out}))
+
+
+def _cc_sweep(esb, torch, timeit, hbm):
+    """The CUDA-core kernels at batch 64: MobileNetV2's depthwise 3x3 layers
+    (fused scale, bias, ReLU6 and requantisation, codes out), the ResNet18
+    stem max pool 112 -> 56 and the global average pools of ResNet18 (7x7x512)
+    and MobileNetV2 (7x7x1280), all ESB(4,2).  Algorithmic bytes = input
+    codes + output codes (+ weights, scale and bias).  Each call reads the next
+    of several input copies (over 3 x L2 in total), so inputs come from HBM;
+    codes are uniformly drawn words (timing only)."""
+    dev = torch.device("cuda")
+    g = torch.Generator(device=dev).manual_seed(0)
+    fx, fw = esb.Fmt(4, 2, False), esb.Fmt(4, 2, True)
+    n = 64
+    span = 3 * 129 * 10 ** 6
+
+    def copies(rows, ld, unsigned):
+        nbytes = rows * ld * 4
+        nx = max(1, min(256, -(-span // nbytes)))
+        c = torch.randint(0, 2 ** 32, (nx * rows, ld), generator=g, device=dev, dtype=torch.int64).to(torch.int32)
+        if unsigned:
+            c &= 0x77777777
+        return [c[i * rows:(i + 1) * rows] for i in range(nx)], nbytes
+
+    res = []
+    for h, c, stride in [(112, 32, 1), (112, 96, 2), (56, 144, 1), (56, 144, 2), (28, 192, 1), (14, 384, 1),
+                         (14, 576, 1), (7, 960, 1)]:
+        ld = esb.esb_row_words(c, 4)
+        P = (h + 2 - 3) // stride + 1
+        Xs, xb = copies(n * h * h, ld, True)
+        W, _ = copies(9, ld, False)
+        W = W[0]
+        scale = torch.full((c,), 1e-3, dtype=torch.float32, device=dev)
+        bias = torch.zeros((c,), dtype=torch.float32, device=dev)
+        ep = esb.Epilogue(scale=scale, bias=bias, act=esb.ESB_ACT_RELU6, alpha_out=0.29, fmt_out=fx)
+        oc = torch.empty((n * P * P, ld), dtype=torch.int32, device=dev)
+        it = [0]
+
+        def f():
+            X = Xs[it[0] % len(Xs)]
+            it[0] += 1
+            esb.esb_conv2d_nhwc(X, fx, W, fw, n, h, h, c, c, 3, 3, stride, 1, groups=c, ep=ep, want_acc=False,
+                                want_codes=True, out_codes=oc)
+
+        us = timeit(f, 20)
+        byt = xb + oc.numel() * 4 + W.numel() * 4 + 8 * c
+        res.append({"dwconv": [n, h, h, c, stride], "fmt": [4, 2], "us": round(us, 2),
+                    "GB/s": round(byt / us / 1e3, 1), "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
+        del Xs, oc
+    Xs, xb = copies(n * 112 * 112, 8, True)
+    Y = torch.empty((n * 56 * 56, 8), dtype=torch.int32, device=dev)
+    it = [0]
+
+    def mp():
+        esb.esb_maxpool_nhwc(Xs[it[0] % len(Xs)], fx, n, 112, 112, 64, 3, 2, 1, out=Y)
+        it[0] += 1
+
+    us = timeit(mp, 20)
+    byt = xb + Y.numel() * 4
+    res.append({"maxpool": [n, 112, 112, 64, 3, 2], "fmt": [4, 2], "us": round(us, 2),
+                "GB/s": round(byt / us / 1e3, 1), "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
+    del Xs, Y
+    for c in (512, 1280):
+        ld = esb.esb_row_words(c, 4)
+        Xs, xb = copies(n * 49, ld, True)
+        it = [0]
+
+        def ap():
+            esb.esb_avgpool_nhwc(Xs[it[0] % len(Xs)], fx, n, 49, c, 1.0 / 49, 0.5, fx)
+            it[0] += 1
+
+        us = timeit(ap, 20)
+        byt = xb + n * ld * 4
+        res.append({"avgpool": [n, 7, 7, c], "fmt": [4, 2], "us": round(us, 2),
+                    "GB/s": round(byt / us / 1e3, 1), "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
+        del Xs
+    res.append({"cc_status": esb.esb_get_status()})
+    return res
 
 
 def main():
@@ -561,8 +643,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--sweeps", nargs="?", const="all", choices=["all", "gemm", "project"],
-                    help="the large-operand sweeps instead of the step (all, or only the GEMM or projection half)")
+    ap.add_argument("--sweeps", nargs="?", const="all", choices=["all", "gemm", "project", "cc"],
+                    help="the sweeps instead of the step (all, or only the GEMM, projection or CUDA-core part)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
