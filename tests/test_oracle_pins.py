@@ -446,3 +446,13 @@ def test_projection_is_the_step_function_of_its_breakpoints(b, k, signed, roundi
     got = step_function_codes(torch.from_numpy(bits), step).numpy()
     bad = np.nonzero(got != exp)[0]
     assert bad.size == 0, [(hex(int(bits[i])), int(exp[i]), int(got[i])) for i in bad[:5]]
+
+
+@pytest.mark.parametrize("b,k", ALL_FORMATS)
+def test_code_rank_is_the_rotated_exponent_field(b, k):
+    # Sec. IV-A's code (e, f) with e = N for the values below one: ordering
+    # the non-negative codes by value is ordering them by (code + 2^k) mod
+    # 2^(b-1), so comparisons of codes (max pooling) need no decode.
+    L = 1 << (b - 1)
+    order = sorted(range(L), key=lambda c: o.decode(c, b, k))
+    assert [(c + (1 << k)) % L for c in order] == list(range(L))
