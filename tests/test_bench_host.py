@@ -66,11 +66,18 @@ def test_reference_arm_json_line():
     _check_reference(_reference_line(r.stdout), 1)
 
 
+def _free_port():
+    import socket
+    with socket.socket(socket.AF_INET, socket.SOCK_STREAM) as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
 def test_reference_arm_under_torchrun_prints_once():
     pytest.importorskip("torch.distributed.run")
     r = subprocess.run([sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
-                        "--master-addr", "127.0.0.1", "--master-port", "29531", "bench.py", "--impl", "reference",
-                        "--gpus", "2", "--steps", "1", "--warmup", "3"],
+                        "--master-addr", "127.0.0.1", "--master-port", str(_free_port()), "bench.py", "--impl",
+                        "reference", "--gpus", "2", "--steps", "1", "--warmup", "3"],
                        cwd=ROOT, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stderr[-2000:]
     _check_reference(_reference_line(r.stdout), 2)
