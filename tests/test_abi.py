@@ -187,3 +187,26 @@ def test_bn_dn_fold_identity():
     xr = acc * 2.0 ** -(kw + ka)
     assert np.allclose(lhs, a_p * xr + b_p, rtol=1e-12, atol=1e-12)
     assert np.allclose(lhs, (scale * acc + bias) / a_next, rtol=1e-12, atol=1e-12)
+
+
+def test_binding_refuses_host_tensors_and_missing_library(monkeypatch):
+    # no CPU fallback: every compute entry point of the binding takes device
+    # tensors only, and a missing libesb.so is an error, not a slower path
+    import torch
+    x = torch.zeros(64, dtype=torch.float32)
+    codes = torch.zeros((1, 8), dtype=torch.int32)
+    f = esb.Fmt(4, 2, True)
+    with pytest.raises(ValueError):
+        esb.esb_project(x, f, alpha=1.0)
+    with pytest.raises(ValueError):
+        esb.esb_calibrate_dda(x, f)
+    with pytest.raises(ValueError):
+        esb.esb_project_dda(x, f)
+    with pytest.raises(ValueError):
+        esb.esb_gemm(codes, f, codes, f, 64)
+    with pytest.raises(ValueError):
+        esb.esb_conv2d_nhwc(codes, f, codes, f, 1, 1, 1, 64, 64, 1, 1, 1, 0)
+    monkeypatch.setattr(esb, "_lib", None)
+    monkeypatch.setattr(esb, "LIB_PATH", os.path.join(ROOT, "no_such_dir", "libesb.so"))
+    with pytest.raises(RuntimeError):
+        esb.lib()
