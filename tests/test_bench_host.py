@@ -81,3 +81,21 @@ def test_reference_arm_under_torchrun_prints_once():
                        cwd=ROOT, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stderr[-2000:]
     _check_reference(_reference_line(r.stdout), 2)
+
+
+def test_cpu_baseline_leg_is_bounded():
+    import time
+    t0 = time.perf_counter()
+    cb = bench.cpu_baseline(budget_s=0.5)
+    assert time.perf_counter() - t0 < 60
+    assert cb["kind"] == "oracle" and cb["unit"] == bench.UNIT and cb["value"] > 0 and cb["cores"] >= 1
+    assert "output rows" in cb["sample"]
+
+
+def test_oracle_sample_ops_scale_with_rows():
+    from concurrent.futures import ThreadPoolExecutor
+    with ThreadPoolExecutor(max_workers=2) as pool:
+        s = bench.OracleSample(pool)
+        per_row = 2 * bench.Q_ * bench.CO_ * bench.R_ * bench.S_ * bench.C_
+        assert s.run(1) == per_row and s.run(3) == 3 * per_row
+        assert 1 <= s.rows_for_budget(0.001) <= s.rows_for_budget(1.0) <= bench.N_ * bench.P_
