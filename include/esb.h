@@ -86,7 +86,7 @@ enum { ESB_ACT_NONE = 0, ESB_ACT_RELU = 1, ESB_ACT_RELU6 = 2 };
  *   y = max(y, 0) (RELU) or min(max(y, 0), 6) (RELU6)
  *   code = projection of y with alpha_out, fmt_out, rounding_out
  *          (same as esb_project)
- * The BN/DN fold of Sec. IV-C becomes scale[n]/bias[n] on the host. */
+ * The BN/DN fold of Sec. IV-C becomes scale[n]/bias[n] (esb_fold_bn_dn). */
 typedef struct esb_epilogue {
     const float* scale;        /* [device] N floats, or NULL -> scale0 for every n */
     const float* alpha_a_dev;  /* [device] 1 float (scale of A / X), or NULL; with alpha_b_dev */
@@ -173,6 +173,26 @@ esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
                              void* workspace, size_t workspace_bytes,
                              float* alpha_out, double* stats_out, void* stream);
 
+/* Statistics and alpha of a tensor that is split into `count` parts, from
+ * the parts' statistics (Sec. III-D "Normalization": the mean and standard
+ * deviation of the whole tensor, then alpha = fl32(alpha*(b,k) * (spread +
+ * 1e-7)) as esb_calibrate_dda computes it).  The parts' statistics combine
+ * by the law of total variance, in fp64:
+ *   n = sum n_i,  mean = sum n_i mean_i / n,
+ *   signed:   n sigma^2 = sum n_i (sigma_i^2 + (mean_i - mean)^2)
+ *   unsigned: n rms^2   = sum n_i rms_i^2
+ * (the mean first, so the second sum has no cancellation).  This is the
+ * one exchange of a data-parallel calibration: every rank gathers all
+ * ranks' stats and calls this, so every rank gets the same alpha.  Host
+ * only, no device work.
+ *   stats      [host] count x 3 doubles {mean, spread, n}, as stats_out of
+ *              esb_calibrate_dda writes them; parts with n == 0 are skipped
+ *   stats_out  [host] 3 doubles {mean, spread, n} of the whole, or NULL
+ *   alpha_out  [host] 1 float, or NULL
+ * Errors: INVALID_ARG (NULL stats, count <= 0, a non-finite entry, a
+ * negative n or spread, total n == 0), UNSUPPORTED (bad format). */
+esb_status esb_dda_combine(const double* stats, int64_t count, esb_format f, double* stats_out, float* alpha_out);
+
 /* Size of the fixed scratch array behind esb_calibrate_dda_noalloc. */
 #define ESB_CALIBRATE_NOALLOC_SCRATCH_BYTES 32768
 
@@ -191,8 +211,9 @@ esb_status esb_calibrate_dda(const float* x, int64_t n, esb_format f,
  *   x          [device] n floats; n > 0
  *   alpha_out  [device] 1 float; stats_out [device] 3 doubles or NULL
  * The first call on a device looks up the array's device address (with
- * that device current) and caches it; make that first call before any
- * stream capture.  All calls share the one array (zero-filled when the
+ * that device current) and caches it for that device's context (a new
+ * context, e.g. after cudaDeviceReset, looks it up again); make that first
+ * call before any stream capture.  All calls share the one array (zero-filled when the
  * library loads; each call leaves its head record zero and overwrites every
  * block record it later reads): calls whose kernels overlap on the GPU (on
  * different streams without ordering) race on it and must be serialised.
@@ -230,9 +251,11 @@ esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx,
  * tensor on chip (shared memory) between them, so x is read from memory
  * once.  The barrier needs every block resident; its wait is bounded, and
  * should another tenant's work keep SMs occupied for seconds the call
- * reports ESB_ERR_TIMEOUT through esb_get_status.  (ESB_FUSED_COOPERATIVE=1
+ * reports ESB_ERR_TIMEOUT through esb_get_status; the workspace must then
+ * be zero-filled again before the next call.  (ESB_FUSED_COOPERATIVE=1
  * in the environment selects a cooperative launch, which waits for the
- * whole device instead.)
+ * whole device instead.  ESB_BARRIER_WAIT_NS, read at every call, can only
+ * shorten the wait's 2 s limit: a test aid that makes the wait run out.)
  *   x          [device] rows x cols floats, contiguous (row stride cols)
  *   workspace  [device] >= esb_calibrate_dda_workspace_bytes(rows * cols),
  *              16-byte aligned, zero-filled before its first use, as for
@@ -305,6 +328,33 @@ esb_status esb_gemm_tiled(int64_t M, int64_t N, int64_t K,
                           const esb_epilogue* ep,
                           int32_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
                           void* workspace, size_t workspace_bytes, void* stream);
+
+/* The "Scale" stage of Sec. IV-C on the host: the fp32 factor that turns
+ * the integer accumulator of codes in formats fa and fb into the product of
+ * their values, fl32(alpha_a * alpha_b) * 2^-(ka+kb) -- the value the
+ * epilogue computes on the device from alpha_a_dev and alpha_b_dev.
+ * Errors: INVALID_ARG (alpha not finite and > 0, NULL out), UNSUPPORTED. */
+esb_status esb_dequant_scale(float alpha_a, esb_format fa, float alpha_b, esb_format fb, float* scale_out);
+
+/* The "BN and DN" fold of Sec. IV-C: batch normalisation (per channel
+ * mean, standard deviation, gamma, beta) and the next layer's data
+ * normalisation (mean dn_mean, standard deviation dn_std) applied to the
+ * dequantised product become one affine map of the integer accumulator,
+ *   DN(BN(Scale(acc))) = scale[n] * acc + bias[n],
+ *   scale[n] = alpha_a 2^-ka alpha_w 2^-kw gamma_n / (std_n dn_std)
+ *   bias[n]  = (std_n beta_n - mean_n gamma_n - std_n dn_mean) / (dn_std std_n),
+ * computed in fp64.  The paper also folds the division by the next
+ * layer's alpha into it; here that division stays in the requantisation
+ * (esb_epilogue.alpha_out), so scale/bias (cast to fp32) are the
+ * epilogue's scale and bias arrays.  Host only.
+ *   bn_*       [host] n doubles each; bn_std > 0
+ *   scale_out, bias_out [host] n doubles each
+ * Errors: INVALID_ARG (NULL pointer, n < 0, non-positive or non-finite
+ * alpha / std), UNSUPPORTED (bad format). */
+esb_status esb_fold_bn_dn(float alpha_a, esb_format fa, float alpha_w, esb_format fw,
+                          const double* bn_mean, const double* bn_std, const double* bn_gamma,
+                          const double* bn_beta, int64_t n, double dn_mean, double dn_std,
+                          double* scale_out, double* bias_out);
 
 /* ---------------------------------------------------------------- conv */
 

@@ -81,7 +81,6 @@ def _load():
         "oracle_D": (f64, [f64, i32, i32]),
         "oracle_alpha_star": (f64, [i32, i32, p]),
         "oracle_dD": (f64, [f64, i32, i32]),
-        "oracle_calibrate": (f32, [p, i64, i32, i32, i32, p]),
         "oracle_calibrate_with": (f32, [p, i64, f64, i32, p]),
         "oracle_gemm_i64": (None, [p, i64, i32, i32, p, i64, i32, i32, i64, i64, i64, p]),
         "oracle_gemm_entry": (i64, [p, i64, i32, i32, p, i64, i32, i32, i64, i64, i64]),

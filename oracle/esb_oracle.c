@@ -333,24 +333,8 @@ double oracle_alpha_star(int b, int k, double *D_out)
  * two passes in fp64.  Signed formats: alpha = fl32(alpha* (sigma + 1e-7)).
  * Unsigned formats (post-ReLU data, the non-negative half of the set):
  * alpha = fl32(alpha* (rms + 1e-7)) with rms = sqrt((1/d) sum x^2), the scale
- * of the underlying normal of a half-normal.  stats = {mu, sigma|rms, d}. */
-float oracle_calibrate(const float *x, int64_t d, int b, int k, int is_signed, double *stats)
-{
-    double s = 0.0;
-    for (int64_t i = 0; i < d; i++) s += (double)x[i];
-    double mu = s / (double)d;
-    double ss = 0.0;
-    for (int64_t i = 0; i < d; i++) {
-        double c = is_signed ? ((double)x[i] - mu) : (double)x[i];
-        ss += c * c;
-    }
-    double spread = sqrt(ss / (double)d);
-    double as = oracle_alpha_star(b, k, NULL);
-    if (stats) { stats[0] = mu; stats[1] = spread; stats[2] = (double)d; }
-    return (float)(as * (spread + 1e-7));
-}
-
-/* Same, with alpha* supplied (avoids re-solving in loops). */
+ * of the underlying normal of a half-normal.  stats = {mu, sigma|rms, d}.
+ * alpha_star is oracle_alpha_star(b, k) of the format, solved once by the caller. */
 float oracle_calibrate_with(const float *x, int64_t d, double alpha_star, int is_signed, double *stats)
 {
     double s = 0.0;
@@ -468,40 +452,9 @@ void oracle_epilogue_array(const int64_t *acc, int64_t M, int64_t N, const float
 /* Sec. IV-B computing logic of a convolution layer, NHWC: X codes are rows
  * of C codes per pixel (ldx words), W codes are rows of C codes per
  * (cout, r, s) (ldw words).  acc[n][p][q][co] = sum_{r,s,c} I(X)*I(W) with
- * zero padding outside the image. */
-void oracle_conv2d_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
-                       const uint32_t *W, int64_t ldw, int bw, int kw,
-                       int Nb, int H, int Wd, int C, int Cout, int R, int S,
-                       int stride, int pad, int P, int Q, int64_t *acc)
-{
-    int cpx = 32 / bx, cpw_ = 32 / bw;
-    uint32_t mx = (1u << bx) - 1u, mw = (1u << bw) - 1u;
-    int64_t tx[256], tw[256];
-    image_table(bx, kx, tx);
-    image_table(bw, kw, tw);
-    for (int n = 0; n < Nb; n++)
-        for (int p = 0; p < P; p++)
-            for (int q = 0; q < Q; q++)
-                for (int co = 0; co < Cout; co++) {
-                    int64_t s = 0;
-                    for (int r = 0; r < R; r++)
-                        for (int t = 0; t < S; t++) {
-                            int h = p * stride - pad + r, w = q * stride - pad + t;
-                            if (h < 0 || h >= H || w < 0 || w >= Wd) continue;
-                            const uint32_t *xr = X + (((int64_t)n * H + h) * Wd + w) * ldx;
-                            const uint32_t *wr = W + (((int64_t)co * R + r) * S + t) * ldw;
-                            for (int c = 0; c < C; c++) {
-                                uint32_t cx = (xr[c / cpx] >> (bx * (c % cpx))) & mx;
-                                uint32_t cw = (wr[c / cpw_] >> (bw * (c % cpw_))) & mw;
-                                s += tx[cx] * tw[cw];
-                            }
-                        }
-                    acc[(((int64_t)n * P + p) * Q + q) * Cout + co] = s;
-                }
-}
-
-/* oracle_conv2d_i64 restricted to output rows p in [p0, p1) (acc holds
- * (p1 - p0) rows per image); used to time bounded samples. */
+ * zero padding outside the image, for the output rows p in [p0, p1) only:
+ * acc holds (p1 - p0) rows per image (the bounded samples of the CPU
+ * baseline).  oracle_conv2d_i64 below is the whole output, p in [0, P). */
 void oracle_conv2d_rows_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
                             const uint32_t *W, int64_t ldw, int bw, int kw,
                             int Nb, int H, int Wd, int C, int Cout, int R, int S,
@@ -533,6 +486,15 @@ void oracle_conv2d_rows_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
                         }
                     acc[(((int64_t)n * rows + (p - p0)) * Q + q) * Cout + co] = s;
                 }
+}
+
+void oracle_conv2d_i64(const uint32_t *X, int64_t ldx, int bx, int kx,
+                       const uint32_t *W, int64_t ldw, int bw, int kw,
+                       int Nb, int H, int Wd, int C, int Cout, int R, int S,
+                       int stride, int pad, int P, int Q, int64_t *acc)
+{
+    oracle_conv2d_rows_i64(X, ldx, bx, kx, W, ldw, bw, kw, Nb, H, Wd, C, Cout, R, S,
+                           stride, pad, P, Q, 0, P, acc);
 }
 
 /* Depthwise convolution (one filter per channel; MobileNetV2's 3x3 layers):

@@ -6,6 +6,7 @@
 #include <cstring>
 #include <mutex>
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include "esb.h"
@@ -16,17 +17,68 @@ namespace esb {
 
 __device__ int g_esb_device_status = 0;
 
+// Id of the current context (unique for the life of the process).  The two
+// driver calls are fetched through the runtime, so the library needs no
+// link-time dependency on the driver library.
+static bool current_context_id(unsigned long long* id)
+{
+    using GetCurrent = CUresult (*)(CUcontext*);
+    using GetId = CUresult (*)(CUcontext, unsigned long long*);
+    static GetCurrent get_current = nullptr;
+    static GetId get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<GetCurrent>(f);
+        f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<GetId>(f);
+    });
+    if (!get_current || !get_id) return false;
+    CUcontext ctx = nullptr;
+    return get_current(&ctx) == CUDA_SUCCESS && ctx && get_id(ctx, id) == CUDA_SUCCESS;
+}
+
+cudaError_t symbol_address(cudaError_t (*lookup)(void**), SymbolCache& cache, void** out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= SymbolCache::kDevices) return cudaErrorInvalidDevice;
+    // The context's id is unique for the life of the process, so a context
+    // created after a cudaDeviceReset (which reloads the module, moving its
+    // arrays) never matches an entry of the one before.
+    unsigned long long id = 0;
+    const bool have_id = current_context_id(&id);
+    std::lock_guard<std::mutex> lk(cache.mu);
+    if (!have_id || !cache.ptr[dev] || cache.ctx_id[dev] != id) {
+        void* p = nullptr;
+        e = lookup(&p);
+        if (e != cudaSuccess) return e;
+        // the lookup makes the device's primary context current if none was
+        if (!have_id && !current_context_id(&id)) {
+            *out = p;  // no id to key on: use the address without caching it
+            return cudaSuccess;
+        }
+        cache.ptr[dev] = p;
+        cache.ctx_id[dev] = id;
+    }
+    *out = cache.ptr[dev];
+    return cudaSuccess;
+}
+
+static cudaError_t lookup_device_status(void** p) { return cudaGetSymbolAddress(p, g_esb_device_status); }
+
 int* device_status_ptr()
 {
-    static int* cache[64] = {nullptr};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    if (!cache[dev]) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_esb_device_status) != cudaSuccess) return nullptr;
-        cache[dev] = static_cast<int*>(p);
-    }
-    return cache[dev];
+    static SymbolCache cache;
+    void* p = nullptr;
+    if (symbol_address(lookup_device_status, cache, &p) != cudaSuccess) return nullptr;
+    return static_cast<int*>(p);
 }
 
 int device_sm_count()
@@ -168,6 +220,70 @@ esb_status esb_calibrate_dda_noalloc(const float* x, int64_t n, esb_format f, fl
     cudaError_t e = launch_calibrate_noalloc(x, n, f.is_signed, as, alpha_out, stats_out,
                                              static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_dda_combine(const double* stats, int64_t count, esb_format f, double* stats_out, float* alpha_out)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (!stats || count <= 0) return ESB_ERR_INVALID_ARG;
+    double n = 0.0, s1 = 0.0;
+    for (int64_t i = 0; i < count; i++) {
+        const double m = stats[3 * i], sp = stats[3 * i + 1], ni = stats[3 * i + 2];
+        if (!std::isfinite(m) || !std::isfinite(sp) || !std::isfinite(ni) || ni < 0.0 || sp < 0.0)
+            return ESB_ERR_INVALID_ARG;
+        n += ni;
+        s1 += ni * m;
+    }
+    if (!(n > 0.0)) return ESB_ERR_INVALID_ARG;
+    const double mean = s1 / n;
+    double m2 = 0.0;
+    for (int64_t i = 0; i < count; i++) {
+        const double m = stats[3 * i], sp = stats[3 * i + 1], ni = stats[3 * i + 2];
+        if (ni == 0.0) continue;
+        m2 += f.is_signed ? ni * (sp * sp + (m - mean) * (m - mean)) : ni * sp * sp;
+    }
+    const double spread = std::sqrt(m2 / n);
+    if (stats_out) {
+        stats_out[0] = mean;
+        stats_out[1] = spread;
+        stats_out[2] = n;
+    }
+    if (alpha_out) {
+        double as = 0.0;
+        alpha_star_cached(f.b, f.k, &as, nullptr);
+        *alpha_out = static_cast<float>(as * (spread + 1e-7));
+    }
+    return ESB_OK;
+}
+
+esb_status esb_dequant_scale(float alpha_a, esb_format fa, float alpha_b, esb_format fb, float* scale_out)
+{
+    if (!fmt_ok(fa) || !fmt_ok(fb)) return ESB_ERR_UNSUPPORTED;
+    if (!scale_out || !(std::isfinite(alpha_a) && alpha_a > 0.0f) || !(std::isfinite(alpha_b) && alpha_b > 0.0f))
+        return ESB_ERR_INVALID_ARG;
+    const float ab = alpha_a * alpha_b;  // one fp32 rounding, as on the device
+    *scale_out = ab * std::ldexp(1.0f, -(fa.k + fb.k));
+    return ESB_OK;
+}
+
+esb_status esb_fold_bn_dn(float alpha_a, esb_format fa, float alpha_w, esb_format fw, const double* bn_mean,
+                          const double* bn_std, const double* bn_gamma, const double* bn_beta, int64_t n,
+                          double dn_mean, double dn_std, double* scale_out, double* bias_out)
+{
+    if (!fmt_ok(fa) || !fmt_ok(fw)) return ESB_ERR_UNSUPPORTED;
+    if (n < 0 || !(std::isfinite(alpha_a) && alpha_a > 0.0f) || !(std::isfinite(alpha_w) && alpha_w > 0.0f) ||
+        !(std::isfinite(dn_std) && dn_std > 0.0) || !std::isfinite(dn_mean))
+        return ESB_ERR_INVALID_ARG;
+    if (n == 0) return ESB_OK;
+    if (!bn_mean || !bn_std || !bn_gamma || !bn_beta || !scale_out || !bias_out) return ESB_ERR_INVALID_ARG;
+    const double s = std::ldexp((double)alpha_a, -fa.k) * std::ldexp((double)alpha_w, -fw.k);
+    for (int64_t i = 0; i < n; i++)
+        if (!(std::isfinite(bn_std[i]) && bn_std[i] > 0.0)) return ESB_ERR_INVALID_ARG;
+    for (int64_t i = 0; i < n; i++) {
+        scale_out[i] = s * bn_gamma[i] / (bn_std[i] * dn_std);
+        bias_out[i] = (bn_std[i] * bn_beta[i] - bn_mean[i] * bn_gamma[i] - bn_std[i] * dn_mean) / (dn_std * bn_std[i]);
+    }
+    return ESB_OK;
 }
 
 esb_status esb_project(const float* x, int64_t rows, int64_t cols, int64_t ldx, float alpha, const float* alpha_dev,

@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <mutex>
 #include <cuda_runtime.h>
 
 #include "esb.h"
@@ -11,6 +12,18 @@
 namespace esb {
 
 int device_sm_count();
+
+// Device address of a __device__ symbol of this library in the current
+// context, cached per device and keyed by the context's id.  `lookup` runs
+// cudaGetSymbolAddress in the symbol's own translation unit (in host code
+// the symbol's name is only a stand-in for the device array).
+struct SymbolCache {
+    static constexpr int kDevices = 64;
+    std::mutex mu;
+    unsigned long long ctx_id[kDevices] = {};
+    void* ptr[kDevices] = {};
+};
+cudaError_t symbol_address(cudaError_t (*lookup)(void**), SymbolCache& cache, void** out);
 
 // Device address of the library status word on the current device.
 int* device_status_ptr();

@@ -747,8 +747,9 @@ __device__ __forceinline__ void cal_depart(CalSync* sync)
 }
 
 // One launch: every block writes its partial record; the block that takes
-// the last ticket (the ticket word is zeroed by a memset before the launch)
-// adds all records in index order and finalises alpha.
+// the last ticket adds all records in index order, finalises alpha and
+// returns the ticket to zero, so the workspace needs zeroing only once,
+// before its first use (never between calls).
 __global__ void __launch_bounds__(kCalThreads, 4)
 calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalPartial* __restrict__ part,
                        CalSync* __restrict__ sync, double alpha_star, int is_signed,
@@ -776,7 +777,7 @@ __global__ void __launch_bounds__(kCalThreads, 4)
 calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols, CalPartial* __restrict__ part,
                          CalSync* __restrict__ sync, double alpha_star, ProjParams p, float* __restrict__ alpha_out,
                          double* __restrict__ stats_out, uint32_t* __restrict__ codes, int64_t ldc,
-                         int* __restrict__ status, int stash_g)
+                         int* __restrict__ status, int stash_g, unsigned long long wait_ns)
 {
     // stash: stash_g granules (512 bytes each) per warp of dynamic shared memory
     extern __shared__ float4 stash_all[];
@@ -818,7 +819,7 @@ calibrate_project_kernel(const float* __restrict__ x, int64_t rows, int64_t cols
         uint32_t it = 0;
         unsigned long long w = *rel;
         while ((w >> 32) == 0ull) {
-            if ((++it & 63u) == 0u && globaltimer_ns() - t0 > 2000000000ull) { timed_out = 1; break; }
+            if ((++it & 63u) == 0u && globaltimer_ns() - t0 > wait_ns) { timed_out = 1; break; }
             __nanosleep(32);
             w = *rel;
         }
@@ -980,9 +981,18 @@ static cudaError_t launch_calibrate_project_b(const float* x, int64_t rows, int6
     CalSync* sync = static_cast<CalSync*>(workspace);
     CalPartial* part = static_cast<CalPartial*>(workspace) + 1;
     int* status = device_status_ptr();
+    // Limit of the grid barrier's wait: 2 s.  ESB_BARRIER_WAIT_NS in the
+    // environment (read at every launch) can only shorten it; tests use that
+    // to make the wait run out.  The wait sits after every bulk copy of the
+    // block has landed, so a block that gives up leaves nothing in flight.
+    unsigned long long wait_ns = 2000000000ull;
+    if (const char* v = getenv("ESB_BARRIER_WAIT_NS")) {
+        const unsigned long long w = strtoull(v, nullptr, 10);
+        if (w > 0 && w < wait_ns) wait_ns = w;
+    }
     void* args[] = {(void*)&x, (void*)&rows, (void*)&cols, (void*)&part, (void*)&sync, (void*)&alpha_star,
                     (void*)&p, (void*)&alpha_out, (void*)&stats_out, (void*)&codes, (void*)&ldc, (void*)&status,
-                    (void*)&stash_g};
+                    (void*)&stash_g, (void*)&wait_ns};
     // The grid is one resident wave (sized by the occupancy query above), so
     // every block becomes resident once the previous kernel of the stream
     // has left the SMs; the grid barrier's wait is bounded and reports
@@ -1052,31 +1062,20 @@ cudaError_t launch_calibrate_project(const float* x, int64_t rows, int64_t cols,
 static_assert(sizeof(CalPartial) == 32, "partial record layout");
 static __device__ __align__(256) unsigned char g_cal_noalloc_scratch[(kCalMaxBlocks + 1) * 32];
 
-namespace {
-std::mutex g_noalloc_mu;
-void* g_noalloc_ptr[64] = {nullptr};
-}  // namespace
-
 size_t calibrate_noalloc_capacity() { return sizeof(g_cal_noalloc_scratch); }
 
 // The host-side name of the array is only a stand-in, never a device
-// address: the address is looked up once per device (with that device
-// current) and cached.
+// address: the address is looked up with the device current and cached per
+// device and context (symbol_address).  The lookup allocates nothing.
+static cudaError_t lookup_noalloc_scratch(void** p)
+{
+    return cudaGetSymbolAddress(p, g_cal_noalloc_scratch);
+}
+
 static cudaError_t noalloc_scratch_address(void** out)
 {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lk(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_cal_noalloc_scratch);
-        if (e != cudaSuccess) return e;
-        g_noalloc_ptr[dev] = p;
-    }
-    *out = g_noalloc_ptr[dev];
-    return cudaSuccess;
+    static SymbolCache cache;
+    return symbol_address(lookup_noalloc_scratch, cache, out);
 }
 
 cudaError_t launch_calibrate_noalloc(const float* x, int64_t n, int is_signed, double alpha_star, float* alpha_out,

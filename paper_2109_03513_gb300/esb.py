@@ -86,6 +86,10 @@ SIGNATURES = {
     "esb_calibrate_dda_workspace_bytes": (_SZ, [_I64]),
     "esb_calibrate_dda": (_I32, [_P, _I64, esb_format, _P, _SZ, _P, _P, _P]),
     "esb_calibrate_dda_noalloc": (_I32, [_P, _I64, esb_format, _P, _P, _P]),
+    "esb_dda_combine": (_I32, [_P, _I64, esb_format, _P, _P]),
+    "esb_dequant_scale": (_I32, [_F32, esb_format, _F32, esb_format, _P]),
+    "esb_fold_bn_dn": (_I32, [_F32, esb_format, _F32, esb_format, _P, _P, _P, _P, _I64, ctypes.c_double,
+                              ctypes.c_double, _P, _P]),
     "esb_project": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _I32, _P, _I64, _P]),
     "esb_project_dda": (_I32, [_P, _I64, _I64, esb_format, _I32, _P, _SZ, _P, _P, _P, _I64, _P]),
     "esb_dequant": (_I32, [_P, _I64, _I64, _I64, _F32, _P, esb_format, _P, _I64, _P]),
@@ -411,25 +415,36 @@ def esb_get_status(stream=None) -> int:
 
 # ------------------------------------------------------------ host helpers
 
-def default_scale(alpha_a: float, fa: Fmt, alpha_b: float, fb: Fmt) -> float:
-    """fp32 multiplier turning the integer accumulator into the real product:
-    alpha_a * 2^-ka * alpha_b * 2^-kb (one fp32 rounding of alpha_a * alpha_b)."""
+def esb_dda_combine(stats, f: Fmt) -> tuple[float, float, float, float]:
+    """(alpha, mean, spread, n) of a tensor from its parts' statistics
+    (an iterable of {mean, spread, n} triples, e.g. esb_calibrate_dda's
+    stats_out of each part)."""
     import numpy as np
-    return float(np.float32(np.float32(alpha_a) * np.float32(alpha_b)) * np.float32(2.0 ** -(fa.k + fb.k)))
+    st = np.ascontiguousarray(np.asarray([[float(v) for v in t] for t in stats], dtype=np.float64).reshape(-1, 3))
+    out = np.zeros(3, dtype=np.float64)
+    a = ctypes.c_float(0.0)
+    _check(lib().esb_dda_combine(st.ctypes.data, st.shape[0], f.c(), out.ctypes.data, ctypes.byref(a)),
+           "esb_dda_combine")
+    return float(a.value), float(out[0]), float(out[1]), float(out[2])
 
 
-def fold_bn_dn(alpha_w: float, kw: int, alpha_a: float, ka: int, bn_mean, bn_std, bn_gamma, bn_beta,
-               dn_mean: float, dn_std: float):
-    """Sec. IV-C "BN and DN" fold for this library's epilogue.  The paper folds
-    Scale, BN and DN (and the division by the next layer's alpha) into one
-    affine a*x + b of the accumulator x; here the division by alpha_out stays
-    in the requantisation, so scale[n] = alpha_out * a_n and bias[n] = alpha_out * b_n:
-      scale = alpha_w 2^-kw alpha_a 2^-ka gamma / (sigma_BN sigma_DN)
-      bias  = (sigma_BN beta - mu_BN gamma - sigma_BN mu_DN) / (sigma_DN sigma_BN)
-    Returns float64 numpy arrays (cast to fp32 by the caller)."""
+def esb_dequant_scale(alpha_a: float, fa: Fmt, alpha_b: float, fb: Fmt) -> float:
+    """fp32 factor turning the integer accumulator into the product of the values."""
+    s = ctypes.c_float(0.0)
+    _check(lib().esb_dequant_scale(alpha_a, fa.c(), alpha_b, fb.c(), ctypes.byref(s)), "esb_dequant_scale")
+    return float(s.value)
+
+
+def esb_fold_bn_dn(alpha_a: float, fa: Fmt, alpha_w: float, fw: Fmt, bn_mean, bn_std, bn_gamma, bn_beta,
+                   dn_mean: float, dn_std: float):
+    """Sec. IV-C "BN and DN" fold -> (scale, bias) float64 numpy arrays of the epilogue."""
     import numpy as np
-    bn_mean, bn_std, bn_gamma, bn_beta = (np.asarray(v, dtype=np.float64) for v in (bn_mean, bn_std, bn_gamma, bn_beta))
-    s = (alpha_w * 2.0 ** -kw) * (alpha_a * 2.0 ** -ka)
-    scale = s * bn_gamma / (bn_std * dn_std)
-    bias = (bn_std * bn_beta - bn_mean * bn_gamma - bn_std * dn_mean) / (dn_std * bn_std)
+    arrs = [np.ascontiguousarray(np.asarray(v, dtype=np.float64).ravel()) for v in (bn_mean, bn_std, bn_gamma, bn_beta)]
+    n = arrs[0].size
+    if any(a.size != n for a in arrs):
+        raise ValueError("bn_mean, bn_std, bn_gamma and bn_beta must have the same length")
+    scale = np.zeros(n, dtype=np.float64)
+    bias = np.zeros(n, dtype=np.float64)
+    _check(lib().esb_fold_bn_dn(alpha_a, fa.c(), alpha_w, fw.c(), *[a.ctypes.data for a in arrs], n, dn_mean, dn_std,
+                                scale.ctypes.data, bias.ctypes.data), "esb_fold_bn_dn")
     return scale, bias

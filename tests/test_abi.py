@@ -3,6 +3,7 @@ points and host-side validation (no device work; runs without a GPU)."""
 import ctypes
 import os
 import re
+from fractions import Fraction
 
 import numpy as np
 import pytest
@@ -172,10 +173,11 @@ def test_host_validation_other_entry_points(lib):
 def test_bn_dn_fold_identity():
     # Sec. IV-C: DN(BN(Scale(x))) / alpha_{l+1} = a x + b with the printed a, b.
     rng = np.random.default_rng(4)
-    aw, ka, aa, kw = 0.37, 2, 1.3, 1
+    aw, ka, aa, kw = np.float32(0.37), 2, np.float32(1.3), 1   # fp32 scales, as the library takes them
+    aw, aa = float(aw), float(aa)
     mu_bn, sd_bn, g, beta = rng.normal(size=5), rng.uniform(0.5, 2, 5), rng.normal(size=5), rng.normal(size=5)
     mu_dn, sd_dn, a_next = 0.3, 1.7, 0.61
-    scale, bias = esb.fold_bn_dn(aw, kw, aa, ka, mu_bn, sd_bn, g, beta, mu_dn, sd_dn)
+    scale, bias = esb.esb_fold_bn_dn(aa, esb.Fmt(8, ka), aw, esb.Fmt(8, kw), mu_bn, sd_bn, g, beta, mu_dn, sd_dn)
     acc = rng.integers(-500, 500, size=5).astype(np.float64)
     x = acc * (aw * 2.0 ** -kw) * (aa * 2.0 ** -ka)          # Scale: dequantised product
     bn = g * (x - mu_bn) / sd_bn + beta                      # BN
@@ -187,6 +189,53 @@ def test_bn_dn_fold_identity():
     xr = acc * 2.0 ** -(kw + ka)
     assert np.allclose(lhs, a_p * xr + b_p, rtol=1e-12, atol=1e-12)
     assert np.allclose(lhs, (scale * acc + bias) / a_next, rtol=1e-12, atol=1e-12)
+
+
+def test_dequant_scale_is_the_scale_stage():
+    # Sec. IV-C "Scale": acc * alpha_a 2^-ka * alpha_b 2^-kb is the product of
+    # the two values; the fp32 factor has one rounding (of alpha_a * alpha_b)
+    rng = np.random.default_rng(9)
+    for _ in range(200):
+        aa, ab = (float(np.float32(v)) for v in rng.uniform(1e-3, 3.0, 2))
+        ka, kb = (int(v) for v in rng.integers(0, 7, 2))
+        s = esb.esb_dequant_scale(aa, esb.Fmt(8, ka), ab, esb.Fmt(8, kb))
+        exact = Fraction(aa) * Fraction(ab) / 2 ** (ka + kb)
+        assert abs(Fraction(s) - exact) <= exact * Fraction(1, 2 ** 24)      # within half an fp32 ulp
+        assert s == float(np.float32(aa * ab)) / 2 ** (ka + kb)
+    f = esb.Fmt(4, 2)
+    with pytest.raises(esb.EsbError):
+        esb.esb_dequant_scale(0.0, f, 1.0, f)
+    with pytest.raises(esb.EsbError):
+        esb.esb_dequant_scale(1.0, esb.Fmt(4, 4), 1.0, f)
+
+
+def test_dda_combine_law_of_total_variance():
+    # Sec. III-D statistics of a whole tensor from its parts: against numpy
+    # fp64 two-pass moments of the concatenation, then alpha = fl32(alpha* (s + 1e-7))
+    rng = np.random.default_rng(10)
+    parts = [rng.normal(3.0, 0.5, 7001), rng.normal(2.5, 2.0, 1), np.abs(rng.normal(size=30000)), np.zeros(0)]
+    for signed in (True, False):
+        f = esb.Fmt(5, 2, signed)
+        st = []
+        for p in parts:
+            if p.size == 0:
+                st.append((0.0, 0.0, 0.0))
+                continue
+            m = p.mean()
+            sp = np.sqrt(((p - m) ** 2).mean()) if signed else np.sqrt((p * p).mean())
+            st.append((m, sp, p.size))
+        a, mean, spread, n = esb.esb_dda_combine(st, f)
+        x = np.concatenate(parts)
+        ref_sp = np.sqrt(((x - x.mean()) ** 2).mean()) if signed else np.sqrt((x * x).mean())
+        assert n == x.size
+        assert abs(mean - x.mean()) <= 1e-12 * abs(x.mean())
+        assert abs(spread - ref_sp) <= 1e-12 * ref_sp
+        astar = esb.esb_alpha_star(5, 2)[0]
+        assert a == float(np.float32(astar * (spread + 1e-7)))
+    with pytest.raises(esb.EsbError):
+        esb.esb_dda_combine([(0.0, 0.0, 0.0)], esb.Fmt(4, 2))
+    with pytest.raises(esb.EsbError):
+        esb.esb_dda_combine([(0.0, -1.0, 5.0)], esb.Fmt(4, 2))
 
 
 def test_binding_refuses_host_tensors_and_missing_library(monkeypatch):

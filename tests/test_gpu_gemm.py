@@ -117,7 +117,7 @@ def test_gemm_fused_epilogue_matches_oracle(M, N, K, act, fo, rnd, per_channel, 
     xb = synth.he_normal((N, K), fan_in=K, seed=N + 2).numpy()
     A, aa = projected_packed(xa, fa, 0)
     B, ab = projected_packed(xb, fb, 0)
-    s0 = esb.default_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2))
+    s0 = esb.esb_dequant_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2))
     if per_channel:
         scale = (np.float32(s0) * synth.normal((N,), seed=3).numpy().__abs__() + np.float32(1e-3)).astype(np.float32)
         bias = (0.1 * synth.normal((N,), seed=4).numpy()).astype(np.float32)
@@ -171,7 +171,7 @@ def test_gemm_codes_only_epilogue(act, fo, bias0, sf):
     fa, fb = (4, 2, False), (4, 2, True)
     A, aa = projected_packed(synth.half_normal((M, K), seed=M + 5).numpy(), fa, 0)
     B, ab = projected_packed(synth.he_normal((N, K), fan_in=K, seed=N + 6).numpy(), fb, 0)
-    s = np.float32(esb.default_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2)) * sf)
+    s = np.float32(esb.esb_dequant_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2)) * sf)
     _, _, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(*fa), dev_i32(B), esb.Fmt(*fb), K, ep=lean_epilogue(fo, act, bias0, s),
                                want_acc=False, want_y=False, want_codes=True)
     acc_o = o.gemm_i64(A, fa[:2], B, fb[:2], M, N, K)
@@ -187,7 +187,7 @@ def test_gemm_codes_only_epilogue_large_accumulators(M, N, K, fab, act):
     fa, fb = (fab[0], fab[1], False), (fab[0], fab[1], True)
     A, aa = projected_packed(synth.half_normal((M, K), seed=K + 1).numpy(), fa, 0)
     B, ab = projected_packed(synth.he_normal((N, K), fan_in=K, seed=K + 2).numpy(), fb, 0)
-    s = np.float32(esb.default_scale(aa, esb.Fmt(*fab), ab, esb.Fmt(*fab)))
+    s = np.float32(esb.esb_dequant_scale(aa, esb.Fmt(*fab), ab, esb.Fmt(*fab)))
     fo = (4, 2, False)
     _, _, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(*fa), dev_i32(B), esb.Fmt(*fb), K,
                                ep=lean_epilogue(fo, act, -0.02, s), want_acc=False, want_codes=True)
@@ -203,7 +203,7 @@ def test_conv_codes_only_epilogue(shape, act, fo, bias0, sf):
     fx, fw = (4, 2, False), (4, 2, True)
     X, ax = projected_packed(synth.half_normal((n * h * w, c), seed=h + c).numpy(), fx, 0)
     W, aw = projected_packed(synth.he_normal((cout * 9, c), fan_in=9 * c, seed=cout).numpy(), fw, 0)
-    s = np.float32(esb.default_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2)) * sf)
+    s = np.float32(esb.esb_dequant_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2)) * sf)
     _, _, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fx), dev_i32(W), esb.Fmt(*fw), n, h, w, c, cout, 3, 3,
                                       stride, 1, ep=lean_epilogue(fo, act, bias0, s), want_acc=False,
                                       want_codes=True)
@@ -221,7 +221,7 @@ def test_codes_store_alignment(ldo_extra, offset_words):
     fx, fw = (4, 2, False), (4, 2, True)
     X, ax = projected_packed(synth.half_normal((n * h * w, c), seed=31).numpy(), fx, 0)
     W, aw = projected_packed(synth.he_normal((cout * 9, c), fan_in=576, seed=32).numpy(), fw, 0)
-    s = np.float32(esb.default_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2)))
+    s = np.float32(esb.esb_dequant_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2)))
     ldo = esb.esb_row_words(cout, 4) + ldo_extra
     M = n * h * w
     buf = torch.full((M * ldo + offset_words + 8,), -1, dtype=torch.int32, device="cuda")
@@ -259,7 +259,7 @@ def check_conv(n, h, w, c, cout, r, s, stride, pad, fx, fw):
     W, aw = projected_packed(wt, fw, 0)
     assert X.shape[1] == ldx and W.shape[1] == ldx
     fo = (fx[0], fx[1], False)
-    s0 = esb.default_scale(ax, esb.Fmt(*fx[:2]), aw, esb.Fmt(*fw[:2]))
+    s0 = esb.esb_dequant_scale(ax, esb.Fmt(*fx[:2]), aw, esb.Fmt(*fw[:2]))
     ep = esb.Epilogue(scale0=s0, bias0=0.0, act=esb.ESB_ACT_RELU, alpha_out=0.7, fmt_out=esb.Fmt(*fo))
     acc, y, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fx), dev_i32(W), esb.Fmt(*fw), n, h, w, c, cout, r, s,
                                         stride, pad, ep=ep, want_acc=True, want_y=True, want_codes=True)
@@ -319,7 +319,7 @@ def test_conv_full_size_sampled_rows():
     wt = synth.he_normal((cout * 9, c), fan_in=576, seed=8).numpy()
     X, ax = projected_packed(x, fu, 0)
     W, aw = projected_packed(wt, fs, 0)
-    s0 = esb.default_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2))
+    s0 = esb.esb_dequant_scale(ax, esb.Fmt(4, 2), aw, esb.Fmt(4, 2))
     ep = esb.Epilogue(scale0=s0, act=esb.ESB_ACT_RELU, alpha_out=0.7, fmt_out=esb.Fmt(4, 2, False))
     acc, _, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fu), dev_i32(W), esb.Fmt(*fs), n, h, w, c, cout, 3, 3,
                                         1, 1, ep=ep, want_acc=True, want_codes=True)
@@ -443,7 +443,7 @@ def test_gemm_tiled_codes_only(act, fo, bias0, sf, tiled_always):
     fa, fb = (4, 2, False), (4, 2, True)
     A, aa = projected_packed(synth.half_normal((M, K), seed=M + 9).numpy(), fa, 0)
     B, ab = projected_packed(synth.he_normal((N, K), fan_in=K, seed=N + 8).numpy(), fb, 0)
-    s = np.float32(esb.default_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2)) * sf)
+    s = np.float32(esb.esb_dequant_scale(aa, esb.Fmt(4, 2), ab, esb.Fmt(4, 2)) * sf)
     _, _, codes = esb.esb_gemm(dev_i32(A), esb.Fmt(*fa), dev_i32(B), esb.Fmt(*fb), K,
                                ep=lean_epilogue(fo, act, bias0, s), want_acc=False, want_codes=True,
                                workspace=tiled_ws(M, N, K))

@@ -101,7 +101,7 @@ class Net:
         c = x.c
         Wd, Wn, aw = self.weights((r * s) if dw else cout * r * s, c, r * s if dw else r * s * c)
         fx, fw = esb.Fmt(*x.f), esb.Fmt(self.b, self.k, True)
-        s0 = esb.default_scale(x.a, fx, aw, fw)
+        s0 = esb.esb_dequant_scale(x.a, fx, aw, fw)
         signed_out = act == esb.ESB_ACT_NONE
         fo = (self.b, self.k, signed_out)
         res_scale = float(np.float32(res.a) * np.float32(2.0 ** -res.f[1])) if res is not None else 0.0
@@ -160,7 +160,7 @@ class Net:
         self.layers += 1
         Wd, Wn, aw = self.weights(nout, x.c, x.c)
         fx, fw = esb.Fmt(*x.f), esb.Fmt(self.b, self.k, True)
-        s0 = esb.default_scale(x.a, fx, aw, fw)
+        s0 = esb.esb_dequant_scale(x.a, fx, aw, fw)
         signed_out = act == esb.ESB_ACT_NONE
         fo = (self.b, self.k, signed_out)
         M, K = x.n, x.c

@@ -289,7 +289,7 @@ def test_workspace_left_zero_and_reusable():
 
 def test_sharded_calibration_from_device_statistics():
     # per-shard statistics from the device (esb_calibrate_dda stats_out),
-    # combined on the host (shard.combine_dda_stats), against the oracle on
+    # combined on the host (esb_dda_combine), against the oracle on
     # the whole tensor
     from paper_2109_03513_gb300 import shard
     for signed, x in [(True, synth.normal((200003,), seed=21, mean=2.0)), (False, synth.half_normal((131072,), seed=22))]:
@@ -300,8 +300,43 @@ def test_sharded_calibration_from_device_statistics():
             st = torch.zeros(3, dtype=torch.float64, device="cuda")
             esb.esb_calibrate_dda(x[cuts[i]:cuts[i + 1]].contiguous().cuda(), f, stats_out=st)
             stats.append(st.cpu().numpy())
-        n, mean, spread = shard.combine_dda_stats(stats, signed)
-        a = shard.dda_alpha(esb.esb_alpha_star(4, 2)[0], spread)
+        a, mean, spread, n = shard.combine_dda_stats(stats, f)
         a_ref, st_ref = o.calibrate(x.numpy(), 4, 2, signed)
         assert n == x.numel()
         assert abs(a - a_ref) <= 1e-6 * a_ref
+
+
+def test_barrier_wait_runs_out_and_recovers(monkeypatch):
+    # The fused projection's grid-barrier wait is bounded.  With its limit cut
+    # to 1 ns (ESB_BARRIER_WAIT_NS, a test aid that can only shorten it),
+    # blocks that arrive before the last one give up after their first
+    # bounded poll: the device status reports ESB_ERR_TIMEOUT and the kernel
+    # returns (no hang, the context stays usable).  After the workspace is
+    # zero-filled again the next call matches the oracle.  The wait sits
+    # after the block's bulk copies have landed, so nothing is in flight.
+    f = esb.Fmt(4, 2, False)
+    x = synth.half_normal((1 << 16, 64), seed=51)
+    xd = x.cuda()
+    ws = torch.zeros(esb.esb_calibrate_dda_workspace_bytes(xd.numel()), dtype=torch.uint8, device="cuda")
+    assert esb.esb_get_status() == 0
+    seen = []
+    monkeypatch.setenv("ESB_BARRIER_WAIT_NS", "1")
+    for _ in range(5):
+        esb.esb_project_dda(xd, f, workspace=ws)
+        seen.append(esb.esb_get_status())
+        ws.zero_()
+        if seen[-1] == esb.ESB_ERR_TIMEOUT:
+            break
+    monkeypatch.delenv("ESB_BARRIER_WAIT_NS")
+    assert esb.ESB_ERR_TIMEOUT in seen, seen
+    assert set(seen) <= {esb.ESB_OK, esb.ESB_ERR_TIMEOUT}
+    codes, a = esb.esb_project_dda(xd, f, workspace=ws)
+    assert esb.esb_get_status() == 0
+    assert int(ws[:32].cpu().sum()) == 0
+    ag = float(a.item())
+    ao, _ = o.calibrate(x.numpy(), 4, 2, False)
+    assert abs(ag - ao) <= 1e-6 * ao
+    idx = np.unique(np.concatenate([np.arange(8), np.arange(x.shape[0] - 8, x.shape[0]),
+                                    np.random.default_rng(5).integers(0, x.shape[0], 1000)]))
+    exp = o.project_packed(x.numpy()[idx], ag, 4, 2, False, ld_words=codes.shape[1])
+    assert np.array_equal(u32(codes)[idx], exp)

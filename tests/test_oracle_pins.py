@@ -332,7 +332,7 @@ def test_conv_and_depthwise_brute_force():
     rng = np.random.default_rng(5)
     fx, fw = (4, 2), (4, 1)
     Nb, H, Wd, C, Cout, R, S = 2, 6, 5, 11, 3, 3, 3
-    for stride, pad in [(1, 1), (2, 1), (1, 0)]:
+    for stride, pad in [(1, 1), (2, 1), (1, 0), (2, 0)]:
         cx = rng.integers(0, 16, size=(Nb, H, Wd, C), dtype=np.uint32)
         cw = rng.integers(0, 16, size=(Cout, R, S, C), dtype=np.uint32)
         X = o.pack(cx.reshape(-1, C), *fx, ld_words=4).reshape(Nb, H, Wd, 4)
@@ -347,6 +347,12 @@ def test_conv_and_depthwise_brute_force():
                 patch = ix[:, r:r + stride * P:stride, s_:s_ + stride * Q:stride, :]
                 exp += np.einsum("npqc,oc->npqo", patch, iw[:, r, s_, :])
         assert np.array_equal(got, exp)
+        # the row-restricted form (the CPU baseline's bounded samples): every
+        # window of output rows, first and last rows included
+        for p0 in range(P):
+            for p1 in range(p0 + 1, P + 1):
+                part = o.conv2d_rows_i64(X, fx, W, fw, Nb, H, Wd, C, Cout, R, S, stride, pad, p0, p1)
+                assert np.array_equal(part, exp[:, p0:p1]), (stride, pad, p0, p1)
         # depthwise with one filter per channel
         cwd = rng.integers(0, 16, size=(R, S, C), dtype=np.uint32)
         Wd_ = o.pack(cwd.reshape(-1, C), *fw, ld_words=4).reshape(R, S, 4)

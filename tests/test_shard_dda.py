@@ -1,7 +1,8 @@
 """Sharded DDA calibration on CPU ranks (gloo, world size 2): each rank
 calibrates its shard with the oracle, the shards' statistics are combined
-with torch.distributed all-reduces, and every rank must get the alpha the
-oracle computes on the whole tensor (Sec. III-D)."""
+with one torch.distributed all-gather and libesb's esb_dda_combine, and
+every rank must get the alpha the oracle computes on the whole tensor
+(Sec. III-D)."""
 import os
 import socket
 
@@ -12,7 +13,7 @@ import torch.distributed as dist
 import torch.multiprocessing as mp
 
 import oracle as o
-from paper_2109_03513_gb300 import shard, synth
+from paper_2109_03513_gb300 import esb, shard, synth
 
 CASES = [
     # (dist, n, b, k, signed)
@@ -43,7 +44,7 @@ def _rank(rank, world, port, case, out_path):
     x = _data(name, n)
     lo, hi = shard.shard_bounds(n, world, rank)
     _, st = o.calibrate(x[lo:hi], b, k, signed)
-    a, mean, spread = shard.allreduce_dda_alpha(st, o.alpha_star_cached(b, k), signed)
+    a, mean, spread = shard.allreduce_dda_alpha(st, esb.Fmt(b, k, signed))
     np.save(f"{out_path}.{rank}.npy", np.array([a, mean, spread], dtype=np.float64))
     dist.barrier()
     dist.destroy_process_group()
@@ -69,8 +70,9 @@ def test_combine_is_exact_on_host():
     x = _data("normal_offset", 30011)
     cuts = [0, 7000, 7001, 30011]
     stats = [o.calibrate(x[cuts[i]:cuts[i + 1]], 4, 2, True)[1] for i in range(3)]
-    n, mean, spread = shard.combine_dda_stats(stats, signed=True)
-    _, st_ref = o.calibrate(x, 4, 2, True)
+    a, mean, spread, n = shard.combine_dda_stats(stats, esb.Fmt(4, 2, True))
+    a_ref, st_ref = o.calibrate(x, 4, 2, True)
     assert n == x.size
+    assert abs(a - a_ref) <= 1e-6 * a_ref
     assert abs(mean - st_ref[0]) <= 1e-9 * abs(st_ref[0])
     assert abs(spread - st_ref[1]) <= 1e-9 * st_ref[1]
