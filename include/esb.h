@@ -290,9 +290,15 @@ esb_status esb_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_
  *   acc_out   [device] M x N int32 (row stride N), or NULL
  *   y_out     [device] M x N floats (row stride N), or NULL
  *   codes_out [device] M rows of ldo words (N codes in fmt_out), or NULL
- * The contraction runs on the tcgen05 tensor cores; it requires both
- * formats to have k <= 3 and b-k-1 <= 4 (every config format qualifies),
- * and K * max|I_A| * max|I_B| < 2^24 (else ESB_ERR_RANGE).
+ * The contraction runs on the tcgen05 tensor cores (kind::f8f6f4, E4M3
+ * operands).  A format with k <= 3 and b-k-1 <= 4 decodes to one exact
+ * E4M3 byte per code; a format with k >= 4 (5 to 8 significant bits, e.g.
+ * (6,4), (7,5), (8,6)) takes the significand split: each code becomes two
+ * exact E4M3 bytes (high and low 4-bit parts of its significand), and the
+ * contraction runs over 2 (one operand split) or 4 (both) planes of K.
+ * Formats with an exponent field of 5 or more bits ((6,0), (7,0), (7,1),
+ * (8,0)..(8,3)) are UNSUPPORTED.  Either way the sum must satisfy
+ * K * max|I_A| * max|I_B| < 2^24 (else ESB_ERR_RANGE).
  * Errors: INVALID_ARG, UNSUPPORTED, RANGE, ALIGN, CUDA. */
 esb_status esb_gemm(int64_t M, int64_t N, int64_t K,
                     const uint32_t* A, int64_t lda, esb_format fa,
@@ -312,7 +318,8 @@ esb_status esb_gemm(int64_t M, int64_t N, int64_t K,
  * exact in fp32) and adds them as integers (the int32 accumulator, and
  * float(acc) rounded to nearest for the epilogue), so the call takes
  * K max|I_A| max|I_B| < 2^31 when the chunks fit (four) and the output
- * codes hold a divisor of 16 per word; RANGE otherwise.  Plus
+ * codes hold a divisor of 16 per word; RANGE otherwise.  Significand-split
+ * formats (k >= 4) always run esb_gemm's kernels, with its 2^24 bound.  Plus
  *   workspace  [device] >= esb_gemm_tiled_workspace_bytes(M, N, K) bytes,
  *              16-byte aligned, contents undefined before and after (the
  *              call overwrites it)
@@ -363,8 +370,11 @@ esb_status esb_fold_bn_dn(float alpha_a, esb_format fa, float alpha_w, esb_forma
  * M = n*P*Q output pixels, N = cout, K = r*s*c, followed by the fused
  * epilogue.  P = (h + 2 pad - r)/stride + 1, Q likewise.
  *   X [device] n*h*w pixel rows of ldx words (c codes each), ldx % 4 == 0
- *   W [device] cout*r*s rows of ldw words (c codes each); ldw == ldx
+ *   W [device] cout*r*s rows of ldw words (c codes each, in fw, which may
+ *     differ from fx in width and k), ldw % 4 == 0
  *   outputs as esb_gemm with M = n*P*Q rows (pixel-major NHWC).
+ * The formats follow esb_gemm (one E4M3 byte per code, or the significand
+ * split for k >= 4), with K = r*s*c real terms in the 2^24 bound.
  * groups == c selects the depthwise path (one r x s filter per channel, W
  * holds r*s rows of ldw words with c codes each, cout == c), which runs on
  * CUDA cores (no dense contraction): exact int32 sums of r*s products, the
@@ -389,7 +399,9 @@ enum {
 
 /* Which of the kernels above esb_conv2d_nhwc launches for geometry d, X
  * row stride ldx and formats fx, fw, when its packed output codes have
- * out_b bits (0: no code output).  The choice depends only on these and on
+ * out_b bits (0: no code output).  The filter stride is taken to be ldx
+ * when fw.b == fx.b and esb_row_words(c, fw.b) otherwise; the halo kernel
+ * needs 4-bit codes of the same layout on both sides.  The choice depends only on these and on
  * the device's shared memory (queried on the current device); results are
  * identical whichever kernel runs.  Setting ESB_CONV_IM2COL=1 in the
  * environment before the first call disables the halo kernel.

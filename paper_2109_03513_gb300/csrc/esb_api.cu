@@ -105,13 +105,17 @@ bool fmt_ok(const esb_format& f)
     return f.b >= 2 && f.b <= 8 && f.k >= 0 && f.k <= f.b - 1 && (f.is_signed == 0 || f.is_signed == 1);
 }
 
-// The tensor-core operand route: the scaled-E4M3 image needs k <= 3 and an
-// exponent field of at most 4 bits, and must avoid the E4M3 NaN pattern
-// (exponent 15 with mantissa 111, i.e. b-k-1 = 4 and k = 3).
+// The tensor-core operand routes: one scaled E4M3 byte per code needs
+// k <= 3 and an exponent field of at most 4 bits, and must avoid the E4M3
+// NaN pattern (exponent 15 with mantissa 111, i.e. b-k-1 = 4 and k = 3);
+// wider significands (k >= 4, at most 8 significant bits, shifts up to 6
+// for b <= 8) take the significand split into two exact E4M3 planes.
+// Other formats (exponent fields of 5+ bits) have images far past the
+// int32 bound and are not contracted.
 bool fmt_tc_ok(const esb_format& f)
 {
     const int ew = f.b - f.k - 1;
-    return f.k <= 3 && ew <= 4 && !(ew == 4 && f.k == 3);
+    return (f.k <= 3 && ew <= 4 && !(ew == 4 && f.k == 3)) || f.k >= 4;
 }
 
 int64_t words_for(int64_t cols, int b) { return (cols + (32 / b) - 1) / (32 / b); }
@@ -432,8 +436,7 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d, const uint32_t* X, int64_t ld
         return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
     }
     if (d->groups != 1) return ESB_ERR_UNSUPPORTED;
-    if (ldw != ldx) return ESB_ERR_INVALID_ARG;
-    if (fx.b != fw.b) return ESB_ERR_UNSUPPORTED;
+    if (ldw < words_for(d->c, fw.b)) return ESB_ERR_INVALID_ARG;
     if (!fmt_tc_ok(fx) || !fmt_tc_ok(fw)) return ESB_ERR_UNSUPPORTED;
     esb_status s = check_epilogue(ep, M, d->cout, want_codes || y_out != nullptr);
     if (s != ESB_OK) return s;
@@ -445,7 +448,7 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d, const uint32_t* X, int64_t ld
     if (M == 0) return ESB_OK;
     if (!X || !W) return ESB_ERR_INVALID_ARG;
     if (!acc_out && !y_out && !codes_out) return ESB_OK;
-    if (!aligned16(X) || !aligned16(W) || (ldx & 3)) return ESB_ERR_ALIGN;
+    if (!aligned16(X) || !aligned16(W) || (ldx & 3) || (ldw & 3)) return ESB_ERR_ALIGN;
     if (M > (int64_t)65535 * 128 * 256) return ESB_ERR_UNSUPPORTED;
     if (!gemm_pick_ok(d->cout, want_codes ? ep->fmt_out.b : 4)) return ESB_ERR_UNSUPPORTED;
     GemmOutputs o{ep, acc_out, y_out, codes_out, ldo};
@@ -468,10 +471,12 @@ esb_status esb_conv2d_kernel(const esb_conv_desc* d, int64_t ldx, esb_format fx,
         *kernel = ESB_CONV_KERNEL_DEPTHWISE;
         return ESB_OK;
     }
-    if (d->groups != 1 || fx.b != fw.b || !fmt_tc_ok(fx) || !fmt_tc_ok(fw) || (ldx & 3)) return ESB_ERR_INVALID_ARG;
+    if (d->groups != 1 || !fmt_tc_ok(fx) || !fmt_tc_ok(fw) || (ldx & 3)) return ESB_ERR_INVALID_ARG;
     const int P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
     const int Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
-    const int k = conv_kernel_choice(*d, P, Q, ldx, fx.b, fx.k, out_b ? out_b : 4);
+    // the filter stride: ldx for the same code width, else the smallest one
+    const int64_t ldw = fw.b == fx.b ? ldx : esb_row_words(d->c, fw.b);
+    const int k = conv_kernel_choice(*d, P, Q, ldx, fx.b, fx.k, ldw, fw.b, fw.k, out_b ? out_b : 4);
     if (k < 0) return ESB_ERR_CUDA;
     *kernel = k;
     return ESB_OK;

@@ -461,7 +461,8 @@ static bool halo_plan(const esb_conv_desc& d, int P, int Q, int64_t ldx, const O
                       HaloPlan* hp, cudaError_t* err)
 {
     *err = cudaSuccess;
-    if (d.stride != 1 || fa.b != 4 || ldx % 4 != 0 || ldx > (1 << 20) || d.pad > d.r - 1 || d.pad > d.s - 1)
+    if (d.stride != 1 || fa.b != 4 || fa.planes != 1 || ldx % 4 != 0 || ldx > (1 << 20) || d.pad > d.r - 1 ||
+        d.pad > d.s - 1)
         return false;
     int lws = 0;
     while ((1 << lws) < d.w + d.pad) lws++;
@@ -540,7 +541,7 @@ bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, i
     if (per_n > m_tiles) per_n = m_tiles;
     const int64_t grid = per_n * n_tiles;
     RowsSrc b{W, (int64_t)d.r * d.s * ldw, N};
-    const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
+    const float acc_scale = ldexpf(1.0f, fa.csc + fb.csc);
     // The specialised instance: 4-bit B, bulk-copied input rows and 4-bit
     // codes as the only output, with a scalar scale and bias, in whole N-tiles
     // and with a monotone requantisation (unsigned codes or an activation).

@@ -99,6 +99,13 @@ struct ConvSrc {
         }
     }
     __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const { return tap_ptr(x, c.r, c.s, c.word); }
+    __host__ __device__ __forceinline__ bool linear() const { return true; }
+    __device__ __forceinline__ const uint32_t* code_word(const Row& x, int64_t kk, int cpw, int& slot) const
+    {
+        const int64_t wi = kk / cpw;
+        slot = (int)(kk - wi * cpw);
+        return words(x, wi);
+    }
 };
 
 // Fast decode of a full b = 4 unit (two words) at a cursor.
@@ -121,7 +128,7 @@ template <class Src>
 __device__ __forceinline__ uint4 decode_unit(const Src& src, const typename Src::Row& row, int64_t k0, int64_t K,
                                              const OpFmt& f)
 {
-    if (f.b == 4 && k0 + 16 <= K) return decode_unit_b4(src, row, src.cursor(k0 >> 3), f);
+    if (f.b == 4 && f.planes == 1 && src.linear() && k0 + 16 <= K) return decode_unit_b4(src, row, src.cursor(k0 >> 3), f);
     return decode_unit_any(src, row, k0, K, f);
 }
 
@@ -396,7 +403,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
             }
             if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
             uint8_t* st = sA + s * kBM * kBK;
-            if (fa.b == 4) {
+            if (fa.b == 4 && fa.planes == 1) {
                 const int64_t kw0 = (int64_t)kb * 16;
                 typename SrcA::Cursor cur[4];
 #pragma unroll
@@ -513,7 +520,7 @@ static cudaError_t launch_tc(const SrcA& a, const SrcB& b, int64_t M, int64_t N,
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
+    const float acc_scale = ldexpf(1.0f, fa.csc + fb.csc);
     dim3 grid((unsigned)((M + kBM - 1) / kBM), (unsigned)((N + BN - 1) / BN));
     esb_gemm_tc_kernel<SrcA, SrcB><<<grid, kGemmThreads, smem, st>>>(a, b, M, N, K, fa, fb, BN, acc_scale, ep);
     return cudaGetLastError();
@@ -556,7 +563,7 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
     if (per_n < 1) per_n = 1;
     if (per_n > m_tiles) per_n = m_tiles;
     const int64_t grid = per_n * n_tiles;
-    const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
+    const float acc_scale = ldexpf(1.0f, fa.csc + fb.csc);
     *err = launch_pdl(esb_gemm_ws_kernel<SrcA>, dim3((unsigned)grid), dim3(kWsThreads), (size_t)L.smem_bytes, st, a, b,
                       M, N, K, fa, fb, BN, L.nkb, L.stages, n_tiles, m_tiles, acc_scale, ep);
     return true;
@@ -616,12 +623,13 @@ cudaError_t launch_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int6
     const int BN = pick_bn(N, ep.out_cpw);
     RowsSrc a{A, lda, M};
     RowsSrc b{B, ldb, N};
-    const OpFmt fa = make_opfmt(ba, ka), fb = make_opfmt(bb, kb);
-    if (K > 0) {
+    OpFmt fa = make_opfmt(ba, ka), fb = make_opfmt(bb, kb);
+    const int64_t Kx = plan_planes(fa, fb, K);        // the kernels' K (significand planes)
+    if (Kx > 0) {
         cudaError_t e = cudaSuccess;
-        if (launch_ws(a, b, M, N, K, fa, fb, BN, ep, st, &e)) return e;
+        if (launch_ws(a, b, M, N, Kx, fa, fb, BN, ep, st, &e)) return e;
     }
-    return launch_tc(a, b, M, N, K, fa, fb, BN, ep, st);
+    return launch_tc(a, b, M, N, Kx, fa, fb, BN, ep, st);
 }
 
 // ESB_CONV_IM2COL=1 in the environment (read once) routes every dense
@@ -650,22 +658,36 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
     a.X = X; a.ldx = (int)ldx; a.rows = (int)M; a.H = d.h; a.W = d.w; a.P = P; a.Q = Q; a.S = d.s;
     a.stride = d.stride; a.pad = d.pad;
     RowsSrc b{W, (int64_t)d.r * d.s * ldw, N};
-    const OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
+    if (bw != bx || ldw != ldx) {
+        // filters of another code width: K runs over taps of the input's
+        // ldx * cpw_x codes; each tap of a filter row holds ldw words
+        b.kp = ldx * (32 / bx);
+        b.ldt = ldw;
+    }
+    OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
+    const int64_t Kx = plan_planes(fa, fb, K);        // the kernels' K (significand planes)
     cudaError_t e = cudaSuccess;
-    if (K > 0 && !conv_force_im2col() && launch_conv_halo(d, P, Q, X, ldx, fa, W, ldw, fb, BN, ep, st, &e)) return e;
-    if (K > 0 && launch_ws(a, b, M, N, K, fa, fb, BN, ep, st, &e)) return e;
-    return launch_tc(a, b, M, N, K, fa, fb, BN, ep, st);
+    if (Kx > 0 && !conv_force_im2col() && fa.planes == 1 && b.linear() &&
+        launch_conv_halo(d, P, Q, X, ldx, fa, W, ldw, fb, BN, ep, st, &e))
+        return e;
+    if (Kx > 0 && launch_ws(a, b, M, N, Kx, fa, fb, BN, ep, st, &e)) return e;
+    return launch_tc(a, b, M, N, Kx, fa, fb, BN, ep, st);
 }
 
-int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int kx, int out_b)
+int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int kx, int64_t ldw, int bw,
+                       int kw, int out_b)
 {
     const int cpw = 32 / out_b;
     const int64_t K = (int64_t)d.r * d.s * ldx * (32 / bx);
-    if (K > 0 && !conv_force_im2col() && conv_halo_ok(d, P, Q, ldx, bx, kx, cpw)) return ESB_CONV_KERNEL_HALO;
+    OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
+    const int64_t Kx = plan_planes(fa, fb, K);
+    const bool same_layout = bw == bx && ldw == ldx && fa.planes == 1;
+    if (Kx > 0 && !conv_force_im2col() && same_layout && conv_halo_ok(d, P, Q, ldx, bx, kx, cpw))
+        return ESB_CONV_KERNEL_HALO;
     cudaError_t e = cudaSuccess;
     const int st = ws_static_smem<ConvSrc>(&e);
     if (st < 0) return -1;
-    if (K > 0 && ws_layout(K, pick_bn(d.cout, cpw), max_dyn_smem() - st).stages >= 3) return ESB_CONV_KERNEL_IM2COL;
+    if (Kx > 0 && ws_layout(Kx, pick_bn(d.cout, cpw), max_dyn_smem() - st).stages >= 3) return ESB_CONV_KERNEL_IM2COL;
     return ESB_CONV_KERNEL_STREAMED;
 }
 

@@ -350,6 +350,8 @@ size_t gemm_tiled_workspace_bytes(int64_t M, int64_t N, int64_t K)
 bool gemm_tiled_ok(int64_t M, int64_t N, int64_t K, int ba, int ka, int bb, int kb, int out_cpw)
 {
     int kbc, nch, BN;
+    // significand-split operands (k >= 4) take esb_gemm's kernels
+    if (fmt_needs_split(ba, ka) || fmt_needs_split(bb, kb)) return false;
     if (M <= 0 || N < kTiledBN || K <= 0 || !tiled_plan(K, ba, ka, bb, kb, &kbc, &nch, &BN)) return false;
     if (kTiledBN % out_cpw != 0 || (nch > 1 && 16 % out_cpw != 0)) return false;
     if (nch > 1) return true;                                     // only this path takes that K
@@ -430,7 +432,7 @@ cudaError_t launch_gemm_tiled(int64_t M, int64_t N, int64_t K, const uint32_t* A
     if (per_n < 1) per_n = 1;
     if (per_n > m_tiles) per_n = m_tiles;
     const int64_t grid = per_n * n_tiles;
-    const float acc_scale = ldexpf(1.0f, fa.k + fb.k + 12);
+    const float acc_scale = ldexpf(1.0f, fa.csc + fb.csc);
     // the specialised epilogue: 4-bit codes as the only output with a scalar
     // scale and bias, whole N-tiles, a monotone requantisation, K in one chunk
     const bool fast = nch == 1 && BN == 256 && ep.codes_out && ep.out.b == 4 && !ep.scale && !ep.bias &&

@@ -73,7 +73,8 @@ cudaError_t launch_gemm_tiled(int64_t M, int64_t N, int64_t K, const uint32_t* A
                               cudaStream_t st);
 // Kernel esb_conv2d_nhwc launches for a dense convolution (an
 // esb_conv_kernel value), or -1 when the device cannot be queried.
-int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int kx, int out_b);
+int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int kx, int64_t ldw, int bw,
+                       int kw, int out_b);
 
 cudaError_t launch_dwconv(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
                           const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st);

@@ -17,16 +17,64 @@ constexpr int kBM = 128;           // rows per tile (TMEM lanes)
 constexpr int kBK = 128;           // codes (= E4M3 bytes) per K-block: one 128-byte swizzle row
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s
 
+// Operand format of a contraction kernel.  A code whose integer image is an
+// exact E4M3 number times 2^-(k+6) (k <= 3, exponent field <= 4 bits) is
+// one E4M3 byte ("whole").  Wider significands (k >= 4: up to 8
+// significant bits) take the significand split: I = (-1)^s m 2^sh with
+// m = 16 m_hi + m_lo becomes two E4M3 bytes, m_hi 2^(sh+4) 2^-9 ("high")
+// and m_lo 2^sh 2^-9 ("low"), each exact (at most 4 significant bits), and
+// the two planes are separate 16-code units of an expanded K.  When either
+// operand is split the logical K of the kernels is planes x K16 (K16 = K
+// rounded up to 16): unit u' of it is plane u' % planes of code unit
+// u' / planes, with the roles of pmap (2 bits per plane: 0 whole, 1 high,
+// 2 low), chosen so that the products of the planes add up to I_A I_B:
+// one split operand [H, L] against [W, W]; both split [H, H, L, L] against
+// [H, L, H, L].  Every product is a multiple of 2^-(csc_A + csc_B), and the
+// sum of their magnitudes is sum |I_A| |I_B| in that unit, so the fp32 TMEM
+// accumulation is exact under the same bound as without the split.
 struct OpFmt {
     int b, k, ew, cpw;
     uint32_t mask;
+    int planes;          // 1, 2 or 4 units of the kernel's K per 16 codes
+    uint32_t pmap;       // role of plane i in bits 2i, 2i+1
+    int csc;             // operand scale: decoded values are I 2^-csc
+    int64_t korig;       // codes per row before the expansion (K tail)
 };
+
+// Significand split needed: the image is not an E4M3 number times a power of two.
+__host__ __device__ inline bool fmt_needs_split(int b, int k)
+{
+    const int ew = b - k - 1;
+    return k > 3 || ew > 4 || (ew == 4 && k == 3);
+}
 
 __host__ inline OpFmt make_opfmt(int b, int k)
 {
     OpFmt o;
     o.b = b; o.k = k; o.ew = b - k - 1; o.cpw = 32 / b; o.mask = (1u << b) - 1u;
+    o.planes = 1; o.pmap = 0u; o.csc = k + 6; o.korig = 0;
     return o;
+}
+
+// The plane layout of a pair of operands (see OpFmt) for a contraction of
+// K codes; returns the kernels' K (K itself when neither is split).
+__host__ inline int64_t plan_planes(OpFmt& fa, OpFmt& fb, int64_t K)
+{
+    const bool sa = fmt_needs_split(fa.b, fa.k), sb = fmt_needs_split(fb.b, fb.k);
+    fa.korig = fb.korig = K;
+    if (!sa && !sb) return K;
+    const int P = (sa && sb) ? 4 : 2;
+    fa.planes = fb.planes = P;
+    if (sa && sb) {
+        fa.pmap = 1u | (1u << 2) | (2u << 4) | (2u << 6);      // H H L L
+        fb.pmap = 1u | (2u << 2) | (1u << 4) | (2u << 6);      // H L H L
+    } else {
+        (sa ? fa : fb).pmap = 1u | (2u << 2);                  // H L
+        (sa ? fb : fa).pmap = 0u;                              // W W
+    }
+    if (sa) fa.csc = 9;
+    if (sb) fb.csc = 9;
+    return (int64_t)P * ((K + 15) / 16) * 16;
 }
 
 // Byte position of code j (0..15) of a 16-code unit.  The fast b = 4
@@ -48,6 +96,26 @@ __device__ __forceinline__ uint32_t code_to_e4m3(uint32_t c, const OpFmt& f)
     return (s << 7) | (E << 3) | (fr << (3 - f.k));
 }
 
+// One code -> the E4M3 byte of one significand plane (role 1: high part,
+// role 2: low part; see OpFmt), value m_part 2^(shift - 9).
+__device__ __forceinline__ uint32_t code_to_e4m3_part(uint32_t c, const OpFmt& f, uint32_t role)
+{
+    const uint32_t s = (c >> (f.b - 1)) & 1u;
+    const uint32_t fr = c & ((1u << f.k) - 1u);
+    const uint32_t N = (1u << f.ew) - 1u;
+    const uint32_t e = f.ew > 0 ? (c >> f.k) & N : N;
+    const uint32_t m = (e == N) ? fr : ((1u << f.k) | fr);
+    const int sh = (e == N) ? 0 : (int)e;
+    const uint32_t part = (role == 1u) ? (m >> 4) : (m & 15u);
+    const int shift = (role == 1u) ? sh + 4 : sh;
+    if (part == 0u) return 0u;
+    const int t = 31 - __clz(part);                                 // 0 .. 3
+    const int E = shift + t - 2;                                    // biased: (shift - 9 + t) + 7
+    const uint32_t mag = (E >= 1) ? (((uint32_t)E << 3) | ((part << (3 - t)) & 7u))
+                                  : (part << shift);                // subnormal: part 2^shift <= 7
+    return (s << 7) | mag;
+}
+
 // 8 four-bit codes (one word) -> 8 scaled E4M3 bytes (lo: codes 0,2,4,6; hi: 1,3,5,7).
 __device__ __forceinline__ void decode_word_b4(uint32_t w, int k, int ew, uint32_t& lo, uint32_t& hi)
 {
@@ -62,36 +130,65 @@ __device__ __forceinline__ void decode_word_b4(uint32_t w, int k, int ew, uint32
 
 // ------------------------------------------------------------ row sources
 
-// Plain K-major rows: logical word w of row r is base[r * ld + w].
+// Plain K-major rows: logical word w of row r is base[r * ld + w].  With
+// kp > 0 the rows are convolution filters whose K runs over taps of kp
+// codes (the input's codes per pixel) while each tap of the row holds ldt
+// words of this operand's width: code kk is channel kk % kp of tap kk / kp,
+// and channels past the tap's words read as zero (mixed code widths).
 struct RowsSrc {
     const uint32_t* base;
     int64_t ld;
     int64_t rows;
+    int64_t kp = 0;
+    int64_t ldt = 0;
     struct Row { const uint32_t* p; };
     struct Cursor { int64_t w; };
+    __host__ __device__ __forceinline__ bool linear() const { return kp == 0; }
     __device__ __forceinline__ Row row(int64_t r) const { Row x; x.p = (r < rows) ? base + r * ld : nullptr; return x; }
     __device__ __forceinline__ const uint32_t* words(const Row& x, int64_t w) const { return x.p ? x.p + w : nullptr; }
+    // Word holding code kk of row x (nullptr: the zero code) and its slot.
+    __device__ __forceinline__ const uint32_t* code_word(const Row& x, int64_t kk, int cpw, int& slot) const
+    {
+        if (kp == 0) {
+            const int64_t wi = kk / cpw;
+            slot = (int)(kk - wi * cpw);
+            return words(x, wi);
+        }
+        const int64_t tap = kk / kp;
+        const int64_t c = kk - tap * kp;
+        const int64_t wi = c / cpw;
+        slot = (int)(c - wi * cpw);
+        return wi < ldt ? words(x, tap * ldt + wi) : nullptr;
+    }
     __device__ __forceinline__ Cursor cursor(int64_t w) const { Cursor c; c.w = w; return c; }
     __device__ __forceinline__ void advance(Cursor& c, int dw) const { c.w += dw; }
     __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const { return x.p ? x.p + c.w : nullptr; }
 };
 
-// General decode of the 16-code unit [k0, k0 + 16) of one row (any b, K tail).
+// General decode of the 16-code unit [k0, k0 + 16) of the kernel's K of
+// one row (any b, K tail, significand planes: see OpFmt).
 template <class Src>
 __device__ __noinline__ uint4 decode_unit_any(const Src& src, const typename Src::Row& row, int64_t k0, int64_t K,
                                               const OpFmt f)
 {
     uint32_t o0 = 0u, o1 = 0u, o2 = 0u, o3 = 0u;
+    uint32_t role = 0u;
+    if (f.planes > 1) {                               // unit k0 / 16 = plane of code unit (k0 / 16) / planes
+        const int64_t u = k0 >> 4;
+        const int64_t cu = u / f.planes;
+        role = (f.pmap >> (2 * (int)(u - cu * f.planes))) & 3u;
+        k0 = cu * 16;
+        K = f.korig;
+    }
 #pragma unroll 1
     for (int j = 0; j < 16; j++) {
         const int64_t kk = k0 + j;
         if (kk >= K) break;
-        const int64_t wi = kk / f.cpw;
-        const int slot = (int)(kk - wi * f.cpw);
-        const uint32_t* p = src.words(row, wi);
+        int slot = 0;
+        const uint32_t* p = src.code_word(row, kk, f.cpw, slot);
         if (!p) continue;
         const uint32_t c = (__ldg(p) >> (f.b * slot)) & f.mask;
-        const uint32_t byte = code_to_e4m3(c, f);
+        const uint32_t byte = role ? code_to_e4m3_part(c, f, role) : code_to_e4m3(c, f);
         const int pos = unit_pos(j);
         const uint32_t v = byte << (8 * (pos & 3));
         switch (pos >> 2) {
@@ -389,7 +486,7 @@ template <bool B4>
 __device__ __forceinline__ void ws_decode_b(const RowsSrc& srcB, int64_t n0, int64_t K, const OpFmt& fb, int BN,
                                             int nkb, uint8_t* sB, int t, int nthreads)
 {
-    if (B4 || fb.b == 4) {
+    if (B4 || (fb.b == 4 && fb.planes == 1 && srcB.linear())) {
         // one row chunk per thread and pass (compact: this code runs cold,
         // once per CTA, on the path to the first MMA)
         const uint32_t zw = fmt_zero_code(4, fb.k) * 0x11111111u;

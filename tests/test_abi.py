@@ -88,8 +88,8 @@ def test_host_validation_without_device(lib):
     ep = esb.Epilogue().c()
     assert lib.esb_gemm(128, 64, 8192, fake, 2048, big, fake, 2048, big, ctypes.byref(ep), fake, null, null, 0,
                         null) == esb.ESB_ERR_RANGE
-    f64 = esb.esb_format(6, 4, 1)     # 5 significant bits: not an E4M3 image
-    assert lib.esb_gemm(128, 64, 64, fake, 16, f64, fake, 16, f64, ctypes.byref(ep), fake, null, null, 0,
+    f71 = esb.esb_format(7, 1, 1)     # 5-bit exponent field: no E4M3 image, no significand split
+    assert lib.esb_gemm(128, 64, 64, fake, 16, f71, fake, 16, f71, ctypes.byref(ep), fake, null, null, 0,
                         null) == esb.ESB_ERR_UNSUPPORTED
     assert lib.esb_gemm(128, 64, 64, fake, 4, f, fake, 8, f, ctypes.byref(ep), fake, null, null, 0,
                         null) == esb.ESB_ERR_INVALID_ARG
@@ -98,8 +98,14 @@ def test_host_validation_without_device(lib):
     assert lib.esb_gemm(0, 64, 64, fake, 8, f, fake, 8, f, ctypes.byref(ep), fake, null, null, 0,
                         null) == esb.ESB_OK
     d = esb.esb_conv_desc(1, 8, 8, 64, 64, 3, 3, 1, 1, 1)
-    assert lib.esb_conv2d_nhwc(ctypes.byref(d), fake, 8, f, fake, 12, f, ctypes.byref(ep), fake, null, null, 0,
+    assert lib.esb_conv2d_nhwc(ctypes.byref(d), fake, 8, f, fake, 7, f, ctypes.byref(ep), fake, null, null, 0,
                                null) == esb.ESB_ERR_INVALID_ARG
+    # filter rows of another width: stride for their own codes, 16-byte multiple
+    f63 = esb.esb_format(6, 3, 1)
+    assert lib.esb_conv2d_nhwc(ctypes.byref(d), fake, 8, f, fake, 12, f63, ctypes.byref(ep), fake, null, null, 0,
+                               null) == esb.ESB_ERR_INVALID_ARG
+    assert lib.esb_conv2d_nhwc(ctypes.byref(d), fake, 8, f, fake, 14, f63, ctypes.byref(ep), fake, null, null, 0,
+                               null) == esb.ESB_ERR_ALIGN
     d2 = esb.esb_conv_desc(1, 8, 8, 64, 64, 3, 3, 1, 3, 1)
     assert lib.esb_conv2d_nhwc(ctypes.byref(d2), fake, 8, f, fake, 8, f, ctypes.byref(ep), fake, null, null, 0,
                                null) == esb.ESB_ERR_INVALID_ARG
