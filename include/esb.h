@@ -411,6 +411,40 @@ enum {
 esb_status esb_conv2d_kernel(const esb_conv_desc* d, int64_t ldx, esb_format fx, esb_format fw, int32_t out_b,
                              int32_t* kernel);
 
+/* ------------------------------------------------- int64 contraction */
+
+/* The ESB contraction on the CUDA cores with exact int64 accumulators, for
+ * formats and sizes outside the tensor-core path (power-of-two-like sets
+ * such as (5,0), (6,1), (6,0), whose images reach 2^30, or sums past
+ * 2^24).  Eq. esb_multiplication: each product of two set elements is the
+ * product of their significands shifted by the sum of their exponents;
+ * every multiply-accumulate here is one small integer product, one 64-bit
+ * shift and one 64-bit add.
+ *   A, lda, fa, B, ldb, fb, ep, y_out, codes_out, ldo: as esb_gemm (any
+ *       formats; no alignment requirement)
+ *   acc_out [device] M x N int64 (row stride N), or NULL
+ * The epilogue takes float(acc) rounded to nearest.  Requires
+ * K * max|I_A| * max|I_B| < 2^62 (else ESB_ERR_RANGE).
+ * Errors: INVALID_ARG, UNSUPPORTED, RANGE, CUDA. */
+esb_status esb_gemm_i64(int64_t M, int64_t N, int64_t K,
+                        const uint32_t* A, int64_t lda, esb_format fa,
+                        const uint32_t* B, int64_t ldb, esb_format fb,
+                        const esb_epilogue* ep,
+                        int64_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
+                        void* stream);
+
+/* esb_conv2d_nhwc (groups == 1) on the int64 path of esb_gemm_i64: any
+ * formats, input and filter codes of different widths, ldx and ldw any
+ * strides that hold c codes; acc_out [device] n*P*Q x cout int64 or NULL.
+ * Requires r*s*c * max|I_X| * max|I_W| < 2^62.
+ * Errors: INVALID_ARG, UNSUPPORTED, RANGE, CUDA. */
+esb_status esb_conv2d_nhwc_i64(const esb_conv_desc* d,
+                               const uint32_t* X, int64_t ldx, esb_format fx,
+                               const uint32_t* W, int64_t ldw, esb_format fw,
+                               const esb_epilogue* ep,
+                               int64_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo,
+                               void* stream);
+
 /* -------------------------------------------------------------- pooling */
 
 /* Max pooling of ESB codes, NHWC (Sec. IV-B "MP" stage with the

@@ -456,6 +456,62 @@ esb_status esb_conv2d_nhwc(const esb_conv_desc* d, const uint32_t* X, int64_t ld
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 
+// Bound of the int64 path: the sum of |I_A| |I_B| over K stays below 2^62.
+static bool i64_bound_ok(int64_t K, esb_format fa, esb_format fb)
+{
+    return (double)K * fmt_max_image(fa.b, fa.k) * fmt_max_image(fb.b, fb.k) < 4611686018427387904.0;
+}
+
+esb_status esb_gemm_i64(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, esb_format fa,
+                        const uint32_t* B, int64_t ldb, esb_format fb, const esb_epilogue* ep, int64_t* acc_out,
+                        float* y_out, uint32_t* codes_out, int64_t ldo, void* stream)
+{
+    if (!fmt_ok(fa) || !fmt_ok(fb)) return ESB_ERR_UNSUPPORTED;
+    if (M < 0 || N < 0 || K < 0) return ESB_ERR_INVALID_ARG;
+    if (lda < words_for(K, fa.b) || ldb < words_for(K, fb.b)) return ESB_ERR_INVALID_ARG;
+    const bool want_codes = codes_out != nullptr;
+    esb_status s = check_epilogue(ep, M, N, want_codes || y_out != nullptr);
+    if (s != ESB_OK) return s;
+    if (want_codes && ldo < words_for(N, ep->fmt_out.b)) return ESB_ERR_INVALID_ARG;
+    if (!i64_bound_ok(K, fa, fb)) return ESB_ERR_RANGE;
+    if (!shiftadd_grid_ok(M, N, want_codes ? ep->fmt_out.b : 4)) return ESB_ERR_UNSUPPORTED;
+    if (M == 0 || N == 0 || (!acc_out && !y_out && !codes_out)) return ESB_OK;
+    if (K > 0 && (!A || !B)) return ESB_ERR_INVALID_ARG;
+    GemmOutputs o{ep, nullptr, y_out, codes_out, ldo};
+    const cudaError_t e = launch_gemm_i64(M, N, K, A, lda, fa.b, fa.k, B, ldb, fb.b, fb.k, acc_out, o,
+                                          static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_conv2d_nhwc_i64(const esb_conv_desc* d, const uint32_t* X, int64_t ldx, esb_format fx,
+                               const uint32_t* W, int64_t ldw, esb_format fw, const esb_epilogue* ep,
+                               int64_t* acc_out, float* y_out, uint32_t* codes_out, int64_t ldo, void* stream)
+{
+    if (!d) return ESB_ERR_INVALID_ARG;
+    if (!fmt_ok(fx) || !fmt_ok(fw)) return ESB_ERR_UNSUPPORTED;
+    if (d->n < 0 || d->h <= 0 || d->w <= 0 || d->c <= 0 || d->cout <= 0 || d->r <= 0 || d->s <= 0 ||
+        d->stride <= 0 || d->pad < 0 || d->pad >= d->r || d->pad >= d->s)
+        return ESB_ERR_INVALID_ARG;
+    if (d->h + 2 * d->pad < d->r || d->w + 2 * d->pad < d->s) return ESB_ERR_INVALID_ARG;
+    if (d->groups != 1) return ESB_ERR_UNSUPPORTED;
+    if (ldx < words_for(d->c, fx.b) || ldw < words_for(d->c, fw.b)) return ESB_ERR_INVALID_ARG;
+    const int P = (d->h + 2 * d->pad - d->r) / d->stride + 1;
+    const int Q = (d->w + 2 * d->pad - d->s) / d->stride + 1;
+    const int64_t M = (int64_t)d->n * P * Q;
+    const bool want_codes = codes_out != nullptr;
+    esb_status s = check_epilogue(ep, M, d->cout, want_codes || y_out != nullptr);
+    if (s != ESB_OK) return s;
+    if (want_codes && ldo < words_for(d->cout, ep->fmt_out.b)) return ESB_ERR_INVALID_ARG;
+    if (!i64_bound_ok((int64_t)d->r * d->s * d->c, fx, fw)) return ESB_ERR_RANGE;
+    if (!shiftadd_grid_ok(M, d->cout, want_codes ? ep->fmt_out.b : 4)) return ESB_ERR_UNSUPPORTED;
+    if (M == 0 || (!acc_out && !y_out && !codes_out)) return ESB_OK;
+    if (!X || !W) return ESB_ERR_INVALID_ARG;
+    GemmOutputs o{ep, nullptr, y_out, codes_out, ldo};
+    const cudaError_t e = launch_conv_i64(*d, P, Q, X, ldx, fx.b, fx.k, W, ldw, fw.b, fw.k, acc_out, o,
+                                          static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
 esb_status esb_conv2d_kernel(const esb_conv_desc* d, int64_t ldx, esb_format fx, esb_format fw, int32_t out_b,
                              int32_t* kernel)
 {

@@ -99,6 +99,9 @@ SIGNATURES = {
                               _P, _SZ, _P]),
     "esb_conv2d_nhwc": (_I32, [_P, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
     "esb_conv2d_kernel": (_I32, [_P, _I64, esb_format, esb_format, _I32, _P]),
+    "esb_gemm_i64": (_I32, [_I64, _I64, _I64, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64,
+                            _P]),
+    "esb_conv2d_nhwc_i64": (_I32, [_P, _P, _I64, esb_format, _P, _I64, esb_format, _P, _P, _P, _P, _I64, _P]),
     "esb_maxpool_nhwc": (_I32, [_P, _I64, esb_format] + [_I32] * 7 + [_P, _I64, _P]),
     "esb_avgpool_nhwc": (_I32, [_P, _I64, esb_format, _I32, _I32, _I32, _F32, _F32, esb_format, _I32, _P, _P, _I64,
                                 _P]),
@@ -335,6 +338,45 @@ def esb_gemm(A: torch.Tensor, fa: Fmt, B: torch.Tensor, fb: Fmt, K: int, ep: Opt
     _check(lib().esb_gemm(M, N, K, _ptr(A), lda, fa.c(), _ptr(B), ldb, fb.c(),
                           ctypes.byref(epc) if epc is not None else None,
                           _ptr(acc), _ptr(y), _ptr(codes), ldo, _stream(stream)), "esb_gemm")
+    return acc, y, codes
+
+
+def esb_gemm_i64(A: torch.Tensor, fa: Fmt, B: torch.Tensor, fb: Fmt, K: int, ep: Optional[Epilogue] = None,
+                 want_acc: bool = True, want_y: bool = False, want_codes: bool = False, stream=None):
+    """CUDA-core contraction with int64 accumulators -> (acc int64 (M,N) | None,
+    y fp32 (M,N) | None, codes int32 (M, ldo) | None)."""
+    _dev(A, "A"); _dev(B, "B")
+    M, lda = A.shape
+    N, ldb = B.shape
+    dev = A.device
+    acc = torch.empty((M, N), dtype=torch.int64, device=dev) if want_acc else None
+    y = torch.empty((M, N), dtype=torch.float32, device=dev) if want_y else None
+    codes = torch.empty((M, esb_row_words(N, ep.fmt_out.b)), dtype=torch.int32, device=dev) if want_codes else None
+    ldo = codes.shape[-1] if codes is not None else 0
+    epc = ep.c() if ep is not None else None
+    _check(lib().esb_gemm_i64(M, N, K, _ptr(A), lda, fa.c(), _ptr(B), ldb, fb.c(),
+                              ctypes.byref(epc) if epc is not None else None, _ptr(acc), _ptr(y), _ptr(codes), ldo,
+                              _stream(stream)), "esb_gemm_i64")
+    return acc, y, codes
+
+
+def esb_conv2d_nhwc_i64(X: torch.Tensor, fx: Fmt, W: torch.Tensor, fw: Fmt, n: int, h: int, w: int, c: int,
+                        cout: int, r: int, s: int, stride: int, pad: int, ep: Optional[Epilogue] = None,
+                        want_acc: bool = True, want_y: bool = False, want_codes: bool = False, stream=None):
+    """esb_conv2d_nhwc on the int64 CUDA-core path; outputs (n*P*Q, cout)-shaped."""
+    _dev(X, "X"); _dev(W, "W")
+    P, Q = conv_out_hw(h, w, r, s, stride, pad)
+    M = n * P * Q
+    dev = X.device
+    acc = torch.empty((M, cout), dtype=torch.int64, device=dev) if want_acc else None
+    y = torch.empty((M, cout), dtype=torch.float32, device=dev) if want_y else None
+    codes = torch.empty((M, esb_row_words(cout, ep.fmt_out.b)), dtype=torch.int32, device=dev) if want_codes else None
+    ldo = codes.shape[-1] if codes is not None else 0
+    d = esb_conv_desc(n, h, w, c, cout, r, s, stride, pad, 1)
+    epc = ep.c() if ep is not None else None
+    _check(lib().esb_conv2d_nhwc_i64(ctypes.byref(d), _ptr(X), X.shape[-1], fx.c(), _ptr(W), W.shape[-1], fw.c(),
+                                     ctypes.byref(epc) if epc is not None else None, _ptr(acc), _ptr(y), _ptr(codes),
+                                     ldo, _stream(stream)), "esb_conv2d_nhwc_i64")
     return acc, y, codes
 
 

@@ -328,6 +328,23 @@ def test_gemm_brute_force(fa, fb):
     assert o.gemm_entry(A, fa, B, fb, K, 3, 4) == exp[3, 4]
 
 
+@pytest.mark.parametrize("fa,fb", [((6, 1), (6, 1)), ((5, 0), (4, 2)), ((6, 0), (3, 1))])
+def test_gemm_large_images_brute_force(fa, fb):
+    # power-of-two-like sets with images up to 2^30: Python integers as truth
+    rng = np.random.default_rng(7)
+    M, N, K = 5, 4, 9
+    ca = rng.integers(0, 2 ** fa[0], size=(M, K), dtype=np.uint32)
+    cb = rng.integers(0, 2 ** fb[0], size=(N, K), dtype=np.uint32)
+    A = o.pack(ca, *fa, ld_words=4)
+    B = o.pack(cb, *fb, ld_words=4)
+    got = o.gemm_i64(A, fa, B, fb, M, N, K)
+    ta = [o.image(c, *fa) for c in range(2 ** fa[0])]
+    tb = [o.image(c, *fb) for c in range(2 ** fb[0])]
+    for m in range(M):
+        for n in range(N):
+            assert int(got[m, n]) == sum(ta[int(ca[m, j])] * tb[int(cb[n, j])] for j in range(K))
+
+
 def test_conv_and_depthwise_brute_force():
     rng = np.random.default_rng(5)
     fx, fw = (4, 2), (4, 1)
