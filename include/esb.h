@@ -223,6 +223,68 @@ esb_status esb_dda_combine(const double* stats, int64_t count, esb_format f, dou
 esb_status esb_calibrate_dda_noalloc(const float* x, int64_t n, esb_format f,
                                      float* alpha_out, double* stats_out, void* stream);
 
+/* ------------------------------------------ DDA for other data densities */
+
+/* Sec. III-D derives alpha* for N(0,1) data ("Resolving extremum": the
+ * paper assumes p(t) is the standard normal).  These entry points run the
+ * same objective, Eq. objective_function_expansion, and the same rule (the
+ * first local minimum of D from small alpha on [1e-4, 4], alpha =
+ * fl32(alpha* (spread + 1e-7))) for other densities of the normalised data
+ * t: a Laplace density with unit variance (heavy tails), or the data's own
+ * density, taken from a histogram of |t|. */
+enum { ESB_DIST_GAUSSIAN = 0, ESB_DIST_LAPLACE = 1 };
+
+/* Most bins of an empirical DDA histogram (one 32-bit shared-memory counter
+ * per bin and block). */
+#define ESB_DDA_MAX_BINS 12288
+
+/* alpha*(b,k) and 2 D(alpha*) for density `dist` (ESB_DIST_*); GAUSSIAN is
+ * esb_alpha_star.  Host only; cached per (b,k); thread-safe.
+ * Errors: UNSUPPORTED (format), INVALID_ARG (dist, NULL alpha_star). */
+esb_status esb_alpha_star_dist(int32_t b, int32_t k, int32_t dist, double* alpha_star, double* dda);
+
+/* esb_calibrate_dda with the alpha* of density `dist` (same statistics,
+ * same arguments and workspace rules). */
+esb_status esb_calibrate_dda_dist(const float* x, int64_t n, esb_format f, int32_t dist,
+                                  void* workspace, size_t workspace_bytes,
+                                  float* alpha_out, double* stats_out, void* stream);
+
+/* Histogram of the normalised magnitudes |t| of x: t = (x - mean) / sigma
+ * for signed formats, x / rms for unsigned ones, with {mean, spread} read
+ * from `stats` (as esb_calibrate_dda's stats_out writes them).  Bin i
+ * counts the values with floor(u) == i, u = |x - mean| * (nbins / (t_max *
+ * spread)) in fp32 (each operation rounded to nearest); values past t_max
+ * go to the last bin, NaN is skipped.
+ *   x       [device] n floats
+ *   stats   [device] 3 doubles
+ *   counts  [device] nbins uint64, overwritten (zero-filled by the call)
+ *   nbins   2 .. ESB_DDA_MAX_BINS;  t_max > 0 (in units of the spread)
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+esb_status esb_dda_histogram(const float* x, int64_t n, esb_format f, const double* stats,
+                             int32_t nbins, float t_max, unsigned long long* counts, void* stream);
+
+/* alpha* of the empirical density: the density of |t| is the histogram's,
+ * even within each bin of width t_max / nbins (half the mass on the
+ * non-negative half, as for the symmetric densities), and D is Eq.
+ * objective_function_expansion with it.  Host only.
+ *   counts [host] nbins uint64 (at least one non-zero)
+ * Errors: UNSUPPORTED (format), INVALID_ARG. */
+esb_status esb_alpha_star_hist(const unsigned long long* counts, int32_t nbins, float t_max,
+                               int32_t b, int32_t k, double* alpha_star, double* dda);
+
+/* DDA calibration with the data's own density: the statistics pass of
+ * esb_calibrate_dda, esb_dda_histogram of x, then esb_alpha_star_hist on
+ * the host and alpha = fl32(alpha* (spread + 1e-7)) written to alpha_out.
+ * Synchronises `stream` (the histogram comes back to the host).
+ *   workspace as esb_calibrate_dda; counts [device] nbins uint64 (scratch);
+ *   stats_out [device] 3 doubles (required); alpha_star_out [host] or NULL.
+ * Errors: INVALID_ARG, UNSUPPORTED, ALIGN (workspace), CUDA. */
+esb_status esb_calibrate_dda_empirical(const float* x, int64_t n, esb_format f,
+                                       void* workspace, size_t workspace_bytes,
+                                       int32_t nbins, float t_max, unsigned long long* counts,
+                                       float* alpha_out, double* stats_out, double* alpha_star_out,
+                                       void* stream);
+
 /* ------------------------------------------------------------- project */
 
 /* Cheap projection operator of Eq. cheap_projection with the
@@ -277,6 +339,50 @@ esb_status esb_project_dda(const float* x, int64_t rows, int64_t cols, esb_forma
 esb_status esb_dequant(const uint32_t* codes, int64_t rows, int64_t cols, int64_t ldc,
                        float alpha, const float* alpha_dev, esb_format f,
                        float* y, int64_t ldy, void* stream);
+
+/* ----------------------------------------- quantisation-aware training */
+
+/* Forward of one tensor in Algorithm 1 (DNN training with ESB): data
+ * normalisation (Sec. III-D "Normalization"), x_hat = (x - mu) / (sigma +
+ * 1e-7), then ESB projection of x_hat with the DDA scale alpha*(b,k) of
+ * N(0,1) data (Eq. optimal_alpha_seeking; the normalised data need no
+ * other scale).  In fp32, each operation rounded to nearest:
+ * x_hat = fl32(fl32(x - fl32(mu)) / fl32(sigma + 1e-7)), code = projection
+ * of x_hat as esb_project with alpha = fl32(alpha*), xq = fl32(alpha * q),
+ * q the code's value (the fake-quantised value the forward multiplies).
+ *   x      [device] rows x cols floats (row stride cols)
+ *   stats  [device] doubles {mu, sigma}: the batch's (stats_out of
+ *          esb_calibrate_dda with a signed format) in training, the moving
+ *          averages of esb_ema_update at test time
+ *   codes  [device] rows x ldc words; xq [device] rows x cols floats or NULL
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+esb_status esb_dn_project(const float* x, int64_t rows, int64_t cols, const double* stats, esb_format f,
+                          int32_t rounding, uint32_t* codes, int64_t ldc, float* xq, void* stream);
+
+/* Backward of esb_dn_project (Algorithm 1, backward loop): the gradient
+ * with respect to the fake-quantised values passes the projection unchanged
+ * (straight-through: Algorithm 1 multiplies no derivative of ESB), then
+ * through DN with the batch's mean and sigma, which depend on every
+ * element: with c = x - mu, s = sigma + 1e-7 and d = n,
+ *   grad_x[j] = (grad[j] - mean(grad)) / s - c[j] sum_i(grad[i] c[i]) / (d sigma s^2)
+ * (the second term is 0 when sigma = 0).  Sums in fp64 in a fixed order;
+ * grad_x rounded to fp32.
+ *   grad, x [device] n floats; stats [device] {mu, sigma} of the forward
+ *   workspace [device] >= esb_dn_backward_workspace_bytes(n), 16-byte aligned
+ *   grad_x [device] n floats
+ * Errors: INVALID_ARG, ALIGN, CUDA. */
+size_t esb_dn_backward_workspace_bytes(int64_t n);
+esb_status esb_dn_backward(const float* grad, const float* x, int64_t n, const double* stats, void* workspace,
+                           size_t workspace_bytes, float* grad_x, void* stream);
+
+/* Exponential moving average of activation statistics (Sec. III-D,
+ * "Normalization", training phase):
+ *   mu <- (1 - gamma) mu + gamma mu_i,  sigma <- (1 - gamma) sigma + gamma sigma_i,
+ * in fp64, each product and sum rounded separately.
+ *   batch_stats [device] {mu_i, sigma_i, ...}; running_stats [device] {mu, sigma}
+ *   gamma in [0, 1] (the paper's momentum coefficient)
+ * Errors: INVALID_ARG, CUDA. */
+esb_status esb_ema_update(const double* batch_stats, double* running_stats, double gamma, void* stream);
 
 /* ---------------------------------------------------------------- gemm */
 

@@ -82,6 +82,14 @@ def _load():
         "oracle_alpha_star": (f64, [i32, i32, p]),
         "oracle_dD": (f64, [f64, i32, i32]),
         "oracle_calibrate_with": (f32, [p, i64, f64, i32, p]),
+        "oracle_D_laplace": (f64, [f64, i32, i32]),
+        "oracle_dn_project": (None, [p, i64, f64, f64, f32, i32, i32, i32, i32, p, p]),
+        "oracle_dn_backward": (None, [p, p, i64, f64, f64, p]),
+        "oracle_ema": (None, [p, p, f64]),
+        "oracle_alpha_star_laplace": (f64, [i32, i32, p]),
+        "oracle_histogram_abs": (None, [p, i64, i32, f64, f64, i32, f32, p]),
+        "oracle_D_hist": (f64, [f64, p, i32, f64, i32, i32]),
+        "oracle_alpha_star_hist": (f64, [p, i32, f64, i32, i32, p]),
         "oracle_gemm_i64": (None, [p, i64, i32, i32, p, i64, i32, i32, i64, i64, i64, p]),
         "oracle_gemm_entry": (i64, [p, i64, i32, i32, p, i64, i32, i32, i64, i64, i64]),
         "oracle_epilogue_one": (f32, [i64, f32, f32, i32, i64, f32, i32, f32, i32, i32, i32, i32, p]),
@@ -254,6 +262,66 @@ def calibrate(x: np.ndarray, b: int, k: int, signed: bool = True) -> tuple[float
     st = np.zeros(3, dtype=np.float64)
     a = _load().oracle_calibrate_with(_ptr(x), x.size, alpha_star_cached(b, k), int(signed), _ptr(st))
     return float(np.float32(a)), st
+
+
+def D_laplace(alpha: float, b: int, k: int) -> float:
+    """D(alpha) of Eq. objective_function_expansion for Laplace data with unit variance."""
+    return _load().oracle_D_laplace(alpha, b, k)
+
+
+def alpha_star_laplace(b: int, k: int) -> tuple[float, float]:
+    """(alpha*, 2 D(alpha*)) for Laplace data with unit variance."""
+    d = ctypes.c_double(0.0)
+    a = _load().oracle_alpha_star_laplace(b, k, ctypes.byref(d))
+    return a, 2.0 * d.value
+
+
+def histogram_abs(x: np.ndarray, signed: bool, mean: float, spread: float, nbins: int, t_max: float) -> np.ndarray:
+    """Counts (uint64, nbins) of the normalised magnitudes of x."""
+    x = np.ascontiguousarray(x, dtype=np.float32).ravel()
+    out = np.zeros(nbins, dtype=np.uint64)
+    _load().oracle_histogram_abs(_ptr(x), x.size, int(signed), float(mean), float(spread), nbins, float(t_max),
+                                 _ptr(out))
+    return out
+
+
+def D_hist(alpha: float, counts: np.ndarray, t_max: float, b: int, k: int) -> float:
+    c = np.ascontiguousarray(counts, dtype=np.uint64)
+    return _load().oracle_D_hist(alpha, _ptr(c), c.size, float(t_max), b, k)
+
+
+def alpha_star_hist(counts: np.ndarray, t_max: float, b: int, k: int) -> tuple[float, float]:
+    """(alpha*, 2 D(alpha*)) of the empirical density of a histogram of |t|."""
+    c = np.ascontiguousarray(counts, dtype=np.uint64)
+    d = ctypes.c_double(0.0)
+    a = _load().oracle_alpha_star_hist(_ptr(c), c.size, float(t_max), b, k, ctypes.byref(d))
+    return a, 2.0 * d.value
+
+
+def dn_project(x: np.ndarray, mu: float, sigma: float, alpha: float, b: int, k: int, signed: bool = True,
+               rounding: int = 0) -> tuple[np.ndarray, np.ndarray]:
+    """(unpacked codes, fake-quantised values) of DN then projection (Algorithm 1 forward)."""
+    x = np.ascontiguousarray(x, dtype=np.float32).ravel()
+    codes = np.zeros(x.size, dtype=np.uint32)
+    xq = np.zeros(x.size, dtype=np.float32)
+    _load().oracle_dn_project(_ptr(x), x.size, float(mu), float(sigma), float(alpha), b, k, int(signed), rounding,
+                              _ptr(codes), _ptr(xq))
+    return codes, xq
+
+
+def dn_backward(g: np.ndarray, x: np.ndarray, mu: float, sigma: float) -> np.ndarray:
+    g = np.ascontiguousarray(g, dtype=np.float32).ravel()
+    x = np.ascontiguousarray(x, dtype=np.float32).ravel()
+    out = np.zeros(x.size, dtype=np.float32)
+    _load().oracle_dn_backward(_ptr(g), _ptr(x), x.size, float(mu), float(sigma), _ptr(out))
+    return out
+
+
+def ema(batch, running, gamma: float) -> np.ndarray:
+    b = np.ascontiguousarray(np.asarray(batch, dtype=np.float64)[:2])
+    r = np.ascontiguousarray(np.asarray(running, dtype=np.float64)[:2]).copy()
+    _load().oracle_ema(_ptr(b), _ptr(r), float(gamma))
+    return r
 
 
 # --------------------------------------------------------- contraction ---

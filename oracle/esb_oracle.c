@@ -587,3 +587,230 @@ void oracle_avgpool_sum_i64(const uint32_t *X, int64_t ldx, int b, int k,
             sums[(int64_t)n * C + c] = s;
         }
 }
+
+/* ---------------------------------------------------------------------- */
+/* DDA for data densities other than N(0,1) (the paper assumes N(0,1) in    */
+/* Sec. III-D "Resolving extremum").  D(alpha) is Eq.                      */
+/* objective_function_expansion with another p(t), written out as the      */
+/* integral of (t - alpha q)^2 p(t) over the cell of each element q of the */
+/* non-negative set; alpha* is its first local minimum from small alpha.   */
+
+/* Composite Simpson rule of (t - q)^2 * p(t) over [lo, hi] with m (even)
+ * subintervals; p(t) = (lam / 2) exp(-lam t), the Laplace density with
+ * unit variance (lam = sqrt 2). */
+static double laplace_cell(double lo, double hi, double q, int m)
+{
+    const double lam = sqrt(2.0);
+    double h = (hi - lo) / m, s = 0.0;
+    for (int i = 0; i <= m; i++) {
+        double t = lo + i * h;
+        double f = (t - q) * (t - q) * 0.5 * lam * exp(-lam * t);
+        s += (i == 0 || i == m) ? f : ((i & 1) ? 4.0 * f : 2.0 * f);
+    }
+    return s * h / 3.0;
+}
+
+/* D(alpha) for Laplace data: the last cell runs to lo + 60 / lam (the tail
+ * beyond holds e^-60 of the mass); m subintervals per cell. */
+static double laplace_D_m(double alpha, int b, int k, int m)
+{
+    double s[ORACLE_MAX_SET];
+    int n = oracle_set_nonneg(b, k, s);
+    double D = 0.0;
+    for (int j = 0; j < n; j++) {
+        double lo = (j == 0) ? 0.0 : alpha * 0.5 * (s[j - 1] + s[j]);
+        double hi = (j == n - 1) ? lo + 60.0 / sqrt(2.0) : alpha * 0.5 * (s[j] + s[j + 1]);
+        D += laplace_cell(lo, hi, alpha * s[j], m);
+    }
+    return D;
+}
+
+double oracle_D_laplace(double alpha, int b, int k) { return laplace_D_m(alpha, b, k, 4000); }
+
+/* First local minimum of f on a geometric grid of G points over [1e-4, 4]
+ * (coarse evaluation fc), refined by golden-section search on f between
+ * the grid neighbours of that point. */
+static double first_minimum_golden(double (*fc)(double, const void *), double (*f)(double, const void *),
+                                   const void *ctx, double *f_out)
+{
+    const int G = 4000;
+    const double lo = 1e-4, hi = 4.0;
+    double prev2 = fc(lo, ctx), a1 = lo * pow(hi / lo, 1.0 / (G - 1)), prev = fc(a1, ctx);
+    double x0 = lo, x1 = hi;
+    for (int i = 2; i < G; i++) {
+        double ai = lo * pow(hi / lo, (double)i / (double)(G - 1));
+        double cur = fc(ai, ctx);
+        if (prev < prev2 && prev <= cur) {
+            x0 = lo * pow(hi / lo, (double)(i - 2) / (double)(G - 1));
+            x1 = ai;
+            break;
+        }
+        prev2 = prev;
+        prev = cur;
+    }
+    const double g = 0.5 * (sqrt(5.0) - 1.0);
+    double c = x1 - g * (x1 - x0), d = x0 + g * (x1 - x0);
+    double fc_ = f(c, ctx), fd = f(d, ctx);
+    for (int it = 0; it < 300 && x1 - x0 > 1e-14 * x1; it++) {
+        if (fc_ < fd) { x1 = d; d = c; fd = fc_; c = x1 - g * (x1 - x0); fc_ = f(c, ctx); }
+        else { x0 = c; c = d; fc_ = fd; d = x0 + g * (x1 - x0); fd = f(d, ctx); }
+    }
+    double as = 0.5 * (x0 + x1);
+    if (f_out) *f_out = f(as, ctx);
+    return as;
+}
+
+typedef struct { int b, k; } bk_ctx;
+
+static double laplace_coarse(double a, const void *c)
+{
+    const bk_ctx *p = (const bk_ctx *)c;
+    return laplace_D_m(a, p->b, p->k, 200);
+}
+
+static double laplace_fine(double a, const void *c)
+{
+    const bk_ctx *p = (const bk_ctx *)c;
+    return oracle_D_laplace(a, p->b, p->k);
+}
+
+/* alpha* for Laplace data with unit variance; D(alpha*) via D_out. */
+double oracle_alpha_star_laplace(int b, int k, double *D_out)
+{
+    bk_ctx c = {b, k};
+    return first_minimum_golden(laplace_coarse, laplace_fine, &c, D_out);
+}
+
+/* Histogram of the normalised magnitudes of x (the empirical density of
+ * the data): t = (x - mean) / spread for signed formats, x / spread for
+ * unsigned ones; bin = floor(u) with u = |x - mean| * (nbins / (t_max *
+ * spread)), each step an fp32 operation rounded to nearest; u >= nbins goes
+ * to the last bin; NaN values are skipped. */
+void oracle_histogram_abs(const float *x, int64_t n, int is_signed, double mean, double spread, int nbins,
+                          float t_max, uint64_t *counts)
+{
+    volatile float m = is_signed ? (float)mean : 0.0f;
+    volatile float sp = (float)spread;
+    volatile float nb = (float)nbins;
+    volatile float den = t_max * sp;
+    volatile float scale = nb / den;
+    for (int i = 0; i < nbins; i++) counts[i] = 0;
+    for (int64_t i = 0; i < n; i++) {
+        if (isnan(x[i])) continue;
+        volatile float d = x[i] - m;
+        volatile float u = fabsf(d) * scale;
+        int bin;
+        if (u < nb) bin = (int)floorf(u);
+        else if (u >= nb) bin = nbins - 1;
+        else bin = 0;
+        counts[bin]++;
+    }
+}
+
+typedef struct { const uint64_t *counts; int nbins; double t_max; int b, k; } hist_ctx;
+
+/* D(alpha) for the empirical density: bin i of width w = t_max / nbins
+ * holds counts[i] / (2 n) of the mass, spread evenly over it (the
+ * non-negative half holds 1/2, as for the symmetric densities).  Each bin
+ * is cut at the cell boundaries alpha (s_j + s_{j+1}) / 2 inside it; on each
+ * piece the integrand (t - alpha q)^2 is a quadratic, which Simpson's rule
+ * with one interval integrates exactly.  q of a piece: the projection of
+ * its midpoint (Eq. thresholing_func). */
+double oracle_D_hist(double alpha, const uint64_t *counts, int nbins, double t_max, int b, int k)
+{
+    double s[ORACLE_MAX_SET];
+    int ns = oracle_set_nonneg(b, k, s);
+    double total = 0.0;
+    for (int i = 0; i < nbins; i++) total += (double)counts[i];
+    double w = t_max / nbins, D = 0.0;
+    int j = 0;                                  /* next boundary index (boundary between s[j], s[j+1]) */
+    for (int i = 0; i < nbins; i++) {
+        double e0 = i * w, e1 = (i + 1) * w;
+        double p = (double)counts[i] / (2.0 * total * w);
+        while (j < ns - 1 && alpha * 0.5 * (s[j] + s[j + 1]) <= e0) j++;
+        double u = e0;
+        for (;;) {
+            int jj = j;
+            double v = e1;
+            while (jj < ns - 1 && alpha * 0.5 * (s[jj] + s[jj + 1]) < e1) {
+                double bd = alpha * 0.5 * (s[jj] + s[jj + 1]);
+                if (bd > u) { v = bd; break; }
+                jj++;
+            }
+            if (p > 0.0) {
+                double tm = 0.5 * (u + v);
+                double q = alpha * lookup_projection(tm / alpha, s, ns, 0);
+                double fu = (u - q) * (u - q), fm = (tm - q) * (tm - q), fv = (v - q) * (v - q);
+                D += p * (v - u) / 6.0 * (fu + 4.0 * fm + fv);
+            }
+            if (v >= e1) break;
+            u = v;
+        }
+    }
+    return D;
+}
+
+static double hist_f(double a, const void *c)
+{
+    const hist_ctx *h = (const hist_ctx *)c;
+    return oracle_D_hist(a, h->counts, h->nbins, h->t_max, h->b, h->k);
+}
+
+/* alpha* of the empirical density (first local minimum of oracle_D_hist). */
+double oracle_alpha_star_hist(const uint64_t *counts, int nbins, double t_max, int b, int k, double *D_out)
+{
+    hist_ctx c = {counts, nbins, t_max, b, k};
+    return first_minimum_golden(hist_f, hist_f, &c, D_out);
+}
+
+/* ---------------------------------------------------------------------- */
+/* Quantisation-aware training (Algorithm 1; Sec. III-D "Normalization").  */
+
+/* Forward of one tensor: DN, x_hat = fl32(fl32(x - fl32(mu)) / fl32(sigma +
+ * 1e-7)), then the projection of x_hat with scale alpha (alpha* of the
+ * format, in fp32): codes (unpacked) and the fake-quantised values
+ * fl32(alpha * q). */
+void oracle_dn_project(const float *x, int64_t n, double mu, double sigma, float alpha, int b, int k, int is_signed,
+                       int rounding, uint32_t *codes, float *xq)
+{
+    volatile float m = (float)mu;
+    volatile float s = (float)(sigma + 1e-7);
+    for (int64_t i = 0; i < n; i++) {
+        volatile float c = x[i] - m;
+        volatile float xh = c / s;
+        double q = oracle_project_value(xh, alpha, b, k, is_signed, rounding);
+        codes[i] = oracle_encode(q, b, k, is_signed);
+        if (xq) xq[i] = alpha * (float)q;
+    }
+}
+
+/* Backward: the straight-through estimator passes the gradient of the
+ * fake-quantised values to x_hat unchanged; DN's derivative, with c = x -
+ * mu, s = sigma + 1e-7 and both mu and sigma functions of all of x:
+ *   d x_hat_i / d x_j = (delta_ij - 1/d) / s - c_i c_j / (d sigma s^2),
+ * so grad_x_j = sum_i g_i d x_hat_i / d x_j (fp64, rounded to fp32 at the
+ * end; the second term is 0 when sigma = 0). */
+void oracle_dn_backward(const float *g, const float *x, int64_t n, double mu, double sigma, float *gx)
+{
+    double s = sigma + 1e-7, sg = 0.0, sgc = 0.0, d = (double)n;
+    for (int64_t i = 0; i < n; i++) {
+        sg += (double)g[i];
+        sgc += (double)g[i] * ((double)x[i] - mu);
+    }
+    for (int64_t j = 0; j < n; j++) {
+        double cj = (double)x[j] - mu;
+        double t = ((double)g[j] - sg / d) / s;
+        if (sigma > 0.0) t -= cj * sgc / (d * sigma * s * s);
+        gx[j] = (float)t;
+    }
+}
+
+/* Exponential moving average of (mu, sigma): r <- (1 - gamma) r + gamma b. */
+void oracle_ema(const double *batch, double *running, double gamma)
+{
+    for (int i = 0; i < 2; i++) {
+        volatile double a = (1.0 - gamma) * running[i];
+        volatile double c = gamma * batch[i];
+        running[i] = a + c;
+    }
+}

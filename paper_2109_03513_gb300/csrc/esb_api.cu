@@ -5,6 +5,7 @@
 #include <cstdint>
 #include <cstring>
 #include <mutex>
+#include <vector>
 
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -127,6 +128,22 @@ double g_astar[9][9];
 double g_dda[9][9];
 bool g_astar_have[9][9];
 
+double g_astar_lap[9][9];
+double g_dda_lap[9][9];
+bool g_astar_lap_have[9][9];
+
+esb_status alpha_star_laplace_cached(int b, int k, double* a, double* d)
+{
+    std::lock_guard<std::mutex> lk(g_astar_mu);
+    if (!g_astar_lap_have[b][k]) {
+        g_astar_lap[b][k] = alpha_star_solve_laplace(b, k, &g_dda_lap[b][k]);
+        g_astar_lap_have[b][k] = true;
+    }
+    if (a) *a = g_astar_lap[b][k];
+    if (d) *d = g_dda_lap[b][k];
+    return ESB_OK;
+}
+
 esb_status alpha_star_cached(int b, int k, double* a, double* d)
 {
     std::lock_guard<std::mutex> lk(g_astar_mu);
@@ -223,6 +240,127 @@ esb_status esb_calibrate_dda_noalloc(const float* x, int64_t n, esb_format f, fl
     alpha_star_cached(f.b, f.k, &as, nullptr);
     cudaError_t e = launch_calibrate_noalloc(x, n, f.is_signed, as, alpha_out, stats_out,
                                              static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_alpha_star_dist(int32_t b, int32_t k, int32_t dist, double* alpha_star, double* dda)
+{
+    if (b < 2 || b > 8 || k < 0 || k > b - 1) return ESB_ERR_UNSUPPORTED;
+    if (!alpha_star) return ESB_ERR_INVALID_ARG;
+    if (dist == ESB_DIST_GAUSSIAN) return alpha_star_cached(b, k, alpha_star, dda);
+    if (dist == ESB_DIST_LAPLACE) return alpha_star_laplace_cached(b, k, alpha_star, dda);
+    return ESB_ERR_INVALID_ARG;
+}
+
+esb_status esb_calibrate_dda_dist(const float* x, int64_t n, esb_format f, int32_t dist, void* workspace,
+                                  size_t workspace_bytes, float* alpha_out, double* stats_out, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (dist != ESB_DIST_GAUSSIAN && dist != ESB_DIST_LAPLACE) return ESB_ERR_INVALID_ARG;
+    if (!x || n <= 0 || !workspace || !alpha_out) return ESB_ERR_INVALID_ARG;
+    if (workspace_bytes < calibrate_workspace_bytes(n)) return ESB_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 15u) != 0) return ESB_ERR_ALIGN;
+    double as = 0.0;
+    esb_alpha_star_dist(f.b, f.k, dist, &as, nullptr);
+    const cudaError_t e = launch_calibrate(x, n, f.is_signed, as, workspace, alpha_out, stats_out,
+                                           static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_dda_histogram(const float* x, int64_t n, esb_format f, const double* stats, int32_t nbins, float t_max,
+                             unsigned long long* counts, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (n < 0 || nbins < 2 || nbins > ESB_DDA_MAX_BINS || !(std::isfinite(t_max) && t_max > 0.0f))
+        return ESB_ERR_INVALID_ARG;
+    if (!stats || !counts || (n > 0 && !x)) return ESB_ERR_INVALID_ARG;
+    const cudaError_t e = launch_dda_histogram(x, n, f.is_signed, stats, nbins, t_max, counts,
+                                               static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_alpha_star_hist(const unsigned long long* counts, int32_t nbins, float t_max, int32_t b, int32_t k,
+                               double* alpha_star, double* dda)
+{
+    if (b < 2 || b > 8 || k < 0 || k > b - 1) return ESB_ERR_UNSUPPORTED;
+    if (!counts || !alpha_star || nbins < 2 || nbins > ESB_DDA_MAX_BINS || !(std::isfinite(t_max) && t_max > 0.0f))
+        return ESB_ERR_INVALID_ARG;
+    unsigned long long total = 0;
+    for (int i = 0; i < nbins; i++) total += counts[i];
+    if (total == 0) return ESB_ERR_INVALID_ARG;
+    *alpha_star = alpha_star_solve_hist(counts, nbins, (double)t_max, b, k, dda);
+    return ESB_OK;
+}
+
+esb_status esb_calibrate_dda_empirical(const float* x, int64_t n, esb_format f, void* workspace,
+                                       size_t workspace_bytes, int32_t nbins, float t_max,
+                                       unsigned long long* counts, float* alpha_out, double* stats_out,
+                                       double* alpha_star_out, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (!x || n <= 0 || !workspace || !alpha_out || !stats_out || !counts) return ESB_ERR_INVALID_ARG;
+    if (nbins < 2 || nbins > ESB_DDA_MAX_BINS || !(std::isfinite(t_max) && t_max > 0.0f)) return ESB_ERR_INVALID_ARG;
+    if (workspace_bytes < calibrate_workspace_bytes(n)) return ESB_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 15u) != 0) return ESB_ERR_ALIGN;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    double as = 0.0;
+    alpha_star_cached(f.b, f.k, &as, nullptr);
+    // 1. statistics (and the Gaussian alpha, overwritten below)
+    cudaError_t e = launch_calibrate(x, n, f.is_signed, as, workspace, alpha_out, stats_out, st);
+    if (e != cudaSuccess) return ESB_ERR_CUDA;
+    // 2. histogram of the normalised magnitudes
+    e = launch_dda_histogram(x, n, f.is_signed, stats_out, nbins, t_max, counts, st);
+    if (e != cudaSuccess) return ESB_ERR_CUDA;
+    // 3. alpha* of the histogram on the host
+    std::vector<unsigned long long> h((size_t)nbins);
+    double stats[3] = {0.0, 0.0, 0.0};
+    if (cudaMemcpyAsync(h.data(), counts, sizeof(unsigned long long) * (size_t)nbins, cudaMemcpyDeviceToHost, st) !=
+            cudaSuccess ||
+        cudaMemcpyAsync(stats, stats_out, sizeof(stats), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return ESB_ERR_CUDA;
+    const double ash = alpha_star_solve_hist(h.data(), nbins, (double)t_max, f.b, f.k, nullptr);
+    if (alpha_star_out) *alpha_star_out = ash;
+    const float alpha = static_cast<float>(ash * (stats[1] + 1e-7));
+    if (cudaMemcpyAsync(alpha_out, &alpha, sizeof(float), cudaMemcpyHostToDevice, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return ESB_ERR_CUDA;
+    return ESB_OK;
+}
+
+esb_status esb_dn_project(const float* x, int64_t rows, int64_t cols, const double* stats, esb_format f,
+                          int32_t rounding, uint32_t* codes, int64_t ldc, float* xq, void* stream)
+{
+    if (!fmt_ok(f)) return ESB_ERR_UNSUPPORTED;
+    if (rows < 0 || cols < 0 || ldc < words_for(cols, f.b)) return ESB_ERR_INVALID_ARG;
+    if (rounding != ESB_ROUND_HALF_AWAY && rounding != ESB_ROUND_HALF_EVEN) return ESB_ERR_INVALID_ARG;
+    if (rows == 0 || ldc == 0) return ESB_OK;
+    if (!stats || !codes || (cols > 0 && !x)) return ESB_ERR_INVALID_ARG;
+    double as = 0.0;
+    alpha_star_cached(f.b, f.k, &as, nullptr);
+    const cudaError_t e = launch_dn_project(x, rows, cols, stats, f.b, f.k, f.is_signed, rounding, (float)as, codes,
+                                            ldc, xq, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+size_t esb_dn_backward_workspace_bytes(int64_t n) { return n > 0 ? dn_grad_workspace_bytes(n) : 0; }
+
+esb_status esb_dn_backward(const float* grad, const float* x, int64_t n, const double* stats, void* workspace,
+                           size_t workspace_bytes, float* grad_x, void* stream)
+{
+    if (n < 0) return ESB_ERR_INVALID_ARG;
+    if (n == 0) return ESB_OK;
+    if (!grad || !x || !stats || !workspace || !grad_x) return ESB_ERR_INVALID_ARG;
+    if (workspace_bytes < dn_grad_workspace_bytes(n)) return ESB_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 15u) != 0) return ESB_ERR_ALIGN;
+    const cudaError_t e = launch_dn_grad(grad, x, n, stats, workspace, grad_x, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_ema_update(const double* batch_stats, double* running_stats, double gamma, void* stream)
+{
+    if (!batch_stats || !running_stats || !(gamma >= 0.0 && gamma <= 1.0)) return ESB_ERR_INVALID_ARG;
+    const cudaError_t e = launch_ema(batch_stats, running_stats, gamma, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 

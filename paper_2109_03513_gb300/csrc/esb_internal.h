@@ -84,7 +84,31 @@ cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
                            float alpha_out, int bo, int ko, int so, int rounding, float* y_out, uint32_t* codes_out,
                            int64_t ldo, cudaStream_t st);
 
+// CUDA-core contraction with int64 accumulators (esb_shiftadd.cu).
+bool shiftadd_grid_ok(int64_t M, int64_t N, int out_b);
+cudaError_t launch_gemm_i64(int64_t M, int64_t N, int64_t K, const uint32_t* A, int64_t lda, int ba, int ka,
+                            const uint32_t* B, int64_t ldb, int bb, int kb, int64_t* acc64, const GemmOutputs& o,
+                            cudaStream_t st);
+cudaError_t launch_conv_i64(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
+                            const uint32_t* W, int64_t ldw, int bw, int kw, int64_t* acc64, const GemmOutputs& o,
+                            cudaStream_t st);
+
+// Quantisation-aware training kernels (esb_qat.cu).
+size_t dn_grad_workspace_bytes(int64_t n);
+cudaError_t launch_dn_project(const float* x, int64_t rows, int64_t cols, const double* stats, int b, int k,
+                              int is_signed, int rounding, float alpha, uint32_t* codes, int64_t ldc, float* xq,
+                              cudaStream_t st);
+cudaError_t launch_dn_grad(const float* g, const float* x, int64_t n, const double* stats, void* workspace, float* gx,
+                           cudaStream_t st);
+cudaError_t launch_ema(const double* batch, double* running, double gamma, cudaStream_t st);
+
 // alpha*(b,k) and 2*D(alpha*) (Sec. III-D), solved on the host in fp64.
 double alpha_star_solve(int b, int k, double* dda);
+// The same for Laplace data with unit variance, and for the empirical
+// density of a histogram of |t| (nbins bins over [0, t_max), t in spreads).
+double alpha_star_solve_laplace(int b, int k, double* dda);
+double alpha_star_solve_hist(const unsigned long long* counts, int nbins, double t_max, int b, int k, double* dda);
+cudaError_t launch_dda_histogram(const float* x, int64_t n, int is_signed, const double* stats, int nbins,
+                                 float t_max, unsigned long long* counts, cudaStream_t st);
 
 }  // namespace esb

@@ -765,6 +765,54 @@ calibrate_pass1_kernel(const float* __restrict__ x, int64_t n, int vec, CalParti
     }
 }
 
+// ------------------------------------------ empirical DDA histogram
+
+// Histogram of |t| for the DDA of the data's own density: t = (x - mean) /
+// sigma (signed formats) or x / rms (unsigned), bins of width t_max / nbins
+// over [0, t_max), values past t_max in the last bin, NaN skipped.  The bin
+// of a value is fixed by these fp32 operations, each rounded to nearest:
+// scale = nbins / (t_max * spread), u = |x - mean| * scale, bin = floor(u).
+// Each block counts into shared memory and adds its counts to the device
+// array (integer additions: the result does not depend on their order).
+__global__ void __launch_bounds__(256)
+dda_histogram_kernel(const float* __restrict__ x, int64_t n, int is_signed, const double* __restrict__ stats,
+                     int nbins, float t_max, unsigned long long* __restrict__ counts)
+{
+    extern __shared__ unsigned int hist[];
+    for (int i = threadIdx.x; i < nbins; i += blockDim.x) hist[i] = 0u;
+    griddep_wait();                                   // stats may come from the previous launch
+    __syncthreads();
+    const float m = is_signed ? (float)__ldg(stats) : 0.0f;
+    const float sp = (float)__ldg(stats + 1);
+    const float nb = (float)nbins;
+    const float scale = __fdiv_rn(nb, __fmul_rn(t_max, sp));
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        const float v = __ldcs(x + i);
+        if (v != v) continue;
+        const float u = __fmul_rn(fabsf(__fsub_rn(v, m)), scale);
+        const int bin = (u < nb) ? (int)u : ((u >= nb) ? nbins - 1 : 0);   // NaN (0 * inf): bin 0
+        atomicAdd(&hist[bin], 1u);
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < nbins; i += blockDim.x)
+        if (hist[i]) atomicAdd(counts + i, (unsigned long long)hist[i]);
+}
+
+cudaError_t launch_dda_histogram(const float* x, int64_t n, int is_signed, const double* stats, int nbins,
+                                 float t_max, unsigned long long* counts, cudaStream_t st)
+{
+    cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(unsigned long long) * (size_t)nbins, st);
+    if (e != cudaSuccess) return e;
+    int64_t blocks = (n + 255) / 256;
+    const int64_t cap = (int64_t)device_sm_count() * 4;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    dda_histogram_kernel<<<(unsigned)blocks, 256, sizeof(unsigned int) * (size_t)nbins, st>>>(
+        x, n, is_signed, stats, nbins, t_max, counts);
+    return cudaGetLastError();
+}
+
 // ------------------------------------- DDA-calibrated projection, fused
 
 // Calibration and projection of the same tensor in one launch of one

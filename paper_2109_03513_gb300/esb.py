@@ -87,6 +87,15 @@ SIGNATURES = {
     "esb_calibrate_dda": (_I32, [_P, _I64, esb_format, _P, _SZ, _P, _P, _P]),
     "esb_calibrate_dda_noalloc": (_I32, [_P, _I64, esb_format, _P, _P, _P]),
     "esb_dda_combine": (_I32, [_P, _I64, esb_format, _P, _P]),
+    "esb_dn_project": (_I32, [_P, _I64, _I64, _P, esb_format, _I32, _P, _I64, _P, _P]),
+    "esb_dn_backward_workspace_bytes": (_SZ, [_I64]),
+    "esb_dn_backward": (_I32, [_P, _P, _I64, _P, _P, _SZ, _P, _P]),
+    "esb_ema_update": (_I32, [_P, _P, ctypes.c_double, _P]),
+    "esb_alpha_star_dist": (_I32, [_I32, _I32, _I32, _P, _P]),
+    "esb_calibrate_dda_dist": (_I32, [_P, _I64, esb_format, _I32, _P, _SZ, _P, _P, _P]),
+    "esb_dda_histogram": (_I32, [_P, _I64, esb_format, _P, _I32, _F32, _P, _P]),
+    "esb_alpha_star_hist": (_I32, [_P, _I32, _F32, _I32, _I32, _P, _P]),
+    "esb_calibrate_dda_empirical": (_I32, [_P, _I64, esb_format, _P, _SZ, _I32, _F32, _P, _P, _P, _P, _P]),
     "esb_dequant_scale": (_I32, [_F32, esb_format, _F32, esb_format, _P]),
     "esb_fold_bn_dn": (_I32, [_F32, esb_format, _F32, esb_format, _P, _P, _P, _P, _I64, ctypes.c_double,
                               ctypes.c_double, _P, _P]),
@@ -206,6 +215,80 @@ def esb_calibrate_dda_noalloc(x: torch.Tensor, f: Fmt, alpha_out: Optional[torch
     return alpha_out, stats_out
 
 
+ESB_DIST_GAUSSIAN = 0
+ESB_DIST_LAPLACE = 1
+
+
+def esb_alpha_star_dist(b: int, k: int, dist: int) -> tuple[float, float]:
+    a = ctypes.c_double(0.0)
+    d = ctypes.c_double(0.0)
+    _check(lib().esb_alpha_star_dist(b, k, dist, ctypes.byref(a), ctypes.byref(d)), "esb_alpha_star_dist")
+    return a.value, d.value
+
+
+def esb_calibrate_dda_dist(x: torch.Tensor, f: Fmt, dist: int, alpha_out: Optional[torch.Tensor] = None,
+                           stats_out: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
+                           stream=None) -> tuple[torch.Tensor, Optional[torch.Tensor]]:
+    """esb_calibrate_dda with the alpha* of another data density (ESB_DIST_*)."""
+    _dev(x, "x")
+    assert x.dtype == torch.float32
+    n = x.numel()
+    if alpha_out is None:
+        alpha_out = torch.empty(1, dtype=torch.float32, device=x.device)
+    if workspace is None:
+        workspace = torch.zeros(max(int(lib().esb_calibrate_dda_workspace_bytes(n)), 16), dtype=torch.uint8,
+                                device=x.device)
+    _check(lib().esb_calibrate_dda_dist(_ptr(x), n, f.c(), dist, _ptr(workspace), workspace.numel(),
+                                        _ptr(alpha_out), _ptr(stats_out), _stream(stream)), "esb_calibrate_dda_dist")
+    return alpha_out, stats_out
+
+
+def esb_dda_histogram(x: torch.Tensor, f: Fmt, stats: torch.Tensor, nbins: int = 8192, t_max: float = 16.0,
+                      counts: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Histogram (int64 CUDA tensor of nbins counts) of the normalised |t| of x."""
+    _dev(x, "x"); _dev(stats, "stats")
+    if counts is None:
+        counts = torch.empty(nbins, dtype=torch.int64, device=x.device)
+    _check(lib().esb_dda_histogram(_ptr(x), x.numel(), f.c(), _ptr(stats), nbins, t_max, _ptr(counts),
+                                   _stream(stream)), "esb_dda_histogram")
+    return counts
+
+
+def esb_alpha_star_hist(counts, t_max: float, b: int, k: int) -> tuple[float, float]:
+    """alpha* and 2 D(alpha*) of a histogram of |t| (host counts, any int array)."""
+    import numpy as np
+    c = np.ascontiguousarray(np.asarray(counts, dtype=np.uint64))
+    a = ctypes.c_double(0.0)
+    d = ctypes.c_double(0.0)
+    _check(lib().esb_alpha_star_hist(c.ctypes.data, c.size, t_max, b, k, ctypes.byref(a), ctypes.byref(d)),
+           "esb_alpha_star_hist")
+    return a.value, d.value
+
+
+def esb_calibrate_dda_empirical(x: torch.Tensor, f: Fmt, nbins: int = 8192, t_max: float = 16.0,
+                                alpha_out: Optional[torch.Tensor] = None, stats_out: Optional[torch.Tensor] = None,
+                                workspace: Optional[torch.Tensor] = None, counts: Optional[torch.Tensor] = None,
+                                stream=None) -> tuple[torch.Tensor, torch.Tensor, float]:
+    """DDA calibration with the data's own density -> (alpha (1,), stats (3,), alpha*).  Synchronises."""
+    _dev(x, "x")
+    n = x.numel()
+    dev = x.device
+    if alpha_out is None:
+        alpha_out = torch.empty(1, dtype=torch.float32, device=dev)
+    if stats_out is None:
+        stats_out = torch.empty(3, dtype=torch.float64, device=dev)
+    if workspace is None:
+        workspace = torch.zeros(max(int(lib().esb_calibrate_dda_workspace_bytes(n)), 16), dtype=torch.uint8,
+                                device=dev)
+    if counts is None:
+        counts = torch.empty(nbins, dtype=torch.int64, device=dev)
+    a = ctypes.c_double(0.0)
+    _check(lib().esb_calibrate_dda_empirical(_ptr(x), n, f.c(), _ptr(workspace), workspace.numel(), nbins, t_max,
+                                             _ptr(counts), _ptr(alpha_out), _ptr(stats_out), ctypes.byref(a),
+                                             _stream(stream)), "esb_calibrate_dda_empirical")
+    return alpha_out, stats_out, a.value
+
+
 def esb_calibrate_dda_workspace_bytes(n: int) -> int:
     return int(lib().esb_calibrate_dda_workspace_bytes(n))
 
@@ -252,6 +335,39 @@ def esb_project_dda(x: torch.Tensor, f: Fmt, rounding: int = ESB_ROUND_HALF_AWAY
                                  _ptr(alpha_out), _ptr(stats_out), _ptr(codes), ldc, _stream(stream)),
            "esb_project_dda")
     return codes, alpha_out
+
+
+def esb_dn_project(x: torch.Tensor, stats: torch.Tensor, f: Fmt, rounding: int = ESB_ROUND_HALF_AWAY,
+                   want_xq: bool = True, stream=None) -> tuple[torch.Tensor, Optional[torch.Tensor]]:
+    """DN then ESB projection with alpha* -> (codes (rows, ldc) int32, fake-quantised values | None)."""
+    _dev(x, "x"); _dev(stats, "stats")
+    x2 = x.reshape(1, -1) if x.dim() == 1 else x.reshape(-1, x.shape[-1])
+    rows, cols = x2.shape
+    ldc = esb_row_words(cols, f.b)
+    codes = torch.empty((rows, ldc), dtype=torch.int32, device=x.device)
+    xq = torch.empty_like(x2) if want_xq else None
+    _check(lib().esb_dn_project(_ptr(x2), rows, cols, _ptr(stats), f.c(), rounding, _ptr(codes), ldc, _ptr(xq),
+                                _stream(stream)), "esb_dn_project")
+    return codes, xq
+
+
+def esb_dn_backward(grad: torch.Tensor, x: torch.Tensor, stats: torch.Tensor,
+                    workspace: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Straight-through + DN backward -> dL/dx (fp32, shape of x)."""
+    _dev(grad, "grad"); _dev(x, "x"); _dev(stats, "stats")
+    n = x.numel()
+    if workspace is None:
+        workspace = torch.empty(max(int(lib().esb_dn_backward_workspace_bytes(n)), 16), dtype=torch.uint8,
+                                device=x.device)
+    gx = torch.empty_like(x)
+    _check(lib().esb_dn_backward(_ptr(grad), _ptr(x), n, _ptr(stats), _ptr(workspace), workspace.numel(), _ptr(gx),
+                                 _stream(stream)), "esb_dn_backward")
+    return gx
+
+
+def esb_ema_update(batch_stats: torch.Tensor, running_stats: torch.Tensor, gamma: float, stream=None) -> None:
+    _dev(batch_stats, "batch_stats"); _dev(running_stats, "running_stats")
+    _check(lib().esb_ema_update(_ptr(batch_stats), _ptr(running_stats), gamma, _stream(stream)), "esb_ema_update")
 
 
 def esb_dequant(codes: torch.Tensor, cols: int, f: Fmt, alpha, stream=None) -> torch.Tensor:

@@ -479,3 +479,144 @@ def test_code_rank_is_the_rotated_exponent_field(b, k):
     L = 1 << (b - 1)
     order = sorted(range(L), key=lambda c: o.decode(c, b, k))
     assert [(c + (1 << k)) % L for c in order] == list(range(L))
+
+
+# ------------------------------------------- DDA for other data densities ---
+
+def test_laplace_ternary_closed_form():
+    # ternary set {0, +-alpha}: alpha* satisfies the centroid condition
+    # alpha = E[t | t > alpha / 2]; the Laplace tail is memoryless, so
+    # E[t | t > c] = c + 1/lam and alpha* = 2 / lam = sqrt 2 (unit variance);
+    # the squared error is then 1 - alpha*^2 P(|t| > alpha*/2) = 1 - 2/e
+    a, dda = o.alpha_star_laplace(2, 0)
+    assert abs(a - math.sqrt(2.0)) <= 1e-7
+    assert abs(dda - (1.0 - 2.0 / math.e)) <= 1e-9
+
+
+@pytest.mark.parametrize("b,k", [(3, 1), (4, 2), (4, 1)])
+def test_laplace_D_against_monte_carlo(b, k):
+    rng = np.random.default_rng(b * 10 + k)
+    t = np.abs(rng.laplace(0.0, 1.0 / math.sqrt(2.0), 2_000_000))    # unit variance
+    s = o.set_nonneg(b, k)
+    for alpha in (0.3, 1.0, 2.0):
+        v = t / alpha
+        idx = np.clip(np.searchsorted(0.5 * (s[1:] + s[:-1]), v, side="right"), 0, len(s) - 1)
+        err = (t - alpha * s[idx]) ** 2
+        mc = 0.5 * err.mean()                     # D covers the half-line: half the mass
+        assert abs(o.D_laplace(alpha, b, k) - mc) <= 4 * 0.5 * err.std() / math.sqrt(t.size)
+
+
+@pytest.mark.parametrize("b", [3, 4])
+def test_laplace_alpha_star_scale_identity(b):
+    # the (b, b-1) set is the (b, b-2) set halved, for any density
+    a1, d1 = o.alpha_star_laplace(b, b - 1)
+    a2, d2 = o.alpha_star_laplace(b, b - 2)
+    assert abs(a1 - 2.0 * a2) <= 1e-7 * a1
+    assert abs(d1 - d2) <= 1e-12
+
+
+def test_laplace_D_limits():
+    # every value projects to (nearly) 0 as alpha -> 0 (the clip) and as
+    # alpha -> infinity: D -> E[t^2] / 2 = 1/2
+    assert abs(o.D_laplace(1e-9, 4, 2) - 0.5) < 1e-6
+    assert abs(o.D_laplace(1e3, 4, 2) - 0.5) < 1e-6       # one wide Simpson cell
+
+
+def test_histogram_bins_follow_their_fp32_definition():
+    rng = np.random.default_rng(3)
+    x = np.concatenate([rng.normal(2.0, 3.0, 100000).astype(np.float32), np.float32([np.nan, np.inf, -np.inf, 2.0])])
+    mean, spread, nb, tmax = 2.0000001, 2.9999, 1000, 8.0
+    got = o.histogram_abs(x, True, mean, spread, nb, tmax)
+    scale = np.float32(nb) / (np.float32(tmax) * np.float32(spread))
+    xv = x[~np.isnan(x)]
+    u = np.abs(xv - np.float32(mean)) * scale
+    bins = np.where(u < nb, np.floor(u), nb - 1).astype(np.int64)
+    assert np.array_equal(got, np.bincount(bins, minlength=nb).astype(np.uint64))
+
+
+def test_histogram_D_of_one_bin_is_the_plain_integral():
+    # all mass in one bin [e0, e1): D = (1/2) (1/w) int (t - alpha q(t))^2 dt
+    nb, tmax, b, k = 64, 4.0, 4, 2
+    counts = np.zeros(nb, np.uint64)
+    counts[13] = 1000
+    w = tmax / nb
+    t = 13 * w + (np.arange(2_000_000) + 0.5) * (w / 2_000_000)     # midpoint rule
+    s = o.set_nonneg(b, k)
+    for alpha in (0.1, 0.37, 1.3):
+        idx = np.clip(np.searchsorted(0.5 * (s[1:] + s[:-1]), t / alpha, side="right"), 0, len(s) - 1)
+        ref = 0.5 * np.mean((t - alpha * s[idx]) ** 2)
+        assert abs(o.D_hist(alpha, counts, tmax, b, k) - ref) <= 1e-9 * max(ref, 1e-12) + 1e-15
+
+
+def test_histogram_alpha_star_of_gaussian_data_is_table_1():
+    # a histogram of 2^23 N(0,1) values recovers the alpha* of Table 1 (D is
+    # flat near its minimum, so a sample moves alpha* by about a percent)
+    x = np.random.default_rng(4).normal(size=1 << 23).astype(np.float32)
+    _, st = o.calibrate(x, 4, 2, True)
+    c = o.histogram_abs(x, True, st[0], st[1], 8192, 16.0)
+    for (b, k), ref in [((4, 2), 1.4136), ((5, 2), 0.4828), ((3, 1), 1.3015)]:
+        a, _ = o.alpha_star_hist(c, 16.0, b, k)
+        assert abs(a - ref) <= 0.02 * ref
+
+
+# ----------------------------------------- quantisation-aware training ---
+
+def test_dn_backward_is_the_derivative_of_dn():
+    # central finite differences of L(x) = sum_i w_i x_hat_i(x), x_hat = DN(x)
+    # in fp64 (mean and sigma recomputed from the perturbed x)
+    rng = np.random.default_rng(12)
+    x = rng.normal(1.5, 2.0, 40)
+    w = rng.normal(size=40)
+
+    def loss(v):
+        mu = v.mean()
+        sig = np.sqrt(((v - mu) ** 2).mean())
+        return float(np.dot(w, (v - mu) / (sig + 1e-7)))
+
+    mu = x.mean()
+    sig = np.sqrt(((x - mu) ** 2).mean())
+    got = o.dn_backward(w.astype(np.float32), x.astype(np.float32), mu, sig).astype(np.float64)
+    h = 1e-6
+    for j in range(40):
+        e = np.zeros(40)
+        e[j] = h
+        fd = (loss(x + e) - loss(x - e)) / (2 * h)
+        # the oracle sees x and g rounded to fp32
+        assert abs(got[j] - fd) <= 1e-4 * max(1.0, abs(fd))
+
+
+def test_dn_backward_kills_shift_and_scale_directions():
+    # DN(x + a) = DN(x) and DN(c x) ~ DN(x): the gradient is orthogonal to
+    # the constant vector and (for eps -> 0) to x - mu
+    rng = np.random.default_rng(13)
+    x = rng.normal(0.3, 1.7, 500).astype(np.float32)
+    g = rng.normal(size=500).astype(np.float32)
+    xd = x.astype(np.float64)
+    mu = xd.mean()
+    sig = np.sqrt(((xd - mu) ** 2).mean())
+    gx = o.dn_backward(g, x, mu, sig).astype(np.float64)
+    assert abs(gx.sum()) <= 1e-4 * np.abs(gx).sum()
+    assert abs(np.dot(gx, xd - mu)) <= 1e-4 * np.abs(gx).sum() * sig
+
+
+def test_ema_closed_form():
+    # T updates with constant batch statistics b: r_T = b + (1 - gamma)^T (r_0 - b)
+    r = np.array([2.0, 0.5])
+    b = np.array([-1.0, 3.0])
+    g = 0.1
+    for _ in range(50):
+        r = o.ema(b, r, g)
+    exp = b + (1 - g) ** 50 * (np.array([2.0, 0.5]) - b)
+    assert np.allclose(r, exp, rtol=1e-13, atol=1e-13)
+
+
+def test_dn_project_is_dn_then_projection():
+    rng = np.random.default_rng(14)
+    x = rng.normal(0.7, 2.5, 3000).astype(np.float32)
+    mu, sig = float(x.astype(np.float64).mean()), float(x.astype(np.float64).std())
+    a = float(np.float32(o.alpha_star(4, 2)[0]))
+    codes, xq = o.dn_project(x, mu, sig, a, 4, 2, True)
+    xh = (x - np.float32(mu)) / np.float32(sig + 1e-7)           # float32 ops
+    assert np.array_equal(codes, o.project_codes(xh, a, 4, 2, True))
+    q = o.project_values(xh, a, 4, 2, True)
+    assert np.array_equal(xq, (np.float32(a) * q.astype(np.float32)))
