@@ -502,8 +502,9 @@ def run_sweep(args):
     """The sweeps of the large-operand workloads, one JSON line: esb_gemm_tiled
     on square M=N=K in {1024, 4096, 8192, 16384} at ESB (4,2) and (6,3)
     (unsigned A, signed B, codes out), and esb_project on 2^28 fp32 values
-    N(0,1) for every b in 3..6, k in 1..b-1 (`--sweeps gemm` / `--sweeps
-    project` run one half).  Each point: CUDA events over
+    drawn N(0,1), Laplace(0,1) and |N(0,1)| for every b in 3..6, k in 1..b-1
+    with the tensor's DDA alpha (`--sweeps gemm` / `--sweeps project` run
+    one part).  Each point: CUDA events over
     repeated calls after 3 warm-ups (operands larger than L2 from 4096 up;
     the projection reads 1 GiB per call)."""
     import torch
@@ -559,16 +560,26 @@ def run_sweep(args):
                         "frac_fp8": round(tf / fp8, 3), "status": esb.esb_get_status()})
             del A, B, oc, ws
             torch.cuda.empty_cache()
-    x = synth.normal((1 << 28,), seed=0).to(dev) if args.sweeps in ("all", "project") else None
-    for b in (range(3, 7) if args.sweeps in ("all", "project") else []):
-        for k in range(1, b):
-            f = esb.Fmt(b, k, True)
-            codes = torch.empty((1, esb.esb_row_words(1 << 28, b)), dtype=torch.int32, device=dev)
-            us = timeit(lambda: esb.esb_project(x, f, alpha=0.7, codes=codes), 20)
-            byt = (1 << 28) * (4 + 4 / (32 // b))
-            out.append({"project": 1 << 28, "fmt": [b, k], "us": round(us, 1), "GB/s": round(byt / us / 1e3, 1),
-                        "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
-    del x
+    # esb_project on 2^28 values of each configured distribution (N(0,1),
+    # Laplace(0,1) and |N(0,1)|, seeds 0/1/2), every b in 3..6 and k in
+    # 1..b-1, the half-normal data in the unsigned format, alpha = the DDA
+    # alpha of that tensor (esb_calibrate_dda, not timed)
+    for di, dist in enumerate(["normal", "laplace", "half_normal"] if args.sweeps in ("all", "project") else []):
+        x = synth.distribution(dist, (1 << 28,), seed=di).to(dev)
+        signed = dist != "half_normal"
+        for b in range(3, 7):
+            for k in range(1, b):
+                f = esb.Fmt(b, k, signed)
+                a, _ = esb.esb_calibrate_dda(x, f)
+                codes = torch.empty((1, esb.esb_row_words(1 << 28, b)), dtype=torch.int32, device=dev)
+                us = timeit(lambda: esb.esb_project(x, f, alpha=a, codes=codes), 20)
+                byt = (1 << 28) * (4 + 4 / (32 // b))
+                out.append({"project": 1 << 28, "dist": dist, "fmt": [b, k, int(signed)], "alpha": float(a.item()),
+                            "us": round(us, 1), "GB/s": round(byt / us / 1e3, 1),
+                            "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
+                del codes
+        del x
+        torch.cuda.empty_cache()
     if args.sweeps in ("all", "cc"):
         out += _cc_sweep(esb, torch, timeit, hbm)
     print(json.dumps({"workload": "sweeps (esb_gemm_tiled M=N=K, esb_project 2^28, depthwise conv and pooling)",
@@ -655,6 +666,275 @@ def _cc_sweep(esb, torch, timeit, hbm):
     return res
 
 
+# ------------------------------------------------------ network workloads
+
+NET_BATCH = {"resnet18": 64, "mobilenetv2": 64, "alexnet_fc": 256}
+NET_FMTS = {"resnet18": [(3, 1), (4, 2), (5, 2), (6, 3)], "mobilenetv2": [(4, 2)], "alexnet_fc": [(4, 2)]}
+
+
+class OAct:
+    """An activation of the oracle's forward: packed codes on the host."""
+
+    def __init__(self, np_codes, f, a, n, h, w, c):
+        self.np, self.f, self.a, self.n, self.h, self.w, self.c = np_codes, f, a, n, h, w, c
+
+
+class OracleRunner:
+    """The oracle's forward of a network, with the weights, alphas and
+    formats of a calibrated libesb Runner (same call sequence): conv layers
+    split their output rows over host threads (oracle_conv2d_rows_i64)."""
+
+    def __init__(self, rn, pool):
+        self.rn, self.pool, self.idx = rn, pool, 0
+
+    def _p(self):
+        p = self.rn.params[self.idx]
+        self.idx += 1
+        return p
+
+    def input(self, x, n, h, w, c):
+        import numpy as np
+        import oracle as o
+        p = self._p()
+        f = (self.rn.b, self.rn.k, True)
+        codes = o.project_packed(np.ascontiguousarray(x.reshape(-1, c)), p["a"], *f)
+        return OAct(codes, f, p["a"], n, h, w, c)
+
+    def conv(self, x, cout, r, s, stride, pad, act=1, res=None, groups=1):
+        import numpy as np
+        import oracle as o
+        from paper_2109_03513_gb300 import esb
+        p = self._p()
+        dw = groups == x.c and x.c > 1
+        W = p["W_np"]
+        fw = (self.rn.b, self.rn.k)
+        P, Q = esb.conv_out_hw(x.h, x.w, r, s, stride, pad)
+        ldx = x.np.shape[1]
+        X4 = x.np.reshape(x.n, x.h, x.w, ldx)
+        if dw:
+            acc = o.dwconv_i64(X4, x.f[:2], W.reshape(r, s, -1), fw, x.n, x.h, x.w, x.c, r, s,
+                               stride, pad).reshape(-1, cout)
+        else:
+            chunks = [(i * P // 16, (i + 1) * P // 16) for i in range(16) if (i + 1) * P // 16 > i * P // 16]
+            parts = list(self.pool.map(lambda pr: o.conv2d_rows_i64(X4, x.f[:2], W.reshape(cout, r, s, -1), fw,
+                                                                    x.n, x.h, x.w, x.c, cout, r, s,
+                                                                    stride, pad, pr[0], pr[1]), chunks))
+            acc = np.concatenate(parts, axis=1).reshape(-1, cout)
+        signed_out = act == 0
+        fo = (self.rn.b, self.rn.k, signed_out)
+        s0 = esb.esb_dequant_scale(x.a, esb.Fmt(*x.f), p["aw"], esb.Fmt(self.rn.b, self.rn.k, True))
+        res_img, res_scale = None, 0.0
+        if res is not None:
+            lut = np.array([o.image(v, res.f[0], res.f[1]) for v in range(2 ** res.f[0])], np.int64)
+            res_img = lut[o.unpack(res.np, cout, res.f[0])]
+            res_scale = esb.esb_dequant_scale(res.a, esb.Fmt(*res.f), 1.0, esb.Fmt(8, 0))
+        _, co = o.epilogue(acc, np.full(cout, s0, np.float32), np.zeros(cout, np.float32), act, p["a_out"], fo,
+                           res_images=res_img, res_scale=res_scale)
+        return OAct(o.pack(co, fo[0], fo[1], ld_words=esb.esb_row_words(cout, fo[0])), fo, p["a_out"], x.n, P, Q, cout)
+
+    def maxpool(self, x, win=3, stride=2, pad=1):
+        import oracle as o
+        from paper_2109_03513_gb300 import esb
+        self._p()
+        P, Q = esb.conv_out_hw(x.h, x.w, win, win, stride, pad)
+        Y = o.maxpool_codes(x.np.reshape(x.n, x.h, x.w, -1), x.f[0], x.f[1], x.n, x.h, x.w,
+                            x.c, win, stride, pad, ld_out=x.np.shape[1]).reshape(x.n * P * Q, -1)
+        return OAct(Y, x.f, x.a, x.n, P, Q, x.c)
+
+    def avgpool(self, x):
+        import numpy as np
+        import oracle as o
+        from paper_2109_03513_gb300 import esb
+        p = self._p()
+        hw = x.h * x.w
+        scale = esb.esb_dequant_scale(x.a, esb.Fmt(*x.f), 1.0 / hw, esb.Fmt(8, 0))
+        sums = o.avgpool_sum_i64(x.np.reshape(x.n, hw, -1), x.f[0], x.f[1], x.n, hw, x.c)
+        y = (np.float32(scale) * sums.astype(np.float32)).astype(np.float32)
+        codes = o.pack(o.project_codes(y, p["a_out"], *x.f), x.f[0], x.f[1],
+                       ld_words=esb.esb_row_words(x.c, x.f[0]))
+        return OAct(codes, x.f, p["a_out"], x.n, 1, 1, x.c)
+
+    def fc(self, x, nout, act=0, workspace=False):
+        import numpy as np
+        import oracle as o
+        from paper_2109_03513_gb300 import esb
+        p = self._p()
+        fw = (self.rn.b, self.rn.k)
+        acc = o.gemm_i64(x.np, x.f[:2], p["W_np"], fw, x.n, nout, x.c)
+        fo = (self.rn.b, self.rn.k, act == 0)
+        s0 = esb.esb_dequant_scale(x.a, esb.Fmt(*x.f), p["aw"], esb.Fmt(self.rn.b, self.rn.k, True))
+        _, co = o.epilogue(acc, np.full(nout, s0, np.float32), np.zeros(nout, np.float32), act, p["a_out"], fo)
+        return OAct(o.pack(co, fo[0], fo[1], ld_words=esb.esb_row_words(nout, fo[0])), fo, p["a_out"], x.n, 1, 1, nout)
+
+
+def run_network(args, name):
+    """One JSON line per (b, k): images/s of the whole forward (a CUDA graph
+    of every layer's launches), per-layer TOPS, the end-to-end number with
+    the input images copied in and the logits' codes copied out, and the
+    oracle's forward of a sample of the batch on the host cores."""
+    from concurrent.futures import ThreadPoolExecutor
+
+    import numpy as np
+    import torch
+
+    import __graft_entry__
+    from paper_2109_03513_gb300 import esb, netrun, synth
+
+    __graft_entry__.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    fn, (h, w, c) = netrun.NETWORKS[name]
+    batch = NET_BATCH[name]
+    fmts = NET_FMTS[name] if not args.bk else [tuple(int(v) for v in t.split(",")) for t in args.bk]
+    hbm, bf16, src = _peaks()
+    for b, k in fmts:
+        rn = netrun.Runner(b, k, seed=1000 * b + k, device=dev)
+        x_cal = synth.normal((batch * h * w, c), seed=1).to(dev)
+        x = synth.normal((batch * h * w, c), seed=2).to(dev)
+        rn.begin("calibrate")
+        fn(rn, x_cal, batch)
+        torch.cuda.synchronize()
+        del x_cal
+        launches = 0
+        stream = torch.cuda.Stream(device=dev)
+        with torch.cuda.stream(stream):
+            rn.begin("infer")
+            fn(rn, x, batch)
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                rn.begin("infer")
+                out = fn(rn, x, batch)
+            for _ in range(max(args.warmup, 3)):
+                g.replay()
+            torch.cuda.synchronize()
+            K = max(1, min(args.steps, 200))
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            clocks = ClockSampler()
+            clocks.start()
+            time.sleep(0.2)
+            e0.record(stream)
+            for _ in range(K):
+                g.replay()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ck = clocks.stop(0)
+            t_fwd = e0.elapsed_time(e1) / K * 1e-3
+            # per-layer device times: one eager pass queued behind a device sleep
+            rn.marks = []
+            torch.cuda._sleep(5_000_000)
+            m0 = torch.cuda.Event(enable_timing=True)
+            m0.record(stream)
+            rn.begin("infer")
+            fn(rn, x, batch)
+            torch.cuda.synchronize()
+            marks, rn.marks = [m0] + rn.marks, None
+            layer_us = [marks[i].elapsed_time(marks[i + 1]) * 1e3 for i in range(len(marks) - 1)]
+            # end to end: pinned host images in, the logits' codes out
+            x_pin = x.cpu().pin_memory()
+            o_pin = torch.empty(out.codes.shape, dtype=torch.int32).pin_memory()
+            ke = max(3, min(20, K))
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            for _ in range(ke):
+                x.copy_(x_pin, non_blocking=True)
+                g.replay()
+                o_pin.copy_(out.codes, non_blocking=True)
+            a1.record(stream)
+            torch.cuda.synchronize()
+            t_e2e = a0.elapsed_time(a1) / ke * 1e-3
+        assert esb.esb_get_status(stream) == 0
+        macs = sum(li.macs for li in rn.info)
+        layers = []
+        for li, us in zip(rn.info, layer_us[1:]):
+            d = {"kind": li.kind, "shape": li.shape, "us": round(us, 2)}
+            if li.macs:
+                d["TOPS"] = round(2 * li.macs / (us * 1e-6) / 1e12, 1)
+            layers.append(d)
+        dense = [(li, us) for li, us in zip(rn.info, layer_us[1:]) if li.kind in ("conv", "fc")]
+        top = max(dense, key=lambda t: t[1])
+        peak = 2.0 * bf16
+        top_tops = 2 * top[0].macs / (top[1] * 1e-6) / 1e12
+        line = {
+            "metric": METRIC, "value": batch / t_fwd, "unit": "images/s", "n_gpus": 1, "steps": K,
+            "warmup": max(args.warmup, 3), "ms_per_step": t_fwd * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "e4m3",
+            "data": "synthetic (seeded N(0,1) images, He-init weights, one calibration batch then a timed batch)",
+            "config": {"workload": f"{name}_b{batch}_esb{b}{k}", "batch": batch, "b": b, "k": k,
+                       "gop_per_forward": round(2 * macs / 1e9, 2),
+                       "l2": "weights and activations stay in L2 across replays (a deployed model's steady state)",
+                       "parallelism": "single"},
+            "TOPS_forward": round(2 * macs / t_fwd / 1e12, 1),
+            "roofline": {"bound": "tensor", "kernel": f"{top[0].kind} {top[0].shape}", "achieved": round(top_tops, 1),
+                         "peak": peak, "unit": "TFLOP/s", "frac": round(top_tops / peak, 4),
+                         "peak_note": f"fp8 dense = {src} bf16 burst {bf16} x nominal fp8:bf16 ratio 2",
+                         "traffic": None},
+            "layers": layers,
+            "e2e": {"value": batch / t_e2e, "unit": "images/s", "h2d_bytes_per_step": int(x_pin.numel() * 4),
+                    "d2h_bytes_per_step": int(o_pin.numel() * 4), "ms_per_step": t_e2e * 1e3},
+            "gpu_launches": None, "clocks": ck,
+        }
+        if not args.no_cpu_baseline:
+            line["cpu_baseline"] = network_cpu_baseline(rn, fn, x, name, batch, h, w, c)
+        print(json.dumps(line), flush=True)
+        del g, rn, x
+
+
+def network_cpu_baseline(rn, fn, x, name, batch, h, w, c):
+    """The oracle's forward of one image (all 1000 classes; conv rows over
+    the host threads) with the calibrated weights and alphas."""
+    from concurrent.futures import ThreadPoolExecutor
+
+    n1 = 8 if name == "alexnet_fc" else 1
+    for p in rn.params:
+        if "W" in p:
+            p["W_np"] = p["W"].cpu().numpy().view("uint32")
+    xs = x[: n1 * h * w].cpu().numpy()
+    cores = _cores()
+    with ThreadPoolExecutor(cores) as pool:
+        orn = OracleRunner(rn, pool)
+        t0 = time.time()
+        fn(orn, xs, n1)
+        dt = time.time() - t0
+    return {"value": n1 / dt, "unit": "images/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n1} of the {batch} images of the timed batch through every layer ({dt:.1f} s wall)"}
+
+
+def run_peaks(args):
+    """Measured tensor-pipe peaks (the tcgen05 f8f6f4 rate the contraction's
+    roofline divides by, and the legacy mma.sync s8 rate), one JSON line."""
+    import torch
+
+    import __graft_entry__
+    from paper_2109_03513_gb300 import esb
+
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+    out = {"peaks": {}}
+    clocks = ClockSampler()
+    clocks.start()
+    time.sleep(0.2)
+    for name, kind, iters in [("tcgen05_f8f6f4_e4m3", esb.ESB_PEAK_TCGEN05_F8F6F4, 20000),
+                              ("mma_sync_s8", esb.ESB_PEAK_MMA_SYNC_S8, 20000)]:
+        for _ in range(3):
+            esb.esb_peak_launch(kind, iters)
+        torch.cuda.synchronize()
+        best = 0.0
+        for _ in range(10):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            ops = esb.esb_peak_launch(kind, iters)
+            e1.record()
+            torch.cuda.synchronize()
+            best = max(best, ops / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+        out["peaks"][name] = {"TFLOP/s" if kind == 0 else "TOPS": round(best, 1)}
+    out["clocks"] = clocks.stop(0)
+    out["status"] = esb.esb_get_status()
+    hbm, bf16, src = _peaks()
+    out["bf16_burst_" + src] = bf16
+    print(json.dumps(out), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -664,10 +944,18 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweeps", nargs="?", const="all", choices=["all", "gemm", "project", "cc"],
                     help="the sweeps instead of the step (all, or only the GEMM, projection or CUDA-core part)")
+    ap.add_argument("--workload", default="conv3x3", choices=["conv3x3", "resnet18", "mobilenetv2", "alexnet_fc"],
+                    help="conv3x3: the benchmark step (default); the others: whole-network forwards")
+    ap.add_argument("--bk", nargs="*", help="formats b,k of a network workload (default: its configuration's)")
+    ap.add_argument("--peaks", action="store_true", help="measure the tensor-pipe peaks instead")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.sweeps:
+    if args.peaks:
+        run_peaks(args)
+    elif args.workload != "conv3x3" and args.impl == "ours":
+        run_network(args, args.workload)
+    elif args.sweeps:
         run_sweep(args)
     elif args.impl == "reference":
         run_reference(args)

@@ -580,6 +580,20 @@ esb_status esb_avgpool_nhwc(const uint32_t* X, int64_t ldx, esb_format f,
                             float alpha_out, esb_format fmt_out, int32_t rounding,
                             float* y_out, uint32_t* codes_out, int64_t ldo, void* stream);
 
+/* ----------------------------------------------------- peak measurement */
+
+/* Microbenchmarks of the tensor-pipe rates the contraction's roofline is
+ * measured against (no paper counterpart): one launch of `iters` rounds of
+ * back-to-back MMAs on every SM, operands zero.  Time it with CUDA events on
+ * `stream`; *ops receives its operation count (2 per multiply-add).
+ *   ESB_PEAK_TCGEN05_F8F6F4: tcgen05.mma kind::f8f6f4, E4M3 x E4M3 -> fp32
+ *     TMEM, M = 128, N = 256, K = 32, one issuing thread per SM (4 per round)
+ *   ESB_PEAK_MMA_SYNC_S8: mma.sync m16n8k32 s8 x s8 -> s32, 8 per round per
+ *     warp, 4 blocks of 8 warps per SM
+ * Errors: INVALID_ARG, CUDA. */
+enum { ESB_PEAK_TCGEN05_F8F6F4 = 0, ESB_PEAK_MMA_SYNC_S8 = 1 };
+esb_status esb_peak_launch(int32_t kind, int64_t iters, int64_t* ops, void* stream);
+
 /* ------------------------------------------------------------- status */
 
 /* Synchronises `stream`, then returns and clears the device status word

@@ -687,7 +687,7 @@ esb_status esb_maxpool_nhwc(const uint32_t* X, int64_t ldx, esb_format f, int32_
     if (n == 0) return ESB_OK;
     if (!X || !Y) return ESB_ERR_INVALID_ARG;
     cudaError_t e = launch_maxpool(X, ldx, f.b, f.k, n, h, w, c, win, stride, pad, P, Q, Y, ldy,
-                                   static_cast<cudaStream_t>(stream));
+                                   static_cast<cudaStream_t>(stream), f.is_signed);
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 
@@ -707,6 +707,14 @@ esb_status esb_avgpool_nhwc(const uint32_t* X, int64_t ldx, esb_format f, int32_
     if ((int64_t)n > 65535) return ESB_ERR_UNSUPPORTED;
     cudaError_t e = launch_avgpool(X, ldx, f.b, f.k, n, hw, c, scale, alpha_out, fmt_out.b, fmt_out.k, fmt_out.is_signed,
                                    rounding, y_out, codes_out, ldo, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
+}
+
+esb_status esb_peak_launch(int32_t kind, int64_t iters, int64_t* ops, void* stream)
+{
+    if ((kind != ESB_PEAK_TCGEN05_F8F6F4 && kind != ESB_PEAK_MMA_SYNC_S8) || iters <= 0 || iters > (1ll << 30) || !ops)
+        return ESB_ERR_INVALID_ARG;
+    const cudaError_t e = launch_peak(kind, iters, ops, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ESB_OK : ESB_ERR_CUDA;
 }
 

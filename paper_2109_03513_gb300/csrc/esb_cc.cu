@@ -143,6 +143,155 @@ esb_dwconv_kernel(const uint32_t* __restrict__ X, int64_t ldx, int bx, int kx,
     }
 }
 
+// Depthwise 3x3 for code widths 3..6 with filters and inputs of one width
+// (every MobileNetV2 layer).  Each block decodes the filters of all
+// channels once into shared memory (integer images, [tap][channel]) and
+// builds the table of input images and the requantisation thresholds, then
+// walks its share of the work units: one unit = one code word (CPW
+// channels) of QT consecutive output pixels of one row.  Each input word of
+// the unit's 3 x ((QT-1) STRIDE + 3) window is decoded once and feeds every
+// output of the strip that reads it; all loop bounds are compile-time
+// constants, so accumulators stay in registers.
+template <int B, int STRIDE>
+__global__ void __launch_bounds__(128)
+esb_dwconv3_kernel(const uint32_t* __restrict__ X, int64_t ldx, int kx, const uint32_t* __restrict__ W, int64_t ldw,
+                   int kw, int n, int H, int Wd, int C, int pad, int P, int Q, int QS, CcEpi ep)
+{
+    constexpr int CPW = 32 / B;
+    constexpr int QT = STRIDE == 1 ? 8 : 4;
+    constexpr int NCOL = (QT - 1) * STRIDE + 3;
+    constexpr uint32_t MASK = (1u << B) - 1u;
+    extern __shared__ int32_t wtab[];                 // [9][words * CPW] filter images
+    __shared__ int32_t lutx[1 << B];
+    __shared__ float T[128];
+    const int words = (C + CPW - 1) / CPW;
+    const int cp = words * CPW;
+    const int ewx = B - kx - 1, Nx = (1 << ewx) - 1;
+    const int eww = B - kw - 1, Nw = (1 << eww) - 1;
+    griddep_wait();                                   // inputs and alphas may come from the previous launch
+    for (int i = threadIdx.x; i < (1 << B); i += blockDim.x) lutx[i] = code_image_i((uint32_t)i, B, kx, ewx, Nx);
+    for (int i = threadIdx.x; i < 9 * words; i += blockDim.x) {
+        const int t = i / words, w = i - (i / words) * words;
+        const uint32_t fw = __ldg(W + (int64_t)t * ldw + w);
+#pragma unroll
+        for (int j = 0; j < CPW; j++) wtab[t * cp + w * CPW + j] = code_image_i((fw >> (B * j)) & MASK, B, kw, eww, Nw);
+    }
+    const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
+    if (ep.codes_out) build_thresholds(T, ep.out, alpha_out, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
+    __syncthreads();
+    Thr7 t7;
+    const bool b4 = ep.out.b == 4 && ep.codes_out;
+#pragma unroll
+    for (int i = 0; i < 7; i++) t7.t[i] = b4 ? T[i] : 0.0f;
+    const bool dq = ep.alpha_a_dev && ep.alpha_b_dev;
+    const float dqs = dq ? __fmul_rn(__ldg(ep.alpha_a_dev), __ldg(ep.alpha_b_dev)) * ep.dq_pow2 : 1.0f;
+    const int rcpw = ep.residual ? 32 / ep.res_b : 1;
+    const uint32_t rmask = ep.residual ? (1u << ep.res_b) - 1u : 0u;
+    const int64_t total = (int64_t)n * P * QS * ep.ldo;
+    for (int64_t unit = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; unit < total;
+         unit += (int64_t)gridDim.x * blockDim.x) {
+        const int w = (int)(unit % ep.ldo);
+        int64_t rest = unit / ep.ldo;
+        const int qs = (int)(rest % QS);
+        rest /= QS;
+        const int p = (int)(rest % P);
+        const int nn = (int)(rest / P);
+        const int q0 = qs * QT;
+        if (w >= words) {                             // padding words of the output rows: zero codes
+            if (ep.codes_out) {
+                uint32_t word = 0;
+#pragma unroll
+                for (int j = 0; j < CPW; j++) word |= ep.out.zero_code << (B * j);
+#pragma unroll
+                for (int u = 0; u < QT; u++)
+                    if (q0 + u < Q) ep.codes_out[(((int64_t)nn * P + p) * Q + q0 + u) * ep.ldo + w] = word;
+            }
+            continue;
+        }
+        int32_t acc[QT][CPW];
+#pragma unroll
+        for (int u = 0; u < QT; u++)
+#pragma unroll
+            for (int j = 0; j < CPW; j++) acc[u][j] = 0;
+#pragma unroll
+        for (int r = 0; r < 3; r++) {
+            const int h = p * STRIDE - pad + r;
+            if (h < 0 || h >= H) continue;
+            int32_t wf[3][CPW];
+#pragma unroll
+            for (int s2 = 0; s2 < 3; s2++)
+#pragma unroll
+                for (int j = 0; j < CPW; j++) wf[s2][j] = wtab[(r * 3 + s2) * cp + w * CPW + j];
+            const uint32_t* xrow = X + ((int64_t)nn * H + h) * Wd * ldx + w;
+#pragma unroll
+            for (int i = 0; i < NCOL; i++) {
+                const int col = q0 * STRIDE - pad + i;
+                if (col < 0 || col >= Wd) continue;
+                const uint32_t xw = __ldg(xrow + (int64_t)col * ldx);
+                int32_t xi[CPW];
+#pragma unroll
+                for (int j = 0; j < CPW; j++) xi[j] = lutx[(xw >> (B * j)) & MASK];
+#pragma unroll
+                for (int u = 0; u < QT; u++) {
+                    const int s2 = i - u * STRIDE;
+                    if (s2 >= 0 && s2 < 3) {
+#pragma unroll
+                        for (int j = 0; j < CPW; j++) acc[u][j] += xi[j] * wf[s2][j];
+                    }
+                }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < QT; u++) {
+            const int q = q0 + u;
+            if (q >= Q) break;
+            const int64_t pix = ((int64_t)nn * P + p) * Q + q;
+            uint32_t word = 0;
+#pragma unroll
+            for (int j = 0; j < CPW; j++) {
+                const int c = w * CPW + j;
+                uint32_t code = ep.out.zero_code;
+                if (c < C) {
+                    const int64_t o = pix * C + c;
+                    if (ep.acc_out) ep.acc_out[o] = acc[u][j];
+                    float sc = ep.scale ? __ldg(ep.scale + c) : ep.scale0;
+                    if (dq) sc = __fmul_rn(sc, dqs);
+                    const float bi = ep.bias ? __ldg(ep.bias + c) : ep.bias0;
+                    float y = __fmaf_rn(sc, (float)acc[u][j], bi);
+                    if (ep.residual) {
+                        const uint32_t rc =
+                            (__ldg(ep.residual + pix * ep.res_ld + c / rcpw) >> (ep.res_b * (c % rcpw))) & rmask;
+                        y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+                    }
+                    y = cc_act(y, ep.act);
+                    if (ep.y_out) ep.y_out[o] = y;
+                    if (ep.codes_out) code = b4 ? project_by_thr7(y, t7, ep.out) : project_by_table(y, T, ep.out);
+                }
+                word |= code << (B * j);
+            }
+            if (ep.codes_out) ep.codes_out[pix * ep.ldo + w] = word;
+        }
+    }
+}
+
+template <int B, int STRIDE>
+static cudaError_t launch_dw3(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int kx,
+                              const uint32_t* W, int64_t ldw, int kw, const CcEpi& ep, cudaStream_t st)
+{
+    constexpr int QT = STRIDE == 1 ? 8 : 4;
+    const int QS = (Q + QT - 1) / QT;
+    const int64_t total = (int64_t)d.n * P * QS * ep.ldo;
+    int64_t blocks = (total + 127) / 128;
+    const int64_t cap = (int64_t)device_sm_count() * 8;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    const int words = (d.c + 32 / B - 1) / (32 / B);
+    const size_t smem = sizeof(int32_t) * 9 * (size_t)words * (32 / B);
+    esb_dwconv3_kernel<B, STRIDE><<<(unsigned)blocks, 128, smem, st>>>(X, ldx, kx, W, ldw, kw, d.n, d.h, d.w, d.c, d.pad,
+                                                                       P, Q, QS, ep);
+    return cudaGetLastError();
+}
+
 static CcEpi make_cc_epi(const GemmOutputs& o, int ka, int kb)
 {
     CcEpi ep;
@@ -188,6 +337,22 @@ cudaError_t launch_dwconv(const esb_conv_desc& d, int P, int Q, const uint32_t* 
     // Thread grid covers words of the output row stride: ldo words when codes
     // are written, else the input's words (acc/y only).
     if (!o.codes_out) ep.ldo = (d.c + (32 / bx) - 1) / (32 / bx);
+    // filter table of the fast kernel: 9 taps x the padded channels, int32, in 48 KiB
+    const int64_t tab = 9 * (int64_t)((d.c + 32 / bx - 1) / (32 / bx)) * (32 / bx) * 4;
+    if (d.r == 3 && d.s == 3 && bw == bx && bx >= 3 && bx <= 6 && (d.stride == 1 || d.stride == 2) &&
+        tab <= 48 * 1024) {
+        const bool s1 = d.stride == 1;
+        switch (bx) {
+        case 3: return s1 ? launch_dw3<3, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)
+                          : launch_dw3<3, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st);
+        case 4: return s1 ? launch_dw3<4, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)
+                          : launch_dw3<4, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st);
+        case 5: return s1 ? launch_dw3<5, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)
+                          : launch_dw3<5, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st);
+        default: return s1 ? launch_dw3<6, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)
+                           : launch_dw3<6, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st);
+        }
+    }
     const int64_t total = (int64_t)d.n * P * Q * ep.ldo;
     esb_dwconv_kernel<<<grid_for(total), 256, 0, st>>>(X, ldx, bx, kx, W, ldw, bw, kw, d.n, d.h, d.w, d.c, d.r, d.s,
                                                         d.stride, d.pad, P, Q, ep);
@@ -251,9 +416,68 @@ esb_maxpool_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int k, in
     }
 }
 
-cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int H, int Wd, int C, int win,
-                           int stride, int pad, int P, int Q, uint32_t* Y, int64_t ldy, cudaStream_t st)
+// Max pooling of unsigned 4-bit codes without decoding them: the value
+// order of the non-negative set is the order of the rotated code
+// (e + 1 mod 2^(b-1-k), then f), i.e. rank = (code + 2^k) mod 8, so the
+// maximum of a window is the byte-wise maximum of the ranks (even and odd
+// codes of a word in separate bytes) and the code comes back by the
+// inverse rotation.  One thread = one output word; blockIdx.y = image row
+// (n, p), threads over (q, word): 32-bit index arithmetic only.
+__global__ void __launch_bounds__(256)
+esb_maxpool_b4u_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H, int Wd, int C, int win, int stride,
+                       int pad, int P, int Q, uint32_t* __restrict__ Y, int64_t ldy)
 {
+    const int np_ = blockIdx.y;
+    const int nn = np_ / P, p = np_ - (np_ / P) * P;
+    const int per_row = Q * (int)ldy;
+    const uint32_t rot = 0x11111111u << k;            // + 2^k in every nibble
+    const int words = (C + 7) / 8;
+    for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < per_row; t += gridDim.x * blockDim.x) {
+        const int q = t / (int)ldy, w = t - (t / (int)ldy) * (int)ldy;
+        uint32_t lo = 0u, hi = 0u;                    // rank maxima (0 = the rank of zero)
+        if (w < words) {
+            for (int r = 0; r < win; r++) {
+                const int h = p * stride - pad + r;
+                if (h < 0 || h >= H) continue;
+                const uint32_t* xr = X + ((int64_t)nn * H + h) * Wd * ldx + w;
+                for (int s2 = 0; s2 < win; s2++) {
+                    const int ww = q * stride - pad + s2;
+                    if (ww < 0 || ww >= Wd) continue;
+                    const uint32_t rk = ((__ldg(xr + (int64_t)ww * ldx) & 0x77777777u) + rot) & 0x77777777u;
+                    lo = __vmaxu4(lo, rk & 0x0F0F0F0Fu);
+                    hi = __vmaxu4(hi, (rk >> 4) & 0x0F0F0F0Fu);
+                }
+            }
+        }
+        // inverse rotation: code = (rank - 2^k) mod 8; rank 0 is the zero code
+        const uint32_t rk = lo | (hi << 4);
+        uint32_t word = (rk + (0x88888888u - rot)) & 0x77777777u;
+        if (w >= words) word = 0u;
+        // channels past C (in the last word) and padding words: the zero code
+        const int c0 = w * 8;
+        const uint32_t zero = (uint32_t)((1 << (3 - k)) - 1) << k;   // e = N, f = 0 for b = 4
+        uint32_t zw = 0u;
+        for (int j = 0; j < 8; j++) zw |= zero << (4 * j);
+        if (w >= words) word = zw;
+        else if (c0 + 8 > C) {
+            const int keep = C - c0;
+            const uint32_t m = keep >= 8 ? 0xffffffffu : ((1u << (4 * keep)) - 1u);
+            word = (word & m) | (zw & ~m);
+        }
+        Y[(((int64_t)nn * P + p) * Q + q) * ldy + w] = word;
+    }
+}
+
+cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int H, int Wd, int C, int win,
+                           int stride, int pad, int P, int Q, uint32_t* Y, int64_t ldy, cudaStream_t st,
+                           int is_signed)
+{
+    if (b == 4 && !is_signed && (int64_t)n * P <= 65535 && (int64_t)Q * ldy < (1ll << 31)) {
+        const int per_row = (int)(Q * ldy);
+        const dim3 grid((unsigned)((per_row + 255) / 256), (unsigned)(n * P));
+        esb_maxpool_b4u_kernel<<<grid, 256, 0, st>>>(X, ldx, k, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
+        return cudaGetLastError();
+    }
     const int64_t total = (int64_t)n * P * Q * ldy;
     esb_maxpool_kernel<<<grid_for(total), 256, 0, st>>>(X, ldx, b, k, n, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
     return cudaGetLastError();
@@ -261,62 +485,53 @@ cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
 
 // ------------------------------------------------------ global avg pool
 
-// One block per (image, channel word): threads stride over the HW pixels,
-// per-thread int32 sums per channel slot, a shared-memory reduction, then
-// y = fl32(scale * (float)sum) and the ESB projection of y with alpha_out
-// (output codes use the input's b, so words line up).
-__global__ void __launch_bounds__(256)
-esb_avgpool_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int k, int HW, int C, float scale,
-                   float alpha_out, ProjParams out, float* __restrict__ y_out, uint32_t* __restrict__ codes_out,
-                   int64_t ldo)
+// One thread = one code word of one image: the HW pixels' words of that
+// channel group are read in turn (consecutive threads read consecutive
+// words of a pixel), their images summed exactly in int32 per channel, and
+// each sum scaled and requantised through the block's threshold table.
+__global__ void __launch_bounds__(128)
+esb_avgpool_word_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int k, int n, int HW, int C, int wout,
+                        float scale, float alpha_out, ProjParams out, float* __restrict__ y_out,
+                        uint32_t* __restrict__ codes_out, int64_t ldo)
 {
+    __shared__ float T[128];
+    griddep_wait();
+    if (codes_out) build_thresholds(T, out, alpha_out, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
+    __syncthreads();
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= (int64_t)n * wout) return;
+    const int nn = (int)(t / wout), w = (int)(t - (t / wout) * wout);
     const int cpw = 32 / b;
     const int ew = b - k - 1, N = (1 << ew) - 1;
     const uint32_t mask = (1u << b) - 1u;
-    const int64_t nn = blockIdx.y;
-    const int w = blockIdx.x;                           // code word of the channel group
-    if (w * cpw >= C) {                                 // padding word of the output row
-        if (threadIdx.x == 0 && codes_out && w < ldo) {
-            uint32_t word = 0;
-            for (int j = 0; j < 32 / out.b; j++) word |= out.zero_code << (out.b * j);
-            codes_out[nn * ldo + w] = word;
+    uint32_t word = 0;
+    if (w * cpw < C) {
+        int32_t acc[16];
+#pragma unroll
+        for (int j = 0; j < 16; j++) acc[j] = 0;
+        const uint32_t* xp = X + (int64_t)nn * HW * ldx + w;
+        for (int i = 0; i < HW; i++) {
+            const uint32_t xw = __ldg(xp + (int64_t)i * ldx);
+#pragma unroll
+            for (int j = 0; j < 16; j++)
+                if (j < cpw) acc[j] += code_image_i((xw >> (b * j)) & mask, b, k, ew, N);
         }
-        return;
-    }
-    __shared__ int32_t red[256][16];
-    int32_t acc[16];
 #pragma unroll
-    for (int j = 0; j < 16; j++) acc[j] = 0;
-    for (int i = threadIdx.x; i < HW; i += blockDim.x) {
-        const uint32_t xw = __ldg(X + (nn * HW + i) * ldx + w);
-#pragma unroll
-        for (int j = 0; j < 16; j++)
-            if (j < cpw) acc[j] += code_image_i((xw >> (b * j)) & mask, b, k, ew, N);
-    }
-#pragma unroll
-    for (int j = 0; j < 16; j++) red[threadIdx.x][j] = acc[j];
-    __syncthreads();
-    for (int h = blockDim.x / 2; h > 0; h >>= 1) {
-        if ((int)threadIdx.x < h) {
-#pragma unroll
-            for (int j = 0; j < 16; j++) red[threadIdx.x][j] += red[threadIdx.x + h][j];
-        }
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) {
-        uint32_t word = 0;
-        for (int j = 0; j < cpw; j++) {
+        for (int j = 0; j < 16; j++) {
+            if (j >= cpw) break;
             const int c = w * cpw + j;
             uint32_t code = out.zero_code;
             if (c < C) {
-                const float y = __fmul_rn(scale, (float)red[0][j]);
-                if (y_out) y_out[nn * C + c] = y;
-                code = project_code(y, alpha_out, out);
+                const float y = __fmul_rn(scale, (float)acc[j]);
+                if (y_out) y_out[(int64_t)nn * C + c] = y;
+                if (codes_out) code = project_by_table(y, T, out);
             }
             word |= code << (out.b * j);
         }
-        if (codes_out && w < ldo) codes_out[nn * ldo + w] = word;
+    } else {
+        for (int j = 0; j < 32 / out.b; j++) word |= out.zero_code << (out.b * j);
     }
+    if (codes_out && w < ldo) codes_out[(int64_t)nn * ldo + w] = word;
 }
 
 cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int HW, int C, float scale,
@@ -326,8 +541,9 @@ cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
     ProjParams out = make_proj_params(bo, ko, so, rounding);
     int64_t words = (C + (32 / b) - 1) / (32 / b);
     if (codes_out && ldo > words) words = ldo;          // also write the row's padding words
-    dim3 grid((unsigned)words, (unsigned)n);
-    esb_avgpool_kernel<<<grid, 256, 0, st>>>(X, ldx, b, k, HW, C, scale, alpha_out, out, y_out, codes_out, ldo);
+    const int64_t total = (int64_t)n * words;
+    esb_avgpool_word_kernel<<<(unsigned)((total + 127) / 128), 128, 0, st>>>(X, ldx, b, k, n, HW, C, (int)words, scale,
+                                                                           alpha_out, out, y_out, codes_out, ldo);
     return cudaGetLastError();
 }
 

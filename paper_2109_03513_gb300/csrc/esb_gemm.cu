@@ -53,6 +53,11 @@ struct ConvSrc {
     int ldx;
     int rows;                     // n * P * Q
     int H, W, P, Q, S, stride, pad;
+    // Words of each pixel in the logical K (<= ldx): the words that hold
+    // channels, so a pixel row's padding words (e.g. the 3 of a first
+    // layer's 4-word rows) take no K.  The logical word w is word w % kw of
+    // tap w / kw.
+    int kw = 0;
     struct Row { int pix0; int h0, w0; bool valid; };
     struct Cursor { int r, s, word; };
     __device__ __forceinline__ Row row(int64_t m64) const
@@ -77,15 +82,15 @@ struct ConvSrc {
     }
     __device__ __forceinline__ const uint32_t* words(const Row& x, int64_t w) const
     {
-        const int tap = (int)(w / ldx);
-        const int word = (int)(w - (int64_t)tap * ldx);
+        const int tap = (int)(w / kw);
+        const int word = (int)(w - (int64_t)tap * kw);
         return tap_ptr(x, tap / S, tap - (tap / S) * S, word);
     }
     __device__ __forceinline__ Cursor cursor(int64_t w) const
     {
         Cursor c;
-        const int tap = (int)(w / ldx);
-        c.word = (int)(w - (int64_t)tap * ldx);
+        const int tap = (int)(w / kw);
+        c.word = (int)(w - (int64_t)tap * kw);
         c.r = tap / S;
         c.s = tap - c.r * S;
         return c;
@@ -93,11 +98,13 @@ struct ConvSrc {
     __device__ __forceinline__ void advance(Cursor& c, int dw) const
     {
         c.word += dw;
-        while (c.word >= ldx) {
-            c.word -= ldx;
+        while (c.word >= kw) {
+            c.word -= kw;
             if (++c.s == S) { c.s = 0; ++c.r; }
         }
     }
+    // 16-byte pieces (4 logical words) are contiguous in memory
+    __host__ __device__ __forceinline__ bool vec4() const { return (kw & 3) == 0; }
     __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const { return tap_ptr(x, c.r, c.s, c.word); }
     __host__ __device__ __forceinline__ bool linear() const { return true; }
     __device__ __forceinline__ const uint32_t* code_word(const Row& x, int64_t kk, int cpw, int& slot) const
@@ -128,7 +135,8 @@ template <class Src>
 __device__ __forceinline__ uint4 decode_unit(const Src& src, const typename Src::Row& row, int64_t k0, int64_t K,
                                              const OpFmt& f)
 {
-    if (f.b == 4 && f.planes == 1 && src.linear() && k0 + 16 <= K) return decode_unit_b4(src, row, src.cursor(k0 >> 3), f);
+    if (f.b == 4 && f.planes == 1 && src.linear() && src.vec4() && k0 + 16 <= K)
+        return decode_unit_b4(src, row, src.cursor(k0 >> 3), f);
     return decode_unit_any(src, row, k0, K, f);
 }
 
@@ -339,6 +347,10 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
     const int64_t my_tiles = (m_tiles > cta_in_n) ? (m_tiles - cta_in_n + ctas_per_n - 1) / ctas_per_n : 0;
     uint32_t tmem_cols = 32;
     while ((int)tmem_cols < 2 * BN) tmem_cols <<= 1;
+    // E4M3 tables of the word-walk decoder (widths other than 4)
+    __shared__ uint8_t luta[256], lutb[256];
+    if (fa.planes == 1) build_e4m3_lut(luta, fa, tid, kWsThreads);
+    if (fb.planes == 1 && fb.b != 4) build_e4m3_lut(lutb, fb, tid, kWsThreads);
     // Epilogue column split: both halves of BN must be whole 16-column chunks
     // and whole output words; otherwise warps 0-3 take every column.
     const int half_cols = BN / 2;
@@ -371,7 +383,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
     // (ws_setup).
     uint32_t tmem_base = 0;
     if (warp < kWsProdWarp0)
-        tmem_base = ws_setup<false>(srcB, n0, K, fb, BN, nkb, sB, thr, ep, tmem_slot, tid);
+        tmem_base = ws_setup<false>(srcB, n0, K, fb, BN, nkb, sB, thr, ep, tmem_slot, tid, lutb);
 
     if (warp >= kWsProdWarp0) {
         // ---------------------------------------------- A producers
@@ -403,7 +415,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
             }
             if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
             uint8_t* st = sA + s * kBM * kBK;
-            if (fa.b == 4 && fa.planes == 1) {
+            if (fa.b == 4 && fa.planes == 1 && srcA.linear() && srcA.vec4()) {
                 const int64_t kw0 = (int64_t)kb * 16;
                 typename SrcA::Cursor cur[4];
 #pragma unroll
@@ -413,6 +425,11 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
                 for (int q = 0; q < 4; q++) load_row_b4(srcA, rows[q], cur, kw0, K, zwa, v[q]);
 #pragma unroll
                 for (int q = 0; q < 4; q++) store_row_b4(st, lane + 32 * q, v[q], kw0, K, fa);
+            } else if (fa.planes == 1 && srcA.linear()) {
+                // other widths: one word walk per row of the K-block
+#pragma unroll 1
+                for (int q = 0; q < 4; q++)
+                    walk_row_kblock(srcA, rows[q], (int64_t)kb * kBK, K, fa, luta, st, lane + 32 * q);
             } else {
                 fill_stage_any(srcA, (cta_in_n + ti * ctas_per_n) * kBM, st, lane, (int64_t)kb * kBK, K, fa);
             }
@@ -644,6 +661,17 @@ static bool conv_force_im2col()
     return v != 0;
 }
 
+// Words of each pixel that enter the implicit GEMM's K: all ldx of them
+// (the halo kernel and the 16-byte decode read whole 4-word pieces) unless
+// at least half are padding (a first layer's 3 channels in a 4-word row),
+// then only the words that hold channels.
+static int conv_k_words(const esb_conv_desc& d, int64_t ldx, int bx)
+{
+    const int cpw = 32 / bx;
+    const int used = (d.c + cpw - 1) / cpw;
+    return (2 * used <= ldx) ? used : (int)ldx;
+}
+
 cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
                            const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st)
 {
@@ -652,16 +680,17 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
     ep.acc_lim = acc_fma_limit((int64_t)d.r * d.s * d.c, bx, kx, bw, kw);   // padding slots add exact zeros
     const int64_t M = (int64_t)d.n * P * Q;
     const int64_t N = d.cout;
-    const int64_t K = (int64_t)d.r * d.s * ldx * (32 / bx);
+    const int kwx = conv_k_words(d, ldx, bx);
+    const int64_t K = (int64_t)d.r * d.s * kwx * (32 / bx);
     const int BN = pick_bn(N, ep.out_cpw);
     ConvSrc a;
     a.X = X; a.ldx = (int)ldx; a.rows = (int)M; a.H = d.h; a.W = d.w; a.P = P; a.Q = Q; a.S = d.s;
-    a.stride = d.stride; a.pad = d.pad;
+    a.stride = d.stride; a.pad = d.pad; a.kw = kwx;
     RowsSrc b{W, (int64_t)d.r * d.s * ldw, N};
-    if (bw != bx || ldw != ldx) {
-        // filters of another code width: K runs over taps of the input's
-        // ldx * cpw_x codes; each tap of a filter row holds ldw words
-        b.kp = ldx * (32 / bx);
+    if (kwx != ldx || bw != bx || ldw != ldx) {
+        // K runs over taps of the input's kwx * cpw_x codes; each tap of a
+        // filter row holds ldw words (of its own code width)
+        b.kp = (int64_t)kwx * (32 / bx);
         b.ldt = ldw;
     }
     OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
@@ -678,10 +707,11 @@ int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx
                        int kw, int out_b)
 {
     const int cpw = 32 / out_b;
-    const int64_t K = (int64_t)d.r * d.s * ldx * (32 / bx);
+    const int kwd = conv_k_words(d, ldx, bx);
+    const int64_t K = (int64_t)d.r * d.s * kwd * (32 / bx);
     OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
     const int64_t Kx = plan_planes(fa, fb, K);
-    const bool same_layout = bw == bx && ldw == ldx && fa.planes == 1;
+    const bool same_layout = bw == bx && ldw == ldx && fa.planes == 1 && kwd == ldx;
     if (Kx > 0 && !conv_force_im2col() && same_layout && conv_halo_ok(d, P, Q, ldx, bx, kx, cpw))
         return ESB_CONV_KERNEL_HALO;
     cudaError_t e = cudaSuccess;

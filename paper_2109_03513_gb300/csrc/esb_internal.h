@@ -79,7 +79,8 @@ int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx
 cudaError_t launch_dwconv(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
                           const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st);
 cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int H, int Wd, int C, int win,
-                           int stride, int pad, int P, int Q, uint32_t* Y, int64_t ldy, cudaStream_t st);
+                           int stride, int pad, int P, int Q, uint32_t* Y, int64_t ldy, cudaStream_t st,
+                           int is_signed);
 cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int HW, int C, float scale,
                            float alpha_out, int bo, int ko, int so, int rounding, float* y_out, uint32_t* codes_out,
                            int64_t ldo, cudaStream_t st);
@@ -101,6 +102,10 @@ cudaError_t launch_dn_project(const float* x, int64_t rows, int64_t cols, const 
 cudaError_t launch_dn_grad(const float* g, const float* x, int64_t n, const double* stats, void* workspace, float* gx,
                            cudaStream_t st);
 cudaError_t launch_ema(const double* batch, double* running, double gamma, cudaStream_t st);
+
+// Tensor-pipe peak microbenchmarks (esb_peak.cu): kind 0 tcgen05 f8f6f4,
+// kind 1 mma.sync s8; *flops receives the operations of the launch.
+cudaError_t launch_peak(int kind, int64_t iters, int64_t* flops, cudaStream_t st);
 
 // alpha*(b,k) and 2*D(alpha*) (Sec. III-D), solved on the host in fp64.
 double alpha_star_solve(int b, int k, double* dda);

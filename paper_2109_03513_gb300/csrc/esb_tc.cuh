@@ -144,6 +144,7 @@ struct RowsSrc {
     struct Row { const uint32_t* p; };
     struct Cursor { int64_t w; };
     __host__ __device__ __forceinline__ bool linear() const { return kp == 0; }
+    __host__ __device__ __forceinline__ bool vec4() const { return true; }
     __device__ __forceinline__ Row row(int64_t r) const { Row x; x.p = (r < rows) ? base + r * ld : nullptr; return x; }
     __device__ __forceinline__ const uint32_t* words(const Row& x, int64_t w) const { return x.p ? x.p + w : nullptr; }
     // Word holding code kk of row x (nullptr: the zero code) and its slot.
@@ -202,6 +203,51 @@ __device__ __noinline__ uint4 decode_unit_any(const Src& src, const typename Src
 }
 
 __device__ __forceinline__ uint32_t swz(int r, int g) { return (uint32_t)(r * 128 + ((g ^ (r & 7)) << 4)); }
+
+// The E4M3 byte of each of the 2^b codes of a whole-byte format (planes ==
+// 1), built by threads t = 0 .. nt-1: the table of the word-walk decoder.
+__device__ __forceinline__ void build_e4m3_lut(uint8_t* lut, const OpFmt& f, int t, int nt)
+{
+    for (int c = t; c < (1 << f.b); c += nt) lut[c] = (uint8_t)code_to_e4m3((uint32_t)c, f);
+}
+
+// Codes [k0, k0 + 128) of one row (a K-block) decoded by walking its words
+// once (a code never straddles two words): eight 16-code units of E4M3
+// bytes, in unit_pos order, stored to the swizzled stage row r.  For code
+// widths other than 4 on linear sources with one plane; codes past K and
+// words outside the operand (rows past M or N, out-of-image taps) give the
+// E4M3 zero.
+template <class Src>
+__device__ __forceinline__ void walk_row_kblock(const Src& src, const typename Src::Row& row, int64_t k0, int64_t K,
+                                                const OpFmt& f, const uint8_t* lut, uint8_t* stage, int r)
+{
+    const int cpw = f.cpw;
+    const int64_t wi = k0 / cpw;
+    int slot = (int)(k0 - wi * cpw);
+    typename Src::Cursor cur = src.cursor(wi);
+    const uint32_t* p = (k0 < K) ? src.at(row, cur) : nullptr;
+    uint32_t w = p ? __ldg(p) : 0u;
+    bool valid = p != nullptr;
+#pragma unroll 1
+    for (int g = 0; g < 8; g++) {
+        uint32_t o[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 16; j++) {
+            const int64_t kk = k0 + g * 16 + j;
+            const uint32_t byte = (valid && kk < K) ? (uint32_t)lut[(w >> (f.b * slot)) & f.mask] : 0u;
+            const int pos = unit_pos(j);
+            o[pos >> 2] |= byte << (8 * (pos & 3));
+            if (++slot == cpw) {
+                slot = 0;
+                src.advance(cur, 1);
+                p = (kk + 1 < K) ? src.at(row, cur) : nullptr;
+                valid = p != nullptr;
+                w = valid ? __ldg(p) : 0u;
+            }
+        }
+        *reinterpret_cast<uint4*>(stage + swz(r, g)) = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
 
 // ------------------------------------------------------------ epilogue
 
@@ -484,7 +530,7 @@ __device__ __forceinline__ void ws_alloc(int warp, uint32_t* tmem_slot, uint32_t
 // (fence_proxy_async_smem) and synchronises before the MMA reads sB.
 template <bool B4>
 __device__ __forceinline__ void ws_decode_b(const RowsSrc& srcB, int64_t n0, int64_t K, const OpFmt& fb, int BN,
-                                            int nkb, uint8_t* sB, int t, int nthreads)
+                                            int nkb, uint8_t* sB, int t, int nthreads, const uint8_t* lutb = nullptr)
 {
     if (B4 || (fb.b == 4 && fb.planes == 1 && srcB.linear())) {
         // one row chunk per thread and pass (compact: this code runs cold,
@@ -502,6 +548,13 @@ __device__ __forceinline__ void ws_decode_b(const RowsSrc& srcB, int64_t n0, int
             uint4 v[4];
             load_row_b4(srcB, row, cur, kw0, K, zw, v);
             store_row_b4(sB + kb * BN * kBK, r, v, kw0, K, fb);
+        }
+    } else if (lutb && fb.planes == 1 && srcB.linear()) {
+        // other widths: one word walk per (K-block, row)
+#pragma unroll 1
+        for (int pr = t; pr < nkb * BN; pr += nthreads) {
+            const int kb = pr / BN, r = pr - kb * BN;
+            walk_row_kblock(srcB, srcB.row(n0 + r), (int64_t)kb * kBK, K, fb, lutb, sB + kb * BN * kBK, r);
         }
     } else {
         for (int u = t; u < nkb * BN * 8; u += nthreads) {
@@ -534,12 +587,12 @@ __device__ __forceinline__ void ws_thresholds(float* thr, const EpiParams& ep, i
 template <bool B4>
 __device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, int64_t K, const OpFmt& fb, int BN,
                                              int nkb, uint8_t* sB, float* thr, const EpiParams& ep,
-                                             uint32_t* tmem_slot, int tid)
+                                             uint32_t* tmem_slot, int tid, const uint8_t* lutb = nullptr)
 {
     constexpr int kSetupThreads = kWsProdWarp0 * 32;
     const int warp = tid >> 5, lane = tid & 31;
     griddep_wait();                                   // B and the alphas may come from the previous launch
-    ws_decode_b<B4>(srcB, n0, K, fb, BN, nkb, sB, tid, kSetupThreads);
+    ws_decode_b<B4>(srcB, n0, K, fb, BN, nkb, sB, tid, kSetupThreads, lutb);
     fence_proxy_async_smem();
     if (warp == kWsMmaWarp) {
         asm volatile("bar.sync 1, %0;" ::"n"(kSetupThreads) : "memory");

@@ -115,6 +115,7 @@ SIGNATURES = {
     "esb_avgpool_nhwc": (_I32, [_P, _I64, esb_format, _I32, _I32, _I32, _F32, _F32, esb_format, _I32, _P, _P, _I64,
                                 _P]),
     "esb_get_status": (_I32, [_P, _P]),
+    "esb_peak_launch": (_I32, [_I32, _I64, _P, _P]),
 }
 
 
@@ -563,6 +564,17 @@ def esb_avgpool_nhwc(X: torch.Tensor, f: Fmt, n: int, hw: int, c: int, scale: fl
     _check(lib().esb_avgpool_nhwc(_ptr(X), ldx, f.c(), n, hw, c, scale, alpha_out, fmt_out.c(), rounding, _ptr(y),
                                   _ptr(codes), ldo, _stream(stream)), "esb_avgpool_nhwc")
     return y, codes
+
+
+ESB_PEAK_TCGEN05_F8F6F4 = 0
+ESB_PEAK_MMA_SYNC_S8 = 1
+
+
+def esb_peak_launch(kind: int, iters: int, stream=None) -> int:
+    """Launch a tensor-pipe peak microbenchmark; returns its operation count."""
+    ops = ctypes.c_int64(0)
+    _check(lib().esb_peak_launch(kind, iters, ctypes.byref(ops), _stream(stream)), "esb_peak_launch")
+    return int(ops.value)
 
 
 def esb_get_status(stream=None) -> int:

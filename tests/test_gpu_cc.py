@@ -82,6 +82,19 @@ def test_maxpool_matches_oracle(n, h, w, c, win, stride, pad, fmt):
     assert np.array_equal(u32(Y), exp)
 
 
+@pytest.mark.parametrize("n,h,w,c,win,stride,pad,k", [(2, 112, 112, 64, 3, 2, 1, 2), (2, 7, 6, 9, 3, 2, 1, 2),
+                                                      (1, 11, 13, 21, 3, 2, 1, 1), (1, 9, 8, 16, 2, 2, 0, 0),
+                                                      (1, 6, 7, 5, 3, 1, 1, 3)])
+def test_maxpool_unsigned_4bit_matches_oracle(n, h, w, c, win, stride, pad, k):
+    # the decode-free path: unsigned 4-bit codes (post-ReLU activations),
+    # window maxima taken on the rotated code ranks
+    codes = synth.uniform_ints((n * h * w, c), 0, 8, seed=h * c + k)
+    X = o.pack(codes, 4, k, ld_words=esb.esb_row_words(c, 4))
+    Y = esb.esb_maxpool_nhwc(dev_i32(X), esb.Fmt(4, k, False), n, h, w, c, win, stride, pad)
+    exp = o.maxpool_codes(X.reshape(n, h, w, -1), 4, k, n, h, w, c, win, stride, pad).reshape(Y.shape[0], -1)
+    assert np.array_equal(u32(Y), exp)
+
+
 @pytest.mark.parametrize("n,hw,c,fmt", [(4, 49, 512, (4, 2)), (3, 49, 1280, (4, 2)), (2, 16, 37, (6, 3)),
                                         (2, 1, 5, (3, 1))])
 def test_avgpool_matches_oracle(n, hw, c, fmt):

@@ -226,6 +226,37 @@ def test_mobilenetv2_blocks_match_oracle():
     assert esb.esb_get_status() == 0
 
 
+# MobileNetV2 (width 1.0) inverted-residual settings: expansion t, output
+# channels c, repeats n, first stride s
+MBV2 = [(1, 16, 1, 1), (6, 24, 2, 2), (6, 32, 3, 2), (6, 64, 4, 2), (6, 96, 3, 1), (6, 160, 3, 2), (6, 320, 1, 1)]
+
+
+def test_mobilenetv2_forward_matches_oracle():
+    # the whole MobileNetV2 at 224 x 224, batch 1: 3x3/2 stem, all 17
+    # bottlenecks (1x1 expand, depthwise 3x3, 1x1 linear projection, residual
+    # where stride 1 and widths match), the 320 -> 1280 1x1 conv, global
+    # average pool and the 1280 -> 1000 classifier, every layer checked
+    net = Net((4, 2), seed=21)
+    r6 = esb.ESB_ACT_RELU6
+    x = net.input(1, 224, 224, 3)
+    x = net.conv(x, 32, 3, 3, 2, 1, act=r6)
+    blocks = 0
+    for t, c, n, s in MBV2:
+        for i in range(n):
+            stride = s if i == 0 else 1
+            h = x if t == 1 else net.conv(x, x.c * t, 1, 1, 1, 0, act=r6)
+            h = net.conv(h, h.c, 3, 3, stride, 1, act=r6, groups=h.c)
+            res = x if (stride == 1 and x.c == c) else None
+            x = net.conv(h, c, 1, 1, 1, 0, act=esb.ESB_ACT_NONE, res=res)
+            blocks += 1
+    assert blocks == 17 and (x.h, x.w, x.c) == (7, 7, 320)
+    x = net.conv(x, 1280, 1, 1, 1, 0, act=r6)
+    x = net.avgpool(x)
+    net.fc(x, 1000)
+    assert net.layers == 1 + 17 * 3 - 1 + 1 + 1
+    assert esb.esb_get_status() == 0
+
+
 def test_alexnet_classifier_matches_oracle(monkeypatch):
     # AlexNet's classifier 9216 -> 4096 -> 4096 -> 1000 (ReLU between), batch
     # 8, through the tiled large-operand GEMM (workspace; every shape to it)
