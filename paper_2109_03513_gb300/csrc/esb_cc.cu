@@ -148,18 +148,16 @@ esb_dwconv_kernel(const uint32_t* __restrict__ X, int64_t ldx, int bx, int kx,
 // channels once into shared memory (integer images, [tap][channel]) and
 // builds the table of input images and the requantisation thresholds, then
 // walks its share of the work units: one unit = one code word (CPW
-// channels) of QT consecutive output pixels of one row.  Each input word of
-// the unit's 3 x ((QT-1) STRIDE + 3) window is decoded once and feeds every
-// output of the strip that reads it; all loop bounds are compile-time
-// constants, so accumulators stay in registers.
+// channels) of QT consecutive output pixels of one row, accumulated in
+// registers.  The taps run in rolled loops so that the kernel's code stays
+// small (fully unrolled strips measured instruction-fetch bound).
 template <int B, int STRIDE>
 __global__ void __launch_bounds__(128)
 esb_dwconv3_kernel(const uint32_t* __restrict__ X, int64_t ldx, int kx, const uint32_t* __restrict__ W, int64_t ldw,
                    int kw, int n, int H, int Wd, int C, int pad, int P, int Q, int QS, CcEpi ep)
 {
     constexpr int CPW = 32 / B;
-    constexpr int QT = STRIDE == 1 ? 8 : 4;
-    constexpr int NCOL = (QT - 1) * STRIDE + 3;
+    constexpr int QT = 4;
     constexpr uint32_t MASK = (1u << B) - 1u;
     extern __shared__ int32_t wtab[];                 // [9][words * CPW] filter images
     __shared__ int32_t lutx[1 << B];
@@ -213,31 +211,26 @@ esb_dwconv3_kernel(const uint32_t* __restrict__ X, int64_t ldx, int kx, const ui
         for (int u = 0; u < QT; u++)
 #pragma unroll
             for (int j = 0; j < CPW; j++) acc[u][j] = 0;
-#pragma unroll
+        // taps in rolled loops (compact code: the instruction cache holds
+        // it), the strip's outputs unrolled; each input word is re-read
+        // from L1 by the up to 3 taps that share it
+#pragma unroll 1
         for (int r = 0; r < 3; r++) {
             const int h = p * STRIDE - pad + r;
             if (h < 0 || h >= H) continue;
-            int32_t wf[3][CPW];
-#pragma unroll
-            for (int s2 = 0; s2 < 3; s2++)
-#pragma unroll
-                for (int j = 0; j < CPW; j++) wf[s2][j] = wtab[(r * 3 + s2) * cp + w * CPW + j];
             const uint32_t* xrow = X + ((int64_t)nn * H + h) * Wd * ldx + w;
+#pragma unroll 1
+            for (int s2 = 0; s2 < 3; s2++) {
+                int32_t wf[CPW];
 #pragma unroll
-            for (int i = 0; i < NCOL; i++) {
-                const int col = q0 * STRIDE - pad + i;
-                if (col < 0 || col >= Wd) continue;
-                const uint32_t xw = __ldg(xrow + (int64_t)col * ldx);
-                int32_t xi[CPW];
-#pragma unroll
-                for (int j = 0; j < CPW; j++) xi[j] = lutx[(xw >> (B * j)) & MASK];
+                for (int j = 0; j < CPW; j++) wf[j] = wtab[(r * 3 + s2) * cp + w * CPW + j];
 #pragma unroll
                 for (int u = 0; u < QT; u++) {
-                    const int s2 = i - u * STRIDE;
-                    if (s2 >= 0 && s2 < 3) {
+                    const int col = (q0 + u) * STRIDE - pad + s2;
+                    if (col < 0 || col >= Wd) continue;
+                    const uint32_t xw = __ldg(xrow + (int64_t)col * ldx);
 #pragma unroll
-                        for (int j = 0; j < CPW; j++) acc[u][j] += xi[j] * wf[s2][j];
-                    }
+                    for (int j = 0; j < CPW; j++) acc[u][j] += lutx[(xw >> (B * j)) & MASK] * wf[j];
                 }
             }
         }
@@ -278,7 +271,7 @@ template <int B, int STRIDE>
 static cudaError_t launch_dw3(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int kx,
                               const uint32_t* W, int64_t ldw, int kw, const CcEpi& ep, cudaStream_t st)
 {
-    constexpr int QT = STRIDE == 1 ? 8 : 4;
+    constexpr int QT = 4;
     const int QS = (Q + QT - 1) / QT;
     const int64_t total = (int64_t)d.n * P * QS * ep.ldo;
     int64_t blocks = (total + 127) / 128;

@@ -177,6 +177,13 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
         const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
         build_thresholds(thr, ep.out, alpha_out, warp, lane, 0, kGemmThreads / 32);
     }
+    // word walks (one row per thread) for widths whose 16-code units are not
+    // 16-byte pieces: 3/5/6-bit codes, 4-bit rows whose words are not contiguous
+    __shared__ uint8_t luta[256], lutb[256];
+    const bool walk_a = fa.planes == 1 && srcA.linear() && !(fa.b == 4 && srcA.vec4());
+    const bool walk_b = fb.planes == 1 && srcB.linear() && !(fb.b == 4 && srcB.vec4());
+    if (walk_a) build_e4m3_lut(luta, fa, tid, kGemmThreads);
+    if (walk_b) build_e4m3_lut(lutb, fb, tid, kGemmThreads);
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_d = *tmem_slot;
@@ -199,15 +206,25 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
         uint8_t* sa = smem + s * stage_bytes;
         uint8_t* sb = sa + a_bytes;
         const int64_t kbase = kb * kBK;
+        if (walk_a) {
+            if (tid < kBM) walk_row_kblock(srcA, srcA.row(m0 + tid), kbase, K, fa, luta, sa, tid);
+        } else {
 #pragma unroll
-        for (int i = 0; i < kAUnits; i++) {
-            const int u = tid + i * kGemmThreads;
-            const int r = u >> 3, g = u & 7;
-            *reinterpret_cast<uint4*>(sa + swz(r, g)) = decode_unit(srcA, arow[i], kbase + g * 16, K, fa);
+            for (int i = 0; i < kAUnits; i++) {
+                const int u = tid + i * kGemmThreads;
+                const int r = u >> 3, g = u & 7;
+                *reinterpret_cast<uint4*>(sa + swz(r, g)) = decode_unit(srcA, arow[i], kbase + g * 16, K, fa);
+            }
         }
-        for (int u = tid; u < BN * 8; u += kGemmThreads) {
-            const int r = u >> 3, g = u & 7;
-            *reinterpret_cast<uint4*>(sb + swz(r, g)) = decode_unit(srcB, srcB.row(n0 + r), kbase + g * 16, K, fb);
+        if (walk_b) {
+            // rows rotated by kBM so that the threads past the A rows start
+            for (int r = (tid + kGemmThreads - kBM) % kGemmThreads; r < BN; r += kGemmThreads)
+                walk_row_kblock(srcB, srcB.row(n0 + r), kbase, K, fb, lutb, sb, r);
+        } else {
+            for (int u = tid; u < BN * 8; u += kGemmThreads) {
+                const int r = u >> 3, g = u & 7;
+                *reinterpret_cast<uint4*>(sb + swz(r, g)) = decode_unit(srcB, srcB.row(n0 + r), kbase + g * 16, K, fb);
+            }
         }
         fence_proxy_async_smem();
         __syncthreads();
@@ -270,6 +287,16 @@ esb_gemm_tc_kernel(SrcA srcA, SrcB srcB, int64_t M, int64_t N, int64_t K, OpFmt 
                     uint32_t word = 0;
                     for (int t = 0; t < cpw; t++) word |= (uint32_t)stage_codes[rr * BN + j * cpw + t] << (ep.out.b * t);
                     ep.codes_out[mm * ep.ldo + wg] = word;
+                }
+            }
+            if (n0 + BN >= N) {                      // the last N-tile fills the rows' padding words
+                uint32_t zw = 0u;
+                for (int t = 0; t < cpw; t++) zw |= ep.out.zero_code << (ep.out.b * t);
+                const int64_t w_end = (n0 + BN) / cpw;
+                for (int rr = tid; rr < kBM; rr += kGemmThreads) {
+                    const int64_t mm = m0 + rr;
+                    if (mm < M)
+                        for (int64_t wq = w_end; wq < ep.ldo; wq++) ep.codes_out[mm * ep.ldo + wq] = zw;
                 }
             }
         }
@@ -492,18 +519,46 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
 int pick_bn(int64_t N, int out_cpw)
 {
     // BN must be a multiple of 16 (MMA N step) and of the output codes per
-    // word (so no packed word straddles two tiles).
-    static const int cands_small[] = {64, 48, 80, 96, 32, 112, 128, 16};
-    static const int cands_big[] = {128, 160, 192, 240, 256, 96, 80, 112, 64, 48, 144, 176, 208, 224};
-    if (N <= 64) {
-        for (int bn : cands_small)
+    // word (so no packed word straddles two tiles).  Up to 256 columns: the
+    // smallest such width that covers N (no wasted MMA columns or epilogue
+    // lanes for narrow layers); wider: the width in [128, 256] that wastes
+    // the fewest columns over the N-tiles, the wider on a tie.
+    int best = 0;
+    if (N <= 256) {
+        for (int bn = 16; bn <= 256; bn += 16)
             if (bn >= N && bn % out_cpw == 0) return bn;
     }
-    for (int bn : cands_big)
-        if (bn % out_cpw == 0) return bn;
+    int64_t waste_best = -1;
+    for (int bn = 256; bn >= 128; bn -= 16) {
+        if (bn % out_cpw) continue;
+        const int64_t waste = ((N + bn - 1) / bn) * bn - N;
+        if (waste_best < 0 || waste < waste_best) { waste_best = waste; best = bn; }
+    }
+    if (best) return best;
     for (int bn = 16; bn <= 256; bn += 16)
         if (bn % out_cpw == 0) return bn;
     return 0;
+}
+
+// N-tile width of the streamed kernel.  Each of its CTAs decodes 128 A rows
+// and BN B rows for every K-block, so a tile costs about 128 + BN row
+// decodes; when M gives few row tiles, narrower N-tiles spread that work
+// over more SMs.  The width (a multiple of 16 and of the output codes per
+// word, at most bn0 = pick_bn's choice, at least 64) that minimises
+// waves x (128 + BN), one CTA per SM; the wider on a tie.
+static int streamed_bn(int64_t M, int64_t N, int out_cpw, int bn0)
+{
+    const int64_t sms = device_sm_count();
+    const int64_t mt = (M + kBM - 1) / kBM;
+    int best = bn0;
+    int64_t cbest = ((mt * ((N + bn0 - 1) / bn0) + sms - 1) / sms) * (128 + bn0);
+    for (int bn = bn0 - 16; bn >= 64; bn -= 16) {
+        if (bn % out_cpw) continue;
+        const int64_t waves = (mt * ((N + bn - 1) / bn) + sms - 1) / sms;
+        const int64_t c = waves * (128 + bn);
+        if (c < cbest) { cbest = c; best = bn; }
+    }
+    return best;
 }
 
 static size_t gemm_smem_bytes(int BN)
@@ -529,6 +584,7 @@ template <class SrcA, class SrcB>
 static cudaError_t launch_tc(const SrcA& a, const SrcB& b, int64_t M, int64_t N, int64_t K, const OpFmt& fa,
                              const OpFmt& fb, int BN, const EpiParams& ep, cudaStream_t st)
 {
+    BN = streamed_bn(M, N, ep.out_cpw, BN);
     const size_t smem = gemm_smem_bytes(BN);
     static bool configured = false;
     if (!configured) {
@@ -641,7 +697,8 @@ cudaError_t launch_gemm(int64_t M, int64_t N, int64_t K, const uint32_t* A, int6
     RowsSrc a{A, lda, M};
     RowsSrc b{B, ldb, N};
     OpFmt fa = make_opfmt(ba, ka), fb = make_opfmt(bb, kb);
-    const int64_t Kx = plan_planes(fa, fb, K);        // the kernels' K (significand planes)
+    int64_t Kx = plan_planes(fa, fb, K);              // the kernels' K (significand planes)
+    if (const int64_t Ks = plan_slots(fa, fb, K, (K + fa.cpw - 1) / fa.cpw)) Kx = Ks;
     if (Kx > 0) {
         cudaError_t e = cudaSuccess;
         if (launch_ws(a, b, M, N, Kx, fa, fb, BN, ep, st, &e)) return e;
@@ -694,7 +751,11 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
         b.ldt = ldw;
     }
     OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
-    const int64_t Kx = plan_planes(fa, fb, K);        // the kernels' K (significand planes)
+    int64_t Kx = plan_planes(fa, fb, K);              // the kernels' K (significand planes)
+    if (b.linear()) {
+        const int64_t words = (int64_t)d.r * d.s * kwx;
+        if (const int64_t Ks = plan_slots(fa, fb, words * fa.cpw, words)) Kx = Ks;
+    }
     cudaError_t e = cudaSuccess;
     if (Kx > 0 && !conv_force_im2col() && fa.planes == 1 && b.linear() &&
         launch_conv_halo(d, P, Q, X, ldx, fa, W, ldw, fb, BN, ep, st, &e))
@@ -710,8 +771,12 @@ int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx
     const int kwd = conv_k_words(d, ldx, bx);
     const int64_t K = (int64_t)d.r * d.s * kwd * (32 / bx);
     OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
-    const int64_t Kx = plan_planes(fa, fb, K);
+    int64_t Kx = plan_planes(fa, fb, K);
     const bool same_layout = bw == bx && ldw == ldx && fa.planes == 1 && kwd == ldx;
+    if (same_layout) {                                // the filter rows are linear (launch_conv_tc)
+        const int64_t words = (int64_t)d.r * d.s * kwd;
+        if (const int64_t Ks = plan_slots(fa, fb, words * fa.cpw, words)) Kx = Ks;
+    }
     if (Kx > 0 && !conv_force_im2col() && same_layout && conv_halo_ok(d, P, Q, ldx, bx, kx, cpw))
         return ESB_CONV_KERNEL_HALO;
     cudaError_t e = cudaSuccess;

@@ -39,6 +39,7 @@ struct OpFmt {
     uint32_t pmap;       // role of plane i in bits 2i, 2i+1
     int csc;             // operand scale: decoded values are I 2^-csc
     int64_t korig;       // codes per row before the expansion (K tail)
+    int spw;             // word-slot layout: kernel-K slots per packed word (0: code-linear K)
 };
 
 // Significand split needed: the image is not an E4M3 number times a power of two.
@@ -52,8 +53,29 @@ __host__ inline OpFmt make_opfmt(int b, int k)
 {
     OpFmt o;
     o.b = b; o.k = k; o.ew = b - k - 1; o.cpw = 32 / b; o.mask = (1u << b) - 1u;
-    o.planes = 1; o.pmap = 0u; o.csc = k + 6; o.korig = 0;
+    o.planes = 1; o.pmap = 0u; o.csc = k + 6; o.korig = 0; o.spw = 0;
     return o;
+}
+
+// Word-slot layout of the kernels' K for a pair of whole-byte operands of
+// widths other than 4 with the same codes per word: packed word w of a row
+// takes the spw slots [w spw, (w + 1) spw) of K (spw = cpw rounded up to a
+// power of two: 16 for 3-bit, 8 for 5/6-bit, 4 for 7/8-bit, 16 for 2-bit),
+// its codes the first cpw of them and the E4M3 zero the rest.  A K-block
+// (128 slots) is then a whole number of words and every code has a fixed
+// byte, so a row decodes word by word without a running code offset.  Both
+// operands use the same slots, so the sums are those of the code-linear K.
+// korig: codes per row (the contraction length; codes of the last word past
+// it count as zero); words: packed words per row that enter K.  Returns the
+// kernels' K, or 0 when the pair keeps the code-linear layout (4-bit,
+// significand planes, different codes per word).
+__host__ inline int64_t plan_slots(OpFmt& fa, OpFmt& fb, int64_t korig, int64_t words)
+{
+    if (fa.planes != 1 || fb.planes != 1 || fa.cpw != fb.cpw || fa.b == 4 || fb.b == 4) return 0;
+    const int spw = fa.cpw > 8 ? 16 : (fa.cpw > 4 ? 8 : 4);
+    fa.spw = fb.spw = spw;
+    fa.korig = fb.korig = korig;
+    return words * spw;
 }
 
 // The plane layout of a pair of operands (see OpFmt) for a contraction of
@@ -173,6 +195,25 @@ __device__ __noinline__ uint4 decode_unit_any(const Src& src, const typename Src
                                               const OpFmt f)
 {
     uint32_t o0 = 0u, o1 = 0u, o2 = 0u, o3 = 0u;
+    if (f.spw) {                                      // word-slot layout: slot j of word k0 / spw + j / spw
+#pragma unroll 1
+        for (int j = 0; j < 16; j++) {
+            const int sl = j % f.spw;
+            const int64_t kk = (k0 / f.spw + j / f.spw) * f.cpw + sl;
+            if (sl >= f.cpw || kk >= f.korig) continue;
+            int slot = 0;
+            const uint32_t* p = src.code_word(row, kk, f.cpw, slot);
+            if (!p) continue;
+            const uint32_t v = code_to_e4m3((__ldg(p) >> (f.b * slot)) & f.mask, f) << (8 * (j & 3));
+            switch (j >> 2) {
+            case 0: o0 |= v; break;
+            case 1: o1 |= v; break;
+            case 2: o2 |= v; break;
+            default: o3 |= v; break;
+            }
+        }
+        return make_uint4(o0, o1, o2, o3);
+    }
     uint32_t role = 0u;
     if (f.planes > 1) {                               // unit k0 / 16 = plane of code unit (k0 / 16) / planes
         const int64_t u = k0 >> 4;
@@ -204,6 +245,15 @@ __device__ __noinline__ uint4 decode_unit_any(const Src& src, const typename Src
 
 __device__ __forceinline__ uint32_t swz(int r, int g) { return (uint32_t)(r * 128 + ((g ^ (r & 7)) << 4)); }
 
+// Byte masks of the decoded lo/hi words of one b = 4 word when only its
+// first v codes (0..8) are inside K.
+__device__ __forceinline__ void tail_masks(int v, uint32_t& mlo, uint32_t& mhi)
+{
+    const int nlo = (v + 1) >> 1, nhi = v >> 1;       // lo holds codes 0,2,4,6; hi 1,3,5,7
+    mlo = nlo >= 4 ? 0xffffffffu : ((1u << (8 * nlo)) - 1u);
+    mhi = nhi >= 4 ? 0xffffffffu : ((1u << (8 * nhi)) - 1u);
+}
+
 // The E4M3 byte of each of the 2^b codes of a whole-byte format (planes ==
 // 1), built by threads t = 0 .. nt-1: the table of the word-walk decoder.
 __device__ __forceinline__ void build_e4m3_lut(uint8_t* lut, const OpFmt& f, int t, int nt)
@@ -211,16 +261,115 @@ __device__ __forceinline__ void build_e4m3_lut(uint8_t* lut, const OpFmt& f, int
     for (int c = t; c < (1 << f.b); c += nt) lut[c] = (uint8_t)code_to_e4m3((uint32_t)c, f);
 }
 
-// Codes [k0, k0 + 128) of one row (a K-block) decoded by walking its words
-// once (a code never straddles two words): eight 16-code units of E4M3
-// bytes, in unit_pos order, stored to the swizzled stage row r.  For code
-// widths other than 4 on linear sources with one plane; codes past K and
-// words outside the operand (rows past M or N, out-of-image taps) give the
-// E4M3 zero.
+// One K-block of a row in the word-slot layout (see plan_slots) for B-bit
+// codes: the block's words are loaded 16 at a time (independent loads in
+// flight), then each word's codes go through the E4M3 table to their fixed
+// bytes.  Words past the row's K words, outside the operand or outside the
+// image, and codes past korig, give the E4M3 zero.
+template <int B, class Src>
+__device__ __forceinline__ void walk_row_slots(const Src& src, const typename Src::Row& row, int64_t k0,
+                                               const OpFmt& f, const uint8_t* lut, uint8_t* stage, int r)
+{
+    constexpr int CPW = 32 / B;
+    constexpr int SPW = CPW > 8 ? 16 : (CPW > 4 ? 8 : 4);
+    constexpr int NW = kBK / SPW;                     // words per K-block: 8, 16 or 32
+    constexpr int CH = NW > 16 ? 16 : NW;             // words per chunk
+    constexpr uint32_t MASK = (1u << B) - 1u;
+    const int64_t w0 = k0 / SPW;
+    typename Src::Cursor cur = src.cursor(w0);
+#pragma unroll 1
+    for (int c0 = 0; c0 < NW; c0 += CH) {
+        const int64_t left = f.korig - (w0 + c0) * CPW;   // codes of this chunk's words inside K
+        const int lim = left < 0 ? 0 : (left > CH * CPW ? CH * CPW : (int)left);
+        uint32_t wv[CH];
+        uint32_t ok = 0u;
+#pragma unroll
+        for (int i = 0; i < CH; i++) {
+            const uint32_t* p = (i * CPW < lim) ? src.at(row, cur) : nullptr;
+            wv[i] = p ? __ldg(p) : 0u;
+            ok |= (p ? 1u : 0u) << i;
+            src.advance(cur, 1);
+        }
+        uint32_t o[CH * SPW / 4];
+#pragma unroll
+        for (int i = 0; i < CH; i++) {
+#pragma unroll
+            for (int q = 0; q < SPW / 4; q++) {
+                uint32_t v = 0u;
+#pragma unroll
+                for (int t = 0; t < 4; t++) {
+                    const int j = q * 4 + t;
+                    if (j < CPW) {
+                        const uint32_t byte = lut[(wv[i] >> (B * j)) & MASK];
+                        v |= ((i * CPW + j < lim) ? byte : 0u) << (8 * t);
+                    }
+                }
+                o[i * (SPW / 4) + q] = ((ok >> i) & 1u) ? v : 0u;
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < CH * SPW / 16; g++)
+            *reinterpret_cast<uint4*>(stage + swz(r, c0 * SPW / 16 + g)) =
+                make_uint4(o[4 * g], o[4 * g + 1], o[4 * g + 2], o[4 * g + 3]);
+    }
+}
+
+// K-block [k0, k0 + 128) of one row decoded by walking its words once (a
+// code never straddles two words): eight 16-code units of E4M3 bytes stored
+// to the swizzled stage row r, in the word-slot layout when f.spw is set,
+// else code-linear in unit_pos order.  For linear sources with one plane;
+// codes past K and words outside the operand (rows past M or N,
+// out-of-image taps) give the E4M3 zero.
 template <class Src>
 __device__ __forceinline__ void walk_row_kblock(const Src& src, const typename Src::Row& row, int64_t k0, int64_t K,
                                                 const OpFmt& f, const uint8_t* lut, uint8_t* stage, int r)
 {
+    if (f.spw) {
+        switch (f.b) {
+        case 2: walk_row_slots<2>(src, row, k0, f, lut, stage, r); return;
+        case 3: walk_row_slots<3>(src, row, k0, f, lut, stage, r); return;
+        case 5: walk_row_slots<5>(src, row, k0, f, lut, stage, r); return;
+        case 6: walk_row_slots<6>(src, row, k0, f, lut, stage, r); return;
+        case 7: walk_row_slots<7>(src, row, k0, f, lut, stage, r); return;
+        default: walk_row_slots<8>(src, row, k0, f, lut, stage, r); return;
+        }
+    }
+    if (f.b == 4) {
+        // 4-bit codes: each 16-code unit is two words (consecutive logical
+        // words may lie in different pixels).  The block's 16 words are
+        // loaded first (independent loads in flight), then decoded 8 codes
+        // at a time.
+        typename Src::Cursor cur = src.cursor(k0 >> 3);
+        uint32_t wv[16];
+        uint32_t ok = 0u;
+#pragma unroll
+        for (int i = 0; i < 16; i++) {
+            const uint32_t* p = (k0 + i * 8 < K) ? src.at(row, cur) : nullptr;
+            wv[i] = p ? __ldg(p) : 0u;
+            ok |= (p ? 1u : 0u) << i;
+            src.advance(cur, 1);
+        }
+#pragma unroll
+        for (int g = 0; g < 8; g++) {
+            uint32_t o[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                const int i = 2 * g + h;
+                if ((ok >> i) & 1u) {
+                    decode_word_b4(wv[i], f.k, f.ew, o[2 * h], o[2 * h + 1]);
+                    const int64_t kk = k0 + i * 8;
+                    if (kk + 8 > K) {                 // K tail: zero the codes past K
+                        uint32_t ml, mh;
+                        tail_masks((int)(K - kk), ml, mh);
+                        o[2 * h] &= ml;
+                        o[2 * h + 1] &= mh;
+                    }
+                }
+            }
+            *reinterpret_cast<uint4*>(stage + swz(r, g)) = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+        return;
+    }
     const int cpw = f.cpw;
     const int64_t wi = k0 / cpw;
     int slot = (int)(k0 - wi * cpw);
@@ -360,14 +509,6 @@ constexpr int kWsProdWarps = 7;
 constexpr int kWsThreads = (kWsProdWarp0 + kWsProdWarps) * 32;   // 512: 4 warps per SM sub-partition
 constexpr int kWsMaxStages = 8;
 
-// Byte masks of the decoded lo/hi words of one b = 4 word when only its
-// first v codes (0..8) are inside K.
-__device__ __forceinline__ void tail_masks(int v, uint32_t& mlo, uint32_t& mhi)
-{
-    const int nlo = (v + 1) >> 1, nhi = v >> 1;       // lo holds codes 0,2,4,6; hi 1,3,5,7
-    mlo = nlo >= 4 ? 0xffffffffu : ((1u << (8 * nlo)) - 1u);
-    mhi = nhi >= 4 ? 0xffffffffu : ((1u << (8 * nhi)) - 1u);
-}
 
 // Decode one 128-code K-block slice (16 words, four 16-byte pieces) of a
 // b = 4 row and store its 8 units to a swizzled stage row.  The loads of
@@ -671,6 +812,11 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
         K0 = k0; K1 = k1; K3 = k3;
         D51 = k5 - k1; D20 = k2 - k0; D40 = k4 - k0; E3 = (k6 - k4) - (k2 - k0);
     }
+    // the warp holding the tile's last columns of the last N-tile writes the padding words
+    const bool pad_words = ep.codes_out && (n0 + BN >= N) && ((n0 + BN) / cpw < ep.ldo) &&
+                           (split ? (warp >> 2) == 1 : true);
+    uint32_t zero_word = 0u;
+    for (int j = 0; j < cpw; j++) zero_word |= ep.out.zero_code << (ep.out.b * j);
     for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
         const int a = (int)(ti & 1);
         if (!wait_or_abort(&tfull[a], (uint32_t)((ti >> 1) & 1), err)) { *err = 1; break; }
@@ -780,6 +926,12 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 }
             }
             c += nc - 16;                             // the loop adds the other 16
+        }
+        // the last N-tile also fills the row's words past its columns (the
+        // output row stride may hold more codes than the tiles cover) with
+        // the zero code
+        if (pad_words && mrow) {
+            for (int64_t wq = (n0 + BN) / cpw; wq < ep.ldo; wq++) ep.codes_out[m * ep.ldo + wq] = zero_word;
         }
     }
 }
