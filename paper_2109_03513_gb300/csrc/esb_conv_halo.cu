@@ -212,7 +212,7 @@ __device__ __noinline__ void halo_fill(const HaloGeom g, int64_t T, int cb, uint
     }
 }
 
-template <bool FAST>
+template <bool FAST, bool GEN>
 __global__ void __launch_bounds__(kWsThreads, 1)
 esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, OpFmt fb, int BN, int nkb,
                      int stages, int n_tiles, int64_t m_tiles, float acc_scale, EpiParams ep)
@@ -417,7 +417,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
             m = ((int64_t)nimg * P + p) * Q + q;
             return q < Q && p < P;
         };
-        ws_epilogue<FAST>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
+        ws_epilogue<FAST, GEN>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
                     warp, lane);
     }
 
@@ -444,12 +444,16 @@ static int halo_static_smem(cudaError_t* err)
 {
     static int v = -1;
     if (v < 0) {
-        cudaFuncAttributes a0, a1;
-        *err = cudaFuncGetAttributes(&a0, esb_conv_halo_kernel<false>);
+        cudaFuncAttributes a0, a1, a2;
+        *err = cudaFuncGetAttributes(&a0, esb_conv_halo_kernel<false, false>);
         if (*err != cudaSuccess) return -1;
-        *err = cudaFuncGetAttributes(&a1, esb_conv_halo_kernel<true>);
+        *err = cudaFuncGetAttributes(&a1, esb_conv_halo_kernel<true, false>);
         if (*err != cudaSuccess) return -1;
-        v = (int)(a0.sharedSizeBytes > a1.sharedSizeBytes ? a0.sharedSizeBytes : a1.sharedSizeBytes);
+        *err = cudaFuncGetAttributes(&a2, esb_conv_halo_kernel<false, true>);
+        if (*err != cudaSuccess) return -1;
+        size_t m = a0.sharedSizeBytes > a1.sharedSizeBytes ? a0.sharedSizeBytes : a1.sharedSizeBytes;
+        if (a2.sharedSizeBytes > m) m = a2.sharedSizeBytes;
+        v = (int)m;
     }
     return v;
 }
@@ -525,10 +529,13 @@ bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, i
     hp.g.X = X;
     static bool configured = false;
     if (!configured) {
-        *err = cudaFuncSetAttribute(esb_conv_halo_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        *err = cudaFuncSetAttribute(esb_conv_halo_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     max_dyn_smem() - halo_static_smem(err));
         if (*err != cudaSuccess) return true;
-        *err = cudaFuncSetAttribute(esb_conv_halo_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        *err = cudaFuncSetAttribute(esb_conv_halo_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    max_dyn_smem() - halo_static_smem(err));
+        if (*err != cudaSuccess) return true;
+        *err = cudaFuncSetAttribute(esb_conv_halo_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     max_dyn_smem() - halo_static_smem(err));
         if (*err != cudaSuccess) return true;
         configured = true;
@@ -550,7 +557,10 @@ bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, i
     const bool fast = fb.b == 4 && hp.g.raw_bytes > 0 && ep.codes_out && ep.out.b == 4 && !ep.scale && !ep.bias &&
                       !ep.residual && !ep.acc_out && !ep.y_out && ep.acc_lim > 0.0f && N % hp.BN == 0 &&
                       (!ep.out.is_signed || ep.act != ESB_ACT_NONE) && (split ? half : hp.BN) % 32 == 0;
-    *err = launch_pdl(fast ? esb_conv_halo_kernel<true> : esb_conv_halo_kernel<false>, dim3((unsigned)grid), dim3(kWsThreads), (size_t)hp.smem, st, hp.g, b, N,
+    const bool gen = !(ep.codes_out && ep.out.b == 4);       // the general-width epilogue instance
+    *err = launch_pdl(fast ? esb_conv_halo_kernel<true, false>
+                           : (gen ? esb_conv_halo_kernel<false, true> : esb_conv_halo_kernel<false, false>),
+                      dim3((unsigned)grid), dim3(kWsThreads), (size_t)hp.smem, st, hp.g, b, N,
                       hp.K, fa, fb, hp.BN, hp.nkb, hp.stages, n_tiles, m_tiles, acc_scale, ep);
     return true;
 }

@@ -58,27 +58,37 @@ struct ConvSrc {
     // layer's 4-word rows) take no K.  The logical word w is word w % kw of
     // tap w / kw.
     int kw = 0;
-    struct Row { int pix0; int h0, w0; bool valid; };
-    struct Cursor { int r, s, word; };
+    // A row: the word offset of its tap (0, 0) (negative at the top-left
+    // border) and the in-image tap ranges r in [rlo, rlo + rn), s in [slo,
+    // slo + sn) (rn = 0 for rows past M).  A cursor follows the word offset
+    // of its (r, s, word) incrementally, so a step costs a few adds.
+    struct Row { int64_t base; int rlo, rn, slo, sn; };
+    struct Cursor { int r, s, word; int64_t off; };
     __device__ __forceinline__ Row row(int64_t m64) const
     {
         Row x;
         const int m = (int)m64;
-        x.valid = m64 < rows;
+        const bool valid = m64 < rows;
         const int pq = P * Q;
-        const int n = x.valid ? m / pq : 0;
-        const int rem = x.valid ? m - n * pq : 0;
+        const int n = valid ? m / pq : 0;
+        const int rem = valid ? m - n * pq : 0;
         const int p = rem / Q, q = rem - (rem / Q) * Q;
-        x.h0 = p * stride - pad;
-        x.w0 = q * stride - pad;
-        x.pix0 = n * H;
+        const int h0 = p * stride - pad, w0 = q * stride - pad;
+        x.base = ((int64_t)(n * H + h0) * W + w0) * ldx;
+        x.rlo = h0 < 0 ? -h0 : 0;
+        x.slo = w0 < 0 ? -w0 : 0;
+        const int rn = H - h0 - x.rlo, sn = W - w0 - x.slo;
+        x.rn = (valid && rn > 0) ? rn : 0;
+        x.sn = sn > 0 ? sn : 0;
         return x;
+    }
+    __device__ __forceinline__ bool inside(const Row& x, int r, int s) const
+    {
+        return (unsigned)(r - x.rlo) < (unsigned)x.rn && (unsigned)(s - x.slo) < (unsigned)x.sn;
     }
     __device__ __forceinline__ const uint32_t* tap_ptr(const Row& x, int r, int s, int word) const
     {
-        const int h = x.h0 + r, ww = x.w0 + s;
-        if (!x.valid || h < 0 || h >= H || ww < 0 || ww >= W) return nullptr;
-        return X + ((int64_t)(x.pix0 + h) * W + ww) * ldx + word;
+        return inside(x, r, s) ? X + x.base + ((int64_t)r * W + s) * ldx + word : nullptr;
     }
     __device__ __forceinline__ const uint32_t* words(const Row& x, int64_t w) const
     {
@@ -93,19 +103,29 @@ struct ConvSrc {
         c.word = (int)(w - (int64_t)tap * kw);
         c.r = tap / S;
         c.s = tap - c.r * S;
+        c.off = ((int64_t)c.r * W + c.s) * ldx + c.word;
         return c;
     }
     __device__ __forceinline__ void advance(Cursor& c, int dw) const
     {
         c.word += dw;
+        c.off += dw;
         while (c.word >= kw) {
             c.word -= kw;
-            if (++c.s == S) { c.s = 0; ++c.r; }
+            c.off += ldx - kw;
+            if (++c.s == S) {
+                c.s = 0;
+                ++c.r;
+                c.off += (int64_t)(W - S) * ldx;
+            }
         }
     }
     // 16-byte pieces (4 logical words) are contiguous in memory
     __host__ __device__ __forceinline__ bool vec4() const { return (kw & 3) == 0; }
-    __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const { return tap_ptr(x, c.r, c.s, c.word); }
+    __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const
+    {
+        return inside(x, c.r, c.s) ? X + x.base + c.off : nullptr;
+    }
     __host__ __device__ __forceinline__ bool linear() const { return true; }
     __device__ __forceinline__ const uint32_t* code_word(const Row& x, int64_t kk, int cpw, int& slot) const
     {
@@ -347,7 +367,7 @@ __device__ __noinline__ void fill_stage_any(const Src src, int64_t m0, uint8_t* 
     }
 }
 
-template <class SrcA>
+template <class SrcA, bool GEN>
 __global__ void __launch_bounds__(kWsThreads, 1)
 esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpFmt fa, OpFmt fb, int BN, int nkb,
                    int stages, int n_tiles, int64_t m_tiles, float acc_scale, EpiParams ep)
@@ -502,7 +522,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
             m = (first + ti * ctas) * kBM + row;
             return m < M;
         };
-        ws_epilogue<false>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
+        ws_epilogue<false, GEN>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty, err,
                     warp, lane);
     }
 
@@ -604,10 +624,12 @@ static int ws_static_smem(cudaError_t* err)
 {
     static int v = -1;
     if (v < 0) {
-        cudaFuncAttributes fa_attr;
-        *err = cudaFuncGetAttributes(&fa_attr, esb_gemm_ws_kernel<SrcA>);
+        cudaFuncAttributes a0, a1;
+        *err = cudaFuncGetAttributes(&a0, esb_gemm_ws_kernel<SrcA, false>);
         if (*err != cudaSuccess) return -1;
-        v = (int)fa_attr.sharedSizeBytes;
+        *err = cudaFuncGetAttributes(&a1, esb_gemm_ws_kernel<SrcA, true>);
+        if (*err != cudaSuccess) return -1;
+        v = (int)(a0.sharedSizeBytes > a1.sharedSizeBytes ? a0.sharedSizeBytes : a1.sharedSizeBytes);
     }
     return v;
 }
@@ -626,7 +648,9 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
     if (L.stages < 3) return false;
     static bool configured = false;
     if (!configured) {
-        *err = cudaFuncSetAttribute(esb_gemm_ws_kernel<SrcA>, cudaFuncAttributeMaxDynamicSharedMemorySize, maxs);
+        *err = cudaFuncSetAttribute(esb_gemm_ws_kernel<SrcA, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, maxs);
+        if (*err != cudaSuccess) return true;
+        *err = cudaFuncSetAttribute(esb_gemm_ws_kernel<SrcA, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, maxs);
         if (*err != cudaSuccess) return true;
         configured = true;
     }
@@ -637,7 +661,8 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
     if (per_n > m_tiles) per_n = m_tiles;
     const int64_t grid = per_n * n_tiles;
     const float acc_scale = ldexpf(1.0f, fa.csc + fb.csc);
-    *err = launch_pdl(esb_gemm_ws_kernel<SrcA>, dim3((unsigned)grid), dim3(kWsThreads), (size_t)L.smem_bytes, st, a, b,
+    const bool gen = !(ep.codes_out && ep.out.b == 4);       // the general-width epilogue instance
+    *err = launch_pdl(gen ? esb_gemm_ws_kernel<SrcA, true> : esb_gemm_ws_kernel<SrcA, false>, dim3((unsigned)grid), dim3(kWsThreads), (size_t)L.smem_bytes, st, a, b,
                       M, N, K, fa, fb, BN, L.nkb, L.stages, n_tiles, m_tiles, acc_scale, ep);
     return true;
 }

@@ -298,7 +298,7 @@ esb_gemm_tiled_kernel(const uint8_t* __restrict__ At, const uint8_t* __restrict_
             m = (first + ti * ctas) * kBM + row;
             return m < M;
         };
-        ws_epilogue<LEAN4>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty,
+        ws_epilogue<LEAN4, false>(ep, thr, rows, my_tiles, n0, N, BN, split, epi_warps, tmem_base, acc_scale, tfull, tempty,
                            err, warp, lane);
     }
 

@@ -755,8 +755,11 @@ __device__ __forceinline__ uint32_t ws_setup(const RowsSrc& srcB, int64_t n0, in
 // and bias (every column chunk inside N, each warp's columns a multiple of
 // 32); the instance then holds just the
 // FMA-pipe requantisation and, for device values that rule it out, the
-// out-of-line per-word path.
-template <bool LEAN4, class RowMap>
+// out-of-line per-word path.  GEN: the output is not 4-bit codes; the
+// instance holds the general-width code path and the out-of-line path for
+// fp32/int32 outputs, and none of the 4-bit code (each instance keeps a
+// small hot loop).
+template <bool LEAN4, bool GEN, class RowMap>
 __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* thr, const RowMap& rows,
                                             int64_t my_tiles, int64_t n0, int64_t N, int BN, bool split,
                                             int epi_warps, uint32_t tmem_base, float acc_scale, uint64_t* tfull,
@@ -786,6 +789,20 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
     if (warp == 0) {
         if (lane == 0) { sh_ep = ep; sh_cx = cx; }
         if (raw_ok && lane < 7) sh_raw[lane] = acc_raw_threshold(sc_fixed, ep.bias0, thr[lane], ep.act, 1.0f / acc_scale);
+    }
+    // Output widths other than 4, codes only ("gen"): per element the
+    // affine map, residual and activation, then the bucket by a bisection
+    // over the 2^(b-1) - 1 thresholds; with a positive scalar scale (and an
+    // unsigned output or an activation) over the same thresholds moved onto
+    // the raw accumulator (gen_raw, as raw_ok above), one compare per level.
+    const bool gen = GEN && !LEAN4 && ep.codes_out && ep.out.b != 4 && !ep.acc_out && !ep.y_out;
+    const bool gen_raw = gen && !ep.scale && !ep.bias && !ep.residual && isfinite(sc_lean) && sc_fixed > 0.0f &&
+                         (!out_signed || ep.act != ESB_ACT_NONE);
+    __shared__ float sh_rawT[128];                    // gen: the thresholds searched (raw or on y)
+    if (gen) {
+        const int nthr = (1 << (ep.out.b - 1)) - 1;
+        for (int i = warp * 32 + lane; i < nthr; i += epi_warps * 32)
+            sh_rawT[i] = gen_raw ? acc_raw_threshold(sc_fixed, ep.bias0, thr[i], ep.act, 1.0f / acc_scale) : thr[i];
     }
     asm volatile("bar.sync 2, %0;" ::"r"(epi_warps * 32) : "memory");   // exactly the epilogue warps in use
     const int cpw = ep.out_cpw;
@@ -826,8 +843,79 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
         const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(a * BN);
         uint32_t wsw[4] = {0u, 0u, (uint32_t)(((n0 + c_lo) / cpw) & 0xffffffff),
                            (uint32_t)(((n0 + c_lo) / cpw) >> 32)};   // general path: word, slot, column
+        uint32_t gword = 0u;                          // gen path: word being packed, its next slot, its column
+        int gslot = 0;
+        int64_t gcol = (n0 + c_lo) / cpw;
         for (int c = c_lo; c < c_hi; c += 16) {
-            if (!LEAN4 && !swar) {
+            if (gen) {
+                uint32_t r[16];
+                const bool live = n0 + c < N;         // a chunk wholly past N only packs zero codes
+                if (live) tmem_ld16(taddr + (uint32_t)c, r);
+                if (c + 16 >= c_hi) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&tempty[a]);
+                }
+                const int ob = ep.out.b, one = 1 << ep.out.k, nlev = ob - 1;
+                const int half = 1 << (ob - 2);
+                const uint32_t nk = (uint32_t)ep.out.N << ep.out.k;
+                // codes of the 16 columns first (no stores in between, so the
+                // 16 searches overlap), then the packing and stores
+                uint32_t cd[16];
+                if (!live) {
+#pragma unroll
+                    for (int j = 0; j < 16; j++) cd[j] = ep.out.zero_code;
+                } else if (gen_raw) {
+#pragma unroll
+                    for (int j = 0; j < 16; j++) {
+                        const float v = __uint_as_float(r[j]);
+                        int jb = 0;
+#pragma unroll
+                        for (int lv = 0; lv < 7; lv++)
+                            if (lv < nlev) jb += (v >= sh_rawT[jb + (half >> lv) - 1]) ? (half >> lv) : 0;
+                        const uint32_t mag = (jb >= one) ? (uint32_t)(jb - one) : (nk | (uint32_t)jb);
+                        cd[j] = (jb != 0 && n0 + c + j < N) ? mag : ep.out.zero_code;
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 16; j++) {
+                        const int64_t n = n0 + c + j;
+                        const int64_t nc = n < N ? n : N - 1;      // in-range index for the loads
+                        float sc = sc_fixed;
+                        if (ep.scale) { sc = __ldg(ep.scale + nc); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
+                        const float bi = ep.bias ? __ldg(ep.bias + nc) : ep.bias0;
+                        float y = __fmaf_rn(sc, __uint_as_float(r[j]) * acc_scale, bi);
+                        if (ep.residual && mrow) {
+                            const int rcpw = 32 / ep.res_b;
+                            const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + nc / rcpw) >>
+                                                 (ep.res_b * (int)(nc % rcpw))) & ((1u << ep.res_b) - 1u);
+                            y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+                        }
+                        y = apply_act(y, ep.act);
+                        const uint32_t sgn = __float_as_uint(y) >> 31;
+                        const float v = fabsf(y);
+                        int jb = 0;
+#pragma unroll
+                        for (int lv = 0; lv < 7; lv++)
+                            if (lv < nlev) jb += (v >= sh_rawT[jb + (half >> lv) - 1]) ? (half >> lv) : 0;
+                        const uint32_t mag = (jb >= one) ? (uint32_t)(jb - one) : (nk | (uint32_t)jb);
+                        const bool zero = jb == 0 || (sgn && !out_signed) || n >= N;
+                        cd[j] = zero ? ep.out.zero_code : (mag | (sgn << (ob - 1)));
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < 16; j++) {
+                    gword |= cd[j] << (ob * gslot);
+                    if (++gslot == cpw) {
+                        if (mrow && gcol < ep.ldo) ep.codes_out[m * ep.ldo + gcol] = gword;
+                        gword = 0u;
+                        gslot = 0;
+                        gcol++;
+                    }
+                }
+                continue;
+            }
+            if (GEN || (!LEAN4 && !swar)) {
                 epi_chunk_any(&sh_ep, &sh_cx, taddr + (uint32_t)c, acc_scale, m, mrow, n0 + c, N, wsw);
                 if (c + 16 >= c_hi) {
                     tc_fence_before();
@@ -836,6 +924,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 }
                 continue;
             }
+            if constexpr (!GEN) {
             // 4-bit output codes: 32 (or 16) columns per TMEM load
             const int nc = LEAN4 ? 16 : ((c + 32 <= c_hi) ? 32 : 16);   // LEAN4: 16 columns a load (compact code)
             uint32_t r[32];
@@ -926,6 +1015,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 }
             }
             c += nc - 16;                             // the loop adds the other 16
+            }
         }
         // the last N-tile also fills the row's words past its columns (the
         // output row stride may hold more codes than the tiles cover) with
