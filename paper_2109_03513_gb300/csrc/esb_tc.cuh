@@ -848,69 +848,82 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
         int64_t gcol = (n0 + c_lo) / cpw;
         for (int c = c_lo; c < c_hi; c += 16) {
             if (gen) {
-                uint32_t r[16];
-                const bool live = n0 + c < N;         // a chunk wholly past N only packs zero codes
-                if (live) tmem_ld16(taddr + (uint32_t)c, r);
-                if (c + 16 >= c_hi) {
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&tempty[a]);
-                }
+                // 16 columns a chunk, in four groups of four (a small loop
+                // body with four independent threshold searches); a chunk
+                // wholly past N only packs zero codes
+                const bool live = n0 + c < N;
                 const int ob = ep.out.b, one = 1 << ep.out.k, nlev = ob - 1;
                 const int half = 1 << (ob - 2);
                 const uint32_t nk = (uint32_t)ep.out.N << ep.out.k;
-                // codes of the 16 columns first (no stores in between, so the
-                // 16 searches overlap), then the packing and stores
-                uint32_t cd[16];
-                if (!live) {
-#pragma unroll
-                    for (int j = 0; j < 16; j++) cd[j] = ep.out.zero_code;
-                } else if (gen_raw) {
-#pragma unroll
-                    for (int j = 0; j < 16; j++) {
-                        const float v = __uint_as_float(r[j]);
-                        int jb = 0;
-#pragma unroll
-                        for (int lv = 0; lv < 7; lv++)
-                            if (lv < nlev) jb += (v >= sh_rawT[jb + (half >> lv) - 1]) ? (half >> lv) : 0;
-                        const uint32_t mag = (jb >= one) ? (uint32_t)(jb - one) : (nk | (uint32_t)jb);
-                        cd[j] = (jb != 0 && n0 + c + j < N) ? mag : ep.out.zero_code;
-                    }
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 16; j++) {
-                        const int64_t n = n0 + c + j;
-                        const int64_t nc = n < N ? n : N - 1;      // in-range index for the loads
-                        float sc = sc_fixed;
-                        if (ep.scale) { sc = __ldg(ep.scale + nc); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
-                        const float bi = ep.bias ? __ldg(ep.bias + nc) : ep.bias0;
-                        float y = __fmaf_rn(sc, __uint_as_float(r[j]) * acc_scale, bi);
-                        if (ep.residual && mrow) {
-                            const int rcpw = 32 / ep.res_b;
-                            const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + nc / rcpw) >>
-                                                 (ep.res_b * (int)(nc % rcpw))) & ((1u << ep.res_b) - 1u);
-                            y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+                const bool last = c + 16 >= c_hi;
+#pragma unroll 1
+                for (int g = 0; g < 4; g++) {
+                    uint32_t cd[4];
+                    if (live) {
+                        uint32_t r[4];
+                        tmem_ld4(taddr + (uint32_t)(c + 4 * g), r);
+                        if (last && g == 3) {
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&tempty[a]);
                         }
-                        y = apply_act(y, ep.act);
-                        const uint32_t sgn = __float_as_uint(y) >> 31;
-                        const float v = fabsf(y);
-                        int jb = 0;
+                        float v[4];
+                        uint32_t sg[4];
 #pragma unroll
-                        for (int lv = 0; lv < 7; lv++)
-                            if (lv < nlev) jb += (v >= sh_rawT[jb + (half >> lv) - 1]) ? (half >> lv) : 0;
-                        const uint32_t mag = (jb >= one) ? (uint32_t)(jb - one) : (nk | (uint32_t)jb);
-                        const bool zero = jb == 0 || (sgn && !out_signed) || n >= N;
-                        cd[j] = zero ? ep.out.zero_code : (mag | (sgn << (ob - 1)));
+                        for (int i = 0; i < 4; i++) {
+                            const int64_t n = n0 + c + 4 * g + i;
+                            if (gen_raw) {
+                                v[i] = __uint_as_float(r[i]);
+                                sg[i] = 0u;
+                            } else {
+                                const int64_t nc = n < N ? n : N - 1;      // in-range index for the loads
+                                float sc = sc_fixed;
+                                if (ep.scale) { sc = __ldg(ep.scale + nc); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
+                                const float bi = ep.bias ? __ldg(ep.bias + nc) : ep.bias0;
+                                float y = __fmaf_rn(sc, __uint_as_float(r[i]) * acc_scale, bi);
+                                if (ep.residual && mrow) {
+                                    const int rcpw = 32 / ep.res_b;
+                                    const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + nc / rcpw) >>
+                                                         (ep.res_b * (int)(nc % rcpw))) & ((1u << ep.res_b) - 1u);
+                                    y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+                                }
+                                y = apply_act(y, ep.act);
+                                sg[i] = (__float_as_uint(y) >> 31) & (out_signed ? 1u : 0u);
+                                // an unsigned set maps negatives to zero: search -1
+                                v[i] = (!out_signed && (__float_as_uint(y) >> 31)) ? -1.0f : fabsf(y);
+                            }
+                        }
+                        int jb[4] = {0, 0, 0, 0};
+#pragma unroll 1
+                        for (int lv = 0; lv < nlev; lv++) {
+                            const int step = half >> lv;
+#pragma unroll
+                            for (int i = 0; i < 4; i++) jb[i] += (v[i] >= sh_rawT[jb[i] + step - 1]) ? step : 0;
+                        }
+#pragma unroll
+                        for (int i = 0; i < 4; i++) {
+                            const uint32_t mag = (jb[i] >= one) ? (uint32_t)(jb[i] - one) : (nk | (uint32_t)jb[i]);
+                            const bool zero = jb[i] == 0 || n0 + c + 4 * g + i >= N;
+                            cd[i] = zero ? ep.out.zero_code : (mag | (sg[i] << (ob - 1)));
+                        }
+                    } else {
+                        if (last && g == 3) {
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(&tempty[a]);
+                        }
+#pragma unroll
+                        for (int i = 0; i < 4; i++) cd[i] = ep.out.zero_code;
                     }
-                }
 #pragma unroll
-                for (int j = 0; j < 16; j++) {
-                    gword |= cd[j] << (ob * gslot);
-                    if (++gslot == cpw) {
-                        if (mrow && gcol < ep.ldo) ep.codes_out[m * ep.ldo + gcol] = gword;
-                        gword = 0u;
-                        gslot = 0;
-                        gcol++;
+                    for (int i = 0; i < 4; i++) {
+                        gword |= cd[i] << (ob * gslot);
+                        if (++gslot == cpw) {
+                            if (mrow && gcol < ep.ldo) ep.codes_out[m * ep.ldo + gcol] = gword;
+                            gword = 0u;
+                            gslot = 0;
+                            gcol++;
+                        }
                     }
                 }
                 continue;
