@@ -754,6 +754,22 @@ static int conv_k_words(const esb_conv_desc& d, int64_t ldx, int bx)
     return (2 * used <= ldx) ? used : (int)ldx;
 }
 
+// Filter rows of the im2col K: plain rows when every tap's ldx input words
+// enter K with filter taps of the same width and stride; otherwise taps of
+// kwx input words (kwx * cpw_x codes) at a tap stride of ldw filter words,
+// walkable word by word when both operands have the same width.
+static RowsSrc conv_filter_rows(const esb_conv_desc& d, const uint32_t* W, int64_t ldx, int bx, int64_t ldw, int bw,
+                                int kwx)
+{
+    RowsSrc b{W, (int64_t)d.r * d.s * ldw, d.cout};
+    if (kwx != ldx || bw != bx || ldw != ldx) {
+        b.kp = (int64_t)kwx * (32 / bx);
+        b.ldt = ldw;
+        if (bw == bx) b.kwt = kwx;
+    }
+    return b;
+}
+
 cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int bx, int kx,
                            const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st)
 {
@@ -768,13 +784,7 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
     ConvSrc a;
     a.X = X; a.ldx = (int)ldx; a.rows = (int)M; a.H = d.h; a.W = d.w; a.P = P; a.Q = Q; a.S = d.s;
     a.stride = d.stride; a.pad = d.pad; a.kw = kwx;
-    RowsSrc b{W, (int64_t)d.r * d.s * ldw, N};
-    if (kwx != ldx || bw != bx || ldw != ldx) {
-        // K runs over taps of the input's kwx * cpw_x codes; each tap of a
-        // filter row holds ldw words (of its own code width)
-        b.kp = (int64_t)kwx * (32 / bx);
-        b.ldt = ldw;
-    }
+    RowsSrc b = conv_filter_rows(d, W, ldx, bx, ldw, bw, kwx);
     OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
     int64_t Kx = plan_planes(fa, fb, K);              // the kernels' K (significand planes)
     if (b.linear()) {
@@ -782,7 +792,7 @@ cudaError_t launch_conv_tc(const esb_conv_desc& d, int P, int Q, const uint32_t*
         if (const int64_t Ks = plan_slots(fa, fb, words * fa.cpw, words)) Kx = Ks;
     }
     cudaError_t e = cudaSuccess;
-    if (Kx > 0 && !conv_force_im2col() && fa.planes == 1 && b.linear() &&
+    if (Kx > 0 && !conv_force_im2col() && fa.planes == 1 && b.kp == 0 &&
         launch_conv_halo(d, P, Q, X, ldx, fa, W, ldw, fb, BN, ep, st, &e))
         return e;
     if (Kx > 0 && launch_ws(a, b, M, N, Kx, fa, fb, BN, ep, st, &e)) return e;
@@ -797,8 +807,9 @@ int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx
     const int64_t K = (int64_t)d.r * d.s * kwd * (32 / bx);
     OpFmt fa = make_opfmt(bx, kx), fb = make_opfmt(bw, kw);
     int64_t Kx = plan_planes(fa, fb, K);
-    const bool same_layout = bw == bx && ldw == ldx && fa.planes == 1 && kwd == ldx;
-    if (same_layout) {                                // the filter rows are linear (launch_conv_tc)
+    const RowsSrc b = conv_filter_rows(d, nullptr, ldx, bx, ldw, bw, kwd);
+    const bool same_layout = b.kp == 0 && fa.planes == 1;
+    if (b.linear()) {                                 // as launch_conv_tc
         const int64_t words = (int64_t)d.r * d.s * kwd;
         if (const int64_t Ks = plan_slots(fa, fb, words * fa.cpw, words)) Kx = Ks;
     }

@@ -161,12 +161,18 @@ struct RowsSrc {
     const uint32_t* base;
     int64_t ld;
     int64_t rows;
+    // Filter rows of an im2col convolution whose K runs over taps of kp
+    // codes (kp = 0: plain rows).  Tap t of a row starts at word t * ldt.
+    // kwt > 0 when a tap's K codes are whole words of this operand (kp =
+    // kwt codes per word x kwt): logical word w is then word w % kwt of tap
+    // w / kwt, and cursors walk the rows word by word.
     int64_t kp = 0;
     int64_t ldt = 0;
+    int64_t kwt = 0;
     struct Row { const uint32_t* p; };
-    struct Cursor { int64_t w; };
-    __host__ __device__ __forceinline__ bool linear() const { return kp == 0; }
-    __host__ __device__ __forceinline__ bool vec4() const { return true; }
+    struct Cursor { int64_t w; int64_t word; };        // w: offset in the row; word: index within the tap
+    __host__ __device__ __forceinline__ bool linear() const { return kp == 0 || kwt > 0; }
+    __host__ __device__ __forceinline__ bool vec4() const { return kp == 0 || ((kwt & 3) == 0 && (ldt & 3) == 0); }
     __device__ __forceinline__ Row row(int64_t r) const { Row x; x.p = (r < rows) ? base + r * ld : nullptr; return x; }
     __device__ __forceinline__ const uint32_t* words(const Row& x, int64_t w) const { return x.p ? x.p + w : nullptr; }
     // Word holding code kk of row x (nullptr: the zero code) and its slot.
@@ -183,8 +189,30 @@ struct RowsSrc {
         slot = (int)(c - wi * cpw);
         return wi < ldt ? words(x, tap * ldt + wi) : nullptr;
     }
-    __device__ __forceinline__ Cursor cursor(int64_t w) const { Cursor c; c.w = w; return c; }
-    __device__ __forceinline__ void advance(Cursor& c, int dw) const { c.w += dw; }
+    __device__ __forceinline__ Cursor cursor(int64_t w) const
+    {
+        Cursor c;
+        if (kwt > 0) {
+            const int64_t tap = w / kwt;
+            c.word = w - tap * kwt;
+            c.w = tap * ldt + c.word;
+        } else {
+            c.w = w;
+            c.word = 0;
+        }
+        return c;
+    }
+    __device__ __forceinline__ void advance(Cursor& c, int dw) const
+    {
+        c.w += dw;
+        if (kwt > 0) {
+            c.word += dw;
+            while (c.word >= kwt) {
+                c.word -= kwt;
+                c.w += ldt - kwt;
+            }
+        }
+    }
     __device__ __forceinline__ const uint32_t* at(const Row& x, const Cursor& c) const { return x.p ? x.p + c.w : nullptr; }
 };
 
@@ -673,7 +701,7 @@ template <bool B4>
 __device__ __forceinline__ void ws_decode_b(const RowsSrc& srcB, int64_t n0, int64_t K, const OpFmt& fb, int BN,
                                             int nkb, uint8_t* sB, int t, int nthreads, const uint8_t* lutb = nullptr)
 {
-    if (B4 || (fb.b == 4 && fb.planes == 1 && srcB.linear())) {
+    if (B4 || (fb.b == 4 && fb.planes == 1 && srcB.linear() && srcB.vec4())) {
         // one row chunk per thread and pass (compact: this code runs cold,
         // once per CTA, on the path to the first MMA)
         const uint32_t zw = fmt_zero_code(4, fb.k) * 0x11111111u;
