@@ -149,7 +149,7 @@ __device__ void tiled_chunked_epilogue(const EpiParams& ep, const float* thr, in
             if (c + 16 >= c_hi) {                        // every column of this warp is in registers
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&tempty[buf]);
+                if (lane == 0) mbar_arrive_tmem_free(&tempty[buf]);
             }
             if (!mrow) continue;
             uint32_t word = 0u;

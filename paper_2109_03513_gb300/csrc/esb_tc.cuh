@@ -528,6 +528,16 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar)
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
+// Arrive without release semantics: for the epilogue's "accumulator buffer
+// free" signal, which orders only its TMEM reads (complete once
+// tcgen05.wait::ld returns, fenced by tcgen05.fence::before_thread_sync)
+// against the next MMA.  A release arrive would first wait for the warp's
+// earlier global stores of output codes to be performed, once per tile.
+__device__ __forceinline__ void mbar_arrive_tmem_free(uint64_t* bar)
+{
+    asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 // ----------------------------------------- resident-B persistent kernel
 
 constexpr int kWsEpiWarps = 8;                 // warps 0-7: epilogue (lanes 32*(w&3).., column half w>>2)
@@ -874,78 +884,72 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
         uint32_t gword = 0u;                          // gen path: word being packed, its next slot, its column
         int gslot = 0;
         int64_t gcol = (n0 + c_lo) / cpw;
-        for (int c = c_lo; c < c_hi; c += 16) {
-            if (gen) {
-                // 16 columns a chunk, in four groups of four (a small loop
-                // body with four independent threshold searches); a chunk
-                // wholly past N only packs zero codes
-                const bool live = n0 + c < N;
-                const int ob = ep.out.b, one = 1 << ep.out.k, nlev = ob - 1;
-                const int half = 1 << (ob - 2);
-                const uint32_t nk = (uint32_t)ep.out.N << ep.out.k;
-                const bool last = c + 16 >= c_hi;
+        if (gen) {
+            // columns [c_lo, c_end) are the warp's chunks holding outputs
+            // inside N, 16 columns a chunk in four groups of four (a small
+            // loop body with four independent threshold searches); the rest
+            // of its columns are zero codes, written as whole words below
+            const int64_t live = N - n0 - c_lo;
+            const int c_end = live <= 0 ? c_lo : (int)((c_hi - c_lo < ((live + 15) >> 4) << 4)
+                                                         ? c_hi : c_lo + (((live + 15) >> 4) << 4));
+            if (c_end == c_lo) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_tmem_free(&tempty[a]);
+            }
+            const int ob = ep.out.b, one = 1 << ep.out.k, nlev = ob - 1;
+            const int half = 1 << (ob - 2);
+            const uint32_t nk = (uint32_t)ep.out.N << ep.out.k;
+            for (int c = c_lo; c < c_end; c += 16) {
+                const bool last = c + 16 >= c_end;
 #pragma unroll 1
                 for (int g = 0; g < 4; g++) {
-                    uint32_t cd[4];
-                    if (live) {
-                        uint32_t r[4];
-                        tmem_ld4(taddr + (uint32_t)(c + 4 * g), r);
-                        if (last && g == 3) {
-                            tc_fence_before();
-                            __syncwarp();
-                            if (lane == 0) mbar_arrive(&tempty[a]);
-                        }
-                        float v[4];
-                        uint32_t sg[4];
+                    uint32_t r[4];
+                    tmem_ld4(taddr + (uint32_t)(c + 4 * g), r);
+                    if (last && g == 3) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive_tmem_free(&tempty[a]);
+                    }
+                    float v[4];
+                    uint32_t sg[4];
 #pragma unroll
-                        for (int i = 0; i < 4; i++) {
-                            const int64_t n = n0 + c + 4 * g + i;
-                            if (gen_raw) {
-                                v[i] = __uint_as_float(r[i]);
-                                sg[i] = 0u;
-                            } else {
-                                const int64_t nc = n < N ? n : N - 1;      // in-range index for the loads
-                                float sc = sc_fixed;
-                                if (ep.scale) { sc = __ldg(ep.scale + nc); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
-                                const float bi = ep.bias ? __ldg(ep.bias + nc) : ep.bias0;
-                                float y = __fmaf_rn(sc, __uint_as_float(r[i]) * acc_scale, bi);
-                                if (ep.residual && mrow) {
-                                    const int rcpw = 32 / ep.res_b;
-                                    const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + nc / rcpw) >>
-                                                         (ep.res_b * (int)(nc % rcpw))) & ((1u << ep.res_b) - 1u);
-                                    y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
-                                }
-                                y = apply_act(y, ep.act);
-                                sg[i] = (__float_as_uint(y) >> 31) & (out_signed ? 1u : 0u);
-                                // an unsigned set maps negatives to zero: search -1
-                                v[i] = (!out_signed && (__float_as_uint(y) >> 31)) ? -1.0f : fabsf(y);
+                    for (int i = 0; i < 4; i++) {
+                        const int64_t n = n0 + c + 4 * g + i;
+                        if (gen_raw) {
+                            v[i] = __uint_as_float(r[i]);
+                            sg[i] = 0u;
+                        } else {
+                            const int64_t nc = n < N ? n : N - 1;      // in-range index for the loads
+                            float sc = sc_fixed;
+                            if (ep.scale) { sc = __ldg(ep.scale + nc); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
+                            const float bi = ep.bias ? __ldg(ep.bias + nc) : ep.bias0;
+                            float y = __fmaf_rn(sc, __uint_as_float(r[i]) * acc_scale, bi);
+                            if (ep.residual && mrow) {
+                                const int rcpw = 32 / ep.res_b;
+                                const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + nc / rcpw) >>
+                                                     (ep.res_b * (int)(nc % rcpw))) & ((1u << ep.res_b) - 1u);
+                                y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
                             }
+                            y = apply_act(y, ep.act);
+                            sg[i] = (__float_as_uint(y) >> 31) & (out_signed ? 1u : 0u);
+                            // an unsigned set maps negatives to zero: search -1
+                            v[i] = (!out_signed && (__float_as_uint(y) >> 31)) ? -1.0f : fabsf(y);
                         }
-                        int jb[4] = {0, 0, 0, 0};
+                    }
+                    int jb[4] = {0, 0, 0, 0};
 #pragma unroll 1
-                        for (int lv = 0; lv < nlev; lv++) {
-                            const int step = half >> lv;
+                    for (int lv = 0; lv < nlev; lv++) {
+                        const int step = half >> lv;
 #pragma unroll
-                            for (int i = 0; i < 4; i++) jb[i] += (v[i] >= sh_rawT[jb[i] + step - 1]) ? step : 0;
-                        }
-#pragma unroll
-                        for (int i = 0; i < 4; i++) {
-                            const uint32_t mag = (jb[i] >= one) ? (uint32_t)(jb[i] - one) : (nk | (uint32_t)jb[i]);
-                            const bool zero = jb[i] == 0 || n0 + c + 4 * g + i >= N;
-                            cd[i] = zero ? ep.out.zero_code : (mag | (sg[i] << (ob - 1)));
-                        }
-                    } else {
-                        if (last && g == 3) {
-                            tc_fence_before();
-                            __syncwarp();
-                            if (lane == 0) mbar_arrive(&tempty[a]);
-                        }
-#pragma unroll
-                        for (int i = 0; i < 4; i++) cd[i] = ep.out.zero_code;
+                        for (int i = 0; i < 4; i++) jb[i] += (v[i] >= sh_rawT[jb[i] + step - 1]) ? step : 0;
                     }
 #pragma unroll
                     for (int i = 0; i < 4; i++) {
-                        gword |= cd[i] << (ob * gslot);
+                        const uint32_t mag = (jb[i] >= one) ? (uint32_t)(jb[i] - one) : (nk | (uint32_t)jb[i]);
+                        const bool zero = jb[i] == 0 || n0 + c + 4 * g + i >= N;
+                        const uint32_t code = zero ? ep.out.zero_code : (mag | (sg[i] << (ob - 1)));
+                        gword |= code << (ob * gslot);
                         if (++gslot == cpw) {
                             if (mrow && gcol < ep.ldo) ep.codes_out[m * ep.ldo + gcol] = gword;
                             gword = 0u;
@@ -954,14 +958,26 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                         }
                     }
                 }
-                continue;
             }
+            // the word in progress and the warp's remaining words: zero codes
+            if (gslot != 0) {
+                for (int j = gslot; j < cpw; j++) gword |= ep.out.zero_code << (ob * j);
+                if (mrow && gcol < ep.ldo) ep.codes_out[m * ep.ldo + gcol] = gword;
+                gword = 0u;
+                gslot = 0;
+                gcol++;
+            }
+            const int64_t wend = (n0 + c_hi) / cpw;
+            if (mrow)
+                for (; gcol < wend && gcol < ep.ldo; gcol++) ep.codes_out[m * ep.ldo + gcol] = zero_word;
+        }
+        for (int c = c_lo; c < (gen ? c_lo : c_hi); c += 16) {
             if (GEN || (!LEAN4 && !swar)) {
                 epi_chunk_any(&sh_ep, &sh_cx, taddr + (uint32_t)c, acc_scale, m, mrow, n0 + c, N, wsw);
                 if (c + 16 >= c_hi) {
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&tempty[a]);
+                    if (lane == 0) mbar_arrive_tmem_free(&tempty[a]);
                 }
                 continue;
             }
@@ -977,7 +993,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
             if (c + nc >= c_hi) {                     // every column of this warp is in registers
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&tempty[a]);
+                if (lane == 0) mbar_arrive_tmem_free(&tempty[a]);
             }
             const bool lean = lean_ok && (n0 + c + nc <= N);
             uint32_t wds[4];
