@@ -43,6 +43,7 @@ struct CcEpi {
     float* y_out;
     uint32_t* codes_out;
     int64_t ldo;
+    int acc24;             // every accumulator below 2^24 in magnitude (exact as fp32)
 };
 
 __device__ __forceinline__ float cc_act(float y, int act)
@@ -147,21 +148,29 @@ esb_dwconv_kernel(const uint32_t* __restrict__ X, int64_t ldx, int bx, int kx,
 // (every MobileNetV2 layer).  Each block decodes the filters of all
 // channels once into shared memory (integer images, [tap][channel]) and
 // builds the table of input images and the requantisation thresholds, then
-// walks its share of the work units: one unit = one code word (CPW
-// channels) of QT consecutive output pixels of one row, accumulated in
-// registers.  The taps run in rolled loops so that the kernel's code stays
-// small (fully unrolled strips measured instruction-fetch bound).
+// walks work items: one item = one code word (CPW channels) of QT
+// consecutive output pixels of one output row (QT = 4 at stride 1, 2 at
+// stride 2).  For each filter row, the item's NIN input words are loaded
+// together (independent loads in flight), each is decoded once and added
+// into every output of the strip that uses it, with the row's three taps
+// in registers.  Index arithmetic is 32-bit (the host checks the sizes).
+// The lean epilogue (4-bit codes only, a positive scalar scale, monotone
+// requantisation) compares the integer accumulator with the 7 thresholds
+// moved onto it and packs a word in one step; everything else takes the
+// per-element path.
 template <int B, int STRIDE>
 __global__ void __launch_bounds__(128)
-esb_dwconv3_kernel(const uint32_t* __restrict__ X, int64_t ldx, int kx, const uint32_t* __restrict__ W, int64_t ldw,
-                   int kw, int n, int H, int Wd, int C, int pad, int P, int Q, int QS, CcEpi ep)
+esb_dwconv3_kernel(const uint32_t* __restrict__ X, int ldx, int kx, const uint32_t* __restrict__ W, int ldw, int kw,
+                   int H, int Wd, int C, int pad, int P, int Q, int QS, int rows, CcEpi ep)
 {
     constexpr int CPW = 32 / B;
-    constexpr int QT = 4;
+    constexpr int QT = STRIDE == 1 ? 4 : 2;
+    constexpr int NIN = (QT - 1) * STRIDE + 3;        // input columns of a strip
     constexpr uint32_t MASK = (1u << B) - 1u;
     extern __shared__ int32_t wtab[];                 // [9][words * CPW] filter images
     __shared__ int32_t lutx[1 << B];
     __shared__ float T[128];
+    __shared__ float Rs[8];
     const int words = (C + CPW - 1) / CPW;
     const int cp = words * CPW;
     const int ewx = B - kx - 1, Nx = (1 << ewx) - 1;
@@ -170,75 +179,110 @@ esb_dwconv3_kernel(const uint32_t* __restrict__ X, int64_t ldx, int kx, const ui
     for (int i = threadIdx.x; i < (1 << B); i += blockDim.x) lutx[i] = code_image_i((uint32_t)i, B, kx, ewx, Nx);
     for (int i = threadIdx.x; i < 9 * words; i += blockDim.x) {
         const int t = i / words, w = i - (i / words) * words;
-        const uint32_t fw = __ldg(W + (int64_t)t * ldw + w);
+        const uint32_t fw = __ldg(W + t * ldw + w);
 #pragma unroll
         for (int j = 0; j < CPW; j++) wtab[t * cp + w * CPW + j] = code_image_i((fw >> (B * j)) & MASK, B, kw, eww, Nw);
     }
     const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
     if (ep.codes_out) build_thresholds(T, ep.out, alpha_out, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
-    __syncthreads();
-    Thr7 t7;
-    const bool b4 = ep.out.b == 4 && ep.codes_out;
-#pragma unroll
-    for (int i = 0; i < 7; i++) t7.t[i] = b4 ? T[i] : 0.0f;
     const bool dq = ep.alpha_a_dev && ep.alpha_b_dev;
     const float dqs = dq ? __fmul_rn(__ldg(ep.alpha_a_dev), __ldg(ep.alpha_b_dev)) * ep.dq_pow2 : 1.0f;
+    const float sc_fixed = ep.scale ? 0.0f : (dq ? __fmul_rn(ep.scale0, dqs) : ep.scale0);
+    const bool b4 = ep.out.b == 4 && ep.codes_out;
+    const bool lean = b4 && ep.acc24 && !ep.scale && !ep.bias && !ep.residual && !ep.acc_out && !ep.y_out &&
+                      sc_fixed > 0.0f && (!ep.out.is_signed || ep.act != ESB_ACT_NONE);
+    __syncthreads();
+    if (lean && threadIdx.x < 7) Rs[threadIdx.x] = acc_raw_threshold(sc_fixed, ep.bias0, T[threadIdx.x], ep.act, 1.0f);
+    __syncthreads();
+    Thr7 t7, r7;
+#pragma unroll
+    for (int i = 0; i < 7; i++) {
+        t7.t[i] = b4 ? T[i] : 0.0f;
+        r7.t[i] = lean ? Rs[i] : 0.0f;
+    }
     const int rcpw = ep.residual ? 32 / ep.res_b : 1;
     const uint32_t rmask = ep.residual ? (1u << ep.res_b) - 1u : 0u;
-    const int64_t total = (int64_t)n * P * QS * ep.ldo;
-    for (int64_t unit = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; unit < total;
-         unit += (int64_t)gridDim.x * blockDim.x) {
-        const int w = (int)(unit % ep.ldo);
-        int64_t rest = unit / ep.ldo;
-        const int qs = (int)(rest % QS);
-        rest /= QS;
-        const int p = (int)(rest % P);
-        const int nn = (int)(rest / P);
+    uint32_t zx = 0u, zo = 0u;                        // zero-code words of the input and output formats
+#pragma unroll
+    for (int j = 0; j < CPW; j++) zx |= (uint32_t)fmt_zero_code(B, kx) << (B * j);
+    for (int j = 0; j < CPW; j++) zo |= ep.out.zero_code << (ep.out.b * j);
+    const int ldo = (int)ep.ldo;
+    const int upr = QS * ldo;
+    const int total = rows * upr;
+    for (int it = blockIdx.x * blockDim.x + threadIdx.x; it < total; it += gridDim.x * blockDim.x) {
+        const int row = it / upr;                     // n * P + p
+        const int u = it - row * upr;
+        const int qs = u / ldo;
+        const int w = u - qs * ldo;
+        const int nn = row / P;
+        const int p = row - nn * P;
         const int q0 = qs * QT;
+        const int64_t obase = ((int64_t)row * Q + q0) * ldo + w;    // output word of pixel q0
         if (w >= words) {                             // padding words of the output rows: zero codes
             if (ep.codes_out) {
-                uint32_t word = 0;
 #pragma unroll
-                for (int j = 0; j < CPW; j++) word |= ep.out.zero_code << (B * j);
-#pragma unroll
-                for (int u = 0; u < QT; u++)
-                    if (q0 + u < Q) ep.codes_out[(((int64_t)nn * P + p) * Q + q0 + u) * ep.ldo + w] = word;
+                for (int uu = 0; uu < QT; uu++)
+                    if (q0 + uu < Q) ep.codes_out[obase + (int64_t)uu * ldo] = zo;
             }
             continue;
         }
         int32_t acc[QT][CPW];
 #pragma unroll
-        for (int u = 0; u < QT; u++)
+        for (int uu = 0; uu < QT; uu++)
 #pragma unroll
-            for (int j = 0; j < CPW; j++) acc[u][j] = 0;
-        // taps in rolled loops (compact code: the instruction cache holds
-        // it), the strip's outputs unrolled; each input word is re-read
-        // from L1 by the up to 3 taps that share it
+            for (int j = 0; j < CPW; j++) acc[uu][j] = 0;
+        const int c0 = q0 * STRIDE - pad;             // first input column of the strip
 #pragma unroll 1
         for (int r = 0; r < 3; r++) {
             const int h = p * STRIDE - pad + r;
-            if (h < 0 || h >= H) continue;
-            const uint32_t* xrow = X + ((int64_t)nn * H + h) * Wd * ldx + w;
-#pragma unroll 1
-            for (int s2 = 0; s2 < 3; s2++) {
-                int32_t wf[CPW];
+            if ((unsigned)h >= (unsigned)H) continue;
+            const uint32_t* xrow = X + (int64_t)(nn * H + h) * Wd * ldx + w;
+            uint32_t xw[NIN];
 #pragma unroll
-                for (int j = 0; j < CPW; j++) wf[j] = wtab[(r * 3 + s2) * cp + w * CPW + j];
+            for (int c = 0; c < NIN; c++) {
+                const int col = c0 + c;
+                xw[c] = ((unsigned)col < (unsigned)Wd) ? __ldg(xrow + (int64_t)col * ldx) : zx;
+            }
+            int32_t wf[3][CPW];
 #pragma unroll
-                for (int u = 0; u < QT; u++) {
-                    const int col = (q0 + u) * STRIDE - pad + s2;
-                    if (col < 0 || col >= Wd) continue;
-                    const uint32_t xw = __ldg(xrow + (int64_t)col * ldx);
+            for (int s2 = 0; s2 < 3; s2++)
 #pragma unroll
-                    for (int j = 0; j < CPW; j++) acc[u][j] += lutx[(xw >> (B * j)) & MASK] * wf[j];
+                for (int j = 0; j < CPW; j++) wf[s2][j] = wtab[(r * 3 + s2) * cp + w * CPW + j];
+#pragma unroll
+            for (int c = 0; c < NIN; c++) {
+                int32_t img[CPW];
+#pragma unroll
+                for (int j = 0; j < CPW; j++) img[j] = lutx[(xw[c] >> (B * j)) & MASK];
+#pragma unroll
+                for (int uu = 0; uu < QT; uu++) {
+                    const int s2 = c - uu * STRIDE;
+                    if (s2 >= 0 && s2 < 3) {
+#pragma unroll
+                        for (int j = 0; j < CPW; j++) acc[uu][j] += img[j] * wf[s2][j];
+                    }
                 }
             }
         }
+        const int cvalid = C - w * CPW;               // channels of this word inside C
 #pragma unroll
-        for (int u = 0; u < QT; u++) {
-            const int q = q0 + u;
-            if (q >= Q) break;
-            const int64_t pix = ((int64_t)nn * P + p) * Q + q;
+        for (int uu = 0; uu < QT; uu++) {
+            if (q0 + uu >= Q) break;
+            const int64_t ow = obase + (int64_t)uu * ldo;
+            if (lean) {
+                uint32_t J = 0u;
+#pragma unroll
+                for (int j = 0; j < CPW; j++) {
+                    const float v = (float)acc[uu][j];
+                    const bool b2 = v >= r7.t[3];
+                    const bool b1 = v >= (b2 ? r7.t[5] : r7.t[1]);
+                    const bool b0 = v >= (b2 ? (b1 ? r7.t[6] : r7.t[4]) : (b1 ? r7.t[2] : r7.t[0]));
+                    const uint32_t jb = (b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u);
+                    J |= (j < cvalid ? jb : 0u) << (4 * j);
+                }
+                ep.codes_out[ow] = codes8_b4(J, 0u, ep.out.k);
+                continue;
+            }
+            const int64_t pix = (int64_t)row * Q + q0 + uu;
             uint32_t word = 0;
 #pragma unroll
             for (int j = 0; j < CPW; j++) {
@@ -246,11 +290,11 @@ esb_dwconv3_kernel(const uint32_t* __restrict__ X, int64_t ldx, int kx, const ui
                 uint32_t code = ep.out.zero_code;
                 if (c < C) {
                     const int64_t o = pix * C + c;
-                    if (ep.acc_out) ep.acc_out[o] = acc[u][j];
+                    if (ep.acc_out) ep.acc_out[o] = acc[uu][j];
                     float sc = ep.scale ? __ldg(ep.scale + c) : ep.scale0;
                     if (dq) sc = __fmul_rn(sc, dqs);
                     const float bi = ep.bias ? __ldg(ep.bias + c) : ep.bias0;
-                    float y = __fmaf_rn(sc, (float)acc[u][j], bi);
+                    float y = __fmaf_rn(sc, (float)acc[uu][j], bi);
                     if (ep.residual) {
                         const uint32_t rc =
                             (__ldg(ep.residual + pix * ep.res_ld + c / rcpw) >> (ep.res_b * (c % rcpw))) & rmask;
@@ -262,7 +306,7 @@ esb_dwconv3_kernel(const uint32_t* __restrict__ X, int64_t ldx, int kx, const ui
                 }
                 word |= code << (B * j);
             }
-            if (ep.codes_out) ep.codes_out[pix * ep.ldo + w] = word;
+            if (ep.codes_out) ep.codes_out[ow] = word;
         }
     }
 }
@@ -271,17 +315,26 @@ template <int B, int STRIDE>
 static cudaError_t launch_dw3(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int kx,
                               const uint32_t* W, int64_t ldw, int kw, const CcEpi& ep, cudaStream_t st)
 {
-    constexpr int QT = 4;
+    constexpr int QT = STRIDE == 1 ? 4 : 2;
     const int QS = (Q + QT - 1) / QT;
-    const int64_t total = (int64_t)d.n * P * QS * ep.ldo;
+    const int rows = d.n * P;
+    const int64_t total = (int64_t)rows * QS * ep.ldo;
     int64_t blocks = (total + 127) / 128;
-    const int64_t cap = (int64_t)device_sm_count() * 8;
+    // one resident wave (each block's set-up -- filter table, thresholds --
+    // is then paid once per block and amortised over many items)
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, esb_dwconv3_kernel<B, STRIDE>, 128,
+                                                      sizeof(int32_t) * 9 * (size_t)((d.c + 32 / B - 1) / (32 / B)) *
+                                                          (32 / B)) != cudaSuccess ||
+        per_sm < 1)
+        per_sm = 4;
+    const int64_t cap = (int64_t)device_sm_count() * per_sm;
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
     const int words = (d.c + 32 / B - 1) / (32 / B);
     const size_t smem = sizeof(int32_t) * 9 * (size_t)words * (32 / B);
-    esb_dwconv3_kernel<B, STRIDE><<<(unsigned)blocks, 128, smem, st>>>(X, ldx, kx, W, ldw, kw, d.n, d.h, d.w, d.c, d.pad,
-                                                                       P, Q, QS, ep);
+    esb_dwconv3_kernel<B, STRIDE><<<(unsigned)blocks, 128, smem, st>>>(X, (int)ldx, kx, W, (int)ldw, kw, d.h, d.w, d.c,
+                                                                       d.pad, P, Q, QS, rows, ep);
     return cudaGetLastError();
 }
 
@@ -311,6 +364,7 @@ static CcEpi make_cc_epi(const GemmOutputs& o, int ka, int kb)
     ep.y_out = o.y_out;
     ep.codes_out = o.codes_out;
     ep.ldo = o.ldo;
+    ep.acc24 = 0;
     return ep;
 }
 
@@ -327,13 +381,19 @@ cudaError_t launch_dwconv(const esb_conv_desc& d, int P, int Q, const uint32_t* 
                           const uint32_t* W, int64_t ldw, int bw, int kw, const GemmOutputs& o, cudaStream_t st)
 {
     CcEpi ep = make_cc_epi(o, kx, kw);
+    ep.acc24 = (double)d.r * d.s * fmt_max_image(bx, kx) * fmt_max_image(bw, kw) < 16777216.0;
     // Thread grid covers words of the output row stride: ldo words when codes
     // are written, else the input's words (acc/y only).
     if (!o.codes_out) ep.ldo = (d.c + (32 / bx) - 1) / (32 / bx);
     // filter table of the fast kernel: 9 taps x the padded channels, int32, in 48 KiB
     const int64_t tab = 9 * (int64_t)((d.c + 32 / bx - 1) / (32 / bx)) * (32 / bx) * 4;
+    // the specialised kernel indexes in 32 bits: work items, input and output words of one image
+    const int P1 = P, Q1 = Q;
+    const int64_t items = (int64_t)d.n * P1 * ((Q1 + 1) / 2) * (o.codes_out ? o.ldo : 1);
+    const bool fits32 = items < (1ll << 31) && (int64_t)d.n * d.h * d.w * ldx < (1ll << 31) && ldx < (1 << 20) &&
+                        ldw < (1 << 20) && ep.ldo < (1 << 20);
     if (d.r == 3 && d.s == 3 && bw == bx && bx >= 3 && bx <= 6 && (d.stride == 1 || d.stride == 2) &&
-        tab <= 48 * 1024) {
+        tab <= 48 * 1024 && fits32) {
         const bool s1 = d.stride == 1;
         switch (bx) {
         case 3: return s1 ? launch_dw3<3, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)

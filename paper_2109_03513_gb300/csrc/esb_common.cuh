@@ -344,6 +344,28 @@ __device__ __forceinline__ uint32_t codes8_b4(uint32_t J, uint32_t S, int k)
     return ((J + C1) & 0x77777777u) | (S & nz);
 }
 
+// Lean-path threshold on the raw accumulator.  For a scale sc > 0,
+// y(a) = fma(sc, a, b) is non-decreasing in the integer accumulator a
+// (|a| < 2^24, checked on the host), and so is the activation of y; an
+// output code's bucket counts the thresholds T_j (all > 0) at or below
+// act(y).  For ReLU and no activation, act(y) >= T  <=>  y >= T (T > 0);
+// ReLU6 never reaches a T above 6.  Returns A * rs for the smallest
+// integer A with y(A) >= T (raw = a * rs exactly), +inf if none, -inf if
+// every accumulator qualifies.  26 bounded bisection steps on integers.
+__device__ __forceinline__ float acc_raw_threshold(float sc, float b, float T, int act, float rs)
+{
+    if (act == ESB_ACT_RELU6 && T > 6.0f) return __int_as_float(0x7f800000);
+    const int lim = 1 << 24;
+    if (!(__fmaf_rn(sc, (float)lim, b) >= T)) return __int_as_float(0x7f800000);
+    if (__fmaf_rn(sc, (float)-lim, b) >= T) return __int_as_float(0xff800000);
+    int lo = -lim, hi = lim;                           // y(lo) < T <= y(hi)
+    for (int it = 0; it < 32 && hi - lo > 1; it++) {
+        const int mid = lo + ((hi - lo) >> 1);
+        if (__fmaf_rn(sc, (float)mid, b) >= T) hi = mid; else lo = mid;
+    }
+    return (float)hi * rs;
+}
+
 // Value of a code in units of alpha (Sec. IV-A, Eq. q), exact in fp32 for b <= 8.
 __device__ __forceinline__ float code_value(uint32_t c, int b, int k)
 {

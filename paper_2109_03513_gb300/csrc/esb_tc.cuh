@@ -630,28 +630,6 @@ static __device__ __noinline__ void epi_chunk_any(const EpiParams* __restrict__ 
 }
 
 
-// Lean-path threshold on the raw accumulator.  For a scale sc > 0,
-// y(a) = fma(sc, a, b) is non-decreasing in the integer accumulator a
-// (|a| < 2^24, checked on the host), and so is the activation of y; an
-// output code's bucket counts the thresholds T_j (all > 0) at or below
-// act(y).  For ReLU and no activation, act(y) >= T  <=>  y >= T (T > 0);
-// ReLU6 never reaches a T above 6.  Returns A * rs for the smallest
-// integer A with y(A) >= T (raw = a * rs exactly), +inf if none, -inf if
-// every accumulator qualifies.  26 bounded bisection steps on integers.
-__device__ __forceinline__ float acc_raw_threshold(float sc, float b, float T, int act, float rs)
-{
-    if (act == ESB_ACT_RELU6 && T > 6.0f) return __int_as_float(0x7f800000);
-    const int lim = 1 << 24;
-    if (!(__fmaf_rn(sc, (float)lim, b) >= T)) return __int_as_float(0x7f800000);
-    if (__fmaf_rn(sc, (float)-lim, b) >= T) return __int_as_float(0xff800000);
-    int lo = -lim, hi = lim;                           // y(lo) < T <= y(hi)
-    for (int it = 0; it < 32 && hi - lo > 1; it++) {
-        const int mid = lo + ((hi - lo) >> 1);
-        if (__fmaf_rn(sc, (float)mid, b) >= T) hi = mid; else lo = mid;
-    }
-    return (float)hi * rs;
-}
-
 struct Raw8 { uint32_t r[8]; };
 
 // One packed word of 4-bit output codes (8 columns from n_first) with
@@ -836,6 +814,15 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
     const bool gen = GEN && !LEAN4 && ep.codes_out && ep.out.b != 4 && !ep.acc_out && !ep.y_out;
     const bool gen_raw = gen && !ep.scale && !ep.bias && !ep.residual && isfinite(sc_lean) && sc_fixed > 0.0f &&
                          (!out_signed || ep.act != ESB_ACT_NONE);
+    // 4-bit codes out with a 4-bit residual and a scalar scale and bias
+    // (ResNet's second conv of a block): per element y = fma(sc, acc, b),
+    // then fma(res_scale, image of the residual code, y), activation and the
+    // 7-threshold bucket, eight codes at a time; the residual's images come
+    // from a 16-entry table.
+    const bool lres = !LEAN4 && swar && !ep.scale && !ep.bias && !ep.acc_out && !ep.y_out && ep.residual &&
+                      ep.res_b == 4 && isfinite(sc_lean) && (sc_lean != 0.0f || sc_fixed == 0.0f);
+    __shared__ float sh_resimg[16];
+    if (lres && warp == 0 && lane < 16) sh_resimg[lane] = code_image_f((uint32_t)lane, 4, ep.res_k);
     __shared__ float sh_rawT[128];                    // gen: the thresholds searched (raw or on y)
     if (gen) {
         const int nthr = (1 << (ep.out.b - 1)) - 1;
@@ -995,12 +982,17 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 __syncwarp();
                 if (lane == 0) mbar_arrive_tmem_free(&tempty[a]);
             }
-            const bool lean = lean_ok && (n0 + c + nc <= N);
+            // columns of the chunk inside N (codes past N are masked to the zero code)
+            const int64_t ncl64 = N - (n0 + c);
+            const int ncl = ncl64 < nc ? (int)ncl64 : nc;
+            const bool lean = lean_ok && ncl > 0;
             uint32_t wds[4];
 #pragma unroll
             for (int h = 0; h < 4; h++) {
                 if (h * 8 >= nc) break;
                 uint32_t J = 0u, S = 0u;
+                const int live_h = ncl - 8 * h;       // nibbles of this word inside N
+                const uint32_t nib = live_h >= 8 ? 0xffffffffu : (live_h <= 0 ? 0u : (1u << (4 * live_h)) - 1u);
                 if (lean && fma_ok) {
                     float jh[2];
 #pragma unroll
@@ -1019,7 +1011,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                         jh[q] = jf + 8388608.0f;                   // integer jf < 2^16 in the low mantissa bits
                     }
                     J = (__float_as_uint(jh[0]) & 0xffffu) | (__float_as_uint(jh[1]) << 16);
-                    wds[h] = codes8_b4(J, 0u, ep.out.k);
+                    wds[h] = codes8_b4(J & nib, 0u, ep.out.k);
                 } else if (!LEAN4 && lean && raw_ok) {
                     // bucket = number of raw thresholds <= raw accumulator
 #pragma unroll
@@ -1030,7 +1022,7 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                         const bool b0 = v >= (b2 ? (b1 ? R6 : R4) : (b1 ? R2 : R0));
                         J |= ((b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u)) << (4 * j);
                     }
-                    wds[h] = codes8_b4(J, 0u, ep.out.k);
+                    wds[h] = codes8_b4(J & nib, 0u, ep.out.k);
                 } else if (!LEAN4 && lean) {
                     // 4-bit output codes only, scalar scale/bias, no residual:
                     // y = fma(scale * 2^(kA+kB+12), raw, bias) equals
@@ -1048,7 +1040,22 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                         J |= ((b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u)) << (4 * j);
                         if (out_signed) S |= (__float_as_uint(y) >> 31) << (4 * j + 3);
                     }
-                    wds[h] = codes8_b4(J, S, ep.out.k);
+                    wds[h] = codes8_b4(J & nib, S & nib, ep.out.k);
+                } else if (!LEAN4 && lres && ncl > 0) {
+                    const uint32_t rw = mrow ? __ldg(ep.residual + m * ep.res_ld + ((n0 + c) >> 3) + h) : 0u;
+#pragma unroll
+                    for (int j = 0; j < 8; j++) {
+                        float y = __fmaf_rn(sc_lean, __uint_as_float(r[8 * h + j]), ep.bias0);
+                        y = __fmaf_rn(ep.res_scale, sh_resimg[(rw >> (4 * j)) & 15u], y);
+                        y = apply_act(y, ep.act);
+                        const float av = out_signed ? fabsf(y) : y;
+                        const bool b2 = av >= T3;
+                        const bool b1 = av >= (b2 ? T5 : T1);
+                        const bool b0 = av >= (b2 ? (b1 ? T6 : T4) : (b1 ? T2 : T0));
+                        J |= ((b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u)) << (4 * j);
+                        if (out_signed) S |= (__float_as_uint(y) >> 31) << (4 * j + 3);
+                    }
+                    wds[h] = codes8_b4(J & nib, S & nib, ep.out.k);
                 } else {
                     Raw8 v;
 #pragma unroll
