@@ -337,6 +337,21 @@ struct WsLayout {
     int smem_bytes;   // total dynamic shared memory incl. alignment slack
 };
 
+// The B-streamed layout: stages of one A block and one B block, no resident B.
+__host__ inline WsLayout ws_layout_streamed(int64_t K, int BN, int max_smem)
+{
+    WsLayout L;
+    L.nkb = (int)((K + kBK - 1) / kBK);
+    L.BN = BN;
+    L.b_bytes = 0;
+    const int fixed = 1024 + 4 * 128 + 512;                      // slack, thresholds, barriers
+    int st = (max_smem - fixed) / ((kBM + BN) * kBK);
+    if (st > kWsMaxStages) st = kWsMaxStages;
+    L.stages = st;
+    L.smem_bytes = fixed + st * (kBM + BN) * kBK;
+    return L;
+}
+
 __host__ inline WsLayout ws_layout(int64_t K, int BN, int max_smem)
 {
     WsLayout L;
@@ -370,13 +385,17 @@ __device__ __noinline__ void fill_stage_any(const Src src, int64_t m0, uint8_t* 
 template <class SrcA, bool GEN>
 __global__ void __launch_bounds__(kWsThreads, 1)
 esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpFmt fa, OpFmt fb, int BN, int nkb,
-                   int stages, int n_tiles, int64_t m_tiles, float acc_scale, EpiParams ep)
+                   int stages, int n_tiles, int64_t m_tiles, float acc_scale, EpiParams ep, int bstream)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sB = smem;                                        // nkb blocks of BN x 128 bytes
-    uint8_t* sA = sB + nkb * BN * kBK;                         // stages x 16 KiB
-    float* thr = reinterpret_cast<float*>(sA + stages * kBM * kBK);
+    // B resident: nkb blocks of BN x 128 bytes, then stages of one A block.
+    // B streamed (bstream, when B's N-tile does not fit): no resident B;
+    // each stage holds the A block and the B block of its K-block.
+    const int stage_bytes = kBM * kBK + (bstream ? BN * kBK : 0);
+    uint8_t* sB = smem;
+    uint8_t* sA = sB + (bstream ? 0 : nkb * BN * kBK);
+    float* thr = reinterpret_cast<float*>(sA + stages * stage_bytes);
     uint64_t* full = reinterpret_cast<uint64_t*>(thr + 128);
     uint64_t* empty = full + kWsMaxStages;
     uint64_t* tfull = empty + kWsMaxStages;
@@ -430,7 +449,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
     // (ws_setup).
     uint32_t tmem_base = 0;
     if (warp < kWsProdWarp0)
-        tmem_base = ws_setup<false>(srcB, n0, K, fb, BN, nkb, sB, thr, ep, tmem_slot, tid, lutb);
+        tmem_base = ws_setup<false>(srcB, n0, K, fb, BN, bstream ? 0 : nkb, sB, thr, ep, tmem_slot, tid, lutb);
 
     if (warp >= kWsProdWarp0) {
         // ---------------------------------------------- A producers
@@ -445,6 +464,8 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
         const int64_t total_it = (p < nprod) ? my_tiles * nkb : 0;
         griddep_wait();                               // A may come from the previous launch
         const uint32_t zwa = fmt_zero_code(4, fa.k) * 0x11111111u;
+        const uint32_t zwb = fmt_zero_code(4, fb.k) * 0x11111111u;
+        const bool b_vec = fb.b == 4 && fb.planes == 1 && srcB.linear() && srcB.vec4();
         int64_t cur_tile = -1;
         typename SrcA::Row rows[4];
         // stage s and its phase ph follow it incrementally (no division in
@@ -461,7 +482,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
                 for (int q = 0; q < 4; q++) rows[q] = srcA.row(m0 + lane + 32 * q);
             }
             if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
-            uint8_t* st = sA + s * kBM * kBK;
+            uint8_t* st = sA + s * stage_bytes;
             if (fa.b == 4 && fa.planes == 1 && srcA.linear() && srcA.vec4()) {
                 const int64_t kw0 = (int64_t)kb * 16;
                 typename SrcA::Cursor cur[4];
@@ -479,6 +500,35 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
                     walk_row_kblock(srcA, rows[q], (int64_t)kb * kBK, K, fa, luta, st, lane + 32 * q);
             } else {
                 fill_stage_any(srcA, (cta_in_n + ti * ctas_per_n) * kBM, st, lane, (int64_t)kb * kBK, K, fa);
+            }
+            if (bstream) {
+                // this K-block of the CTA's B rows n0 .. n0 + BN, two rows per lane in flight
+                uint8_t* sb = st + kBM * kBK;
+                const int64_t k0 = (int64_t)kb * kBK;
+                if (b_vec) {
+                    const int64_t kw0 = (int64_t)kb * 16;
+                    RowsSrc::Cursor cur[4];
+#pragma unroll
+                    for (int pc = 0; pc < 4; pc++) cur[pc] = srcB.cursor(kw0 + 4 * pc);
+#pragma unroll 1
+                    for (int r = lane; r < BN; r += 64) {
+                        const bool two = r + 32 < BN;
+                        uint4 v0[4], v1[4];
+                        load_row_b4(srcB, srcB.row(n0 + r), cur, kw0, K, zwb, v0);
+                        if (two) load_row_b4(srcB, srcB.row(n0 + r + 32), cur, kw0, K, zwb, v1);
+                        store_row_b4(sb, r, v0, kw0, K, fb);
+                        if (two) store_row_b4(sb, r + 32, v1, kw0, K, fb);
+                    }
+                } else if (fb.planes == 1 && srcB.linear()) {
+#pragma unroll 1
+                    for (int r = lane; r < BN; r += 32) walk_row_kblock(srcB, srcB.row(n0 + r), k0, K, fb, lutb, sb, r);
+                } else {
+#pragma unroll 1
+                    for (int u = lane; u < BN * 8; u += 32) {
+                        const int r = u >> 3, g = u & 7;
+                        *reinterpret_cast<uint4*>(sb + swz(r, g)) = decode_unit_any(srcB, srcB.row(n0 + r), k0 + g * 16, K, fb);
+                    }
+                }
             }
             fence_proxy_async_smem();
             __syncwarp();
@@ -501,8 +551,8 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
                 for (int kb = 0; kb < nkb; kb++) {
                     if (!wait_or_abort(&full[s], ph, err)) { *err = 1; break; }
                     tc_fence_after();
-                    const uint32_t a0 = a_base + (uint32_t)(s * kBM * kBK);
-                    const uint32_t b0 = b_base + (uint32_t)(kb * BN * kBK);
+                    const uint32_t a0 = a_base + (uint32_t)(s * stage_bytes);
+                    const uint32_t b0 = bstream ? a0 + (uint32_t)(kBM * kBK) : b_base + (uint32_t)(kb * BN * kBK);
 #pragma unroll
                     for (int j = 0; j < kBK / 32; j++)
                         mma_f8f6f4(d, smem_desc_sw128(a0 + j * 32), smem_desc_sw128(b0 + j * 32), idesc,
@@ -634,8 +684,9 @@ static int ws_static_smem(cudaError_t* err)
     return v;
 }
 
-// Resident-B launch when B's N-tile fits in shared memory with at least
-// three A stages; returns false (nothing launched) otherwise.
+// Warp-specialised launch: B resident when its N-tile fits in shared
+// memory with at least three A stages, else streamed with A through the
+// stages; returns false (nothing launched) when neither fits.
 template <class SrcA>
 static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int64_t K, const OpFmt& fa,
                       const OpFmt& fb, int BN, const EpiParams& ep, cudaStream_t st, cudaError_t* err)
@@ -644,8 +695,16 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
     const int static_smem = ws_static_smem<SrcA>(err);
     if (static_smem < 0) return true;
     const int maxs = max_dyn_smem() - static_smem;
-    const WsLayout L = ws_layout(K, BN, maxs);
-    if (L.stages < 3) return false;
+    WsLayout L = ws_layout(K, BN, maxs);
+    int bstream = 0;
+    if (L.stages < 3) {
+        // B's N-tile does not fit beside three A stages: stream B through
+        // the stages with A, at the N-tile width that suits the row tiles
+        BN = streamed_bn(M, N, ep.out_cpw, BN);
+        L = ws_layout_streamed(K, BN, maxs);
+        if (L.stages < 3) return false;
+        bstream = 1;
+    }
     static bool configured = false;
     if (!configured) {
         *err = cudaFuncSetAttribute(esb_gemm_ws_kernel<SrcA, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, maxs);
@@ -663,7 +722,7 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
     const float acc_scale = ldexpf(1.0f, fa.csc + fb.csc);
     const bool gen = !(ep.codes_out && ep.out.b == 4);       // the general-width epilogue instance
     *err = launch_pdl(gen ? esb_gemm_ws_kernel<SrcA, true> : esb_gemm_ws_kernel<SrcA, false>, dim3((unsigned)grid), dim3(kWsThreads), (size_t)L.smem_bytes, st, a, b,
-                      M, N, K, fa, fb, BN, L.nkb, L.stages, n_tiles, m_tiles, acc_scale, ep);
+                      M, N, K, fa, fb, BN, L.nkb, L.stages, n_tiles, m_tiles, acc_scale, ep, bstream);
     return true;
 }
 

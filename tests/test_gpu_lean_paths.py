@@ -43,7 +43,7 @@ def random_codes(rows, cols, b, seed, signed=True):
 
 
 @pytest.mark.parametrize("fa,fb,K,extra", [((3, 1), (3, 1), 77, 3), ((5, 2), (5, 2), 131, 5), ((6, 3), (6, 3), 259, 4),
-                                           ((7, 3), (8, 3), 300, 2), ((2, 0), (2, 0), 515, 9), ((6, 2), (6, 3), 129, 1)])
+                                           ((7, 3), (7, 3), 15, 2), ((8, 4), (7, 3), 8, 3), ((2, 0), (2, 0), 515, 9), ((6, 2), (6, 3), 129, 1)])
 def test_gemm_word_slots_ignore_codes_past_k(fa, fb, K, extra):
     """Rows hold K + extra random codes; the contraction takes the first K."""
     M, N = 150, 70
