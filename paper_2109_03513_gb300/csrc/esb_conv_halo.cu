@@ -74,14 +74,47 @@ __device__ __forceinline__ void halo_mma_fixed(uint32_t d, uint32_t a_st, uint32
     }
 }
 
+// One packed word of a 5- or 6-bit format in the word-slot layout (8 K
+// slots per word, see plan_slots): code j to byte j through the E4M3 table,
+// the slots past the word's codes zero.
+__device__ __forceinline__ void decode_word_slot8(uint32_t w, const uint8_t* lut, int b, uint32_t& lo, uint32_t& hi)
+{
+    const int cpw = 32 / b;
+    const uint32_t mask = (1u << b) - 1u;
+    uint32_t o[2] = {0u, 0u};
+#pragma unroll
+    for (int j = 0; j < 8; j++)
+        if (j < cpw) o[j >> 2] |= (uint32_t)lut[(w >> (b * j)) & mask] << (8 * (j & 3));
+    lo = o[0];
+    hi = o[1];
+}
+
+// The two 16-byte chunks (planes 2pc, 2pc + 1) of one 4-word piece.
+template <bool SLOT>
+__device__ __forceinline__ void decode_piece(const uint4 v, int k, int ew, const uint8_t* lut, int b, uint4& c0,
+                                             uint4& c1)
+{
+    if (SLOT) {
+        decode_word_slot8(v.x, lut, b, c0.x, c0.y);
+        decode_word_slot8(v.y, lut, b, c0.z, c0.w);
+        decode_word_slot8(v.z, lut, b, c1.x, c1.y);
+        decode_word_slot8(v.w, lut, b, c1.z, c1.w);
+    } else {
+        decode_word_b4(v.x, k, ew, c0.x, c0.y);
+        decode_word_b4(v.y, k, ew, c0.z, c0.w);
+        decode_word_b4(v.z, k, ew, c1.x, c1.y);
+        decode_word_b4(v.w, k, ew, c1.z, c1.w);
+    }
+}
+
 // Producer: decode one channel block of one tile's halo into stage st.
 // Lane l owns slots l, l + 32, ...; each slot takes NPC 16-byte pieces
 // (4 words = two 16-code chunks each) of its pixel.  The pieces of up to
 // 16 / NPC slot groups are loaded before any decode, so a fill makes at
 // most a few round trips to memory.
-template <int NPC>
+template <int NPC, bool SLOT>
 __device__ __forceinline__ void halo_fill_t(const HaloGeom& g, int p0, const uint32_t* xi, uint8_t* st, int lane,
-                                            int k, int ew)
+                                            int k, int ew, const uint8_t* lut, int b)
 {
     constexpr int GB = 16 / NPC;                                   // slot groups per batch
     const int groups = (g.ns + 31) >> 5;
@@ -113,12 +146,7 @@ __device__ __forceinline__ void halo_fill_t(const HaloGeom& g, int p0, const uin
 #pragma unroll
             for (int pc = 0; pc < NPC; pc++) {
                 uint4 c0 = make_uint4(0u, 0u, 0u, 0u), c1 = c0;
-                if (ok) {
-                    decode_word_b4(v[u][pc].x, k, ew, c0.x, c0.y);
-                    decode_word_b4(v[u][pc].y, k, ew, c0.z, c0.w);
-                    decode_word_b4(v[u][pc].z, k, ew, c1.x, c1.y);
-                    decode_word_b4(v[u][pc].w, k, ew, c1.z, c1.w);
-                }
+                if (ok) decode_piece<SLOT>(v[u][pc], k, ew, lut, b, c0, c1);
                 uint8_t* dst = st + (2 * pc) * g.pb + slot * 16;
                 *reinterpret_cast<uint4*>(dst) = c0;
                 *reinterpret_cast<uint4*>(dst + g.pb) = c1;
@@ -153,9 +181,9 @@ __device__ __forceinline__ void halo_issue_rows(const HaloGeom& g, int64_t T, ui
 
 // The decoders' share of one bulk-filled tile: slots first, first + stride,
 // ... (zeros for padding slots and rows outside the image).
-template <int NPC>
+template <int NPC, bool SLOT>
 __device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint8_t* st, int first, int stride, int k,
-                                              int ew)
+                                              int ew, const uint8_t* lut, int b)
 {
     const int nimg = (int)(T / g.tpi);
     const int p0 = (int)(T - (int64_t)nimg * g.tpi) * g.rows_out;
@@ -172,13 +200,7 @@ __device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint
 #pragma unroll
         for (int pc = 0; pc < NPC; pc++) {
             uint4 c0 = make_uint4(0u, 0u, 0u, 0u), c1 = c0;
-            if (ok) {
-                const uint4 v = src[pc];
-                decode_word_b4(v.x, k, ew, c0.x, c0.y);
-                decode_word_b4(v.y, k, ew, c0.z, c0.w);
-                decode_word_b4(v.z, k, ew, c1.x, c1.y);
-                decode_word_b4(v.w, k, ew, c1.z, c1.w);
-            }
+            if (ok) decode_piece<SLOT>(src[pc], k, ew, lut, b, c0, c1);
             uint8_t* dst = st + (2 * pc) * g.pb + slot * 16;
             *reinterpret_cast<uint4*>(dst) = c0;
             *reinterpret_cast<uint4*>(dst + g.pb) = c1;
@@ -186,29 +208,50 @@ __device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint
     }
 }
 
-__device__ __noinline__ void halo_decode(const HaloGeom g, int64_t T, uint8_t* st, int first, int stride, int k, int ew)
+// lut: the E4M3 table of a 5/6-bit word-slot input (nullptr: 4-bit codes).
+__device__ __noinline__ void halo_decode(const HaloGeom g, int64_t T, uint8_t* st, int first, int stride, int k, int ew,
+                                         const uint8_t* lut, int b)
 {
+    if (lut) {
+        switch (g.ldx >> 2) {
+        case 1: halo_decode_t<1, true>(g, T, st, first, stride, k, ew, lut, b); break;
+        case 2: halo_decode_t<2, true>(g, T, st, first, stride, k, ew, lut, b); break;
+        case 3: halo_decode_t<3, true>(g, T, st, first, stride, k, ew, lut, b); break;
+        default: halo_decode_t<4, true>(g, T, st, first, stride, k, ew, lut, b); break;
+        }
+        return;
+    }
     switch (g.ldx >> 2) {
-    case 1: halo_decode_t<1>(g, T, st, first, stride, k, ew); break;
-    case 2: halo_decode_t<2>(g, T, st, first, stride, k, ew); break;
-    case 3: halo_decode_t<3>(g, T, st, first, stride, k, ew); break;
-    default: halo_decode_t<4>(g, T, st, first, stride, k, ew); break;
+    case 1: halo_decode_t<1, false>(g, T, st, first, stride, k, ew, lut, b); break;
+    case 2: halo_decode_t<2, false>(g, T, st, first, stride, k, ew, lut, b); break;
+    case 3: halo_decode_t<3, false>(g, T, st, first, stride, k, ew, lut, b); break;
+    default: halo_decode_t<4, false>(g, T, st, first, stride, k, ew, lut, b); break;
     }
 }
 
 // Channel block cb (words 16 cb .. of each pixel) of tile T's halo.
-__device__ __noinline__ void halo_fill(const HaloGeom g, int64_t T, int cb, uint8_t* st, int lane, int k, int ew)
+__device__ __noinline__ void halo_fill(const HaloGeom g, int64_t T, int cb, uint8_t* st, int lane, int k, int ew,
+                                       const uint8_t* lut, int b)
 {
     const int nimg = (int)(T / g.tpi);
     const int p0 = (int)(T - (int64_t)nimg * g.tpi) * g.rows_out;
     const int w0 = cb * 16;
     const int npc = min(16, g.ldx - w0) >> 2;                      // pieces per slot (1..4)
     const uint32_t* xi = g.X + (int64_t)nimg * g.H * g.W * g.ldx + w0;
+    if (lut) {
+        switch (npc) {
+        case 1: halo_fill_t<1, true>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        case 2: halo_fill_t<2, true>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        case 3: halo_fill_t<3, true>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        default: halo_fill_t<4, true>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        }
+        return;
+    }
     switch (npc) {
-    case 1: halo_fill_t<1>(g, p0, xi, st, lane, k, ew); break;
-    case 2: halo_fill_t<2>(g, p0, xi, st, lane, k, ew); break;
-    case 3: halo_fill_t<3>(g, p0, xi, st, lane, k, ew); break;
-    default: halo_fill_t<4>(g, p0, xi, st, lane, k, ew); break;
+    case 1: halo_fill_t<1, false>(g, p0, xi, st, lane, k, ew, lut, b); break;
+    case 2: halo_fill_t<2, false>(g, p0, xi, st, lane, k, ew, lut, b); break;
+    case 3: halo_fill_t<3, false>(g, p0, xi, st, lane, k, ew, lut, b); break;
+    default: halo_fill_t<4, false>(g, p0, xi, st, lane, k, ew, lut, b); break;
     }
 }
 
@@ -244,6 +287,11 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
     const bool split = (half_cols % 16 == 0) && (half_cols % ep.out_cpw == 0);
     const int epi_warps = split ? 8 : 4;
     const int cbs = g.cblocks;
+    // E4M3 tables of 5/6-bit word-slot operands (4-bit codes decode by SWAR)
+    __shared__ uint8_t lut_a[64], lut_b[64];
+    const bool slot_a = fa.spw != 0;
+    if (slot_a) build_e4m3_lut(lut_a, fa, tid, kWsThreads);
+    if (fb.spw != 0) build_e4m3_lut(lut_b, fb, tid, kWsThreads);
     // the layout above must fit the dynamic allocation (uniform for the CTA)
     if ((uintptr_t)(reinterpret_cast<const volatile uint8_t*>(err) + 4 - smem_raw) > dynamic_smem_bytes()) {
         if (tid == 0) record_status(ep.status, ESB_ERR_INTERNAL);
@@ -288,7 +336,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
     if (!(bulk && warp == kWsProdWarp0)) {
         const int nbdec = bulk ? kWsThreads - 32 : kWsThreads;
         const int t = (bulk && warp > kWsProdWarp0) ? tid - 32 : tid;
-        ws_decode_b<FAST>(srcB, n0, K, fb, BN, nkb, sB, t, nbdec);
+        ws_decode_b<FAST>(srcB, n0, K, fb, BN, nkb, sB, t, nbdec, fb.spw ? lut_b : nullptr);
         fence_proxy_async_smem();
         if (warp == kWsMmaWarp) asm volatile("bar.sync 1, %0;" ::"r"(nbdec) : "memory");
         else asm volatile("bar.arrive 1, %0;" ::"r"(nbdec) : "memory");
@@ -320,7 +368,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
                 for (int64_t ti = 0; ti < my_tiles && !*err; ti++) {
                     if (!wait_or_abort(&rawb[s], ph, err)) { *err = 1; break; }
                     halo_decode(g, cta_in_n + ti * ctas_per_n, sA + s * g.stage_bytes, d * 32 + lane,
-                                kHaloDecoders * 32, fa.k, fa.ew);
+                                kHaloDecoders * 32, fa.k, fa.ew, slot_a ? lut_a : nullptr, fa.b);
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&full[s]);
@@ -342,7 +390,8 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
             const int64_t ti = (cbs == 1) ? it : it / cbs;
             const int cb = (int)(it - ti * cbs);
             if (!wait_or_abort(&empty[s], ph ^ 1u, err)) { *err = 1; break; }
-            halo_fill(g, cta_in_n + ti * ctas_per_n, cb, sA + s * g.stage_bytes, lane, fa.k, fa.ew);
+            halo_fill(g, cta_in_n + ti * ctas_per_n, cb, sA + s * g.stage_bytes, lane, fa.k, fa.ew,
+                      slot_a ? lut_a : nullptr, fa.b);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&full[s]);
@@ -465,8 +514,11 @@ static bool halo_plan(const esb_conv_desc& d, int P, int Q, int64_t ldx, const O
                       HaloPlan* hp, cudaError_t* err)
 {
     *err = cudaSuccess;
-    if (d.stride != 1 || fa.b != 4 || fa.planes != 1 || ldx % 4 != 0 || ldx > (1 << 20) || d.pad > d.r - 1 ||
-        d.pad > d.s - 1)
+    // 4-bit codes, or 5/6-bit codes in the word-slot layout (8 K slots per
+    // word, the same K per pixel word as 4-bit codes)
+    const bool slot8 = fa.spw == 8 && (fa.b == 5 || fa.b == 6);
+    if (d.stride != 1 || !(fa.b == 4 || slot8) || fa.planes != 1 || ldx % 4 != 0 || ldx > (1 << 20) ||
+        d.pad > d.r - 1 || d.pad > d.s - 1)
         return false;
     int lws = 0;
     while ((1 << lws) < d.w + d.pad) lws++;
@@ -513,7 +565,9 @@ bool conv_halo_ok(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int
 {
     HaloPlan hp;
     cudaError_t e;
-    return halo_plan(d, P, Q, ldx, make_opfmt(bx, kx), pick_bn(d.cout, out_cpw), out_cpw, &hp, &e);
+    OpFmt fa = make_opfmt(bx, kx);
+    if (bx == 5 || bx == 6) fa.spw = 8;               // as plan_slots for same-width input and filters
+    return halo_plan(d, P, Q, ldx, fa, pick_bn(d.cout, out_cpw), out_cpw, &hp, &e);
 }
 
 bool launch_conv_halo(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, const OpFmt& fa,

@@ -18,18 +18,19 @@
 //
 // Two kernels here share the decode and the epilogue (esb_tc.cuh) with the
 // halo convolution of esb_conv_halo.cu:
-//  * esb_gemm_ws_kernel (B resident): persistent, warp-specialised.  The
-//    CTA decodes its N-tile of B once into shared memory; 7 producer warps
-//    decode A K-blocks into a ring of up to 8 shared-memory stages; one MMA
-//    warp issues tcgen05.mma (M = 128, N = BN, K = 32) into one of two TMEM
-//    accumulators and commits each stage to the mbarrier that frees it;
-//    8 epilogue warps drain the other accumulator with tcgen05.ld, so the
-//    post-processing of tile i overlaps the MMAs of tile i+1 and the decode
-//    of later tiles (the paper's ping-pong buffers and overlapped timing
-//    graph, Sec. IV-C/IV-D).
-//  * esb_gemm_tc_kernel (B streamed): one 128 x BN tile per CTA; all warps
+//  * esb_gemm_ws_kernel: persistent, warp-specialised.  The CTA decodes
+//    its N-tile of B once into shared memory when it fits beside three A
+//    stages (B resident), else each stage carries the B block of its
+//    K-block too (B streamed); 7 producer warps decode the stages of a ring
+//    of up to 8; one MMA warp issues tcgen05.mma (M = 128, N = BN, K = 32)
+//    into one of two TMEM accumulators and commits each stage to the
+//    mbarrier that frees it; 8 epilogue warps drain the other accumulator
+//    with tcgen05.ld, so the post-processing of tile i overlaps the MMAs of
+//    tile i+1 and the decode of later tiles (the paper's ping-pong buffers
+//    and overlapped timing graph, Sec. IV-C/IV-D).
+//  * esb_gemm_tc_kernel (fallback): one 128 x BN tile per CTA; all warps
 //    decode A and B K-blocks into a ring of stages, one thread issues the
-//    MMAs.  Used when B does not fit in shared memory.
+//    MMAs.
 // Every mbarrier wait is bounded (kWaitLimitNs); on expiry the kernel records
 // ESB_ERR_TIMEOUT, stops issuing work, frees TMEM and returns.
 #include <cstdint>

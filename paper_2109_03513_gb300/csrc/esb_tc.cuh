@@ -496,7 +496,8 @@ __device__ __forceinline__ uint32_t epi_element(const EpiParams& ep, const EpiCt
     float y = __fmaf_rn(sc, af, bi);
     if (ep.residual) {
         const int rcpw = 32 / ep.res_b;
-        const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >> (ep.res_b * (int)(n % rcpw))) &
+        const int nq = (int)n / rcpw;                 // 32-bit: a column index is below 2^31
+        const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + nq) >> (ep.res_b * ((int)n - nq * rcpw))) &
                             ((1u << ep.res_b) - 1u);
         y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
     }
@@ -654,7 +655,8 @@ static __device__ __noinline__ uint32_t epi_word_b4(const EpiParams* __restrict_
             float y = __fmaf_rn(sc, af, bi);
             if (ep.residual) {
                 const int rcpw = 32 / ep.res_b;
-                const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + n / rcpw) >> (ep.res_b * (int)(n % rcpw))) &
+                const int nq = (int)n / rcpw;                 // 32-bit: a column index is below 2^31
+        const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + nq) >> (ep.res_b * ((int)n - nq * rcpw))) &
                                     ((1u << ep.res_b) - 1u);
                 y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
             }
@@ -824,6 +826,11 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
     __shared__ float sh_resimg[16];
     if (lres && warp == 0 && lane < 16) sh_resimg[lane] = code_image_f((uint32_t)lane, 4, ep.res_k);
     __shared__ float sh_rawT[128];                    // gen: the thresholds searched (raw or on y)
+    __shared__ float sh_gres[GEN ? 256 : 1];          // gen: images of the residual's codes
+    const bool gres = gen && !gen_raw && ep.residual;
+    if (gres)
+        for (int i = warp * 32 + lane; i < (1 << ep.res_b); i += epi_warps * 32)
+            sh_gres[i] = code_image_f((uint32_t)i, ep.res_b, ep.res_k);
     if (gen) {
         const int nthr = (1 << (ep.out.b - 1)) - 1;
         for (int i = warp * 32 + lane; i < nthr; i += epi_warps * 32)
@@ -900,6 +907,18 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                     }
                     float v[4];
                     uint32_t sg[4];
+                    // residual codes of the group's four columns: at most two words, one load each
+                    const int rcpw = gres ? 32 / ep.res_b : 1;
+                    uint32_t rw0 = 0u, rw1 = 0u;
+                    int rsl0 = 0;
+                    if (gres && mrow) {
+                        const int col0 = (int)(n0 + c + 4 * g);
+                        const int wq = col0 / rcpw;
+                        rsl0 = col0 - wq * rcpw;
+                        const uint32_t* rp = ep.residual + m * ep.res_ld + wq;
+                        rw0 = __ldg(rp);
+                        rw1 = (rsl0 + 3 >= rcpw && (int64_t)(wq + 1) * rcpw < N) ? __ldg(rp + 1) : rw0;
+                    }
 #pragma unroll
                     for (int i = 0; i < 4; i++) {
                         const int64_t n = n0 + c + 4 * g + i;
@@ -912,11 +931,12 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                             if (ep.scale) { sc = __ldg(ep.scale + nc); if (cx.dq) sc = __fmul_rn(sc, cx.dqs); }
                             const float bi = ep.bias ? __ldg(ep.bias + nc) : ep.bias0;
                             float y = __fmaf_rn(sc, __uint_as_float(r[i]) * acc_scale, bi);
-                            if (ep.residual && mrow) {
-                                const int rcpw = 32 / ep.res_b;
-                                const uint32_t rc = (__ldg(ep.residual + m * ep.res_ld + nc / rcpw) >>
-                                                     (ep.res_b * (int)(nc % rcpw))) & ((1u << ep.res_b) - 1u);
-                                y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+                            if (gres && mrow) {
+                                const int sl = rsl0 + i;
+                                const uint32_t wd = sl < rcpw ? rw0 : rw1;
+                                const uint32_t rc = (wd >> (ep.res_b * (sl < rcpw ? sl : sl - rcpw))) &
+                                                    ((1u << ep.res_b) - 1u);
+                                y = __fmaf_rn(ep.res_scale, sh_gres[rc], y);
                             }
                             y = apply_act(y, ep.act);
                             sg[i] = (__float_as_uint(y) >> 31) & (out_signed ? 1u : 0u);

@@ -154,3 +154,34 @@ def test_conv_filter_rows_walked_by_tap(c, fmt, r, stride):
     acc_o = o.conv2d_i64(X.reshape(n, h, w, ldx), fmt, W.reshape(cout, r, r, ldx), fmt, n, h, w, c, cout, r, r,
                          stride, pad).reshape(-1, cout)
     assert np.array_equal(acc.cpu().numpy().astype(np.int64), acc_o)
+
+
+@pytest.mark.parametrize("n,h,w,c,cout,r,pad,fmt", [
+    (2, 14, 14, 64, 64, 3, 1, (6, 3)),            # ResNet18 layer shape, one channel block
+    (2, 28, 28, 128, 96, 3, 1, (5, 2)),           # two channel blocks (register fill path)
+    (1, 14, 14, 128, 64, 3, 1, (6, 3)),           # two channel blocks, 6-bit
+    (2, 15, 30, 40, 48, 5, 2, (5, 2)),            # ragged channels, 5x5
+    (2, 16, 31, 96, 80, 1, 0, (6, 3)),            # 1x1
+])
+def test_conv_halo_word_slots(n, h, w, c, cout, r, pad, fmt):
+    """Stride-1 convolution of 5/6-bit codes on the halo kernel (word-slot K)."""
+    fx, fw = (fmt[0], fmt[1], False), (fmt[0], fmt[1], True)
+    assert esb.esb_conv2d_kernel(n, h, w, c, cout, r, r, 1, pad, esb.Fmt(*fx), esb.Fmt(*fw),
+                                 out_b=fmt[0]) == esb.ESB_CONV_KERNEL_HALO
+    x = synth.half_normal((n * h * w, c), seed=c + h).numpy()
+    wt = synth.he_normal((cout * r * r, c), fan_in=r * r * c, seed=cout + r).numpy()
+    ldx = esb.esb_row_words(c, fmt[0])
+    ax, _ = o.calibrate(x, *fx)
+    aw, _ = o.calibrate(wt, *fw)
+    X = o.project_packed(x, ax, *fx, ld_words=ldx)
+    W = o.project_packed(wt, aw, *fw, ld_words=ldx)
+    s0 = esb.esb_dequant_scale(ax, esb.Fmt(*fmt), aw, esb.Fmt(*fmt))
+    fo = (fmt[0], fmt[1], False)
+    ep = esb.Epilogue(scale0=s0, bias0=0.0, act=esb.ESB_ACT_RELU, alpha_out=0.6, fmt_out=esb.Fmt(*fo))
+    acc, _, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fx), dev_i32(W), esb.Fmt(*fw), n, h, w, c, cout, r, r,
+                                        1, pad, ep=ep, want_acc=True, want_codes=True)
+    acc_o = o.conv2d_i64(X.reshape(n, h, w, ldx), fmt, W.reshape(cout, r, r, ldx), fmt, n, h, w, c, cout, r, r,
+                         1, pad).reshape(-1, cout)
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), acc_o)
+    _, co = o.epilogue(acc_o, np.full(cout, s0, np.float32), np.zeros(cout, np.float32), esb.ESB_ACT_RELU, 0.6, fo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
