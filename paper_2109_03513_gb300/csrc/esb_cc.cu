@@ -264,6 +264,18 @@ esb_dwconv3_kernel(const uint32_t* __restrict__ X, int ldx, int kx, const uint32
             }
         }
         const int cvalid = C - w * CPW;               // channels of this word inside C
+        // per-channel scale and bias of the word's channels, once per item
+        float scv[CPW], biv[CPW];
+        if (!lean) {
+#pragma unroll
+            for (int j = 0; j < CPW; j++) {
+                const int c = w * CPW + j < C ? w * CPW + j : C - 1;
+                float sc = ep.scale ? __ldg(ep.scale + c) : ep.scale0;
+                if (dq) sc = __fmul_rn(sc, dqs);
+                scv[j] = sc;
+                biv[j] = ep.bias ? __ldg(ep.bias + c) : ep.bias0;
+            }
+        }
 #pragma unroll
         for (int uu = 0; uu < QT; uu++) {
             if (q0 + uu >= Q) break;
@@ -291,10 +303,7 @@ esb_dwconv3_kernel(const uint32_t* __restrict__ X, int ldx, int kx, const uint32
                 if (c < C) {
                     const int64_t o = pix * C + c;
                     if (ep.acc_out) ep.acc_out[o] = acc[uu][j];
-                    float sc = ep.scale ? __ldg(ep.scale + c) : ep.scale0;
-                    if (dq) sc = __fmul_rn(sc, dqs);
-                    const float bi = ep.bias ? __ldg(ep.bias + c) : ep.bias0;
-                    float y = __fmaf_rn(sc, (float)acc[uu][j], bi);
+                    float y = __fmaf_rn(scv[j], (float)acc[uu][j], biv[j]);
                     if (ep.residual) {
                         const uint32_t rc =
                             (__ldg(ep.residual + pix * ep.res_ld + c / rcpw) >> (ep.res_b * (c % rcpw))) & rmask;
@@ -538,10 +547,13 @@ cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
 
 // ------------------------------------------------------ global avg pool
 
-// One thread = one code word of one image: the HW pixels' words of that
-// channel group are read in turn (consecutive threads read consecutive
-// words of a pixel), their images summed exactly in int32 per channel, and
-// each sum scaled and requantised through the block's threshold table.
+// kPoolLanes threads = one code word of one image: each reads every
+// kPoolLanes-th pixel's word of that channel group and sums the images
+// exactly in int32 per channel; the partial sums are added by shuffles and
+// the first lane scales and requantises each sum through the block's
+// threshold table.
+constexpr int kPoolLanes = 8;
+
 __global__ void __launch_bounds__(128)
 esb_avgpool_word_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int k, int n, int HW, int C, int wout,
                         float scale, float alpha_out, ProjParams out, float* __restrict__ y_out,
@@ -551,24 +563,38 @@ esb_avgpool_word_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int 
     griddep_wait();
     if (codes_out) build_thresholds(T, out, alpha_out, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
     __syncthreads();
+    // kPoolLanes consecutive lanes share one (image, word): each sums every
+    // kPoolLanes-th pixel, then the partial sums meet by shuffles (integer
+    // sums: the result does not depend on the split)
     const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (t >= (int64_t)n * wout) return;
-    const int nn = (int)(t / wout), w = (int)(t - (t / wout) * wout);
+    const int sub = threadIdx.x & (kPoolLanes - 1);
+    const int64_t grp = t / kPoolLanes;
+    const bool live = grp < (int64_t)n * wout;
+    const int nn = live ? (int)(grp / wout) : 0, w = live ? (int)(grp - (grp / wout) * wout) : 0;
     const int cpw = 32 / b;
     const int ew = b - k - 1, N = (1 << ew) - 1;
     const uint32_t mask = (1u << b) - 1u;
     uint32_t word = 0;
-    if (w * cpw < C) {
-        int32_t acc[16];
+    const bool has = live && w * cpw < C;
+    int32_t acc[16];
 #pragma unroll
-        for (int j = 0; j < 16; j++) acc[j] = 0;
+    for (int j = 0; j < 16; j++) acc[j] = 0;
+    if (has) {
         const uint32_t* xp = X + (int64_t)nn * HW * ldx + w;
-        for (int i = 0; i < HW; i++) {
+        for (int i = sub; i < HW; i += kPoolLanes) {
             const uint32_t xw = __ldg(xp + (int64_t)i * ldx);
 #pragma unroll
             for (int j = 0; j < 16; j++)
                 if (j < cpw) acc[j] += code_image_i((xw >> (b * j)) & mask, b, k, ew, N);
         }
+    }
+#pragma unroll
+    for (int o = kPoolLanes / 2; o > 0; o >>= 1)
+#pragma unroll
+        for (int j = 0; j < 16; j++)
+            if (j < cpw) acc[j] += __shfl_xor_sync(0xffffffffu, acc[j], o);
+    if (!live || sub != 0) return;
+    if (has) {
 #pragma unroll
         for (int j = 0; j < 16; j++) {
             if (j >= cpw) break;
@@ -594,7 +620,7 @@ cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
     ProjParams out = make_proj_params(bo, ko, so, rounding);
     int64_t words = (C + (32 / b) - 1) / (32 / b);
     if (codes_out && ldo > words) words = ldo;          // also write the row's padding words
-    const int64_t total = (int64_t)n * words;
+    const int64_t total = (int64_t)n * words * kPoolLanes;
     esb_avgpool_word_kernel<<<(unsigned)((total + 127) / 128), 128, 0, st>>>(X, ldx, b, k, n, HW, C, (int)words, scale,
                                                                            alpha_out, out, y_out, codes_out, ldo);
     return cudaGetLastError();

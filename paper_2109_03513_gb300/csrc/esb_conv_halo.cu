@@ -44,6 +44,7 @@ struct HaloGeom {
     int ns;              // slots per plane (128 + (R-1) * Ws + S - 1)
     int pb;              // bytes per plane (ns * 16)
     int cblocks;         // channel blocks of 16 words
+    int spw;             // K slots per input word: 8 (4-bit codes, 5/6-bit word slots) or 16 (2/3-bit word slots)
     int stage_bytes;     // planes of one channel block (<= 8 planes), then raw rows
     int planes_bytes;    // the planes part of a stage
     int raw_bytes;       // raw code rows of a tile (one channel block only), or 0: register path
@@ -89,22 +90,55 @@ __device__ __forceinline__ void decode_word_slot8(uint32_t w, const uint8_t* lut
     hi = o[1];
 }
 
-// The two 16-byte chunks (planes 2pc, 2pc + 1) of one 4-word piece.
-template <bool SLOT>
-__device__ __forceinline__ void decode_piece(const uint4 v, int k, int ew, const uint8_t* lut, int b, uint4& c0,
-                                             uint4& c1)
+// One packed word of a 2- or 3-bit format in the word-slot layout (16 K
+// slots per word): a whole 16-byte plane entry.
+__device__ __forceinline__ uint4 decode_word_slot16(uint32_t w, const uint8_t* lut, int b)
 {
-    if (SLOT) {
-        decode_word_slot8(v.x, lut, b, c0.x, c0.y);
-        decode_word_slot8(v.y, lut, b, c0.z, c0.w);
-        decode_word_slot8(v.z, lut, b, c1.x, c1.y);
-        decode_word_slot8(v.w, lut, b, c1.z, c1.w);
-    } else {
-        decode_word_b4(v.x, k, ew, c0.x, c0.y);
-        decode_word_b4(v.y, k, ew, c0.z, c0.w);
-        decode_word_b4(v.z, k, ew, c1.x, c1.y);
-        decode_word_b4(v.w, k, ew, c1.z, c1.w);
+    const int cpw = 32 / b;
+    const uint32_t mask = (1u << b) - 1u;
+    uint32_t o[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int j = 0; j < 16; j++)
+        if (j < cpw) o[j >> 2] |= (uint32_t)lut[(w >> (b * j)) & mask] << (8 * (j & 3));
+    return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// Decode modes of the halo fill: 4-bit codes (SWAR), 5/6-bit word slots
+// (8 per word), 2/3-bit word slots (16 per word).
+enum { kHaloB4 = 0, kHaloSlot8 = 1, kHaloSlot16 = 2 };
+
+// One 4-word piece (piece pc of the pixel in slot `slot`) into its planes:
+// 2 planes (pc * 2 ..) for 8-slot words, 4 planes (pc * 4 ..) for 16-slot
+// words; ok = false writes the E4M3 zero (outside the image).
+template <int MODE>
+__device__ __forceinline__ void halo_store_piece(uint8_t* st, int pb, int slot, int pc, bool ok, const uint4 v, int k,
+                                                 int ew, const uint8_t* lut, int b)
+{
+    if (MODE == kHaloSlot16) {
+        uint8_t* dst = st + (4 * pc) * pb + slot * 16;
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; i++)
+            *reinterpret_cast<uint4*>(dst + i * pb) = ok ? decode_word_slot16(w[i], lut, b) : make_uint4(0u, 0u, 0u, 0u);
+        return;
     }
+    uint4 c0 = make_uint4(0u, 0u, 0u, 0u), c1 = c0;
+    if (ok) {
+        if (MODE == kHaloSlot8) {
+            decode_word_slot8(v.x, lut, b, c0.x, c0.y);
+            decode_word_slot8(v.y, lut, b, c0.z, c0.w);
+            decode_word_slot8(v.z, lut, b, c1.x, c1.y);
+            decode_word_slot8(v.w, lut, b, c1.z, c1.w);
+        } else {
+            decode_word_b4(v.x, k, ew, c0.x, c0.y);
+            decode_word_b4(v.y, k, ew, c0.z, c0.w);
+            decode_word_b4(v.z, k, ew, c1.x, c1.y);
+            decode_word_b4(v.w, k, ew, c1.z, c1.w);
+        }
+    }
+    uint8_t* dst = st + (2 * pc) * pb + slot * 16;
+    *reinterpret_cast<uint4*>(dst) = c0;
+    *reinterpret_cast<uint4*>(dst + pb) = c1;
 }
 
 // Producer: decode one channel block of one tile's halo into stage st.
@@ -112,7 +146,7 @@ __device__ __forceinline__ void decode_piece(const uint4 v, int k, int ew, const
 // (4 words = two 16-code chunks each) of its pixel.  The pieces of up to
 // 16 / NPC slot groups are loaded before any decode, so a fill makes at
 // most a few round trips to memory.
-template <int NPC, bool SLOT>
+template <int NPC, int MODE>
 __device__ __forceinline__ void halo_fill_t(const HaloGeom& g, int p0, const uint32_t* xi, uint8_t* st, int lane,
                                             int k, int ew, const uint8_t* lut, int b)
 {
@@ -144,13 +178,7 @@ __device__ __forceinline__ void halo_fill_t(const HaloGeom& g, int p0, const uin
             if (u >= per || slot >= g.ns) break;
             const bool ok = (okm >> u) & 1u;
 #pragma unroll
-            for (int pc = 0; pc < NPC; pc++) {
-                uint4 c0 = make_uint4(0u, 0u, 0u, 0u), c1 = c0;
-                if (ok) decode_piece<SLOT>(v[u][pc], k, ew, lut, b, c0, c1);
-                uint8_t* dst = st + (2 * pc) * g.pb + slot * 16;
-                *reinterpret_cast<uint4*>(dst) = c0;
-                *reinterpret_cast<uint4*>(dst + g.pb) = c1;
-            }
+            for (int pc = 0; pc < NPC; pc++) halo_store_piece<MODE>(st, g.pb, slot, pc, ok, v[u][pc], k, ew, lut, b);
         }
     }
 }
@@ -181,7 +209,7 @@ __device__ __forceinline__ void halo_issue_rows(const HaloGeom& g, int64_t T, ui
 
 // The decoders' share of one bulk-filled tile: slots first, first + stride,
 // ... (zeros for padding slots and rows outside the image).
-template <int NPC, bool SLOT>
+template <int NPC, int MODE>
 __device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint8_t* st, int first, int stride, int k,
                                               int ew, const uint8_t* lut, int b)
 {
@@ -198,13 +226,8 @@ __device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint
         const bool ok = rel >= 0 && hi < g.hr && j < g.W && (unsigned)h < (unsigned)g.H;
         const uint4* src = reinterpret_cast<const uint4*>(raw + ((size_t)hi * g.W + j) * g.ldx * 4);
 #pragma unroll
-        for (int pc = 0; pc < NPC; pc++) {
-            uint4 c0 = make_uint4(0u, 0u, 0u, 0u), c1 = c0;
-            if (ok) decode_piece<SLOT>(src[pc], k, ew, lut, b, c0, c1);
-            uint8_t* dst = st + (2 * pc) * g.pb + slot * 16;
-            *reinterpret_cast<uint4*>(dst) = c0;
-            *reinterpret_cast<uint4*>(dst + g.pb) = c1;
-        }
+        for (int pc = 0; pc < NPC; pc++)
+            halo_store_piece<MODE>(st, g.pb, slot, pc, ok, ok ? src[pc] : make_uint4(0u, 0u, 0u, 0u), k, ew, lut, b);
     }
 }
 
@@ -212,20 +235,29 @@ __device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint
 __device__ __noinline__ void halo_decode(const HaloGeom g, int64_t T, uint8_t* st, int first, int stride, int k, int ew,
                                          const uint8_t* lut, int b)
 {
+    if (lut && g.spw == 16) {
+        switch (g.ldx >> 2) {
+        case 1: halo_decode_t<1, kHaloSlot16>(g, T, st, first, stride, k, ew, lut, b); break;
+        case 2: halo_decode_t<2, kHaloSlot16>(g, T, st, first, stride, k, ew, lut, b); break;
+        case 3: halo_decode_t<3, kHaloSlot16>(g, T, st, first, stride, k, ew, lut, b); break;
+        default: halo_decode_t<4, kHaloSlot16>(g, T, st, first, stride, k, ew, lut, b); break;
+        }
+        return;
+    }
     if (lut) {
         switch (g.ldx >> 2) {
-        case 1: halo_decode_t<1, true>(g, T, st, first, stride, k, ew, lut, b); break;
-        case 2: halo_decode_t<2, true>(g, T, st, first, stride, k, ew, lut, b); break;
-        case 3: halo_decode_t<3, true>(g, T, st, first, stride, k, ew, lut, b); break;
-        default: halo_decode_t<4, true>(g, T, st, first, stride, k, ew, lut, b); break;
+        case 1: halo_decode_t<1, kHaloSlot8>(g, T, st, first, stride, k, ew, lut, b); break;
+        case 2: halo_decode_t<2, kHaloSlot8>(g, T, st, first, stride, k, ew, lut, b); break;
+        case 3: halo_decode_t<3, kHaloSlot8>(g, T, st, first, stride, k, ew, lut, b); break;
+        default: halo_decode_t<4, kHaloSlot8>(g, T, st, first, stride, k, ew, lut, b); break;
         }
         return;
     }
     switch (g.ldx >> 2) {
-    case 1: halo_decode_t<1, false>(g, T, st, first, stride, k, ew, lut, b); break;
-    case 2: halo_decode_t<2, false>(g, T, st, first, stride, k, ew, lut, b); break;
-    case 3: halo_decode_t<3, false>(g, T, st, first, stride, k, ew, lut, b); break;
-    default: halo_decode_t<4, false>(g, T, st, first, stride, k, ew, lut, b); break;
+    case 1: halo_decode_t<1, kHaloB4>(g, T, st, first, stride, k, ew, lut, b); break;
+    case 2: halo_decode_t<2, kHaloB4>(g, T, st, first, stride, k, ew, lut, b); break;
+    case 3: halo_decode_t<3, kHaloB4>(g, T, st, first, stride, k, ew, lut, b); break;
+    default: halo_decode_t<4, kHaloB4>(g, T, st, first, stride, k, ew, lut, b); break;
     }
 }
 
@@ -238,20 +270,29 @@ __device__ __noinline__ void halo_fill(const HaloGeom g, int64_t T, int cb, uint
     const int w0 = cb * 16;
     const int npc = min(16, g.ldx - w0) >> 2;                      // pieces per slot (1..4)
     const uint32_t* xi = g.X + (int64_t)nimg * g.H * g.W * g.ldx + w0;
+    if (lut && g.spw == 16) {
+        switch (npc) {
+        case 1: halo_fill_t<1, kHaloSlot16>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        case 2: halo_fill_t<2, kHaloSlot16>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        case 3: halo_fill_t<3, kHaloSlot16>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        default: halo_fill_t<4, kHaloSlot16>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        }
+        return;
+    }
     if (lut) {
         switch (npc) {
-        case 1: halo_fill_t<1, true>(g, p0, xi, st, lane, k, ew, lut, b); break;
-        case 2: halo_fill_t<2, true>(g, p0, xi, st, lane, k, ew, lut, b); break;
-        case 3: halo_fill_t<3, true>(g, p0, xi, st, lane, k, ew, lut, b); break;
-        default: halo_fill_t<4, true>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        case 1: halo_fill_t<1, kHaloSlot8>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        case 2: halo_fill_t<2, kHaloSlot8>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        case 3: halo_fill_t<3, kHaloSlot8>(g, p0, xi, st, lane, k, ew, lut, b); break;
+        default: halo_fill_t<4, kHaloSlot8>(g, p0, xi, st, lane, k, ew, lut, b); break;
         }
         return;
     }
     switch (npc) {
-    case 1: halo_fill_t<1, false>(g, p0, xi, st, lane, k, ew, lut, b); break;
-    case 2: halo_fill_t<2, false>(g, p0, xi, st, lane, k, ew, lut, b); break;
-    case 3: halo_fill_t<3, false>(g, p0, xi, st, lane, k, ew, lut, b); break;
-    default: halo_fill_t<4, false>(g, p0, xi, st, lane, k, ew, lut, b); break;
+    case 1: halo_fill_t<1, kHaloB4>(g, p0, xi, st, lane, k, ew, lut, b); break;
+    case 2: halo_fill_t<2, kHaloB4>(g, p0, xi, st, lane, k, ew, lut, b); break;
+    case 3: halo_fill_t<3, kHaloB4>(g, p0, xi, st, lane, k, ew, lut, b); break;
+    default: halo_fill_t<4, kHaloB4>(g, p0, xi, st, lane, k, ew, lut, b); break;
     }
 }
 
@@ -409,7 +450,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
             const uint32_t idesc = idesc_e4m3_f32(BN);
             const uint32_t b_base = smem_u32(sB), a_base = smem_u32(sA);
             const int ws = 1 << g.lws;
-            const int units_tap = g.ldx >> 2;                  // 32-code K steps per tap
+            const int units_tap = (g.ldx * g.spw) >> 5;        // 32-slot K steps per tap
             const bool r3 = g.R == 3 && g.S == 3;
             int s = 0;                                         // stage and phase of the next K-block
             uint32_t ph = 0u;
@@ -424,7 +465,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
                     tc_fence_after();
                     const uint32_t a_st = a_base + (uint32_t)(s * g.stage_bytes);
                     const uint32_t b_blk = b_base + (uint32_t)(cb * BN * kBK);   // block cb: 4 K steps on
-                    const int pairs = min(16, g.ldx - cb * 16) >> 2;
+                    const int pairs = (min(16, g.ldx - cb * 16) * g.spw) >> 5;   // K steps (plane pairs) of the block
                     if (r3 && ws == 64 && units_tap == 2 && BN == 64) {           // 56 x 56 x 64
                         halo_mma_fixed<64, 3, 3, 2, 2, 64>(d, a_st, b_blk, idesc, acc);
                     } else if (r3 && ws == 32 && units_tap == 4 && BN == 128) {   // 28 x 28 x 128
@@ -435,7 +476,7 @@ esb_conv_halo_kernel(HaloGeom g, RowsSrc srcB, int64_t N, int64_t K, OpFmt fa, O
                         for (int r = 0; r < g.R; r++) {
                             for (int sx = 0; sx < g.S; sx++) {
                                 const uint32_t at = a_st + (uint32_t)((r * ws + sx) * 16);
-                                const int kq0 = (r * g.S + sx) * units_tap + cb * 4;
+                                const int kq0 = (r * g.S + sx) * units_tap + cb * (g.spw >> 1);
                                 for (int j = 0; j < pairs; j++) {
                                     const int kq = kq0 + j;
                                     const uint32_t bb = b_base + (uint32_t)((kq >> 2) * BN * kBK + (kq & 3) * 32);
@@ -517,7 +558,8 @@ static bool halo_plan(const esb_conv_desc& d, int P, int Q, int64_t ldx, const O
     // 4-bit codes, or 5/6-bit codes in the word-slot layout (8 K slots per
     // word, the same K per pixel word as 4-bit codes)
     const bool slot8 = fa.spw == 8 && (fa.b == 5 || fa.b == 6);
-    if (d.stride != 1 || !(fa.b == 4 || slot8) || fa.planes != 1 || ldx % 4 != 0 || ldx > (1 << 20) ||
+    const bool slot16 = fa.spw == 16 && (fa.b == 2 || fa.b == 3);
+    if (d.stride != 1 || !(fa.b == 4 || slot8 || slot16) || fa.planes != 1 || ldx % 4 != 0 || ldx > (1 << 20) ||
         d.pad > d.r - 1 || d.pad > d.s - 1)
         return false;
     int lws = 0;
@@ -534,7 +576,8 @@ static bool halo_plan(const esb_conv_desc& d, int P, int Q, int64_t ldx, const O
     g.ns = kBM + (d.r - 1) * ws + d.s - 1;
     g.pb = g.ns * 16;
     g.cblocks = (int)((ldx + 15) / 16);
-    const int planes = (int)(ldx >= 16 ? 8 : ldx / 2);
+    g.spw = slot16 ? 16 : 8;
+    const int planes = (int)((ldx >= 16 ? 16 : ldx) * g.spw / 16);      // planes of one channel block
     g.planes_bytes = ((planes * g.pb + 127) / 128) * 128;
     // one channel block: the fill bulk-copies whole input rows to a raw area of the stage
     g.raw_bytes = (g.cblocks == 1) ? ((g.hr * d.w * (int)ldx * 4 + 127) / 128) * 128 : 0;
@@ -543,7 +586,7 @@ static bool halo_plan(const esb_conv_desc& d, int P, int Q, int64_t ldx, const O
     const int st_smem = halo_static_smem(err);
     if (st_smem < 0) return false;
     const int maxs = max_dyn_smem() - st_smem;
-    hp->K = (int64_t)d.r * d.s * ldx * 8;
+    hp->K = (int64_t)d.r * d.s * ldx * g.spw;
     hp->nkb = (int)((hp->K + kBK - 1) / kBK);
     static const int cands[] = {256, 240, 224, 208, 192, 176, 160, 144, 128, 112, 96, 80, 64, 48, 32, 16};
     for (int i = -1; i < (int)(sizeof(cands) / sizeof(cands[0])); i++) {
@@ -567,6 +610,7 @@ bool conv_halo_ok(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx, int
     cudaError_t e;
     OpFmt fa = make_opfmt(bx, kx);
     if (bx == 5 || bx == 6) fa.spw = 8;               // as plan_slots for same-width input and filters
+    if (bx == 2 || bx == 3) fa.spw = 16;
     return halo_plan(d, P, Q, ldx, fa, pick_bn(d.cout, out_cpw), out_cpw, &hp, &e);
 }
 

@@ -162,6 +162,9 @@ def test_conv_filter_rows_walked_by_tap(c, fmt, r, stride):
     (1, 14, 14, 128, 64, 3, 1, (6, 3)),           # two channel blocks, 6-bit
     (2, 15, 30, 40, 48, 5, 2, (5, 2)),            # ragged channels, 5x5
     (2, 16, 31, 96, 80, 1, 0, (6, 3)),            # 1x1
+    (2, 14, 14, 64, 64, 3, 1, (3, 1)),            # 3-bit: 16 K slots per word, one plane per word
+    (2, 14, 14, 96, 32, 3, 1, (3, 1)),            # 3-bit, 12-word pixels
+    (2, 15, 30, 40, 48, 3, 1, (2, 0)),            # 2-bit
 ])
 def test_conv_halo_word_slots(n, h, w, c, cout, r, pad, fmt):
     """Stride-1 convolution of 5/6-bit codes on the halo kernel (word-slot K)."""
