@@ -39,6 +39,8 @@
 
 #include "esb_tc.cuh"
 
+#include <type_traits>
+
 namespace esb {
 
 constexpr int kStages = 4;         // streamed kernel
@@ -135,6 +137,85 @@ struct ConvSrc {
         return words(x, wi);
     }
 };
+
+template <class T>
+constexpr bool kIsConv = std::is_same<T, ConvSrc>::value;
+
+// ---------------------------------------- im2col rows through a tap table
+//
+// The words of one K-block sit at the same taps and offsets in every row of
+// the tile, so the producer warp builds a table of them once per stage
+// (lane i: word w0 + i -> tap (r, s) and word offset from a row's tap-(0,0)
+// base) and each row's loads then need no running cursor: independent
+// address adds and loads, all in flight together.
+__device__ __forceinline__ void conv_tap_table(const ConvSrc& src, int64_t w0, int n, int4* tab, int lane)
+{
+    __syncwarp();                                     // the previous stage's readers are done
+    if (lane < n) {
+        const ConvSrc::Cursor c = src.cursor(w0 + lane);
+        tab[lane] = make_int4(c.r, c.s, (int)c.off, 0);
+    }
+    __syncwarp();
+}
+
+// 4-bit codes: the K-block's 16 words of row `row` (rows past M and taps
+// outside the image give the E4M3 zero), decoded and stored to stage row r.
+__device__ __forceinline__ void walk_b4_tab(const ConvSrc& src, const ConvSrc::Row& row, const int4* tab, int64_t k0,
+                                            int64_t K, const OpFmt& f, uint8_t* stage, int r)
+{
+    uint32_t wv[16];
+    uint32_t ok = 0u;
+#pragma unroll
+    for (int i = 0; i < 16; i++) {
+        const int4 e = tab[i];
+        const bool in = (k0 + i * 8 < K) && src.inside(row, e.x, e.y);
+        wv[i] = in ? __ldg(src.X + (row.base + e.z)) : 0u;
+        ok |= (in ? 1u : 0u) << i;
+    }
+    store_b4_words(wv, ok, k0, K, f, stage, r);
+}
+
+// Word-slot codes (see plan_slots): the K-block's NW words, CH at a time.
+template <int B>
+__device__ __forceinline__ void walk_slots_tab(const ConvSrc& src, const ConvSrc::Row& row, const int4* tab,
+                                               int64_t k0, const OpFmt& f, const uint8_t* lut, uint8_t* stage, int r)
+{
+    constexpr int CPW = 32 / B;
+    constexpr int SPW = CPW > 8 ? 16 : (CPW > 4 ? 8 : 4);
+    constexpr int NW = kBK / SPW;
+    constexpr int CH = NW > 16 ? 16 : NW;
+    const int64_t w0 = k0 / SPW;
+#pragma unroll 1
+    for (int c0 = 0; c0 < NW; c0 += CH) {
+        const int64_t left = f.korig - (w0 + c0) * CPW;
+        const int lim = left < 0 ? 0 : (left > CH * CPW ? CH * CPW : (int)left);
+        uint32_t wv[CH];
+        uint32_t ok = 0u;
+#pragma unroll
+        for (int i = 0; i < CH; i++) {
+            const int4 e = tab[c0 + i];
+            const bool in = (i * CPW < lim) && src.inside(row, e.x, e.y);
+            wv[i] = in ? __ldg(src.X + (row.base + e.z)) : 0u;
+            ok |= (in ? 1u : 0u) << i;
+        }
+        store_slot_words<B, CH>(wv, ok, lim, lut, stage, r, c0 * SPW / 16);
+    }
+}
+
+__device__ __forceinline__ void walk_row_tab(const ConvSrc& src, const ConvSrc::Row& row, const int4* tab,
+                                             int64_t k0, int64_t K, const OpFmt& f, const uint8_t* lut, uint8_t* stage,
+                                             int r)
+{
+    if (f.b == 4) { walk_b4_tab(src, row, tab, k0, K, f, stage, r); return; }
+    switch (f.b) {
+    case 2: walk_slots_tab<2>(src, row, tab, k0, f, lut, stage, r); return;
+    case 3: walk_slots_tab<3>(src, row, tab, k0, f, lut, stage, r); return;
+    case 5: walk_slots_tab<5>(src, row, tab, k0, f, lut, stage, r); return;
+    case 6: walk_slots_tab<6>(src, row, tab, k0, f, lut, stage, r); return;
+    case 7: walk_slots_tab<7>(src, row, tab, k0, f, lut, stage, r); return;
+    default: walk_slots_tab<8>(src, row, tab, k0, f, lut, stage, r); return;
+    }
+}
 
 // Fast decode of a full b = 4 unit (two words) at a cursor.
 template <class Src>
@@ -416,6 +497,7 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
     while ((int)tmem_cols < 2 * BN) tmem_cols <<= 1;
     // E4M3 tables of the word-walk decoder (widths other than 4)
     __shared__ uint8_t luta[256], lutb[256];
+    __shared__ int4 ptab[kWsProdWarps][32];          // producers' per-stage tap tables (im2col rows)
     if (fa.planes == 1) build_e4m3_lut(luta, fa, tid, kWsThreads);
     if (fb.planes == 1 && fb.b != 4) build_e4m3_lut(lutb, fb, tid, kWsThreads);
     // Epilogue column split: both halves of BN must be whole 16-column chunks
@@ -495,10 +577,25 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
 #pragma unroll
                 for (int q = 0; q < 4; q++) store_row_b4(st, lane + 32 * q, v[q], kw0, K, fa);
             } else if (fa.planes == 1 && srcA.linear()) {
-                // other widths: one word walk per row of the K-block
+                bool done = false;
+                if constexpr (kIsConv<SrcA>) {
+                    if (fa.b == 4 || fa.spw) {
+                        // im2col rows: the K-block's words through a tap table
+                        const int nw = kBK / (fa.b == 4 ? 8 : fa.spw);
+                        int4* tab = ptab[p];
+                        conv_tap_table(srcA, (int64_t)kb * nw, nw, tab, lane);
 #pragma unroll 1
-                for (int q = 0; q < 4; q++)
-                    walk_row_kblock(srcA, rows[q], (int64_t)kb * kBK, K, fa, luta, st, lane + 32 * q);
+                        for (int q = 0; q < 4; q++)
+                            walk_row_tab(srcA, rows[q], tab, (int64_t)kb * kBK, K, fa, luta, st, lane + 32 * q);
+                        done = true;
+                    }
+                }
+                if (!done) {
+                    // other widths: one word walk per row of the K-block
+#pragma unroll 1
+                    for (int q = 0; q < 4; q++)
+                        walk_row_kblock(srcA, rows[q], (int64_t)kb * kBK, K, fa, luta, st, lane + 32 * q);
+                }
             } else {
                 fill_stage_any(srcA, (cta_in_n + ti * ctas_per_n) * kBM, st, lane, (int64_t)kb * kBK, K, fa);
             }

@@ -289,6 +289,65 @@ __device__ __forceinline__ void build_e4m3_lut(uint8_t* lut, const OpFmt& f, int
     for (int c = t; c < (1 << f.b); c += nt) lut[c] = (uint8_t)code_to_e4m3((uint32_t)c, f);
 }
 
+// CH loaded words of B-bit codes in the word-slot layout (ok: word i
+// exists; lim: codes of the chunk inside K) -> their E4M3 slots, stored as
+// 16-byte units from unit g0 of stage row r.
+template <int B, int CH>
+__device__ __forceinline__ void store_slot_words(const uint32_t (&wv)[CH], uint32_t ok, int lim, const uint8_t* lut,
+                                                 uint8_t* stage, int r, int g0)
+{
+    constexpr int CPW = 32 / B;
+    constexpr int SPW = CPW > 8 ? 16 : (CPW > 4 ? 8 : 4);
+    constexpr uint32_t MASK = (1u << B) - 1u;
+    uint32_t o[CH * SPW / 4];
+#pragma unroll
+    for (int i = 0; i < CH; i++) {
+#pragma unroll
+        for (int q = 0; q < SPW / 4; q++) {
+            uint32_t v = 0u;
+#pragma unroll
+            for (int t = 0; t < 4; t++) {
+                const int j = q * 4 + t;
+                if (j < CPW) {
+                    const uint32_t byte = lut[(wv[i] >> (B * j)) & MASK];
+                    v |= ((i * CPW + j < lim) ? byte : 0u) << (8 * t);
+                }
+            }
+            o[i * (SPW / 4) + q] = ((ok >> i) & 1u) ? v : 0u;
+        }
+    }
+#pragma unroll
+    for (int g = 0; g < CH * SPW / 16; g++)
+        *reinterpret_cast<uint4*>(stage + swz(r, g0 + g)) = make_uint4(o[4 * g], o[4 * g + 1], o[4 * g + 2], o[4 * g + 3]);
+}
+
+// The 16 loaded words of a 4-bit K-block (ok: word i exists) decoded 8
+// codes at a time and stored as the 8 units of stage row r; codes past K
+// give the E4M3 zero.
+__device__ __forceinline__ void store_b4_words(const uint32_t (&wv)[16], uint32_t ok, int64_t k0, int64_t K,
+                                               const OpFmt& f, uint8_t* stage, int r)
+{
+#pragma unroll
+    for (int g = 0; g < 8; g++) {
+        uint32_t o[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+            const int i = 2 * g + h;
+            if ((ok >> i) & 1u) {
+                decode_word_b4(wv[i], f.k, f.ew, o[2 * h], o[2 * h + 1]);
+                const int64_t kk = k0 + i * 8;
+                if (kk + 8 > K) {                     // K tail: zero the codes past K
+                    uint32_t ml, mh;
+                    tail_masks((int)(K - kk), ml, mh);
+                    o[2 * h] &= ml;
+                    o[2 * h + 1] &= mh;
+                }
+            }
+        }
+        *reinterpret_cast<uint4*>(stage + swz(r, g)) = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
 // One K-block of a row in the word-slot layout (see plan_slots) for B-bit
 // codes: the block's words are loaded 16 at a time (independent loads in
 // flight), then each word's codes go through the E4M3 table to their fixed
@@ -318,27 +377,7 @@ __device__ __forceinline__ void walk_row_slots(const Src& src, const typename Sr
             ok |= (p ? 1u : 0u) << i;
             src.advance(cur, 1);
         }
-        uint32_t o[CH * SPW / 4];
-#pragma unroll
-        for (int i = 0; i < CH; i++) {
-#pragma unroll
-            for (int q = 0; q < SPW / 4; q++) {
-                uint32_t v = 0u;
-#pragma unroll
-                for (int t = 0; t < 4; t++) {
-                    const int j = q * 4 + t;
-                    if (j < CPW) {
-                        const uint32_t byte = lut[(wv[i] >> (B * j)) & MASK];
-                        v |= ((i * CPW + j < lim) ? byte : 0u) << (8 * t);
-                    }
-                }
-                o[i * (SPW / 4) + q] = ((ok >> i) & 1u) ? v : 0u;
-            }
-        }
-#pragma unroll
-        for (int g = 0; g < CH * SPW / 16; g++)
-            *reinterpret_cast<uint4*>(stage + swz(r, c0 * SPW / 16 + g)) =
-                make_uint4(o[4 * g], o[4 * g + 1], o[4 * g + 2], o[4 * g + 3]);
+        store_slot_words<B, CH>(wv, ok, lim, lut, stage, r, c0 * SPW / 16);
     }
 }
 
@@ -377,25 +416,7 @@ __device__ __forceinline__ void walk_row_kblock(const Src& src, const typename S
             ok |= (p ? 1u : 0u) << i;
             src.advance(cur, 1);
         }
-#pragma unroll
-        for (int g = 0; g < 8; g++) {
-            uint32_t o[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-            for (int h = 0; h < 2; h++) {
-                const int i = 2 * g + h;
-                if ((ok >> i) & 1u) {
-                    decode_word_b4(wv[i], f.k, f.ew, o[2 * h], o[2 * h + 1]);
-                    const int64_t kk = k0 + i * 8;
-                    if (kk + 8 > K) {                 // K tail: zero the codes past K
-                        uint32_t ml, mh;
-                        tail_masks((int)(K - kk), ml, mh);
-                        o[2 * h] &= ml;
-                        o[2 * h + 1] &= mh;
-                    }
-                }
-            }
-            *reinterpret_cast<uint4*>(stage + swz(r, g)) = make_uint4(o[0], o[1], o[2], o[3]);
-        }
+        store_b4_words(wv, ok, k0, K, f, stage, r);
         return;
     }
     const int cpw = f.cpw;
