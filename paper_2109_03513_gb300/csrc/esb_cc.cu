@@ -530,10 +530,81 @@ esb_maxpool_b4u_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H
     }
 }
 
+// Max pool of unsigned B-bit codes (B != 4) by the same rank rotation:
+// rank = (code + 2^k) mod 2^(B-1) orders the non-negative set (rank 0 is
+// the zero code), so each channel slot keeps the largest rank of its
+// window and the code comes back by the inverse rotation.  One thread =
+// one output word; blockIdx.y = image row (n, p); 32-bit indices.
+template <int B>
+__global__ void __launch_bounds__(256)
+esb_maxpool_rank_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H, int Wd, int C, int win, int stride,
+                        int pad, int P, int Q, uint32_t* __restrict__ Y, int64_t ldy)
+{
+    constexpr int CPW = 32 / B;
+    constexpr uint32_t RM = (1u << (B - 1)) - 1u;     // ranks live in B - 1 bits
+    const int np_ = blockIdx.y;
+    const int nn = np_ / P, p = np_ - (np_ / P) * P;
+    const int per_row = Q * (int)ldy;
+    const uint32_t rot = 1u << k;
+    const int words = (C + CPW - 1) / CPW;
+    const uint32_t zero = (uint32_t)((1 << (B - 1 - k)) - 1) << k;   // e = N, f = 0
+    for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < per_row; t += gridDim.x * blockDim.x) {
+        const int q = t / (int)ldy, w = t - (t / (int)ldy) * (int)ldy;
+        uint32_t best[CPW];
+#pragma unroll
+        for (int j = 0; j < CPW; j++) best[j] = 0u;
+        if (w < words) {
+            for (int r = 0; r < win; r++) {
+                const int h = p * stride - pad + r;
+                if (h < 0 || h >= H) continue;
+                const uint32_t* xr = X + ((int64_t)nn * H + h) * Wd * ldx + w;
+                for (int s2 = 0; s2 < win; s2++) {
+                    const int ww = q * stride - pad + s2;
+                    if (ww < 0 || ww >= Wd) continue;
+                    const uint32_t xw = __ldg(xr + (int64_t)ww * ldx);
+#pragma unroll
+                    for (int j = 0; j < CPW; j++) {
+                        const uint32_t rk = (((xw >> (B * j)) & RM) + rot) & RM;
+                        best[j] = best[j] > rk ? best[j] : rk;
+                    }
+                }
+            }
+        }
+        uint32_t word = 0u;
+#pragma unroll
+        for (int j = 0; j < CPW; j++) {
+            const bool in = w < words && w * CPW + j < C;
+            const uint32_t code = in ? ((best[j] + (RM + 1u) - rot) & RM) : zero;
+            word |= code << (B * j);
+        }
+        Y[(((int64_t)nn * P + p) * Q + q) * ldy + w] = word;
+    }
+}
+
+template <int B>
+static void launch_maxpool_rank(const uint32_t* X, int64_t ldx, int k, int n, int H, int Wd, int C, int win,
+                                int stride, int pad, int P, int Q, uint32_t* Y, int64_t ldy, cudaStream_t st)
+{
+    const int per_row = (int)(Q * ldy);
+    const dim3 grid((unsigned)((per_row + 255) / 256), (unsigned)(n * P));
+    esb_maxpool_rank_kernel<B><<<grid, 256, 0, st>>>(X, ldx, k, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
+}
+
 cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int H, int Wd, int C, int win,
                            int stride, int pad, int P, int Q, uint32_t* Y, int64_t ldy, cudaStream_t st,
                            int is_signed)
 {
+    if (b != 4 && !is_signed && (int64_t)n * P <= 65535 && (int64_t)Q * ldy < (1ll << 31)) {
+        switch (b) {
+        case 2: launch_maxpool_rank<2>(X, ldx, k, n, H, Wd, C, win, stride, pad, P, Q, Y, ldy, st); break;
+        case 3: launch_maxpool_rank<3>(X, ldx, k, n, H, Wd, C, win, stride, pad, P, Q, Y, ldy, st); break;
+        case 5: launch_maxpool_rank<5>(X, ldx, k, n, H, Wd, C, win, stride, pad, P, Q, Y, ldy, st); break;
+        case 6: launch_maxpool_rank<6>(X, ldx, k, n, H, Wd, C, win, stride, pad, P, Q, Y, ldy, st); break;
+        case 7: launch_maxpool_rank<7>(X, ldx, k, n, H, Wd, C, win, stride, pad, P, Q, Y, ldy, st); break;
+        default: launch_maxpool_rank<8>(X, ldx, k, n, H, Wd, C, win, stride, pad, P, Q, Y, ldy, st); break;
+        }
+        return cudaGetLastError();
+    }
     if (b == 4 && !is_signed && (int64_t)n * P <= 65535 && (int64_t)Q * ldy < (1ll << 31)) {
         const int per_row = (int)(Q * ldy);
         const dim3 grid((unsigned)((per_row + 255) / 256), (unsigned)(n * P));

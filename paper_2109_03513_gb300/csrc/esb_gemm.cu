@@ -729,6 +729,34 @@ static int streamed_bn(int64_t M, int64_t N, int out_cpw, int bn0)
     return best;
 }
 
+// N-tile width of the warp-specialised kernel with B resident when the
+// tiles do not fill the SMs (small M: a classifier, the last stages of a
+// network at small batch).  A CTA then decodes the A rows of its few tiles
+// (128 rows each, again for every N-tile) and its BN rows of B once; the
+// width (a multiple of 16 and of the output codes per word, at most bn0)
+// that minimises waves x tiles per CTA x (128 + BN), the wider on a tie.
+static int resident_bn(int64_t M, int64_t N, int out_cpw, int bn0)
+{
+    const int64_t sms = device_sm_count();
+    const int64_t mt = (M + kBM - 1) / kBM;
+    auto cost = [&](int bn) {
+        const int64_t nt = (N + bn - 1) / bn;
+        const int64_t per_n = nt >= sms ? 1 : sms / nt;
+        const int64_t waves = (nt + sms - 1) / sms;
+        const int64_t my = (mt + per_n - 1) / per_n;
+        return waves * my * (128 + bn);
+    };
+    if (mt * ((N + bn0 - 1) / bn0) >= sms) return bn0;
+    int best = bn0;
+    int64_t cbest = cost(bn0);
+    for (int bn = bn0 - 16; bn >= 16; bn -= 16) {
+        if (bn % out_cpw) continue;
+        const int64_t c = cost(bn);
+        if (c < cbest) { cbest = c; best = bn; }
+    }
+    return best;
+}
+
 static size_t gemm_smem_bytes(int BN)
 {
     return 1024 + (size_t)kStages * (kBM * kBK + (size_t)BN * kBK) + kStages * 8 + 16 + 512;
@@ -793,6 +821,7 @@ static bool launch_ws(const SrcA& a, const RowsSrc& b, int64_t M, int64_t N, int
     const int static_smem = ws_static_smem<SrcA>(err);
     if (static_smem < 0) return true;
     const int maxs = max_dyn_smem() - static_smem;
+    BN = resident_bn(M, N, ep.out_cpw, BN);
     WsLayout L = ws_layout(K, BN, maxs);
     int bstream = 0;
     if (L.stages < 3) {
@@ -975,7 +1004,8 @@ int conv_kernel_choice(const esb_conv_desc& d, int P, int Q, int64_t ldx, int bx
     cudaError_t e = cudaSuccess;
     const int st = ws_static_smem<ConvSrc>(&e);
     if (st < 0) return -1;
-    if (Kx > 0 && ws_layout(Kx, pick_bn(d.cout, cpw), max_dyn_smem() - st).stages >= 3) return ESB_CONV_KERNEL_IM2COL;
+    const int bn = resident_bn((int64_t)d.n * P * Q, d.cout, cpw, pick_bn(d.cout, cpw));   // as launch_ws
+    if (Kx > 0 && ws_layout(Kx, bn, max_dyn_smem() - st).stages >= 3) return ESB_CONV_KERNEL_IM2COL;
     return ESB_CONV_KERNEL_STREAMED;
 }
 

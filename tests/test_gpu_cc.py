@@ -95,6 +95,19 @@ def test_maxpool_unsigned_4bit_matches_oracle(n, h, w, c, win, stride, pad, k):
     assert np.array_equal(u32(Y), exp)
 
 
+@pytest.mark.parametrize("n,h,w,c,win,stride,pad,fmt", [(2, 56, 56, 64, 3, 2, 1, (3, 1)), (1, 11, 13, 23, 3, 2, 1, (5, 2)),
+                                                        (1, 9, 8, 16, 2, 2, 0, (6, 3)), (1, 6, 7, 5, 3, 1, 1, (2, 0)),
+                                                        (1, 7, 9, 30, 3, 2, 1, (7, 2)), (1, 5, 6, 9, 3, 1, 1, (8, 4))])
+def test_maxpool_unsigned_rank_matches_oracle(n, h, w, c, win, stride, pad, fmt):
+    # unsigned codes of widths other than 4: window maxima on the rotated ranks
+    b, k = fmt
+    codes = synth.uniform_ints((n * h * w, c), 0, 2 ** (b - 1), seed=h * c + b)
+    X = o.pack(codes, b, k, ld_words=esb.esb_row_words(c, b))
+    Y = esb.esb_maxpool_nhwc(dev_i32(X), esb.Fmt(b, k, False), n, h, w, c, win, stride, pad)
+    exp = o.maxpool_codes(X.reshape(n, h, w, -1), b, k, n, h, w, c, win, stride, pad).reshape(Y.shape[0], -1)
+    assert np.array_equal(u32(Y), exp)
+
+
 @pytest.mark.parametrize("n,hw,c,fmt", [(4, 49, 512, (4, 2)), (3, 49, 1280, (4, 2)), (2, 16, 37, (6, 3)),
                                         (2, 1, 5, (3, 1))])
 def test_avgpool_matches_oracle(n, hw, c, fmt):
