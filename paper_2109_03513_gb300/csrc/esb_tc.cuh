@@ -361,7 +361,6 @@ __device__ __forceinline__ void walk_row_slots(const Src& src, const typename Sr
     constexpr int SPW = CPW > 8 ? 16 : (CPW > 4 ? 8 : 4);
     constexpr int NW = kBK / SPW;                     // words per K-block: 8, 16 or 32
     constexpr int CH = NW > 16 ? 16 : NW;             // words per chunk
-    constexpr uint32_t MASK = (1u << B) - 1u;
     const int64_t w0 = k0 / SPW;
     typename Src::Cursor cur = src.cursor(w0);
 #pragma unroll 1
