@@ -571,11 +571,15 @@ esb_gemm_ws_kernel(SrcA srcA, RowsSrc srcB, int64_t M, int64_t N, int64_t K, OpF
                 typename SrcA::Cursor cur[4];
 #pragma unroll
                 for (int pc = 0; pc < 4; pc++) cur[pc] = srcA.cursor(kw0 + 4 * pc);
-                uint4 v[4][4];
-#pragma unroll
-                for (int q = 0; q < 4; q++) load_row_b4(srcA, rows[q], cur, kw0, K, zwa, v[q]);
-#pragma unroll
-                for (int q = 0; q < 4; q++) store_row_b4(st, lane + 32 * q, v[q], kw0, K, fa);
+                // one row at a time: a rolled loop keeps the producers' code
+                // small (the SM's instruction caches hold every role's loop;
+                // measured faster than four rows' loads in flight unrolled)
+#pragma unroll 1
+                for (int q = 0; q < 4; q++) {
+                    uint4 v[4];
+                    load_row_b4(srcA, rows[q], cur, kw0, K, zwa, v);
+                    store_row_b4(st, lane + 32 * q, v, kw0, K, fa);
+                }
             } else if (fa.planes == 1 && srcA.linear()) {
                 bool done = false;
                 if constexpr (kIsConv<SrcA>) {

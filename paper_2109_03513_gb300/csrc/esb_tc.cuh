@@ -1009,14 +1009,11 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 continue;
             }
             if constexpr (!GEN) {
-            // 4-bit output codes: 32 (or 16) columns per TMEM load
-            const int nc = LEAN4 ? 16 : ((c + 32 <= c_hi) ? 32 : 16);   // LEAN4: 16 columns a load (compact code)
-            uint32_t r[32];
-            if (nc == 32) {
-                tmem_ld32(taddr + (uint32_t)c, r);
-            } else {
-                tmem_ld16(taddr + (uint32_t)c, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-            }
+            // 4-bit output codes: 16 columns (two code words) per TMEM load
+            // (compact code: measured faster than 32-column loads)
+            constexpr int nc = 16;
+            uint32_t r[16];
+            tmem_ld16(taddr + (uint32_t)c, r);
             if (c + nc >= c_hi) {                     // every column of this warp is in registers
                 tc_fence_before();
                 __syncwarp();
@@ -1026,10 +1023,9 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
             const int64_t ncl64 = N - (n0 + c);
             const int ncl = ncl64 < nc ? (int)ncl64 : nc;
             const bool lean = lean_ok && ncl > 0;
-            uint32_t wds[4];
+            uint32_t wds[2];
 #pragma unroll
-            for (int h = 0; h < 4; h++) {
-                if (h * 8 >= nc) break;
+            for (int h = 0; h < 2; h++) {
                 uint32_t J = 0u, S = 0u;
                 const int live_h = ncl - 8 * h;       // nibbles of this word inside N
                 const uint32_t nib = live_h >= 8 ? 0xffffffffu : (live_h <= 0 ? 0u : (1u << (4 * live_h)) - 1u);
@@ -1104,21 +1100,17 @@ __device__ __forceinline__ void ws_epilogue(const EpiParams& ep, const float* th
                 }
             }
             if (mrow) {
-                // words w0 .. w0 + nc/8 - 1 of row m; vector stores only where
-                // the address is aligned and every word is inside the row
+                // words w0, w0 + 1 of row m; a vector store only where the
+                // address is aligned and both words are inside the row
                 const int64_t w0 = (n0 + c) >> 3;
                 uint32_t* dst = ep.codes_out + m * ep.ldo + w0;
-                const int nw = nc >> 3;
-                if (nw == 4 && ep.codes_vec >= 4 && (w0 & 3) == 0 && w0 + 4 <= ep.ldo) {
-                    *reinterpret_cast<uint4*>(dst) = make_uint4(wds[0], wds[1], wds[2], wds[3]);
-                } else if (ep.codes_vec >= 2 && (w0 & 1) == 0 && w0 + nw <= ep.ldo) {
-                    for (int q = 0; q < nw; q += 2) *reinterpret_cast<uint2*>(dst + q) = make_uint2(wds[q], wds[q + 1]);
+                if (ep.codes_vec >= 2 && (w0 & 1) == 0 && w0 + 2 <= ep.ldo) {
+                    *reinterpret_cast<uint2*>(dst) = make_uint2(wds[0], wds[1]);
                 } else {
-                    for (int q = 0; q < nw; q++)
+                    for (int q = 0; q < 2; q++)
                         if (w0 + q < ep.ldo) dst[q] = wds[q];
                 }
             }
-            c += nc - 16;                             // the loop adds the other 16
             }
         }
         // the last N-tile also fills the row's words past its columns (the
