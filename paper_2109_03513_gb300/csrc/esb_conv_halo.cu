@@ -225,7 +225,7 @@ __device__ __forceinline__ void halo_decode_t(const HaloGeom& g, int64_t T, uint
         const int h = p0 - g.pad + hi;
         const bool ok = rel >= 0 && hi < g.hr && j < g.W && (unsigned)h < (unsigned)g.H;
         const uint4* src = reinterpret_cast<const uint4*>(raw + ((size_t)hi * g.W + j) * g.ldx * 4);
-#pragma unroll
+#pragma unroll 1                                      // one piece at a time: a small loop body
         for (int pc = 0; pc < NPC; pc++)
             halo_store_piece<MODE>(st, g.pb, slot, pc, ok, ok ? src[pc] : make_uint4(0u, 0u, 0u, 0u), k, ew, lut, b);
     }

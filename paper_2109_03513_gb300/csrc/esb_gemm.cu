@@ -163,16 +163,20 @@ __device__ __forceinline__ void conv_tap_table(const ConvSrc& src, int64_t w0, i
 __device__ __forceinline__ void walk_b4_tab(const ConvSrc& src, const ConvSrc::Row& row, const int4* tab, int64_t k0,
                                             int64_t K, const OpFmt& f, uint8_t* stage, int r)
 {
-    uint32_t wv[16];
-    uint32_t ok = 0u;
+#pragma unroll 1
+    for (int hf = 0; hf < 2; hf++) {                  // two halves of 8 words: a small loop body
+        uint32_t wv[8];
+        uint32_t ok = 0u;
+        const int64_t kh = k0 + hf * 64;
 #pragma unroll
-    for (int i = 0; i < 16; i++) {
-        const int4 e = tab[i];
-        const bool in = (k0 + i * 8 < K) && src.inside(row, e.x, e.y);
-        wv[i] = in ? __ldg(src.X + (row.base + e.z)) : 0u;
-        ok |= (in ? 1u : 0u) << i;
+        for (int i = 0; i < 8; i++) {
+            const int4 e = tab[8 * hf + i];
+            const bool in = (kh + i * 8 < K) && src.inside(row, e.x, e.y);
+            wv[i] = in ? __ldg(src.X + (row.base + e.z)) : 0u;
+            ok |= (in ? 1u : 0u) << i;
+        }
+        store_b4_words<8>(wv, ok, kh, K, f, stage, r, 4 * hf);
     }
-    store_b4_words(wv, ok, k0, K, f, stage, r);
 }
 
 // Word-slot codes (see plan_slots): the K-block's NW words, CH at a time.
@@ -183,7 +187,7 @@ __device__ __forceinline__ void walk_slots_tab(const ConvSrc& src, const ConvSrc
     constexpr int CPW = 32 / B;
     constexpr int SPW = CPW > 8 ? 16 : (CPW > 4 ? 8 : 4);
     constexpr int NW = kBK / SPW;
-    constexpr int CH = NW > 16 ? 16 : NW;
+    constexpr int CH = 8;                             // words per chunk (a small loop body)
     const int64_t w0 = k0 / SPW;
 #pragma unroll 1
     for (int c0 = 0; c0 < NW; c0 += CH) {

@@ -321,14 +321,15 @@ __device__ __forceinline__ void store_slot_words(const uint32_t (&wv)[CH], uint3
         *reinterpret_cast<uint4*>(stage + swz(r, g0 + g)) = make_uint4(o[4 * g], o[4 * g + 1], o[4 * g + 2], o[4 * g + 3]);
 }
 
-// The 16 loaded words of a 4-bit K-block (ok: word i exists) decoded 8
-// codes at a time and stored as the 8 units of stage row r; codes past K
-// give the E4M3 zero.
-__device__ __forceinline__ void store_b4_words(const uint32_t (&wv)[16], uint32_t ok, int64_t k0, int64_t K,
-                                               const OpFmt& f, uint8_t* stage, int r)
+// NW loaded words of a 4-bit K-block from code k0 (ok: word i exists)
+// decoded 8 codes at a time and stored as the NW / 2 units of stage row r
+// from unit g0; codes past K give the E4M3 zero.
+template <int NW>
+__device__ __forceinline__ void store_b4_words(const uint32_t (&wv)[NW], uint32_t ok, int64_t k0, int64_t K,
+                                               const OpFmt& f, uint8_t* stage, int r, int g0)
 {
 #pragma unroll
-    for (int g = 0; g < 8; g++) {
+    for (int g = 0; g < NW / 2; g++) {
         uint32_t o[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
         for (int h = 0; h < 2; h++) {
@@ -344,7 +345,7 @@ __device__ __forceinline__ void store_b4_words(const uint32_t (&wv)[16], uint32_
                 }
             }
         }
-        *reinterpret_cast<uint4*>(stage + swz(r, g)) = make_uint4(o[0], o[1], o[2], o[3]);
+        *reinterpret_cast<uint4*>(stage + swz(r, g0 + g)) = make_uint4(o[0], o[1], o[2], o[3]);
     }
 }
 
@@ -360,7 +361,7 @@ __device__ __forceinline__ void walk_row_slots(const Src& src, const typename Sr
     constexpr int CPW = 32 / B;
     constexpr int SPW = CPW > 8 ? 16 : (CPW > 4 ? 8 : 4);
     constexpr int NW = kBK / SPW;                     // words per K-block: 8, 16 or 32
-    constexpr int CH = NW > 16 ? 16 : NW;             // words per chunk
+    constexpr int CH = 8;                             // words per chunk (a small loop body)
     const int64_t w0 = k0 / SPW;
     typename Src::Cursor cur = src.cursor(w0);
 #pragma unroll 1
@@ -415,7 +416,7 @@ __device__ __forceinline__ void walk_row_kblock(const Src& src, const typename S
             ok |= (p ? 1u : 0u) << i;
             src.advance(cur, 1);
         }
-        store_b4_words(wv, ok, k0, K, f, stage, r);
+        store_b4_words<16>(wv, ok, k0, K, f, stage, r, 0);
         return;
     }
     const int cpw = f.cpw;
