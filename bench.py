@@ -622,9 +622,10 @@ def _cc_sweep(esb, torch, timeit, hbm):
     (fused scale, bias, ReLU6 and requantisation, codes out), the ResNet18
     stem max pool 112 -> 56 and the global average pools of ResNet18 (7x7x512)
     and MobileNetV2 (7x7x1280), all ESB(4,2).  Algorithmic bytes = input
-    codes + output codes (+ weights, scale and bias).  Each call reads the next
-    of several input copies (over 3 x L2 in total), so inputs come from HBM;
-    codes are uniformly drawn words (timing only)."""
+    codes + output codes (+ weights, scale and bias).  Each point is a CUDA
+    graph of one call per input copy (over 3 x L2 of copies in total, so
+    inputs come from HBM), replayed; the figure is device time per call,
+    without host launch gaps.  Codes are uniformly drawn words (timing only)."""
     dev = torch.device("cuda")
     g = torch.Generator(device=dev).manual_seed(0)
     fx, fw = esb.Fmt(4, 2, False), esb.Fmt(4, 2, True)
@@ -633,11 +634,24 @@ def _cc_sweep(esb, torch, timeit, hbm):
 
     def copies(rows, ld, unsigned):
         nbytes = rows * ld * 4
-        nx = max(1, min(256, -(-span // nbytes)))
+        nx = max(3, min(256, -(-span // nbytes)))
         c = torch.randint(0, 2 ** 32, (nx * rows, ld), generator=g, device=dev, dtype=torch.int64).to(torch.int32)
         if unsigned:
             c &= 0x77777777
         return [c[i * rows:(i + 1) * rows] for i in range(nx)], nbytes
+
+    def graphed(calls, reps=5):
+        s_ = torch.cuda.Stream()
+        s_.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s_):
+            for f in calls[:3]:
+                f()
+        torch.cuda.current_stream().wait_stream(s_)
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr):
+            for f in calls:
+                f()
+        return timeit(gr.replay, reps) / len(calls)
 
     res = []
     for h, c, stride in [(112, 32, 1), (112, 96, 2), (56, 144, 1), (56, 144, 2), (28, 192, 1), (14, 384, 1),
@@ -651,28 +665,23 @@ def _cc_sweep(esb, torch, timeit, hbm):
         bias = torch.zeros((c,), dtype=torch.float32, device=dev)
         ep = esb.Epilogue(scale=scale, bias=bias, act=esb.ESB_ACT_RELU6, alpha_out=0.29, fmt_out=fx)
         oc = torch.empty((n * P * P, ld), dtype=torch.int32, device=dev)
-        it = [0]
 
-        def f():
-            X = Xs[it[0] % len(Xs)]
-            it[0] += 1
-            esb.esb_conv2d_nhwc(X, fx, W, fw, n, h, h, c, c, 3, 3, stride, 1, groups=c, ep=ep, want_acc=False,
-                                want_codes=True, out_codes=oc)
+        def dw(X):
+            return lambda: esb.esb_conv2d_nhwc(X, fx, W, fw, n, h, h, c, c, 3, 3, stride, 1, groups=c, ep=ep,
+                                               want_acc=False, want_codes=True, out_codes=oc)
 
-        us = timeit(f, 20)
+        us = graphed([dw(X) for X in Xs])
         byt = xb + oc.numel() * 4 + W.numel() * 4 + 8 * c
         res.append({"dwconv": [n, h, h, c, stride], "fmt": [4, 2], "us": round(us, 2),
                     "GB/s": round(byt / us / 1e3, 1), "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
         del Xs, oc
     Xs, xb = copies(n * 112 * 112, 8, True)
     Y = torch.empty((n * 56 * 56, 8), dtype=torch.int32, device=dev)
-    it = [0]
 
-    def mp():
-        esb.esb_maxpool_nhwc(Xs[it[0] % len(Xs)], fx, n, 112, 112, 64, 3, 2, 1, out=Y)
-        it[0] += 1
+    def mp(X):
+        return lambda: esb.esb_maxpool_nhwc(X, fx, n, 112, 112, 64, 3, 2, 1, out=Y)
 
-    us = timeit(mp, 20)
+    us = graphed([mp(X) for X in Xs])
     byt = xb + Y.numel() * 4
     res.append({"maxpool": [n, 112, 112, 64, 3, 2], "fmt": [4, 2], "us": round(us, 2),
                 "GB/s": round(byt / us / 1e3, 1), "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
@@ -680,13 +689,11 @@ def _cc_sweep(esb, torch, timeit, hbm):
     for c in (512, 1280):
         ld = esb.esb_row_words(c, 4)
         Xs, xb = copies(n * 49, ld, True)
-        it = [0]
 
-        def ap():
-            esb.esb_avgpool_nhwc(Xs[it[0] % len(Xs)], fx, n, 49, c, 1.0 / 49, 0.5, fx)
-            it[0] += 1
+        def ap(X):
+            return lambda: esb.esb_avgpool_nhwc(X, fx, n, 49, c, 1.0 / 49, 0.5, fx)
 
-        us = timeit(ap, 20)
+        us = graphed([ap(X) for X in Xs], reps=20)
         byt = xb + n * ld * 4
         res.append({"avgpool": [n, 7, 7, c], "fmt": [4, 2], "us": round(us, 2),
                     "GB/s": round(byt / us / 1e3, 1), "frac_hbm": round(byt / us / 1e3 / hbm, 3)})
@@ -828,7 +835,9 @@ def run_network(args, name):
         stream = torch.cuda.Stream(device=dev)
         with torch.cuda.stream(stream):
             rn.begin("infer")
+            t_host = time.perf_counter()
             fn(rn, x, batch)
+            t_host = time.perf_counter() - t_host         # host time to enqueue one eager pass
             torch.cuda.synchronize()
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g, stream=stream):
@@ -850,8 +859,10 @@ def run_network(args, name):
             ck = clocks.stop(0)
             t_fwd = e0.elapsed_time(e1) / K * 1e-3
             # per-layer device times: one eager pass queued behind a device sleep
+            # that outlasts its host enqueue time (3x margin at up to 2.1 GHz), so
+            # that every layer is queued before the device reaches it
             rn.marks = []
-            torch.cuda._sleep(5_000_000)
+            torch.cuda._sleep(int(min(2e9, max(5e6, 3.0 * t_host * 2.1e9))))
             m0 = torch.cuda.Event(enable_timing=True)
             m0.record(stream)
             rn.begin("infer")

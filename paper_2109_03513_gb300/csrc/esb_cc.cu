@@ -7,6 +7,7 @@
 //   * global average pooling: exact integer sum of the images per channel,
 //     then one fp32 scale and ESB requantisation.
 #include <cstdint>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
 #include "esb_common.cuh"
@@ -320,31 +321,251 @@ esb_dwconv3_kernel(const uint32_t* __restrict__ X, int ldx, int kx, const uint32
     }
 }
 
-template <int B, int STRIDE>
-static cudaError_t launch_dw3(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int kx,
-                              const uint32_t* W, int64_t ldw, int kw, const CcEpi& ep, cudaStream_t st)
+// Depthwise 3x3 of 4-bit codes on packed fp16 pairs.  Every 4-bit image is
+// an integer of magnitude at most 12, so every partial sum of the 9 taps is
+// an integer of magnitude at most 9 * 12 * 12 = 1296 < 2^11: fp16 holds each
+// one exactly and a fused multiply-add of two such pairs never rounds (the
+// host takes this kernel only when 9 * max|Ix| * max|Iw| <= 2048).  One
+// half2 = the images of two neighbouring channels (one byte of a code
+// word), so one instruction does two channels' multiply-adds and one table
+// load decodes two codes.  The sums never take the value -0 (they start at
+// +0, and an exact zero sum rounds to +0), so their conversion to float is
+// the integer accumulator's.  Work items, the strip walk and the epilogue
+// are those of the integer kernel above; the next filter row's input words
+// are loaded while the current row is multiplied.
+template <int STRIDE>
+__global__ void __launch_bounds__(128, 6)
+esb_dwconv3_b4h_kernel(const uint32_t* __restrict__ X, int ldx, int kx, const uint32_t* __restrict__ W, int ldw,
+                       int kw, int H, int Wd, int C, int pad, int P, int Q, int QS, int rows, CcEpi ep)
 {
     constexpr int QT = STRIDE == 1 ? 4 : 2;
-    const int QS = (Q + QT - 1) / QT;
-    const int rows = d.n * P;
-    const int64_t total = (int64_t)rows * QS * ep.ldo;
-    int64_t blocks = (total + 127) / 128;
-    // one resident wave (each block's set-up -- filter table, thresholds --
-    // is then paid once per block and amortised over many items)
+    constexpr int NIN = (QT - 1) * STRIDE + 3;
+    extern __shared__ __half2 wtab2[];                // [9][words * 4] filter images, channel pairs
+    __shared__ __half2 lut2[256];                     // code byte -> (image of low nibble, image of high nibble)
+    __shared__ float T[128];
+    __shared__ float Rs[8];
+    const int words = (C + 7) / 8;
+    const int cp2 = words * 4;
+    const int ewx = 3 - kx, Nx = (1 << ewx) - 1;
+    const int eww = 3 - kw, Nw = (1 << eww) - 1;
+    griddep_wait();
+    for (int i = threadIdx.x; i < 256; i += blockDim.x)
+        lut2[i] = __halves2half2(__int2half_rn(code_image_i((uint32_t)i & 15u, 4, kx, ewx, Nx)),
+                                 __int2half_rn(code_image_i((uint32_t)i >> 4, 4, kx, ewx, Nx)));
+    for (int i = threadIdx.x; i < 9 * words; i += blockDim.x) {
+        const int t = i / words, w = i - (i / words) * words;
+        const uint32_t fw = __ldg(W + t * ldw + w);
+#pragma unroll
+        for (int m = 0; m < 4; m++)
+            wtab2[t * cp2 + w * 4 + m] =
+                __halves2half2(__int2half_rn(code_image_i((fw >> (8 * m)) & 15u, 4, kw, eww, Nw)),
+                               __int2half_rn(code_image_i((fw >> (8 * m + 4)) & 15u, 4, kw, eww, Nw)));
+    }
+    const float alpha_out = ep.alpha_out_dev ? __ldg(ep.alpha_out_dev) : ep.alpha_out;
+    if (ep.codes_out) build_thresholds(T, ep.out, alpha_out, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
+    const bool dq = ep.alpha_a_dev && ep.alpha_b_dev;
+    const float dqs = dq ? __fmul_rn(__ldg(ep.alpha_a_dev), __ldg(ep.alpha_b_dev)) * ep.dq_pow2 : 1.0f;
+    const float sc_fixed = ep.scale ? 0.0f : (dq ? __fmul_rn(ep.scale0, dqs) : ep.scale0);
+    const bool b4 = ep.out.b == 4 && ep.codes_out;
+    const bool lean = b4 && ep.acc24 && !ep.scale && !ep.bias && !ep.residual && !ep.acc_out && !ep.y_out &&
+                      sc_fixed > 0.0f && (!ep.out.is_signed || ep.act != ESB_ACT_NONE);
+    // codes only, any scale and bias: the word's 8 codes from their buckets at once
+    const bool words8 = b4 && !lean && !ep.residual && !ep.acc_out && !ep.y_out;
+    const uint32_t sgn_out = ep.out.is_signed ? 1u : 0u;
+    __syncthreads();
+    if (lean && threadIdx.x < 7) Rs[threadIdx.x] = acc_raw_threshold(sc_fixed, ep.bias0, T[threadIdx.x], ep.act, 1.0f);
+    __syncthreads();
+    Thr7 t7, r7;
+#pragma unroll
+    for (int i = 0; i < 7; i++) {
+        t7.t[i] = b4 ? T[i] : 0.0f;
+        r7.t[i] = lean ? Rs[i] : 0.0f;
+    }
+    const int rcpw = ep.residual ? 32 / ep.res_b : 1;
+    const uint32_t rmask = ep.residual ? (1u << ep.res_b) - 1u : 0u;
+    const uint32_t zx = 0x11111111u * (uint32_t)fmt_zero_code(4, kx);
+    uint32_t zo = 0u;
+    for (int j = 0; j < 32 / ep.out.b; j++) zo |= ep.out.zero_code << (ep.out.b * j);
+    const int ldo = (int)ep.ldo;
+    const int upr = QS * ldo;
+    const int total = rows * upr;
+    for (int it = blockIdx.x * blockDim.x + threadIdx.x; it < total; it += gridDim.x * blockDim.x) {
+        const int row = it / upr;                     // n * P + p
+        const int u = it - row * upr;
+        const int qs = u / ldo;
+        const int w = u - qs * ldo;
+        const int nn = row / P;
+        const int p = row - nn * P;
+        const int q0 = qs * QT;
+        const int64_t obase = ((int64_t)row * Q + q0) * ldo + w;
+        if (w >= words) {
+            if (ep.codes_out) {
+#pragma unroll
+                for (int uu = 0; uu < QT; uu++)
+                    if (q0 + uu < Q) ep.codes_out[obase + (int64_t)uu * ldo] = zo;
+            }
+            continue;
+        }
+        const int c0 = q0 * STRIDE - pad;
+        const int h0 = p * STRIDE - pad;
+        const uint32_t* xim = X + (int64_t)nn * H * Wd * ldx + w;
+        // input words of filter row r (rows outside the image read as zero codes)
+        auto load_row = [&](uint32_t (&xv)[NIN], int r) {
+            const int h = h0 + r;
+            const bool hin = (unsigned)h < (unsigned)H;
+            const uint32_t* xrow = xim + (int64_t)h * Wd * ldx;
+#pragma unroll
+            for (int c = 0; c < NIN; c++) {
+                const int col = c0 + c;
+                xv[c] = (hin && (unsigned)col < (unsigned)Wd) ? __ldg(xrow + (int64_t)col * ldx) : zx;
+            }
+        };
+        __half2 acc[QT][4];
+#pragma unroll
+        for (int uu = 0; uu < QT; uu++)
+#pragma unroll
+            for (int m = 0; m < 4; m++) acc[uu][m] = __float2half2_rn(0.0f);
+        uint32_t xw[NIN], xn[NIN];
+        load_row(xw, 0);
+#pragma unroll 1
+        for (int r = 0; r < 3; r++) {
+            if (r < 2) load_row(xn, r + 1);
+            __half2 wf[3][4];
+#pragma unroll
+            for (int s2 = 0; s2 < 3; s2++)
+#pragma unroll
+                for (int m = 0; m < 4; m++) wf[s2][m] = wtab2[(r * 3 + s2) * cp2 + w * 4 + m];
+#pragma unroll
+            for (int c = 0; c < NIN; c++) {
+                __half2 img[4];
+#pragma unroll
+                for (int m = 0; m < 4; m++) img[m] = lut2[__byte_perm(xw[c], 0u, 0x4440u + (uint32_t)m)];
+#pragma unroll
+                for (int uu = 0; uu < QT; uu++) {
+                    const int s2 = c - uu * STRIDE;
+                    if (s2 >= 0 && s2 < 3) {
+#pragma unroll
+                        for (int m = 0; m < 4; m++) acc[uu][m] = __hfma2(img[m], wf[s2][m], acc[uu][m]);
+                    }
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < NIN; c++) xw[c] = xn[c];
+        }
+        const int cvalid = C - w * 8;
+        float scv[8], biv[8];
+        if (!lean) {
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                const int c = w * 8 + j < C ? w * 8 + j : C - 1;
+                float sc = ep.scale ? __ldg(ep.scale + c) : ep.scale0;
+                if (dq) sc = __fmul_rn(sc, dqs);
+                scv[j] = sc;
+                biv[j] = ep.bias ? __ldg(ep.bias + c) : ep.bias0;
+            }
+        }
+#pragma unroll
+        for (int uu = 0; uu < QT; uu++) {
+            if (q0 + uu >= Q) break;
+            const int64_t ow = obase + (int64_t)uu * ldo;
+            float a[8];
+#pragma unroll
+            for (int m = 0; m < 4; m++) {
+                const float2 f2 = __half22float2(acc[uu][m]);
+                a[2 * m] = f2.x;
+                a[2 * m + 1] = f2.y;
+            }
+            if (lean) {
+                uint32_t J = 0u;
+#pragma unroll
+                for (int j = 0; j < 8; j++) {
+                    const float v = a[j];
+                    const bool b2 = v >= r7.t[3];
+                    const bool b1 = v >= (b2 ? r7.t[5] : r7.t[1]);
+                    const bool b0 = v >= (b2 ? (b1 ? r7.t[6] : r7.t[4]) : (b1 ? r7.t[2] : r7.t[0]));
+                    const uint32_t jb = (b2 ? 4u : 0u) | (b1 ? 2u : 0u) | (b0 ? 1u : 0u);
+                    J |= (j < cvalid ? jb : 0u) << (4 * j);
+                }
+                ep.codes_out[ow] = codes8_b4(J, 0u, ep.out.k);
+                continue;
+            }
+            if (words8) {
+                // per element: y = fma(scale, acc, bias), the activation, then
+                // the bucket of |y| (zero for negatives of an unsigned set);
+                // codes8_b4 turns buckets and signs into the word (zero
+                // buckets keep sign 0), as project_by_thr7 does per code
+                uint32_t J = 0u, S = 0u;
+#pragma unroll
+                for (int j = 0; j < 8; j++) {
+                    const uint32_t u = __float_as_uint(cc_act(__fmaf_rn(scv[j], a[j], biv[j]), ep.act));
+                    const uint32_t neg = u >> 31;
+                    const uint32_t jb = bucket7(__uint_as_float(u & 0x7fffffffu), t7);
+                    J |= ((j < cvalid && (sgn_out | (neg ^ 1u))) ? jb : 0u) << (4 * j);
+                    S |= (neg & sgn_out) << (4 * j + 3);
+                }
+                ep.codes_out[ow] = codes8_b4(J, S, ep.out.k);
+                continue;
+            }
+            const int64_t pix = (int64_t)row * Q + q0 + uu;
+            uint32_t word = 0;
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                const int c = w * 8 + j;
+                uint32_t code = ep.out.zero_code;
+                if (c < C) {
+                    const int64_t o = pix * C + c;
+                    if (ep.acc_out) ep.acc_out[o] = (int32_t)a[j];
+                    float y = __fmaf_rn(scv[j], a[j], biv[j]);
+                    if (ep.residual) {
+                        const uint32_t rc =
+                            (__ldg(ep.residual + pix * ep.res_ld + c / rcpw) >> (ep.res_b * (c % rcpw))) & rmask;
+                        y = __fmaf_rn(ep.res_scale, code_image_f(rc, ep.res_b, ep.res_k), y);
+                    }
+                    y = cc_act(y, ep.act);
+                    if (ep.y_out) ep.y_out[o] = y;
+                    if (ep.codes_out) code = b4 ? project_by_thr7(y, t7, ep.out) : project_by_table(y, T, ep.out);
+                }
+                word |= code << (ep.out.b * j);
+            }
+            if (ep.codes_out) ep.codes_out[ow] = word;
+        }
+    }
+}
+
+// One resident wave of blocks (each block's set-up -- filter table,
+// thresholds -- is then paid once per block and amortised over many items).
+template <class Kern>
+static cudaError_t launch_dw_wave(Kern kern, size_t smem, int64_t items, const esb_conv_desc& d, int P, int Q, int QS,
+                                  const uint32_t* X, int64_t ldx, int kx, const uint32_t* W, int64_t ldw, int kw,
+                                  const CcEpi& ep, cudaStream_t st)
+{
+    int64_t blocks = (items + 127) / 128;
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, esb_dwconv3_kernel<B, STRIDE>, 128,
-                                                      sizeof(int32_t) * 9 * (size_t)((d.c + 32 / B - 1) / (32 / B)) *
-                                                          (32 / B)) != cudaSuccess ||
-        per_sm < 1)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 128, smem) != cudaSuccess || per_sm < 1)
         per_sm = 4;
     const int64_t cap = (int64_t)device_sm_count() * per_sm;
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    const int words = (d.c + 32 / B - 1) / (32 / B);
-    const size_t smem = sizeof(int32_t) * 9 * (size_t)words * (32 / B);
-    esb_dwconv3_kernel<B, STRIDE><<<(unsigned)blocks, 128, smem, st>>>(X, (int)ldx, kx, W, (int)ldw, kw, d.h, d.w, d.c,
-                                                                       d.pad, P, Q, QS, rows, ep);
+    kern<<<(unsigned)blocks, 128, smem, st>>>(X, (int)ldx, kx, W, (int)ldw, kw, d.h, d.w, d.c, d.pad, P, Q, QS,
+                                              d.n * P, ep);
     return cudaGetLastError();
+}
+
+template <int B, int STRIDE>
+static cudaError_t launch_dw3(const esb_conv_desc& d, int P, int Q, const uint32_t* X, int64_t ldx, int kx,
+                              const uint32_t* W, int64_t ldw, int kw, const CcEpi& ep, bool h16, cudaStream_t st)
+{
+    constexpr int QT = STRIDE == 1 ? 4 : 2;
+    const int QS = (Q + QT - 1) / QT;
+    const int64_t items = (int64_t)d.n * P * QS * ep.ldo;
+    const int words = (d.c + 32 / B - 1) / (32 / B);
+    if constexpr (B == 4) {
+        if (h16)
+            return launch_dw_wave(esb_dwconv3_b4h_kernel<STRIDE>, sizeof(__half2) * 9 * (size_t)words * 4, items, d, P,
+                                  Q, QS, X, ldx, kx, W, ldw, kw, ep, st);
+    }
+    return launch_dw_wave(esb_dwconv3_kernel<B, STRIDE>, sizeof(int32_t) * 9 * (size_t)words * (32 / B), items, d, P,
+                          Q, QS, X, ldx, kx, W, ldw, kw, ep, st);
 }
 
 static CcEpi make_cc_epi(const GemmOutputs& o, int ka, int kb)
@@ -404,15 +625,17 @@ cudaError_t launch_dwconv(const esb_conv_desc& d, int P, int Q, const uint32_t* 
     if (d.r == 3 && d.s == 3 && bw == bx && bx >= 3 && bx <= 6 && (d.stride == 1 || d.stride == 2) &&
         tab <= 48 * 1024 && fits32) {
         const bool s1 = d.stride == 1;
+        // packed fp16 sums are exact while every partial sum stays below 2^11
+        const bool h16 = 9.0 * fmt_max_image(bx, kx) * fmt_max_image(bw, kw) <= 2048.0;
         switch (bx) {
-        case 3: return s1 ? launch_dw3<3, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)
-                          : launch_dw3<3, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st);
-        case 4: return s1 ? launch_dw3<4, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)
-                          : launch_dw3<4, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st);
-        case 5: return s1 ? launch_dw3<5, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)
-                          : launch_dw3<5, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st);
-        default: return s1 ? launch_dw3<6, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st)
-                           : launch_dw3<6, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, st);
+        case 3: return s1 ? launch_dw3<3, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, false, st)
+                          : launch_dw3<3, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, false, st);
+        case 4: return s1 ? launch_dw3<4, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, h16, st)
+                          : launch_dw3<4, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, h16, st);
+        case 5: return s1 ? launch_dw3<5, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, false, st)
+                          : launch_dw3<5, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, false, st);
+        default: return s1 ? launch_dw3<6, 1>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, false, st)
+                           : launch_dw3<6, 2>(d, P, Q, X, ldx, kx, W, ldw, kw, ep, false, st);
         }
     }
     const int64_t total = (int64_t)d.n * P * Q * ep.ldo;
@@ -478,6 +701,44 @@ esb_maxpool_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int k, in
     }
 }
 
+// Window walk of the rank max pools: calls take(word) for every input word
+// of output pixel (q, p) of image nn at word w.  With WIN > 0 (the 3x3
+// window of ResNet18's stem pool) all WIN*WIN loads are issued before the
+// first maximum; taps outside the image read the zero-code word, whose
+// ranks are all 0 (the minimum), so they change nothing.
+template <int WIN, class Take>
+__device__ __forceinline__ void pool_window(const uint32_t* __restrict__ X, int64_t ldx, int nn, int p, int q, int w,
+                                            int H, int Wd, int win, int stride, int pad, uint32_t zw, Take take)
+{
+    if constexpr (WIN > 0) {
+        uint32_t xv[WIN * WIN];
+#pragma unroll
+        for (int r = 0; r < WIN; r++) {
+            const int h = p * stride - pad + r;
+            const bool hin = (unsigned)h < (unsigned)H;
+            const uint32_t* xr = X + ((int64_t)nn * H + (hin ? h : 0)) * Wd * ldx + w;
+#pragma unroll
+            for (int s2 = 0; s2 < WIN; s2++) {
+                const int ww = q * stride - pad + s2;
+                xv[r * WIN + s2] = (hin && (unsigned)ww < (unsigned)Wd) ? __ldg(xr + (int64_t)ww * ldx) : zw;
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < WIN * WIN; i++) take(xv[i]);
+    } else {
+        for (int r = 0; r < win; r++) {
+            const int h = p * stride - pad + r;
+            if (h < 0 || h >= H) continue;
+            const uint32_t* xr = X + ((int64_t)nn * H + h) * Wd * ldx + w;
+            for (int s2 = 0; s2 < win; s2++) {
+                const int ww = q * stride - pad + s2;
+                if (ww < 0 || ww >= Wd) continue;
+                take(__ldg(xr + (int64_t)ww * ldx));
+            }
+        }
+    }
+}
+
 // Max pooling of unsigned 4-bit codes without decoding them: the value
 // order of the non-negative set is the order of the rotated code
 // (e + 1 mod 2^(b-1-k), then f), i.e. rank = (code + 2^k) mod 8, so the
@@ -485,6 +746,7 @@ esb_maxpool_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int k, in
 // codes of a word in separate bytes) and the code comes back by the
 // inverse rotation.  One thread = one output word; blockIdx.y = image row
 // (n, p), threads over (q, word): 32-bit index arithmetic only.
+template <int WIN>
 __global__ void __launch_bounds__(256)
 esb_maxpool_b4u_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H, int Wd, int C, int win, int stride,
                        int pad, int P, int Q, uint32_t* __restrict__ Y, int64_t ldy)
@@ -494,32 +756,22 @@ esb_maxpool_b4u_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H
     const int per_row = Q * (int)ldy;
     const uint32_t rot = 0x11111111u << k;            // + 2^k in every nibble
     const int words = (C + 7) / 8;
+    const uint32_t zero = (uint32_t)((1 << (3 - k)) - 1) << k;   // e = N, f = 0 for b = 4
+    const uint32_t zw = 0x11111111u * zero;
     for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < per_row; t += gridDim.x * blockDim.x) {
         const int q = t / (int)ldy, w = t - (t / (int)ldy) * (int)ldy;
         uint32_t lo = 0u, hi = 0u;                    // rank maxima (0 = the rank of zero)
-        if (w < words) {
-            for (int r = 0; r < win; r++) {
-                const int h = p * stride - pad + r;
-                if (h < 0 || h >= H) continue;
-                const uint32_t* xr = X + ((int64_t)nn * H + h) * Wd * ldx + w;
-                for (int s2 = 0; s2 < win; s2++) {
-                    const int ww = q * stride - pad + s2;
-                    if (ww < 0 || ww >= Wd) continue;
-                    const uint32_t rk = ((__ldg(xr + (int64_t)ww * ldx) & 0x77777777u) + rot) & 0x77777777u;
-                    lo = __vmaxu4(lo, rk & 0x0F0F0F0Fu);
-                    hi = __vmaxu4(hi, (rk >> 4) & 0x0F0F0F0Fu);
-                }
-            }
-        }
+        if (w < words)
+            pool_window<WIN>(X, ldx, nn, p, q, w, H, Wd, win, stride, pad, zw, [&](uint32_t xw) {
+                const uint32_t rk = ((xw & 0x77777777u) + rot) & 0x77777777u;
+                lo = __vmaxu4(lo, rk & 0x0F0F0F0Fu);
+                hi = __vmaxu4(hi, (rk >> 4) & 0x0F0F0F0Fu);
+            });
         // inverse rotation: code = (rank - 2^k) mod 8; rank 0 is the zero code
         const uint32_t rk = lo | (hi << 4);
         uint32_t word = (rk + (0x88888888u - rot)) & 0x77777777u;
-        if (w >= words) word = 0u;
         // channels past C (in the last word) and padding words: the zero code
         const int c0 = w * 8;
-        const uint32_t zero = (uint32_t)((1 << (3 - k)) - 1) << k;   // e = N, f = 0 for b = 4
-        uint32_t zw = 0u;
-        for (int j = 0; j < 8; j++) zw |= zero << (4 * j);
         if (w >= words) word = zw;
         else if (c0 + 8 > C) {
             const int keep = C - c0;
@@ -535,7 +787,7 @@ esb_maxpool_b4u_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H
 // the zero code), so each channel slot keeps the largest rank of its
 // window and the code comes back by the inverse rotation.  One thread =
 // one output word; blockIdx.y = image row (n, p); 32-bit indices.
-template <int B>
+template <int B, int WIN>
 __global__ void __launch_bounds__(256)
 esb_maxpool_rank_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H, int Wd, int C, int win, int stride,
                         int pad, int P, int Q, uint32_t* __restrict__ Y, int64_t ldy)
@@ -548,28 +800,22 @@ esb_maxpool_rank_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int 
     const uint32_t rot = 1u << k;
     const int words = (C + CPW - 1) / CPW;
     const uint32_t zero = (uint32_t)((1 << (B - 1 - k)) - 1) << k;   // e = N, f = 0
+    uint32_t zw = 0u;
+#pragma unroll
+    for (int j = 0; j < CPW; j++) zw |= zero << (B * j);
     for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < per_row; t += gridDim.x * blockDim.x) {
         const int q = t / (int)ldy, w = t - (t / (int)ldy) * (int)ldy;
         uint32_t best[CPW];
 #pragma unroll
         for (int j = 0; j < CPW; j++) best[j] = 0u;
-        if (w < words) {
-            for (int r = 0; r < win; r++) {
-                const int h = p * stride - pad + r;
-                if (h < 0 || h >= H) continue;
-                const uint32_t* xr = X + ((int64_t)nn * H + h) * Wd * ldx + w;
-                for (int s2 = 0; s2 < win; s2++) {
-                    const int ww = q * stride - pad + s2;
-                    if (ww < 0 || ww >= Wd) continue;
-                    const uint32_t xw = __ldg(xr + (int64_t)ww * ldx);
+        if (w < words)
+            pool_window<WIN>(X, ldx, nn, p, q, w, H, Wd, win, stride, pad, zw, [&](uint32_t xw) {
 #pragma unroll
-                    for (int j = 0; j < CPW; j++) {
-                        const uint32_t rk = (((xw >> (B * j)) & RM) + rot) & RM;
-                        best[j] = best[j] > rk ? best[j] : rk;
-                    }
+                for (int j = 0; j < CPW; j++) {
+                    const uint32_t rk = (((xw >> (B * j)) & RM) + rot) & RM;
+                    best[j] = best[j] > rk ? best[j] : rk;
                 }
-            }
-        }
+            });
         uint32_t word = 0u;
 #pragma unroll
         for (int j = 0; j < CPW; j++) {
@@ -587,7 +833,10 @@ static void launch_maxpool_rank(const uint32_t* X, int64_t ldx, int k, int n, in
 {
     const int per_row = (int)(Q * ldy);
     const dim3 grid((unsigned)((per_row + 255) / 256), (unsigned)(n * P));
-    esb_maxpool_rank_kernel<B><<<grid, 256, 0, st>>>(X, ldx, k, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
+    if (win == 3)
+        esb_maxpool_rank_kernel<B, 3><<<grid, 256, 0, st>>>(X, ldx, k, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
+    else
+        esb_maxpool_rank_kernel<B, 0><<<grid, 256, 0, st>>>(X, ldx, k, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
 }
 
 cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int H, int Wd, int C, int win,
@@ -608,7 +857,10 @@ cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
     if (b == 4 && !is_signed && (int64_t)n * P <= 65535 && (int64_t)Q * ldy < (1ll << 31)) {
         const int per_row = (int)(Q * ldy);
         const dim3 grid((unsigned)((per_row + 255) / 256), (unsigned)(n * P));
-        esb_maxpool_b4u_kernel<<<grid, 256, 0, st>>>(X, ldx, k, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
+        if (win == 3)
+            esb_maxpool_b4u_kernel<3><<<grid, 256, 0, st>>>(X, ldx, k, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
+        else
+            esb_maxpool_b4u_kernel<0><<<grid, 256, 0, st>>>(X, ldx, k, H, Wd, C, win, stride, pad, P, Q, Y, ldy);
         return cudaGetLastError();
     }
     const int64_t total = (int64_t)n * P * Q * ldy;
@@ -618,70 +870,77 @@ cudaError_t launch_maxpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
 
 // ------------------------------------------------------ global avg pool
 
-// kPoolLanes threads = one code word of one image: each reads every
-// kPoolLanes-th pixel's word of that channel group and sums the images
-// exactly in int32 per channel; the partial sums are added by shuffles and
-// the first lane scales and requantises each sum through the block's
-// threshold table.
-constexpr int kPoolLanes = 8;
+// One block = 32 consecutive code words (lanes) of one image; its
+// kPoolWarps warps split the image's pixels (warp i takes pixels i, i + 8,
+// ...), so each warp load reads 128 contiguous bytes and a lane's loads are
+// independent.  Codes decode through a 2^B-entry table of integer images;
+// each lane sums its CPW channels exactly in int32; the partial sums of
+// warps 1..7 meet warp 0's in shared memory (integer sums: the result does
+// not depend on the split), and warp 0 scales and requantises each sum
+// through the block's threshold table.
+constexpr int kPoolWarps = 8;
 
-__global__ void __launch_bounds__(128)
-esb_avgpool_word_kernel(const uint32_t* __restrict__ X, int64_t ldx, int b, int k, int n, int HW, int C, int wout,
-                        float scale, float alpha_out, ProjParams out, float* __restrict__ y_out,
-                        uint32_t* __restrict__ codes_out, int64_t ldo)
+template <int B>
+__global__ void __launch_bounds__(kPoolWarps * 32)
+esb_avgpool_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int n, int HW, int C, int wout, float scale,
+                   float alpha_out, ProjParams out, float* __restrict__ y_out, uint32_t* __restrict__ codes_out,
+                   int64_t ldo)
 {
+    constexpr int CPW = 32 / B;
+    constexpr uint32_t MASK = (1u << B) - 1u;
     __shared__ float T[128];
+    __shared__ int32_t lut[1 << B];
+    __shared__ int32_t part[kPoolWarps - 1][CPW][32]; // [warp - 1][channel slot][lane]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     griddep_wait();
-    if (codes_out) build_thresholds(T, out, alpha_out, threadIdx.x >> 5, threadIdx.x & 31, 0, blockDim.x >> 5);
+    const int ew = B - k - 1, N = (1 << ew) - 1;
+    for (int i = threadIdx.x; i < (1 << B); i += blockDim.x) lut[i] = code_image_i((uint32_t)i, B, k, ew, N);
+    if (codes_out) build_thresholds(T, out, alpha_out, warp, lane, 0, kPoolWarps);
     __syncthreads();
-    // kPoolLanes consecutive lanes share one (image, word): each sums every
-    // kPoolLanes-th pixel, then the partial sums meet by shuffles (integer
-    // sums: the result does not depend on the split)
-    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int sub = threadIdx.x & (kPoolLanes - 1);
-    const int64_t grp = t / kPoolLanes;
-    const bool live = grp < (int64_t)n * wout;
-    const int nn = live ? (int)(grp / wout) : 0, w = live ? (int)(grp - (grp / wout) * wout) : 0;
-    const int cpw = 32 / b;
-    const int ew = b - k - 1, N = (1 << ew) - 1;
-    const uint32_t mask = (1u << b) - 1u;
-    uint32_t word = 0;
-    const bool has = live && w * cpw < C;
-    int32_t acc[16];
+    const int w = blockIdx.x * 32 + lane;
+    const bool has = w < wout && w * CPW < C;
+    for (int nn = blockIdx.y; nn < n; nn += gridDim.y) {
+        int32_t acc[CPW];
 #pragma unroll
-    for (int j = 0; j < 16; j++) acc[j] = 0;
-    if (has) {
-        const uint32_t* xp = X + (int64_t)nn * HW * ldx + w;
-        for (int i = sub; i < HW; i += kPoolLanes) {
-            const uint32_t xw = __ldg(xp + (int64_t)i * ldx);
+        for (int j = 0; j < CPW; j++) acc[j] = 0;
+        if (has) {
+            const uint32_t* xp = X + (int64_t)nn * HW * ldx + w;
+#pragma unroll 4
+            for (int i = warp; i < HW; i += kPoolWarps) {
+                const uint32_t xw = __ldg(xp + (int64_t)i * ldx);
 #pragma unroll
-            for (int j = 0; j < 16; j++)
-                if (j < cpw) acc[j] += code_image_i((xw >> (b * j)) & mask, b, k, ew, N);
-        }
-    }
-#pragma unroll
-    for (int o = kPoolLanes / 2; o > 0; o >>= 1)
-#pragma unroll
-        for (int j = 0; j < 16; j++)
-            if (j < cpw) acc[j] += __shfl_xor_sync(0xffffffffu, acc[j], o);
-    if (!live || sub != 0) return;
-    if (has) {
-#pragma unroll
-        for (int j = 0; j < 16; j++) {
-            if (j >= cpw) break;
-            const int c = w * cpw + j;
-            uint32_t code = out.zero_code;
-            if (c < C) {
-                const float y = __fmul_rn(scale, (float)acc[j]);
-                if (y_out) y_out[(int64_t)nn * C + c] = y;
-                if (codes_out) code = project_by_table(y, T, out);
+                for (int j = 0; j < CPW; j++) acc[j] += lut[(xw >> (B * j)) & MASK];
             }
-            word |= code << (out.b * j);
         }
-    } else {
-        for (int j = 0; j < 32 / out.b; j++) word |= out.zero_code << (out.b * j);
+        if (warp > 0) {
+#pragma unroll
+            for (int j = 0; j < CPW; j++) part[warp - 1][j][lane] = acc[j];
+        }
+        __syncthreads();                              // partial sums ready
+        if (warp == 0 && w < wout) {
+            uint32_t word = 0;
+            if (has) {
+#pragma unroll 1
+                for (int j = 0; j < CPW; j++) {
+                    int32_t sum = acc[j];
+#pragma unroll
+                    for (int v = 0; v < kPoolWarps - 1; v++) sum += part[v][j][lane];
+                    const int c = w * CPW + j;
+                    uint32_t code = out.zero_code;
+                    if (c < C) {
+                        const float y = __fmul_rn(scale, (float)sum);
+                        if (y_out) y_out[(int64_t)nn * C + c] = y;
+                        if (codes_out) code = project_by_table(y, T, out);
+                    }
+                    word |= code << (out.b * j);
+                }
+            } else {
+                for (int j = 0; j < 32 / out.b; j++) word |= out.zero_code << (out.b * j);
+            }
+            if (codes_out && w < ldo) codes_out[(int64_t)nn * ldo + w] = word;
+        }
+        __syncthreads();                              // part is rewritten by the next image
     }
-    if (codes_out && w < ldo) codes_out[(int64_t)nn * ldo + w] = word;
 }
 
 cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, int HW, int C, float scale,
@@ -691,9 +950,24 @@ cudaError_t launch_avgpool(const uint32_t* X, int64_t ldx, int b, int k, int n, 
     ProjParams out = make_proj_params(bo, ko, so, rounding);
     int64_t words = (C + (32 / b) - 1) / (32 / b);
     if (codes_out && ldo > words) words = ldo;          // also write the row's padding words
-    const int64_t total = (int64_t)n * words * kPoolLanes;
-    esb_avgpool_word_kernel<<<(unsigned)((total + 127) / 128), 128, 0, st>>>(X, ldx, b, k, n, HW, C, (int)words, scale,
-                                                                           alpha_out, out, y_out, codes_out, ldo);
+    const dim3 grid((unsigned)((words + 31) / 32), (unsigned)(n < 65535 ? n : 65535));
+    const int wo = (int)words;
+    switch (b) {
+    case 2: esb_avgpool_kernel<2><<<grid, kPoolWarps * 32, 0, st>>>(X, ldx, k, n, HW, C, wo, scale, alpha_out, out,
+                                                                     y_out, codes_out, ldo); break;
+    case 3: esb_avgpool_kernel<3><<<grid, kPoolWarps * 32, 0, st>>>(X, ldx, k, n, HW, C, wo, scale, alpha_out, out,
+                                                                     y_out, codes_out, ldo); break;
+    case 4: esb_avgpool_kernel<4><<<grid, kPoolWarps * 32, 0, st>>>(X, ldx, k, n, HW, C, wo, scale, alpha_out, out,
+                                                                     y_out, codes_out, ldo); break;
+    case 5: esb_avgpool_kernel<5><<<grid, kPoolWarps * 32, 0, st>>>(X, ldx, k, n, HW, C, wo, scale, alpha_out, out,
+                                                                     y_out, codes_out, ldo); break;
+    case 6: esb_avgpool_kernel<6><<<grid, kPoolWarps * 32, 0, st>>>(X, ldx, k, n, HW, C, wo, scale, alpha_out, out,
+                                                                     y_out, codes_out, ldo); break;
+    case 7: esb_avgpool_kernel<7><<<grid, kPoolWarps * 32, 0, st>>>(X, ldx, k, n, HW, C, wo, scale, alpha_out, out,
+                                                                     y_out, codes_out, ldo); break;
+    default: esb_avgpool_kernel<8><<<grid, kPoolWarps * 32, 0, st>>>(X, ldx, k, n, HW, C, wo, scale, alpha_out, out,
+                                                                      y_out, codes_out, ldo); break;
+    }
     return cudaGetLastError();
 }
 

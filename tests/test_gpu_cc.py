@@ -63,6 +63,72 @@ def test_depthwise_matches_oracle(n, h, w, c, stride, fx, fw, act):
     assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
 
 
+@pytest.mark.parametrize("n,h,w,c,stride,fo,act", [
+    (2, 14, 14, 96, 1, (4, 2, False), esb.ESB_ACT_RELU6),      # MobileNetV2: per-channel BN fold, ReLU6
+    (2, 13, 15, 44, 2, (4, 2, False), esb.ESB_ACT_RELU6),      # stride 2, ragged channels
+    (2, 9, 11, 40, 1, (4, 1, True), esb.ESB_ACT_NONE),         # signed outputs: sign bits, negative zero buckets
+    (2, 9, 10, 24, 1, (4, 3, False), esb.ESB_ACT_NONE),        # unsigned outputs of negative values: the zero code
+    (1, 7, 7, 960, 1, (4, 2, False), esb.ESB_ACT_RELU),
+])
+def test_depthwise_codes_only_per_channel(n, h, w, c, stride, fo, act):
+    """4-bit codes out with per-channel scale and bias and no other output:
+    the word-at-a-time requantisation (buckets of |y| packed into a word)."""
+    r = s = 3
+    pad = 1
+    x = synth.normal((n * h * w, c), seed=c + h + 1).numpy()
+    wt = synth.he_normal((r * s, c), fan_in=9, seed=c + 3).numpy()
+    fx, fw = (4, 2, True), (4, 2, True)
+    ldx = esb.esb_row_words(c, 4)
+    ax, _ = o.calibrate(x, *fx)
+    aw, _ = o.calibrate(wt, *fw)
+    X = o.project_packed(x, ax, *fx, ld_words=ldx)
+    W = o.project_packed(wt, aw, *fw, ld_words=ldx)
+    scale = (np.float32(ax * aw / 16) * (1 + 0.2 * synth.normal((c,), seed=7).numpy())).astype(np.float32)
+    bias = (0.1 * synth.normal((c,), seed=8).numpy()).astype(np.float32)
+    ep = esb.Epilogue(scale=torch.from_numpy(scale).cuda(), bias=torch.from_numpy(bias).cuda(), act=act,
+                      alpha_out=0.31, fmt_out=esb.Fmt(*fo))
+    _, _, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fx), dev_i32(W), esb.Fmt(*fw), n, h, w, c, c, r, s,
+                                      stride, pad, groups=c, ep=ep, want_acc=False, want_codes=True)
+    acc_o = o.dwconv_i64(X.reshape(n, h, w, ldx), fx[:2], W.reshape(r, s, -1), fw[:2], n, h, w, c, r, s, stride,
+                         pad).reshape(-1, c)
+    _, co = o.epilogue(acc_o, scale, bias, act, 0.31, fo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
+@pytest.mark.parametrize("stride", [1, 2])
+def test_depthwise_b4_largest_sums(stride):
+    """4-bit (4,1) images reach 12 in magnitude, so 3x3 sums reach 9 * 144 =
+    1296: the bound under which 4-bit depthwise sums are exact in fp16.
+    Image 0 holds the largest positive image in half the channels, against
+    filters of the largest positive and negative images; the rest is every
+    code pattern drawn uniformly (negative zero and subnormal codes too)."""
+    n, h, w, c = 2, 10, 13, 72
+    r = s = 3
+    pad = 1
+    ldx = esb.esb_row_words(c, 4)
+    xc = synth.uniform_ints((n * h * w, c), 0, 16, seed=11 + stride)
+    wc = synth.uniform_ints((r * s, c), 0, 16, seed=12 + stride)
+    xc[:h * w, :c // 2] = 5                       # code 0101 of (4,1): image +12
+    wc[:, :c // 4] = 5
+    wc[:, c // 4:c // 2] = 13                     # code 1101: image -12
+    X = o.pack(xc, 4, 1, ld_words=ldx)
+    W = o.pack(wc, 4, 1, ld_words=ldx)
+    scale = np.full(c, 1e-3, np.float32)
+    bias = np.zeros(c, np.float32)
+    fo = (4, 1, True)
+    ep = esb.Epilogue(scale=torch.from_numpy(scale).cuda(), bias=torch.from_numpy(bias).cuda(),
+                      act=esb.ESB_ACT_NONE, alpha_out=0.5, fmt_out=esb.Fmt(*fo))
+    acc, y, codes = esb.esb_conv2d_nhwc(dev_i32(X), esb.Fmt(*fo), dev_i32(W), esb.Fmt(*fo), n, h, w, c, c, r, s,
+                                        stride, pad, groups=c, ep=ep, want_acc=True, want_y=True, want_codes=True)
+    acc_o = o.dwconv_i64(X.reshape(n, h, w, ldx), (4, 1), W.reshape(r, s, -1), (4, 1), n, h, w, c, r, s, stride,
+                         pad).reshape(-1, c)
+    assert acc_o.max() == 1296 and acc_o.min() == -1296
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), acc_o)
+    yo, co = o.epilogue(acc_o, scale, bias, esb.ESB_ACT_NONE, 0.5, fo)
+    assert np.array_equal(y.cpu().numpy(), yo)
+    assert np.array_equal(u32(codes), o.pack(co, fo[0], fo[1], ld_words=codes.shape[1]))
+
+
 POOL_CASES = [
     # n, h, w, c, win, stride, pad, fmt
     (2, 112, 112, 64, 3, 2, 1, (4, 2)),     # ResNet18 stem pool
@@ -109,7 +175,7 @@ def test_maxpool_unsigned_rank_matches_oracle(n, h, w, c, win, stride, pad, fmt)
 
 
 @pytest.mark.parametrize("n,hw,c,fmt", [(4, 49, 512, (4, 2)), (3, 49, 1280, (4, 2)), (2, 16, 37, (6, 3)),
-                                        (2, 1, 5, (3, 1))])
+                                        (2, 1, 5, (3, 1)), (3, 25, 530, (2, 0)), (2, 100, 300, (5, 2))])
 def test_avgpool_matches_oracle(n, hw, c, fmt):
     b, k = fmt
     x = synth.half_normal((n * hw, c), seed=c).numpy()
