@@ -975,6 +975,46 @@ def run_peaks(args):
     print(json.dumps(out), flush=True)
 
 
+def run_cc_profile(args):
+    """A few launches of each CUDA-core kernel, untimed: the target of an ncu
+    capture (`-k regex:"dwconv3_b4h|maxpool_b4u|avgpool_kernel"`).  Depthwise
+    3x3 112x112x32 at batch 32 (per-channel scale and bias, ReLU6, codes
+    out), the ResNet18 stem max pool at batch 32 and the 7x7x1280 global
+    average pool at batch 64, ESB(4,2), four rounds."""
+    import torch
+
+    from paper_2109_03513_gb300 import esb
+    import __graft_entry__
+
+    __graft_entry__.build()
+    dev = torch.device("cuda:0")
+    g = torch.Generator(device=dev).manual_seed(0)
+    fx, fw = esb.Fmt(4, 2, False), esb.Fmt(4, 2, True)
+
+    def words(rows, ld, unsigned=True):
+        c = torch.randint(0, 2 ** 32, (rows, ld), generator=g, device=dev, dtype=torch.int64).to(torch.int32)
+        return c & 0x77777777 if unsigned else c
+
+    n, h, c = 32, 112, 32
+    ld = esb.esb_row_words(c, 4)
+    X, W = words(n * h * h, ld), words(9, ld, False)
+    ep = esb.Epilogue(scale=torch.full((c,), 1e-3, device=dev), bias=torch.zeros((c,), device=dev),
+                      act=esb.ESB_ACT_RELU6, alpha_out=0.29, fmt_out=fx)
+    oc = torch.empty((n * h * h, ld), dtype=torch.int32, device=dev)
+    Xm, Y = words(n * 112 * 112, 8), torch.empty((n * 56 * 56, 8), dtype=torch.int32, device=dev)
+    Xa = words(64 * 49, esb.esb_row_words(1280, 4))
+    for _ in range(4):
+        esb.esb_conv2d_nhwc(X, fx, W, fw, n, h, h, c, c, 3, 3, 1, 1, groups=c, ep=ep, want_acc=False,
+                            want_codes=True, out_codes=oc)
+        esb.esb_maxpool_nhwc(Xm, fx, n, 112, 112, 64, 3, 2, 1, out=Y)
+        esb.esb_avgpool_nhwc(Xa, fx, 64, 49, 1280, 1.0 / 49, 0.5, fx)
+    torch.cuda.synchronize()
+    st = esb.esb_get_status()
+    print(json.dumps({"cc_profile": "done", "status": st}), flush=True)
+    if st != 0:
+        raise SystemExit(1)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -988,10 +1028,14 @@ def main():
                     help="conv3x3: the benchmark step (default); the others: whole-network forwards")
     ap.add_argument("--bk", nargs="*", help="formats b,k of a network workload (default: its configuration's)")
     ap.add_argument("--peaks", action="store_true", help="measure the tensor-pipe peaks instead")
+    ap.add_argument("--cc-profile", action="store_true",
+                    help="a few untimed launches of the CUDA-core kernels (an ncu capture target)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.peaks:
+    if args.cc_profile:
+        run_cc_profile(args)
+    elif args.peaks:
         run_peaks(args)
     elif args.workload != "conv3x3" and args.impl == "ours":
         run_network(args, args.workload)
