@@ -330,9 +330,10 @@ esb_dwconv3_kernel(const uint32_t* __restrict__ X, int ldx, int kx, const uint32
 // word), so one instruction does two channels' multiply-adds and one table
 // load decodes two codes.  The sums never take the value -0 (they start at
 // +0, and an exact zero sum rounds to +0), so their conversion to float is
-// the integer accumulator's.  Work items, the strip walk and the epilogue
-// are those of the integer kernel above; the next filter row's input words
-// are loaded while the current row is multiplied.
+// the integer accumulator's.  Work items, the strip walk and the epilogues
+// are those of the integer kernel above, plus a word-at-a-time one for
+// codes-only outputs with per-channel scale and bias; the next filter row's
+// input words are loaded while the current row is multiplied.
 template <int STRIDE>
 __global__ void __launch_bounds__(128, 6)
 esb_dwconv3_b4h_kernel(const uint32_t* __restrict__ X, int ldx, int kx, const uint32_t* __restrict__ W, int ldw,
