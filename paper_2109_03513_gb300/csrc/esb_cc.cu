@@ -743,10 +743,12 @@ __device__ __forceinline__ void pool_window(const uint32_t* __restrict__ X, int6
 // Max pooling of unsigned 4-bit codes without decoding them: the value
 // order of the non-negative set is the order of the rotated code
 // (e + 1 mod 2^(b-1-k), then f), i.e. rank = (code + 2^k) mod 8, so the
-// maximum of a window is the byte-wise maximum of the ranks (even and odd
-// codes of a word in separate bytes) and the code comes back by the
-// inverse rotation.  One thread = one output word; blockIdx.y = image row
-// (n, p), threads over (q, word): 32-bit index arithmetic only.
+// maximum of a window is the nibble-wise maximum of the ranks and the code
+// comes back by the inverse rotation.  The eight 3-bit ranks of a word are
+// compared at once: (best | 8) - rank in each nibble lies in 1..15 (no
+// borrow crosses a nibble) and keeps bit 3 exactly where best >= rank,
+// which selects the larger of the two.  One thread = one output word;
+// blockIdx.y = image row (n, p), threads over (q, word).
 template <int WIN>
 __global__ void __launch_bounds__(256)
 esb_maxpool_b4u_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H, int Wd, int C, int win, int stride,
@@ -761,16 +763,16 @@ esb_maxpool_b4u_kernel(const uint32_t* __restrict__ X, int64_t ldx, int k, int H
     const uint32_t zw = 0x11111111u * zero;
     for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < per_row; t += gridDim.x * blockDim.x) {
         const int q = t / (int)ldy, w = t - (t / (int)ldy) * (int)ldy;
-        uint32_t lo = 0u, hi = 0u;                    // rank maxima (0 = the rank of zero)
+        uint32_t best = 0u;                           // rank maxima, one per nibble (0 = the rank of zero)
         if (w < words)
             pool_window<WIN>(X, ldx, nn, p, q, w, H, Wd, win, stride, pad, zw, [&](uint32_t xw) {
                 const uint32_t rk = ((xw & 0x77777777u) + rot) & 0x77777777u;
-                lo = __vmaxu4(lo, rk & 0x0F0F0F0Fu);
-                hi = __vmaxu4(hi, (rk >> 4) & 0x0F0F0F0Fu);
+                const uint32_t ge = ((best | 0x88888888u) - rk) & 0x88888888u;   // bit 3: best >= rk
+                const uint32_t keep = ge - (ge >> 3);                            // 7 where best >= rk
+                best = (best & keep) | (rk & ~keep);
             });
         // inverse rotation: code = (rank - 2^k) mod 8; rank 0 is the zero code
-        const uint32_t rk = lo | (hi << 4);
-        uint32_t word = (rk + (0x88888888u - rot)) & 0x77777777u;
+        uint32_t word = (best + (0x88888888u - rot)) & 0x77777777u;
         // channels past C (in the last word) and padding words: the zero code
         const int c0 = w * 8;
         if (w >= words) word = zw;
