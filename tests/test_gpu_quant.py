@@ -67,7 +67,8 @@ def test_project_b4_flat_probes(k, signed):
     C = o.C_of(4, k)
     base = np.concatenate([probe_values(4, k), synth.normal((4000,), seed=40 + k).numpy() * np.float32(C)])
     for alpha in (1.0, 0.7310585, 3.0, 2.0 ** -20, 1e-35, 1e35, 6.0e-8):
-        pts = np.concatenate([base * np.float32(alpha), base]).astype(np.float32)
+        with np.errstate(over="ignore"):                # alpha = 1e35 sends probes to infinity on purpose
+            pts = np.concatenate([base * np.float32(alpha), base]).astype(np.float32)
         pts = pts[: pts.size // 64 * 64]
         for shape in ((1, pts.size), (pts.size // 64, 64)):
             xs = pts.reshape(shape)
@@ -92,7 +93,8 @@ def test_project_cell_table_probes(b, k, signed):
     C = o.C_of(b, k)
     base = np.concatenate([probe_values(b, k), synth.normal((3000,), seed=50 + 8 * b + k).numpy() * np.float32(C)])
     for alpha in (1.0, 0.7310585, 3.0, 2.0 ** -20, 1e-35, 1e35, 6.0e-8):
-        pts = np.concatenate([base * np.float32(alpha), base]).astype(np.float32)
+        with np.errstate(over="ignore"):                # alpha = 1e35 sends probes to infinity on purpose
+            pts = np.concatenate([base * np.float32(alpha), base]).astype(np.float32)
         for rounding in (0, 1):
             for shape in ((1, pts.size), (pts.size // 96, 96)):
                 xs = np.ascontiguousarray(pts[: int(np.prod(shape))].reshape(shape))
